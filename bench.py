@@ -1,0 +1,355 @@
+#!/usr/bin/env python3
+"""Benchmark of carry-through-protected CNN inference on one or more GPUs.
+
+One step = one batch through the whole inference path on each GPU:
+ct_infer (carry-through convolutions, FC layers with the checksum neurons,
+per-image verification) followed by ct_reexecute of the flagged images
+(fault-free run: the flagged images are the false alarms of the
+distribution-based threshold, alpha = 1%).  The same model built without
+carry-through filters gives the unprotected throughput and the overhead.
+
+Prints ONE JSON line (rank 0).  Multi-GPU (torchrun): independent replicas,
+each rank runs its own batch; only the barrier and the max-over-ranks timing
+use a collective.
+
+  python bench.py [--workload NAME] [--steps K] [--warmup W] [--gpus N]
+  python bench.py --impl reference ...   # the CPU oracle on a bounded sample
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+METRIC = "protected images/sec and checksum overhead % vs unprotected; conv % of GB300 peak"
+DEFAULT_WORKLOAD = "resnet18_imagenet"
+# bounded oracle samples (images) per workload: roughly 10-30 s of CPU work
+ORACLE_SAMPLE = {"lenet5": 256, "resnet18_cifar": 24, "campaign_resnet18_cifar": 24,
+                 "resnet18_imagenet": 16, "vgg16": 3}
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        return json.load(open(p)), "measured"
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+            "sm_max_mhz": 2070.0}, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons, sampled during the timed region."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.rows = []
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.Q,
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.rows.append([c.strip() for c in line.split(",")])
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        ok = [r for r in self.rows if len(r) >= 9]
+        sm = [float(r[1]) for r in ok if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in ok if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = set()
+        for r in ok:
+            for nm, v in zip(names, r[5:9]):
+                if v.strip().lower() in ("active", "1"):
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def conv_flops(wl) -> float:
+    sh = synth.shapes(wl.layers, wl.in_shape)
+    f = 0.0
+    for L in wl.layers:
+        if L.op == "conv":
+            _, P, Q = sh[L.dst]
+            f += 2.0 * P * Q * L.cout * L.cin * L.k * L.k
+    return f * wl.batch
+
+
+def oracle_rate(wl, n_img: int):
+    """Oracle images/s on n_img images of the workload (CPU, as it stands)."""
+    import oracle
+    net = oracle.build_workload(wl)
+    x = synth.make_input(wl, batch=n_img)
+    t = time.perf_counter()
+    oracle.forward(net, x)
+    dt = time.perf_counter() - t
+    return n_img / dt, oracle.get_threads(), dt
+
+
+def run_reference(args, wl, rank, world):
+    """--impl reference: the CPU oracle, timed on bounded samples of the workload."""
+    if rank != 0:
+        return
+    import oracle
+    n = max(1, ORACLE_SAMPLE.get(wl.name, 4) // max(1, args.steps))
+    net = oracle.build_workload(wl)
+    x = synth.make_input(wl, batch=n)
+    for _ in range(min(args.warmup, 1)):
+        oracle.forward(net, x[:1])
+    times = []
+    for _ in range(args.steps):
+        t = time.perf_counter()
+        oracle.forward(net, x)
+        times.append(time.perf_counter() - t)
+    total = sum(times)
+    v = n * args.steps / total
+    line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "images/s",
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * total / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None,
+            "dtype": "f16" if wl.precision == "fp16" else "f32",
+            "data": "synthetic", "config": {"workload": wl.name, "batch": n,
+                                            "precision": wl.precision},
+            "cpu_baseline": {"value": v, "unit": "images/s", "cores": oracle.get_threads(),
+                             "kind": "oracle",
+                             "sample": "%d steps x %d images of %s" % (args.steps, n, wl.name)},
+            "e2e": {"value": v, "unit": "images/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
+    ap.add_argument("--simt-only", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    wl = synth.workload(args.workload)
+
+    if args.impl == "reference":
+        run_reference(args, wl, rank, world)
+        return
+
+    import torch
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+
+    from paper_2609_16742_gb300 import build as _build
+    if rank == 0:
+        _build.build()
+    if dist is not None:
+        dist.barrier()
+    import paper_2609_16742_gb300 as ct
+
+    B = wl.batch
+    params = synth.make_params(wl.layers, wl.seed)
+    mp = ct.ct_build_workload(wl, params, device=local, simt_only=args.simt_only)
+    mu = ct.ct_build_workload(wl, params, device=local, simt_only=args.simt_only, protect=False)
+
+    # calibration (Sec. II-C, distribution-based, alpha = 1%) on seeded fault-free images
+    calib_n = 2 * B
+    xc = torch.from_numpy(synth.make_input(wl, batch=calib_n, seed=wl.calib_seed)).cuda()
+    Sc = torch.empty(calib_n, device="cuda")
+    lc = torch.empty(B, wl.n_classes, device="cuda")
+    for i in range(0, calib_n, B):
+        ct.ct_infer(mp, xc[i:i + B], B, lc, Sc[i:i + B], None)
+    torch.cuda.synchronize()
+    r, tau = ct.ct_calibrate(Sc.cpu().numpy(), 0.01)
+    ct.ct_set_threshold(mp, r, tau)
+    del xc
+
+    # evaluation batch for this rank (a distinct slice of the seeded set per rank)
+    x_host = synth.make_input(wl, batch=B, first=rank * B)
+    x = torch.from_numpy(x_host).cuda()
+    logits = torch.empty(B, wl.n_classes, device="cuda")
+    S = torch.empty(B, device="cuda")
+    flag = torch.empty(B, dtype=torch.uint8, device="cuda")
+    stream = torch.cuda.current_stream()
+
+    def step_protected():
+        ct.ct_infer(mp, x, B, logits, S, flag, stream)
+        return ct.ct_reexecute(mp, x, B, flag, logits, S, stream)
+
+    def step_unprotected():
+        ct.ct_infer(mu, x, B, logits, None, None, stream)
+        return 0
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    def timed(fn, steps):
+        barrier()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        n_re = 0
+        for _ in range(steps):
+            n_re += fn()
+        e1.record(stream)
+        barrier()
+        ms = e0.elapsed_time(e1)
+        if dist is not None:
+            t = torch.tensor([ms], device="cuda")
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            ms = float(t.item())
+        return ms, n_re
+
+    for _ in range(max(args.warmup, 3)):
+        step_protected()
+        step_unprotected()
+    torch.cuda.synchronize()
+
+    # unprotected reference (same kernels, no carry-through filters)
+    ms_u, _ = timed(step_unprotected, args.steps)
+
+    # protected, timed, with clocks sampled and per-kernel events on the launch stream
+    clk = ClockSampler(local if "CUDA_VISIBLE_DEVICES" not in os.environ else
+                       int(os.environ["CUDA_VISIBLE_DEVICES"].split(",")[local]))
+    ct.ct_profile_enable(mp, True)
+    for fam in range(5):
+        ct.ct_profile_read(mp, fam)
+    clk.start()
+    ms_p, n_rerun = timed(step_protected, args.steps)
+    clocks = clk.stop()
+    ct.ct_profile_enable(mp, False)
+    fam_stats = {fam: ct.ct_profile_read(mp, fam) for fam in range(5)}
+    err = ct.ct_device_error(mp)
+
+    # end to end through the public host API: H2D input, infer, re-execute, D2H results
+    xh = torch.from_numpy(x_host).pin_memory()
+    lh = torch.empty(B, wl.n_classes, dtype=torch.float32).pin_memory()
+    sh = torch.empty(B, dtype=torch.float32).pin_memory()
+    fh = torch.empty(B, dtype=torch.uint8).pin_memory()
+    xn, ln, sn, fn_ = xh.numpy(), lh.numpy(), sh.numpy(), fh.numpy()
+    for _ in range(2):
+        ct.ct_run_host(mp, xn, ln, sn, fn_, stream)
+    barrier()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        ct.ct_run_host(mp, xn, ln, sn, fn_, stream)
+    barrier()
+    e2e_s = time.perf_counter() - t0
+    if dist is not None:
+        t = torch.tensor([e2e_s], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_s = float(t.item())
+
+    if rank != 0:
+        if dist is not None:
+            dist.destroy_process_group()
+        return
+
+    pk, pk_kind = peaks()
+    value = world * B * args.steps / (ms_p / 1e3)
+    value_u = world * B * args.steps / (ms_u / 1e3)
+    props = torch.cuda.get_device_properties(local)
+    # dominant kernel: the convolution family that carries the FLOPs
+    tc_n, tc_ms, tc_fl = fam_stats[0]
+    si_n, si_ms, si_fl = fam_stats[1]
+    if tc_ms >= si_ms and tc_n:
+        roof = {"kernel": "conv_tc_kernel (tcgen05, fp16 in / fp32 acc)", "bound": "tensor",
+                "achieved": tc_fl / (tc_ms / 1e3) / 1e12, "peak": pk["bf16_tflops"],
+                "unit": "TFLOP/s",
+                "peak_source": "%s bf16 dense burst; fp16 has the bf16 rate" % pk_kind,
+                "launches": tc_n, "avg_launch_us": 1e3 * tc_ms / tc_n,
+                "flops_per_launch": tc_fl / tc_n}
+    else:
+        clock = pk.get("sm_max_mhz", 2070.0) * 1e6
+        peak = props.multi_processor_count * 128 * 2 * clock / 1e12
+        roof = {"kernel": "conv_simt_kernel (FFMA)", "bound": "alu",
+                "achieved": si_fl / (si_ms / 1e3) / 1e12 if si_ms else 0.0,
+                "peak": peak, "unit": "TFLOP/s",
+                "peak_source": "%d SMs x 128 FFMA/clk x 2 flop x %.0f MHz (%s max SM clock)"
+                               % (props.multi_processor_count, clock / 1e6, pk_kind),
+                "launches": si_n, "avg_launch_us": 1e3 * si_ms / max(si_n, 1),
+                "flops_per_launch": si_fl / max(si_n, 1)}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["traffic"] = None
+    roof["conv_share_of_step"] = (tc_ms + si_ms) / ms_p if ms_p else None
+    launches = int(sum(v[0] for v in fam_stats.values()))
+
+    cpu = None
+    if not args.no_cpu_baseline:
+        n_img = ORACLE_SAMPLE.get(wl.name, 4)
+        v, cores, dt = oracle_rate(wl, n_img)
+        cpu = {"value": v, "unit": "images/s", "cores": cores, "kind": "oracle",
+               "sample": "%d images of %s, one forward pass (%.1f s)" % (n_img, wl.name, dt)}
+
+    in_bytes = B * int(np.prod(wl.in_shape)) * 4
+    out_bytes = B * (wl.n_classes * 4 + 4 + 1)
+    line = {
+        "metric": METRIC, "value": value, "unit": "images/s", "n_gpus": world,
+        "steps": args.steps, "warmup": max(args.warmup, 3), "ms_per_step": ms_p / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f16" if wl.precision == "fp16" else "f32", "data": "synthetic",
+        "config": {"workload": wl.name, "batch_per_gpu": B, "in_shape": list(wl.in_shape),
+                   "precision": wl.precision + (" storage, fp32 accumulate"
+                                                if wl.precision == "fp16" else ""),
+                   "parallelism": "replicas x%d" % world, "alpha": 0.01,
+                   "l2": "inputs and activations larger than L2 (no flush)",
+                   "simt_only": bool(args.simt_only)},
+        "unprotected_value": value_u,
+        "overhead_pct": 100.0 * (ms_p / ms_u - 1.0),
+        "reexecuted_images_per_step": n_rerun / args.steps,
+        "conv_tflop_per_batch": conv_flops(wl) / 1e12,
+        "roofline": roof,
+        "cpu_baseline": cpu,
+        "e2e": {"value": world * B * args.steps / e2e_s, "unit": "images/s",
+                "h2d_bytes_per_step": in_bytes, "d2h_bytes_per_step": out_bytes},
+        "gpu_launches": launches,
+        "clocks": clocks,
+        "device_error": err,
+        "threshold": {"reference": r, "tau": tau},
+    }
+    print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,228 @@
+/*
+ * ct.h -- C ABI of the carry-through checksum inference library (libct.so).
+ *
+ * The library runs CNN inference in which convolutional layers carry the
+ * carry-through filter of Sec. II-A (an extra output filter with a single 1
+ * at the kernel centre over every input channel), propagates the resulting
+ * checksum channel through bias, activation, pooling and the classifier,
+ * sums it in the accumulated-checksum neuron of Sec. II-B, and flags every
+ * image whose neuron deviates from a reference by more than a threshold.
+ * A bit-flip injector (Sec. III-A) and re-execution of flagged images
+ * (Sec. II-B, last paragraph) complete the path.
+ *
+ * Conventions shared by every entry point:
+ *   - Status codes only; nothing is thrown across the ABI.
+ *   - "_dev" pointers are CUDA device pointers on the model's device; the
+ *     caller owns them and keeps them valid until the stream work that uses
+ *     them has finished.  "_host" pointers are host memory.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream).  Calls are asynchronous on that stream unless stated.
+ *   - The library owns all weights, activation workspaces and scratch.
+ *   - A model is not thread-safe: one host thread at a time per model.
+ */
+#ifndef CT_H
+#define CT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    CT_OK = 0,
+    CT_EINVAL = 1,       /* bad argument or malformed description */
+    CT_ENOMEM = 2,       /* device or host allocation failed */
+    CT_ECUDA = 3,        /* a CUDA runtime/driver call failed */
+    CT_ESTATE = 4,       /* call not valid in the model's current state */
+    CT_ERANGE = 5,       /* index, batch or bit outside the allowed range */
+    CT_EUNSUPPORTED = 6, /* shape the kernels do not implement */
+    CT_EDEVICE = 7       /* a kernel reported a device-side error (bounded wait expired) */
+} ct_status;
+
+typedef enum { CT_FP32 = 0, CT_FP16 = 1 } ct_precision;
+
+typedef enum { CT_OP_CONV = 0, CT_OP_MAXPOOL = 1, CT_OP_GAP = 2, CT_OP_FC = 3 } ct_op;
+
+/* Role of a convolution in the scheme (Sec. II-A):
+ *   CT_ROLE_CT   carries a carry-through filter (new last output channel);
+ *   CT_ROLE_NONE carries none: the first convolution of a residual block,
+ *                whose input is also the block's shortcut (Sec. II-A, last
+ *                paragraph);
+ *   CT_ROLE_PASS a 1x1 downsample shortcut: its checksum output is the
+ *                incoming checksum at the sampled position (or nothing when
+ *                the model is built with CT_DS_ZERO). */
+typedef enum { CT_ROLE_CT = 0, CT_ROLE_NONE = 1, CT_ROLE_PASS = 2 } ct_role;
+
+typedef enum { CT_BUF_WEIGHT = 0, CT_BUF_ACT = 1 } ct_buf_kind;
+
+typedef enum { CT_DS_PASS = 0, CT_DS_ZERO = 1 } ct_ds_mode;
+
+/* One operation over numbered tensor slots; slot 0 is the network input.
+ *   CONV    y = act(conv(x[src]) * BN + res[res]) with kernel k x k, stride,
+ *           pad; res = -1 for none; weights OIHW [cout, cin, k, k].
+ *   MAXPOOL k x k window, stride, pad (padding never wins).
+ *   GAP     global average pool to a vector of cin features.
+ *   FC      y = act(W x + b), W [cout, cin] with cin counted in the
+ *           PyTorch flatten order (C, H, W) of the data channels; `final`
+ *           marks the classifier, which gets the accumulated-checksum neuron.
+ * ct_shift: the layer's carry-through coefficients are 2^-ct_shift instead
+ * of 1 (keeps an FP16 checksum neuron inside the FP16 range). */
+typedef struct {
+    int32_t op, src, dst, res;
+    int32_t cin, cout, k, stride, pad;
+    int32_t role;
+    int32_t bn, relu, final;
+    int32_t ct_shift;
+} ct_layer_desc;
+
+typedef struct {
+    int32_t n_layers;
+    const ct_layer_desc *layers;
+    int32_t in_c, in_h, in_w;     /* input image shape (NCHW without N) */
+    int32_t n_classes;
+    double bn_eps;                /* epsilon of Eq. 1 */
+} ct_model_desc;
+
+/* Weight pointers: `weights[6*i + j]` for layer i, host FP32, read-only,
+ * copied by ct_build:
+ *   j = 0  conv: W [cout, cin, k, k] (OIHW); fc: W [cout, cin]
+ *   j = 1  bias [cout] or NULL (zero)
+ *   j = 2..5  BatchNorm gamma, beta, running mean, running var [cout]
+ *          (conv with bn = 1 only; otherwise NULL). */
+#define CT_WEIGHTS_PER_LAYER 6
+
+/* flags for ct_build_opts.flags */
+#define CT_FLAG_SIMT_ONLY 1u      /* use the CUDA-core conv kernels everywhere */
+
+typedef struct {
+    int32_t precision;   /* ct_precision: storage type of weights and activations */
+    int32_t protect;     /* 1: add carry-through filters and the checksum neuron;
+                            0: the same network and kernels without them */
+    int32_t ds_mode;     /* ct_ds_mode */
+    int32_t device;      /* CUDA device ordinal */
+    int32_t max_batch;   /* workspaces are sized for this many images */
+    uint32_t flags;
+} ct_build_opts;
+
+typedef struct ct_model ct_model;
+
+/* ct_build -- Sec. II-A/II-B construction.  Folds BatchNorm (Eq. 1) into the
+ * convolutions in double precision with the identity (scale exactly 1, bias
+ * 0) on every checksum channel; appends a carry-through filter to every
+ * CT_ROLE_CT convolution; leaves the checksum input out of every data filter
+ * (its zero slice is structural); adds one all-ones neuron to every hidden
+ * FC layer and the accumulated-checksum neuron to the final one; rounds to
+ * the storage precision; converts to the device layouts and uploads.
+ * Synchronous.  On success *out owns device memory until ct_destroy.
+ * Errors: CT_EINVAL (malformed description), CT_EUNSUPPORTED, CT_ENOMEM,
+ * CT_ECUDA.  Nothing is allocated on failure. */
+ct_status ct_build(const ct_model_desc *desc, const float *const *weights,
+                   const ct_build_opts *opts, ct_model **out);
+
+/* ct_set_threshold -- Sec. II-B detection rule: an image is flagged when
+ * NOT(|S - reference| <= tau), so a NaN or infinite S is always flagged.
+ * tau must be >= 0 (CT_EINVAL otherwise).  A new model has tau = +inf. */
+ct_status ct_set_threshold(ct_model *m, double reference, double tau);
+ct_status ct_get_threshold(const ct_model *m, double *reference, double *tau);
+
+/* ct_infer -- Sec. II-B.  Runs `batch` images through the network.
+ *   input_dev  FP32 NCHW [batch, in_c, in_h, in_w], read-only.
+ *   logits_dev FP32 [batch, n_classes], written.
+ *   S_dev      FP32 [batch]: the accumulated-checksum neuron (NULL allowed;
+ *              NaN for an unprotected model).
+ *   flag_dev   uint8 [batch]: 1 = flagged (NULL allowed; 0 when unprotected).
+ * An armed fault (ct_inject) is applied during this call and disarmed:
+ * a weight fault flips the stored word before the layer runs and flips it
+ * back after; an activation fault flips the stored word of the layer's
+ * input tensor after its producer wrote it and before any reader.
+ * Errors: CT_ERANGE if batch < 1 or batch > max_batch; CT_ECUDA. */
+ct_status ct_infer(ct_model *m, const float *input_dev, int32_t batch, float *logits_dev,
+                   float *S_dev, uint8_t *flag_dev, void *stream);
+
+/* ct_inject -- Sec. III-A fault model: arms ONE transient single-bit flip
+ * for the next ct_infer.  `layer` indexes desc->layers and must be a CONV.
+ * `element` is a flat index into the literal layout of the protected
+ * network, where the checksum is the last channel:
+ *   CT_BUF_WEIGHT: [C_out_tot, C_in_tot, k, k] of that layer (carry-through
+ *     row and zero checksum slice included);
+ *   CT_BUF_ACT:    [batch, C_tot, H, W] of that layer's input tensor, for
+ *     the batch of the next ct_infer.
+ * `bit` is in [0, 32) for FP32 and [0, 16) for FP16 storage.
+ * Errors: CT_EINVAL (not a conv layer, bad kind), CT_ERANGE (element or bit
+ * out of range; an activation element is range-checked again by ct_infer
+ * against its batch). */
+ct_status ct_inject(ct_model *m, int32_t kind, int32_t layer, int64_t element, int32_t bit);
+ct_status ct_clear_faults(ct_model *m);
+
+/* ct_reexecute -- Sec. II-B mitigation.  Re-runs, fault-free, only the
+ * images whose flag_dev entry is non-zero and overwrites their rows of
+ * logits_dev and S_dev (the re-run's own flags are ignored; flag_dev is not
+ * modified).  Synchronises `stream` once to read the flags.  *n_rerun
+ * (host) receives the number of images re-run.  Same buffers as ct_infer.
+ * An armed fault stays armed for the next ct_infer. */
+ct_status ct_reexecute(ct_model *m, const float *input_dev, int32_t batch,
+                       const uint8_t *flag_dev, float *logits_dev, float *S_dev,
+                       int32_t *n_rerun, void *stream);
+
+/* ct_run_host -- end-to-end call for callers with host buffers: copies the
+ * input from host memory, runs ct_infer and ct_reexecute, and copies
+ * logits, S and flags back.  Returns after the results are in host memory.
+ * Pinned host memory gives asynchronous copies; pageable memory works. */
+ct_status ct_run_host(ct_model *m, const float *input_host, int32_t batch, float *logits_host,
+                      float *S_host, uint8_t *flag_host, int32_t *n_rerun, void *stream);
+
+/* ct_calibrate -- Sec. II-C distribution-based threshold, host arithmetic:
+ * reference = mean of the n fault-free S values, tau = the nearest-rank
+ * ceil((1 - alpha) * n)-th smallest |S - reference|.  CT_EINVAL for n < 1,
+ * alpha outside [0, 1) or a non-finite S. */
+ct_status ct_calibrate(const float *S_host, int64_t n, double alpha, double *reference,
+                       double *tau);
+
+/* Fault-able buffers of the protected network for a given batch, in the
+ * order used by campaign drivers: every conv weight tensor, then every
+ * distinct tensor read by a convolution (the network input excluded),
+ * addressed by the first convolution that reads it. */
+ct_status ct_buffer_count(const ct_model *m, int32_t batch, int32_t *n);
+ct_status ct_buffer_info(const ct_model *m, int32_t batch, int32_t i, int32_t *kind,
+                         int32_t *layer, int64_t *n_elements, int32_t *bits);
+
+/* Per-launch kernel timing with CUDA events recorded on the launch stream
+ * (off by default).  ct_profile_read returns, for one kernel family, the
+ * launches, milliseconds and algorithmic FLOPs accumulated since the last
+ * read of that family, then resets it.  It synchronises on the recorded
+ * events.  Families: 0 = tensor-core conv, 1 = CUDA-core conv, 2 = FC,
+ * 3 = pooling, 4 = other. */
+ct_status ct_profile_enable(ct_model *m, int32_t on);
+ct_status ct_profile_read(ct_model *m, int32_t family, int64_t *launches, double *ms,
+                          double *flops);
+
+/* Number of kernels one fault-free ct_infer of this model launches. */
+ct_status ct_launches_per_infer(const ct_model *m, int32_t *n);
+
+/* ct_copy_activation -- diagnostic read of an intermediate tensor of the
+ * last ct_infer on `stream`: slot `slot` (0 = converted input; the `dst` of
+ * a layer otherwise) for the first `batch` images.  data_host receives the
+ * data channels in the device layout, NHWC [batch, H, W, C] (FP32 features
+ * [batch, C] after a global average pool, [batch, n] after a hidden FC), in
+ * the slot's storage type (FP32, or FP16 words as uint16); cs_host (may be
+ * NULL) receives the checksum plane [batch, H, W] in the same type.
+ * *C, *H, *W, *has_cs and *elem_bytes describe the slot (any may be NULL; call
+ * first with data_host = NULL to query).  Synchronous.  CT_ERANGE for a slot
+ * that is not stored (the classifier output) or batch > max_batch. */
+ct_status ct_copy_activation(ct_model *m, int32_t slot, int32_t batch, void *data_host, void *cs_host,
+                             int32_t *C, int32_t *H, int32_t *W, int32_t *has_cs,
+                             int32_t *elem_bytes, void *stream);
+
+/* Reads and clears the model's device-side error word (set by a kernel whose
+ * bounded wait expired).  Synchronises the model's device. */
+ct_status ct_device_error(ct_model *m, uint32_t *code);
+
+void ct_destroy(ct_model *m);
+const char *ct_strerror(ct_status s);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* CT_H */

@@ -1,0 +1,494 @@
+// Tensor-core (tcgen05) implicit-GEMM convolution with the carry-through
+// filter, FP16 storage, FP32 accumulation in TMEM.
+//
+// GEMM view: D[m, n] = sum_k A[m, k] B[n, k] with m = output pixel (n, p, q),
+// n = output channel, k = (tap, channel), channels innermost.
+//   A (128 pixels x 64 channels of one tap) is fetched by TMA in im2col mode
+//     from the NHWC input: the TMA unit walks consecutive output pixels,
+//     applies stride and zero padding, and writes the 128-byte swizzled
+//     K-major tile the MMA reads.
+//   B (BN channels x 64) is fetched by tiled TMA from the KRSC weights.
+//   The carry-through filter of Sec. II-A is one more GEMM row: coef at the
+//     centre tap of every input channel, 0 elsewhere.  Its non-zero part is a
+//     constant 16-row tile (row 0 = coef, rows 1-15 = 0) kept in shared
+//     memory, so the tensor core itself computes the checksum column on the
+//     centre-tap K blocks, which the K loop visits first: as 16 extra columns
+//     of the same MMA when BN + 16 <= 256, else as a separate N = 16 MMA.
+//   The incoming checksum plane (weight coef at the centre) and the
+//   epilogue (bias, residual, ReLU) are applied by the epilogue warps.
+//
+// Warp roles (192 threads): warp 0 issues TMA, warp 1 allocates TMEM and
+// issues tcgen05.mma (one elected lane), warps 2-5 read the accumulator
+// (each thread owns one output pixel) and store data and checksum.
+// Every mbarrier wait is bounded; on expiry the kernel records an error code
+// in a device word, stops issuing work and exits after releasing TMEM.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <string.h>
+
+#include <mutex>
+
+#include "ct_internal.h"
+
+namespace ct {
+
+namespace {
+
+constexpr int BM = 128;            // output pixels per tile (TMEM lanes)
+constexpr int BK = 64;             // channels per K block (128 bytes of fp16)
+constexpr int A_BYTES = BM * BK * 2;
+constexpr int NTHREADS = 192;
+constexpr uint64_t WAIT_NS = 2000000000ull;   // 2 s bound on any single wait
+
+enum CtMode { CT_NONE_ = 0, CT_MERGED = 1, CT_SEPARATE = 2 };
+
+struct TcGeom {
+    int M, PQ, Q, stride, pad, C, K, RSC;
+    int n_kb, cpb, ctr_tap, S;
+    int ct_mode;
+    int tmem_cols;
+    uint16_t coef_h;
+};
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ uint64_t globaltimer() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count));
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Bounded wait: true on completion, false (and error code recorded) after WAIT_NS.
+__device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint32_t *err, uint32_t code) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = globaltimer();
+    for (uint32_t it = 0;; ++it) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if ((it & 63) == 63) {
+            if (globaltimer() - t0 > WAIT_NS) {
+                atomicOr(err, code);
+                return false;
+            }
+            __nanosleep(128);
+        }
+    }
+}
+
+__device__ __forceinline__ void tma_load_im2col(uint32_t dst, const CUtensorMap *map, uint32_t bar, int c,
+                                                int w, int h, int n, uint16_t ow, uint16_t oh) {
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.im2col.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3, %4, %5}], [%6], {%7, %8};" ::"r"(dst),
+        "l"((uint64_t)map), "r"(c), "r"(w), "r"(h), "r"(n), "r"(bar), "h"(ow), "h"(oh)
+        : "memory");
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, uint32_t bar, int x, int y) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+        "l"((uint64_t)map), "r"(x), "r"(y), "r"(bar)
+        : "memory");
+}
+
+// UMMA shared-memory descriptor: K-major operand, 128-byte swizzle, 8-row
+// atoms of 1024 bytes (SBO), start address in 16-byte units.
+__device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t addr) {
+    uint64_t d = 0;
+    d |= (uint64_t)((addr >> 4) & 0x3FFF);
+    d |= (uint64_t)1 << 16;                 // LBO (unused for swizzled K-major)
+    d |= (uint64_t)(1024 >> 4) << 32;       // SBO: 8 rows x 128 B
+    d |= (uint64_t)1 << 46;                 // descriptor version
+    d |= (uint64_t)2 << 61;                 // SWIZZLE_128B
+    return d;
+}
+
+// Instruction descriptor: kind::f16, A = B = F16, D = F32, both K-major.
+__host__ __device__ constexpr uint32_t idesc_f16(int M, int N) {
+    return (1u << 4) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+__device__ __forceinline__ void umma_f16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(a), "l"(b), "r"(idesc), "r"(acc));
+}
+
+__device__ __forceinline__ void umma_commit(uint32_t bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+                 : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float *v) {
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+__device__ __forceinline__ float tmem_ld1(uint32_t taddr) {
+    uint32_t r;
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(r) : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+    return __uint_as_float(r);
+}
+
+__device__ __forceinline__ float relu_keep_nan(float v) { return v < 0.f ? 0.f : v; }
+
+__device__ __forceinline__ float ldh(const __half *p, size_t i) { return __half2float(p[i]); }
+
+// tap visited at K-block kb: the centre tap first, the others in order
+__device__ __forceinline__ int tap_of(int t, int ctr) { return t == 0 ? ctr : (t <= ctr ? t - 1 : t); }
+
+template <int BN, int STAGES>
+__global__ void __launch_bounds__(NTHREADS, BN <= 128 ? 2 : 1)
+conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
+               const ConvArgs a, const TcGeom g) {
+    constexpr int B_ROWS = BN + 16;                       // 16 constant carry-through rows
+    constexpr int B_BYTES_STAGE = B_ROWS * BK * 2;
+    constexpr int B_TMA_BYTES = BN * BK * 2;
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint8_t *As = smem;
+    uint8_t *Bs = As + STAGES * A_BYTES;
+    uint8_t *CTt = Bs + STAGES * B_BYTES_STAGE;           // separate 16-row carry-through tile
+    uint64_t *full = (uint64_t *)(CTt + 16 * BK * 2);
+    uint64_t *empty = full + STAGES;
+    uint64_t *accum = empty + STAGES;
+    uint32_t *tmem_holder = (uint32_t *)(accum + 1);
+    volatile uint32_t *abort_flag = tmem_holder + 1;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int m0 = blockIdx.x * BM;
+    const int n_tile = blockIdx.y;
+    const bool ct_here = g.ct_mode != CT_NONE_ && n_tile == 0;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(smem_u32(&full[s]), 1);
+            mbar_init(smem_u32(&empty[s]), 1);
+        }
+        mbar_init(smem_u32(accum), 1);
+        *abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_holder)),
+                     "r"((uint32_t)g.tmem_cols));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    if (warp >= 2) {
+        // constant carry-through rows: row 0 = coef, rows 1..15 = 0 (swizzle-invariant)
+        const uint32_t coef2 = (uint32_t)g.coef_h | ((uint32_t)g.coef_h << 16);
+        const int t = threadIdx.x - 64;
+        for (int s = 0; s < STAGES; ++s) {
+            uint32_t *rows = (uint32_t *)(Bs + s * B_BYTES_STAGE + BN * BK * 2);
+            for (int i = t; i < 16 * BK / 2; i += 128) rows[i] = (i < BK / 2) ? coef2 : 0u;
+        }
+        uint32_t *ctt = (uint32_t *)CTt;
+        for (int i = t; i < 16 * BK / 2; i += 128) ctt[i] = (i < BK / 2) ? coef2 : 0u;
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tmem = *tmem_holder;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            // ---------------- TMA producer ----------------
+            const int nimg = m0 / g.PQ, rem = m0 % g.PQ;
+            const int p = rem / g.Q, q = rem % g.Q;
+            const int w0 = q * g.stride - g.pad, h0 = p * g.stride - g.pad;
+            for (int kb = 0; kb < g.n_kb; ++kb) {
+                const int s = kb % STAGES;
+                const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
+                if (!mbar_wait(smem_u32(&empty[s]), ph ^ 1u, a.err, 1u)) { *abort_flag = 1; break; }
+                if (*abort_flag) break;
+                const int tap = tap_of(kb / g.cpb, g.ctr_tap);
+                const int c0 = (kb % g.cpb) * BK;
+                const int r = tap / g.S, sx = tap % g.S;
+                const uint32_t fb = smem_u32(&full[s]);
+                mbar_expect_tx(fb, A_BYTES + B_TMA_BYTES);
+                tma_load_im2col(smem_u32(As + s * A_BYTES), &amap, fb, c0, w0, h0, nimg, (uint16_t)sx, (uint16_t)r);
+                tma_load_2d(smem_u32(Bs + s * B_BYTES_STAGE), &bmap, fb, tap * g.C + c0, n_tile * BN);
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            // ---------------- MMA issuer ----------------
+            const uint32_t id_main = idesc_f16(BM, BN);
+            const uint32_t id_merged = idesc_f16(BM, BN + 16);
+            const uint32_t id_ct = idesc_f16(BM, 16);
+            const int n_centre = g.cpb;
+            for (int kb = 0; kb < g.n_kb; ++kb) {
+                const int s = kb % STAGES;
+                const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
+                if (!mbar_wait(smem_u32(&full[s]), ph, a.err, 2u)) { *abort_flag = 1; break; }
+                if (*abort_flag) break;
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                const bool centre = kb < n_centre;
+                const uint32_t a_base = smem_u32(As + s * A_BYTES);
+                const uint32_t b_base = smem_u32(Bs + s * B_BYTES_STAGE);
+#pragma unroll
+                for (int k16 = 0; k16 < BK / 16; ++k16) {
+                    const uint64_t ad = smem_desc_sw128(a_base + k16 * 32);
+                    const uint64_t bd = smem_desc_sw128(b_base + k16 * 32);
+                    const uint32_t acc = (kb > 0 || k16 > 0) ? 1u : 0u;
+                    if (ct_here && centre && g.ct_mode == CT_MERGED) {
+                        umma_f16(tmem, ad, bd, id_merged, acc);
+                    } else {
+                        umma_f16(tmem, ad, bd, id_main, acc);
+                        if (ct_here && centre && g.ct_mode == CT_SEPARATE)
+                            umma_f16(tmem + BN, ad, smem_desc_sw128(smem_u32(CTt) + k16 * 32), id_ct, acc);
+                    }
+                }
+                umma_commit(smem_u32(&empty[s]));
+            }
+            umma_commit(smem_u32(accum));      // fires when every MMA issued above has completed
+        }
+    } else {
+        // ---------------- epilogue: warps 2..5, one output pixel per thread ----------------
+        const int quad = warp & 3;
+        const int row = quad * 32 + lane;
+        const int m = m0 + row;
+        bool ok = mbar_wait(smem_u32(accum), 0u, a.err, 4u) && !*abort_flag;
+        ok = __all_sync(0xffffffffu, ok);          // tcgen05.ld below is warp-collective
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        if (ok) {
+            const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
+            const bool valid = m < g.M;
+            const int mm = valid ? m : 0;
+            const int nimg = mm / g.PQ, rem = mm % g.PQ, p = rem / g.Q, q = rem % g.Q;
+            const __half *x = static_cast<const __half *>(a.x);
+            const __half *res = static_cast<const __half *>(a.res);
+            __half *y = static_cast<__half *>(a.y);
+            const FaultDelta fd = a.fd;
+            float fsrc = 0.f;
+            if (fd.active) {
+                const int h = p * g.stride + fd.r - g.pad, w = q * g.stride + fd.s - g.pad;
+                if (h >= 0 && h < a.H && w >= 0 && w < a.W) {
+                    if (fd.cin < g.C) fsrc = ldh(x, (((size_t)nimg * a.H + h) * a.W + w) * g.C + fd.cin);
+                    else if (a.cs_in) fsrc = ldh(static_cast<const __half *>(a.cs_in), ((size_t)nimg * a.H + h) * a.W + w);
+                }
+            }
+            const int n0 = n_tile * BN;
+#pragma unroll 1
+            for (int ch = 0; ch < BN; ch += 16) {
+                float v[16];
+                tmem_ld16(trow + ch, v);
+                if (valid) {
+                    const size_t base = (size_t)m * g.K + n0 + ch;
+                    float rv[16];
+                    if (res) {
+                        const uint4 *rp = reinterpret_cast<const uint4 *>(res + base);
+                        uint4 r0 = rp[0], r1 = rp[1];
+                        const __half2 *h0 = reinterpret_cast<const __half2 *>(&r0);
+                        const __half2 *h1 = reinterpret_cast<const __half2 *>(&r1);
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) {
+                            float2 f0 = __half22float2(h0[i]), f1 = __half22float2(h1[i]);
+                            rv[2 * i] = f0.x; rv[2 * i + 1] = f0.y; rv[8 + 2 * i] = f1.x; rv[8 + 2 * i + 1] = f1.y;
+                        }
+                    }
+                    uint32_t packed[8];
+#pragma unroll
+                    for (int i = 0; i < 16; i += 2) {
+                        float o[2];
+#pragma unroll
+                        for (int j = 0; j < 2; ++j) {
+                            const int k = n0 + ch + i + j;
+                            float t = v[i + j] + a.bias[k];
+                            if (fd.active && fd.kout == k) t += fd.dv * fsrc;
+                            if (res) t += rv[i + j];
+                            if (a.relu) t = relu_keep_nan(t);
+                            o[j] = t;
+                        }
+                        __half2 hh = __floats2half2_rn(o[0], o[1]);
+                        packed[i / 2] = *reinterpret_cast<uint32_t *>(&hh);
+                    }
+                    uint4 *yp = reinterpret_cast<uint4 *>(y + base);
+                    yp[0] = make_uint4(packed[0], packed[1], packed[2], packed[3]);
+                    yp[1] = make_uint4(packed[4], packed[5], packed[6], packed[7]);
+                }
+            }
+            // checksum output
+            if (a.cs_out != nullptr && n_tile == 0) {
+                float ctv = 0.f;
+                if (g.ct_mode != CT_NONE_) ctv = tmem_ld1(trow + BN);
+                if (valid) {
+                    const __half *csi = static_cast<const __half *>(a.cs_in);
+                    const int ctr_r = g.ctr_tap / g.S, ctr_s = g.ctr_tap % g.S;
+                    const int hc = p * g.stride + ctr_r - g.pad, wc = q * g.stride + ctr_s - g.pad;
+                    const bool inb = hc >= 0 && hc < a.H && wc >= 0 && wc < a.W;
+                    const float cin = (csi && inb) ? ldh(csi, ((size_t)nimg * a.H + hc) * a.W + wc) : 0.f;
+                    float o = 0.f;
+                    if (a.role == CT_ROLE_CT) o = ctv + a.coef * cin;
+                    else if (a.role == CT_ROLE_PASS) o = cin;
+                    if (fd.active && fd.kout == g.K) o += fd.dv * fsrc;
+                    if (a.res_cs) o += ldh(static_cast<const __half *>(a.res_cs), (size_t)m);
+                    if (a.relu) o = relu_keep_nan(o);
+                    static_cast<__half *>(a.cs_out)[m] = __float2half_rn(o);
+                }
+            }
+        }
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if (warp == 1) {
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)g.tmem_cols));
+    }
+}
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+
+PFN_cuTensorMapEncodeTiled_v12000 g_encode_tiled = nullptr;
+PFN_cuTensorMapEncodeIm2col_v12000 g_encode_im2col = nullptr;
+std::once_flag g_once;
+
+bool load_encoders() {
+    std::call_once(g_once, [] {
+        cudaDriverEntryPointQueryResult q;
+        void *p = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess && q == cudaDriverEntryPointSuccess)
+            g_encode_tiled = (PFN_cuTensorMapEncodeTiled_v12000)p;
+        p = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeIm2col", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess && q == cudaDriverEntryPointSuccess)
+            g_encode_im2col = (PFN_cuTensorMapEncodeIm2col_v12000)p;
+    });
+    return g_encode_tiled && g_encode_im2col;
+}
+
+template <int BN, int STAGES>
+size_t smem_bytes() {
+    return 1024 + (size_t)STAGES * (A_BYTES + (BN + 16) * BK * 2) + 16 * BK * 2 + 8 * (2 * STAGES + 1) + 16;
+}
+
+uint16_t coef_half_bits(float c) {
+    __half h = __float2half_rn(c);        // exact: coefficients are powers of two
+    uint16_t b;
+    memcpy(&b, &h, 2);
+    return b;
+}
+
+}  // namespace
+
+struct TcPlan {
+    CUtensorMap amap;
+    CUtensorMap bmap;
+    TcGeom g;
+    int BN, stages, n_tiles;
+    size_t smem;
+};
+
+bool tc_supported(int C, int K, int R, int S, int stride, int pad, std::string *why) {
+    if (C % BK != 0) { if (why) *why = "input channels not a multiple of 64"; return false; }
+    if (!(K == 64 || K == 128 || K % 256 == 0)) { if (why) *why = "output channels"; return false; }
+    if (R != S || R > 7 || stride < 1 || stride > 2 || pad > 3 || pad > R / 2 + 1) {
+        if (why) *why = "filter geometry";
+        return false;
+    }
+    return true;
+}
+
+TcPlan *tc_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, const void *x_dev, std::string *why) {
+    if (!load_encoders()) { if (why) *why = "tensor-map encoders unavailable"; return nullptr; }
+    TcPlan *pl = new TcPlan();
+    memset(pl, 0, sizeof(*pl));
+    pl->BN = a.K <= 256 ? a.K : 256;
+    pl->n_tiles = a.K / pl->BN;
+    pl->stages = pl->BN == 128 ? 3 : 4;
+    TcGeom &g = pl->g;
+    g.PQ = a.P * a.Q; g.Q = a.Q; g.stride = a.stride; g.pad = a.pad; g.C = a.C; g.K = a.K;
+    g.RSC = a.R * a.S * a.C; g.S = a.S;
+    g.cpb = a.C / BK;
+    g.n_kb = a.R * a.S * g.cpb;
+    g.ctr_tap = ((a.R - 1) / 2) * a.S + (a.S - 1) / 2;
+    g.ct_mode = a.role != CT_ROLE_CT ? CT_NONE_ : (pl->BN + 16 <= 256 && pl->n_tiles == 1 ? CT_MERGED : CT_SEPARATE);
+    const int cols = pl->BN + (g.ct_mode != CT_NONE_ ? 16 : 0);
+    g.tmem_cols = cols <= 32 ? 32 : cols <= 64 ? 64 : cols <= 128 ? 128 : cols <= 256 ? 256 : 512;
+    g.coef_h = coef_half_bits(a.coef);
+    // A: im2col view of the NHWC input [max_batch, H, W, C]
+    cuuint64_t gdim[4] = {(cuuint64_t)a.C, (cuuint64_t)a.W, (cuuint64_t)a.H, (cuuint64_t)max_batch};
+    cuuint64_t gstr[3] = {(cuuint64_t)a.C * 2, (cuuint64_t)a.W * a.C * 2, (cuuint64_t)a.H * a.W * a.C * 2};
+    int lower[2] = {-a.pad, -a.pad};
+    int upper[2] = {a.pad - (a.S - 1), a.pad - (a.R - 1)};
+    cuuint32_t estr[4] = {1, (cuuint32_t)a.stride, (cuuint32_t)a.stride, 1};
+    CUresult r = g_encode_im2col(&pl->amap, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<void *>(x_dev), gdim, gstr,
+                                 lower, upper, BK, BM, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                                 CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) { if (why) *why = "im2col tensor map"; delete pl; return nullptr; }
+    // B: weights [K, R*S*C] fp16, K-major rows
+    cuuint64_t bdim[2] = {(cuuint64_t)g.RSC, (cuuint64_t)a.K};
+    cuuint64_t bstr[1] = {(cuuint64_t)g.RSC * 2};
+    cuuint32_t box[2] = {BK, (cuuint32_t)pl->BN};
+    cuuint32_t bes[2] = {1, 1};
+    r = g_encode_tiled(&pl->bmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void *>(w_dev), bdim, bstr, box, bes,
+                       CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                       CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) { if (why) *why = "weight tensor map"; delete pl; return nullptr; }
+    cudaError_t e;
+    if (pl->BN == 64) {
+        pl->smem = smem_bytes<64, 4>();
+        e = cudaFuncSetAttribute(conv_tc_kernel<64, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
+    } else if (pl->BN == 128) {
+        pl->smem = smem_bytes<128, 3>();
+        e = cudaFuncSetAttribute(conv_tc_kernel<128, 3>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
+    } else {
+        pl->smem = smem_bytes<256, 4>();
+        e = cudaFuncSetAttribute(conv_tc_kernel<256, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
+    }
+    if (e != cudaSuccess) { if (why) *why = "shared memory attribute"; delete pl; return nullptr; }
+    return pl;
+}
+
+void tc_plan_destroy(TcPlan *p) { delete p; }
+
+cudaError_t launch_conv_tc(const ConvArgs &a, const void *plan, cudaStream_t st) {
+    const TcPlan *pl = static_cast<const TcPlan *>(plan);
+    TcGeom g = pl->g;
+    g.M = a.N * a.P * a.Q;
+    dim3 grid((g.M + BM - 1) / BM, pl->n_tiles);
+    if (pl->BN == 64) conv_tc_kernel<64, 4><<<grid, NTHREADS, pl->smem, st>>>(pl->amap, pl->bmap, a, g);
+    else if (pl->BN == 128) conv_tc_kernel<128, 3><<<grid, NTHREADS, pl->smem, st>>>(pl->amap, pl->bmap, a, g);
+    else conv_tc_kernel<256, 4><<<grid, NTHREADS, pl->smem, st>>>(pl->amap, pl->bmap, a, g);
+    return cudaGetLastError();
+}
+
+}  // namespace ct

@@ -1,0 +1,810 @@
+// libct C ABI: model construction (Sec. II-A/II-B), inference orchestration,
+// fault injection (Sec. III-A), re-execution (Sec. II-B) and calibration
+// (Sec. II-C).  Every arithmetic step of inference runs in this library's
+// CUDA kernels; the host only builds weights and launches.
+#include <math.h>
+#include <string.h>
+
+#include <algorithm>
+#include <memory>
+#include <new>
+#include <vector>
+
+#include "ct_internal.h"
+
+using namespace ct;
+
+namespace {
+
+// ---------------------------------------------------------------------------
+// storage rounding (host)
+// ---------------------------------------------------------------------------
+
+// IEEE binary64 -> binary16, round to nearest even, directly (no float step).
+uint16_t double_to_half_bits(double d) {
+    uint64_t u;
+    memcpy(&u, &d, 8);
+    const uint16_t sign = (uint16_t)((u >> 48) & 0x8000u);
+    const uint64_t mag = u & 0x7FFFFFFFFFFFFFFFull;
+    if (mag >= 0x7FF0000000000000ull) return sign | (mag > 0x7FF0000000000000ull ? 0x7E00 : 0x7C00);
+    const int e = (int)(mag >> 52) - 1023;
+    if (e == -1023) return sign;                                // binary64 subnormal: below half's range
+    const uint64_t full = (mag & ((1ull << 52) - 1)) | (1ull << 52);   // 53-bit significand
+    if (e >= 16) return sign | 0x7C00;
+    if (e >= -14) {                                             // half normal range
+        uint64_t hm = full >> 42, rem = full & ((1ull << 42) - 1), hlf = 1ull << 41;
+        int ee = e;
+        if (rem > hlf || (rem == hlf && (hm & 1))) ++hm;
+        if (hm == 2048) { hm = 1024; ++ee; }
+        if (ee >= 16) return sign | 0x7C00;
+        return (uint16_t)(sign | ((ee + 15) << 10) | (hm & 0x3FF));
+    }
+    const int shift = 28 - e;                                   // value / 2^-24 = full >> shift
+    if (shift >= 54) return sign;
+    uint64_t m = full >> shift, rem = full & ((1ull << shift) - 1), hlf = 1ull << (shift - 1);
+    if (rem > hlf || (rem == hlf && (m & 1))) ++m;
+    return (uint16_t)(sign | m);                               // m == 1024 encodes 2^-14
+}
+
+float half_bits_to_float(uint16_t h) {
+    const uint32_t sign = (uint32_t)(h & 0x8000) << 16;
+    const uint32_t e = (h >> 10) & 0x1F, m = h & 0x3FF;
+    uint32_t bits;
+    if (e == 0x1F) bits = sign | 0x7F800000u | (m << 13);
+    else if (e == 0) {
+        if (m == 0) bits = sign;
+        else {
+            float v = ldexpf((float)m, -24);
+            memcpy(&bits, &v, 4);
+            bits |= sign;
+        }
+    } else bits = sign | ((e + 112) << 23) | (m << 13);
+    float f;
+    memcpy(&f, &bits, 4);
+    return f;
+}
+
+uint32_t float_bits(float f) { uint32_t u; memcpy(&u, &f, 4); return u; }
+float bits_float(uint32_t u) { float f; memcpy(&f, &u, 4); return f; }
+
+// ---------------------------------------------------------------------------
+// model
+// ---------------------------------------------------------------------------
+
+struct Slot {
+    int C = 0, H = 0, W = 0;
+    bool has_cs = false;
+    bool is_float = false;       // GAP output: fp32 features whatever the precision
+    void *data = nullptr;
+    void *cs = nullptr;
+};
+
+struct LayerRT {
+    ct_layer_desc d{};
+    int role = CT_ROLE_NONE;     // effective role (protect / ds_mode applied)
+    // conv
+    int C = 0, K = 0, R = 0, S = 0, H = 0, W = 0, P = 0, Q = 0;
+    bool cs_in = false, cs_out = false;
+    float coef = 1.f;
+    void *w = nullptr;
+    float *bias = nullptr;
+    bool tc = false;
+    TcPlan *plan = nullptr;
+    // fc
+    int n_in = 0, n_cs = 0, n_out = 0;
+    bool x_float = false;
+};
+
+struct EvRec { int fam; int ev; double flops; };
+
+}  // namespace
+
+struct ct_model {
+    int device = 0;
+    int prec = CT_FP32;
+    bool protect = true;
+    int ds_mode = CT_DS_PASS;
+    int max_batch = 0;
+    uint32_t flags = 0;
+    int in_c = 0, in_h = 0, in_w = 0, n_classes = 0;
+    std::vector<LayerRT> L;
+    std::vector<Slot> slots;
+    double ref = 0.0, tau = INFINITY;
+    // armed fault
+    bool armed = false;
+    int f_kind = 0, f_layer = 0, f_bit = 0;
+    int64_t f_elem = 0;
+    // scratch owned by the library
+    float *re_input = nullptr, *re_logits = nullptr, *re_S = nullptr;
+    uint8_t *re_flag = nullptr;
+    int32_t *re_idx = nullptr;
+    uint8_t *h_flags = nullptr;
+    int32_t *h_idx = nullptr;
+    float *rh_input = nullptr, *rh_logits = nullptr, *rh_S = nullptr;
+    uint8_t *rh_flag = nullptr;
+    uint32_t *d_err = nullptr;
+    std::vector<void *> dev_allocs;
+    // profiling
+    bool prof = false;
+    std::vector<std::pair<cudaEvent_t, cudaEvent_t>> ev_pool;
+    std::vector<int> ev_free;
+    std::vector<EvRec> recs;
+
+    size_t esz() const { return prec == CT_FP16 ? 2 : 4; }
+};
+
+namespace {
+
+#define CUDA_TRY(x)                                   \
+    do {                                              \
+        cudaError_t e__ = (x);                        \
+        if (e__ != cudaSuccess) return CT_ECUDA;      \
+    } while (0)
+
+struct DeviceGuard {
+    int prev = -1;
+    explicit DeviceGuard(int dev) {
+        if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
+        cudaSetDevice(dev);
+    }
+    ~DeviceGuard() { if (prev >= 0) cudaSetDevice(prev); }
+};
+
+ct_status dalloc(ct_model *m, void **p, size_t bytes) {
+    if (bytes == 0) bytes = 16;
+    if (cudaMalloc(p, bytes) != cudaSuccess) { cudaGetLastError(); return CT_ENOMEM; }
+    m->dev_allocs.push_back(*p);
+    return CT_OK;
+}
+
+void free_all(ct_model *m) {
+    for (auto &l : m->L)
+        if (l.plan) tc_plan_destroy(l.plan);
+    for (void *p : m->dev_allocs) cudaFree(p);
+    m->dev_allocs.clear();
+    if (m->h_flags) cudaFreeHost(m->h_flags);
+    if (m->h_idx) cudaFreeHost(m->h_idx);
+    for (auto &e : m->ev_pool) { cudaEventDestroy(e.first); cudaEventDestroy(e.second); }
+    m->ev_pool.clear();
+}
+
+// store a double as the storage word (fp32 or fp16) into a byte buffer
+void put(std::vector<uint8_t> &buf, size_t i, double v, int prec) {
+    if (prec == CT_FP16) {
+        uint16_t h = double_to_half_bits(v);
+        memcpy(&buf[i * 2], &h, 2);
+    } else {
+        float f = (float)v;
+        memcpy(&buf[i * 4], &f, 4);
+    }
+}
+
+// value of a storage word after flipping `bit`, as float
+float flipped(double stored, int bit, int prec) {
+    if (prec == CT_FP16) return half_bits_to_float((uint16_t)(double_to_half_bits(stored) ^ (1u << bit)));
+    return bits_float(float_bits((float)stored) ^ (1u << bit));
+}
+
+// ---------------------------------------------------------------------------
+// profiling helpers
+// ---------------------------------------------------------------------------
+
+template <typename F>
+cudaError_t launch(ct_model *m, int fam, double flops, cudaStream_t st, F &&fn) {
+    if (!m->prof) return fn();
+    int ev;
+    if (!m->ev_free.empty()) { ev = m->ev_free.back(); m->ev_free.pop_back(); }
+    else {
+        cudaEvent_t a, b;
+        if (cudaEventCreate(&a) != cudaSuccess) return cudaErrorMemoryAllocation;
+        if (cudaEventCreate(&b) != cudaSuccess) { cudaEventDestroy(a); return cudaErrorMemoryAllocation; }
+        m->ev_pool.push_back({a, b});
+        ev = (int)m->ev_pool.size() - 1;
+    }
+    cudaEventRecord(m->ev_pool[ev].first, st);
+    cudaError_t e = fn();
+    cudaEventRecord(m->ev_pool[ev].second, st);
+    m->recs.push_back({fam, ev, flops});
+    return e;
+}
+
+// ---------------------------------------------------------------------------
+// build
+// ---------------------------------------------------------------------------
+
+ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const *wts) {
+    const int nL = desc->n_layers;
+    int max_slot = 0;
+    for (int i = 0; i < nL; ++i) {
+        const ct_layer_desc &d = desc->layers[i];
+        if (d.src < 0 || d.dst <= 0) return CT_EINVAL;
+        max_slot = std::max(max_slot, std::max(d.dst, d.src));
+    }
+    std::vector<int> defined(max_slot + 1, 0);
+    m->slots.assign(max_slot + 1, Slot());
+    Slot &in = m->slots[0];
+    in.C = desc->in_c; in.H = desc->in_h; in.W = desc->in_w;
+    defined[0] = 1;
+    const int prec = m->prec;
+    const size_t esz = m->esz();
+    const int B = m->max_batch;
+    int n_final = 0;
+
+    for (int i = 0; i < nL; ++i) {
+        const ct_layer_desc &d = desc->layers[i];
+        if (!defined[d.src] || defined[d.dst]) return CT_EINVAL;
+        if (d.res >= 0 && (d.res > max_slot || !defined[d.res])) return CT_EINVAL;
+        Slot &src = m->slots[d.src];
+        Slot &dst = m->slots[d.dst];
+        LayerRT l;
+        l.d = d;
+        const float *W = wts[CT_WEIGHTS_PER_LAYER * i + 0];
+        const float *bias = wts[CT_WEIGHTS_PER_LAYER * i + 1];
+        if (d.op == CT_OP_CONV) {
+            if (src.is_float || d.cin != src.C || d.k < 1 || d.stride < 1 || d.pad < 0 || d.cout < 1 || !W)
+                return CT_EINVAL;
+            int role = m->protect ? d.role : CT_ROLE_NONE;
+            if (role == CT_ROLE_PASS && m->ds_mode == CT_DS_ZERO) role = CT_ROLE_NONE;
+            if (role < CT_ROLE_CT || role > CT_ROLE_PASS) return CT_EINVAL;
+            l.role = role;
+            l.C = d.cin; l.K = d.cout; l.R = l.S = d.k;
+            l.H = src.H; l.W = src.W;
+            l.P = (src.H + 2 * d.pad - d.k) / d.stride + 1;
+            l.Q = (src.W + 2 * d.pad - d.k) / d.stride + 1;
+            if (l.P < 1 || l.Q < 1) return CT_EINVAL;
+            l.cs_in = src.has_cs;
+            const bool res_cs = d.res >= 0 && m->slots[d.res].has_cs;
+            if (d.res >= 0) {
+                const Slot &r = m->slots[d.res];
+                if (r.C != l.K || r.H != l.P || r.W != l.Q || r.is_float) return CT_EINVAL;
+            }
+            l.cs_out = role == CT_ROLE_CT || role == CT_ROLE_PASS || res_cs;
+            l.coef = ldexpf(1.f, -d.ct_shift);
+            dst.C = l.K; dst.H = l.P; dst.W = l.Q; dst.has_cs = l.cs_out;
+            // ---- weights: BN fold in double (Eq. 1); the checksum channel keeps
+            // scale 1 and bias 0 because its filter is never folded ----
+            const int RSC = l.R * l.S * l.C;
+            std::string why;
+            l.tc = prec == CT_FP16 && !(m->flags & CT_FLAG_SIMT_ONLY) &&
+                   tc_supported(l.C, l.K, l.R, l.S, d.stride, d.pad, &why);
+            std::vector<uint8_t> hw((size_t)l.K * RSC * esz, 0);
+            std::vector<float> hb(l.K, 0.f);
+            for (int k = 0; k < l.K; ++k) {
+                double scale = 1.0, shift = bias ? (double)bias[k] : 0.0;
+                if (d.bn) {
+                    const float *g = wts[CT_WEIGHTS_PER_LAYER * i + 2], *be = wts[CT_WEIGHTS_PER_LAYER * i + 3];
+                    const float *mu = wts[CT_WEIGHTS_PER_LAYER * i + 4], *var = wts[CT_WEIGHTS_PER_LAYER * i + 5];
+                    if (!g || !be || !mu || !var) return CT_EINVAL;
+                    scale = (double)g[k] / sqrt((double)var[k] + desc->bn_eps);
+                    double t = (shift - (double)mu[k]) * scale;
+                    shift = t + (double)be[k];
+                }
+                hb[k] = (float)shift;
+                for (int c = 0; c < l.C; ++c)
+                    for (int r = 0; r < l.R; ++r)
+                        for (int s = 0; s < l.S; ++s) {
+                            double v = (double)W[(((size_t)k * l.C + c) * l.R + r) * l.S + s] * scale;
+                            put(hw, (size_t)k * RSC + ((size_t)r * l.S + s) * l.C + c, v, prec);
+                        }
+            }
+            ct_status st;
+            if ((st = dalloc(m, &l.w, hw.size())) != CT_OK) return st;
+            if ((st = dalloc(m, (void **)&l.bias, sizeof(float) * l.K)) != CT_OK) return st;
+            CUDA_TRY(cudaMemcpy(l.w, hw.data(), hw.size(), cudaMemcpyHostToDevice));
+            CUDA_TRY(cudaMemcpy(l.bias, hb.data(), sizeof(float) * l.K, cudaMemcpyHostToDevice));
+        } else if (d.op == CT_OP_MAXPOOL) {
+            if (src.is_float || d.k < 1 || d.stride < 1 || d.pad < 0 || d.pad >= d.k) return CT_EINVAL;
+            dst.C = src.C;
+            dst.H = (src.H + 2 * d.pad - d.k) / d.stride + 1;
+            dst.W = (src.W + 2 * d.pad - d.k) / d.stride + 1;
+            dst.has_cs = src.has_cs;
+            if (dst.H < 1 || dst.W < 1) return CT_EINVAL;
+        } else if (d.op == CT_OP_GAP) {
+            if (src.is_float) return CT_EINVAL;
+            dst.C = src.C; dst.H = dst.W = 1; dst.has_cs = src.has_cs; dst.is_float = true;
+        } else if (d.op == CT_OP_FC) {
+            const int HW = src.H * src.W;
+            if (d.cin != src.C * HW || d.cout < 1 || !W) return CT_EINVAL;
+            l.n_in = d.cin; l.n_out = d.cout;
+            l.n_cs = src.has_cs ? HW : 0;
+            l.x_float = src.is_float;
+            l.coef = ldexpf(1.f, -d.ct_shift);
+            if (d.final) { ++n_final; if (d.cout != desc->n_classes || i != nL - 1) return CT_EINVAL; }
+            dst.C = l.n_out; dst.H = dst.W = 1;
+            dst.has_cs = m->protect && !d.final;
+            // weights: columns permuted from (c, h, w) to the NHWC flatten (h, w, c)
+            std::vector<uint8_t> hw((size_t)l.n_out * l.n_in * esz);
+            std::vector<float> hb(l.n_out, 0.f);
+            for (int j = 0; j < l.n_out; ++j) {
+                hb[j] = bias ? bias[j] : 0.f;
+                for (int c = 0; c < src.C; ++c)
+                    for (int p = 0; p < HW; ++p)
+                        put(hw, (size_t)j * l.n_in + (size_t)p * src.C + c,
+                            (double)W[(size_t)j * l.n_in + (size_t)c * HW + p], prec);
+            }
+            ct_status st;
+            if ((st = dalloc(m, &l.w, hw.size())) != CT_OK) return st;
+            if ((st = dalloc(m, (void **)&l.bias, sizeof(float) * l.n_out)) != CT_OK) return st;
+            CUDA_TRY(cudaMemcpy(l.w, hw.data(), hw.size(), cudaMemcpyHostToDevice));
+            CUDA_TRY(cudaMemcpy(l.bias, hb.data(), sizeof(float) * l.n_out, cudaMemcpyHostToDevice));
+        } else {
+            return CT_EINVAL;
+        }
+        defined[d.dst] = 1;
+        m->L.push_back(l);
+    }
+    if (n_final != 1) return CT_EINVAL;
+    // ---- activation slots ----
+    for (size_t s = 0; s < m->slots.size(); ++s) {
+        Slot &sl = m->slots[s];
+        if (!defined[s]) continue;
+        bool is_final_out = false;
+        for (auto &l : m->L) if (l.d.op == CT_OP_FC && l.d.final && l.d.dst == (int)s) is_final_out = true;
+        if (is_final_out) continue;
+        const size_t e = sl.is_float ? 4 : esz;
+        ct_status st;
+        if ((st = dalloc(m, &sl.data, (size_t)B * sl.H * sl.W * sl.C * e)) != CT_OK) return st;
+        if (sl.has_cs && (st = dalloc(m, &sl.cs, (size_t)B * sl.H * sl.W * e)) != CT_OK) return st;
+    }
+    // ---- tensor-core plans ----
+    for (auto &l : m->L) {
+        if (!l.tc) continue;
+        ConvArgs a{};
+        a.N = B; a.H = l.H; a.W = l.W; a.C = l.C; a.K = l.K; a.R = l.R; a.S = l.S;
+        a.stride = l.d.stride; a.pad = l.d.pad; a.P = l.P; a.Q = l.Q; a.role = l.role; a.coef = l.coef;
+        std::string why;
+        l.plan = tc_plan_create(a, B, l.w, m->slots[l.d.src].data, &why);
+        if (!l.plan) return CT_ECUDA;
+    }
+    // ---- scratch for re-execution and host runs ----
+    const size_t per_img = (size_t)m->in_c * m->in_h * m->in_w;
+    ct_status st;
+    if ((st = dalloc(m, (void **)&m->re_input, sizeof(float) * per_img * B)) != CT_OK) return st;
+    if ((st = dalloc(m, (void **)&m->re_logits, sizeof(float) * m->n_classes * B)) != CT_OK) return st;
+    if ((st = dalloc(m, (void **)&m->re_S, sizeof(float) * B)) != CT_OK) return st;
+    if ((st = dalloc(m, (void **)&m->re_flag, B)) != CT_OK) return st;
+    if ((st = dalloc(m, (void **)&m->re_idx, sizeof(int32_t) * B)) != CT_OK) return st;
+    if ((st = dalloc(m, (void **)&m->rh_input, sizeof(float) * per_img * B)) != CT_OK) return st;
+    if ((st = dalloc(m, (void **)&m->rh_logits, sizeof(float) * m->n_classes * B)) != CT_OK) return st;
+    if ((st = dalloc(m, (void **)&m->rh_S, sizeof(float) * B)) != CT_OK) return st;
+    if ((st = dalloc(m, (void **)&m->rh_flag, B)) != CT_OK) return st;
+    if ((st = dalloc(m, (void **)&m->d_err, sizeof(uint32_t))) != CT_OK) return st;
+    CUDA_TRY(cudaMemset(m->d_err, 0, sizeof(uint32_t)));
+    if (cudaMallocHost((void **)&m->h_flags, B) != cudaSuccess) return CT_ENOMEM;
+    if (cudaMallocHost((void **)&m->h_idx, sizeof(int32_t) * B) != cudaSuccess) return CT_ENOMEM;
+    CUDA_TRY(cudaDeviceSynchronize());
+    return CT_OK;
+}
+
+// ---------------------------------------------------------------------------
+// fault resolution
+// ---------------------------------------------------------------------------
+
+struct WeightFault {
+    bool explicit_word = false;   // XOR a device word
+    int64_t word = 0;
+    FaultDelta fd{};
+};
+
+// Map a literal weight element [K_tot, C_tot, R, S] of conv layer l to the
+// device representation: an explicit stored word (a data filter weight), or
+// an implicit weight of the construction (zero checksum slice, carry-through
+// or pass-through row), whose flipped value enters the epilogue as
+// dv * input, dv = flipped - stored.
+WeightFault resolve_weight_fault(const ct_model *m, const LayerRT &l, int64_t e, int bit) {
+    const int Ct = l.C + (l.cs_in ? 1 : 0);
+    const int RS = l.R * l.S;
+    const int k = (int)(e / ((int64_t)Ct * RS));
+    const int c = (int)((e / RS) % Ct);
+    const int r = (int)((e / l.S) % l.R), s = (int)(e % l.S);
+    const int RSC = l.R * l.S * l.C;
+    const bool centre = r == (l.R - 1) / 2 && s == (l.S - 1) / 2;
+    WeightFault f;
+    if (k < l.K && c < l.C) {
+        f.explicit_word = true;
+        f.word = (int64_t)k * RSC + ((int64_t)r * l.S + s) * l.C + c;
+        return f;
+    }
+    double stored = 0.0;                      // zero slice and off-centre taps
+    if (k == l.K && l.role == CT_ROLE_CT && centre) stored = l.coef;
+    if (k == l.K && l.role == CT_ROLE_PASS && centre && c == l.C) stored = 1.0;
+    const float v = flipped(stored, bit, m->prec);
+    f.fd.active = 1;
+    f.fd.kout = k;
+    f.fd.cin = c;
+    f.fd.r = r;
+    f.fd.s = s;
+    f.fd.dv = v - (float)stored;
+    return f;
+}
+
+ct_status act_fault_word(const ct_model *m, int slot, int batch, int64_t e, void **base, int64_t *word) {
+    const Slot &sl = m->slots[slot];
+    const int Ct = sl.C + (sl.has_cs ? 1 : 0);
+    const int64_t HW = (int64_t)sl.H * sl.W;
+    if (e < 0 || e >= (int64_t)batch * Ct * HW) return CT_ERANGE;
+    const int64_t n = e / (Ct * HW);
+    const int c = (int)((e / HW) % Ct);
+    const int64_t hw = e % HW;
+    if (c < sl.C) { *base = sl.data; *word = (n * HW + hw) * sl.C + c; }
+    else { *base = sl.cs; *word = n * HW + hw; }
+    return CT_OK;
+}
+
+// ---------------------------------------------------------------------------
+// inference
+// ---------------------------------------------------------------------------
+
+ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, float *S,
+                     uint8_t *flag, cudaStream_t st) {
+    const bool half = m->prec == CT_FP16;
+    const int wb = half ? 2 : 4;
+    const bool armed = m->armed;
+    m->armed = false;
+    int act_slot = -1;
+    void *act_base = nullptr;
+    int64_t act_word = 0;
+    if (armed && m->f_kind == CT_BUF_ACT) {
+        act_slot = m->L[m->f_layer].d.src;
+        if (act_fault_word(m, act_slot, batch, m->f_elem, &act_base, &act_word) != CT_OK) return CT_ERANGE;
+    }
+    Slot &s0 = m->slots[0];
+    CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] {
+        return launch_convert_input(input, s0.data, batch, s0.C, s0.H, s0.W, half, st);
+    }));
+    if (act_slot == 0) CUDA_TRY(launch_xor_bit(act_base, act_word, m->f_bit, wb, st));
+    for (size_t i = 0; i < m->L.size(); ++i) {
+        LayerRT &l = m->L[i];
+        const ct_layer_desc &d = l.d;
+        Slot &src = m->slots[d.src];
+        Slot &dst = m->slots[d.dst];
+        if (d.op == CT_OP_CONV) {
+            ConvArgs a{};
+            a.x = src.data; a.cs_in = src.has_cs ? src.cs : nullptr; a.w = l.w; a.bias = l.bias;
+            if (d.res >= 0) {
+                a.res = m->slots[d.res].data;
+                a.res_cs = m->slots[d.res].has_cs ? m->slots[d.res].cs : nullptr;
+            }
+            a.y = dst.data; a.cs_out = dst.has_cs ? dst.cs : nullptr;
+            a.N = batch; a.H = l.H; a.W = l.W; a.C = l.C; a.K = l.K; a.R = l.R; a.S = l.S;
+            a.stride = d.stride; a.pad = d.pad; a.P = l.P; a.Q = l.Q;
+            a.role = l.role; a.relu = d.relu; a.coef = l.coef; a.err = m->d_err;
+            WeightFault wf;
+            const bool wfault = armed && m->f_kind == CT_BUF_WEIGHT && m->f_layer == (int)i;
+            if (wfault) {
+                wf = resolve_weight_fault(m, l, m->f_elem, m->f_bit);
+                if (wf.explicit_word) CUDA_TRY(launch_xor_bit(l.w, wf.word, m->f_bit, wb, st));
+                else a.fd = wf.fd;
+            }
+            const double flops = 2.0 * batch * l.P * l.Q * (double)l.K * l.R * l.S * l.C;
+            if (l.tc) CUDA_TRY(launch(m, FAM_TC, flops, st, [&] { return launch_conv_tc(a, l.plan, st); }));
+            else CUDA_TRY(launch(m, FAM_SIMT, flops, st, [&] { return launch_conv_simt(a, half, st); }));
+            if (wfault && wf.explicit_word) CUDA_TRY(launch_xor_bit(l.w, wf.word, m->f_bit, wb, st));
+        } else if (d.op == CT_OP_MAXPOOL || d.op == CT_OP_GAP) {
+            PoolArgs a{};
+            a.x = src.data; a.cs_in = src.has_cs ? src.cs : nullptr;
+            a.y = dst.data; a.cs_out = dst.has_cs ? dst.cs : nullptr;
+            a.N = batch; a.H = src.H; a.W = src.W; a.C = src.C; a.P = dst.H; a.Q = dst.W;
+            a.k = d.k; a.stride = d.stride; a.pad = d.pad;
+            if (d.op == CT_OP_MAXPOOL) CUDA_TRY(launch(m, FAM_POOL, 0, st, [&] { return launch_maxpool(a, half, st); }));
+            else CUDA_TRY(launch(m, FAM_POOL, 0, st, [&] { return launch_gap(a, half, st); }));
+        } else {
+            FcArgs a{};
+            a.x = src.data; a.xcs = src.has_cs ? src.cs : nullptr; a.w = l.w; a.bias = l.bias;
+            a.B = batch; a.n_in = l.n_in; a.n_cs = l.n_cs; a.n_out = l.n_out;
+            a.relu = d.relu; a.final_layer = d.final; a.protect = m->protect; a.coef = l.coef;
+            a.ref = m->ref; a.tau = m->tau;
+            if (d.final) { a.y = logits; a.S = S; a.flag = flag; }
+            else { a.y = dst.data; a.ycs = dst.has_cs ? dst.cs : nullptr; }
+            const double flops = 2.0 * batch * (double)l.n_in * l.n_out;
+            CUDA_TRY(launch(m, FAM_FC, flops, st, [&] { return launch_fc(a, half, l.x_float, st); }));
+        }
+        if (act_slot == d.dst) CUDA_TRY(launch_xor_bit(act_base, act_word, m->f_bit, wb, st));
+    }
+    return CT_OK;
+}
+
+ct_status reexec_impl(ct_model *m, const float *input, int batch, const uint8_t *flag, float *logits,
+                      float *S, int *n_rerun, cudaStream_t st) {
+    CUDA_TRY(cudaMemcpyAsync(m->h_flags, flag, batch, cudaMemcpyDeviceToHost, st));
+    CUDA_TRY(cudaStreamSynchronize(st));
+    int n = 0;
+    for (int i = 0; i < batch; ++i)
+        if (m->h_flags[i]) m->h_idx[n++] = i;
+    if (n_rerun) *n_rerun = n;
+    if (n == 0) return CT_OK;
+    CUDA_TRY(cudaMemcpyAsync(m->re_idx, m->h_idx, sizeof(int32_t) * n, cudaMemcpyHostToDevice, st));
+    const int64_t per = (int64_t)m->in_c * m->in_h * m->in_w;
+    CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] { return launch_gather_images(input, m->re_input, m->re_idx, n, per, st); }));
+    // fault-free re-run: an armed fault stays armed for the next ct_infer
+    const bool armed = m->armed;
+    m->armed = false;
+    ct_status s = infer_impl(m, m->re_input, n, m->re_logits, m->re_S, m->re_flag, st);
+    m->armed = armed;
+    if (s != CT_OK) return s;
+    CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] { return launch_scatter_rows(m->re_logits, logits, m->re_idx, n, m->n_classes, st); }));
+    if (S) CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] { return launch_scatter_rows(m->re_S, S, m->re_idx, n, 1, st); }));
+    return CT_OK;
+}
+
+}  // namespace
+
+// ===========================================================================
+// C ABI
+// ===========================================================================
+
+extern "C" {
+
+ct_status ct_build(const ct_model_desc *desc, const float *const *weights, const ct_build_opts *opts,
+                   ct_model **out) {
+    if (!desc || !weights || !opts || !out || desc->n_layers < 1 || !desc->layers) return CT_EINVAL;
+    if (opts->precision != CT_FP32 && opts->precision != CT_FP16) return CT_EINVAL;
+    if (opts->max_batch < 1 || desc->in_c < 1 || desc->in_h < 1 || desc->in_w < 1 || desc->n_classes < 1)
+        return CT_EINVAL;
+    *out = nullptr;
+    int ndev = 0;
+    if (cudaGetDeviceCount(&ndev) != cudaSuccess || opts->device < 0 || opts->device >= ndev) {
+        cudaGetLastError();
+        return CT_ECUDA;
+    }
+    DeviceGuard g(opts->device);
+    ct_model *m = new (std::nothrow) ct_model();
+    if (!m) return CT_ENOMEM;
+    m->device = opts->device;
+    m->prec = opts->precision;
+    m->protect = opts->protect != 0;
+    m->ds_mode = opts->ds_mode;
+    m->max_batch = opts->max_batch;
+    m->flags = opts->flags;
+    m->in_c = desc->in_c; m->in_h = desc->in_h; m->in_w = desc->in_w;
+    m->n_classes = desc->n_classes;
+    ct_status s = build_impl(m, desc, weights);
+    if (s != CT_OK) {
+        free_all(m);
+        delete m;
+        return s;
+    }
+    *out = m;
+    return CT_OK;
+}
+
+ct_status ct_set_threshold(ct_model *m, double reference, double tau) {
+    if (!m || !(tau >= 0.0) || reference != reference) return CT_EINVAL;
+    m->ref = reference;
+    m->tau = tau;
+    return CT_OK;
+}
+
+ct_status ct_get_threshold(const ct_model *m, double *reference, double *tau) {
+    if (!m || !reference || !tau) return CT_EINVAL;
+    *reference = m->ref;
+    *tau = m->tau;
+    return CT_OK;
+}
+
+ct_status ct_infer(ct_model *m, const float *input_dev, int32_t batch, float *logits_dev, float *S_dev,
+                   uint8_t *flag_dev, void *stream) {
+    if (!m || !input_dev || !logits_dev) return CT_EINVAL;
+    if (batch < 1 || batch > m->max_batch) return CT_ERANGE;
+    DeviceGuard g(m->device);
+    return infer_impl(m, input_dev, batch, logits_dev, S_dev, flag_dev, (cudaStream_t)stream);
+}
+
+ct_status ct_inject(ct_model *m, int32_t kind, int32_t layer, int64_t element, int32_t bit) {
+    if (!m || layer < 0 || layer >= (int)m->L.size()) return CT_EINVAL;
+    const LayerRT &l = m->L[layer];
+    if (l.d.op != CT_OP_CONV) return CT_EINVAL;
+    if (kind != CT_BUF_WEIGHT && kind != CT_BUF_ACT) return CT_EINVAL;
+    const int bits = m->prec == CT_FP16 ? 16 : 32;
+    if (bit < 0 || bit >= bits) return CT_ERANGE;
+    if (kind == CT_BUF_WEIGHT) {
+        const int Kt = l.K + ((l.role == CT_ROLE_CT || l.role == CT_ROLE_PASS) ? 1 : 0);
+        const int Ct = l.C + (l.cs_in ? 1 : 0);
+        if (element < 0 || element >= (int64_t)Kt * Ct * l.R * l.S) return CT_ERANGE;
+    } else {
+        const Slot &sl = m->slots[l.d.src];
+        const int Ct = sl.C + (sl.has_cs ? 1 : 0);
+        if (element < 0 || element >= (int64_t)m->max_batch * Ct * sl.H * sl.W) return CT_ERANGE;
+    }
+    m->armed = true;
+    m->f_kind = kind; m->f_layer = layer; m->f_elem = element; m->f_bit = bit;
+    return CT_OK;
+}
+
+ct_status ct_clear_faults(ct_model *m) {
+    if (!m) return CT_EINVAL;
+    m->armed = false;
+    return CT_OK;
+}
+
+ct_status ct_reexecute(ct_model *m, const float *input_dev, int32_t batch, const uint8_t *flag_dev,
+                       float *logits_dev, float *S_dev, int32_t *n_rerun, void *stream) {
+    if (!m || !input_dev || !flag_dev || !logits_dev) return CT_EINVAL;
+    if (batch < 1 || batch > m->max_batch) return CT_ERANGE;
+    DeviceGuard g(m->device);
+    int n = 0;
+    ct_status s = reexec_impl(m, input_dev, batch, flag_dev, logits_dev, S_dev, &n, (cudaStream_t)stream);
+    if (n_rerun) *n_rerun = n;
+    return s;
+}
+
+ct_status ct_run_host(ct_model *m, const float *input_host, int32_t batch, float *logits_host,
+                      float *S_host, uint8_t *flag_host, int32_t *n_rerun, void *stream) {
+    if (!m || !input_host || !logits_host) return CT_EINVAL;
+    if (batch < 1 || batch > m->max_batch) return CT_ERANGE;
+    DeviceGuard g(m->device);
+    cudaStream_t st = (cudaStream_t)stream;
+    const size_t per = (size_t)m->in_c * m->in_h * m->in_w;
+    CUDA_TRY(cudaMemcpyAsync(m->rh_input, input_host, sizeof(float) * per * batch, cudaMemcpyHostToDevice, st));
+    ct_status s = infer_impl(m, m->rh_input, batch, m->rh_logits, m->rh_S, m->rh_flag, st);
+    if (s != CT_OK) return s;
+    int n = 0;
+    if (m->protect) {
+        s = reexec_impl(m, m->rh_input, batch, m->rh_flag, m->rh_logits, m->rh_S, &n, st);
+        if (s != CT_OK) return s;
+    }
+    if (n_rerun) *n_rerun = n;
+    CUDA_TRY(cudaMemcpyAsync(logits_host, m->rh_logits, sizeof(float) * m->n_classes * batch,
+                             cudaMemcpyDeviceToHost, st));
+    if (S_host) CUDA_TRY(cudaMemcpyAsync(S_host, m->rh_S, sizeof(float) * batch, cudaMemcpyDeviceToHost, st));
+    if (flag_host) CUDA_TRY(cudaMemcpyAsync(flag_host, m->rh_flag, batch, cudaMemcpyDeviceToHost, st));
+    CUDA_TRY(cudaStreamSynchronize(st));
+    return CT_OK;
+}
+
+ct_status ct_calibrate(const float *S_host, int64_t n, double alpha, double *reference, double *tau) {
+    if (!S_host || n < 1 || !(alpha >= 0.0 && alpha < 1.0) || !reference || !tau) return CT_EINVAL;
+    double sum = 0.0;
+    for (int64_t i = 0; i < n; ++i) {
+        if (!isfinite(S_host[i])) return CT_EINVAL;
+        sum += (double)S_host[i];
+    }
+    const double r = sum / (double)n;
+    std::vector<double> dev(n);
+    for (int64_t i = 0; i < n; ++i) dev[i] = fabs((double)S_host[i] - r);
+    std::sort(dev.begin(), dev.end());
+    int64_t rank = (int64_t)ceil((1.0 - alpha) * (double)n);
+    rank = std::min<int64_t>(std::max<int64_t>(rank, 1), n);
+    *reference = r;
+    *tau = dev[rank - 1];
+    return CT_OK;
+}
+
+ct_status ct_buffer_count(const ct_model *m, int32_t batch, int32_t *n) {
+    if (!m || !n || batch < 1) return CT_EINVAL;
+    int cnt = 0;
+    std::vector<int> seen;
+    for (auto &l : m->L)
+        if (l.d.op == CT_OP_CONV) ++cnt;
+    for (auto &l : m->L)
+        if (l.d.op == CT_OP_CONV && l.d.src != 0 &&
+            std::find(seen.begin(), seen.end(), l.d.src) == seen.end()) {
+            seen.push_back(l.d.src);
+            ++cnt;
+        }
+    *n = cnt;
+    return CT_OK;
+}
+
+ct_status ct_buffer_info(const ct_model *m, int32_t batch, int32_t i, int32_t *kind, int32_t *layer,
+                         int64_t *n_elements, int32_t *bits) {
+    if (!m || batch < 1 || !kind || !layer || !n_elements || !bits) return CT_EINVAL;
+    const int b = m->prec == CT_FP16 ? 16 : 32;
+    int idx = 0;
+    for (size_t li = 0; li < m->L.size(); ++li) {
+        const LayerRT &l = m->L[li];
+        if (l.d.op != CT_OP_CONV) continue;
+        if (idx++ == i) {
+            const int Kt = l.K + ((l.role == CT_ROLE_CT || l.role == CT_ROLE_PASS) ? 1 : 0);
+            const int Ct = l.C + (l.cs_in ? 1 : 0);
+            *kind = CT_BUF_WEIGHT; *layer = (int)li; *n_elements = (int64_t)Kt * Ct * l.R * l.S; *bits = b;
+            return CT_OK;
+        }
+    }
+    std::vector<int> seen;
+    for (size_t li = 0; li < m->L.size(); ++li) {
+        const LayerRT &l = m->L[li];
+        if (l.d.op != CT_OP_CONV || l.d.src == 0) continue;
+        if (std::find(seen.begin(), seen.end(), l.d.src) != seen.end()) continue;
+        seen.push_back(l.d.src);
+        if (idx++ == i) {
+            const Slot &sl = m->slots[l.d.src];
+            *kind = CT_BUF_ACT; *layer = (int)li;
+            *n_elements = (int64_t)batch * (sl.C + (sl.has_cs ? 1 : 0)) * sl.H * sl.W;
+            *bits = b;
+            return CT_OK;
+        }
+    }
+    return CT_ERANGE;
+}
+
+ct_status ct_profile_enable(ct_model *m, int32_t on) {
+    if (!m) return CT_EINVAL;
+    m->prof = on != 0;
+    return CT_OK;
+}
+
+ct_status ct_profile_read(ct_model *m, int32_t family, int64_t *launches, double *ms, double *flops) {
+    if (!m || family < 0 || family >= FAM_COUNT || !launches || !ms) return CT_EINVAL;
+    DeviceGuard g(m->device);
+    int64_t n = 0;
+    double t = 0.0, f = 0.0;
+    std::vector<EvRec> keep;
+    for (const EvRec &r : m->recs) {
+        if (r.fam != family) { keep.push_back(r); continue; }
+        float e = 0.f;
+        CUDA_TRY(cudaEventSynchronize(m->ev_pool[r.ev].second));
+        CUDA_TRY(cudaEventElapsedTime(&e, m->ev_pool[r.ev].first, m->ev_pool[r.ev].second));
+        t += e;
+        f += r.flops;
+        ++n;
+        m->ev_free.push_back(r.ev);
+    }
+    m->recs.swap(keep);
+    *launches = n;
+    *ms = t;
+    if (flops) *flops = f;
+    return CT_OK;
+}
+
+ct_status ct_launches_per_infer(const ct_model *m, int32_t *n) {
+    if (!m || !n) return CT_EINVAL;
+    *n = 1 + (int)m->L.size();
+    return CT_OK;
+}
+
+ct_status ct_copy_activation(ct_model *m, int32_t slot, int32_t batch, void *data_host, void *cs_host,
+                             int32_t *C, int32_t *H, int32_t *W, int32_t *has_cs, int32_t *elem_bytes,
+                             void *stream) {
+    if (!m) return CT_EINVAL;
+    if (slot < 0 || slot >= (int)m->slots.size() || batch < 1 || batch > m->max_batch) return CT_ERANGE;
+    const Slot &sl = m->slots[slot];
+    if (!sl.data) return CT_ERANGE;
+    const size_t e = sl.is_float ? 4 : m->esz();
+    if (C) *C = sl.C;
+    if (H) *H = sl.H;
+    if (W) *W = sl.W;
+    if (has_cs) *has_cs = sl.has_cs ? 1 : 0;
+    if (elem_bytes) *elem_bytes = (int32_t)e;
+    if (!data_host) return CT_OK;
+    DeviceGuard g(m->device);
+    cudaStream_t st = (cudaStream_t)stream;
+    const size_t hw = (size_t)batch * sl.H * sl.W;
+    CUDA_TRY(cudaMemcpyAsync(data_host, sl.data, hw * sl.C * e, cudaMemcpyDeviceToHost, st));
+    if (cs_host && sl.has_cs) CUDA_TRY(cudaMemcpyAsync(cs_host, sl.cs, hw * e, cudaMemcpyDeviceToHost, st));
+    CUDA_TRY(cudaStreamSynchronize(st));
+    return CT_OK;
+}
+
+ct_status ct_device_error(ct_model *m, uint32_t *code) {
+    if (!m || !code) return CT_EINVAL;
+    DeviceGuard g(m->device);
+    CUDA_TRY(cudaDeviceSynchronize());
+    CUDA_TRY(cudaMemcpy(code, m->d_err, sizeof(uint32_t), cudaMemcpyDeviceToHost));
+    CUDA_TRY(cudaMemset(m->d_err, 0, sizeof(uint32_t)));
+    return CT_OK;
+}
+
+void ct_destroy(ct_model *m) {
+    if (!m) return;
+    DeviceGuard g(m->device);
+    cudaDeviceSynchronize();
+    free_all(m);
+    delete m;
+}
+
+const char *ct_strerror(ct_status s) {
+    switch (s) {
+        case CT_OK: return "ok";
+        case CT_EINVAL: return "invalid argument or model description";
+        case CT_ENOMEM: return "out of memory";
+        case CT_ECUDA: return "CUDA call failed";
+        case CT_ESTATE: return "invalid state";
+        case CT_ERANGE: return "index, batch or bit out of range";
+        case CT_EUNSUPPORTED: return "unsupported shape";
+        case CT_EDEVICE: return "device-side error (bounded wait expired)";
+    }
+    return "unknown status";
+}
+
+}  // extern "C"

@@ -1,0 +1,87 @@
+// Internal structures of libct (not part of the ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_fp16.h>
+#include <stdint.h>
+
+#include <string>
+#include <vector>
+
+#include "../../include/ct.h"
+
+namespace ct {
+
+// Implicit weight of the carry-through construction hit by a fault: output
+// channel `kout` (== K for the checksum output) gains dv * input[cin] at tap
+// (r, s), where cin == C means the incoming checksum plane.
+struct FaultDelta {
+    int active;
+    int kout, cin, r, s;
+    float dv;
+};
+
+// Arguments of every convolution kernel.  Activations are NHWC, the checksum
+// plane is [N, H, W]; weights are KRSC (C innermost).
+struct ConvArgs {
+    const void *x;        // [N, H, W, C]
+    const void *cs_in;    // [N, H, W] or null
+    const void *w;        // [K, R, S, C]
+    const float *bias;    // [K]
+    const void *res;      // [N, P, Q, K] or null
+    const void *res_cs;   // [N, P, Q] or null
+    void *y;              // [N, P, Q, K]
+    void *cs_out;         // [N, P, Q] or null
+    int N, H, W, C, K, R, S, stride, pad, P, Q;
+    int role;             // ct_role after ds_mode is applied
+    int relu;
+    float coef;           // carry-through coefficient 2^-ct_shift
+    FaultDelta fd;
+    uint32_t *err;        // device error word
+};
+
+struct FcArgs {
+    const void *x;        // [B, n_in] data features
+    const void *xcs;      // [B, n_cs] checksum features or null
+    const void *w;        // [n_out, n_in]
+    const float *bias;    // [n_out]
+    void *y;              // [B, n_out]  (final: float logits)
+    void *ycs;            // [B] carry-through neuron (hidden) or null
+    float *S;             // final: [B] or null
+    uint8_t *flag;        // final: [B] or null
+    int B, n_in, n_cs, n_out;
+    int relu, final_layer, protect;
+    float coef;
+    double ref, tau;
+};
+
+struct PoolArgs {
+    const void *x; const void *cs_in;
+    void *y; void *cs_out;
+    int N, H, W, C, P, Q, k, stride, pad;
+};
+
+enum Family { FAM_TC = 0, FAM_SIMT = 1, FAM_FC = 2, FAM_POOL = 3, FAM_OTHER = 4, FAM_COUNT = 5 };
+
+// kernel launchers; each returns cudaGetLastError()
+cudaError_t launch_conv_simt(const ConvArgs &a, bool half, cudaStream_t st);
+cudaError_t launch_conv_tc(const ConvArgs &a, const void *tc_plan, cudaStream_t st);
+cudaError_t launch_fc(const FcArgs &a, bool half, bool x_float, cudaStream_t st);
+cudaError_t launch_maxpool(const PoolArgs &a, bool half, cudaStream_t st);
+cudaError_t launch_gap(const PoolArgs &a, bool half, cudaStream_t st);
+cudaError_t launch_convert_input(const float *in, void *out, int N, int C, int H, int W, bool half,
+                                 cudaStream_t st);
+cudaError_t launch_xor_bit(void *base, int64_t word, int bit, int word_bytes, cudaStream_t st);
+cudaError_t launch_gather_images(const float *in, float *out, const int32_t *idx, int n,
+                                 int64_t per_image, cudaStream_t st);
+cudaError_t launch_scatter_rows(const float *src, float *dst, const int32_t *idx, int n, int row,
+                                cudaStream_t st);
+
+// tensor-core conv plan (opaque outside conv_tc.cu)
+struct TcPlan;
+TcPlan *tc_plan_create(const ConvArgs &shape_args, int max_batch, const void *w_dev, const void *x_dev,
+                       std::string *why);
+void tc_plan_destroy(TcPlan *p);
+bool tc_supported(int C, int K, int R, int S, int stride, int pad, std::string *why);
+
+}  // namespace ct

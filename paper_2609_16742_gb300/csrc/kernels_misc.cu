@@ -1,0 +1,304 @@
+// FC layers with the carry-through neuron and the output verification,
+// pooling, layout conversion, fault injection and re-execution gathers.
+#include "ct_internal.h"
+
+namespace ct {
+namespace {
+
+__device__ __forceinline__ float to_f(float v) { return v; }
+__device__ __forceinline__ float to_f(__half v) { return __half2float(v); }
+template <typename T> __device__ __forceinline__ T from_f(float v);
+template <> __device__ __forceinline__ float from_f<float>(float v) { return v; }
+template <> __device__ __forceinline__ __half from_f<__half>(float v) { return __float2half_rn(v); }
+__device__ __forceinline__ float relu_keep_nan(float v) { return v < 0.f ? 0.f : v; }
+
+// ---------------------------------------------------------------------------
+// FC: y[b, j] = act(sum_i W[j, i] x[b, i] + bias[j]) over the data features
+// only (the checksum features are structural zeros of every data neuron,
+// Sec. II-A); the carry-through neuron (hidden layers) or the
+// accumulated-checksum neuron S (final layer, Sec. II-B) is coef times the
+// sum of every input, checksum features included.  The final layer also
+// writes the verdict flag = NOT(|S - ref| <= tau), compared in double.
+//
+// Block: 256 threads = 8 warps, 16 neurons x 64 images.  Lanes own images
+// (l and l + 32), warps split the K chunk, so one staged x value feeds 16
+// FMAs and one staged weight value is a broadcast.
+// ---------------------------------------------------------------------------
+constexpr int FC_J = 16, FC_IMG = 64, FC_KC = 64, FC_WARPS = 8;
+static_assert((FC_KC * (FC_IMG + 1)) % 4 == 0, "weight tile must start 16-byte aligned (float4 reads)");
+
+template <typename TX, typename TW, typename TY>
+__global__ void __launch_bounds__(256) fc_kernel(FcArgs a) {
+    extern __shared__ __align__(16) float smem[];
+    float *Xs = smem;                              // [FC_KC][FC_IMG + 1]
+    float *Ws = Xs + FC_KC * (FC_IMG + 1);         // [FC_KC][FC_J]; offset 4160 floats: 16-byte aligned
+    float *red = Ws + FC_KC * FC_J;                // [FC_WARPS][FC_J + 1][FC_IMG]
+    const TX *x = static_cast<const TX *>(a.x);
+    const TW *w = static_cast<const TW *>(a.w);
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int j0 = blockIdx.x * FC_J, b0 = blockIdx.y * FC_IMG;
+    const bool ct_block = a.protect && blockIdx.x == 0;
+
+    float acc[FC_J][2];
+    float act[2] = {0.f, 0.f};
+#pragma unroll
+    for (int j = 0; j < FC_J; ++j) acc[j][0] = acc[j][1] = 0.f;
+
+    for (int k0 = 0; k0 < a.n_in; k0 += FC_KC) {
+        // stage x[b0 .. b0+63][k0 .. k0+63] transposed, and W[j0..j0+15][k0..k0+63]
+        for (int e = tid; e < FC_KC * FC_IMG; e += 256) {
+            int kk = e % FC_KC, bb = e / FC_KC;
+            int b = b0 + bb, k = k0 + kk;
+            Xs[kk * (FC_IMG + 1) + bb] = (b < a.B && k < a.n_in) ? to_f(x[(size_t)b * a.n_in + k]) : 0.f;
+        }
+        for (int e = tid; e < FC_KC * FC_J; e += 256) {
+            int kk = e % FC_KC, jj = e / FC_KC;
+            int j = j0 + jj, k = k0 + kk;
+            Ws[kk * FC_J + jj] = (j < a.n_out && k < a.n_in) ? to_f(w[(size_t)j * a.n_in + k]) : 0.f;
+        }
+        __syncthreads();
+#pragma unroll 2
+        for (int kk = warp; kk < FC_KC; kk += FC_WARPS) {
+            float x0 = Xs[kk * (FC_IMG + 1) + lane], x1 = Xs[kk * (FC_IMG + 1) + lane + 32];
+            const float4 *wr = reinterpret_cast<const float4 *>(&Ws[kk * FC_J]);
+#pragma unroll
+            for (int q = 0; q < FC_J / 4; ++q) {
+                float4 wv = wr[q];
+                acc[4 * q + 0][0] = fmaf(wv.x, x0, acc[4 * q + 0][0]);
+                acc[4 * q + 0][1] = fmaf(wv.x, x1, acc[4 * q + 0][1]);
+                acc[4 * q + 1][0] = fmaf(wv.y, x0, acc[4 * q + 1][0]);
+                acc[4 * q + 1][1] = fmaf(wv.y, x1, acc[4 * q + 1][1]);
+                acc[4 * q + 2][0] = fmaf(wv.z, x0, acc[4 * q + 2][0]);
+                acc[4 * q + 2][1] = fmaf(wv.z, x1, acc[4 * q + 2][1]);
+                acc[4 * q + 3][0] = fmaf(wv.w, x0, acc[4 * q + 3][0]);
+                acc[4 * q + 3][1] = fmaf(wv.w, x1, acc[4 * q + 3][1]);
+            }
+            if (ct_block) { act[0] += x0; act[1] += x1; }
+        }
+        __syncthreads();
+    }
+    // cross-warp reduction
+#pragma unroll
+    for (int j = 0; j < FC_J; ++j) {
+        red[(warp * (FC_J + 1) + j) * FC_IMG + lane] = acc[j][0];
+        red[(warp * (FC_J + 1) + j) * FC_IMG + lane + 32] = acc[j][1];
+    }
+    red[(warp * (FC_J + 1) + FC_J) * FC_IMG + lane] = act[0];
+    red[(warp * (FC_J + 1) + FC_J) * FC_IMG + lane + 32] = act[1];
+    __syncthreads();
+    for (int e = tid; e < FC_J * FC_IMG; e += 256) {
+        int jj = e / FC_IMG, bb = e % FC_IMG;
+        int j = j0 + jj, b = b0 + bb;
+        if (j >= a.n_out || b >= a.B) continue;
+        float s = 0.f;
+        for (int wv = 0; wv < FC_WARPS; ++wv) s += red[(wv * (FC_J + 1) + jj) * FC_IMG + bb];
+        s += a.bias[j];
+        if (a.relu) s = relu_keep_nan(s);
+        static_cast<TY *>(a.y)[(size_t)b * a.n_out + j] = from_f<TY>(s);
+    }
+    if (!ct_block) {
+        if (a.final_layer && blockIdx.x == 0 && !a.protect) {
+            for (int bb = tid; bb < FC_IMG; bb += 256) {
+                int b = b0 + bb;
+                if (b >= a.B) continue;
+                if (a.S) a.S[b] = __int_as_float(0x7fc00000);
+                if (a.flag) a.flag[b] = 0;
+            }
+        }
+        return;
+    }
+    const TX *xcs = static_cast<const TX *>(a.xcs);
+    for (int bb = tid; bb < FC_IMG; bb += 256) {
+        int b = b0 + bb;
+        if (b >= a.B) continue;
+        float s = 0.f;
+        for (int wv = 0; wv < FC_WARPS; ++wv) s += red[(wv * (FC_J + 1) + FC_J) * FC_IMG + bb];
+        if (xcs)
+            for (int i = 0; i < a.n_cs; ++i) s += to_f(xcs[(size_t)b * a.n_cs + i]);
+        s *= a.coef;
+        if (a.final_layer) {
+            if (a.S) a.S[b] = s;
+            if (a.flag) a.flag[b] = !(fabs((double)s - a.ref) <= a.tau);
+        } else {
+            if (a.relu) s = relu_keep_nan(s);
+            static_cast<TY *>(a.ycs)[b] = from_f<TY>(s);
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Max-pool over NHWC data and the [N, H, W] checksum plane together.  The
+// window maximum is taken on stored values (exact); padding never wins; a
+// NaN anywhere in the window gives NaN.
+// ---------------------------------------------------------------------------
+template <typename T>
+__global__ void maxpool_kernel(PoolArgs a) {
+    const int64_t n_data = (int64_t)a.N * a.P * a.Q * a.C;
+    const int64_t n_cs = a.cs_in ? (int64_t)a.N * a.P * a.Q : 0;
+    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n_data + n_cs;
+         e += (int64_t)gridDim.x * blockDim.x) {
+        const bool is_cs = e >= n_data;
+        const int64_t i = is_cs ? e - n_data : e;
+        const int C = is_cs ? 1 : a.C;
+        const int c = (int)(i % C);
+        int64_t t = i / C;
+        const int q = (int)(t % a.Q); t /= a.Q;
+        const int p = (int)(t % a.P);
+        const int n = (int)(t / a.P);
+        const T *src = static_cast<const T *>(is_cs ? a.cs_in : a.x);
+        float m = -INFINITY;
+        bool nan = false;
+        for (int r = 0; r < a.k; ++r) {
+            int h = p * a.stride + r - a.pad;
+            if (h < 0 || h >= a.H) continue;
+            for (int s = 0; s < a.k; ++s) {
+                int w = q * a.stride + s - a.pad;
+                if (w < 0 || w >= a.W) continue;
+                float v = to_f(src[(((size_t)n * a.H + h) * a.W + w) * C + c]);
+                nan |= (v != v);
+                m = v > m ? v : m;
+            }
+        }
+        if (nan) m = __int_as_float(0x7fc00000);
+        T *dst = static_cast<T *>(is_cs ? a.cs_out : a.y);
+        dst[i] = from_f<T>(m);
+    }
+}
+
+// Global average pool: float [N, C] features (+ float [N] checksum feature).
+template <typename T>
+__global__ void gap_kernel(PoolArgs a) {
+    const int HW = a.H * a.W;
+    const int n = blockIdx.y;
+    const int c = blockIdx.x * blockDim.x + threadIdx.x;
+    const T *x = static_cast<const T *>(a.x);
+    if (c < a.C) {
+        float s = 0.f;
+        for (int i = 0; i < HW; ++i) s += to_f(x[((size_t)n * HW + i) * a.C + c]);
+        static_cast<float *>(a.y)[(size_t)n * a.C + c] = s / (float)HW;
+    } else if (c == a.C && a.cs_in) {
+        const T *cs = static_cast<const T *>(a.cs_in);
+        float s = 0.f;
+        for (int i = 0; i < HW; ++i) s += to_f(cs[(size_t)n * HW + i]);
+        static_cast<float *>(a.cs_out)[n] = s / (float)HW;
+    }
+}
+
+template <typename T>
+__global__ void convert_input_kernel(const float *in, T *out, int N, int C, int H, int W) {
+    const int64_t total = (int64_t)N * C * H * W;
+    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
+         e += (int64_t)gridDim.x * blockDim.x) {
+        int c = (int)(e % C);
+        int64_t t = e / C;
+        int w = (int)(t % W); t /= W;
+        int h = (int)(t % H);
+        int n = (int)(t / H);
+        out[e] = from_f<T>(in[(((size_t)n * C + c) * H + h) * W + w]);
+    }
+}
+
+__global__ void xor_bit_kernel(void *base, int64_t word, int bit, int word_bytes) {
+    if (word_bytes == 2) static_cast<uint16_t *>(base)[word] ^= (uint16_t)(1u << bit);
+    else static_cast<uint32_t *>(base)[word] ^= (1u << bit);
+}
+
+// Copies image idx[i] of `in` to row i of `out` (NCHW float rows of `per`
+// elements).  16-byte vectors when every row starts 16-byte aligned.
+__global__ void gather_images_kernel(const float *in, float *out, const int32_t *idx, int64_t per) {
+    const int i = blockIdx.y;
+    const float *s = in + (size_t)idx[i] * per;
+    float *d = out + (size_t)i * per;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    const int64_t t0 = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+    if (per % 4 == 0) {
+        const float4 *src = reinterpret_cast<const float4 *>(s);
+        float4 *dst = reinterpret_cast<float4 *>(d);
+        for (int64_t e = t0; e < per / 4; e += stride) dst[e] = src[e];
+    } else {
+        for (int64_t e = t0; e < per; e += stride) d[e] = s[e];
+    }
+}
+
+__global__ void scatter_rows_kernel(const float *src, float *dst, const int32_t *idx, int n, int row) {
+    for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < n * row; e += gridDim.x * blockDim.x) {
+        int i = e / row, c = e % row;
+        dst[(size_t)idx[i] * row + c] = src[e];
+    }
+}
+
+int grid_for(int64_t n, int threads) {
+    int64_t g = (n + threads - 1) / threads;
+    if (g > 152 * 32) g = 152 * 32;
+    return (int)(g < 1 ? 1 : g);
+}
+
+template <typename TX, typename TW, typename TY>
+cudaError_t fc_go(const FcArgs &a, cudaStream_t st) {
+    const size_t smem =
+        sizeof(float) * (FC_KC * (FC_IMG + 1) + FC_KC * FC_J + FC_WARPS * (FC_J + 1) * FC_IMG);
+    static bool attr = false;
+    if (!attr) {
+        cudaError_t e = cudaFuncSetAttribute(fc_kernel<TX, TW, TY>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        attr = true;
+    }
+    dim3 grid((a.n_out + FC_J - 1) / FC_J, (a.B + FC_IMG - 1) / FC_IMG);
+    fc_kernel<TX, TW, TY><<<grid, 256, smem, st>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_fc(const FcArgs &a, bool half, bool x_float, cudaStream_t st) {
+    if (!half) return fc_go<float, float, float>(a, st);
+    if (a.final_layer)
+        return x_float ? fc_go<float, __half, float>(a, st) : fc_go<__half, __half, float>(a, st);
+    return x_float ? fc_go<float, __half, __half>(a, st) : fc_go<__half, __half, __half>(a, st);
+}
+
+cudaError_t launch_maxpool(const PoolArgs &a, bool half, cudaStream_t st) {
+    int64_t n = (int64_t)a.N * a.P * a.Q * (a.C + (a.cs_in ? 1 : 0));
+    if (half) maxpool_kernel<__half><<<grid_for(n, 256), 256, 0, st>>>(a);
+    else maxpool_kernel<float><<<grid_for(n, 256), 256, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_gap(const PoolArgs &a, bool half, cudaStream_t st) {
+    dim3 grid((a.C + 1 + 127) / 128, a.N);
+    if (half) gap_kernel<__half><<<grid, 128, 0, st>>>(a);
+    else gap_kernel<float><<<grid, 128, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_convert_input(const float *in, void *out, int N, int C, int H, int W, bool half,
+                                 cudaStream_t st) {
+    int64_t n = (int64_t)N * C * H * W;
+    if (half) convert_input_kernel<__half><<<grid_for(n, 256), 256, 0, st>>>(in, (__half *)out, N, C, H, W);
+    else convert_input_kernel<float><<<grid_for(n, 256), 256, 0, st>>>(in, (float *)out, N, C, H, W);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_xor_bit(void *base, int64_t word, int bit, int word_bytes, cudaStream_t st) {
+    xor_bit_kernel<<<1, 1, 0, st>>>(base, word, bit, word_bytes);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_gather_images(const float *in, float *out, const int32_t *idx, int n,
+                                 int64_t per_image, cudaStream_t st) {
+    if (n <= 0) return cudaSuccess;
+    const int64_t blocks = (per_image / 4 + 255) / 256 + 1;
+    dim3 grid((unsigned)(blocks > 64 ? 64 : blocks), n);
+    gather_images_kernel<<<grid, 256, 0, st>>>(in, out, idx, per_image);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_scatter_rows(const float *src, float *dst, const int32_t *idx, int n, int row,
+                                cudaStream_t st) {
+    if (n <= 0) return cudaSuccess;
+    scatter_rows_kernel<<<grid_for((int64_t)n * row, 256), 256, 0, st>>>(src, dst, idx, n, row);
+    return cudaGetLastError();
+}
+
+}  // namespace ct

@@ -1,0 +1,82 @@
+"""CPU checks of the C-ABI library: it builds, loads and exports every symbol
+that include/ct.h declares; host-only entry points behave as specified."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def ct():
+    from paper_2609_16742_gb300 import build
+    build.build()
+    import paper_2609_16742_gb300 as ct
+    return ct
+
+
+def declared_symbols():
+    src = ""
+    inc = os.path.join(ROOT, "include")
+    for f in sorted(os.listdir(inc)):
+        if f.endswith(".h"):
+            src += open(os.path.join(inc, f)).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(ct_[a-z0-9_]+)\s*\(", src)))
+
+
+def test_header_declares_the_boundary():
+    syms = declared_symbols()
+    for s in ("ct_build", "ct_infer", "ct_inject", "ct_reexecute", "ct_set_threshold"):
+        assert s in syms
+
+
+def test_library_exports_every_declared_symbol(ct):
+    lib = ctypes.CDLL(ct.LIB_PATH)
+    missing = [s for s in declared_symbols() if not hasattr(lib, s)]
+    assert not missing, missing
+    assert sorted(ct.EXPORTS) == declared_symbols()
+
+
+def test_strerror(ct):
+    assert ct.lib().ct_strerror(0) == b"ok"
+    assert b"range" in ct.lib().ct_strerror(5)
+
+
+def test_calibrate_matches_hand_example(ct):
+    S = np.arange(100, dtype=np.float32)
+    r, tau = ct.ct_calibrate(S, 0.10)
+    assert r == 49.5 and tau == 44.5
+
+
+def test_calibrate_agrees_with_oracle(ct):
+    rng = np.random.default_rng(1)
+    for n, alpha in [(1, 0.0), (7, 0.3), (1000, 0.01), (4096, 0.05)]:
+        S = (rng.standard_normal(n) * 40 + 1000).astype(np.float32)
+        r1, t1 = ct.ct_calibrate(S, alpha)
+        r2, t2 = oracle.calibrate(S.astype(np.float64), alpha)
+        assert abs(r1 - r2) <= 1e-12 * abs(r2)
+        assert abs(t1 - t2) <= 1e-9 * max(abs(t2), 1.0)
+
+
+def test_calibrate_rejects_bad_input(ct):
+    with pytest.raises(ct.CtError):
+        ct.ct_calibrate(np.array([1.0, np.nan], np.float32), 0.01)
+    with pytest.raises(ct.CtError):
+        ct.ct_calibrate(np.array([1.0], np.float32), 1.0)
+
+
+def test_build_without_device_fails_cleanly(ct):
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a device is present")
+    import synth
+    wl = synth.workload("lenet5")
+    with pytest.raises(ct.CtError) as ei:
+        ct.ct_build_workload(wl)
+    assert ei.value.status == 3          # CT_ECUDA

@@ -1,0 +1,52 @@
+"""Layer-by-layer GPU parity: every stored tensor of one inference (data
+channels and checksum plane) against the oracle's stored tensors."""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from _cache import inputs
+from _gpu import TOL, ct, model, onet, run
+
+pytestmark = pytest.mark.gpu
+
+
+def layer_errors(name, prec, batch, simt_only=False, first=0):
+    """[(slot, op, data_rel_err, cs_rel_err)] for one inference; raises on a device error."""
+    wl = synth.workload(name)
+    m = model(name, prec=prec, simt_only=simt_only, max_batch=batch)
+    x = inputs(name, batch, first)
+    run(m, x)
+    code = ct().ct_device_error(m)
+    assert code == 0, "device error word %#x" % code
+    o = oracle.forward(onet(name, prec), x, keep=True)
+    out = []
+    for L in wl.layers:
+        if L.op == "fc" and L.final:
+            continue
+        gd, gc = ct().ct_copy_activation(m, L.dst, batch)
+        ed = ec = 0.0
+        for n in range(batch):
+            a = o["acts"][n][L.dst]
+            nd = gd.shape[1]
+            ref = a[:nd].reshape(nd, -1)
+            got = gd[n].reshape(nd, -1)
+            ed = max(ed, float(np.abs(got - ref).max() / max(np.abs(ref).max(), 1e-6)))
+            if gc is not None:
+                rc = a[nd].reshape(-1)
+                ec = max(ec, float(np.abs(gc[n].reshape(-1) - rc).max() / max(np.abs(rc).max(), 1e-6)))
+        out.append((L.dst, L.op, ed, ec))
+    return out
+
+
+@pytest.mark.parametrize("name,prec,batch,simt_only", [
+    ("resnet18_cifar", "fp16", 3, False),
+    ("resnet18_cifar", "fp16", 3, True),
+    ("resnet18_cifar", "fp32", 2, False),
+    ("resnet18_imagenet", "fp16", 2, False),
+    ("lenet5", "fp32", 5, False),
+])
+def test_every_stored_tensor_matches_oracle(name, prec, batch, simt_only):
+    errs = layer_errors(name, prec, batch, simt_only)
+    bad = [e for e in errs if e[2] > TOL[prec] or e[3] > TOL[prec]]
+    assert not bad, bad

@@ -1,0 +1,100 @@
+"""GPU parity: the CUDA path, called through the C ABI, against the oracle on
+the same seeded inputs, element by element (logits, S, verdicts)."""
+import numpy as np
+import pytest
+
+import oracle
+from _cache import inputs
+from _gpu import assert_parity, ct, model, onet, run
+
+pytestmark = pytest.mark.gpu
+
+
+def _oracle(name, prec, x, protected=True):
+    return oracle.forward(onet(name, prec, protected), x)
+
+
+def test_lenet5_full_batch():
+    m = model("lenet5")
+    x = inputs("lenet5", 64)
+    lg, S, flag = run(m, x)
+    o = _oracle("lenet5", "fp32", x)
+    assert_parity(lg, S, o["logits"], o["S"], "fp32", "lenet5")
+
+
+@pytest.mark.parametrize("simt_only", [False, True])
+def test_resnet18_cifar_fp32_full_batch_sampled(simt_only):
+    m = model("resnet18_cifar", simt_only=simt_only)
+    x = inputs("resnet18_cifar", 128)
+    lg, S, _ = run(m, x)
+    idx = [0, 1, 64, 127]
+    o = _oracle("resnet18_cifar", "fp32", x[idx])
+    assert_parity(lg[idx], S[idx], o["logits"], o["S"], "fp32", "resnet18_cifar")
+
+
+@pytest.mark.parametrize("prec,simt_only", [("fp32", False), ("fp16", False), ("fp16", True)])
+@pytest.mark.parametrize("batch", [1, 3])
+def test_resnet18_cifar_ragged_batches(prec, simt_only, batch):
+    m = model("resnet18_cifar", prec=prec, simt_only=simt_only, max_batch=4)
+    x = inputs("resnet18_cifar", batch, 5)
+    lg, S, _ = run(m, x)
+    o = _oracle("resnet18_cifar", prec, x)
+    assert_parity(lg, S, o["logits"], o["S"], prec, "resnet18_cifar %s b%d" % (prec, batch))
+
+
+def test_resnet18_imagenet_fp16_full_batch_sampled():
+    m = model("resnet18_imagenet")
+    x = inputs("resnet18_imagenet", 256)
+    lg, S, _ = run(m, x)
+    idx = [0, 129, 255]
+    o = _oracle("resnet18_imagenet", "fp16", x[idx])
+    assert_parity(lg[idx], S[idx], o["logits"], o["S"], "fp16", "resnet18_imagenet")
+
+
+def test_vgg16_fp16_full_batch_sampled():
+    m = model("vgg16")
+    x = inputs("vgg16", 64)
+    lg, S, _ = run(m, x)
+    idx = [0, 63]
+    o = _oracle("vgg16", "fp16", x[idx])
+    assert_parity(lg[idx], S[idx], o["logits"], o["S"], "fp16", "vgg16")
+    assert np.isfinite(S).all() and np.abs(S).max() < 65504
+
+
+@pytest.mark.parametrize("prec", ["fp32", "fp16"])
+def test_protected_data_path_equals_unprotected(prec):
+    x = inputs("resnet18_cifar", 8)
+    lp, Sp, fp = run(model("resnet18_cifar", prec=prec, max_batch=8), x)
+    lu, Su, fu = run(model("resnet18_cifar", prec=prec, protect=False, max_batch=8), x)
+    assert np.array_equal(lp, lu)           # the checksum never enters a data channel
+    assert np.isnan(Su).all() and (fu == 0).all()
+    assert np.isfinite(Sp).all()
+
+
+def test_downsample_zero_mode():
+    x = inputs("resnet18_cifar", 2)
+    m = model("resnet18_cifar", max_batch=2, ds_mode="zero")
+    lg, S, _ = run(m, x)
+    o = oracle.forward(onet("resnet18_cifar", "fp32", True, "zero"), x)
+    assert_parity(lg, S, o["logits"], o["S"], "fp32", "ds zero")
+
+
+def test_verdict_parity_with_shared_threshold():
+    x = inputs("resnet18_cifar", 32)
+    m = model("resnet18_cifar", max_batch=32)
+    o = _oracle("resnet18_cifar", "fp32", x)
+    r = float(np.median(o["S"]))
+    tau = float(np.median(np.abs(o["S"] - r)))      # about half the images flagged
+    ct().ct_set_threshold(m, r, tau)
+    _, S, flag = run(m, x)
+    of = oracle.verdict(o["S"], r, tau)
+    near = np.abs(np.abs(o["S"] - r) - tau) <= 0.01 * tau
+    assert (flag[~near].astype(bool) == of[~near]).all()
+    assert 0 < flag.sum() < len(flag)
+
+
+def test_fault_buffers_match_oracle():
+    m = model("resnet18_cifar")
+    assert ct().ct_buffers(m, 128) == oracle.fault_buffers(onet("resnet18_cifar", "fp32"), 128)
+    m16 = model("resnet18_imagenet", max_batch=2)
+    assert ct().ct_buffers(m16, 2) == oracle.fault_buffers(onet("resnet18_imagenet", "fp16"), 2)
