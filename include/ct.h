@@ -166,6 +166,36 @@ ct_status ct_reexecute(ct_model *m, const float *input_dev, int32_t batch,
                        const uint8_t *flag_dev, float *logits_dev, float *S_dev,
                        int32_t *n_rerun, void *stream);
 
+/* ct_reexecute_noalloc -- the same re-execution as ct_reexecute, for callers
+ * that must not allocate device memory while they run: real-time loops whose
+ * device memory is fixed at start-up so that a request can never fail for
+ * want of memory, and plug-ins whose host application owns the device
+ * allocator and forbids allocations behind its back.  (The paper has no
+ * counterpart; this is a deployment variant of the mitigation step.)
+ *
+ * It allocates nothing.  ct_reexecute keeps its scratch (the gather index
+ * list and the compacted batch of flagged images with their logits, S and
+ * flags) in buffers made by ct_build; this entry point keeps that scratch
+ * in one static device array of CT_NOALLOC_SCRATCH_BYTES that every GPU
+ * loading the library holds until the process exits.  The model's weights
+ * and activation workspaces are the ones ct_build allocated.
+ *   - The scratch must hold the compacted batch: 256-byte aligned parts of
+ *     4*n (indices), 4*n*in_c*in_h*in_w (images), 4*n*n_classes (logits),
+ *     4*n (S) and n (flags) bytes for n flagged images.  If it does not,
+ *     or batch > 65536, the call returns CT_ERANGE and runs nothing.
+ *   - The first call on a device looks up the array's device address
+ *     (cudaGetSymbolAddress) with that device current; make that first
+ *     call before any stream capture.
+ *   - Every call on a device shares the one array and it keeps the last
+ *     call's contents; calls that can overlap on the GPU race on it, so
+ *     serialise them (one stream, or a wait between streams).  Host-side
+ *     flag and index lists are static too: one host thread at a time.
+ * Arguments, results and synchronisation are those of ct_reexecute. */
+#define CT_NOALLOC_SCRATCH_BYTES (16u * 1024u * 1024u)
+ct_status ct_reexecute_noalloc(ct_model *m, const float *input_dev, int32_t batch,
+                               const uint8_t *flag_dev, float *logits_dev, float *S_dev,
+                               int32_t *n_rerun, void *stream);
+
 /* ct_run_host -- end-to-end call for callers with host buffers: copies the
  * input from host memory, runs ct_infer and ct_reexecute, and copies
  * logits, S and flags back.  Returns after the results are in host memory.

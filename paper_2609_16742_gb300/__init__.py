@@ -35,7 +35,10 @@ _STATUS = {0: "CT_OK", 1: "CT_EINVAL", 2: "CT_ENOMEM", 3: "CT_ECUDA", 4: "CT_EST
 EXPORTS = ["ct_build", "ct_set_threshold", "ct_get_threshold", "ct_infer", "ct_inject",
            "ct_clear_faults", "ct_reexecute", "ct_run_host", "ct_calibrate", "ct_buffer_count",
            "ct_buffer_info", "ct_profile_enable", "ct_profile_read", "ct_launches_per_infer",
-           "ct_copy_activation", "ct_device_error", "ct_destroy", "ct_strerror"]
+           "ct_copy_activation", "ct_device_error", "ct_destroy", "ct_strerror",
+           "ct_reexecute_noalloc"]
+
+CT_NOALLOC_SCRATCH_BYTES = 16 * 1024 * 1024
 
 
 class CtError(RuntimeError):
@@ -83,6 +86,7 @@ def lib():
             "ct_inject": [vp, i32, i32, i64, i32],
             "ct_clear_faults": [vp],
             "ct_reexecute": [vp, vp, i32, vp, vp, vp, P(i32), vp],
+            "ct_reexecute_noalloc": [vp, vp, i32, vp, vp, vp, P(i32), vp],
             "ct_run_host": [vp, vp, i32, vp, vp, vp, P(i32), vp],
             "ct_calibrate": [vp, i64, dbl, P(dbl), P(dbl)],
             "ct_buffer_count": [vp, i32, P(i32)],
@@ -230,6 +234,16 @@ def ct_reexecute(m: Model, input_dev, batch: int, flag_dev, logits_dev, S_dev=No
     n = ctypes.c_int32()
     _check(lib().ct_reexecute(m.handle, _ptr(input_dev), batch, _ptr(flag_dev), _ptr(logits_dev),
                               _ptr(S_dev), ctypes.byref(n), _stream(stream)), "ct_reexecute")
+    return n.value
+
+
+def ct_reexecute_noalloc(m: Model, input_dev, batch: int, flag_dev, logits_dev, S_dev=None,
+                         stream=None) -> int:
+    """ct_reexecute without allocation: its scratch is a static device array."""
+    n = ctypes.c_int32()
+    _check(lib().ct_reexecute_noalloc(m.handle, _ptr(input_dev), batch, _ptr(flag_dev),
+                                      _ptr(logits_dev), _ptr(S_dev), ctypes.byref(n),
+                                      _stream(stream)), "ct_reexecute_noalloc")
     return n.value
 
 

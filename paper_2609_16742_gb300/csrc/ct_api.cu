@@ -529,6 +529,30 @@ ct_status reexec_impl(ct_model *m, const float *input, int batch, const uint8_t 
 
 }  // namespace
 
+namespace ct {
+
+ct_status model_info(const ct_model *m, ModelInfo *out) {
+    if (!m || !out) return CT_EINVAL;
+    out->device = m->device;
+    out->in_c = m->in_c; out->in_h = m->in_h; out->in_w = m->in_w;
+    out->n_classes = m->n_classes;
+    out->max_batch = m->max_batch;
+    out->protect = m->protect ? 1 : 0;
+    return CT_OK;
+}
+
+ct_status infer_fault_free(ct_model *m, const float *input, int batch, float *logits, float *S,
+                           uint8_t *flag, cudaStream_t st) {
+    if (!m || batch < 1 || batch > m->max_batch) return CT_ERANGE;
+    const bool armed = m->armed;
+    m->armed = false;
+    ct_status s = infer_impl(m, input, batch, logits, S, flag, st);
+    m->armed = armed;
+    return s;
+}
+
+}  // namespace ct
+
 // ===========================================================================
 // C ABI
 // ===========================================================================

@@ -77,6 +77,15 @@ cudaError_t launch_gather_images(const float *in, float *out, const int32_t *idx
 cudaError_t launch_scatter_rows(const float *src, float *dst, const int32_t *idx, int n, int row,
                                 cudaStream_t st);
 
+// Model facts and a fault-free inference for code outside ct_api.cu.
+struct ModelInfo {
+    int device, in_c, in_h, in_w, n_classes, max_batch, protect;
+};
+ct_status model_info(const ct_model *m, ModelInfo *out);
+// ct_infer on device buffers with any armed fault left armed for the next ct_infer.
+ct_status infer_fault_free(ct_model *m, const float *input, int batch, float *logits, float *S,
+                           uint8_t *flag, cudaStream_t st);
+
 // tensor-core conv plan (opaque outside conv_tc.cu)
 struct TcPlan;
 TcPlan *tc_plan_create(const ConvArgs &shape_args, int max_batch, const void *w_dev, const void *x_dev,

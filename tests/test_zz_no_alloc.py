@@ -1,0 +1,70 @@
+"""ct_reexecute_noalloc: re-execution for callers that cannot allocate device
+memory at run time (device memory fixed at start-up, or an allocator owned
+by the host application).  Its scratch is a static device array instead of
+buffers made by ct_build; its results must equal ct_reexecute's.  This file
+is collected last on purpose."""
+import numpy as np
+import pytest
+
+from _cache import inputs
+from _gpu import TOL, ct, model, run
+
+pytestmark = pytest.mark.gpu
+
+
+def _flagging_threshold(m, S):
+    """A threshold that flags roughly half of the images (both entry points
+    then re-run the same, non-trivial set)."""
+    r = float(np.median(S))
+    ct().ct_set_threshold(m, r, float(np.median(np.abs(S - r))))
+
+
+def test_noalloc_reexecute_matches_reexecute_twice():
+    import torch
+    name, B = "resnet18_cifar", 16
+    m = model(name, max_batch=B)
+    x = inputs(name, B)
+    _, S0, _ = run(m, x)
+    _flagging_threshold(m, S0)
+    xd = torch.from_numpy(x).cuda()
+    for call in range(2):                       # two calls in a row
+        lg = torch.empty(B, m.n_classes, device="cuda")
+        S = torch.empty(B, device="cuda")
+        fl = torch.empty(B, dtype=torch.uint8, device="cuda")
+        # corrupt the rows first so that a re-run that writes nothing is caught
+        ct().ct_infer(m, xd, B, lg, S, fl)
+        flags = fl.clone()
+        lg_a, S_a = lg.clone(), S.clone()
+        lg_a[flags.bool()] = float("nan")
+        S_a[flags.bool()] = float("nan")
+        lg_b, S_b = lg_a.clone(), S_a.clone()
+        n_a = ct().ct_reexecute(m, xd, B, flags, lg_a, S_a)
+        n_b = ct().ct_reexecute_noalloc(m, xd, B, flags, lg_b, S_b)
+        torch.cuda.synchronize()
+        assert 0 < n_a < B and n_b == n_a, (call, n_a, n_b)
+        a, b = lg_a.cpu().numpy(), lg_b.cpu().numpy()
+        assert np.isfinite(b).all()
+        err = np.abs(a - b).max(axis=1) / np.maximum(np.abs(a).max(axis=1), 1e-6)
+        assert (err <= TOL["fp32"]).all(), (call, err.max())
+        sa, sb = S_a.cpu().numpy(), S_b.cpu().numpy()
+        assert (np.abs(sa - sb) <= TOL["fp32"] * np.abs(sa)).all(), call
+
+
+def test_noalloc_rejects_a_batch_beyond_its_scratch():
+    import torch
+    # 3 x 224 x 224 fp32 images are 602,112 bytes: 32 flagged images need
+    # about 19 MB of scratch, more than the 16 MiB array
+    name, B = "resnet18_imagenet", 32
+    m = model(name, max_batch=B)
+    xd = torch.from_numpy(inputs(name, B)).cuda()
+    fl = torch.ones(B, dtype=torch.uint8, device="cuda")
+    lg = torch.zeros(B, m.n_classes, device="cuda")
+    S = torch.zeros(B, device="cuda")
+    with pytest.raises(ct().CtError) as ei:
+        ct().ct_reexecute_noalloc(m, xd, B, fl, lg, S)
+    assert ei.value.status == 5                # CT_ERANGE
+    assert float(lg.abs().sum()) == 0.0        # nothing ran
+    fl[2:] = 0                                  # two images fit
+    assert ct().ct_reexecute_noalloc(m, xd, B, fl, lg, S) == 2
+    torch.cuda.synchronize()
+    assert np.isfinite(lg[:2].cpu().numpy()).all() and float(lg[2:].abs().sum()) == 0.0
