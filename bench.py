@@ -247,6 +247,12 @@ def main():
     # unprotected reference (same kernels, no carry-through filters)
     ms_u, _ = timed(step_unprotected, args.steps)
 
+    # protected inference alone (no re-execution): the cost of the filters
+    def step_protected_infer():
+        ct.ct_infer(mp, x, B, logits, S, flag, stream)
+        return 0
+    ms_pi, _ = timed(step_protected_infer, args.steps)
+
     # protected, timed, with clocks sampled and per-kernel events on the launch stream
     clk = ClockSampler(local if "CUDA_VISIBLE_DEVICES" not in os.environ else
                        int(os.environ["CUDA_VISIBLE_DEVICES"].split(",")[local]))
@@ -335,12 +341,17 @@ def main():
                    "simt_only": bool(args.simt_only)},
         "unprotected_value": value_u,
         "overhead_pct": 100.0 * (ms_p / ms_u - 1.0),
+        "overhead_filters_pct": 100.0 * (ms_pi / ms_u - 1.0),
+        "overhead_reexec_pct": 100.0 * (ms_p - ms_pi) / ms_u,
         "reexecuted_images_per_step": n_rerun / args.steps,
         "conv_tflop_per_batch": conv_flops(wl) / 1e12,
         "roofline": roof,
         "cpu_baseline": cpu,
         "e2e": {"value": world * B * args.steps / e2e_s, "unit": "images/s",
                 "h2d_bytes_per_step": in_bytes, "d2h_bytes_per_step": out_bytes},
+        "kernel_families": {nm: {"launches": fam_stats[i][0], "ms": fam_stats[i][1],
+                                 "tflop": fam_stats[i][2] / 1e12}
+                            for i, nm in enumerate(["conv_tc", "conv_simt", "fc", "pool", "other"])},
         "gpu_launches": launches,
         "clocks": clocks,
         "device_error": err,

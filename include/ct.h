@@ -238,6 +238,9 @@ ct_status ct_launches_per_infer(const ct_model *m, int32_t *n);
  * [batch, C] after a global average pool, [batch, n] after a hidden FC), in
  * the slot's storage type (FP32, or FP16 words as uint16); cs_host (may be
  * NULL) receives the checksum plane [batch, H, W] in the same type.
+ * When the first convolution runs on the tensor-core path for images with at
+ * most 4 channels, slot 0 is stored with 4 channels (the extra ones zero)
+ * and *C reports 4.
  * *C, *H, *W, *has_cs and *elem_bytes describe the slot (any may be NULL; call
  * first with data_host = NULL to query).  Synchronous.  CT_ERANGE for a slot
  * that is not stored (the classifier output) or batch > max_batch. */

@@ -372,6 +372,216 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
 }
 
 // ---------------------------------------------------------------------------
+// First layers with at most 4 input channels (the image): the input is
+// stored NHWC with its channels padded to 4 (8 bytes per pixel) and the GEMM
+// K index runs over (tap, channel of 4), 16 taps per 64-wide K block.  TMA
+// im2col cannot fetch 8-byte pixels, so four producer warps build the A tile
+// in shared memory: each thread owns one output pixel, loads one 8-byte
+// input pixel per tap and writes the 128-byte swizzled row the MMA reads.
+// Output channels: 64.  The carry-through row is coef at the centre tap's
+// real channels: 16 constant rows after the 64 weight rows of every B stage,
+// used (N = 80) on the centre tap's K block, which the loop visits first.
+// ---------------------------------------------------------------------------
+constexpr int SM_THREADS = 288;     // warps 0-3 producers, 4 MMA, 5-8 epilogue
+constexpr int SM_STAGES = 6;
+constexpr int SM_BN = 64;
+
+struct TcGeomS {
+    int M, PQ, Q, stride, pad, C, H, W, R, S;
+    int n_kb, kb_ct, col_ct, ct;
+    int tmem_cols;
+    uint16_t coef_h;
+};
+
+__device__ __forceinline__ void mbar_expect_tx_only(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__global__ void __launch_bounds__(SM_THREADS, 1)
+conv_tc_small_kernel(const __grid_constant__ CUtensorMap bmap, const ConvArgs a, const TcGeomS g) {
+    constexpr int B_ROWS = SM_BN + 16;
+    constexpr int B_BYTES_STAGE = B_ROWS * BK * 2;
+    constexpr int B_TMA_BYTES = SM_BN * BK * 2;
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint8_t *As = smem;
+    uint8_t *Bs = As + SM_STAGES * A_BYTES;
+    uint64_t *full = (uint64_t *)(Bs + SM_STAGES * B_BYTES_STAGE);
+    uint64_t *empty = full + SM_STAGES;
+    uint64_t *accum = empty + SM_STAGES;
+    uint32_t *tmem_holder = (uint32_t *)(accum + 1);
+    volatile uint32_t *abort_flag = tmem_holder + 1;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int m0 = blockIdx.x * BM;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < SM_STAGES; ++s) {
+            mbar_init(smem_u32(&full[s]), 128);
+            mbar_init(smem_u32(&empty[s]), 1);
+        }
+        mbar_init(smem_u32(accum), 1);
+        *abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 4) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_holder)),
+                     "r"((uint32_t)g.tmem_cols));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    if (warp >= 5) {
+        // constant rows 64..79 of every B stage: row 64 = coef at the centre
+        // tap's real channels (columns col_ct .. col_ct + C - 1), the rest 0;
+        // rows whose index is a multiple of 8 are not permuted by the swizzle
+        const int t = threadIdx.x - 160;
+        const __half ch = __ushort_as_half(g.coef_h);
+        for (int s = 0; s < SM_STAGES; ++s) {
+            __half *rows = (__half *)(Bs + s * B_BYTES_STAGE + SM_BN * BK * 2);
+            for (int i = t; i < 16 * BK; i += 128)
+                rows[i] = (g.ct && i >= g.col_ct && i < g.col_ct + g.C) ? ch : __ushort_as_half((unsigned short)0);
+        }
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tmem = *tmem_holder;
+    const __half *x = static_cast<const __half *>(a.x);
+
+    if (warp < 4) {
+        // ---------------- software im2col producers ----------------
+        const int row = threadIdx.x;
+        const int m = m0 + row;
+        const bool valid = m < g.M;
+        const int mm = valid ? m : 0;
+        const int nimg = mm / g.PQ, rem = mm % g.PQ, p = rem / g.Q, q = rem % g.Q;
+        const int h0 = p * g.stride - g.pad, w0 = q * g.stride - g.pad;
+        const int taps = g.R * g.S;
+        for (int it = 0; it < g.n_kb; ++it) {
+            const int kb = (it + g.kb_ct) % g.n_kb;
+            const int s = it % SM_STAGES;
+            const uint32_t ph = (uint32_t)(it / SM_STAGES) & 1u;
+            if (!mbar_wait(smem_u32(&empty[s]), ph ^ 1u, a.err, 1u)) { *abort_flag = 1; break; }
+            if (*abort_flag) break;
+            const uint32_t fb = smem_u32(&full[s]);
+            if (row == 0) {
+                mbar_expect_tx_only(fb, B_TMA_BYTES);
+                tma_load_2d(smem_u32(Bs + s * B_BYTES_STAGE), &bmap, fb, kb * BK, 0);
+            }
+            uint8_t *arow = As + s * A_BYTES + row * 128;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                uint2 v[2];
+#pragma unroll
+                for (int u = 0; u < 2; ++u) {
+                    const int tp = kb * 16 + 2 * j + u;
+                    v[u] = make_uint2(0u, 0u);
+                    if (valid && tp < taps) {
+                        const int h = h0 + tp / g.S, w = w0 + tp % g.S;
+                        if (h >= 0 && h < g.H && w >= 0 && w < g.W)
+                            v[u] = *reinterpret_cast<const uint2 *>(x + (((size_t)nimg * g.H + h) * g.W + w) * 4);
+                    }
+                }
+                *reinterpret_cast<uint4 *>(arow + ((j ^ (row & 7)) << 4)) = make_uint4(v[0].x, v[0].y, v[1].x, v[1].y);
+            }
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            mbar_arrive(fb);
+        }
+    } else if (warp == 4) {
+        if (lane == 0) {
+            // ---------------- MMA issuer ----------------
+            const uint32_t id_main = idesc_f16(BM, SM_BN);
+            const uint32_t id_merged = idesc_f16(BM, SM_BN + 16);
+            for (int it = 0; it < g.n_kb; ++it) {
+                const int s = it % SM_STAGES;
+                const uint32_t ph = (uint32_t)(it / SM_STAGES) & 1u;
+                if (!mbar_wait(smem_u32(&full[s]), ph, a.err, 2u)) { *abort_flag = 1; break; }
+                if (*abort_flag) break;
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                const uint32_t a_base = smem_u32(As + s * A_BYTES);
+                const uint32_t b_base = smem_u32(Bs + s * B_BYTES_STAGE);
+#pragma unroll
+                for (int k16 = 0; k16 < BK / 16; ++k16) {
+                    const uint64_t ad = smem_desc_sw128(a_base + k16 * 32);
+                    const uint64_t bd = smem_desc_sw128(b_base + k16 * 32);
+                    const uint32_t acc = (it > 0 || k16 > 0) ? 1u : 0u;
+                    umma_f16(tmem, ad, bd, (it == 0 && g.ct) ? id_merged : id_main, acc);
+                }
+                umma_commit(smem_u32(&empty[s]));
+            }
+            umma_commit(smem_u32(accum));
+        }
+    } else {
+        // ---------------- epilogue: warps 5..8 ----------------
+        const int quad = warp & 3;
+        const int row = quad * 32 + lane;
+        const int m = m0 + row;
+        bool ok = mbar_wait(smem_u32(accum), 0u, a.err, 4u) && !*abort_flag;
+        ok = __all_sync(0xffffffffu, ok);
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        if (ok) {
+            const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
+            const bool valid = m < g.M;
+            const int mm = valid ? m : 0;
+            const int nimg = mm / g.PQ, rem = mm % g.PQ, p = rem / g.Q, q = rem % g.Q;
+            __half *y = static_cast<__half *>(a.y);
+            const FaultDelta fd = a.fd;
+            float fsrc = 0.f;
+            if (fd.active) {
+                const int h = p * g.stride + fd.r - g.pad, w = q * g.stride + fd.s - g.pad;
+                if (fd.cin < g.C && h >= 0 && h < g.H && w >= 0 && w < g.W)
+                    fsrc = ldh(x, (((size_t)nimg * g.H + h) * g.W + w) * 4 + fd.cin);
+            }
+#pragma unroll 1
+            for (int ch = 0; ch < SM_BN; ch += 16) {
+                float v[16];
+                tmem_ld16(trow + ch, v);
+                if (valid) {
+                    uint32_t packed[8];
+#pragma unroll
+                    for (int i = 0; i < 16; i += 2) {
+                        float o[2];
+#pragma unroll
+                        for (int j = 0; j < 2; ++j) {
+                            const int k = ch + i + j;
+                            float t = v[i + j] + a.bias[k];
+                            if (fd.active && fd.kout == k) t += fd.dv * fsrc;
+                            if (a.relu) t = relu_keep_nan(t);
+                            o[j] = t;
+                        }
+                        __half2 hh = __floats2half2_rn(o[0], o[1]);
+                        packed[i / 2] = *reinterpret_cast<uint32_t *>(&hh);
+                    }
+                    uint4 *yp = reinterpret_cast<uint4 *>(y + (size_t)m * SM_BN + ch);
+                    yp[0] = make_uint4(packed[0], packed[1], packed[2], packed[3]);
+                    yp[1] = make_uint4(packed[4], packed[5], packed[6], packed[7]);
+                }
+            }
+            if (a.cs_out != nullptr) {
+                float ctv = 0.f;
+                if (g.ct) ctv = tmem_ld1(trow + SM_BN);
+                if (valid) {
+                    float o = (a.role == CT_ROLE_CT) ? ctv : 0.f;
+                    if (fd.active && fd.kout == SM_BN) o += fd.dv * fsrc;
+                    if (a.relu) o = relu_keep_nan(o);
+                    static_cast<__half *>(a.cs_out)[m] = __float2half_rn(o);
+                }
+            }
+        }
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if (warp == 4) {
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)g.tmem_cols));
+    }
+}
+
+// ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
 
@@ -476,6 +686,61 @@ TcPlan *tc_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, cons
     }
     if (e != cudaSuccess) { if (why) *why = "shared memory attribute"; delete pl; return nullptr; }
     return pl;
+}
+
+bool tc_small_supported(int C, int K, int R, int S, int stride, int pad) {
+    return C >= 1 && C <= 4 && K == SM_BN && R == S && R <= 7 && stride >= 1 && stride <= 2 && pad <= 3;
+}
+
+int tc_small_kpad(int R, int S) { return ((R * S * 4 + BK - 1) / BK) * BK; }
+
+struct TcSmallPlan {
+    CUtensorMap bmap;
+    TcGeomS g;
+    size_t smem;
+};
+
+TcSmallPlan *tc_small_plan_create(const ConvArgs &a, const void *w_dev, std::string *why) {
+    if (!load_encoders()) { if (why) *why = "tensor-map encoders unavailable"; return nullptr; }
+    TcSmallPlan *pl = new TcSmallPlan();
+    memset(pl, 0, sizeof(*pl));
+    TcGeomS &g = pl->g;
+    g.PQ = a.P * a.Q; g.Q = a.Q; g.stride = a.stride; g.pad = a.pad; g.C = a.C;
+    g.H = a.H; g.W = a.W; g.R = a.R; g.S = a.S;
+    const int kp = tc_small_kpad(a.R, a.S);
+    g.n_kb = kp / BK;
+    const int ctr_tap = ((a.R - 1) / 2) * a.S + (a.S - 1) / 2;
+    g.kb_ct = (ctr_tap * 4) / BK;
+    g.col_ct = (ctr_tap * 4) % BK;
+    g.ct = a.role == CT_ROLE_CT ? 1 : 0;
+    g.tmem_cols = 128;
+    g.coef_h = coef_half_bits(a.coef);
+    cuuint64_t bdim[2] = {(cuuint64_t)kp, (cuuint64_t)SM_BN};
+    cuuint64_t bstr[1] = {(cuuint64_t)kp * 2};
+    cuuint32_t box[2] = {BK, (cuuint32_t)SM_BN};
+    cuuint32_t bes[2] = {1, 1};
+    CUresult r = g_encode_tiled(&pl->bmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void *>(w_dev), bdim, bstr,
+                                box, bes, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                                CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) { if (why) *why = "weight tensor map"; delete pl; return nullptr; }
+    pl->smem = 1024 + (size_t)SM_STAGES * (A_BYTES + (SM_BN + 16) * BK * 2) + 8 * (2 * SM_STAGES + 1) + 16;
+    if (cudaFuncSetAttribute(conv_tc_small_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem) !=
+        cudaSuccess) {
+        if (why) *why = "shared memory attribute";
+        delete pl;
+        return nullptr;
+    }
+    return pl;
+}
+
+void tc_small_plan_destroy(TcSmallPlan *p) { delete p; }
+
+cudaError_t launch_conv_tc_small(const ConvArgs &a, const TcSmallPlan *pl, cudaStream_t st) {
+    TcGeomS g = pl->g;
+    g.M = a.N * a.P * a.Q;
+    dim3 grid((g.M + BM - 1) / BM);
+    conv_tc_small_kernel<<<grid, SM_THREADS, pl->smem, st>>>(pl->bmap, a, g);
+    return cudaGetLastError();
 }
 
 void tc_plan_destroy(TcPlan *p) { delete p; }

@@ -73,6 +73,7 @@ float bits_float(uint32_t u) { float f; memcpy(&f, &u, 4); return f; }
 
 struct Slot {
     int C = 0, H = 0, W = 0;
+    int cp = 0;                  // channel pitch of the NHWC data (C, or 4 for a padded image)
     bool has_cs = false;
     bool is_float = false;       // GAP output: fp32 features whatever the precision
     void *data = nullptr;
@@ -90,6 +91,9 @@ struct LayerRT {
     float *bias = nullptr;
     bool tc = false;
     TcPlan *plan = nullptr;
+    bool tc_small = false;       // first layer with <= 4 input channels on the tensor cores
+    TcSmallPlan *splan = nullptr;
+    int w_ld = 0, c_stride = 0;  // weight row length and channel stride within a tap
     // fc
     int n_in = 0, n_cs = 0, n_out = 0;
     bool x_float = false;
@@ -158,8 +162,10 @@ ct_status dalloc(ct_model *m, void **p, size_t bytes) {
 }
 
 void free_all(ct_model *m) {
-    for (auto &l : m->L)
+    for (auto &l : m->L) {
         if (l.plan) tc_plan_destroy(l.plan);
+        if (l.splan) tc_small_plan_destroy(l.splan);
+    }
     for (void *p : m->dev_allocs) cudaFree(p);
     m->dev_allocs.clear();
     if (m->h_flags) cudaFreeHost(m->h_flags);
@@ -267,7 +273,17 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
             std::string why;
             l.tc = prec == CT_FP16 && !(m->flags & CT_FLAG_SIMT_ONLY) &&
                    tc_supported(l.C, l.K, l.R, l.S, d.stride, d.pad, &why);
-            std::vector<uint8_t> hw((size_t)l.K * RSC * esz, 0);
+            if (prec == CT_FP16 && !(m->flags & CT_FLAG_SIMT_ONLY) && d.src == 0 &&
+                tc_small_supported(l.C, l.K, l.R, l.S, d.stride, d.pad)) {
+                int readers = 0;               // the padded image must have no other reader
+                for (int j = 0; j < nL; ++j)
+                    readers += (desc->layers[j].src == 0) + (desc->layers[j].res == 0);
+                l.tc_small = readers == 1;
+            }
+            l.w_ld = l.tc_small ? tc_small_kpad(l.R, l.S) : RSC;
+            l.c_stride = l.tc_small ? 4 : l.C;
+            if (l.tc_small) src.cp = 4;
+            std::vector<uint8_t> hw((size_t)l.K * l.w_ld * esz, 0);
             std::vector<float> hb(l.K, 0.f);
             for (int k = 0; k < l.K; ++k) {
                 double scale = 1.0, shift = bias ? (double)bias[k] : 0.0;
@@ -284,7 +300,7 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
                     for (int r = 0; r < l.R; ++r)
                         for (int s = 0; s < l.S; ++s) {
                             double v = (double)W[(((size_t)k * l.C + c) * l.R + r) * l.S + s] * scale;
-                            put(hw, (size_t)k * RSC + ((size_t)r * l.S + s) * l.C + c, v, prec);
+                            put(hw, (size_t)k * l.w_ld + ((size_t)r * l.S + s) * l.c_stride + c, v, prec);
                         }
             }
             ct_status st;
@@ -342,12 +358,22 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
         for (auto &l : m->L) if (l.d.op == CT_OP_FC && l.d.final && l.d.dst == (int)s) is_final_out = true;
         if (is_final_out) continue;
         const size_t e = sl.is_float ? 4 : esz;
+        if (sl.cp < sl.C) sl.cp = sl.C;
         ct_status st;
-        if ((st = dalloc(m, &sl.data, (size_t)B * sl.H * sl.W * sl.C * e)) != CT_OK) return st;
+        if ((st = dalloc(m, &sl.data, (size_t)B * sl.H * sl.W * sl.cp * e)) != CT_OK) return st;
         if (sl.has_cs && (st = dalloc(m, &sl.cs, (size_t)B * sl.H * sl.W * e)) != CT_OK) return st;
     }
     // ---- tensor-core plans ----
     for (auto &l : m->L) {
+        if (l.tc_small) {
+            ConvArgs a{};
+            a.N = B; a.H = l.H; a.W = l.W; a.C = l.C; a.K = l.K; a.R = l.R; a.S = l.S;
+            a.stride = l.d.stride; a.pad = l.d.pad; a.P = l.P; a.Q = l.Q; a.role = l.role; a.coef = l.coef;
+            std::string why;
+            l.splan = tc_small_plan_create(a, l.w, &why);
+            if (!l.splan) return CT_ECUDA;
+            continue;
+        }
         if (!l.tc) continue;
         ConvArgs a{};
         a.N = B; a.H = l.H; a.W = l.W; a.C = l.C; a.K = l.K; a.R = l.R; a.S = l.S;
@@ -397,12 +423,11 @@ WeightFault resolve_weight_fault(const ct_model *m, const LayerRT &l, int64_t e,
     const int k = (int)(e / ((int64_t)Ct * RS));
     const int c = (int)((e / RS) % Ct);
     const int r = (int)((e / l.S) % l.R), s = (int)(e % l.S);
-    const int RSC = l.R * l.S * l.C;
     const bool centre = r == (l.R - 1) / 2 && s == (l.S - 1) / 2;
     WeightFault f;
     if (k < l.K && c < l.C) {
         f.explicit_word = true;
-        f.word = (int64_t)k * RSC + ((int64_t)r * l.S + s) * l.C + c;
+        f.word = (int64_t)k * l.w_ld + ((int64_t)r * l.S + s) * l.c_stride + c;
         return f;
     }
     double stored = 0.0;                      // zero slice and off-centre taps
@@ -426,7 +451,7 @@ ct_status act_fault_word(const ct_model *m, int slot, int batch, int64_t e, void
     const int64_t n = e / (Ct * HW);
     const int c = (int)((e / HW) % Ct);
     const int64_t hw = e % HW;
-    if (c < sl.C) { *base = sl.data; *word = (n * HW + hw) * sl.C + c; }
+    if (c < sl.C) { *base = sl.data; *word = (n * HW + hw) * sl.cp + c; }
     else { *base = sl.cs; *word = n * HW + hw; }
     return CT_OK;
 }
@@ -450,7 +475,7 @@ ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, 
     }
     Slot &s0 = m->slots[0];
     CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] {
-        return launch_convert_input(input, s0.data, batch, s0.C, s0.H, s0.W, half, st);
+        return launch_convert_input(input, s0.data, batch, s0.C, s0.cp, s0.H, s0.W, half, st);
     }));
     if (act_slot == 0) CUDA_TRY(launch_xor_bit(act_base, act_word, m->f_bit, wb, st));
     for (size_t i = 0; i < m->L.size(); ++i) {
@@ -477,7 +502,8 @@ ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, 
                 else a.fd = wf.fd;
             }
             const double flops = 2.0 * batch * l.P * l.Q * (double)l.K * l.R * l.S * l.C;
-            if (l.tc) CUDA_TRY(launch(m, FAM_TC, flops, st, [&] { return launch_conv_tc(a, l.plan, st); }));
+            if (l.tc_small) CUDA_TRY(launch(m, FAM_TC, flops, st, [&] { return launch_conv_tc_small(a, l.splan, st); }));
+            else if (l.tc) CUDA_TRY(launch(m, FAM_TC, flops, st, [&] { return launch_conv_tc(a, l.plan, st); }));
             else CUDA_TRY(launch(m, FAM_SIMT, flops, st, [&] { return launch_conv_simt(a, half, st); }));
             if (wfault && wf.explicit_word) CUDA_TRY(launch_xor_bit(l.w, wf.word, m->f_bit, wb, st));
         } else if (d.op == CT_OP_MAXPOOL || d.op == CT_OP_GAP) {
@@ -785,7 +811,7 @@ ct_status ct_copy_activation(ct_model *m, int32_t slot, int32_t batch, void *dat
     const Slot &sl = m->slots[slot];
     if (!sl.data) return CT_ERANGE;
     const size_t e = sl.is_float ? 4 : m->esz();
-    if (C) *C = sl.C;
+    if (C) *C = sl.cp;
     if (H) *H = sl.H;
     if (W) *W = sl.W;
     if (has_cs) *has_cs = sl.has_cs ? 1 : 0;
@@ -794,7 +820,7 @@ ct_status ct_copy_activation(ct_model *m, int32_t slot, int32_t batch, void *dat
     DeviceGuard g(m->device);
     cudaStream_t st = (cudaStream_t)stream;
     const size_t hw = (size_t)batch * sl.H * sl.W;
-    CUDA_TRY(cudaMemcpyAsync(data_host, sl.data, hw * sl.C * e, cudaMemcpyDeviceToHost, st));
+    CUDA_TRY(cudaMemcpyAsync(data_host, sl.data, hw * sl.cp * e, cudaMemcpyDeviceToHost, st));
     if (cs_host && sl.has_cs) CUDA_TRY(cudaMemcpyAsync(cs_host, sl.cs, hw * e, cudaMemcpyDeviceToHost, st));
     CUDA_TRY(cudaStreamSynchronize(st));
     return CT_OK;

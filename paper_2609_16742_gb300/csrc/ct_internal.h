@@ -69,7 +69,7 @@ cudaError_t launch_conv_tc(const ConvArgs &a, const void *tc_plan, cudaStream_t 
 cudaError_t launch_fc(const FcArgs &a, bool half, bool x_float, cudaStream_t st);
 cudaError_t launch_maxpool(const PoolArgs &a, bool half, cudaStream_t st);
 cudaError_t launch_gap(const PoolArgs &a, bool half, cudaStream_t st);
-cudaError_t launch_convert_input(const float *in, void *out, int N, int C, int H, int W, bool half,
+cudaError_t launch_convert_input(const float *in, void *out, int N, int C, int Cp, int H, int W, bool half,
                                  cudaStream_t st);
 cudaError_t launch_xor_bit(void *base, int64_t word, int bit, int word_bytes, cudaStream_t st);
 cudaError_t launch_gather_images(const float *in, float *out, const int32_t *idx, int n,
@@ -92,5 +92,15 @@ TcPlan *tc_plan_create(const ConvArgs &shape_args, int max_batch, const void *w_
                        std::string *why);
 void tc_plan_destroy(TcPlan *p);
 bool tc_supported(int C, int K, int R, int S, int stride, int pad, std::string *why);
+
+// tensor-core conv for first layers with at most 4 input channels (input
+// stored NHWC with 4 channels; weights [64][tc_small_kpad] with K index
+// tap * 4 + channel)
+struct TcSmallPlan;
+bool tc_small_supported(int C, int K, int R, int S, int stride, int pad);
+int tc_small_kpad(int R, int S);
+TcSmallPlan *tc_small_plan_create(const ConvArgs &shape_args, const void *w_dev, std::string *why);
+void tc_small_plan_destroy(TcSmallPlan *p);
+cudaError_t launch_conv_tc_small(const ConvArgs &a, const TcSmallPlan *plan, cudaStream_t st);
 
 }  // namespace ct

@@ -129,10 +129,68 @@ __global__ void __launch_bounds__(256) fc_kernel(FcArgs a) {
 // ---------------------------------------------------------------------------
 // Max-pool over NHWC data and the [N, H, W] checksum plane together.  The
 // window maximum is taken on stored values (exact); padding never wins; a
-// NaN anywhere in the window gives NaN.
+// NaN anywhere in the window gives NaN.  Data: one thread per output pixel
+// and 8 (fp16) or 4 (fp32) consecutive channels, 16-byte loads and stores;
+// the checksum plane: one thread per output pixel.
 // ---------------------------------------------------------------------------
+__device__ __forceinline__ void vmax(float &m, float v) { m = (v > m || v != v) ? v : m; }
+
 template <typename T>
 __global__ void maxpool_kernel(PoolArgs a) {
+    constexpr int VE = 16 / sizeof(T);
+    using V = uint4;
+    const int CV = a.C / VE;                       // vectors per pixel (C % VE == 0)
+    const int n_pix = a.N * a.P * a.Q;
+    const int n_data = n_pix * CV;
+    const int n_all = n_data + (a.cs_in ? n_pix : 0);
+    for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < n_all; e += gridDim.x * blockDim.x) {
+        const bool is_cs = e >= n_data;
+        const int i = is_cs ? e - n_data : e;
+        const int cv = is_cs ? 0 : i % CV;
+        const int pix = is_cs ? i : i / CV;
+        const int q = pix % a.Q, t = pix / a.Q, p = t % a.P, n = t / a.P;
+        if (is_cs) {
+            const T *src = static_cast<const T *>(a.cs_in);
+            float m = -INFINITY;
+            for (int r = 0; r < a.k; ++r) {
+                const int h = p * a.stride + r - a.pad;
+                if (h < 0 || h >= a.H) continue;
+                for (int s = 0; s < a.k; ++s) {
+                    const int w = q * a.stride + s - a.pad;
+                    if (w < 0 || w >= a.W) continue;
+                    vmax(m, to_f(src[((size_t)n * a.H + h) * a.W + w]));
+                }
+            }
+            static_cast<T *>(a.cs_out)[pix] = from_f<T>(m);
+            continue;
+        }
+        float m[VE];
+#pragma unroll
+        for (int j = 0; j < VE; ++j) m[j] = -INFINITY;
+        const T *src = static_cast<const T *>(a.x);
+        for (int r = 0; r < a.k; ++r) {
+            const int h = p * a.stride + r - a.pad;
+            if (h < 0 || h >= a.H) continue;
+            for (int s = 0; s < a.k; ++s) {
+                const int w = q * a.stride + s - a.pad;
+                if (w < 0 || w >= a.W) continue;
+                const V v = *reinterpret_cast<const V *>(src + (((size_t)n * a.H + h) * a.W + w) * a.C + cv * VE);
+                const T *tv = reinterpret_cast<const T *>(&v);
+#pragma unroll
+                for (int j = 0; j < VE; ++j) vmax(m[j], to_f(tv[j]));
+            }
+        }
+        V o;
+        T *to = reinterpret_cast<T *>(&o);
+#pragma unroll
+        for (int j = 0; j < VE; ++j) to[j] = from_f<T>(m[j]);
+        *reinterpret_cast<V *>(static_cast<T *>(a.y) + (size_t)pix * a.C + cv * VE) = o;
+    }
+}
+
+// Scalar fallback for channel counts that are not a multiple of the vector.
+template <typename T>
+__global__ void maxpool_scalar_kernel(PoolArgs a) {
     const int64_t n_data = (int64_t)a.N * a.P * a.Q * a.C;
     const int64_t n_cs = a.cs_in ? (int64_t)a.N * a.P * a.Q : 0;
     for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n_data + n_cs;
@@ -147,19 +205,15 @@ __global__ void maxpool_kernel(PoolArgs a) {
         const int n = (int)(t / a.P);
         const T *src = static_cast<const T *>(is_cs ? a.cs_in : a.x);
         float m = -INFINITY;
-        bool nan = false;
         for (int r = 0; r < a.k; ++r) {
             int h = p * a.stride + r - a.pad;
             if (h < 0 || h >= a.H) continue;
             for (int s = 0; s < a.k; ++s) {
                 int w = q * a.stride + s - a.pad;
                 if (w < 0 || w >= a.W) continue;
-                float v = to_f(src[(((size_t)n * a.H + h) * a.W + w) * C + c]);
-                nan |= (v != v);
-                m = v > m ? v : m;
+                vmax(m, to_f(src[(((size_t)n * a.H + h) * a.W + w) * C + c]));
             }
         }
-        if (nan) m = __int_as_float(0x7fc00000);
         T *dst = static_cast<T *>(is_cs ? a.cs_out : a.y);
         dst[i] = from_f<T>(m);
     }
@@ -184,17 +238,17 @@ __global__ void gap_kernel(PoolArgs a) {
     }
 }
 
+// NCHW fp32 -> NHWC storage type, one thread per pixel; channels C..Cp-1
+// of the output (padding to Cp channels) are written as zeros.
 template <typename T>
-__global__ void convert_input_kernel(const float *in, T *out, int N, int C, int H, int W) {
-    const int64_t total = (int64_t)N * C * H * W;
-    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
-         e += (int64_t)gridDim.x * blockDim.x) {
-        int c = (int)(e % C);
-        int64_t t = e / C;
-        int w = (int)(t % W); t /= W;
-        int h = (int)(t % H);
-        int n = (int)(t / H);
-        out[e] = from_f<T>(in[(((size_t)n * C + c) * H + h) * W + w]);
+__global__ void convert_input_kernel(const float *in, T *out, int N, int C, int Cp, int H, int W) {
+    const int HW = H * W;
+    const int total = N * HW;
+    for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < total; e += gridDim.x * blockDim.x) {
+        const int n = e / HW, hw = e % HW;
+        const float *src = in + (size_t)n * C * HW + hw;
+        T *dst = out + (size_t)e * Cp;
+        for (int c = 0; c < Cp; ++c) dst[c] = from_f<T>(c < C ? src[(size_t)c * HW] : 0.f);
     }
 }
 
@@ -259,9 +313,17 @@ cudaError_t launch_fc(const FcArgs &a, bool half, bool x_float, cudaStream_t st)
 }
 
 cudaError_t launch_maxpool(const PoolArgs &a, bool half, cudaStream_t st) {
-    int64_t n = (int64_t)a.N * a.P * a.Q * (a.C + (a.cs_in ? 1 : 0));
-    if (half) maxpool_kernel<__half><<<grid_for(n, 256), 256, 0, st>>>(a);
-    else maxpool_kernel<float><<<grid_for(n, 256), 256, 0, st>>>(a);
+    const int ve = half ? 8 : 4;
+    const int64_t pix = (int64_t)a.N * a.P * a.Q;
+    if (a.C % ve == 0 && pix * (a.C / ve + 1) < (1ll << 31)) {
+        const int64_t n = pix * (a.C / ve + (a.cs_in ? 1 : 0));
+        if (half) maxpool_kernel<__half><<<grid_for(n, 256), 256, 0, st>>>(a);
+        else maxpool_kernel<float><<<grid_for(n, 256), 256, 0, st>>>(a);
+    } else {
+        const int64_t n = pix * (a.C + (a.cs_in ? 1 : 0));
+        if (half) maxpool_scalar_kernel<__half><<<grid_for(n, 256), 256, 0, st>>>(a);
+        else maxpool_scalar_kernel<float><<<grid_for(n, 256), 256, 0, st>>>(a);
+    }
     return cudaGetLastError();
 }
 
@@ -272,11 +334,11 @@ cudaError_t launch_gap(const PoolArgs &a, bool half, cudaStream_t st) {
     return cudaGetLastError();
 }
 
-cudaError_t launch_convert_input(const float *in, void *out, int N, int C, int H, int W, bool half,
+cudaError_t launch_convert_input(const float *in, void *out, int N, int C, int Cp, int H, int W, bool half,
                                  cudaStream_t st) {
-    int64_t n = (int64_t)N * C * H * W;
-    if (half) convert_input_kernel<__half><<<grid_for(n, 256), 256, 0, st>>>(in, (__half *)out, N, C, H, W);
-    else convert_input_kernel<float><<<grid_for(n, 256), 256, 0, st>>>(in, (float *)out, N, C, H, W);
+    const int64_t n = (int64_t)N * H * W;
+    if (half) convert_input_kernel<__half><<<grid_for(n, 256), 256, 0, st>>>(in, (__half *)out, N, C, Cp, H, W);
+    else convert_input_kernel<float><<<grid_for(n, 256), 256, 0, st>>>(in, (float *)out, N, C, Cp, H, W);
     return cudaGetLastError();
 }
 

@@ -45,6 +45,7 @@ def layer_errors(name, prec, batch, simt_only=False, first=0):
     ("resnet18_cifar", "fp32", 2, False),
     ("resnet18_imagenet", "fp16", 2, False),
     ("lenet5", "fp32", 5, False),
+    ("vgg16", "fp16", 1, False),
 ])
 def test_every_stored_tensor_matches_oracle(name, prec, batch, simt_only):
     errs = layer_errors(name, prec, batch, simt_only)
