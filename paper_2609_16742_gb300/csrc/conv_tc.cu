@@ -17,9 +17,18 @@
 //   The incoming checksum plane (weight coef at the centre) and the
 //   epilogue (bias, residual, ReLU) are applied by the epilogue warps.
 //
-// Warp roles (192 threads): warp 0 issues TMA, warp 1 allocates TMEM and
-// issues tcgen05.mma (one elected lane), warps 2-5 read the accumulator
-// (each thread owns one output pixel) and store data and checksum.
+// The kernels are persistent: one CTA per SM walks a static list of output
+// tiles.  The TMA producer runs ahead across tile boundaries through a ring
+// of shared-memory stages.  Consecutive K blocks accumulate into up to four
+// independent TMEM accumulators (chains), because back-to-back MMAs into one
+// accumulator wait on each other; the epilogue sums the chains, and for
+// N <= 128 releases TMEM before its global stores so that the next tile's
+// MMAs overlap them.
+//
+// Warp roles (320 threads): warp 0 issues TMA, warp 1 allocates TMEM and
+// issues tcgen05.mma (one elected lane), warps 2-9 read the accumulator:
+// each TMEM lane quadrant (32 output pixels) is read by two warps, each
+// taking half of the tile's channels.
 // Every mbarrier wait is bounded; on expiry the kernel records an error code
 // in a device word, stops issuing work and exits after releasing TMEM.
 #include <cuda.h>
@@ -37,8 +46,11 @@ namespace {
 constexpr int BM = 128;            // output pixels per tile (TMEM lanes)
 constexpr int BK = 64;             // channels per K block (128 bytes of fp16)
 constexpr int A_BYTES = BM * BK * 2;
-constexpr int NTHREADS = 192;
-constexpr uint64_t WAIT_NS = 2000000000ull;   // 2 s bound on any single wait
+constexpr int NTHREADS = 320;      // 1 TMA warp, 1 MMA warp, 8 epilogue warps
+constexpr int N_EPI_WARPS = 8;
+// Bound on any single wait: 2^32 SM cycles (about 2 to 3 s at the clocks
+// this part runs at), measured with the cheap per-SM cycle counter.
+constexpr long long WAIT_CYCLES = 1ll << 32;
 
 enum CtMode { CT_NONE_ = 0, CT_MERGED = 1, CT_SEPARATE = 2 };
 
@@ -47,6 +59,7 @@ struct TcGeom {
     int n_kb, cpb, ctr_tap, S;
     int ct_mode;
     int tmem_cols;
+    int m_tiles, n_tiles;
     uint16_t coef_h;
 };
 
@@ -54,19 +67,21 @@ __device__ __forceinline__ uint32_t smem_u32(const void *p) {
     return (uint32_t)__cvta_generic_to_shared(p);
 }
 
-__device__ __forceinline__ uint64_t globaltimer() {
-    uint64_t t;
-    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-    return t;
-}
-
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count));
 }
 
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
                  : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx_only(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }
 
 __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
@@ -81,20 +96,38 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
     return ok != 0;
 }
 
-// Bounded wait: true on completion, false (and error code recorded) after WAIT_NS.
-__device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint32_t *err, uint32_t code) {
+// Bounded wait: true on completion, false (and error code recorded) after
+// WAIT_CYCLES.  try_wait suspends the thread until the phase completes or a
+// short hardware time limit passes; the cycle counter is read only every 256
+// polls so that the common case costs nothing extra.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint32_t *err, uint32_t code) {
     if (mbar_try_wait(bar, parity)) return true;
-    const uint64_t t0 = globaltimer();
-    for (uint32_t it = 0;; ++it) {
+    const long long t0 = clock64();
+    for (uint32_t it = 1;; ++it) {
         if (mbar_try_wait(bar, parity)) return true;
-        if ((it & 63) == 63) {
-            if (globaltimer() - t0 > WAIT_NS) {
-                atomicOr(err, code);
-                return false;
-            }
-            __nanosleep(128);
+        if ((it & 255) == 0 && clock64() - t0 > WAIT_CYCLES) {
+            atomicOr(err, code);
+            return false;
         }
     }
+}
+
+// One lane of a converged warp: issues TMA / tcgen05 instructions while the
+// whole warp computes their (warp-uniform) operands.
+__device__ __forceinline__ bool elect_one() {
+    uint32_t pred;
+    asm volatile(
+        "{\n\t.reg .pred P;\n\t"
+        "elect.sync _|P, 0xffffffff;\n\t"
+        "selp.b32 %0, 1, 0, P;\n\t}"
+        : "=r"(pred));
+    return pred != 0;
+}
+
+// Bounded wait by a whole warp; true only if every lane saw the phase complete.
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, uint32_t *err, uint32_t code) {
+    const bool ok = mbar_wait(bar, parity, err, code);
+    return __all_sync(0xffffffffu, ok);
 }
 
 __device__ __forceinline__ void tma_load_im2col(uint32_t dst, const CUtensorMap *map, uint32_t bar, int c,
@@ -170,35 +203,108 @@ __device__ __forceinline__ float ldh(const __half *p, size_t i) { return __half2
 // tap visited at K-block kb: the centre tap first, the others in order
 __device__ __forceinline__ int tap_of(int t, int ctr) { return t == 0 ? ctr : (t <= ctr ? t - 1 : t); }
 
-template <int BN, int STAGES>
-__global__ void __launch_bounds__(NTHREADS, BN <= 128 ? 2 : 1)
+// Epilogue of one 16-channel chunk for one output pixel m: bias, fault delta,
+// residual, ReLU, fp16 store (32 bytes).
+__device__ __forceinline__ void store_chunk(const float *v, const ConvArgs &a, int K, size_t m, int k0,
+                                            float fsrc) {
+    const __half *res = static_cast<const __half *>(a.res);
+    const size_t base = m * K + k0;
+    float rv[16];
+    if (res) {
+        const uint4 *rp = reinterpret_cast<const uint4 *>(res + base);
+        uint4 r0 = rp[0], r1 = rp[1];
+        const __half2 *h0 = reinterpret_cast<const __half2 *>(&r0);
+        const __half2 *h1 = reinterpret_cast<const __half2 *>(&r1);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            float2 f0 = __half22float2(h0[i]), f1 = __half22float2(h1[i]);
+            rv[2 * i] = f0.x; rv[2 * i + 1] = f0.y; rv[8 + 2 * i] = f1.x; rv[8 + 2 * i + 1] = f1.y;
+        }
+    }
+    const FaultDelta &fd = a.fd;
+    uint32_t packed[8];
+#pragma unroll
+    for (int i = 0; i < 16; i += 2) {
+        float o[2];
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+            const int k = k0 + i + j;
+            float t = v[i + j] + __ldg(a.bias + k);
+            if (fd.active && fd.kout == k) t += fd.dv * fsrc;
+            if (res) t += rv[i + j];
+            if (a.relu) t = relu_keep_nan(t);
+            o[j] = t;
+        }
+        __half2 hh = __floats2half2_rn(o[0], o[1]);
+        packed[i / 2] = *reinterpret_cast<uint32_t *>(&hh);
+    }
+    uint4 *yp = reinterpret_cast<uint4 *>(static_cast<__half *>(a.y) + base);
+    yp[0] = make_uint4(packed[0], packed[1], packed[2], packed[3]);
+    yp[1] = make_uint4(packed[4], packed[5], packed[6], packed[7]);
+}
+
+// The checksum output of one pixel: carry-through column + coef * incoming
+// checksum (centre pixel, or the sum of an FC layer's checksum features),
+// fault delta, residual checksum, ReLU.
+__device__ __forceinline__ void store_checksum(float ctv, const ConvArgs &a, const TcGeom &g, int m, int nimg,
+                                               int p, int q, float fsrc) {
+    const __half *csi = static_cast<const __half *>(a.cs_in);
+    const int ctr_r = g.ctr_tap / g.S, ctr_s = g.ctr_tap % g.S;
+    const int hc = p * g.stride + ctr_r - g.pad, wc = q * g.stride + ctr_s - g.pad;
+    const bool inb = hc >= 0 && hc < a.H && wc >= 0 && wc < a.W;
+    float cin = 0.f;
+    if (csi && a.cs_rowsum > 0) {                  // FC layer: every incoming checksum feature
+        for (int i = 0; i < a.cs_rowsum; ++i) cin += ldh(csi, (size_t)m * a.cs_rowsum + i);
+    } else if (csi && inb) {
+        cin = ldh(csi, ((size_t)nimg * a.H + hc) * a.W + wc);
+    }
+    float o = 0.f;
+    if (a.role == CT_ROLE_CT) o = ctv + a.coef * cin;
+    else if (a.role == CT_ROLE_PASS) o = cin;
+    if (a.fd.active && a.fd.kout == g.K) o += a.fd.dv * fsrc;
+    if (a.res_cs) o += ldh(static_cast<const __half *>(a.res_cs), (size_t)m);
+    if (a.relu) o = relu_keep_nan(o);
+    static_cast<__half *>(a.cs_out)[m] = __float2half_rn(o);
+}
+
+// K-block kb accumulates into chain kb % NCH: back-to-back MMAs into one
+// TMEM accumulator serialise on it, so NCH independent chains keep the
+// tensor pipe busy when one 128 x BN x 16 MMA is short (BN = 64, 128).  The
+// epilogue adds the chains.  SUB K-blocks share one pipeline stage (one
+// barrier round trip).  A single TMEM buffer holds the chains; for
+// BN <= 128 the epilogue copies it to registers and releases it before its
+// global stores, so the next tile's MMAs overlap the stores.
+template <int BN, int STAGES, int SUB, int NCH>
+__global__ void __launch_bounds__(NTHREADS, 1)
 conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
                const ConvArgs a, const TcGeom g) {
     constexpr int B_ROWS = BN + 16;                       // 16 constant carry-through rows
-    constexpr int B_BYTES_STAGE = B_ROWS * BK * 2;
+    constexpr int B_SUB_BYTES = B_ROWS * BK * 2;
     constexpr int B_TMA_BYTES = BN * BK * 2;
+    constexpr int CH = BN + 16;                           // TMEM columns per chain
+    constexpr bool EARLY = BN <= 128;                     // release TMEM before the stores
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-    uint8_t *As = smem;
-    uint8_t *Bs = As + STAGES * A_BYTES;
-    uint8_t *CTt = Bs + STAGES * B_BYTES_STAGE;           // separate 16-row carry-through tile
+    uint8_t *As = smem;                                   // [STAGES][SUB][A_BYTES]
+    uint8_t *Bs = As + STAGES * SUB * A_BYTES;            // [STAGES][SUB][B_SUB_BYTES]
+    uint8_t *CTt = Bs + STAGES * SUB * B_SUB_BYTES;       // separate 16-row carry-through tile
     uint64_t *full = (uint64_t *)(CTt + 16 * BK * 2);
     uint64_t *empty = full + STAGES;
-    uint64_t *accum = empty + STAGES;
-    uint32_t *tmem_holder = (uint32_t *)(accum + 1);
+    uint64_t *acc_full = empty + STAGES;
+    uint64_t *acc_empty = acc_full + 1;
+    uint32_t *tmem_holder = (uint32_t *)(acc_empty + 1);
     volatile uint32_t *abort_flag = tmem_holder + 1;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int m0 = blockIdx.x * BM;
-    const int n_tile = blockIdx.y;
-    const bool ct_here = g.ct_mode != CT_NONE_ && n_tile == 0;
+    const int num_tiles = g.m_tiles * g.n_tiles;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(smem_u32(&full[s]), 1);
             mbar_init(smem_u32(&empty[s]), 1);
         }
-        mbar_init(smem_u32(accum), 1);
+        mbar_init(smem_u32(acc_full), 1);
+        mbar_init(smem_u32(acc_empty), N_EPI_WARPS);
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -211,12 +317,12 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
         // constant carry-through rows: row 0 = coef, rows 1..15 = 0 (swizzle-invariant)
         const uint32_t coef2 = (uint32_t)g.coef_h | ((uint32_t)g.coef_h << 16);
         const int t = threadIdx.x - 64;
-        for (int s = 0; s < STAGES; ++s) {
-            uint32_t *rows = (uint32_t *)(Bs + s * B_BYTES_STAGE + BN * BK * 2);
-            for (int i = t; i < 16 * BK / 2; i += 128) rows[i] = (i < BK / 2) ? coef2 : 0u;
+        for (int sb = 0; sb < STAGES * SUB; ++sb) {
+            uint32_t *rows = (uint32_t *)(Bs + sb * B_SUB_BYTES + BN * BK * 2);
+            for (int i = t; i < 16 * BK / 2; i += 32 * N_EPI_WARPS) rows[i] = (i < BK / 2) ? coef2 : 0u;
         }
         uint32_t *ctt = (uint32_t *)CTt;
-        for (int i = t; i < 16 * BK / 2; i += 128) ctt[i] = (i < BK / 2) ? coef2 : 0u;
+        for (int i = t; i < 16 * BK / 2; i += 32 * N_EPI_WARPS) ctt[i] = (i < BK / 2) ? coef2 : 0u;
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     }
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -225,75 +331,118 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
     const uint32_t tmem = *tmem_holder;
 
     if (warp == 0) {
-        if (lane == 0) {
-            // ---------------- TMA producer ----------------
+        // ---------------- TMA producer (whole warp, one lane issues) ----------------
+        if (elect_one()) {
+            asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&amap) : "memory");
+            asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&bmap) : "memory");
+        }
+        __syncwarp();
+        int it = 0;
+        for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
+            if (__any_sync(0xffffffffu, *abort_flag)) break;
+            const int m0 = (tile / g.n_tiles) * BM, n_tile = tile % g.n_tiles;
             const int nimg = m0 / g.PQ, rem = m0 % g.PQ;
             const int p = rem / g.Q, q = rem % g.Q;
             const int w0 = q * g.stride - g.pad, h0 = p * g.stride - g.pad;
-            for (int kb = 0; kb < g.n_kb; ++kb) {
-                const int s = kb % STAGES;
-                const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
-                if (!mbar_wait(smem_u32(&empty[s]), ph ^ 1u, a.err, 1u)) { *abort_flag = 1; break; }
-                if (*abort_flag) break;
-                const int tap = tap_of(kb / g.cpb, g.ctr_tap);
-                const int c0 = (kb % g.cpb) * BK;
-                const int r = tap / g.S, sx = tap % g.S;
+            bool ok = true;
+            for (int kb0 = 0; kb0 < g.n_kb; kb0 += SUB, ++it) {
+                const int s = it % STAGES;
+                const uint32_t ph = (uint32_t)(it / STAGES) & 1u;
+                if (!warp_wait(smem_u32(&empty[s]), ph ^ 1u, a.err, 1u)) { ok = false; break; }
+                const int nsub = min(SUB, g.n_kb - kb0);
                 const uint32_t fb = smem_u32(&full[s]);
-                mbar_expect_tx(fb, A_BYTES + B_TMA_BYTES);
-                tma_load_im2col(smem_u32(As + s * A_BYTES), &amap, fb, c0, w0, h0, nimg, (uint16_t)sx, (uint16_t)r);
-                tma_load_2d(smem_u32(Bs + s * B_BYTES_STAGE), &bmap, fb, tap * g.C + c0, n_tile * BN);
-            }
-        }
-    } else if (warp == 1) {
-        if (lane == 0) {
-            // ---------------- MMA issuer ----------------
-            const uint32_t id_main = idesc_f16(BM, BN);
-            const uint32_t id_merged = idesc_f16(BM, BN + 16);
-            const uint32_t id_ct = idesc_f16(BM, 16);
-            const int n_centre = g.cpb;
-            for (int kb = 0; kb < g.n_kb; ++kb) {
-                const int s = kb % STAGES;
-                const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
-                if (!mbar_wait(smem_u32(&full[s]), ph, a.err, 2u)) { *abort_flag = 1; break; }
-                if (*abort_flag) break;
-                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-                const bool centre = kb < n_centre;
-                const uint32_t a_base = smem_u32(As + s * A_BYTES);
-                const uint32_t b_base = smem_u32(Bs + s * B_BYTES_STAGE);
-#pragma unroll
-                for (int k16 = 0; k16 < BK / 16; ++k16) {
-                    const uint64_t ad = smem_desc_sw128(a_base + k16 * 32);
-                    const uint64_t bd = smem_desc_sw128(b_base + k16 * 32);
-                    const uint32_t acc = (kb > 0 || k16 > 0) ? 1u : 0u;
-                    if (ct_here && centre && g.ct_mode == CT_MERGED) {
-                        umma_f16(tmem, ad, bd, id_merged, acc);
-                    } else {
-                        umma_f16(tmem, ad, bd, id_main, acc);
-                        if (ct_here && centre && g.ct_mode == CT_SEPARATE)
-                            umma_f16(tmem + BN, ad, smem_desc_sw128(smem_u32(CTt) + k16 * 32), id_ct, acc);
+                if (elect_one()) {
+                    mbar_arrive_expect_tx(fb, nsub * (A_BYTES + B_TMA_BYTES));
+                    for (int j = 0; j < nsub; ++j) {
+                        const int kb = kb0 + j;
+                        const int tap = tap_of(kb / g.cpb, g.ctr_tap);
+                        const int c0 = (kb % g.cpb) * BK;
+                        const int r = tap / g.S, sx = tap % g.S;
+                        tma_load_im2col(smem_u32(As + (s * SUB + j) * A_BYTES), &amap, fb, c0, w0, h0, nimg,
+                                        (uint16_t)sx, (uint16_t)r);
+                        tma_load_2d(smem_u32(Bs + (s * SUB + j) * B_SUB_BYTES), &bmap, fb, tap * g.C + c0,
+                                    n_tile * BN);
                     }
                 }
-                umma_commit(smem_u32(&empty[s]));
+                __syncwarp();
             }
-            umma_commit(smem_u32(accum));      // fires when every MMA issued above has completed
+            if (!ok) { if (lane == 0) *abort_flag = 1; break; }
+        }
+    } else if (warp == 1) {
+        // ---------------- MMA issuer (whole warp, one lane issues) ----------------
+        const uint32_t id_main = idesc_f16(BM, BN);
+        const uint32_t id_merged = idesc_f16(BM, BN + 16);
+        const uint32_t id_ct = idesc_f16(BM, 16);
+        const uint32_t ct_base = smem_u32(CTt);
+        int it = 0, lt = 0;
+        for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++lt) {
+            if (__any_sync(0xffffffffu, *abort_flag)) break;
+            const int n_tile = tile % g.n_tiles;
+            const bool ct_here = g.ct_mode != CT_NONE_ && n_tile == 0;
+            if (!warp_wait(smem_u32(acc_empty), ((uint32_t)lt & 1u) ^ 1u, a.err, 8u)) {
+                if (lane == 0) *abort_flag = 1;
+                break;
+            }
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            bool ok = true;
+            for (int kb0 = 0; kb0 < g.n_kb; kb0 += SUB, ++it) {
+                const int s = it % STAGES;
+                const uint32_t ph = (uint32_t)(it / STAGES) & 1u;
+                if (!warp_wait(smem_u32(&full[s]), ph, a.err, 2u)) { ok = false; break; }
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                const int nsub = min(SUB, g.n_kb - kb0);
+                const bool leader = elect_one();
+                for (int j = 0; j < nsub; ++j) {
+                    const int kb = kb0 + j;
+                    const uint32_t d = tmem + (uint32_t)((kb % NCH) * CH);
+                    const bool centre = kb < g.cpb;
+                    const uint32_t a_base = smem_u32(As + (s * SUB + j) * A_BYTES);
+                    const uint32_t b_base = smem_u32(Bs + (s * SUB + j) * B_SUB_BYTES);
+#pragma unroll
+                    for (int k16 = 0; k16 < BK / 16; ++k16) {
+                        const uint64_t ad = smem_desc_sw128(a_base + k16 * 32);
+                        const uint64_t bd = smem_desc_sw128(b_base + k16 * 32);
+                        const uint32_t acc = (kb >= NCH || k16 > 0) ? 1u : 0u;   // first use of the chain
+                        if (leader) {
+                            if (ct_here && centre && g.ct_mode == CT_MERGED) {
+                                umma_f16(d, ad, bd, id_merged, acc);
+                            } else {
+                                umma_f16(d, ad, bd, id_main, acc);
+                                if (ct_here && centre && g.ct_mode == CT_SEPARATE)
+                                    umma_f16(d + BN, ad, smem_desc_sw128(ct_base + k16 * 32), id_ct, acc);
+                            }
+                        }
+                    }
+                }
+                if (leader) umma_commit(smem_u32(&empty[s]));
+                __syncwarp();
+            }
+            if (!ok) { if (lane == 0) *abort_flag = 1; break; }
+            if (elect_one()) umma_commit(smem_u32(acc_full));   // fires when the tile's MMAs have completed
+            __syncwarp();
         }
     } else {
-        // ---------------- epilogue: warps 2..5, one output pixel per thread ----------------
-        const int quad = warp & 3;
+        // ---------------- epilogue: warps 2..9 ----------------
+        const int ep = warp - 2;
+        const int quad = warp & 3;                 // TMEM lanes this warp may read
+        const int half = ep >> 2;                  // which half of the tile's channels
         const int row = quad * 32 + lane;
-        const int m = m0 + row;
-        bool ok = mbar_wait(smem_u32(accum), 0u, a.err, 4u) && !*abort_flag;
-        ok = __all_sync(0xffffffffu, ok);          // tcgen05.ld below is warp-collective
-        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        if (ok) {
+        const __half *x = static_cast<const __half *>(a.x);
+        const FaultDelta fd = a.fd;
+        const int chains = min(NCH, g.n_kb);                       // chains that received MMAs
+        const int ct_chains = min(NCH, g.cpb);                     // chains holding a carry-through column
+        int lt = 0;
+        for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++lt) {
+            const int m0 = (tile / g.n_tiles) * BM, n_tile = tile % g.n_tiles;
+            bool ok = mbar_wait(smem_u32(acc_full), (uint32_t)lt & 1u, a.err, 4u) && !*abort_flag;
+            ok = __all_sync(0xffffffffu, ok);      // tcgen05.ld below is warp-collective
+            if (!ok) break;
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
             const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
+            const int m = m0 + row;
             const bool valid = m < g.M;
             const int mm = valid ? m : 0;
             const int nimg = mm / g.PQ, rem = mm % g.PQ, p = rem / g.Q, q = rem % g.Q;
-            const __half *x = static_cast<const __half *>(a.x);
-            const __half *res = static_cast<const __half *>(a.res);
-            __half *y = static_cast<__half *>(a.y);
-            const FaultDelta fd = a.fd;
             float fsrc = 0.f;
             if (fd.active) {
                 const int h = p * g.stride + fd.r - g.pad, w = q * g.stride + fd.s - g.pad;
@@ -303,63 +452,50 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
                 }
             }
             const int n0 = n_tile * BN;
+            const bool do_cs = half == 0 && a.cs_out != nullptr && n_tile == 0;
+            float ctv = 0.f;
+            if (EARLY) {
+                float vals[BN / 2];
+#pragma unroll
+                for (int c = 0; c < BN / 2; c += 16) {
+                    tmem_ld16(trow + half * (BN / 2) + c, vals + c);
+                    for (int ch = 1; ch < chains; ++ch) {
+                        float t[16];
+                        tmem_ld16(trow + ch * CH + half * (BN / 2) + c, t);
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) vals[c + i] += t[i];
+                    }
+                }
+                if (do_cs && g.ct_mode != CT_NONE_)
+                    for (int ch = 0; ch < ct_chains; ++ch) ctv += tmem_ld1(trow + ch * CH + BN);
+                asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(acc_empty));   // accumulators free for the next tile
+                if (valid) {
+#pragma unroll
+                    for (int c = 0; c < BN / 2; c += 16)
+                        store_chunk(vals + c, a, g.K, (size_t)m, n0 + half * (BN / 2) + c, fsrc);
+                    if (do_cs) store_checksum(ctv, a, g, m, nimg, p, q, fsrc);
+                }
+            } else {
 #pragma unroll 1
-            for (int ch = 0; ch < BN; ch += 16) {
-                float v[16];
-                tmem_ld16(trow + ch, v);
-                if (valid) {
-                    const size_t base = (size_t)m * g.K + n0 + ch;
-                    float rv[16];
-                    if (res) {
-                        const uint4 *rp = reinterpret_cast<const uint4 *>(res + base);
-                        uint4 r0 = rp[0], r1 = rp[1];
-                        const __half2 *h0 = reinterpret_cast<const __half2 *>(&r0);
-                        const __half2 *h1 = reinterpret_cast<const __half2 *>(&r1);
+                for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 16) {
+                    float v[16];
+                    tmem_ld16(trow + c, v);
+                    for (int ch = 1; ch < chains; ++ch) {
+                        float t[16];
+                        tmem_ld16(trow + ch * CH + c, t);
 #pragma unroll
-                        for (int i = 0; i < 4; ++i) {
-                            float2 f0 = __half22float2(h0[i]), f1 = __half22float2(h1[i]);
-                            rv[2 * i] = f0.x; rv[2 * i + 1] = f0.y; rv[8 + 2 * i] = f1.x; rv[8 + 2 * i + 1] = f1.y;
-                        }
+                        for (int i = 0; i < 16; ++i) v[i] += t[i];
                     }
-                    uint32_t packed[8];
-#pragma unroll
-                    for (int i = 0; i < 16; i += 2) {
-                        float o[2];
-#pragma unroll
-                        for (int j = 0; j < 2; ++j) {
-                            const int k = n0 + ch + i + j;
-                            float t = v[i + j] + a.bias[k];
-                            if (fd.active && fd.kout == k) t += fd.dv * fsrc;
-                            if (res) t += rv[i + j];
-                            if (a.relu) t = relu_keep_nan(t);
-                            o[j] = t;
-                        }
-                        __half2 hh = __floats2half2_rn(o[0], o[1]);
-                        packed[i / 2] = *reinterpret_cast<uint32_t *>(&hh);
-                    }
-                    uint4 *yp = reinterpret_cast<uint4 *>(y + base);
-                    yp[0] = make_uint4(packed[0], packed[1], packed[2], packed[3]);
-                    yp[1] = make_uint4(packed[4], packed[5], packed[6], packed[7]);
+                    if (valid) store_chunk(v, a, g.K, (size_t)m, n0 + c, fsrc);
                 }
-            }
-            // checksum output
-            if (a.cs_out != nullptr && n_tile == 0) {
-                float ctv = 0.f;
-                if (g.ct_mode != CT_NONE_) ctv = tmem_ld1(trow + BN);
-                if (valid) {
-                    const __half *csi = static_cast<const __half *>(a.cs_in);
-                    const int ctr_r = g.ctr_tap / g.S, ctr_s = g.ctr_tap % g.S;
-                    const int hc = p * g.stride + ctr_r - g.pad, wc = q * g.stride + ctr_s - g.pad;
-                    const bool inb = hc >= 0 && hc < a.H && wc >= 0 && wc < a.W;
-                    const float cin = (csi && inb) ? ldh(csi, ((size_t)nimg * a.H + hc) * a.W + wc) : 0.f;
-                    float o = 0.f;
-                    if (a.role == CT_ROLE_CT) o = ctv + a.coef * cin;
-                    else if (a.role == CT_ROLE_PASS) o = cin;
-                    if (fd.active && fd.kout == g.K) o += fd.dv * fsrc;
-                    if (a.res_cs) o += ldh(static_cast<const __half *>(a.res_cs), (size_t)m);
-                    if (a.relu) o = relu_keep_nan(o);
-                    static_cast<__half *>(a.cs_out)[m] = __float2half_rn(o);
-                }
+                if (do_cs && g.ct_mode != CT_NONE_)
+                    for (int ch = 0; ch < ct_chains; ++ch) ctv += tmem_ld1(trow + ch * CH + BN);
+                if (do_cs && valid) store_checksum(ctv, a, g, m, nimg, p, q, fsrc);
+                asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(acc_empty));
             }
         }
     }
@@ -381,50 +517,46 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
 // Output channels: 64.  The carry-through row is coef at the centre tap's
 // real channels: 16 constant rows after the 64 weight rows of every B stage,
 // used (N = 80) on the centre tap's K block, which the loop visits first.
+// Persistent, double-buffered accumulators, as above.
 // ---------------------------------------------------------------------------
 constexpr int SM_THREADS = 288;     // warps 0-3 producers, 4 MMA, 5-8 epilogue
-constexpr int SM_STAGES = 6;
+constexpr int SM_STAGES = 8;
 constexpr int SM_BN = 64;
 
 struct TcGeomS {
     int M, PQ, Q, stride, pad, C, H, W, R, S;
     int n_kb, kb_ct, col_ct, ct;
-    int tmem_cols;
+    int tmem_cols, m_tiles;
     uint16_t coef_h;
 };
-
-__device__ __forceinline__ void mbar_expect_tx_only(uint32_t bar, uint32_t bytes) {
-    asm volatile("mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
-}
-
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
 
 __global__ void __launch_bounds__(SM_THREADS, 1)
 conv_tc_small_kernel(const __grid_constant__ CUtensorMap bmap, const ConvArgs a, const TcGeomS g) {
     constexpr int B_ROWS = SM_BN + 16;
     constexpr int B_BYTES_STAGE = B_ROWS * BK * 2;
     constexpr int B_TMA_BYTES = SM_BN * BK * 2;
+    constexpr int NCH = 4;                                // accumulator chains (see conv_tc_kernel)
+    constexpr int CH = SM_BN + 16;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint8_t *As = smem;
     uint8_t *Bs = As + SM_STAGES * A_BYTES;
     uint64_t *full = (uint64_t *)(Bs + SM_STAGES * B_BYTES_STAGE);
     uint64_t *empty = full + SM_STAGES;
-    uint64_t *accum = empty + SM_STAGES;
-    uint32_t *tmem_holder = (uint32_t *)(accum + 1);
+    uint64_t *acc_full = empty + SM_STAGES;
+    uint64_t *acc_empty = acc_full + 1;
+    uint32_t *tmem_holder = (uint32_t *)(acc_empty + 1);
     volatile uint32_t *abort_flag = tmem_holder + 1;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int m0 = blockIdx.x * BM;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < SM_STAGES; ++s) {
             mbar_init(smem_u32(&full[s]), 128);
             mbar_init(smem_u32(&empty[s]), 1);
         }
-        mbar_init(smem_u32(accum), 1);
+        mbar_init(smem_u32(acc_full), 1);
+        mbar_init(smem_u32(acc_empty), 4);
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -455,116 +587,123 @@ conv_tc_small_kernel(const __grid_constant__ CUtensorMap bmap, const ConvArgs a,
     if (warp < 4) {
         // ---------------- software im2col producers ----------------
         const int row = threadIdx.x;
-        const int m = m0 + row;
-        const bool valid = m < g.M;
-        const int mm = valid ? m : 0;
-        const int nimg = mm / g.PQ, rem = mm % g.PQ, p = rem / g.Q, q = rem % g.Q;
-        const int h0 = p * g.stride - g.pad, w0 = q * g.stride - g.pad;
+        if (row == 0) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&bmap) : "memory");
         const int taps = g.R * g.S;
-        for (int it = 0; it < g.n_kb; ++it) {
-            const int kb = (it + g.kb_ct) % g.n_kb;
-            const int s = it % SM_STAGES;
-            const uint32_t ph = (uint32_t)(it / SM_STAGES) & 1u;
-            if (!mbar_wait(smem_u32(&empty[s]), ph ^ 1u, a.err, 1u)) { *abort_flag = 1; break; }
-            if (*abort_flag) break;
-            const uint32_t fb = smem_u32(&full[s]);
-            if (row == 0) {
-                mbar_expect_tx_only(fb, B_TMA_BYTES);
-                tma_load_2d(smem_u32(Bs + s * B_BYTES_STAGE), &bmap, fb, kb * BK, 0);
-            }
-            uint8_t *arow = As + s * A_BYTES + row * 128;
+        int it = 0;
+        for (int tile = blockIdx.x; tile < g.m_tiles && !*abort_flag; tile += gridDim.x) {
+            const int m = tile * BM + row;
+            const bool valid = m < g.M;
+            const int mm = valid ? m : 0;
+            const int nimg = mm / g.PQ, rem = mm % g.PQ, p = rem / g.Q, q = rem % g.Q;
+            const int h0 = p * g.stride - g.pad, w0 = q * g.stride - g.pad;
+            const __half *ximg = x + (size_t)nimg * g.H * g.W * 4;
+            for (int i = 0; i < g.n_kb; ++i, ++it) {
+                const int kb = (i + g.kb_ct) % g.n_kb;
+                // all 16 taps of this K block are fetched before any shared-memory
+                // store, so their global-load latencies overlap
+                uint2 v[16];
+                int r = (kb * 16) / g.S, sx = (kb * 16) % g.S;
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                uint2 v[2];
-#pragma unroll
-                for (int u = 0; u < 2; ++u) {
-                    const int tp = kb * 16 + 2 * j + u;
+                for (int u = 0; u < 16; ++u) {
                     v[u] = make_uint2(0u, 0u);
-                    if (valid && tp < taps) {
-                        const int h = h0 + tp / g.S, w = w0 + tp % g.S;
-                        if (h >= 0 && h < g.H && w >= 0 && w < g.W)
-                            v[u] = *reinterpret_cast<const uint2 *>(x + (((size_t)nimg * g.H + h) * g.W + w) * 4);
-                    }
+                    const int h = h0 + r, w = w0 + sx;
+                    if (valid && kb * 16 + u < taps && h >= 0 && h < g.H && w >= 0 && w < g.W)
+                        v[u] = __ldg(reinterpret_cast<const uint2 *>(ximg + ((size_t)h * g.W + w) * 4));
+                    if (++sx == g.S) { sx = 0; ++r; }
                 }
-                *reinterpret_cast<uint4 *>(arow + ((j ^ (row & 7)) << 4)) = make_uint4(v[0].x, v[0].y, v[1].x, v[1].y);
-            }
-            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-            mbar_arrive(fb);
-        }
-    } else if (warp == 4) {
-        if (lane == 0) {
-            // ---------------- MMA issuer ----------------
-            const uint32_t id_main = idesc_f16(BM, SM_BN);
-            const uint32_t id_merged = idesc_f16(BM, SM_BN + 16);
-            for (int it = 0; it < g.n_kb; ++it) {
                 const int s = it % SM_STAGES;
                 const uint32_t ph = (uint32_t)(it / SM_STAGES) & 1u;
-                if (!mbar_wait(smem_u32(&full[s]), ph, a.err, 2u)) { *abort_flag = 1; break; }
-                if (*abort_flag) break;
+                if (!mbar_wait(smem_u32(&empty[s]), ph ^ 1u, a.err, 1u)) { *abort_flag = 1; break; }
+                const uint32_t fb = smem_u32(&full[s]);
+                if (row == 0) {
+                    mbar_expect_tx_only(fb, B_TMA_BYTES);
+                    tma_load_2d(smem_u32(Bs + s * B_BYTES_STAGE), &bmap, fb, kb * BK, 0);
+                }
+                uint8_t *arow = As + s * A_BYTES + row * 128;
+#pragma unroll
+                for (int j = 0; j < 8; ++j)
+                    *reinterpret_cast<uint4 *>(arow + ((j ^ (row & 7)) << 4)) =
+                        make_uint4(v[2 * j].x, v[2 * j].y, v[2 * j + 1].x, v[2 * j + 1].y);
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                mbar_arrive(fb);
+            }
+        }
+    } else if (warp == 4) {
+        // ---------------- MMA issuer (whole warp, one lane issues) ----------------
+        const uint32_t id_main = idesc_f16(BM, SM_BN);
+        const uint32_t id_merged = idesc_f16(BM, SM_BN + 16);
+        int it = 0, lt = 0;
+        for (int tile = blockIdx.x; tile < g.m_tiles; tile += gridDim.x, ++lt) {
+            if (__any_sync(0xffffffffu, *abort_flag)) break;
+            if (!warp_wait(smem_u32(acc_empty), ((uint32_t)lt & 1u) ^ 1u, a.err, 8u)) {
+                if (lane == 0) *abort_flag = 1;
+                break;
+            }
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            bool ok = true;
+            for (int i = 0; i < g.n_kb; ++i, ++it) {
+                const uint32_t d = tmem + (uint32_t)((i % NCH) * CH);
+                const int s = it % SM_STAGES;
+                const uint32_t ph = (uint32_t)(it / SM_STAGES) & 1u;
+                if (!warp_wait(smem_u32(&full[s]), ph, a.err, 2u)) { ok = false; break; }
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                 const uint32_t a_base = smem_u32(As + s * A_BYTES);
                 const uint32_t b_base = smem_u32(Bs + s * B_BYTES_STAGE);
+                const bool leader = elect_one();
 #pragma unroll
                 for (int k16 = 0; k16 < BK / 16; ++k16) {
                     const uint64_t ad = smem_desc_sw128(a_base + k16 * 32);
                     const uint64_t bd = smem_desc_sw128(b_base + k16 * 32);
-                    const uint32_t acc = (it > 0 || k16 > 0) ? 1u : 0u;
-                    umma_f16(tmem, ad, bd, (it == 0 && g.ct) ? id_merged : id_main, acc);
+                    const uint32_t acc = (i >= NCH || k16 > 0) ? 1u : 0u;   // first use of the chain
+                    if (leader) umma_f16(d, ad, bd, (i == 0 && g.ct) ? id_merged : id_main, acc);
                 }
-                umma_commit(smem_u32(&empty[s]));
+                if (leader) umma_commit(smem_u32(&empty[s]));
+                __syncwarp();
             }
-            umma_commit(smem_u32(accum));
+            if (!ok) { if (lane == 0) *abort_flag = 1; break; }
+            if (elect_one()) umma_commit(smem_u32(acc_full));
+            __syncwarp();
         }
     } else {
         // ---------------- epilogue: warps 5..8 ----------------
         const int quad = warp & 3;
         const int row = quad * 32 + lane;
-        const int m = m0 + row;
-        bool ok = mbar_wait(smem_u32(accum), 0u, a.err, 4u) && !*abort_flag;
-        ok = __all_sync(0xffffffffu, ok);
-        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        if (ok) {
+        const FaultDelta fd = a.fd;
+        const int chains = min(NCH, g.n_kb);
+        int lt = 0;
+        for (int tile = blockIdx.x; tile < g.m_tiles; tile += gridDim.x, ++lt) {
+            bool ok = mbar_wait(smem_u32(acc_full), (uint32_t)lt & 1u, a.err, 4u) && !*abort_flag;
+            ok = __all_sync(0xffffffffu, ok);
+            if (!ok) break;
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
             const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
-            const bool valid = m < g.M;
-            const int mm = valid ? m : 0;
-            const int nimg = mm / g.PQ, rem = mm % g.PQ, p = rem / g.Q, q = rem % g.Q;
-            __half *y = static_cast<__half *>(a.y);
-            const FaultDelta fd = a.fd;
-            float fsrc = 0.f;
-            if (fd.active) {
-                const int h = p * g.stride + fd.r - g.pad, w = q * g.stride + fd.s - g.pad;
-                if (fd.cin < g.C && h >= 0 && h < g.H && w >= 0 && w < g.W)
-                    fsrc = ldh(x, (((size_t)nimg * g.H + h) * g.W + w) * 4 + fd.cin);
-            }
-#pragma unroll 1
-            for (int ch = 0; ch < SM_BN; ch += 16) {
-                float v[16];
-                tmem_ld16(trow + ch, v);
-                if (valid) {
-                    uint32_t packed[8];
+            float vals[SM_BN];
 #pragma unroll
-                    for (int i = 0; i < 16; i += 2) {
-                        float o[2];
+            for (int c = 0; c < SM_BN; c += 16) {
+                tmem_ld16(trow + c, vals + c);
+                for (int ch = 1; ch < chains; ++ch) {
+                    float t[16];
+                    tmem_ld16(trow + ch * CH + c, t);
 #pragma unroll
-                        for (int j = 0; j < 2; ++j) {
-                            const int k = ch + i + j;
-                            float t = v[i + j] + a.bias[k];
-                            if (fd.active && fd.kout == k) t += fd.dv * fsrc;
-                            if (a.relu) t = relu_keep_nan(t);
-                            o[j] = t;
-                        }
-                        __half2 hh = __floats2half2_rn(o[0], o[1]);
-                        packed[i / 2] = *reinterpret_cast<uint32_t *>(&hh);
-                    }
-                    uint4 *yp = reinterpret_cast<uint4 *>(y + (size_t)m * SM_BN + ch);
-                    yp[0] = make_uint4(packed[0], packed[1], packed[2], packed[3]);
-                    yp[1] = make_uint4(packed[4], packed[5], packed[6], packed[7]);
+                    for (int i = 0; i < 16; ++i) vals[c + i] += t[i];
                 }
             }
-            if (a.cs_out != nullptr) {
-                float ctv = 0.f;
-                if (g.ct) ctv = tmem_ld1(trow + SM_BN);
-                if (valid) {
+            const float ctv = (a.cs_out != nullptr && g.ct) ? tmem_ld1(trow + SM_BN) : 0.f;   // chain 0 only
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(acc_empty));
+            const int m = tile * BM + row;
+            if (m < g.M) {
+                const int nimg = m / g.PQ, rem = m % g.PQ, p = rem / g.Q, q = rem % g.Q;
+                float fsrc = 0.f;
+                if (fd.active) {
+                    const int h = p * g.stride + fd.r - g.pad, w = q * g.stride + fd.s - g.pad;
+                    if (fd.cin < g.C && h >= 0 && h < g.H && w >= 0 && w < g.W)
+                        fsrc = ldh(x, (((size_t)nimg * g.H + h) * g.W + w) * 4 + fd.cin);
+                }
+#pragma unroll
+                for (int c = 0; c < SM_BN; c += 16) store_chunk(vals + c, a, SM_BN, (size_t)m, c, fsrc);
+                if (a.cs_out != nullptr) {
                     float o = (a.role == CT_ROLE_CT) ? ctv : 0.f;
                     if (fd.active && fd.kout == SM_BN) o += fd.dv * fsrc;
                     if (a.relu) o = relu_keep_nan(o);
@@ -604,9 +743,9 @@ bool load_encoders() {
     return g_encode_tiled && g_encode_im2col;
 }
 
-template <int BN, int STAGES>
+template <int BN, int STAGES, int SUB>
 size_t smem_bytes() {
-    return 1024 + (size_t)STAGES * (A_BYTES + (BN + 16) * BK * 2) + 16 * BK * 2 + 8 * (2 * STAGES + 1) + 16;
+    return 1024 + (size_t)STAGES * SUB * (A_BYTES + (BN + 16) * BK * 2) + 16 * BK * 2 + 8 * (2 * STAGES + 2) + 16;
 }
 
 uint16_t coef_half_bits(float c) {
@@ -616,13 +755,21 @@ uint16_t coef_half_bits(float c) {
     return b;
 }
 
+int sm_count() {
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1)
+        return 148;
+    return n;
+}
+
 }  // namespace
 
 struct TcPlan {
     CUtensorMap amap;
     CUtensorMap bmap;
     TcGeom g;
-    int BN, stages, n_tiles;
+    int BN, n_tiles, sms;
     size_t smem;
 };
 
@@ -642,7 +789,7 @@ TcPlan *tc_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, cons
     memset(pl, 0, sizeof(*pl));
     pl->BN = a.K <= 256 ? a.K : 256;
     pl->n_tiles = a.K / pl->BN;
-    pl->stages = pl->BN == 128 ? 3 : 4;
+    pl->sms = sm_count();
     TcGeom &g = pl->g;
     g.PQ = a.P * a.Q; g.Q = a.Q; g.stride = a.stride; g.pad = a.pad; g.C = a.C; g.K = a.K;
     g.RSC = a.R * a.S * a.C; g.S = a.S;
@@ -650,8 +797,8 @@ TcPlan *tc_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, cons
     g.n_kb = a.R * a.S * g.cpb;
     g.ctr_tap = ((a.R - 1) / 2) * a.S + (a.S - 1) / 2;
     g.ct_mode = a.role != CT_ROLE_CT ? CT_NONE_ : (pl->BN + 16 <= 256 && pl->n_tiles == 1 ? CT_MERGED : CT_SEPARATE);
-    const int cols = pl->BN + (g.ct_mode != CT_NONE_ ? 16 : 0);
-    g.tmem_cols = cols <= 32 ? 32 : cols <= 64 ? 64 : cols <= 128 ? 128 : cols <= 256 ? 256 : 512;
+    g.tmem_cols = 512;
+    g.n_tiles = pl->n_tiles;
     g.coef_h = coef_half_bits(a.coef);
     // A: im2col view of the NHWC input [max_batch, H, W, C]
     cuuint64_t gdim[4] = {(cuuint64_t)a.C, (cuuint64_t)a.W, (cuuint64_t)a.H, (cuuint64_t)max_batch};
@@ -675,17 +822,30 @@ TcPlan *tc_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, cons
     if (r != CUDA_SUCCESS) { if (why) *why = "weight tensor map"; delete pl; return nullptr; }
     cudaError_t e;
     if (pl->BN == 64) {
-        pl->smem = smem_bytes<64, 4>();
-        e = cudaFuncSetAttribute(conv_tc_kernel<64, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
+        pl->smem = smem_bytes<64, 4, 2>();
+        e = cudaFuncSetAttribute(conv_tc_kernel<64, 4, 2, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
     } else if (pl->BN == 128) {
-        pl->smem = smem_bytes<128, 3>();
-        e = cudaFuncSetAttribute(conv_tc_kernel<128, 3>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
+        pl->smem = smem_bytes<128, 3, 2>();
+        e = cudaFuncSetAttribute(conv_tc_kernel<128, 3, 2, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
     } else {
-        pl->smem = smem_bytes<256, 4>();
-        e = cudaFuncSetAttribute(conv_tc_kernel<256, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
+        pl->smem = smem_bytes<256, 4, 1>();
+        e = cudaFuncSetAttribute(conv_tc_kernel<256, 4, 1, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
     }
     if (e != cudaSuccess) { if (why) *why = "shared memory attribute"; delete pl; return nullptr; }
     return pl;
+}
+
+cudaError_t launch_conv_tc(const ConvArgs &a, const void *plan, cudaStream_t st) {
+    const TcPlan *pl = static_cast<const TcPlan *>(plan);
+    TcGeom g = pl->g;
+    g.M = a.N * a.P * a.Q;
+    g.m_tiles = (g.M + BM - 1) / BM;
+    const int tiles = g.m_tiles * g.n_tiles;
+    dim3 grid(tiles < pl->sms ? tiles : pl->sms);
+    if (pl->BN == 64) conv_tc_kernel<64, 4, 2, 4><<<grid, NTHREADS, pl->smem, st>>>(pl->amap, pl->bmap, a, g);
+    else if (pl->BN == 128) conv_tc_kernel<128, 3, 2, 2><<<grid, NTHREADS, pl->smem, st>>>(pl->amap, pl->bmap, a, g);
+    else conv_tc_kernel<256, 4, 1, 1><<<grid, NTHREADS, pl->smem, st>>>(pl->amap, pl->bmap, a, g);
+    return cudaGetLastError();
 }
 
 bool tc_small_supported(int C, int K, int R, int S, int stride, int pad) {
@@ -697,6 +857,7 @@ int tc_small_kpad(int R, int S) { return ((R * S * 4 + BK - 1) / BK) * BK; }
 struct TcSmallPlan {
     CUtensorMap bmap;
     TcGeomS g;
+    int sms;
     size_t smem;
 };
 
@@ -704,6 +865,7 @@ TcSmallPlan *tc_small_plan_create(const ConvArgs &a, const void *w_dev, std::str
     if (!load_encoders()) { if (why) *why = "tensor-map encoders unavailable"; return nullptr; }
     TcSmallPlan *pl = new TcSmallPlan();
     memset(pl, 0, sizeof(*pl));
+    pl->sms = sm_count();
     TcGeomS &g = pl->g;
     g.PQ = a.P * a.Q; g.Q = a.Q; g.stride = a.stride; g.pad = a.pad; g.C = a.C;
     g.H = a.H; g.W = a.W; g.R = a.R; g.S = a.S;
@@ -713,7 +875,7 @@ TcSmallPlan *tc_small_plan_create(const ConvArgs &a, const void *w_dev, std::str
     g.kb_ct = (ctr_tap * 4) / BK;
     g.col_ct = (ctr_tap * 4) % BK;
     g.ct = a.role == CT_ROLE_CT ? 1 : 0;
-    g.tmem_cols = 128;
+    g.tmem_cols = 512;
     g.coef_h = coef_half_bits(a.coef);
     cuuint64_t bdim[2] = {(cuuint64_t)kp, (cuuint64_t)SM_BN};
     cuuint64_t bstr[1] = {(cuuint64_t)kp * 2};
@@ -723,7 +885,7 @@ TcSmallPlan *tc_small_plan_create(const ConvArgs &a, const void *w_dev, std::str
                                 box, bes, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                                 CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) { if (why) *why = "weight tensor map"; delete pl; return nullptr; }
-    pl->smem = 1024 + (size_t)SM_STAGES * (A_BYTES + (SM_BN + 16) * BK * 2) + 8 * (2 * SM_STAGES + 1) + 16;
+    pl->smem = 1024 + (size_t)SM_STAGES * (A_BYTES + (SM_BN + 16) * BK * 2) + 8 * (2 * SM_STAGES + 2) + 16;
     if (cudaFuncSetAttribute(conv_tc_small_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem) !=
         cudaSuccess) {
         if (why) *why = "shared memory attribute";
@@ -738,22 +900,12 @@ void tc_small_plan_destroy(TcSmallPlan *p) { delete p; }
 cudaError_t launch_conv_tc_small(const ConvArgs &a, const TcSmallPlan *pl, cudaStream_t st) {
     TcGeomS g = pl->g;
     g.M = a.N * a.P * a.Q;
-    dim3 grid((g.M + BM - 1) / BM);
+    g.m_tiles = (g.M + BM - 1) / BM;
+    dim3 grid(g.m_tiles < pl->sms ? g.m_tiles : pl->sms);
     conv_tc_small_kernel<<<grid, SM_THREADS, pl->smem, st>>>(pl->bmap, a, g);
     return cudaGetLastError();
 }
 
 void tc_plan_destroy(TcPlan *p) { delete p; }
-
-cudaError_t launch_conv_tc(const ConvArgs &a, const void *plan, cudaStream_t st) {
-    const TcPlan *pl = static_cast<const TcPlan *>(plan);
-    TcGeom g = pl->g;
-    g.M = a.N * a.P * a.Q;
-    dim3 grid((g.M + BM - 1) / BM, pl->n_tiles);
-    if (pl->BN == 64) conv_tc_kernel<64, 4><<<grid, NTHREADS, pl->smem, st>>>(pl->amap, pl->bmap, a, g);
-    else if (pl->BN == 128) conv_tc_kernel<128, 3><<<grid, NTHREADS, pl->smem, st>>>(pl->amap, pl->bmap, a, g);
-    else conv_tc_kernel<256, 4><<<grid, NTHREADS, pl->smem, st>>>(pl->amap, pl->bmap, a, g);
-    return cudaGetLastError();
-}
 
 }  // namespace ct

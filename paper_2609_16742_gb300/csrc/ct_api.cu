@@ -97,6 +97,7 @@ struct LayerRT {
     // fc
     int n_in = 0, n_cs = 0, n_out = 0;
     bool x_float = false;
+    bool fc_tc = false;          // hidden FC run on the tensor-core conv kernel as a 1x1 conv
 };
 
 struct EvRec { int fam; int ev; double flops; };
@@ -328,6 +329,9 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
             if (d.final) { ++n_final; if (d.cout != desc->n_classes || i != nL - 1) return CT_EINVAL; }
             dst.C = l.n_out; dst.H = dst.W = 1;
             dst.has_cs = m->protect && !d.final;
+            std::string why;
+            l.fc_tc = prec == CT_FP16 && !(m->flags & CT_FLAG_SIMT_ONLY) && !d.final && !src.is_float &&
+                      tc_supported(l.n_in, l.n_out, 1, 1, 1, 0, &why);
             // weights: columns permuted from (c, h, w) to the NHWC flatten (h, w, c)
             std::vector<uint8_t> hw((size_t)l.n_out * l.n_in * esz);
             std::vector<float> hb(l.n_out, 0.f);
@@ -372,6 +376,16 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
             std::string why;
             l.splan = tc_small_plan_create(a, l.w, &why);
             if (!l.splan) return CT_ECUDA;
+            continue;
+        }
+        if (l.fc_tc) {
+            ConvArgs a{};
+            a.N = B; a.H = a.W = 1; a.C = l.n_in; a.K = l.n_out; a.R = a.S = 1;
+            a.stride = 1; a.pad = 0; a.P = a.Q = 1;
+            a.role = m->protect ? CT_ROLE_CT : CT_ROLE_NONE; a.coef = l.coef;
+            std::string why;
+            l.plan = tc_plan_create(a, B, l.w, m->slots[l.d.src].data, &why);
+            if (!l.plan) return CT_ECUDA;
             continue;
         }
         if (!l.tc) continue;
@@ -514,6 +528,19 @@ ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, 
             a.k = d.k; a.stride = d.stride; a.pad = d.pad;
             if (d.op == CT_OP_MAXPOOL) CUDA_TRY(launch(m, FAM_POOL, 0, st, [&] { return launch_maxpool(a, half, st); }));
             else CUDA_TRY(launch(m, FAM_POOL, 0, st, [&] { return launch_gap(a, half, st); }));
+        } else if (l.fc_tc) {
+            // hidden FC as a 1x1 convolution over [batch, 1, 1, n_in]: the carry-through
+            // neuron is the kernel's carry-through column plus the sum of the incoming
+            // checksum features
+            ConvArgs a{};
+            a.x = src.data; a.cs_in = src.has_cs ? src.cs : nullptr; a.w = l.w; a.bias = l.bias;
+            a.y = dst.data; a.cs_out = dst.has_cs ? dst.cs : nullptr;
+            a.N = batch; a.H = a.W = 1; a.C = l.n_in; a.K = l.n_out; a.R = a.S = 1;
+            a.stride = 1; a.pad = 0; a.P = a.Q = 1;
+            a.role = m->protect ? CT_ROLE_CT : CT_ROLE_NONE; a.relu = d.relu; a.coef = l.coef;
+            a.err = m->d_err; a.cs_rowsum = l.n_cs;
+            const double flops = 2.0 * batch * (double)l.n_in * l.n_out;
+            CUDA_TRY(launch(m, FAM_FC, flops, st, [&] { return launch_conv_tc(a, l.plan, st); }));
         } else {
             FcArgs a{};
             a.x = src.data; a.xcs = src.has_cs ? src.cs : nullptr; a.w = l.w; a.bias = l.bias;

@@ -38,6 +38,8 @@ struct ConvArgs {
     float coef;           // carry-through coefficient 2^-ct_shift
     FaultDelta fd;
     uint32_t *err;        // device error word
+    int cs_rowsum;        // > 0: an FC layer run as a 1x1 convolution; its checksum input
+                          // is the sum of cs_in[m * cs_rowsum .. m * cs_rowsum + cs_rowsum)
 };
 
 struct FcArgs {
