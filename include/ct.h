@@ -115,6 +115,10 @@ typedef struct ct_model ct_model;
  * (its zero slice is structural); adds one all-ones neuron to every hidden
  * FC layer and the accumulated-checksum neuron to the final one; rounds to
  * the storage precision; converts to the device layouts and uploads.
+ * With FP16 storage, a first 7x7 stride-2 convolution on an image of at most
+ * 4 channels with 64 filters, followed by a 3x3 stride-2 padding-1 max-pool
+ * that is its only reader, runs as one fused kernel: the FP16 copy of the
+ * image and the unpooled convolution output are then never stored.
  * Synchronous.  On success *out owns device memory until ct_destroy.
  * Errors: CT_EINVAL (malformed description), CT_EUNSUPPORTED, CT_ENOMEM,
  * CT_ECUDA.  Nothing is allocated on failure. */
@@ -151,8 +155,9 @@ ct_status ct_infer(ct_model *m, const float *input_dev, int32_t batch, float *lo
  *     the batch of the next ct_infer.
  * `bit` is in [0, 32) for FP32 and [0, 16) for FP16 storage.
  * Errors: CT_EINVAL (not a conv layer, bad kind), CT_ERANGE (element or bit
- * out of range; an activation element is range-checked again by ct_infer
- * against its batch). */
+ * out of range, or an activation tensor that is not stored: the image of a
+ * model with a fused stem; an activation element is range-checked again by
+ * ct_infer against its batch). */
 ct_status ct_inject(ct_model *m, int32_t kind, int32_t layer, int64_t element, int32_t bit);
 ct_status ct_clear_faults(ct_model *m);
 
@@ -243,7 +248,9 @@ ct_status ct_launches_per_infer(const ct_model *m, int32_t *n);
  * and *C reports 4.
  * *C, *H, *W, *has_cs and *elem_bytes describe the slot (any may be NULL; call
  * first with data_host = NULL to query).  Synchronous.  CT_ERANGE for a slot
- * that is not stored (the classifier output) or batch > max_batch. */
+ * that is not kept (the classifier output) or batch > max_batch; CT_ESTATE
+ * for a tensor that a fused kernel computes without storing (slot 0 and the
+ * unpooled stem output of a model with a fused stem). */
 ct_status ct_copy_activation(ct_model *m, int32_t slot, int32_t batch, void *data_host, void *cs_host,
                              int32_t *C, int32_t *H, int32_t *W, int32_t *has_cs,
                              int32_t *elem_bytes, void *stream);

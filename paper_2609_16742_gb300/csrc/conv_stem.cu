@@ -1,0 +1,510 @@
+// Fused image stem: input conversion, 7x7 stride-2 convolution with the
+// carry-through filter on the tensor cores (tcgen05, FP32 accumulation in
+// TMEM), bias, ReLU, and the 3x3 stride-2 max-pool that follows it, in one
+// persistent kernel.  Only the pooled tensor and its checksum plane reach
+// HBM; the unpooled convolution output and the FP16 copy of the image are
+// never stored.  Rounding to FP16 before the max-pool and after it give the
+// same result (rounding is monotone), so this equals conv -> store -> pool.
+//
+// GEMM view of one convolution output row (n, p): M = 128 output columns q
+// (Q <= 128; rows q >= Q are computed and dropped), N = 64 filters plus the
+// carry-through row, K = 7 filter rows x 2 steps x 16.  Step 0 of filter row
+// r covers taps s = 0..3 and step 1 taps s = 3..6 (the weight of tap 3 is 0
+// in step 1), each tap with 4 channels (the image's C <= 4 channels, then
+// zeros).
+//
+// No im2col tile is built.  The producer warps convert input rows from FP32
+// NCHW to FP16 pixels of 4 channels (8 bytes) in a ring of shared-memory
+// rows.  With stride 2, output column q reads input pixels 2q + s - 3, so in
+// such a row the A operand of one step is a strided view: A row q starts
+// 16 bytes after row q - 1 and each 8-element K chunk (2 taps) 16 bytes after
+// the previous one.  That is a no-swizzle K-major UMMA descriptor with row
+// pitch 16, LBO = 16 and SBO = 128 over overlapping rows.  Step 0 reads copy
+// E of the row (pixel x at byte 8 (x + 3)), step 1 reads copy O (pixel x at
+// byte 8 (x + 4)), so that both start on a 16-byte boundary.
+//
+// Work unit: one pooled output row (n, i), which takes convolution rows
+// 2i - 1, 2i, 2i + 1.  Each CTA owns a contiguous range of units and computes
+// their convolution rows in order, so a row shared by two units is computed
+// once (plus one row at the start of each CTA's range in an image).  The
+// epilogue keeps the column-pooled row of the previous odd convolution row
+// in registers and writes each pooled row when its last convolution row is
+// done.
+//
+// Warp roles (416 threads): warps 0-3 fill ring rows (entry e goes to warp
+// e % 4), warp 4 allocates TMEM and issues tcgen05.mma (one elected lane),
+// warps 5-12 are the epilogue: each TMEM lane quadrant is read by two warps,
+// each taking 32 of the 64 channels.  Two TMEM accumulators alternate
+// between consecutive convolution rows.  Every mbarrier wait is bounded; on
+// expiry the kernel records an error code, stops and frees TMEM.
+#include "ct_internal.h"
+#include "tc_common.cuh"
+
+namespace ct {
+
+namespace {
+
+using namespace tc;
+
+constexpr int ST_K = 64;                     // filters
+constexpr int ST_NB = ST_K + 16;             // B rows: filters, carry-through row, 15 zero rows
+constexpr int ST_R = 7;                      // filter rows and columns
+constexpr int ST_KSTEPS = 2 * ST_R;          // K16 steps
+constexpr int ST_KLEN = 16 * ST_KSTEPS;      // 224: weight row length
+constexpr int ST_RP = 264;                   // ring row pitch in pixels (8 bytes each)
+constexpr int ST_ROW_BYTES = ST_RP * 8;      // one copy of one input row
+constexpr int ST_SLOT_BYTES = 2 * ST_ROW_BYTES;
+constexpr int ST_NSLOT = 16;                 // ring rows
+constexpr int ST_B_STEP = ST_NB * 32;        // B bytes per K16 step (two core-matrix columns)
+constexpr int ST_B_LBO = ST_NB * 16;         // between the two K chunks of a step
+constexpr int ST_PIX_H = 72;                 // halves per pixel in the epilogue row buffer (144 B)
+constexpr int ST_THREADS = 416;
+constexpr int ST_EPI0 = 160;                 // first epilogue thread
+constexpr int ST_EPI = 256;                  // epilogue threads
+constexpr int ST_TMEM_COLS = 256;            // two accumulators of 128 columns
+
+constexpr size_t ST_OFF_B = (size_t)ST_NSLOT * ST_SLOT_BYTES;
+constexpr size_t ST_OFF_ROW = ST_OFF_B + (size_t)ST_KSTEPS * ST_B_STEP;
+constexpr size_t ST_OFF_CS = ST_OFF_ROW + 2ull * 128 * ST_PIX_H * 2;
+constexpr size_t ST_OFF_BAR = ST_OFF_CS + 2ull * 128 * 2;
+constexpr size_t ST_SMEM = 1024 + ST_OFF_BAR + 8 * (2 * ST_NSLOT + 5) + 16;
+
+struct StemGeom {
+    int N, C, H, W, P, Q, P2, Q2;
+    int ct;              // carry-through column computed
+    uint16_t coef_h;
+};
+
+// Walks the convolution rows of one CTA's unit range [u, u_end) in order.
+struct StemJobs {
+    int u, u_end;
+    int n, p, p_end;
+    bool seg_start;      // first row of a run within one image
+
+    __device__ bool start_seg(const StemGeom &g) {
+        if (u >= u_end) return false;
+        n = u / g.P2;
+        const int ia = u % g.P2;
+        const int ib = min(g.P2 - 1, u_end - 1 - n * g.P2);
+        p = ia == 0 ? 0 : 2 * ia - 1;
+        p_end = min(2 * ib + 1, g.P - 1);
+        u = (n + 1) * g.P2;
+        seg_start = true;
+        return true;
+    }
+    __device__ bool first(int u0, int u1, const StemGeom &g) {
+        u = u0;
+        u_end = u1;
+        return start_seg(g);
+    }
+    __device__ bool next(const StemGeom &g) {
+        if (p < p_end) {
+            ++p;
+            seg_start = false;
+            return true;
+        }
+        return start_seg(g);
+    }
+};
+
+// barrier among the epilogue warps that also ORs one predicate over them
+__device__ __forceinline__ bool epi_bar_or(bool pred) {
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\t"
+        "setp.ne.u32 p, %1, 0;\n\t"
+        "barrier.red.or.pred q, 1, %2, p;\n\t"
+        "selp.u32 %0, 1, 0, q;\n\t}"
+        : "=r"(r)
+        : "r"((uint32_t)pred), "n"(ST_EPI)
+        : "memory");
+    return r != 0;
+}
+
+__device__ __forceinline__ uint32_t hmax2u(uint32_t a, uint32_t b) {
+    __half2 r = __hmax2_nan(*reinterpret_cast<__half2 *>(&a), *reinterpret_cast<__half2 *>(&b));
+    return *reinterpret_cast<uint32_t *>(&r);
+}
+
+__device__ __forceinline__ float image_half(const float *x, const StemGeom &g, int n, int c, int h, int w) {
+    if (c >= g.C || h < 0 || h >= g.H || w < 0 || w >= g.W) return 0.f;
+    return __half2float(__float2half_rn(x[(((size_t)n * g.C + c) * g.H + h) * g.W + w]));
+}
+
+__global__ void __launch_bounds__(ST_THREADS, 1)
+stem_pool_kernel(const ConvArgs a, const StemGeom g) {
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint8_t *ring = smem;
+    uint8_t *Bs = smem + ST_OFF_B;
+    __half *rowbuf = (__half *)(smem + ST_OFF_ROW);
+    __half *csbuf = (__half *)(smem + ST_OFF_CS);
+    uint64_t *full = (uint64_t *)(smem + ST_OFF_BAR);
+    uint64_t *empty = full + ST_NSLOT;
+    uint64_t *acc_full = empty + ST_NSLOT;
+    uint64_t *acc_empty = acc_full + 2;
+    uint64_t *mma_done = acc_empty + 2;
+    uint32_t *tmem_holder = (uint32_t *)(mma_done + 1);
+    volatile uint32_t *abort_flag = tmem_holder + 1;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const float *x = static_cast<const float *>(a.x);
+    const int units = g.N * g.P2;
+    const int u0 = (int)((long long)blockIdx.x * units / gridDim.x);
+    const int u1 = (int)((long long)(blockIdx.x + 1) * units / gridDim.x);
+
+    // ---- set-up: zero the ring (its padding columns stay zero), weights to
+    // the canonical no-swizzle layout, the carry-through row ----
+    for (int i = threadIdx.x; i < (int)(ST_OFF_B / 16); i += ST_THREADS)
+        reinterpret_cast<uint4 *>(ring)[i] = make_uint4(0u, 0u, 0u, 0u);
+    {
+        const __half *w = static_cast<const __half *>(a.w);
+        const __half coef = __ushort_as_half(g.coef_h);
+        const __half zero = __ushort_as_half((unsigned short)0);
+        for (int i = threadIdx.x; i < ST_NB * (ST_KLEN / 8); i += ST_THREADS) {
+            const int nrow = i / (ST_KLEN / 8), k8 = i % (ST_KLEN / 8);
+            uint4 v = make_uint4(0u, 0u, 0u, 0u);
+            if (nrow < ST_K) {
+                v = *reinterpret_cast<const uint4 *>(w + (size_t)nrow * ST_KLEN + k8 * 8);
+            } else if (nrow == ST_K && g.ct) {
+                // centre tap (r = 3, s = 3) lies in step 0 of filter row 3:
+                // K index 3 * 32 + 3 * 4 + c
+                __half h[8];
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    const int k = k8 * 8 + e;
+                    h[e] = (k >= 108 && k < 108 + g.C) ? coef : zero;
+                }
+                v = *reinterpret_cast<uint4 *>(h);
+            }
+            const int t = k8 / 2, kc = k8 % 2;
+            *reinterpret_cast<uint4 *>(Bs + t * ST_B_STEP + kc * ST_B_LBO + (nrow / 8) * 128 + (nrow % 8) * 16) = v;
+        }
+    }
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < ST_NSLOT; ++s) {
+            mbar_init(smem_u32(&full[s]), 32);
+            mbar_init(smem_u32(&empty[s]), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(smem_u32(&acc_full[b]), 1);
+            mbar_init(smem_u32(&acc_empty[b]), ST_EPI / 32);
+        }
+        mbar_init(smem_u32(mma_done), 1);
+        *abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 4) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_holder)),
+                     "r"((uint32_t)ST_TMEM_COLS));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tmem = *tmem_holder;
+
+    if (warp < 4) {
+        // ---------------- ring producers ----------------
+        StemJobs jb;
+        bool have = jb.first(u0, u1, g);
+        int ecount = 0;
+        while (have) {
+            if (__any_sync(0xffffffffu, *abort_flag)) break;
+            const int n_new = jb.seg_start ? 7 : 2;
+            const int y0 = jb.seg_start ? 2 * jb.p - 3 : 2 * jb.p + 2;
+            bool ok = true;
+            for (int t = 0; t < n_new; ++t) {
+                const int e = ecount + t;
+                if ((e & 3) != warp) continue;
+                const int slot = e % ST_NSLOT;
+                const uint32_t ph = (uint32_t)(e / ST_NSLOT) & 1u;
+                if (!warp_wait(smem_u32(&empty[slot]), ph ^ 1u, a.err, 1u)) { ok = false; break; }
+                const int y = y0 + t;
+                const bool row_ok = y >= 0 && y < g.H;
+                float v[8][4];
+#pragma unroll
+                for (int it = 0; it < 8; ++it) {
+                    const int col = lane + 32 * it;
+#pragma unroll
+                    for (int c = 0; c < 4; ++c) {
+                        v[it][c] = 0.f;
+                        if (row_ok && col < g.W && c < g.C)
+                            v[it][c] = __ldg(x + (((size_t)jb.n * g.C + c) * g.H + y) * g.W + col);
+                    }
+                }
+                uint8_t *E = ring + slot * ST_SLOT_BYTES;
+                uint8_t *O = E + ST_ROW_BYTES;
+#pragma unroll
+                for (int it = 0; it < 8; ++it) {
+                    const int col = lane + 32 * it;
+                    if (col < g.W) {
+                        __half2 lo = __floats2half2_rn(v[it][0], v[it][1]);
+                        __half2 hi = __floats2half2_rn(v[it][2], v[it][3]);
+                        const uint2 pk = make_uint2(*reinterpret_cast<uint32_t *>(&lo), *reinterpret_cast<uint32_t *>(&hi));
+                        *reinterpret_cast<uint2 *>(E + (col + 3) * 8) = pk;
+                        *reinterpret_cast<uint2 *>(O + (col + 4) * 8) = pk;
+                    }
+                }
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                mbar_arrive(smem_u32(&full[slot]));
+            }
+            if (!ok) { if (lane == 0) *abort_flag = 1; break; }
+            ecount += n_new;
+            have = jb.next(g);
+        }
+    } else if (warp == 4) {
+        // ---------------- MMA issuer (whole warp, one lane issues) ----------------
+        const uint32_t id64 = idesc_f16(128, ST_K);
+        const uint32_t id80 = idesc_f16(128, ST_NB);
+        const uint32_t ring_base = smem_u32(ring), b_base = smem_u32(Bs);
+        StemJobs jb;
+        bool have = jb.first(u0, u1, g);
+        int ecount = 0, j = 0;
+        bool issued = false;
+        while (have) {
+            if (__any_sync(0xffffffffu, *abort_flag)) break;
+            const int wstart = jb.seg_start ? ecount : ecount - 5;
+            ecount += jb.seg_start ? 7 : 2;
+            StemJobs nx = jb;
+            const bool have_next = nx.next(g);
+            const int nrel = (have_next && !nx.seg_start) ? 2 : 7;
+            const int ab = j & 1;
+            const uint32_t use = (uint32_t)(j >> 1) & 1u;
+            bool ok = warp_wait(smem_u32(&acc_empty[ab]), use ^ 1u, a.err, 8u);
+            for (int r = 0; r < ST_R && ok; ++r) {
+                const int e = wstart + r;
+                ok = warp_wait(smem_u32(&full[e % ST_NSLOT]), (uint32_t)(e / ST_NSLOT) & 1u, a.err, 2u);
+            }
+            if (!ok) { if (lane == 0) *abort_flag = 1; break; }
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            if (elect_one()) {
+                const uint32_t d = tmem + (uint32_t)(ab * 128);
+#pragma unroll
+                for (int i = 0; i < ST_R; ++i) {
+                    const int r = i == 0 ? 3 : (i <= 3 ? i - 1 : i);    // centre row first
+                    const uint32_t row = ring_base + (uint32_t)(((wstart + r) % ST_NSLOT) * ST_SLOT_BYTES);
+                    const uint64_t a0 = smem_desc_noswz(row, 16, 128);
+                    const uint64_t a1 = smem_desc_noswz(row + ST_ROW_BYTES + 32, 16, 128);
+                    const uint64_t b0 = smem_desc_noswz(b_base + (2 * r) * ST_B_STEP, ST_B_LBO, 128);
+                    const uint64_t b1 = smem_desc_noswz(b_base + (2 * r + 1) * ST_B_STEP, ST_B_LBO, 128);
+                    // the first MMA (centre row) writes all 80 columns when the
+                    // carry-through row is present
+                    umma_f16(d, a0, b0, (i == 0 && g.ct) ? id80 : id64, i > 0 ? 1u : 0u);
+                    umma_f16(d, a1, b1, id64, 1u);
+                }
+                umma_commit(smem_u32(&acc_full[ab]));
+                for (int t = 0; t < nrel; ++t) umma_commit(smem_u32(&empty[(wstart + t) % ST_NSLOT]));
+            }
+            __syncwarp();
+            issued = true;
+            jb = nx;
+            have = have_next;
+            ++j;
+        }
+        // every issued MMA has completed before TMEM can be freed
+        if (issued) {
+            if (elect_one()) umma_commit(smem_u32(mma_done));
+            __syncwarp();
+            warp_wait(smem_u32(mma_done), 0u, a.err, 16u);
+        }
+    } else {
+        // ---------------- epilogue: warps 5..12 ----------------
+        const int et = threadIdx.x - ST_EPI0;
+        const int quad = warp & 3;
+        const int half_id = (warp - 5) >> 2;            // channels 32 * half_id ..
+        const int q = quad * 32 + lane;                 // output column of this thread
+        const int k0 = 32 * half_id;
+        const FaultDelta fd = a.fd;
+        float bias[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) bias[i] = __ldg(a.bias + k0 + i);
+        const bool has_cs = a.cs_out != nullptr;
+        // pooling role: column jj, channels 16 * cq .. 16 * cq + 15
+        const int jj = et >> 2, cq = et & 3;
+        const bool pool_data = jj < g.Q2;
+        const bool pool_cs = has_cs && et < g.Q2;
+        uint32_t accv[8], carry[8];
+        __half acc_cs = __ushort_as_half((unsigned short)0xFC00), carry_cs = acc_cs;
+        bool acc_valid = false, has_carry = false;
+        StemJobs jb;
+        bool have = jb.first(u0, u1, g);
+        int j = 0;
+        while (have) {
+            const int ab = j & 1;
+            const uint32_t use = (uint32_t)(j >> 1) & 1u;
+            bool ok = mbar_wait(smem_u32(&acc_full[ab]), use, a.err, 4u);
+            ok = __all_sync(0xffffffffu, ok) && !*abort_flag;
+            __half *rb = rowbuf + (size_t)(j & 1) * 128 * ST_PIX_H;
+            __half *cb = csbuf + (j & 1) * 128;
+            if (ok) {
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                const uint32_t trow = tmem + (uint32_t)(ab * 128) + ((uint32_t)(quad * 32) << 16);
+                float v[32];
+                tmem_ld16(trow + k0, v);
+                tmem_ld16(trow + k0 + 16, v + 16);
+                const float ctv = (has_cs && g.ct && half_id == 0) ? tmem_ld1(trow + ST_K) : 0.f;
+                asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&acc_empty[ab]));
+                if (q < g.Q) {
+                    float fsrc = 0.f;
+                    if (fd.active)
+                        fsrc = image_half(x, g, jb.n, fd.cin, 2 * jb.p + fd.r - 3, 2 * q + fd.s - 3);
+                    uint32_t pk[16];
+#pragma unroll
+                    for (int i = 0; i < 32; i += 2) {
+                        float o[2];
+#pragma unroll
+                        for (int t = 0; t < 2; ++t) {
+                            float s = v[i + t] + bias[i + t];
+                            if (fd.active && fd.kout == k0 + i + t) s += fd.dv * fsrc;
+                            if (a.relu) s = relu_keep_nan(s);
+                            o[t] = s;
+                        }
+                        __half2 hh = __floats2half2_rn(o[0], o[1]);
+                        pk[i / 2] = *reinterpret_cast<uint32_t *>(&hh);
+                    }
+                    uint4 *dst = reinterpret_cast<uint4 *>(rb + q * ST_PIX_H + k0);
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+                    if (has_cs && half_id == 0) {
+                        float o = (a.role == CT_ROLE_CT) ? ctv : 0.f;
+                        if (fd.active && fd.kout == ST_K) o += fd.dv * fsrc;
+                        if (a.relu) o = relu_keep_nan(o);
+                        cb[q] = __float2half_rn(o);
+                    }
+                }
+            }
+            if (epi_bar_or(!ok)) {
+                if (et == 0) *abort_flag = 1;
+                break;
+            }
+            // ---- column max over 2jj - 1 .. 2jj + 1, then the row logic ----
+            const int p = jb.p;
+            const bool close_even = (p & 1) == 0 && p == g.P - 1;
+            if (jb.seg_start) { acc_valid = false; has_carry = false; }
+            if (pool_data) {
+                uint32_t h[8];
+#pragma unroll
+                for (int i = 0; i < 8; ++i) h[i] = 0xFC00FC00u;
+#pragma unroll
+                for (int dc = -1; dc <= 1; ++dc) {
+                    const int col = 2 * jj + dc;
+                    if (col < 0 || col >= g.Q) continue;
+                    const uint4 *src = reinterpret_cast<const uint4 *>(rb + col * ST_PIX_H + 16 * cq);
+                    const uint4 s0 = src[0], s1 = src[1];
+                    h[0] = hmax2u(h[0], s0.x); h[1] = hmax2u(h[1], s0.y);
+                    h[2] = hmax2u(h[2], s0.z); h[3] = hmax2u(h[3], s0.w);
+                    h[4] = hmax2u(h[4], s1.x); h[5] = hmax2u(h[5], s1.y);
+                    h[6] = hmax2u(h[6], s1.z); h[7] = hmax2u(h[7], s1.w);
+                }
+                bool store = false;
+                if (p & 1) {
+                    if (acc_valid) {
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) accv[i] = hmax2u(accv[i], h[i]);
+                        store = true;
+                    }
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) carry[i] = h[i];
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) accv[i] = has_carry ? hmax2u(carry[i], h[i]) : h[i];
+                    store = close_even;
+                }
+                if (store) {
+                    const int i2 = (p & 1) ? (p - 1) / 2 : p / 2;
+                    uint4 *dst = reinterpret_cast<uint4 *>(static_cast<__half *>(a.y) +
+                                                            (((size_t)jb.n * g.P2 + i2) * g.Q2 + jj) * ST_K + 16 * cq);
+                    dst[0] = make_uint4(accv[0], accv[1], accv[2], accv[3]);
+                    dst[1] = make_uint4(accv[4], accv[5], accv[6], accv[7]);
+                }
+            }
+            if (pool_cs) {
+                __half h = __ushort_as_half((unsigned short)0xFC00);
+                for (int dc = -1; dc <= 1; ++dc) {
+                    const int col = 2 * et + dc;
+                    if (col >= 0 && col < g.Q) h = __hmax_nan(h, cb[col]);
+                }
+                bool store = false;
+                if (p & 1) {
+                    if (acc_valid) { acc_cs = __hmax_nan(acc_cs, h); store = true; }
+                    carry_cs = h;
+                } else {
+                    acc_cs = has_carry ? __hmax_nan(carry_cs, h) : h;
+                    store = close_even;
+                }
+                if (store) {
+                    const int i2 = (p & 1) ? (p - 1) / 2 : p / 2;
+                    static_cast<__half *>(a.cs_out)[((size_t)jb.n * g.P2 + i2) * g.Q2 + et] = acc_cs;
+                }
+            }
+            if (p & 1) { acc_valid = false; has_carry = true; }
+            else { acc_valid = !close_even; }
+            have = jb.next(g);
+            ++j;
+        }
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if (warp == 4) {
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)ST_TMEM_COLS));
+    }
+}
+
+}  // namespace
+
+struct StemPlan {
+    StemGeom g;
+    int sms;
+};
+
+int stem_kidx(int r, int s, int c) { return r * 32 + (s <= 3 ? s * 4 : 16 + (s - 3) * 4) + c; }
+int stem_klen() { return ST_KLEN; }
+
+bool stem_pool_supported(int C, int K, int R, int S, int stride, int pad, int H, int W) {
+    if (C < 1 || C > 4 || K != ST_K || R != ST_R || S != ST_R || stride != 2 || pad != 3) return false;
+    const int P = (H + 2 * pad - R) / stride + 1, Q = (W + 2 * pad - S) / stride + 1;
+    return P >= 2 && Q >= 2 && Q <= 128 && W + 4 <= ST_RP && W <= 256;
+}
+
+StemPlan *stem_plan_create(const ConvArgs &a, std::string *why) {
+    if (!stem_pool_supported(a.C, a.K, a.R, a.S, a.stride, a.pad, a.H, a.W)) {
+        if (why) *why = "shape not supported by the fused stem";
+        return nullptr;
+    }
+    StemPlan *pl = new (std::nothrow) StemPlan();
+    if (!pl) return nullptr;
+    StemGeom &g = pl->g;
+    g.C = a.C; g.H = a.H; g.W = a.W; g.P = a.P; g.Q = a.Q;
+    g.P2 = (g.P + 2 - 3) / 2 + 1;
+    g.Q2 = (g.Q + 2 - 3) / 2 + 1;
+    g.ct = a.role == CT_ROLE_CT;
+    __half h = __float2half_rn(a.coef);          // exact: coefficients are powers of two
+    memcpy(&g.coef_h, &h, 2);
+    pl->sms = device_sm_count();
+    if (cudaFuncSetAttribute(stem_pool_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ST_SMEM) !=
+        cudaSuccess) {
+        cudaGetLastError();
+        if (why) *why = "cannot reserve shared memory for the fused stem";
+        delete pl;
+        return nullptr;
+    }
+    return pl;
+}
+
+void stem_plan_destroy(StemPlan *p) { delete p; }
+
+cudaError_t launch_stem_pool(const ConvArgs &a, const StemPlan *pl, cudaStream_t st) {
+    StemGeom g = pl->g;
+    g.N = a.N;
+    const int units = g.N * g.P2;
+    const int grid = std::min(pl->sms, units);
+    stem_pool_kernel<<<grid, ST_THREADS, ST_SMEM, st>>>(a, g);
+    return cudaGetLastError();
+}
+
+}  // namespace ct

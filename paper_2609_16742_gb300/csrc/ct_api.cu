@@ -76,6 +76,7 @@ struct Slot {
     int cp = 0;                  // channel pitch of the NHWC data (C, or 4 for a padded image)
     bool has_cs = false;
     bool is_float = false;       // GAP output: fp32 features whatever the precision
+    bool stored = true;          // false: computed inside a fused kernel, never in HBM
     void *data = nullptr;
     void *cs = nullptr;
 };
@@ -93,6 +94,9 @@ struct LayerRT {
     TcPlan *plan = nullptr;
     bool tc_small = false;       // first layer with <= 4 input channels on the tensor cores
     TcSmallPlan *splan = nullptr;
+    bool stem = false;           // fused image stem: this conv and the max-pool after it
+    StemPlan *stplan = nullptr;
+    bool fused = false;          // max-pool computed by the preceding fused stem
     int w_ld = 0, c_stride = 0;  // weight row length and channel stride within a tap
     // fc
     int n_in = 0, n_cs = 0, n_out = 0;
@@ -166,6 +170,7 @@ void free_all(ct_model *m) {
     for (auto &l : m->L) {
         if (l.plan) tc_plan_destroy(l.plan);
         if (l.splan) tc_small_plan_destroy(l.splan);
+        if (l.stplan) stem_plan_destroy(l.stplan);
     }
     for (void *p : m->dev_allocs) cudaFree(p);
     m->dev_allocs.clear();
@@ -190,6 +195,12 @@ void put(std::vector<uint8_t> &buf, size_t i, double v, int prec) {
 float flipped(double stored, int bit, int prec) {
     if (prec == CT_FP16) return half_bits_to_float((uint16_t)(double_to_half_bits(stored) ^ (1u << bit)));
     return bits_float(float_bits((float)stored) ^ (1u << bit));
+}
+
+// stored word of data-filter weight (k, r, s, c) in the device weight array
+int64_t weight_word(const LayerRT &l, int k, int r, int s, int c) {
+    if (l.stem) return (int64_t)k * l.w_ld + stem_kidx(r, s, c);
+    return (int64_t)k * l.w_ld + ((int64_t)r * l.S + s) * l.c_stride + c;
 }
 
 // ---------------------------------------------------------------------------
@@ -274,14 +285,28 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
             std::string why;
             l.tc = prec == CT_FP16 && !(m->flags & CT_FLAG_SIMT_ONLY) &&
                    tc_supported(l.C, l.K, l.R, l.S, d.stride, d.pad, &why);
-            if (prec == CT_FP16 && !(m->flags & CT_FLAG_SIMT_ONLY) && d.src == 0 &&
+            if (prec == CT_FP16 && !(m->flags & CT_FLAG_SIMT_ONLY) && d.src == 0 && d.res < 0 && i + 1 < nL &&
+                stem_pool_supported(l.C, l.K, l.R, l.S, d.stride, d.pad, l.H, l.W)) {
+                // the image and the unpooled output must have no other reader
+                const ct_layer_desc &nx = desc->layers[i + 1];
+                int readers_in = 0, readers_mid = 0;
+                for (int j = 0; j < nL; ++j) {
+                    readers_in += (desc->layers[j].src == 0) + (desc->layers[j].res == 0);
+                    readers_mid += (desc->layers[j].src == d.dst) + (desc->layers[j].res == d.dst);
+                }
+                l.stem = nx.op == CT_OP_MAXPOOL && nx.src == d.dst && nx.k == 3 && nx.stride == 2 &&
+                         nx.pad == 1 && readers_in == 1 && readers_mid == 1;
+                if (l.stem) { src.stored = false; dst.stored = false; }
+            }
+            if (!l.stem && prec == CT_FP16 && !(m->flags & CT_FLAG_SIMT_ONLY) && d.src == 0 &&
                 tc_small_supported(l.C, l.K, l.R, l.S, d.stride, d.pad)) {
                 int readers = 0;               // the padded image must have no other reader
                 for (int j = 0; j < nL; ++j)
                     readers += (desc->layers[j].src == 0) + (desc->layers[j].res == 0);
                 l.tc_small = readers == 1;
             }
-            l.w_ld = l.tc_small ? tc_small_kpad(l.R, l.S) : RSC;
+            if (l.stem) l.tc = false;
+            l.w_ld = l.stem ? stem_klen() : l.tc_small ? tc_small_kpad(l.R, l.S) : RSC;
             l.c_stride = l.tc_small ? 4 : l.C;
             if (l.tc_small) src.cp = 4;
             std::vector<uint8_t> hw((size_t)l.K * l.w_ld * esz, 0);
@@ -301,7 +326,7 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
                     for (int r = 0; r < l.R; ++r)
                         for (int s = 0; s < l.S; ++s) {
                             double v = (double)W[(((size_t)k * l.C + c) * l.R + r) * l.S + s] * scale;
-                            put(hw, (size_t)k * l.w_ld + ((size_t)r * l.S + s) * l.c_stride + c, v, prec);
+                            put(hw, (size_t)weight_word(l, k, r, s, c), v, prec);
                         }
             }
             ct_status st;
@@ -311,6 +336,7 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
             CUDA_TRY(cudaMemcpy(l.bias, hb.data(), sizeof(float) * l.K, cudaMemcpyHostToDevice));
         } else if (d.op == CT_OP_MAXPOOL) {
             if (src.is_float || d.k < 1 || d.stride < 1 || d.pad < 0 || d.pad >= d.k) return CT_EINVAL;
+            l.fused = !m->L.empty() && m->L.back().stem && m->L.back().d.dst == d.src;
             dst.C = src.C;
             dst.H = (src.H + 2 * d.pad - d.k) / d.stride + 1;
             dst.W = (src.W + 2 * d.pad - d.k) / d.stride + 1;
@@ -357,7 +383,7 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
     // ---- activation slots ----
     for (size_t s = 0; s < m->slots.size(); ++s) {
         Slot &sl = m->slots[s];
-        if (!defined[s]) continue;
+        if (!defined[s] || !sl.stored) continue;
         bool is_final_out = false;
         for (auto &l : m->L) if (l.d.op == CT_OP_FC && l.d.final && l.d.dst == (int)s) is_final_out = true;
         if (is_final_out) continue;
@@ -369,6 +395,15 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
     }
     // ---- tensor-core plans ----
     for (auto &l : m->L) {
+        if (l.stem) {
+            ConvArgs a{};
+            a.N = B; a.H = l.H; a.W = l.W; a.C = l.C; a.K = l.K; a.R = l.R; a.S = l.S;
+            a.stride = l.d.stride; a.pad = l.d.pad; a.P = l.P; a.Q = l.Q; a.role = l.role; a.coef = l.coef;
+            std::string why;
+            l.stplan = stem_plan_create(a, &why);
+            if (!l.stplan) return CT_ECUDA;
+            continue;
+        }
         if (l.tc_small) {
             ConvArgs a{};
             a.N = B; a.H = l.H; a.W = l.W; a.C = l.C; a.K = l.K; a.R = l.R; a.S = l.S;
@@ -441,7 +476,7 @@ WeightFault resolve_weight_fault(const ct_model *m, const LayerRT &l, int64_t e,
     WeightFault f;
     if (k < l.K && c < l.C) {
         f.explicit_word = true;
-        f.word = (int64_t)k * l.w_ld + ((int64_t)r * l.S + s) * l.c_stride + c;
+        f.word = weight_word(l, k, r, s, c);
         return f;
     }
     double stored = 0.0;                      // zero slice and off-centre taps
@@ -461,7 +496,7 @@ ct_status act_fault_word(const ct_model *m, int slot, int batch, int64_t e, void
     const Slot &sl = m->slots[slot];
     const int Ct = sl.C + (sl.has_cs ? 1 : 0);
     const int64_t HW = (int64_t)sl.H * sl.W;
-    if (e < 0 || e >= (int64_t)batch * Ct * HW) return CT_ERANGE;
+    if (!sl.stored || e < 0 || e >= (int64_t)batch * Ct * HW) return CT_ERANGE;
     const int64_t n = e / (Ct * HW);
     const int c = (int)((e / HW) % Ct);
     const int64_t hw = e % HW;
@@ -488,9 +523,10 @@ ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, 
         if (act_fault_word(m, act_slot, batch, m->f_elem, &act_base, &act_word) != CT_OK) return CT_ERANGE;
     }
     Slot &s0 = m->slots[0];
-    CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] {
-        return launch_convert_input(input, s0.data, batch, s0.C, s0.cp, s0.H, s0.W, half, st);
-    }));
+    if (s0.stored)
+        CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] {
+            return launch_convert_input(input, s0.data, batch, s0.C, s0.cp, s0.H, s0.W, half, st);
+        }));
     if (act_slot == 0) CUDA_TRY(launch_xor_bit(act_base, act_word, m->f_bit, wb, st));
     for (size_t i = 0; i < m->L.size(); ++i) {
         LayerRT &l = m->L[i];
@@ -516,10 +552,19 @@ ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, 
                 else a.fd = wf.fd;
             }
             const double flops = 2.0 * batch * l.P * l.Q * (double)l.K * l.R * l.S * l.C;
-            if (l.tc_small) CUDA_TRY(launch(m, FAM_TC, flops, st, [&] { return launch_conv_tc_small(a, l.splan, st); }));
+            if (l.stem) {
+                // the fused kernel reads the FP32 image and writes the max-pool's output
+                const Slot &po = m->slots[m->L[i + 1].d.dst];
+                a.x = input;
+                a.y = po.data;
+                a.cs_out = po.has_cs ? po.cs : nullptr;
+                CUDA_TRY(launch(m, FAM_TC, flops, st, [&] { return launch_stem_pool(a, l.stplan, st); }));
+            } else if (l.tc_small) CUDA_TRY(launch(m, FAM_TC, flops, st, [&] { return launch_conv_tc_small(a, l.splan, st); }));
             else if (l.tc) CUDA_TRY(launch(m, FAM_TC, flops, st, [&] { return launch_conv_tc(a, l.plan, st); }));
             else CUDA_TRY(launch(m, FAM_SIMT, flops, st, [&] { return launch_conv_simt(a, half, st); }));
             if (wfault && wf.explicit_word) CUDA_TRY(launch_xor_bit(l.w, wf.word, m->f_bit, wb, st));
+        } else if (l.fused) {
+            // computed by the fused stem
         } else if (d.op == CT_OP_MAXPOOL || d.op == CT_OP_GAP) {
             PoolArgs a{};
             a.x = src.data; a.cs_in = src.has_cs ? src.cs : nullptr;
@@ -681,7 +726,7 @@ ct_status ct_inject(ct_model *m, int32_t kind, int32_t layer, int64_t element, i
     } else {
         const Slot &sl = m->slots[l.d.src];
         const int Ct = sl.C + (sl.has_cs ? 1 : 0);
-        if (element < 0 || element >= (int64_t)m->max_batch * Ct * sl.H * sl.W) return CT_ERANGE;
+        if (!sl.stored || element < 0 || element >= (int64_t)m->max_batch * Ct * sl.H * sl.W) return CT_ERANGE;
     }
     m->armed = true;
     m->f_kind = kind; m->f_layer = layer; m->f_elem = element; m->f_bit = bit;
@@ -826,7 +871,9 @@ ct_status ct_profile_read(ct_model *m, int32_t family, int64_t *launches, double
 
 ct_status ct_launches_per_infer(const ct_model *m, int32_t *n) {
     if (!m || !n) return CT_EINVAL;
-    *n = 1 + (int)m->L.size();
+    int cnt = m->slots[0].stored ? 1 : 0;
+    for (auto &l : m->L) cnt += l.fused ? 0 : 1;
+    *n = cnt;
     return CT_OK;
 }
 
@@ -836,6 +883,7 @@ ct_status ct_copy_activation(ct_model *m, int32_t slot, int32_t batch, void *dat
     if (!m) return CT_EINVAL;
     if (slot < 0 || slot >= (int)m->slots.size() || batch < 1 || batch > m->max_batch) return CT_ERANGE;
     const Slot &sl = m->slots[slot];
+    if (!sl.stored) return CT_ESTATE;
     if (!sl.data) return CT_ERANGE;
     const size_t e = sl.is_float ? 4 : m->esz();
     if (C) *C = sl.cp;

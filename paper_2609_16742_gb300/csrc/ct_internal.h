@@ -88,6 +88,9 @@ ct_status model_info(const ct_model *m, ModelInfo *out);
 ct_status infer_fault_free(ct_model *m, const float *input, int batch, float *logits, float *S,
                            uint8_t *flag, cudaStream_t st);
 
+// number of SMs of the current device (148 if the query fails)
+int device_sm_count();
+
 // tensor-core conv plan (opaque outside conv_tc.cu)
 struct TcPlan;
 TcPlan *tc_plan_create(const ConvArgs &shape_args, int max_batch, const void *w_dev, const void *x_dev,
@@ -104,5 +107,17 @@ int tc_small_kpad(int R, int S);
 TcSmallPlan *tc_small_plan_create(const ConvArgs &shape_args, const void *w_dev, std::string *why);
 void tc_small_plan_destroy(TcSmallPlan *p);
 cudaError_t launch_conv_tc_small(const ConvArgs &a, const TcSmallPlan *plan, cudaStream_t st);
+
+// Fused image stem (7x7 stride-2 convolution, C <= 4, 64 filters, followed
+// by a 3x3 stride-2 padding-1 max-pool): reads the FP32 NCHW image, writes
+// the pooled NHWC tensor and its checksum plane.  Weights [64][stem_klen()]
+// with K index stem_kidx(r, s, c).
+struct StemPlan;
+bool stem_pool_supported(int C, int K, int R, int S, int stride, int pad, int H, int W);
+int stem_kidx(int r, int s, int c);
+int stem_klen();
+StemPlan *stem_plan_create(const ConvArgs &shape_args, std::string *why);
+void stem_plan_destroy(StemPlan *p);
+cudaError_t launch_stem_pool(const ConvArgs &a, const StemPlan *p, cudaStream_t st);
 
 }  // namespace ct

@@ -10,6 +10,8 @@ from _gpu import TOL, ct, model, onet, run
 
 pytestmark = pytest.mark.gpu
 
+CT_ESTATE = 4
+
 
 def layer_errors(name, prec, batch, simt_only=False, first=0):
     """[(slot, op, data_rel_err, cs_rel_err)] for one inference; raises on a device error."""
@@ -24,7 +26,12 @@ def layer_errors(name, prec, batch, simt_only=False, first=0):
     for L in wl.layers:
         if L.op == "fc" and L.final:
             continue
-        gd, gc = ct().ct_copy_activation(m, L.dst, batch)
+        try:
+            gd, gc = ct().ct_copy_activation(m, L.dst, batch)
+        except ct().CtError as e:
+            if e.status == CT_ESTATE:          # computed inside a fused kernel, never stored
+                continue
+            raise
         ed = ec = 0.0
         for n in range(batch):
             a = o["acts"][n][L.dst]
