@@ -166,7 +166,14 @@ ct_status ct_clear_faults(ct_model *m);
  * logits_dev and S_dev (the re-run's own flags are ignored; flag_dev is not
  * modified).  Synchronises `stream` once to read the flags.  *n_rerun
  * (host) receives the number of images re-run.  Same buffers as ct_infer.
- * An armed fault stays armed for the next ct_infer. */
+ * The re-run batch is padded to the next power of two by repeating the
+ * last flagged image.  Its inference is captured into a CUDA graph on a
+ * model-owned stream the first time that padded size occurs (that call is
+ * slower) and replayed afterwards; with profiling on (ct_profile_enable) the
+ * kernels are launched one by one instead.  A re-run row equals a fault-free
+ * ct_infer of the padded batch; because small batches split K differently,
+ * it can differ from the same image's row of a full batch by summation
+ * order.  An armed fault stays armed for the next ct_infer. */
 ct_status ct_reexecute(ct_model *m, const float *input_dev, int32_t batch,
                        const uint8_t *flag_dev, float *logits_dev, float *S_dev,
                        int32_t *n_rerun, void *stream);
@@ -233,8 +240,17 @@ ct_status ct_profile_enable(ct_model *m, int32_t on);
 ct_status ct_profile_read(ct_model *m, int32_t family, int64_t *launches, double *ms,
                           double *flops);
 
-/* Number of kernels one fault-free ct_infer of this model launches. */
+/* Number of library kernels the most recent inference of this model
+ * launched (fault-injection bit flips not counted); a layer whose K
+ * dimension is split across CTAs (small batches) launches two.  Before the
+ * first inference: the count without split K. */
 ct_status ct_launches_per_infer(const ct_model *m, int32_t *n);
+
+/* ct_kernel_count -- number of library kernels launched for this model since
+ * the previous call (directly, or as nodes of the re-execution graphs that
+ * ct_reexecute replays), fault-injection bit flips included; resets the
+ * count.  Host bookkeeping only: no synchronisation. */
+ct_status ct_kernel_count(ct_model *m, int64_t *n);
 
 /* ct_copy_activation -- diagnostic read of an intermediate tensor of the
  * last ct_infer on `stream`: slot `slot` (0 = converted input; the `dst` of

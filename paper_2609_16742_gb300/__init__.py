@@ -34,7 +34,7 @@ _STATUS = {0: "CT_OK", 1: "CT_EINVAL", 2: "CT_ENOMEM", 3: "CT_ECUDA", 4: "CT_EST
 # every exported symbol of include/ct.h
 EXPORTS = ["ct_build", "ct_set_threshold", "ct_get_threshold", "ct_infer", "ct_inject",
            "ct_clear_faults", "ct_reexecute", "ct_run_host", "ct_calibrate", "ct_buffer_count",
-           "ct_buffer_info", "ct_profile_enable", "ct_profile_read", "ct_launches_per_infer",
+           "ct_buffer_info", "ct_profile_enable", "ct_profile_read", "ct_launches_per_infer", "ct_kernel_count",
            "ct_copy_activation", "ct_device_error", "ct_destroy", "ct_strerror",
            "ct_reexecute_noalloc"]
 
@@ -94,6 +94,7 @@ def lib():
             "ct_profile_enable": [vp, i32],
             "ct_profile_read": [vp, i32, P(i64), P(dbl), P(dbl)],
             "ct_launches_per_infer": [vp, P(i32)],
+            "ct_kernel_count": [vp, P(i64)],
             "ct_copy_activation": [vp, i32, i32, vp, vp, P(i32), P(i32), P(i32), P(i32), P(i32), vp],
             "ct_device_error": [vp, P(ctypes.c_uint32)],
         }
@@ -288,6 +289,13 @@ def ct_profile_read(m: Model, family: int):
     _check(lib().ct_profile_read(m.handle, family, ctypes.byref(n), ctypes.byref(ms),
                                  ctypes.byref(fl)), "ct_profile_read")
     return n.value, ms.value, fl.value
+
+
+def ct_kernel_count(m: Model) -> int:
+    """Library kernels launched for m since the previous call (then reset)."""
+    n = ctypes.c_int64()
+    _check(lib().ct_kernel_count(m.handle, ctypes.byref(n)), "ct_kernel_count")
+    return n.value
 
 
 def ct_launches_per_infer(m: Model) -> int:

@@ -174,13 +174,18 @@ conv_simt_kernel(ConvArgs a) {
         for (int j = 0; j < TN; ++j) acc[i][j] = 0.f;
     }
 
-    const int nk = (Ktot + BK - 1) / BK;
-    load_tiles(0);
-    store_tiles(0);
+    // K tiles of this block: all of them, or one split's range (gridDim.z > 1)
+    const int nk_all = (Ktot + BK - 1) / BK;
+    const int kps = (nk_all + gridDim.z - 1) / gridDim.z;
+    const int kt_lo = blockIdx.z * kps, kt_hi = min(nk_all, kt_lo + kps);
+    if (kt_lo < kt_hi) {
+        load_tiles(kt_lo);
+        store_tiles(0);
+    }
     __syncthreads();
-    for (int kt = 0; kt < nk; ++kt) {
-        const int buf = kt & 1;
-        if (kt + 1 < nk) load_tiles(kt + 1);
+    for (int kt = kt_lo; kt < kt_hi; ++kt) {
+        const int buf = (kt - kt_lo) & 1;
+        if (kt + 1 < kt_hi) load_tiles(kt + 1);
         const int k0 = kt * BK;
 #pragma unroll
         for (int kk = 0; kk < BK; ++kk) {
@@ -207,8 +212,27 @@ conv_simt_kernel(ConvArgs a) {
                 }
             }
         }
-        if (kt + 1 < nk) store_tiles(buf ^ 1);
+        if (kt + 1 < kt_hi) store_tiles(buf ^ 1);
         __syncthreads();
+    }
+
+    if (gridDim.z > 1) {
+        // split-K: FP32 partial sums; the reduction kernel applies the epilogue
+        const int ws_ld = (a.K + 1 + 3) & ~3;
+        float *wz = a.ws + (size_t)blockIdx.z * M * ws_ld;
+#pragma unroll
+        for (int i = 0; i < TM; ++i) {
+            const int m = m0 + ty * TM + i;
+            if (m >= M) break;
+#pragma unroll
+            for (int j = 0; j < TN; ++j) {
+                const int k = n0 + tx * TN + j;
+                if (k < a.K) wz[(size_t)m * ws_ld + k] = acc[i][j];
+            }
+            if (a.cs_out != nullptr && blockIdx.y == 0 && tx == 0)
+                wz[(size_t)m * ws_ld + a.K] = do_cs ? a.coef * csum[i] : 0.f;
+        }
+        return;
     }
 
     // ---- epilogue ----
@@ -287,30 +311,46 @@ conv_simt_kernel(ConvArgs a) {
     }
 }
 
+int sm_count_cached() {
+    static int n = 0;
+    if (n == 0) n = device_sm_count();
+    return n;
+}
+
 template <typename T, int BM, int BN, int BK, int TM, int TN, bool VEC>
-cudaError_t go(const ConvArgs &a, cudaStream_t st) {
+cudaError_t go(const ConvArgs &a, cudaStream_t st, int *n_kernels) {
     const int M = a.N * a.P * a.Q;
-    dim3 grid((M + BM - 1) / BM, (a.K + BN - 1) / BN);
+    const int gx = (M + BM - 1) / BM, gy = (a.K + BN - 1) / BN;
+    // split K when the output tiles leave most SMs idle (at least 8 K tiles per split)
+    const int ws_ld = (a.K + 1 + 3) & ~3;
+    const int nk = (a.R * a.S * a.C + BK - 1) / BK;
+    const int splits = (a.K % 8 == 0) ? splitk_choose(gx * gy, nk, 8, 2 * sm_count_cached(), M, ws_ld,
+                                                      a.ws ? a.ws_bytes : 0) : 1;
+    dim3 grid(gx, gy, splits);
     conv_simt_kernel<T, BM, BN, BK, TM, TN, VEC><<<grid, (BM / TM) * (BN / TN), 0, st>>>(a);
-    return cudaGetLastError();
+    cudaError_t e = cudaGetLastError();
+    if (n_kernels) *n_kernels = 1;
+    if (e != cudaSuccess || splits == 1) return e;
+    if (n_kernels) *n_kernels = 2;
+    return launch_splitk_reduce(a, splits, ws_ld, sizeof(T) == 2, st);
 }
 
 template <typename T>
-cudaError_t dispatch(const ConvArgs &a, cudaStream_t st) {
+cudaError_t dispatch(const ConvArgs &a, cudaStream_t st, int *nk) {
     constexpr int VE = Vec<T>::n;
     const bool vec = (a.C % 16 == 0) && (a.C % VE == 0);
     if (vec) {
-        if (a.K >= 128) return go<T, 128, 128, 16, 8, 8, true>(a, st);
-        return go<T, 128, 64, 16, 8, 4, true>(a, st);
+        if (a.K >= 128) return go<T, 128, 128, 16, 8, 8, true>(a, st, nk);
+        return go<T, 128, 64, 16, 8, 4, true>(a, st, nk);
     }
-    if (a.K <= 16) return go<T, 64, 16, 16, 4, 4, false>(a, st);
-    return go<T, 128, 64, 16, 8, 4, false>(a, st);
+    if (a.K <= 16) return go<T, 64, 16, 16, 4, 4, false>(a, st, nk);
+    return go<T, 128, 64, 16, 8, 4, false>(a, st, nk);
 }
 
 }  // namespace
 
-cudaError_t launch_conv_simt(const ConvArgs &a, bool half, cudaStream_t st) {
-    return half ? dispatch<__half>(a, st) : dispatch<float>(a, st);
+cudaError_t launch_conv_simt(const ConvArgs &a, bool half, cudaStream_t st, int *n_kernels) {
+    return half ? dispatch<__half>(a, st, n_kernels) : dispatch<float>(a, st, n_kernels);
 }
 
 }  // namespace ct

@@ -60,8 +60,25 @@ struct TcGeom {
     int ct_mode;
     int tmem_cols;
     int m_tiles, n_tiles;
+    int splits, kps, ws_ld;      // split-K: K blocks per split, workspace row length
     uint16_t coef_h;
 };
+
+// K-block range [lo, hi) and output tile of persistent work item `tile`
+struct TileRef {
+    int m0, n_tile, sp, kb_lo, kb_hi;
+};
+__device__ __forceinline__ TileRef tile_ref(int tile, const TcGeom &g) {
+    TileRef t;
+    const int per = g.m_tiles * g.n_tiles;
+    t.sp = tile / per;
+    const int rt = tile - t.sp * per;
+    t.m0 = (rt / g.n_tiles) * BM;
+    t.n_tile = rt % g.n_tiles;
+    t.kb_lo = t.sp * g.kps;
+    t.kb_hi = min(g.n_kb, t.kb_lo + g.kps);
+    return t;
+}
 
 
 // tap visited at K-block kb: the centre tap first, the others in order
@@ -160,7 +177,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
     volatile uint32_t *abort_flag = tmem_holder + 1;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int num_tiles = g.m_tiles * g.n_tiles;
+    const int num_tiles = g.m_tiles * g.n_tiles * g.splits;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -204,16 +221,17 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
         int it = 0;
         for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
             if (__any_sync(0xffffffffu, *abort_flag)) break;
-            const int m0 = (tile / g.n_tiles) * BM, n_tile = tile % g.n_tiles;
+            const TileRef tr = tile_ref(tile, g);
+            const int m0 = tr.m0, n_tile = tr.n_tile;
             const int nimg = m0 / g.PQ, rem = m0 % g.PQ;
             const int p = rem / g.Q, q = rem % g.Q;
             const int w0 = q * g.stride - g.pad, h0 = p * g.stride - g.pad;
             bool ok = true;
-            for (int kb0 = 0; kb0 < g.n_kb; kb0 += SUB, ++it) {
+            for (int kb0 = tr.kb_lo; kb0 < tr.kb_hi; kb0 += SUB, ++it) {
                 const int s = it % STAGES;
                 const uint32_t ph = (uint32_t)(it / STAGES) & 1u;
                 if (!warp_wait(smem_u32(&empty[s]), ph ^ 1u, a.err, 1u)) { ok = false; break; }
-                const int nsub = min(SUB, g.n_kb - kb0);
+                const int nsub = min(SUB, tr.kb_hi - kb0);
                 const uint32_t fb = smem_u32(&full[s]);
                 if (elect_one()) {
                     mbar_arrive_expect_tx(fb, nsub * (A_BYTES + B_TMA_BYTES));
@@ -241,7 +259,8 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
         int it = 0, lt = 0;
         for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++lt) {
             if (__any_sync(0xffffffffu, *abort_flag)) break;
-            const int n_tile = tile % g.n_tiles;
+            const TileRef tr = tile_ref(tile, g);
+            const int n_tile = tr.n_tile;
             const bool ct_here = g.ct_mode != CT_NONE_ && n_tile == 0;
             if (!warp_wait(smem_u32(acc_empty), ((uint32_t)lt & 1u) ^ 1u, a.err, 8u)) {
                 if (lane == 0) *abort_flag = 1;
@@ -249,16 +268,17 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
             }
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
             bool ok = true;
-            for (int kb0 = 0; kb0 < g.n_kb; kb0 += SUB, ++it) {
+            for (int kb0 = tr.kb_lo; kb0 < tr.kb_hi; kb0 += SUB, ++it) {
                 const int s = it % STAGES;
                 const uint32_t ph = (uint32_t)(it / STAGES) & 1u;
                 if (!warp_wait(smem_u32(&full[s]), ph, a.err, 2u)) { ok = false; break; }
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-                const int nsub = min(SUB, g.n_kb - kb0);
+                const int nsub = min(SUB, tr.kb_hi - kb0);
                 const bool leader = elect_one();
                 for (int j = 0; j < nsub; ++j) {
                     const int kb = kb0 + j;
-                    const uint32_t d = tmem + (uint32_t)((kb % NCH) * CH);
+                    const int kr = kb - tr.kb_lo;               // position within this split
+                    const uint32_t d = tmem + (uint32_t)((kr % NCH) * CH);
                     const bool centre = kb < g.cpb;
                     const uint32_t a_base = smem_u32(As + (s * SUB + j) * A_BYTES);
                     const uint32_t b_base = smem_u32(Bs + (s * SUB + j) * B_SUB_BYTES);
@@ -266,7 +286,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
                     for (int k16 = 0; k16 < BK / 16; ++k16) {
                         const uint64_t ad = smem_desc_sw128(a_base + k16 * 32);
                         const uint64_t bd = smem_desc_sw128(b_base + k16 * 32);
-                        const uint32_t acc = (kb >= NCH || k16 > 0) ? 1u : 0u;   // first use of the chain
+                        const uint32_t acc = (kr >= NCH || k16 > 0) ? 1u : 0u;   // first use of the chain
                         if (leader) {
                             if (ct_here && centre && g.ct_mode == CT_MERGED) {
                                 umma_f16(d, ad, bd, id_merged, acc);
@@ -293,11 +313,14 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
         const int row = quad * 32 + lane;
         const __half *x = static_cast<const __half *>(a.x);
         const FaultDelta fd = a.fd;
-        const int chains = min(NCH, g.n_kb);                       // chains that received MMAs
-        const int ct_chains = min(NCH, g.cpb);                     // chains holding a carry-through column
+        const bool split = g.splits > 1;
         int lt = 0;
         for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++lt) {
-            const int m0 = (tile / g.n_tiles) * BM, n_tile = tile % g.n_tiles;
+            const TileRef tr = tile_ref(tile, g);
+            const int m0 = tr.m0, n_tile = tr.n_tile;
+            const int chains = min(NCH, tr.kb_hi - tr.kb_lo);                    // chains that received MMAs
+            // chains whose first K block is a centre block hold a carry-through column
+            const int ct_chains = max(0, min(NCH, min(g.cpb, tr.kb_hi) - tr.kb_lo));
             bool ok = mbar_wait(smem_u32(acc_full), (uint32_t)lt & 1u, a.err, 4u) && !*abort_flag;
             ok = __all_sync(0xffffffffu, ok);      // tcgen05.ld below is warp-collective
             if (!ok) break;
@@ -308,7 +331,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
             const int mm = valid ? m : 0;
             const int nimg = mm / g.PQ, rem = mm % g.PQ, p = rem / g.Q, q = rem % g.Q;
             float fsrc = 0.f;
-            if (fd.active) {
+            if (fd.active && !split) {
                 const int h = p * g.stride + fd.r - g.pad, w = q * g.stride + fd.s - g.pad;
                 if (h >= 0 && h < a.H && w >= 0 && w < a.W) {
                     if (fd.cin < g.C) fsrc = ldh(x, (((size_t)nimg * a.H + h) * a.W + w) * g.C + fd.cin);
@@ -335,7 +358,14 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
                 asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
                 __syncwarp();
                 if (lane == 0) mbar_arrive(smem_u32(acc_empty));   // accumulators free for the next tile
-                if (valid) {
+                if (valid && split) {
+                    float *wrow = a.ws + ((size_t)tr.sp * g.M + m) * g.ws_ld;
+#pragma unroll
+                    for (int c = 0; c < BN / 2; c += 4)
+                        *reinterpret_cast<float4 *>(wrow + n0 + half * (BN / 2) + c) =
+                            make_float4(vals[c], vals[c + 1], vals[c + 2], vals[c + 3]);
+                    if (do_cs) wrow[g.K] = ctv;
+                } else if (valid) {
 #pragma unroll
                     for (int c = 0; c < BN / 2; c += 16)
                         store_chunk(vals + c, a, g.K, (size_t)m, n0 + half * (BN / 2) + c, fsrc);
@@ -352,11 +382,18 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
 #pragma unroll
                         for (int i = 0; i < 16; ++i) v[i] += t[i];
                     }
-                    if (valid) store_chunk(v, a, g.K, (size_t)m, n0 + c, fsrc);
+                    if (valid && split) {
+                        float4 *wp = reinterpret_cast<float4 *>(a.ws + ((size_t)tr.sp * g.M + m) * g.ws_ld + n0 + c);
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) wp[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+                    } else if (valid) {
+                        store_chunk(v, a, g.K, (size_t)m, n0 + c, fsrc);
+                    }
                 }
                 if (do_cs && g.ct_mode != CT_NONE_)
                     for (int ch = 0; ch < ct_chains; ++ch) ctv += tmem_ld1(trow + ch * CH + BN);
-                if (do_cs && valid) store_checksum(ctv, a, g, m, nimg, p, q, fsrc);
+                if (do_cs && valid && split) a.ws[((size_t)tr.sp * g.M + m) * g.ws_ld + g.K] = ctv;
+                else if (do_cs && valid) store_checksum(ctv, a, g, m, nimg, p, q, fsrc);
                 asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
                 __syncwarp();
                 if (lane == 0) mbar_arrive(smem_u32(acc_empty));
@@ -701,17 +738,26 @@ TcPlan *tc_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, cons
     return pl;
 }
 
-cudaError_t launch_conv_tc(const ConvArgs &a, const void *plan, cudaStream_t st) {
+cudaError_t launch_conv_tc(const ConvArgs &a, const void *plan, cudaStream_t st, int *n_kernels) {
     const TcPlan *pl = static_cast<const TcPlan *>(plan);
     TcGeom g = pl->g;
     g.M = a.N * a.P * a.Q;
     g.m_tiles = (g.M + BM - 1) / BM;
     const int tiles = g.m_tiles * g.n_tiles;
-    dim3 grid(tiles < pl->sms ? tiles : pl->sms);
+    // split K when the output tiles leave most SMs idle (at least 4 K blocks per split)
+    g.ws_ld = (g.K + 1 + 3) & ~3;
+    g.splits = (a.K % 8 == 0) ? splitk_choose(tiles, g.n_kb, 4, pl->sms, g.M, g.ws_ld, a.ws ? a.ws_bytes : 0) : 1;
+    g.kps = (g.n_kb + g.splits - 1) / g.splits;
+    const int items = tiles * g.splits;
+    dim3 grid(items < pl->sms ? items : pl->sms);
     if (pl->BN == 64) conv_tc_kernel<64, 4, 2, 4><<<grid, NTHREADS, pl->smem, st>>>(pl->amap, pl->bmap, a, g);
     else if (pl->BN == 128) conv_tc_kernel<128, 3, 2, 2><<<grid, NTHREADS, pl->smem, st>>>(pl->amap, pl->bmap, a, g);
     else conv_tc_kernel<256, 4, 1, 1><<<grid, NTHREADS, pl->smem, st>>>(pl->amap, pl->bmap, a, g);
-    return cudaGetLastError();
+    cudaError_t e = cudaGetLastError();
+    if (n_kernels) *n_kernels = 1;
+    if (e != cudaSuccess || g.splits == 1) return e;
+    if (n_kernels) *n_kernels = 2;
+    return launch_splitk_reduce(a, g.splits, g.ws_ld, true, st);
 }
 
 bool tc_small_supported(int C, int K, int R, int S, int stride, int pad) {

@@ -104,7 +104,10 @@ struct LayerRT {
     bool fc_tc = false;          // hidden FC run on the tensor-core conv kernel as a 1x1 conv
 };
 
-struct EvRec { int fam; int ev; double flops; };
+struct EvRec { int fam; int ev; double flops; int nk; };
+
+// split-K workspace of a model (FP32 partial sums of one layer at a time)
+constexpr size_t SPLITK_WS_BYTES = 32ull << 20;
 
 }  // namespace
 
@@ -132,6 +135,14 @@ struct ct_model {
     float *rh_input = nullptr, *rh_logits = nullptr, *rh_S = nullptr;
     uint8_t *rh_flag = nullptr;
     uint32_t *d_err = nullptr;
+    float *ws = nullptr;         // split-K partial sums
+    // re-execution: one captured inference graph per power-of-two batch
+    cudaStream_t cap_stream = nullptr;
+    std::vector<cudaGraphExec_t> re_graph;
+    std::vector<int> re_graph_nk;        // kernels in each graph
+    int64_t kernels_total = 0;           // kernels launched since the last ct_kernel_count
+    int n_kernels_last = -1;     // kernels launched by the last inference
+    int n_kernels_run = 0;
     std::vector<void *> dev_allocs;
     // profiling
     bool prof = false;
@@ -178,6 +189,11 @@ void free_all(ct_model *m) {
     if (m->h_idx) cudaFreeHost(m->h_idx);
     for (auto &e : m->ev_pool) { cudaEventDestroy(e.first); cudaEventDestroy(e.second); }
     m->ev_pool.clear();
+    for (cudaGraphExec_t g : m->re_graph)
+        if (g) cudaGraphExecDestroy(g);
+    m->re_graph.clear();
+    if (m->cap_stream) cudaStreamDestroy(m->cap_stream);
+    m->cap_stream = nullptr;
 }
 
 // store a double as the storage word (fp32 or fp16) into a byte buffer
@@ -207,9 +223,20 @@ int64_t weight_word(const LayerRT &l, int k, int r, int s, int c) {
 // profiling helpers
 // ---------------------------------------------------------------------------
 
+// fault-injection bit flip (counted, not timed)
+cudaError_t xor_bit(ct_model *m, void *base, int64_t word, int bit, int word_bytes, cudaStream_t st) {
+    ++m->kernels_total;
+    return launch_xor_bit(base, word, bit, word_bytes, st);
+}
+
 template <typename F>
-cudaError_t launch(ct_model *m, int fam, double flops, cudaStream_t st, F &&fn) {
-    if (!m->prof) return fn();
+cudaError_t launch(ct_model *m, int fam, double flops, cudaStream_t st, F &&fn, const int *nk = nullptr) {
+    if (!m->prof) {
+        cudaError_t e = fn();
+        m->n_kernels_run += nk ? *nk : 1;
+        m->kernels_total += nk ? *nk : 1;
+        return e;
+    }
     int ev;
     if (!m->ev_free.empty()) { ev = m->ev_free.back(); m->ev_free.pop_back(); }
     else {
@@ -222,7 +249,10 @@ cudaError_t launch(ct_model *m, int fam, double flops, cudaStream_t st, F &&fn) 
     cudaEventRecord(m->ev_pool[ev].first, st);
     cudaError_t e = fn();
     cudaEventRecord(m->ev_pool[ev].second, st);
-    m->recs.push_back({fam, ev, flops});
+    const int n = nk ? *nk : 1;
+    m->recs.push_back({fam, ev, flops, n});
+    m->n_kernels_run += n;
+    m->kernels_total += n;
     return e;
 }
 
@@ -444,6 +474,7 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
     if ((st = dalloc(m, (void **)&m->rh_S, sizeof(float) * B)) != CT_OK) return st;
     if ((st = dalloc(m, (void **)&m->rh_flag, B)) != CT_OK) return st;
     if ((st = dalloc(m, (void **)&m->d_err, sizeof(uint32_t))) != CT_OK) return st;
+    if ((st = dalloc(m, (void **)&m->ws, SPLITK_WS_BYTES)) != CT_OK) return st;
     CUDA_TRY(cudaMemset(m->d_err, 0, sizeof(uint32_t)));
     if (cudaMallocHost((void **)&m->h_flags, B) != cudaSuccess) return CT_ENOMEM;
     if (cudaMallocHost((void **)&m->h_idx, sizeof(int32_t) * B) != cudaSuccess) return CT_ENOMEM;
@@ -515,6 +546,7 @@ ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, 
     const int wb = half ? 2 : 4;
     const bool armed = m->armed;
     m->armed = false;
+    m->n_kernels_run = 0;
     int act_slot = -1;
     void *act_base = nullptr;
     int64_t act_word = 0;
@@ -527,7 +559,7 @@ ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, 
         CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] {
             return launch_convert_input(input, s0.data, batch, s0.C, s0.cp, s0.H, s0.W, half, st);
         }));
-    if (act_slot == 0) CUDA_TRY(launch_xor_bit(act_base, act_word, m->f_bit, wb, st));
+    if (act_slot == 0) CUDA_TRY(xor_bit(m, act_base, act_word, m->f_bit, wb, st));
     for (size_t i = 0; i < m->L.size(); ++i) {
         LayerRT &l = m->L[i];
         const ct_layer_desc &d = l.d;
@@ -548,7 +580,7 @@ ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, 
             const bool wfault = armed && m->f_kind == CT_BUF_WEIGHT && m->f_layer == (int)i;
             if (wfault) {
                 wf = resolve_weight_fault(m, l, m->f_elem, m->f_bit);
-                if (wf.explicit_word) CUDA_TRY(launch_xor_bit(l.w, wf.word, m->f_bit, wb, st));
+                if (wf.explicit_word) CUDA_TRY(xor_bit(m, l.w, wf.word, m->f_bit, wb, st));
                 else a.fd = wf.fd;
             }
             const double flops = 2.0 * batch * l.P * l.Q * (double)l.K * l.R * l.S * l.C;
@@ -559,10 +591,15 @@ ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, 
                 a.y = po.data;
                 a.cs_out = po.has_cs ? po.cs : nullptr;
                 CUDA_TRY(launch(m, FAM_TC, flops, st, [&] { return launch_stem_pool(a, l.stplan, st); }));
-            } else if (l.tc_small) CUDA_TRY(launch(m, FAM_TC, flops, st, [&] { return launch_conv_tc_small(a, l.splan, st); }));
-            else if (l.tc) CUDA_TRY(launch(m, FAM_TC, flops, st, [&] { return launch_conv_tc(a, l.plan, st); }));
-            else CUDA_TRY(launch(m, FAM_SIMT, flops, st, [&] { return launch_conv_simt(a, half, st); }));
-            if (wfault && wf.explicit_word) CUDA_TRY(launch_xor_bit(l.w, wf.word, m->f_bit, wb, st));
+            } else if (l.tc_small) {
+                CUDA_TRY(launch(m, FAM_TC, flops, st, [&] { return launch_conv_tc_small(a, l.splan, st); }));
+            } else {
+                a.ws = m->ws; a.ws_bytes = SPLITK_WS_BYTES;
+                int nk = 1;
+                if (l.tc) CUDA_TRY(launch(m, FAM_TC, flops, st, [&] { return launch_conv_tc(a, l.plan, st, &nk); }, &nk));
+                else CUDA_TRY(launch(m, FAM_SIMT, flops, st, [&] { return launch_conv_simt(a, half, st, &nk); }, &nk));
+            }
+            if (wfault && wf.explicit_word) CUDA_TRY(xor_bit(m, l.w, wf.word, m->f_bit, wb, st));
         } else if (l.fused) {
             // computed by the fused stem
         } else if (d.op == CT_OP_MAXPOOL || d.op == CT_OP_GAP) {
@@ -584,8 +621,10 @@ ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, 
             a.stride = 1; a.pad = 0; a.P = a.Q = 1;
             a.role = m->protect ? CT_ROLE_CT : CT_ROLE_NONE; a.relu = d.relu; a.coef = l.coef;
             a.err = m->d_err; a.cs_rowsum = l.n_cs;
+            a.ws = m->ws; a.ws_bytes = SPLITK_WS_BYTES;
             const double flops = 2.0 * batch * (double)l.n_in * l.n_out;
-            CUDA_TRY(launch(m, FAM_FC, flops, st, [&] { return launch_conv_tc(a, l.plan, st); }));
+            int nk = 1;
+            CUDA_TRY(launch(m, FAM_FC, flops, st, [&] { return launch_conv_tc(a, l.plan, st, &nk); }, &nk));
         } else {
             FcArgs a{};
             a.x = src.data; a.xcs = src.has_cs ? src.cs : nullptr; a.w = l.w; a.bias = l.bias;
@@ -597,9 +636,44 @@ ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, 
             const double flops = 2.0 * batch * (double)l.n_in * l.n_out;
             CUDA_TRY(launch(m, FAM_FC, flops, st, [&] { return launch_fc(a, half, l.x_float, st); }));
         }
-        if (act_slot == d.dst) CUDA_TRY(launch_xor_bit(act_base, act_word, m->f_bit, wb, st));
+        if (act_slot == d.dst) CUDA_TRY(xor_bit(m, act_base, act_word, m->f_bit, wb, st));
     }
+    m->n_kernels_last = m->n_kernels_run;
     return CT_OK;
+}
+
+// Fault-free inference of the first `bucket` images of the re-execution
+// scratch, replayed from a graph captured on first use of this batch size:
+// one graph launch instead of one host launch per kernel.  Falls back to
+// direct launches if capture or instantiation fails.
+cudaGraphExec_t reexec_graph(ct_model *m, int bucket) {
+    int slot = 0;
+    while ((1 << slot) < bucket) ++slot;
+    if ((int)m->re_graph.size() <= slot) {
+        m->re_graph.resize(slot + 1, nullptr);
+        m->re_graph_nk.resize(slot + 1, 0);
+    }
+    if (m->re_graph[slot]) return m->re_graph[slot];
+    if (!m->cap_stream && cudaStreamCreateWithFlags(&m->cap_stream, cudaStreamNonBlocking) != cudaSuccess) {
+        cudaGetLastError();
+        return nullptr;
+    }
+    if (cudaStreamBeginCapture(m->cap_stream, cudaStreamCaptureModeThreadLocal) != cudaSuccess) {
+        cudaGetLastError();
+        return nullptr;
+    }
+    const int64_t before = m->kernels_total;
+    const ct_status s = infer_impl(m, m->re_input, bucket, m->re_logits, m->re_S, m->re_flag, m->cap_stream);
+    m->re_graph_nk[slot] = (int)(m->kernels_total - before);
+    m->kernels_total = before;           // captured, not launched
+    cudaGraph_t g = nullptr;
+    const cudaError_t e = cudaStreamEndCapture(m->cap_stream, &g);
+    cudaGraphExec_t ex = nullptr;
+    if (s == CT_OK && e == cudaSuccess && g && cudaGraphInstantiate(&ex, g, 0) != cudaSuccess) ex = nullptr;
+    if (g) cudaGraphDestroy(g);
+    cudaGetLastError();
+    m->re_graph[slot] = ex;
+    return ex;
 }
 
 ct_status reexec_impl(ct_model *m, const float *input, int batch, const uint8_t *flag, float *logits,
@@ -611,13 +685,28 @@ ct_status reexec_impl(ct_model *m, const float *input, int batch, const uint8_t 
         if (m->h_flags[i]) m->h_idx[n++] = i;
     if (n_rerun) *n_rerun = n;
     if (n == 0) return CT_OK;
-    CUDA_TRY(cudaMemcpyAsync(m->re_idx, m->h_idx, sizeof(int32_t) * n, cudaMemcpyHostToDevice, st));
+    // the re-run batch is padded to a power of two by repeating the last
+    // flagged image; only the first n rows are scattered back
+    int bucket = 1;
+    while (bucket < n) bucket <<= 1;
+    if (bucket > m->max_batch) bucket = n;
+    for (int i = n; i < bucket; ++i) m->h_idx[i] = m->h_idx[n - 1];
+    CUDA_TRY(cudaMemcpyAsync(m->re_idx, m->h_idx, sizeof(int32_t) * bucket, cudaMemcpyHostToDevice, st));
     const int64_t per = (int64_t)m->in_c * m->in_h * m->in_w;
-    CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] { return launch_gather_images(input, m->re_input, m->re_idx, n, per, st); }));
+    CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] { return launch_gather_images(input, m->re_input, m->re_idx, bucket, per, st); }));
     // fault-free re-run: an armed fault stays armed for the next ct_infer
     const bool armed = m->armed;
     m->armed = false;
-    ct_status s = infer_impl(m, m->re_input, n, m->re_logits, m->re_S, m->re_flag, st);
+    ct_status s = CT_OK;
+    cudaGraphExec_t ex = m->prof ? nullptr : reexec_graph(m, bucket);
+    if (ex) {
+        int slot = 0;
+        while ((1 << slot) < bucket) ++slot;
+        if (cudaGraphLaunch(ex, st) != cudaSuccess) s = CT_ECUDA;
+        else m->kernels_total += m->re_graph_nk[slot];
+    } else {
+        s = infer_impl(m, m->re_input, bucket, m->re_logits, m->re_S, m->re_flag, st);
+    }
     m->armed = armed;
     if (s != CT_OK) return s;
     CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] { return launch_scatter_rows(m->re_logits, logits, m->re_idx, n, m->n_classes, st); }));
@@ -859,7 +948,7 @@ ct_status ct_profile_read(ct_model *m, int32_t family, int64_t *launches, double
         CUDA_TRY(cudaEventElapsedTime(&e, m->ev_pool[r.ev].first, m->ev_pool[r.ev].second));
         t += e;
         f += r.flops;
-        ++n;
+        n += r.nk;
         m->ev_free.push_back(r.ev);
     }
     m->recs.swap(keep);
@@ -869,8 +958,16 @@ ct_status ct_profile_read(ct_model *m, int32_t family, int64_t *launches, double
     return CT_OK;
 }
 
+ct_status ct_kernel_count(ct_model *m, int64_t *n) {
+    if (!m || !n) return CT_EINVAL;
+    *n = m->kernels_total;
+    m->kernels_total = 0;
+    return CT_OK;
+}
+
 ct_status ct_launches_per_infer(const ct_model *m, int32_t *n) {
     if (!m || !n) return CT_EINVAL;
+    if (m->n_kernels_last >= 0) { *n = m->n_kernels_last; return CT_OK; }
     int cnt = m->slots[0].stored ? 1 : 0;
     for (auto &l : m->L) cnt += l.fused ? 0 : 1;
     *n = cnt;

@@ -40,6 +40,8 @@ struct ConvArgs {
     uint32_t *err;        // device error word
     int cs_rowsum;        // > 0: an FC layer run as a 1x1 convolution; its checksum input
                           // is the sum of cs_in[m * cs_rowsum .. m * cs_rowsum + cs_rowsum)
+    float *ws;            // split-K workspace (null: never split)
+    size_t ws_bytes;
 };
 
 struct FcArgs {
@@ -66,8 +68,16 @@ struct PoolArgs {
 enum Family { FAM_TC = 0, FAM_SIMT = 1, FAM_FC = 2, FAM_POOL = 3, FAM_OTHER = 4, FAM_COUNT = 5 };
 
 // kernel launchers; each returns cudaGetLastError()
-cudaError_t launch_conv_simt(const ConvArgs &a, bool half, cudaStream_t st);
-cudaError_t launch_conv_tc(const ConvArgs &a, const void *tc_plan, cudaStream_t st);
+// conv launchers report in *n_kernels (may be null) how many kernels they
+// launched: 2 when K is split (the conv kernel and the split-K reduction)
+cudaError_t launch_conv_simt(const ConvArgs &a, bool half, cudaStream_t st, int *n_kernels);
+cudaError_t launch_conv_tc(const ConvArgs &a, const void *tc_plan, cudaStream_t st, int *n_kernels);
+// Split-K: number of K splits for `tiles` output tiles over n_kblocks K
+// blocks (1 = no split); partial sums [splits][M][ws_ld] must fit ws_bytes.
+int splitk_choose(int tiles, int n_kblocks, int min_kb_per_split, int target_ctas, int M, int ws_ld,
+                  size_t ws_bytes);
+// Adds the partials in a.ws and applies the conv epilogue (data and checksum).
+cudaError_t launch_splitk_reduce(const ConvArgs &a, int splits, int ws_ld, bool half, cudaStream_t st);
 cudaError_t launch_fc(const FcArgs &a, bool half, bool x_float, cudaStream_t st);
 cudaError_t launch_maxpool(const PoolArgs &a, bool half, cudaStream_t st);
 cudaError_t launch_gap(const PoolArgs &a, bool half, cudaStream_t st);

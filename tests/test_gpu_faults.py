@@ -124,8 +124,15 @@ def test_reexecute_restores_flagged_rows():
     assert flags[5] == 1 and flags.sum() == 1, flags
     n = ct().ct_reexecute(m, xd, 16, fl, lg, S)
     assert n == 1
-    assert np.array_equal(lg.cpu().numpy(), g_lg.astype(np.float32))
-    assert np.array_equal(S.cpu().numpy(), g_S.astype(np.float32))
+    # rows of unflagged images are untouched; the re-run row is a fault-free
+    # result (a batch of one image may split K differently, so it equals the
+    # batch-16 row up to summation order)
+    lgn, Sn = lg.cpu().numpy(), S.cpu().numpy()
+    keep = [i for i in range(16) if i != 5]
+    assert np.array_equal(lgn[keep], g_lg[keep].astype(np.float32))
+    assert np.array_equal(Sn[keep], g_S[keep].astype(np.float32))
+    assert rel_err_rows(lgn[5], g_lg[5])[0] <= 1e-5
+    assert abs(Sn[5] - g_S[5]) <= 1e-5 * abs(g_S[5])
 
 
 def test_run_host_matches_device_path():
