@@ -124,28 +124,98 @@ __device__ __forceinline__ void store_chunk(const float *v, const ConvArgs &a, i
     yp[1] = make_uint4(packed[4], packed[5], packed[6], packed[7]);
 }
 
+// Residual of 16 channels of one pixel, loaded before the accumulator is
+// ready so that its memory latency overlaps the MMAs.
+struct Res16 {
+    uint4 r0, r1;
+};
+__device__ __forceinline__ Res16 load_res16(const ConvArgs &a, int K, size_t m, int k0) {
+    Res16 r;
+    if (a.res) {
+        const uint4 *rp = reinterpret_cast<const uint4 *>(static_cast<const __half *>(a.res) + m * K + k0);
+        r.r0 = rp[0];
+        r.r1 = rp[1];
+    } else {
+        r.r0 = r.r1 = make_uint4(0u, 0u, 0u, 0u);
+    }
+    return r;
+}
+
+// store_chunk with the residual already loaded
+__device__ __forceinline__ void store_chunk_pre(const float *v, const Res16 &r, const ConvArgs &a, int K, size_t m,
+                                                int k0, float fsrc) {
+    float rv[16];
+    {
+        const __half2 *h0 = reinterpret_cast<const __half2 *>(&r.r0);
+        const __half2 *h1 = reinterpret_cast<const __half2 *>(&r.r1);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            float2 f0 = __half22float2(h0[i]), f1 = __half22float2(h1[i]);
+            rv[2 * i] = f0.x; rv[2 * i + 1] = f0.y; rv[8 + 2 * i] = f1.x; rv[8 + 2 * i + 1] = f1.y;
+        }
+    }
+    const bool res = a.res != nullptr;
+    const FaultDelta &fd = a.fd;
+    uint32_t packed[8];
+#pragma unroll
+    for (int i = 0; i < 16; i += 2) {
+        float o[2];
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+            const int k = k0 + i + j;
+            float t = v[i + j] + __ldg(a.bias + k);
+            if (fd.active && fd.kout == k) t += fd.dv * fsrc;
+            if (res) t += rv[i + j];
+            if (a.relu) t = relu_keep_nan(t);
+            o[j] = t;
+        }
+        __half2 hh = __floats2half2_rn(o[0], o[1]);
+        packed[i / 2] = *reinterpret_cast<uint32_t *>(&hh);
+    }
+    uint4 *yp = reinterpret_cast<uint4 *>(static_cast<__half *>(a.y) + m * K + k0);
+    yp[0] = make_uint4(packed[0], packed[1], packed[2], packed[3]);
+    yp[1] = make_uint4(packed[4], packed[5], packed[6], packed[7]);
+}
+
 // The checksum output of one pixel: carry-through column + coef * incoming
 // checksum (centre pixel, or the sum of an FC layer's checksum features),
 // fault delta, residual checksum, ReLU.
-__device__ __forceinline__ void store_checksum(float ctv, const ConvArgs &a, const TcGeom &g, int m, int nimg,
-                                               int p, int q, float fsrc) {
+// Inputs of a checksum output other than the carry-through column: the
+// incoming checksum at the centre pixel (or the sum of an FC layer's
+// checksum features) and the residual checksum.  Loaded before the
+// accumulator is ready so that their latency overlaps the MMAs.
+struct CsIn {
+    float cin, rcs;
+};
+__device__ __forceinline__ CsIn load_cs_inputs(const ConvArgs &a, const TcGeom &g, int m, int nimg, int p, int q) {
+    CsIn c{0.f, 0.f};
     const __half *csi = static_cast<const __half *>(a.cs_in);
     const int ctr_r = g.ctr_tap / g.S, ctr_s = g.ctr_tap % g.S;
     const int hc = p * g.stride + ctr_r - g.pad, wc = q * g.stride + ctr_s - g.pad;
     const bool inb = hc >= 0 && hc < a.H && wc >= 0 && wc < a.W;
-    float cin = 0.f;
     if (csi && a.cs_rowsum > 0) {                  // FC layer: every incoming checksum feature
-        for (int i = 0; i < a.cs_rowsum; ++i) cin += ldh(csi, (size_t)m * a.cs_rowsum + i);
+        for (int i = 0; i < a.cs_rowsum; ++i) c.cin += ldh(csi, (size_t)m * a.cs_rowsum + i);
     } else if (csi && inb) {
-        cin = ldh(csi, ((size_t)nimg * a.H + hc) * a.W + wc);
+        c.cin = ldh(csi, ((size_t)nimg * a.H + hc) * a.W + wc);
     }
+    if (a.res_cs) c.rcs = ldh(static_cast<const __half *>(a.res_cs), (size_t)m);
+    return c;
+}
+
+__device__ __forceinline__ void store_checksum_pre(float ctv, const CsIn &c, const ConvArgs &a, const TcGeom &g,
+                                                   int m, float fsrc) {
     float o = 0.f;
-    if (a.role == CT_ROLE_CT) o = ctv + a.coef * cin;
-    else if (a.role == CT_ROLE_PASS) o = cin;
+    if (a.role == CT_ROLE_CT) o = ctv + a.coef * c.cin;
+    else if (a.role == CT_ROLE_PASS) o = c.cin;
     if (a.fd.active && a.fd.kout == g.K) o += a.fd.dv * fsrc;
-    if (a.res_cs) o += ldh(static_cast<const __half *>(a.res_cs), (size_t)m);
+    if (a.res_cs) o += c.rcs;
     if (a.relu) o = relu_keep_nan(o);
     static_cast<__half *>(a.cs_out)[m] = __float2half_rn(o);
+}
+
+__device__ __forceinline__ void store_checksum(float ctv, const ConvArgs &a, const TcGeom &g, int m, int nimg,
+                                               int p, int q, float fsrc) {
+    store_checksum_pre(ctv, load_cs_inputs(a, g, m, nimg, p, q), a, g, m, fsrc);
 }
 
 // K-block kb accumulates into chain kb % NCH: back-to-back MMAs into one
@@ -318,6 +388,24 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
         for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++lt) {
             const TileRef tr = tile_ref(tile, g);
             const int m0 = tr.m0, n_tile = tr.n_tile;
+            // residual loads in flight while the MMAs run
+            Res16 rs[BN / 32];
+            {
+                const int mp = m0 + row;
+#pragma unroll
+                for (int c = 0; c < BN / 32; ++c)
+                    rs[c] = (mp < g.M && g.splits == 1)
+                                ? load_res16(a, g.K, (size_t)mp, n_tile * BN + half * (BN / 2) + 16 * c)
+                                : Res16{make_uint4(0u, 0u, 0u, 0u), make_uint4(0u, 0u, 0u, 0u)};
+            }
+            CsIn csv{0.f, 0.f};
+            {
+                const int mp = m0 + row;
+                if (half == 0 && a.cs_out != nullptr && n_tile == 0 && mp < g.M && g.splits == 1) {
+                    const int ni = mp / g.PQ, rm = mp % g.PQ;
+                    csv = load_cs_inputs(a, g, mp, ni, rm / g.Q, rm % g.Q);
+                }
+            }
             const int chains = min(NCH, tr.kb_hi - tr.kb_lo);                    // chains that received MMAs
             // chains whose first K block is a centre block hold a carry-through column
             const int ct_chains = max(0, min(NCH, min(g.cpb, tr.kb_hi) - tr.kb_lo));
@@ -368,11 +456,11 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
                 } else if (valid) {
 #pragma unroll
                     for (int c = 0; c < BN / 2; c += 16)
-                        store_chunk(vals + c, a, g.K, (size_t)m, n0 + half * (BN / 2) + c, fsrc);
-                    if (do_cs) store_checksum(ctv, a, g, m, nimg, p, q, fsrc);
+                        store_chunk_pre(vals + c, rs[c / 16], a, g.K, (size_t)m, n0 + half * (BN / 2) + c, fsrc);
+                    if (do_cs) store_checksum_pre(ctv, csv, a, g, m, fsrc);
                 }
             } else {
-#pragma unroll 1
+#pragma unroll
                 for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 16) {
                     float v[16];
                     tmem_ld16(trow + c, v);
@@ -387,13 +475,13 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
 #pragma unroll
                         for (int i = 0; i < 4; ++i) wp[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
                     } else if (valid) {
-                        store_chunk(v, a, g.K, (size_t)m, n0 + c, fsrc);
+                        store_chunk_pre(v, rs[(c - half * (BN / 2)) / 16], a, g.K, (size_t)m, n0 + c, fsrc);
                     }
                 }
                 if (do_cs && g.ct_mode != CT_NONE_)
                     for (int ch = 0; ch < ct_chains; ++ch) ctv += tmem_ld1(trow + ch * CH + BN);
                 if (do_cs && valid && split) a.ws[((size_t)tr.sp * g.M + m) * g.ws_ld + g.K] = ctv;
-                else if (do_cs && valid) store_checksum(ctv, a, g, m, nimg, p, q, fsrc);
+                else if (do_cs && valid) store_checksum_pre(ctv, csv, a, g, m, fsrc);
                 asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
                 __syncwarp();
                 if (lane == 0) mbar_arrive(smem_u32(acc_empty));
@@ -622,6 +710,286 @@ conv_tc_small_kernel(const __grid_constant__ CUtensorMap bmap, const ConvArgs a,
 }
 
 // ---------------------------------------------------------------------------
+// Stride-1 3x3 convolutions from a halo tile.  An output tile of 16 rows x
+// 8 columns (M = 128) needs an 18 x 10 pixel patch of its input; one tiled
+// TMA per 64-channel block copies it to shared memory (128-byte rows,
+// 128-byte swizzle, zero fill outside the image), and the nine taps are
+// nine views of that patch: the A descriptor of tap (r, s) starts r patch
+// rows and s pixels into it, and its 8-row groups (one output row each) are
+// one patch row (1280 bytes) apart.  The 128-byte swizzle follows the
+// absolute shared-memory address, so shifted starts read the rows the TMA
+// wrote.  Each input pixel thus crosses L2 -> SM once per tile instead of
+// once per tap (im2col).  B (64 x BN per tap and channel block) streams
+// through its own ring, or stays resident for the whole kernel when the
+// layer has one channel block and one N tile (C = K = 64).  The
+// carry-through row is merged into the centre tap's MMAs as in
+// conv_tc_kernel; two TMEM accumulators alternate between tiles.
+// ---------------------------------------------------------------------------
+constexpr int HT_TH = 16, HT_TW = 8;                    // output tile
+constexpr int HT_PH = HT_TH + 2, HT_PW = HT_TW + 2;     // input patch with a one-pixel halo
+constexpr int HT_A_BYTES = HT_PH * HT_PW * BK * 2;      // 23040
+constexpr int HT_A_STAGE = 23 * 1024;                   // stage pitch (1024-byte aligned)
+constexpr int HT_ROW = HT_PW * BK * 2;                  // 1280: one patch row, the A group stride
+
+struct HaloGeom {
+    int N, H, W, C, K;
+    int ncb, n_tiles, ty_tiles, tx_tiles;
+    int ct;
+    int tmem_cols;
+    uint16_t coef_h;
+};
+
+__device__ __forceinline__ uint64_t smem_desc_sw128_sbo(uint32_t addr, uint32_t sbo) {
+    uint64_t d = 0;
+    d |= (uint64_t)((addr >> 4) & 0x3FFF);
+    d |= (uint64_t)1 << 16;
+    d |= (uint64_t)((sbo >> 4) & 0x3FFF) << 32;
+    d |= (uint64_t)1 << 46;
+    d |= (uint64_t)2 << 61;
+    return d;
+}
+
+__device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap *map, uint32_t bar, int c, int x,
+                                            int y, int n) {
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(dst),
+        "l"((uint64_t)map), "r"(c), "r"(x), "r"(y), "r"(n), "r"(bar)
+        : "memory");
+}
+
+struct HaloTile {
+    int n, y0, x0, nt;
+};
+__device__ __forceinline__ HaloTile halo_tile(int t, const HaloGeom &hg) {
+    HaloTile h;
+    h.nt = t % hg.n_tiles;
+    const int r1 = t / hg.n_tiles;
+    h.x0 = (r1 % hg.tx_tiles) * HT_TW;
+    const int r2 = r1 / hg.tx_tiles;
+    h.y0 = (r2 % hg.ty_tiles) * HT_TH;
+    h.n = r2 / hg.ty_tiles;
+    return h;
+}
+
+template <int BN, bool BRES, int NA, int NB>
+__global__ void __launch_bounds__(NTHREADS, 1)
+conv_tc_halo_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
+                    const ConvArgs a, const HaloGeom hg, const TcGeom g) {
+    constexpr int B_ROWS = BN + 16;                       // 16 constant carry-through rows
+    constexpr int B_STAGE = B_ROWS * BK * 2;
+    constexpr int B_TMA = BN * BK * 2;
+    constexpr int NBS = BRES ? 9 : NB;
+    constexpr int CH = BN + 16;
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint8_t *As = smem;
+    uint8_t *Bs = As + NA * HT_A_STAGE;
+    uint64_t *a_full = (uint64_t *)(Bs + NBS * B_STAGE);
+    uint64_t *a_empty = a_full + NA;
+    uint64_t *b_full = a_empty + NA;
+    uint64_t *b_empty = b_full + NBS;
+    uint64_t *acc_full = b_empty + NBS;
+    uint64_t *acc_empty = acc_full + 2;
+    uint32_t *tmem_holder = (uint32_t *)(acc_empty + 2);
+    volatile uint32_t *abort_flag = tmem_holder + 1;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int num_tiles = hg.N * hg.ty_tiles * hg.tx_tiles * hg.n_tiles;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < NA; ++s) {
+            mbar_init(smem_u32(&a_full[s]), 1);
+            mbar_init(smem_u32(&a_empty[s]), 1);
+        }
+        for (int s = 0; s < NBS; ++s) {
+            mbar_init(smem_u32(&b_full[s]), 1);
+            mbar_init(smem_u32(&b_empty[s]), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(smem_u32(&acc_full[b]), 1);
+            mbar_init(smem_u32(&acc_empty[b]), N_EPI_WARPS);
+        }
+        *abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_holder)),
+                     "r"((uint32_t)hg.tmem_cols));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    if (warp >= 2) {
+        // constant carry-through rows after the BN weight rows of every B stage:
+        // row 0 = coef, rows 1..15 = 0 (swizzle-invariant)
+        const uint32_t coef2 = (uint32_t)hg.coef_h | ((uint32_t)hg.coef_h << 16);
+        const int t = threadIdx.x - 64;
+        for (int sb = 0; sb < NBS; ++sb) {
+            uint32_t *rows = (uint32_t *)(Bs + sb * B_STAGE + BN * BK * 2);
+            for (int i = t; i < 16 * BK / 2; i += 32 * N_EPI_WARPS) rows[i] = (i < BK / 2) ? coef2 : 0u;
+        }
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tmem = *tmem_holder;
+
+    if (warp == 0) {
+        // ---------------- TMA producer (whole warp, one lane issues) ----------------
+        if (elect_one()) {
+            asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&amap) : "memory");
+            asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&bmap) : "memory");
+            if (BRES) {
+                for (int i = 0; i < 9; ++i) {
+                    mbar_arrive_expect_tx(smem_u32(&b_full[i]), B_TMA);
+                    tma_load_2d(smem_u32(Bs + i * B_STAGE), &bmap, smem_u32(&b_full[i]), tap_of(i, 4) * hg.C, 0);
+                }
+            }
+        }
+        __syncwarp();
+        int ai = 0, bi = 0;
+        bool ok = true;
+        for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
+            if (__any_sync(0xffffffffu, *abort_flag)) break;
+            const HaloTile ht = halo_tile(tile, hg);
+            for (int cb = 0; cb < hg.ncb && ok; ++cb) {
+                const int as = ai % NA;
+                if (!warp_wait(smem_u32(&a_empty[as]), ((uint32_t)(ai / NA) & 1u) ^ 1u, a.err, 1u)) { ok = false; break; }
+                if (elect_one()) {
+                    mbar_arrive_expect_tx(smem_u32(&a_full[as]), HT_A_BYTES);
+                    tma_load_4d(smem_u32(As + as * HT_A_STAGE), &amap, smem_u32(&a_full[as]), cb * BK, ht.x0 - 1,
+                                ht.y0 - 1, ht.n);
+                }
+                __syncwarp();
+                ++ai;
+                if (!BRES) {
+                    for (int i = 0; i < 9; ++i) {
+                        const int bs = bi % NBS;
+                        if (!warp_wait(smem_u32(&b_empty[bs]), ((uint32_t)(bi / NBS) & 1u) ^ 1u, a.err, 1u)) {
+                            ok = false;
+                            break;
+                        }
+                        if (elect_one()) {
+                            mbar_arrive_expect_tx(smem_u32(&b_full[bs]), B_TMA);
+                            tma_load_2d(smem_u32(Bs + bs * B_STAGE), &bmap, smem_u32(&b_full[bs]),
+                                        tap_of(i, 4) * hg.C + cb * BK, ht.nt * BN);
+                        }
+                        __syncwarp();
+                        ++bi;
+                    }
+                }
+            }
+        }
+        if (!ok && lane == 0) *abort_flag = 1;
+    } else if (warp == 1) {
+        // ---------------- MMA issuer (whole warp, one lane issues) ----------------
+        const uint32_t id_main = idesc_f16(BM, BN);
+        const uint32_t id_merged = idesc_f16(BM, BN + 16);
+        int ai = 0, bi = 0, lt = 0;
+        bool ok = true;
+        for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x, ++lt) {
+            if (__any_sync(0xffffffffu, *abort_flag)) break;
+            const HaloTile ht = halo_tile(tile, hg);
+            const bool ct_here = hg.ct && ht.nt == 0;
+            const int ab = lt & 1;
+            if (!warp_wait(smem_u32(&acc_empty[ab]), ((uint32_t)(lt >> 1) & 1u) ^ 1u, a.err, 8u)) { ok = false; break; }
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            const uint32_t d = tmem + (uint32_t)(ab * CH);
+            for (int cb = 0; cb < hg.ncb && ok; ++cb) {
+                const int as = ai % NA;
+                if (!warp_wait(smem_u32(&a_full[as]), (uint32_t)(ai / NA) & 1u, a.err, 2u)) { ok = false; break; }
+                const uint32_t a_base = smem_u32(As + as * HT_A_STAGE);
+                for (int i = 0; i < 9; ++i) {
+                    const int bs = BRES ? i : bi % NBS;
+                    const uint32_t bph = BRES ? 0u : (uint32_t)(bi / NBS) & 1u;
+                    if (!warp_wait(smem_u32(&b_full[bs]), bph, a.err, 2u)) { ok = false; break; }
+                    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                    const int tap = tap_of(i, 4);
+                    const uint32_t a_tap = a_base + (uint32_t)(((tap / 3) * HT_PW + tap % 3) * BK * 2);
+                    const uint32_t b_base = smem_u32(Bs + bs * B_STAGE);
+                    const bool merged = ct_here && i == 0;
+                    if (elect_one()) {
+#pragma unroll
+                        for (int k16 = 0; k16 < BK / 16; ++k16) {
+                            const uint64_t ad = smem_desc_sw128_sbo(a_tap + k16 * 32, HT_ROW);
+                            const uint64_t bd = smem_desc_sw128(b_base + k16 * 32);
+                            const uint32_t acc = (cb > 0 || i > 0 || k16 > 0) ? 1u : 0u;
+                            umma_f16(d, ad, bd, merged ? id_merged : id_main, acc);
+                        }
+                        if (!BRES) umma_commit(smem_u32(&b_empty[bs]));
+                    }
+                    __syncwarp();
+                    if (!BRES) ++bi;
+                }
+                if (!ok) break;
+                if (elect_one()) umma_commit(smem_u32(&a_empty[as]));
+                __syncwarp();
+                ++ai;
+            }
+            if (!ok) break;
+            if (elect_one()) umma_commit(smem_u32(&acc_full[ab]));   // fires when the tile's MMAs have completed
+            __syncwarp();
+        }
+        if (!ok && lane == 0) *abort_flag = 1;
+    } else {
+        // ---------------- epilogue: warps 2..9 ----------------
+        const int ep = warp - 2;
+        const int quad = warp & 3;
+        const int half = ep >> 2;
+        const int row = quad * 32 + lane;
+        const __half *x = static_cast<const __half *>(a.x);
+        const FaultDelta fd = a.fd;
+        int lt = 0;
+        for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++lt) {
+            const HaloTile ht = halo_tile(tile, hg);
+            const int ab = lt & 1;
+            const int p = ht.y0 + row / HT_TW, q = ht.x0 + row % HT_TW;
+            const bool valid = p < hg.H && q < hg.W;
+            const int m = valid ? (ht.n * hg.H + p) * hg.W + q : 0;
+            const int n0 = ht.nt * BN + half * (BN / 2);
+            // residual loads in flight while the MMAs run
+            Res16 rs[BN / 32];
+#pragma unroll
+            for (int c = 0; c < BN / 32; ++c)
+                rs[c] = valid ? load_res16(a, hg.K, (size_t)m, n0 + 16 * c) : Res16{make_uint4(0u, 0u, 0u, 0u), make_uint4(0u, 0u, 0u, 0u)};
+            const bool do_cs = half == 0 && a.cs_out != nullptr && ht.nt == 0;
+            const CsIn csv = (do_cs && valid) ? load_cs_inputs(a, g, m, ht.n, p, q) : CsIn{0.f, 0.f};
+            bool ok = mbar_wait(smem_u32(&acc_full[ab]), (uint32_t)(lt >> 1) & 1u, a.err, 4u) && !*abort_flag;
+            ok = __all_sync(0xffffffffu, ok);
+            if (!ok) break;
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            const uint32_t trow = tmem + (uint32_t)(ab * CH) + ((uint32_t)(quad * 32) << 16);
+            float vals[BN / 2];
+#pragma unroll
+            for (int c = 0; c < BN / 2; c += 16) tmem_ld16(trow + half * (BN / 2) + c, vals + c);
+            const float ctv = (do_cs && hg.ct) ? tmem_ld1(trow + BN) : 0.f;
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&acc_empty[ab]));
+            if (valid) {
+                float fsrc = 0.f;
+                if (fd.active) {
+                    const int h = p + fd.r - 1, w = q + fd.s - 1;
+                    if (h >= 0 && h < hg.H && w >= 0 && w < hg.W) {
+                        if (fd.cin < hg.C) fsrc = ldh(x, (((size_t)ht.n * hg.H + h) * hg.W + w) * hg.C + fd.cin);
+                        else if (a.cs_in) fsrc = ldh(static_cast<const __half *>(a.cs_in), ((size_t)ht.n * hg.H + h) * hg.W + w);
+                    }
+                }
+#pragma unroll
+                for (int c = 0; c < BN / 2; c += 16) store_chunk_pre(vals + c, rs[c / 16], a, hg.K, (size_t)m, n0 + c, fsrc);
+                if (do_cs) store_checksum_pre(ctv, csv, a, g, m, fsrc);
+            }
+        }
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if (warp == 1) {
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)hg.tmem_cols));
+    }
+}
+
+// ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
 
@@ -819,5 +1187,103 @@ cudaError_t launch_conv_tc_small(const ConvArgs &a, const TcSmallPlan *pl, cudaS
 }
 
 void tc_plan_destroy(TcPlan *p) { delete p; }
+
+// ---------------------------------------------------------------------------
+// halo-tile plans
+// ---------------------------------------------------------------------------
+struct HaloPlan {
+    CUtensorMap amap;
+    CUtensorMap bmap;
+    HaloGeom hg;
+    TcGeom g;
+    int BN, kind, sms;
+    size_t smem;
+};
+
+template <int BN, bool BRES, int NA, int NB>
+size_t halo_smem() {
+    const int nbs = BRES ? 9 : NB;
+    return 1024 + (size_t)NA * HT_A_STAGE + (size_t)nbs * (BN + 16) * BK * 2 + 8 * (2 * NA + 2 * nbs + 4) + 16;
+}
+
+// Tiles that overhang the image waste MMA rows: require whole 8-column tiles
+// and at most one partly filled row of tiles on a tall image.
+bool halo_supported(int C, int K, int R, int S, int stride, int pad, int H, int W) {
+    return R == 3 && S == 3 && stride == 1 && pad == 1 && C % BK == 0 && (K == 64 || K == 128) && W % HT_TW == 0 &&
+           (H % HT_TH == 0 || H >= 3 * HT_TH);
+}
+
+HaloPlan *halo_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, const void *x_dev, std::string *why) {
+    if (!halo_supported(a.C, a.K, a.R, a.S, a.stride, a.pad, a.H, a.W)) { if (why) *why = "shape"; return nullptr; }
+    if (!load_encoders()) { if (why) *why = "tensor-map encoders unavailable"; return nullptr; }
+    HaloPlan *pl = new HaloPlan();
+    memset(pl, 0, sizeof(*pl));
+    pl->BN = a.K;
+    pl->sms = sm_count();
+    HaloGeom &hg = pl->hg;
+    hg.H = a.H; hg.W = a.W; hg.C = a.C; hg.K = a.K;
+    hg.ncb = a.C / BK;
+    hg.n_tiles = 1;
+    hg.ty_tiles = (a.H + HT_TH - 1) / HT_TH;
+    hg.tx_tiles = (a.W + HT_TW - 1) / HT_TW;
+    hg.ct = a.role == CT_ROLE_CT ? 1 : 0;
+    hg.tmem_cols = 2 * (pl->BN + 16) <= 256 ? 256 : 512;
+    hg.coef_h = coef_half_bits(a.coef);
+    // geometry the shared epilogue helpers read
+    TcGeom &g = pl->g;
+    g.PQ = a.P * a.Q; g.Q = a.Q; g.stride = 1; g.pad = 1; g.C = a.C; g.K = a.K; g.S = 3; g.ctr_tap = 4;
+    // A: the NHWC input [max_batch, H, W, C] as tiles of 64 channels x 10 x 18 pixels
+    cuuint64_t gdim[4] = {(cuuint64_t)a.C, (cuuint64_t)a.W, (cuuint64_t)a.H, (cuuint64_t)max_batch};
+    cuuint64_t gstr[3] = {(cuuint64_t)a.C * 2, (cuuint64_t)a.W * a.C * 2, (cuuint64_t)a.H * a.W * a.C * 2};
+    cuuint32_t abox[4] = {BK, HT_PW, HT_PH, 1};
+    cuuint32_t aes[4] = {1, 1, 1, 1};
+    CUresult r = g_encode_tiled(&pl->amap, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<void *>(x_dev), gdim, gstr,
+                                abox, aes, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                                CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) { if (why) *why = "patch tensor map"; delete pl; return nullptr; }
+    const int RSC = 9 * a.C;
+    cuuint64_t bdim[2] = {(cuuint64_t)RSC, (cuuint64_t)a.K};
+    cuuint64_t bstr[1] = {(cuuint64_t)RSC * 2};
+    cuuint32_t box[2] = {BK, (cuuint32_t)pl->BN};
+    cuuint32_t bes[2] = {1, 1};
+    r = g_encode_tiled(&pl->bmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void *>(w_dev), bdim, bstr, box, bes,
+                       CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                       CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) { if (why) *why = "weight tensor map"; delete pl; return nullptr; }
+    cudaError_t e;
+    if (pl->BN == 64 && hg.ncb == 1) {
+        pl->kind = 0;
+        pl->smem = halo_smem<64, true, 4, 0>();
+        e = cudaFuncSetAttribute(conv_tc_halo_kernel<64, true, 4, 0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
+    } else if (pl->BN == 64) {
+        pl->kind = 1;
+        pl->smem = halo_smem<64, false, 4, 8>();
+        e = cudaFuncSetAttribute(conv_tc_halo_kernel<64, false, 4, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
+    } else {
+        pl->kind = 2;
+        pl->smem = halo_smem<128, false, 3, 6>();
+        e = cudaFuncSetAttribute(conv_tc_halo_kernel<128, false, 3, 6>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
+    }
+    if (e != cudaSuccess) { cudaGetLastError(); if (why) *why = "shared memory attribute"; delete pl; return nullptr; }
+    return pl;
+}
+
+int halo_tiles(const HaloPlan *pl, int batch) { return batch * pl->hg.ty_tiles * pl->hg.tx_tiles * pl->hg.n_tiles; }
+int halo_sms(const HaloPlan *pl) { return pl->sms; }
+
+cudaError_t launch_conv_tc_halo(const ConvArgs &a, const HaloPlan *pl, cudaStream_t st) {
+    HaloGeom hg = pl->hg;
+    hg.N = a.N;
+    TcGeom g = pl->g;
+    g.M = a.N * a.P * a.Q;
+    const int tiles = halo_tiles(pl, a.N);
+    dim3 grid(tiles < pl->sms ? tiles : pl->sms);
+    if (pl->kind == 0) conv_tc_halo_kernel<64, true, 4, 0><<<grid, NTHREADS, pl->smem, st>>>(pl->amap, pl->bmap, a, hg, g);
+    else if (pl->kind == 1) conv_tc_halo_kernel<64, false, 4, 8><<<grid, NTHREADS, pl->smem, st>>>(pl->amap, pl->bmap, a, hg, g);
+    else conv_tc_halo_kernel<128, false, 3, 6><<<grid, NTHREADS, pl->smem, st>>>(pl->amap, pl->bmap, a, hg, g);
+    return cudaGetLastError();
+}
+
+void halo_plan_destroy(HaloPlan *p) { delete p; }
 
 }  // namespace ct

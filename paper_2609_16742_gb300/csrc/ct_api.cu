@@ -92,6 +92,7 @@ struct LayerRT {
     float *bias = nullptr;
     bool tc = false;
     TcPlan *plan = nullptr;
+    HaloPlan *hplan = nullptr;   // stride-1 3x3 layers: halo tiles when the batch fills the GPU
     bool tc_small = false;       // first layer with <= 4 input channels on the tensor cores
     TcSmallPlan *splan = nullptr;
     bool stem = false;           // fused image stem: this conv and the max-pool after it
@@ -182,6 +183,7 @@ void free_all(ct_model *m) {
         if (l.plan) tc_plan_destroy(l.plan);
         if (l.splan) tc_small_plan_destroy(l.splan);
         if (l.stplan) stem_plan_destroy(l.stplan);
+        if (l.hplan) halo_plan_destroy(l.hplan);
     }
     for (void *p : m->dev_allocs) cudaFree(p);
     m->dev_allocs.clear();
@@ -460,6 +462,10 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
         std::string why;
         l.plan = tc_plan_create(a, B, l.w, m->slots[l.d.src].data, &why);
         if (!l.plan) return CT_ECUDA;
+        if (halo_supported(l.C, l.K, l.R, l.S, l.d.stride, l.d.pad, l.H, l.W) && m->slots[l.d.src].cp == l.C) {
+            l.hplan = halo_plan_create(a, B, l.w, m->slots[l.d.src].data, &why);
+            if (!l.hplan) return CT_ECUDA;
+        }
     }
     // ---- scratch for re-execution and host runs ----
     const size_t per_img = (size_t)m->in_c * m->in_h * m->in_w;
@@ -596,7 +602,9 @@ ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, 
             } else {
                 a.ws = m->ws; a.ws_bytes = SPLITK_WS_BYTES;
                 int nk = 1;
-                if (l.tc) CUDA_TRY(launch(m, FAM_TC, flops, st, [&] { return launch_conv_tc(a, l.plan, st, &nk); }, &nk));
+                if (l.hplan && halo_tiles(l.hplan, batch) >= halo_sms(l.hplan))
+                    CUDA_TRY(launch(m, FAM_TC, flops, st, [&] { return launch_conv_tc_halo(a, l.hplan, st); }));
+                else if (l.tc) CUDA_TRY(launch(m, FAM_TC, flops, st, [&] { return launch_conv_tc(a, l.plan, st, &nk); }, &nk));
                 else CUDA_TRY(launch(m, FAM_SIMT, flops, st, [&] { return launch_conv_simt(a, half, st, &nk); }, &nk));
             }
             if (wfault && wf.explicit_word) CUDA_TRY(xor_bit(m, l.w, wf.word, m->f_bit, wb, st));
@@ -633,8 +641,10 @@ ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, 
             a.ref = m->ref; a.tau = m->tau;
             if (d.final) { a.y = logits; a.S = S; a.flag = flag; }
             else { a.y = dst.data; a.ycs = dst.has_cs ? dst.cs : nullptr; }
+            a.ws = m->ws; a.ws_bytes = SPLITK_WS_BYTES;
             const double flops = 2.0 * batch * (double)l.n_in * l.n_out;
-            CUDA_TRY(launch(m, FAM_FC, flops, st, [&] { return launch_fc(a, half, l.x_float, st); }));
+            int nk = 1;
+            CUDA_TRY(launch(m, FAM_FC, flops, st, [&] { return launch_fc(a, half, l.x_float, st, &nk); }, &nk));
         }
         if (act_slot == d.dst) CUDA_TRY(xor_bit(m, act_base, act_word, m->f_bit, wb, st));
     }

@@ -57,6 +57,8 @@ struct FcArgs {
     int relu, final_layer, protect;
     float coef;
     double ref, tau;
+    float *ws;            // split-K workspace (null: never split)
+    size_t ws_bytes;
 };
 
 struct PoolArgs {
@@ -78,7 +80,7 @@ int splitk_choose(int tiles, int n_kblocks, int min_kb_per_split, int target_cta
                   size_t ws_bytes);
 // Adds the partials in a.ws and applies the conv epilogue (data and checksum).
 cudaError_t launch_splitk_reduce(const ConvArgs &a, int splits, int ws_ld, bool half, cudaStream_t st);
-cudaError_t launch_fc(const FcArgs &a, bool half, bool x_float, cudaStream_t st);
+cudaError_t launch_fc(const FcArgs &a, bool half, bool x_float, cudaStream_t st, int *n_kernels);
 cudaError_t launch_maxpool(const PoolArgs &a, bool half, cudaStream_t st);
 cudaError_t launch_gap(const PoolArgs &a, bool half, cudaStream_t st);
 cudaError_t launch_convert_input(const float *in, void *out, int N, int C, int Cp, int H, int W, bool half,
@@ -117,6 +119,17 @@ int tc_small_kpad(int R, int S);
 TcSmallPlan *tc_small_plan_create(const ConvArgs &shape_args, const void *w_dev, std::string *why);
 void tc_small_plan_destroy(TcSmallPlan *p);
 cudaError_t launch_conv_tc_small(const ConvArgs &a, const TcSmallPlan *plan, cudaStream_t st);
+
+// Stride-1 3x3 convolution (C a multiple of 64, K = 64 or 128) from halo
+// tiles of 16 x 8 output pixels: one patch load per tile and channel block.
+struct HaloPlan;
+bool halo_supported(int C, int K, int R, int S, int stride, int pad, int H, int W);
+HaloPlan *halo_plan_create(const ConvArgs &shape_args, int max_batch, const void *w_dev, const void *x_dev,
+                           std::string *why);
+void halo_plan_destroy(HaloPlan *p);
+int halo_tiles(const HaloPlan *p, int batch);
+int halo_sms(const HaloPlan *p);
+cudaError_t launch_conv_tc_halo(const ConvArgs &a, const HaloPlan *p, cudaStream_t st);
 
 // Fused image stem (7x7 stride-2 convolution, C <= 4, 64 filters, followed
 // by a 3x3 stride-2 padding-1 max-pool): reads the FP32 NCHW image, writes

@@ -44,17 +44,21 @@ __global__ void __launch_bounds__(256) fc_kernel(FcArgs a) {
 #pragma unroll
     for (int j = 0; j < FC_J; ++j) acc[j][0] = acc[j][1] = 0.f;
 
-    for (int k0 = 0; k0 < a.n_in; k0 += FC_KC) {
+    // K range of this block: all inputs, or one split's range (gridDim.z > 1)
+    const int nkc = (a.n_in + FC_KC - 1) / FC_KC;
+    const int kc_per = (nkc + gridDim.z - 1) / gridDim.z;
+    const int k_lo = blockIdx.z * kc_per * FC_KC, k_hi = min(a.n_in, k_lo + kc_per * FC_KC);
+    for (int k0 = k_lo; k0 < k_hi; k0 += FC_KC) {
         // stage x[b0 .. b0+63][k0 .. k0+63] transposed, and W[j0..j0+15][k0..k0+63]
         for (int e = tid; e < FC_KC * FC_IMG; e += 256) {
             int kk = e % FC_KC, bb = e / FC_KC;
             int b = b0 + bb, k = k0 + kk;
-            Xs[kk * (FC_IMG + 1) + bb] = (b < a.B && k < a.n_in) ? to_f(x[(size_t)b * a.n_in + k]) : 0.f;
+            Xs[kk * (FC_IMG + 1) + bb] = (b < a.B && k < k_hi) ? to_f(x[(size_t)b * a.n_in + k]) : 0.f;
         }
         for (int e = tid; e < FC_KC * FC_J; e += 256) {
             int kk = e % FC_KC, jj = e / FC_KC;
             int j = j0 + jj, k = k0 + kk;
-            Ws[kk * FC_J + jj] = (j < a.n_out && k < a.n_in) ? to_f(w[(size_t)j * a.n_in + k]) : 0.f;
+            Ws[kk * FC_J + jj] = (j < a.n_out && k < k_hi) ? to_f(w[(size_t)j * a.n_in + k]) : 0.f;
         }
         __syncthreads();
 #pragma unroll 2
@@ -86,6 +90,24 @@ __global__ void __launch_bounds__(256) fc_kernel(FcArgs a) {
     red[(warp * (FC_J + 1) + FC_J) * FC_IMG + lane] = act[0];
     red[(warp * (FC_J + 1) + FC_J) * FC_IMG + lane + 32] = act[1];
     __syncthreads();
+    if (gridDim.z > 1) {
+        // split K: FP32 partial sums [z][B][n_out + 1] (column n_out: the
+        // carry-through neuron's sum of data inputs); fc_reduce_kernel finishes
+        const int ldw = a.n_out + 1;
+        float *wz = a.ws + (size_t)blockIdx.z * a.B * ldw;
+        for (int e = tid; e < (FC_J + 1) * FC_IMG; e += 256) {
+            const int jj = e / FC_IMG, bb = e % FC_IMG;
+            const int b = b0 + bb;
+            if (b >= a.B) continue;
+            if (jj == FC_J && !ct_block) continue;
+            const int j = jj == FC_J ? a.n_out : j0 + jj;
+            if (jj < FC_J && j >= a.n_out) continue;
+            float sum = 0.f;
+            for (int wv = 0; wv < FC_WARPS; ++wv) sum += red[(wv * (FC_J + 1) + jj) * FC_IMG + bb];
+            wz[(size_t)b * ldw + j] = sum;
+        }
+        return;
+    }
     for (int e = tid; e < FC_J * FC_IMG; e += 256) {
         int jj = e / FC_IMG, bb = e % FC_IMG;
         int j = j0 + jj, b = b0 + bb;
@@ -113,6 +135,50 @@ __global__ void __launch_bounds__(256) fc_kernel(FcArgs a) {
         if (b >= a.B) continue;
         float s = 0.f;
         for (int wv = 0; wv < FC_WARPS; ++wv) s += red[(wv * (FC_J + 1) + FC_J) * FC_IMG + bb];
+        if (xcs)
+            for (int i = 0; i < a.n_cs; ++i) s += to_f(xcs[(size_t)b * a.n_cs + i]);
+        s *= a.coef;
+        if (a.final_layer) {
+            if (a.S) a.S[b] = s;
+            if (a.flag) a.flag[b] = !(fabs((double)s - a.ref) <= a.tau);
+        } else {
+            if (a.relu) s = relu_keep_nan(s);
+            static_cast<TY *>(a.ycs)[b] = from_f<TY>(s);
+        }
+    }
+}
+
+// Split-K FC: adds the partials in split order, then bias and ReLU (data
+// neurons), and the carry-through / accumulated-checksum neuron:
+// coef * (sum of data inputs + sum of checksum inputs), with the verdict
+// for the final layer.  One thread per (image, neuron), neuron n_out = the
+// checksum neuron.
+template <typename TX, typename TY>
+__global__ void fc_reduce_kernel(FcArgs a, int splits) {
+    const int ldw = a.n_out + 1;
+    const long long total = (long long)a.B * ldw;
+    const size_t plane = (size_t)a.B * ldw;
+    for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
+         e += (long long)gridDim.x * blockDim.x) {
+        const int b = (int)(e / ldw), j = (int)(e % ldw);
+        if (j < a.n_out) {
+            float s = 0.f;
+            for (int z = 0; z < splits; ++z) s += a.ws[z * plane + (size_t)b * ldw + j];
+            s += a.bias[j];
+            if (a.relu) s = relu_keep_nan(s);
+            static_cast<TY *>(a.y)[(size_t)b * a.n_out + j] = from_f<TY>(s);
+            continue;
+        }
+        if (!a.protect) {
+            if (a.final_layer) {
+                if (a.S) a.S[b] = __int_as_float(0x7fc00000);
+                if (a.flag) a.flag[b] = 0;
+            }
+            continue;
+        }
+        float s = 0.f;
+        for (int z = 0; z < splits; ++z) s += a.ws[z * plane + (size_t)b * ldw + j];
+        const TX *xcs = static_cast<const TX *>(a.xcs);
         if (xcs)
             for (int i = 0; i < a.n_cs; ++i) s += to_f(xcs[(size_t)b * a.n_cs + i]);
         s *= a.coef;
@@ -288,7 +354,7 @@ int grid_for(int64_t n, int threads) {
 }
 
 template <typename TX, typename TW, typename TY>
-cudaError_t fc_go(const FcArgs &a, cudaStream_t st) {
+cudaError_t fc_go(const FcArgs &a, cudaStream_t st, int *n_kernels) {
     const size_t smem =
         sizeof(float) * (FC_KC * (FC_IMG + 1) + FC_KC * FC_J + FC_WARPS * (FC_J + 1) * FC_IMG);
     static bool attr = false;
@@ -298,18 +364,30 @@ cudaError_t fc_go(const FcArgs &a, cudaStream_t st) {
         if (e != cudaSuccess) return e;
         attr = true;
     }
-    dim3 grid((a.n_out + FC_J - 1) / FC_J, (a.B + FC_IMG - 1) / FC_IMG);
+    const int gx = (a.n_out + FC_J - 1) / FC_J, gy = (a.B + FC_IMG - 1) / FC_IMG;
+    // split K when the output blocks leave most SMs idle (at least 4 chunks of 64 inputs each)
+    static int sms = 0;
+    if (sms == 0) sms = device_sm_count();
+    const int nkc = (a.n_in + FC_KC - 1) / FC_KC;
+    const int splits = splitk_choose(gx * gy, nkc, 4, 2 * sms, a.B, a.n_out + 1, a.ws ? a.ws_bytes : 0);
+    dim3 grid(gx, gy, splits);
     fc_kernel<TX, TW, TY><<<grid, 256, smem, st>>>(a);
+    cudaError_t e = cudaGetLastError();
+    if (n_kernels) *n_kernels = 1;
+    if (e != cudaSuccess || splits == 1) return e;
+    if (n_kernels) *n_kernels = 2;
+    const long long total = (long long)a.B * (a.n_out + 1);
+    fc_reduce_kernel<TX, TY><<<(int)std::min<long long>((total + 255) / 256, 4096), 256, 0, st>>>(a, splits);
     return cudaGetLastError();
 }
 
 }  // namespace
 
-cudaError_t launch_fc(const FcArgs &a, bool half, bool x_float, cudaStream_t st) {
-    if (!half) return fc_go<float, float, float>(a, st);
+cudaError_t launch_fc(const FcArgs &a, bool half, bool x_float, cudaStream_t st, int *n_kernels) {
+    if (!half) return fc_go<float, float, float>(a, st, n_kernels);
     if (a.final_layer)
-        return x_float ? fc_go<float, __half, float>(a, st) : fc_go<__half, __half, float>(a, st);
-    return x_float ? fc_go<float, __half, __half>(a, st) : fc_go<__half, __half, __half>(a, st);
+        return x_float ? fc_go<float, __half, float>(a, st, n_kernels) : fc_go<__half, __half, float>(a, st, n_kernels);
+    return x_float ? fc_go<float, __half, __half>(a, st, n_kernels) : fc_go<__half, __half, __half>(a, st, n_kernels);
 }
 
 cudaError_t launch_maxpool(const PoolArgs &a, bool half, cudaStream_t st) {

@@ -53,6 +53,10 @@ def layer_errors(name, prec, batch, simt_only=False, first=0):
     ("resnet18_imagenet", "fp16", 2, False),
     ("lenet5", "fp32", 5, False),
     ("vgg16", "fp16", 1, False),
+    # batches whose stride-1 3x3 layers fill the GPU with halo tiles
+    ("resnet18_imagenet", "fp16", 8, False),
+    ("resnet18_cifar", "fp16", 20, False),
+    ("vgg16", "fp16", 2, False),
 ])
 def test_every_stored_tensor_matches_oracle(name, prec, batch, simt_only):
     errs = layer_errors(name, prec, batch, simt_only)
