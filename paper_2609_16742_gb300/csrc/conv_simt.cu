@@ -57,6 +57,8 @@ __device__ __forceinline__ float load_x(const T *x, int n, int h, int w, int c, 
 template <typename T, int BM, int BN, int BK, int TM, int TN, bool VEC>
 __global__ void __launch_bounds__((BM / TM) * (BN / TN))
 conv_simt_kernel(ConvArgs a) {
+    pdl_wait();
+    pdl_trigger();
     constexpr int NT = (BM / TM) * (BN / TN);
     constexpr int VE = Vec<T>::n;                 // elements per 16-byte vector
     constexpr int UPR = VEC ? BK / VE : 1;        // load units per tile row
@@ -327,7 +329,7 @@ cudaError_t go(const ConvArgs &a, cudaStream_t st, int *n_kernels) {
     const int splits = (a.K % 8 == 0) ? splitk_choose(gx * gy, nk, 8, 2 * sm_count_cached(), M, ws_ld,
                                                       a.ws ? a.ws_bytes : 0) : 1;
     dim3 grid(gx, gy, splits);
-    conv_simt_kernel<T, BM, BN, BK, TM, TN, VEC><<<grid, (BM / TM) * (BN / TN), 0, st>>>(a);
+    pdl_launch(conv_simt_kernel<T, BM, BN, BK, TM, TN, VEC>, grid, (BM / TM) * (BN / TN), 0, st, a);
     cudaError_t e = cudaGetLastError();
     if (n_kernels) *n_kernels = 1;
     if (e != cudaSuccess || splits == 1) return e;

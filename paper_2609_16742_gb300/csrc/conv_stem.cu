@@ -34,8 +34,9 @@
 // Warp roles (416 threads): warps 0-3 fill ring rows (entry e goes to warp
 // e % 4), warp 4 allocates TMEM and issues tcgen05.mma (one elected lane),
 // warps 5-12 are the epilogue: each TMEM lane quadrant is read by two warps,
-// each taking 32 of the 64 channels.  Two TMEM accumulators alternate
-// between consecutive convolution rows.  Every mbarrier wait is bounded; on
+// each taking 32 of the 64 channels.  Four TMEM accumulators rotate over
+// consecutive convolution rows, so the MMAs run up to three rows ahead of
+// the epilogue.  Every mbarrier wait is bounded; on
 // expiry the kernel records an error code, stops and frees TMEM.
 #include "ct_internal.h"
 #include "tc_common.cuh"
@@ -61,13 +62,14 @@ constexpr int ST_PIX_H = 72;                 // halves per pixel in the epilogue
 constexpr int ST_THREADS = 416;
 constexpr int ST_EPI0 = 160;                 // first epilogue thread
 constexpr int ST_EPI = 256;                  // epilogue threads
-constexpr int ST_TMEM_COLS = 256;            // two accumulators of 128 columns
+constexpr int ST_NACC = 4;                   // TMEM accumulators (rows in flight between MMA and epilogue)
+constexpr int ST_TMEM_COLS = 128 * ST_NACC;
 
 constexpr size_t ST_OFF_B = (size_t)ST_NSLOT * ST_SLOT_BYTES;
 constexpr size_t ST_OFF_ROW = ST_OFF_B + (size_t)ST_KSTEPS * ST_B_STEP;
 constexpr size_t ST_OFF_CS = ST_OFF_ROW + 2ull * 128 * ST_PIX_H * 2;
 constexpr size_t ST_OFF_BAR = ST_OFF_CS + 2ull * 128 * 2;
-constexpr size_t ST_SMEM = 1024 + ST_OFF_BAR + 8 * (2 * ST_NSLOT + 5) + 16;
+constexpr size_t ST_SMEM = 1024 + ST_OFF_BAR + 8 * (2 * ST_NSLOT + 2 * ST_NACC + 1) + 16;
 
 struct StemGeom {
     int N, C, H, W, P, Q, P2, Q2;
@@ -133,6 +135,8 @@ __device__ __forceinline__ float image_half(const float *x, const StemGeom &g, i
 
 __global__ void __launch_bounds__(ST_THREADS, 1)
 stem_pool_kernel(const ConvArgs a, const StemGeom g) {
+    pdl_wait();
+    pdl_trigger();
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint8_t *ring = smem;
@@ -142,8 +146,8 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
     uint64_t *full = (uint64_t *)(smem + ST_OFF_BAR);
     uint64_t *empty = full + ST_NSLOT;
     uint64_t *acc_full = empty + ST_NSLOT;
-    uint64_t *acc_empty = acc_full + 2;
-    uint64_t *mma_done = acc_empty + 2;
+    uint64_t *acc_empty = acc_full + ST_NACC;
+    uint64_t *mma_done = acc_empty + ST_NACC;
     uint32_t *tmem_holder = (uint32_t *)(mma_done + 1);
     volatile uint32_t *abort_flag = tmem_holder + 1;
 
@@ -187,7 +191,7 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
             mbar_init(smem_u32(&full[s]), 32);
             mbar_init(smem_u32(&empty[s]), 1);
         }
-        for (int b = 0; b < 2; ++b) {
+        for (int b = 0; b < ST_NACC; ++b) {
             mbar_init(smem_u32(&acc_full[b]), 1);
             mbar_init(smem_u32(&acc_empty[b]), ST_EPI / 32);
         }
@@ -270,10 +274,12 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
             StemJobs nx = jb;
             const bool have_next = nx.next(g);
             const int nrel = (have_next && !nx.seg_start) ? 2 : 7;
-            const int ab = j & 1;
-            const uint32_t use = (uint32_t)(j >> 1) & 1u;
+            const int ab = j % ST_NACC;
+            const uint32_t use = (uint32_t)(j / ST_NACC) & 1u;
             bool ok = warp_wait(smem_u32(&acc_empty[ab]), use ^ 1u, a.err, 8u);
-            for (int r = 0; r < ST_R && ok; ++r) {
+            // only the rows new to this window: the others were waited for by
+            // an earlier row of the run and stay until it releases them
+            for (int r = jb.seg_start ? 0 : ST_R - 2; r < ST_R && ok; ++r) {
                 const int e = wstart + r;
                 ok = warp_wait(smem_u32(&full[e % ST_NSLOT]), (uint32_t)(e / ST_NSLOT) & 1u, a.err, 2u);
             }
@@ -332,8 +338,8 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
         bool have = jb.first(u0, u1, g);
         int j = 0;
         while (have) {
-            const int ab = j & 1;
-            const uint32_t use = (uint32_t)(j >> 1) & 1u;
+            const int ab = j % ST_NACC;
+            const uint32_t use = (uint32_t)(j / ST_NACC) & 1u;
             bool ok = mbar_wait(smem_u32(&acc_full[ab]), use, a.err, 4u);
             ok = __all_sync(0xffffffffu, ok) && !*abort_flag;
             __half *rb = rowbuf + (size_t)(j & 1) * 128 * ST_PIX_H;
@@ -503,7 +509,7 @@ cudaError_t launch_stem_pool(const ConvArgs &a, const StemPlan *pl, cudaStream_t
     g.N = a.N;
     const int units = g.N * g.P2;
     const int grid = std::min(pl->sms, units);
-    stem_pool_kernel<<<grid, ST_THREADS, ST_SMEM, st>>>(a, g);
+    pdl_launch(stem_pool_kernel, grid, ST_THREADS, ST_SMEM, st, a, g);
     return cudaGetLastError();
 }
 

@@ -213,10 +213,6 @@ __device__ __forceinline__ void store_checksum_pre(float ctv, const CsIn &c, con
     static_cast<__half *>(a.cs_out)[m] = __float2half_rn(o);
 }
 
-__device__ __forceinline__ void store_checksum(float ctv, const ConvArgs &a, const TcGeom &g, int m, int nimg,
-                                               int p, int q, float fsrc) {
-    store_checksum_pre(ctv, load_cs_inputs(a, g, m, nimg, p, q), a, g, m, fsrc);
-}
 
 // K-block kb accumulates into chain kb % NCH: back-to-back MMAs into one
 // TMEM accumulator serialise on it, so NCH independent chains keep the
@@ -280,6 +276,9 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
     __syncthreads();
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem = *tmem_holder;
+    // the previous kernel's outputs (and any fault flip) are visible from here
+    pdl_wait();
+    pdl_trigger();
 
     if (warp == 0) {
         // ---------------- TMA producer (whole warp, one lane issues) ----------------
@@ -571,6 +570,9 @@ conv_tc_small_kernel(const __grid_constant__ CUtensorMap bmap, const ConvArgs a,
     __syncthreads();
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem = *tmem_holder;
+    // the previous kernel's outputs (and any fault flip) are visible from here
+    pdl_wait();
+    pdl_trigger();
     const __half *x = static_cast<const __half *>(a.x);
 
     if (warp < 4) {
@@ -736,6 +738,7 @@ struct HaloGeom {
     int ncb, n_tiles, ty_tiles, tx_tiles;
     int ct;
     int tmem_cols;
+    int res, csin, rescs;       // epilogue operands fetched by TMA into the R ring
     uint16_t coef_h;
 };
 
@@ -758,6 +761,14 @@ __device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap *map
         : "memory");
 }
 
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *map, uint32_t bar, int x, int y, int n) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
+        "l"((uint64_t)map), "r"(x), "r"(y), "r"(n), "r"(bar)
+        : "memory");
+}
+
 struct HaloTile {
     int n, y0, x0, nt;
 };
@@ -772,30 +783,53 @@ __device__ __forceinline__ HaloTile halo_tile(int t, const HaloGeom &hg) {
     return h;
 }
 
-template <int BN, bool BRES, int NA, int NB>
+// tensor maps of one halo plan: patch (A), weights (B), and the epilogue
+// operands: residual tile [16 x 8 x BN], incoming and residual checksum
+// planes [16 x 8]
+struct HaloMaps {
+    CUtensorMap amap, bmap, rmap, cmap, qmap;
+};
+
+// Epilogue operand ring (R): per tile, the residual tile (BN channels of
+// its 128 pixels, pixel-major) and the incoming / residual checksum values
+// of its pixels, fetched by the producer warp with TMA several tiles ahead
+// so that the epilogue reads them from shared memory.
+template <int BN>
+struct HaloR {
+    static constexpr int RES = 128 * BN * 2;
+    static constexpr int CS = 128 * 2;
+    static constexpr int STAGE = RES + 2 * CS;       // multiple of 128
+};
+
+template <int BN, bool BRES, int NA, int NB, int NR>
 __global__ void __launch_bounds__(NTHREADS, 1)
-conv_tc_halo_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
-                    const ConvArgs a, const HaloGeom hg, const TcGeom g) {
+conv_tc_halo_kernel(const __grid_constant__ HaloMaps maps, const ConvArgs a, const HaloGeom hg, const TcGeom g) {
     constexpr int B_ROWS = BN + 16;                       // 16 constant carry-through rows
     constexpr int B_STAGE = B_ROWS * BK * 2;
     constexpr int B_TMA = BN * BK * 2;
     constexpr int NBS = BRES ? 9 : NB;
     constexpr int CH = BN + 16;
+    using R = HaloR<BN>;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint8_t *As = smem;
     uint8_t *Bs = As + NA * HT_A_STAGE;
-    uint64_t *a_full = (uint64_t *)(Bs + NBS * B_STAGE);
+    uint8_t *Rs = Bs + NBS * B_STAGE;
+    uint64_t *a_full = (uint64_t *)(Rs + NR * R::STAGE);
     uint64_t *a_empty = a_full + NA;
     uint64_t *b_full = a_empty + NA;
     uint64_t *b_empty = b_full + NBS;
-    uint64_t *acc_full = b_empty + NBS;
+    uint64_t *r_full = b_empty + NBS;
+    uint64_t *r_empty = r_full + NR;
+    uint64_t *acc_full = r_empty + NR;
     uint64_t *acc_empty = acc_full + 2;
     uint32_t *tmem_holder = (uint32_t *)(acc_empty + 2);
     volatile uint32_t *abort_flag = tmem_holder + 1;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int num_tiles = hg.N * hg.ty_tiles * hg.tx_tiles * hg.n_tiles;
+    const bool ring = hg.res || hg.csin || hg.rescs;
+    const uint32_t r_bytes = (hg.res ? R::RES : 0) + (hg.csin ? R::CS : 0) + (hg.rescs ? R::CS : 0);
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < NA; ++s) {
@@ -805,6 +839,10 @@ conv_tc_halo_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
         for (int s = 0; s < NBS; ++s) {
             mbar_init(smem_u32(&b_full[s]), 1);
             mbar_init(smem_u32(&b_empty[s]), 1);
+        }
+        for (int s = 0; s < NR; ++s) {
+            mbar_init(smem_u32(&r_full[s]), 1);
+            mbar_init(smem_u32(&r_empty[s]), N_EPI_WARPS);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(smem_u32(&acc_full[b]), 1);
@@ -833,21 +871,24 @@ conv_tc_halo_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
     __syncthreads();
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem = *tmem_holder;
+    // the previous kernel's outputs (and any fault flip) are visible from here
+    pdl_wait();
+    pdl_trigger();
 
     if (warp == 0) {
         // ---------------- TMA producer (whole warp, one lane issues) ----------------
         if (elect_one()) {
-            asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&amap) : "memory");
-            asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&bmap) : "memory");
+            asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&maps.amap) : "memory");
+            asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&maps.bmap) : "memory");
             if (BRES) {
                 for (int i = 0; i < 9; ++i) {
                     mbar_arrive_expect_tx(smem_u32(&b_full[i]), B_TMA);
-                    tma_load_2d(smem_u32(Bs + i * B_STAGE), &bmap, smem_u32(&b_full[i]), tap_of(i, 4) * hg.C, 0);
+                    tma_load_2d(smem_u32(Bs + i * B_STAGE), &maps.bmap, smem_u32(&b_full[i]), tap_of(i, 4) * hg.C, 0);
                 }
             }
         }
         __syncwarp();
-        int ai = 0, bi = 0;
+        int ai = 0, bi = 0, ri = 0;
         bool ok = true;
         for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
             if (__any_sync(0xffffffffu, *abort_flag)) break;
@@ -857,11 +898,26 @@ conv_tc_halo_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
                 if (!warp_wait(smem_u32(&a_empty[as]), ((uint32_t)(ai / NA) & 1u) ^ 1u, a.err, 1u)) { ok = false; break; }
                 if (elect_one()) {
                     mbar_arrive_expect_tx(smem_u32(&a_full[as]), HT_A_BYTES);
-                    tma_load_4d(smem_u32(As + as * HT_A_STAGE), &amap, smem_u32(&a_full[as]), cb * BK, ht.x0 - 1,
+                    tma_load_4d(smem_u32(As + as * HT_A_STAGE), &maps.amap, smem_u32(&a_full[as]), cb * BK, ht.x0 - 1,
                                 ht.y0 - 1, ht.n);
                 }
                 __syncwarp();
                 ++ai;
+                if (cb == 0 && ring) {
+                    // epilogue operands of this tile, behind its first patch
+                    const int rs = ri % NR;
+                    if (!warp_wait(smem_u32(&r_empty[rs]), ((uint32_t)(ri / NR) & 1u) ^ 1u, a.err, 1u)) { ok = false; break; }
+                    if (elect_one()) {
+                        const uint32_t rb = smem_u32(&r_full[rs]);
+                        uint8_t *st = Rs + rs * R::STAGE;
+                        mbar_arrive_expect_tx(rb, r_bytes);
+                        if (hg.res) tma_load_4d(smem_u32(st), &maps.rmap, rb, ht.nt * BN, ht.x0, ht.y0, ht.n);
+                        if (hg.csin) tma_load_3d(smem_u32(st + R::RES), &maps.cmap, rb, ht.x0, ht.y0, ht.n);
+                        if (hg.rescs) tma_load_3d(smem_u32(st + R::RES + R::CS), &maps.qmap, rb, ht.x0, ht.y0, ht.n);
+                    }
+                    __syncwarp();
+                    ++ri;
+                }
                 if (!BRES) {
                     for (int i = 0; i < 9; ++i) {
                         const int bs = bi % NBS;
@@ -871,7 +927,7 @@ conv_tc_halo_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
                         }
                         if (elect_one()) {
                             mbar_arrive_expect_tx(smem_u32(&b_full[bs]), B_TMA);
-                            tma_load_2d(smem_u32(Bs + bs * B_STAGE), &bmap, smem_u32(&b_full[bs]),
+                            tma_load_2d(smem_u32(Bs + bs * B_STAGE), &maps.bmap, smem_u32(&b_full[bs]),
                                         tap_of(i, 4) * hg.C + cb * BK, ht.nt * BN);
                         }
                         __syncwarp();
@@ -887,18 +943,44 @@ conv_tc_halo_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
         const uint32_t id_merged = idesc_f16(BM, BN + 16);
         int ai = 0, bi = 0, lt = 0;
         bool ok = true;
+        if (BRES) {
+            // resident weights: wait for all nine tiles once
+            for (int i = 0; i < 9 && ok; ++i) ok = warp_wait(smem_u32(&b_full[i]), 0u, a.err, 2u);
+        }
         for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x, ++lt) {
             if (__any_sync(0xffffffffu, *abort_flag)) break;
             const HaloTile ht = halo_tile(tile, hg);
             const bool ct_here = hg.ct && ht.nt == 0;
             const int ab = lt & 1;
             if (!warp_wait(smem_u32(&acc_empty[ab]), ((uint32_t)(lt >> 1) & 1u) ^ 1u, a.err, 8u)) { ok = false; break; }
-            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
             const uint32_t d = tmem + (uint32_t)(ab * CH);
             for (int cb = 0; cb < hg.ncb && ok; ++cb) {
                 const int as = ai % NA;
                 if (!warp_wait(smem_u32(&a_full[as]), (uint32_t)(ai / NA) & 1u, a.err, 2u)) { ok = false; break; }
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                 const uint32_t a_base = smem_u32(As + as * HT_A_STAGE);
+                if constexpr (BRES) {
+                    // all 36 MMAs of the tile in one burst from one lane
+                    if (elect_one()) {
+                        const uint32_t b0 = smem_u32(Bs);
+#pragma unroll
+                        for (int i = 0; i < 9; ++i) {
+                            const int tap = tap_of(i, 4);
+                            const uint32_t a_tap = a_base + (uint32_t)(((tap / 3) * HT_PW + tap % 3) * BK * 2);
+                            const uint32_t b_base = b0 + (uint32_t)(i * B_STAGE);
+#pragma unroll
+                            for (int k16 = 0; k16 < BK / 16; ++k16) {
+                                const uint64_t ad = smem_desc_sw128_sbo(a_tap + k16 * 32, HT_ROW);
+                                const uint64_t bd = smem_desc_sw128(b_base + k16 * 32);
+                                const uint32_t acc = (cb > 0 || i > 0 || k16 > 0) ? 1u : 0u;
+                                umma_f16(d, ad, bd, (ct_here && i == 0) ? id_merged : id_main, acc);
+                            }
+                        }
+                        umma_commit(smem_u32(&a_empty[as]));
+                    }
+                    __syncwarp();
+                    ++ai;
+                } else {
                 for (int i = 0; i < 9; ++i) {
                     const int bs = BRES ? i : bi % NBS;
                     const uint32_t bph = BRES ? 0u : (uint32_t)(bi / NBS) & 1u;
@@ -925,6 +1007,7 @@ conv_tc_halo_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
                 if (elect_one()) umma_commit(smem_u32(&a_empty[as]));
                 __syncwarp();
                 ++ai;
+                }
             }
             if (!ok) break;
             if (elect_one()) umma_commit(smem_u32(&acc_full[ab]));   // fires when the tile's MMAs have completed
@@ -947,14 +1030,10 @@ conv_tc_halo_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
             const bool valid = p < hg.H && q < hg.W;
             const int m = valid ? (ht.n * hg.H + p) * hg.W + q : 0;
             const int n0 = ht.nt * BN + half * (BN / 2);
-            // residual loads in flight while the MMAs run
-            Res16 rs[BN / 32];
-#pragma unroll
-            for (int c = 0; c < BN / 32; ++c)
-                rs[c] = valid ? load_res16(a, hg.K, (size_t)m, n0 + 16 * c) : Res16{make_uint4(0u, 0u, 0u, 0u), make_uint4(0u, 0u, 0u, 0u)};
             const bool do_cs = half == 0 && a.cs_out != nullptr && ht.nt == 0;
-            const CsIn csv = (do_cs && valid) ? load_cs_inputs(a, g, m, ht.n, p, q) : CsIn{0.f, 0.f};
             bool ok = mbar_wait(smem_u32(&acc_full[ab]), (uint32_t)(lt >> 1) & 1u, a.err, 4u) && !*abort_flag;
+            const int rsl = lt % NR;
+            if (ring) ok = ok && mbar_wait(smem_u32(&r_full[rsl]), (uint32_t)(lt / NR) & 1u, a.err, 4u);
             ok = __all_sync(0xffffffffu, ok);
             if (!ok) break;
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
@@ -966,6 +1045,28 @@ conv_tc_halo_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
             asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&acc_empty[ab]));
+            // epilogue operands from the R ring
+            const uint8_t *rst = Rs + rsl * R::STAGE;
+            Res16 rs[BN / 32];
+#pragma unroll
+            for (int c = 0; c < BN / 32; ++c) {
+                if (hg.res) {
+                    const uint4 *rp = reinterpret_cast<const uint4 *>(rst + ((size_t)row * BN + half * (BN / 2) + 16 * c) * 2);
+                    rs[c].r0 = rp[0];
+                    rs[c].r1 = rp[1];
+                } else {
+                    rs[c].r0 = rs[c].r1 = make_uint4(0u, 0u, 0u, 0u);
+                }
+            }
+            CsIn csv{0.f, 0.f};
+            if (do_cs) {
+                if (hg.csin) csv.cin = __half2float(reinterpret_cast<const __half *>(rst + R::RES)[row]);
+                if (hg.rescs) csv.rcs = __half2float(reinterpret_cast<const __half *>(rst + R::RES + R::CS)[row]);
+            }
+            if (ring) {
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&r_empty[rsl]));
+            }
             if (valid) {
                 float fsrc = 0.f;
                 if (fd.active) {
@@ -1118,9 +1219,9 @@ cudaError_t launch_conv_tc(const ConvArgs &a, const void *plan, cudaStream_t st,
     g.kps = (g.n_kb + g.splits - 1) / g.splits;
     const int items = tiles * g.splits;
     dim3 grid(items < pl->sms ? items : pl->sms);
-    if (pl->BN == 64) conv_tc_kernel<64, 4, 2, 4><<<grid, NTHREADS, pl->smem, st>>>(pl->amap, pl->bmap, a, g);
-    else if (pl->BN == 128) conv_tc_kernel<128, 3, 2, 2><<<grid, NTHREADS, pl->smem, st>>>(pl->amap, pl->bmap, a, g);
-    else conv_tc_kernel<256, 4, 1, 1><<<grid, NTHREADS, pl->smem, st>>>(pl->amap, pl->bmap, a, g);
+    if (pl->BN == 64) pdl_launch(conv_tc_kernel<64, 4, 2, 4>, grid, NTHREADS, pl->smem, st, pl->amap, pl->bmap, a, g);
+    else if (pl->BN == 128) pdl_launch(conv_tc_kernel<128, 3, 2, 2>, grid, NTHREADS, pl->smem, st, pl->amap, pl->bmap, a, g);
+    else pdl_launch(conv_tc_kernel<256, 4, 1, 1>, grid, NTHREADS, pl->smem, st, pl->amap, pl->bmap, a, g);
     cudaError_t e = cudaGetLastError();
     if (n_kernels) *n_kernels = 1;
     if (e != cudaSuccess || g.splits == 1) return e;
@@ -1182,7 +1283,7 @@ cudaError_t launch_conv_tc_small(const ConvArgs &a, const TcSmallPlan *pl, cudaS
     g.M = a.N * a.P * a.Q;
     g.m_tiles = (g.M + BM - 1) / BM;
     dim3 grid(g.m_tiles < pl->sms ? g.m_tiles : pl->sms);
-    conv_tc_small_kernel<<<grid, SM_THREADS, pl->smem, st>>>(pl->bmap, a, g);
+    pdl_launch(conv_tc_small_kernel, grid, SM_THREADS, pl->smem, st, pl->bmap, a, g);
     return cudaGetLastError();
 }
 
@@ -1192,18 +1293,19 @@ void tc_plan_destroy(TcPlan *p) { delete p; }
 // halo-tile plans
 // ---------------------------------------------------------------------------
 struct HaloPlan {
-    CUtensorMap amap;
-    CUtensorMap bmap;
+    HaloMaps maps;
     HaloGeom hg;
     TcGeom g;
     int BN, kind, sms;
     size_t smem;
+    const void *res, *csin, *rescs;   // tensors the R-ring maps point at
 };
 
-template <int BN, bool BRES, int NA, int NB>
+template <int BN, bool BRES, int NA, int NB, int NR>
 size_t halo_smem() {
     const int nbs = BRES ? 9 : NB;
-    return 1024 + (size_t)NA * HT_A_STAGE + (size_t)nbs * (BN + 16) * BK * 2 + 8 * (2 * NA + 2 * nbs + 4) + 16;
+    return 1024 + (size_t)NA * HT_A_STAGE + (size_t)nbs * (BN + 16) * BK * 2 + (size_t)NR * HaloR<BN>::STAGE +
+           8 * (2 * NA + 2 * nbs + 2 * NR + 4) + 16;
 }
 
 // Tiles that overhang the image waste MMA rows: require whole 8-column tiles
@@ -1213,13 +1315,26 @@ bool halo_supported(int C, int K, int R, int S, int stride, int pad, int H, int 
            (H % HT_TH == 0 || H >= 3 * HT_TH);
 }
 
-HaloPlan *halo_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, const void *x_dev, std::string *why) {
+static bool encode_plane_map(CUtensorMap *map, const void *plane, int N, int H, int W) {
+    // [N, H, W] fp16 plane as boxes of 8 x 16 pixels
+    cuuint64_t dim[3] = {(cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)N};
+    cuuint64_t str[2] = {(cuuint64_t)W * 2, (cuuint64_t)H * W * 2};
+    cuuint32_t box[3] = {HT_TW, HT_TH, 1};
+    cuuint32_t es[3] = {1, 1, 1};
+    return g_encode_tiled(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 3, const_cast<void *>(plane), dim, str, box, es,
+                          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+HaloPlan *halo_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, const void *x_dev, const void *res_dev,
+                           const void *csin_dev, const void *rescs_dev, std::string *why) {
     if (!halo_supported(a.C, a.K, a.R, a.S, a.stride, a.pad, a.H, a.W)) { if (why) *why = "shape"; return nullptr; }
     if (!load_encoders()) { if (why) *why = "tensor-map encoders unavailable"; return nullptr; }
     HaloPlan *pl = new HaloPlan();
     memset(pl, 0, sizeof(*pl));
     pl->BN = a.K;
     pl->sms = sm_count();
+    pl->res = res_dev; pl->csin = csin_dev; pl->rescs = rescs_dev;
     HaloGeom &hg = pl->hg;
     hg.H = a.H; hg.W = a.W; hg.C = a.C; hg.K = a.K;
     hg.ncb = a.C / BK;
@@ -1229,6 +1344,7 @@ HaloPlan *halo_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, 
     hg.ct = a.role == CT_ROLE_CT ? 1 : 0;
     hg.tmem_cols = 2 * (pl->BN + 16) <= 256 ? 256 : 512;
     hg.coef_h = coef_half_bits(a.coef);
+    hg.res = res_dev != nullptr; hg.csin = csin_dev != nullptr; hg.rescs = rescs_dev != nullptr;
     // geometry the shared epilogue helpers read
     TcGeom &g = pl->g;
     g.PQ = a.P * a.Q; g.Q = a.Q; g.stride = 1; g.pad = 1; g.C = a.C; g.K = a.K; g.S = 3; g.ctr_tap = 4;
@@ -1237,8 +1353,8 @@ HaloPlan *halo_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, 
     cuuint64_t gstr[3] = {(cuuint64_t)a.C * 2, (cuuint64_t)a.W * a.C * 2, (cuuint64_t)a.H * a.W * a.C * 2};
     cuuint32_t abox[4] = {BK, HT_PW, HT_PH, 1};
     cuuint32_t aes[4] = {1, 1, 1, 1};
-    CUresult r = g_encode_tiled(&pl->amap, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<void *>(x_dev), gdim, gstr,
-                                abox, aes, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+    CUresult r = g_encode_tiled(&pl->maps.amap, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<void *>(x_dev), gdim,
+                                gstr, abox, aes, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                                 CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) { if (why) *why = "patch tensor map"; delete pl; return nullptr; }
     const int RSC = 9 * a.C;
@@ -1246,23 +1362,42 @@ HaloPlan *halo_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, 
     cuuint64_t bstr[1] = {(cuuint64_t)RSC * 2};
     cuuint32_t box[2] = {BK, (cuuint32_t)pl->BN};
     cuuint32_t bes[2] = {1, 1};
-    r = g_encode_tiled(&pl->bmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void *>(w_dev), bdim, bstr, box, bes,
-                       CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+    r = g_encode_tiled(&pl->maps.bmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void *>(w_dev), bdim, bstr, box,
+                       bes, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) { if (why) *why = "weight tensor map"; delete pl; return nullptr; }
+    if (res_dev) {
+        // residual [max_batch, H, W, K]: boxes of BN channels x 8 x 16 pixels, pixel-major
+        cuuint64_t rdim[4] = {(cuuint64_t)a.K, (cuuint64_t)a.W, (cuuint64_t)a.H, (cuuint64_t)max_batch};
+        cuuint64_t rstr[3] = {(cuuint64_t)a.K * 2, (cuuint64_t)a.W * a.K * 2, (cuuint64_t)a.H * a.W * a.K * 2};
+        cuuint32_t rbox[4] = {(cuuint32_t)pl->BN, HT_TW, HT_TH, 1};
+        if (g_encode_tiled(&pl->maps.rmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<void *>(res_dev), rdim, rstr,
+                           rbox, aes, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                           CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS) {
+            if (why) *why = "residual tensor map";
+            delete pl;
+            return nullptr;
+        }
+    }
+    if ((csin_dev && !encode_plane_map(&pl->maps.cmap, csin_dev, max_batch, a.H, a.W)) ||
+        (rescs_dev && !encode_plane_map(&pl->maps.qmap, rescs_dev, max_batch, a.H, a.W))) {
+        if (why) *why = "checksum tensor map";
+        delete pl;
+        return nullptr;
+    }
     cudaError_t e;
     if (pl->BN == 64 && hg.ncb == 1) {
         pl->kind = 0;
-        pl->smem = halo_smem<64, true, 4, 0>();
-        e = cudaFuncSetAttribute(conv_tc_halo_kernel<64, true, 4, 0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
+        pl->smem = halo_smem<64, true, 3, 0, 3>();
+        e = cudaFuncSetAttribute(conv_tc_halo_kernel<64, true, 3, 0, 3>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
     } else if (pl->BN == 64) {
         pl->kind = 1;
-        pl->smem = halo_smem<64, false, 4, 8>();
-        e = cudaFuncSetAttribute(conv_tc_halo_kernel<64, false, 4, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
+        pl->smem = halo_smem<64, false, 3, 6, 3>();
+        e = cudaFuncSetAttribute(conv_tc_halo_kernel<64, false, 3, 6, 3>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
     } else {
         pl->kind = 2;
-        pl->smem = halo_smem<128, false, 3, 6>();
-        e = cudaFuncSetAttribute(conv_tc_halo_kernel<128, false, 3, 6>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
+        pl->smem = halo_smem<128, false, 3, 4, 2>();
+        e = cudaFuncSetAttribute(conv_tc_halo_kernel<128, false, 3, 4, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
     }
     if (e != cudaSuccess) { cudaGetLastError(); if (why) *why = "shared memory attribute"; delete pl; return nullptr; }
     return pl;
@@ -1272,15 +1407,19 @@ int halo_tiles(const HaloPlan *pl, int batch) { return batch * pl->hg.ty_tiles *
 int halo_sms(const HaloPlan *pl) { return pl->sms; }
 
 cudaError_t launch_conv_tc_halo(const ConvArgs &a, const HaloPlan *pl, cudaStream_t st) {
+    // the R-ring maps were encoded for these tensors
+    if (a.res != pl->res || (a.cs_out && a.cs_in != pl->csin) || (a.cs_out && a.res_cs != pl->rescs))
+        return cudaErrorInvalidValue;
     HaloGeom hg = pl->hg;
     hg.N = a.N;
+    if (!a.cs_out) hg.csin = hg.rescs = 0;
     TcGeom g = pl->g;
     g.M = a.N * a.P * a.Q;
     const int tiles = halo_tiles(pl, a.N);
     dim3 grid(tiles < pl->sms ? tiles : pl->sms);
-    if (pl->kind == 0) conv_tc_halo_kernel<64, true, 4, 0><<<grid, NTHREADS, pl->smem, st>>>(pl->amap, pl->bmap, a, hg, g);
-    else if (pl->kind == 1) conv_tc_halo_kernel<64, false, 4, 8><<<grid, NTHREADS, pl->smem, st>>>(pl->amap, pl->bmap, a, hg, g);
-    else conv_tc_halo_kernel<128, false, 3, 6><<<grid, NTHREADS, pl->smem, st>>>(pl->amap, pl->bmap, a, hg, g);
+    if (pl->kind == 0) pdl_launch(conv_tc_halo_kernel<64, true, 3, 0, 3>, grid, NTHREADS, pl->smem, st, pl->maps, a, hg, g);
+    else if (pl->kind == 1) pdl_launch(conv_tc_halo_kernel<64, false, 3, 6, 3>, grid, NTHREADS, pl->smem, st, pl->maps, a, hg, g);
+    else pdl_launch(conv_tc_halo_kernel<128, false, 3, 4, 2>, grid, NTHREADS, pl->smem, st, pl->maps, a, hg, g);
     return cudaGetLastError();
 }
 

@@ -463,7 +463,12 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
         l.plan = tc_plan_create(a, B, l.w, m->slots[l.d.src].data, &why);
         if (!l.plan) return CT_ECUDA;
         if (halo_supported(l.C, l.K, l.R, l.S, l.d.stride, l.d.pad, l.H, l.W) && m->slots[l.d.src].cp == l.C) {
-            l.hplan = halo_plan_create(a, B, l.w, m->slots[l.d.src].data, &why);
+            const Slot &sx = m->slots[l.d.src];
+            const Slot *sr = l.d.res >= 0 ? &m->slots[l.d.res] : nullptr;
+            const bool cs_out = l.cs_out;
+            l.hplan = halo_plan_create(a, B, l.w, sx.data, sr ? sr->data : nullptr,
+                                       (cs_out && sx.has_cs) ? sx.cs : nullptr,
+                                       (cs_out && sr && sr->has_cs) ? sr->cs : nullptr, &why);
             if (!l.hplan) return CT_ECUDA;
         }
     }

@@ -6,6 +6,7 @@
 #include <stdint.h>
 
 #include <string>
+#include <utility>
 #include <vector>
 
 #include "../../include/ct.h"
@@ -69,6 +70,33 @@ struct PoolArgs {
 
 enum Family { FAM_TC = 0, FAM_SIMT = 1, FAM_FC = 2, FAM_POOL = 3, FAM_OTHER = 4, FAM_COUNT = 5 };
 
+// Programmatic dependent launch: every kernel is launched so that it may
+// start while the previous kernel in the stream finishes; it calls
+// pdl_wait() before its first access to global memory (which returns once
+// the previous kernel has completed and its writes are visible) and
+// pdl_trigger() to let the next kernel start early.  Only prologues that
+// touch no global memory (barrier set-up, TMEM allocation) overlap.
+#ifdef __CUDACC__
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+#endif
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t pdl_launch(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                              Args &&...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
 // kernel launchers; each returns cudaGetLastError()
 // conv launchers report in *n_kernels (may be null) how many kernels they
 // launched: 2 when K is split (the conv kernel and the split-K reduction)
@@ -124,8 +152,10 @@ cudaError_t launch_conv_tc_small(const ConvArgs &a, const TcSmallPlan *plan, cud
 // tiles of 16 x 8 output pixels: one patch load per tile and channel block.
 struct HaloPlan;
 bool halo_supported(int C, int K, int R, int S, int stride, int pad, int H, int W);
+// res_dev / csin_dev / rescs_dev: residual tensor, incoming and residual
+// checksum planes the layer reads (null if none); launches must pass them.
 HaloPlan *halo_plan_create(const ConvArgs &shape_args, int max_batch, const void *w_dev, const void *x_dev,
-                           std::string *why);
+                           const void *res_dev, const void *csin_dev, const void *rescs_dev, std::string *why);
 void halo_plan_destroy(HaloPlan *p);
 int halo_tiles(const HaloPlan *p, int batch);
 int halo_sms(const HaloPlan *p);

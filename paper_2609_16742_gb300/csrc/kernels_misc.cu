@@ -29,6 +29,8 @@ static_assert((FC_KC * (FC_IMG + 1)) % 4 == 0, "weight tile must start 16-byte a
 
 template <typename TX, typename TW, typename TY>
 __global__ void __launch_bounds__(256) fc_kernel(FcArgs a) {
+    pdl_wait();
+    pdl_trigger();
     extern __shared__ __align__(16) float smem[];
     float *Xs = smem;                              // [FC_KC][FC_IMG + 1]
     float *Ws = Xs + FC_KC * (FC_IMG + 1);         // [FC_KC][FC_J]; offset 4160 floats: 16-byte aligned
@@ -155,6 +157,8 @@ __global__ void __launch_bounds__(256) fc_kernel(FcArgs a) {
 // checksum neuron.
 template <typename TX, typename TY>
 __global__ void fc_reduce_kernel(FcArgs a, int splits) {
+    pdl_wait();
+    pdl_trigger();
     const int ldw = a.n_out + 1;
     const long long total = (long long)a.B * ldw;
     const size_t plane = (size_t)a.B * ldw;
@@ -203,6 +207,8 @@ __device__ __forceinline__ void vmax(float &m, float v) { m = (v > m || v != v) 
 
 template <typename T>
 __global__ void maxpool_kernel(PoolArgs a) {
+    pdl_wait();
+    pdl_trigger();
     constexpr int VE = 16 / sizeof(T);
     using V = uint4;
     const int CV = a.C / VE;                       // vectors per pixel (C % VE == 0)
@@ -257,6 +263,8 @@ __global__ void maxpool_kernel(PoolArgs a) {
 // Scalar fallback for channel counts that are not a multiple of the vector.
 template <typename T>
 __global__ void maxpool_scalar_kernel(PoolArgs a) {
+    pdl_wait();
+    pdl_trigger();
     const int64_t n_data = (int64_t)a.N * a.P * a.Q * a.C;
     const int64_t n_cs = a.cs_in ? (int64_t)a.N * a.P * a.Q : 0;
     for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n_data + n_cs;
@@ -288,6 +296,8 @@ __global__ void maxpool_scalar_kernel(PoolArgs a) {
 // Global average pool: float [N, C] features (+ float [N] checksum feature).
 template <typename T>
 __global__ void gap_kernel(PoolArgs a) {
+    pdl_wait();
+    pdl_trigger();
     const int HW = a.H * a.W;
     const int n = blockIdx.y;
     const int c = blockIdx.x * blockDim.x + threadIdx.x;
@@ -308,6 +318,8 @@ __global__ void gap_kernel(PoolArgs a) {
 // of the output (padding to Cp channels) are written as zeros.
 template <typename T>
 __global__ void convert_input_kernel(const float *in, T *out, int N, int C, int Cp, int H, int W) {
+    pdl_wait();
+    pdl_trigger();
     const int HW = H * W;
     const int total = N * HW;
     for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < total; e += gridDim.x * blockDim.x) {
@@ -319,6 +331,8 @@ __global__ void convert_input_kernel(const float *in, T *out, int N, int C, int 
 }
 
 __global__ void xor_bit_kernel(void *base, int64_t word, int bit, int word_bytes) {
+    pdl_wait();
+    pdl_trigger();
     if (word_bytes == 2) static_cast<uint16_t *>(base)[word] ^= (uint16_t)(1u << bit);
     else static_cast<uint32_t *>(base)[word] ^= (1u << bit);
 }
@@ -326,6 +340,8 @@ __global__ void xor_bit_kernel(void *base, int64_t word, int bit, int word_bytes
 // Copies image idx[i] of `in` to row i of `out` (NCHW float rows of `per`
 // elements).  16-byte vectors when every row starts 16-byte aligned.
 __global__ void gather_images_kernel(const float *in, float *out, const int32_t *idx, int64_t per) {
+    pdl_wait();
+    pdl_trigger();
     const int i = blockIdx.y;
     const float *s = in + (size_t)idx[i] * per;
     float *d = out + (size_t)i * per;
@@ -341,6 +357,8 @@ __global__ void gather_images_kernel(const float *in, float *out, const int32_t 
 }
 
 __global__ void scatter_rows_kernel(const float *src, float *dst, const int32_t *idx, int n, int row) {
+    pdl_wait();
+    pdl_trigger();
     for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < n * row; e += gridDim.x * blockDim.x) {
         int i = e / row, c = e % row;
         dst[(size_t)idx[i] * row + c] = src[e];
@@ -371,13 +389,13 @@ cudaError_t fc_go(const FcArgs &a, cudaStream_t st, int *n_kernels) {
     const int nkc = (a.n_in + FC_KC - 1) / FC_KC;
     const int splits = splitk_choose(gx * gy, nkc, 4, 2 * sms, a.B, a.n_out + 1, a.ws ? a.ws_bytes : 0);
     dim3 grid(gx, gy, splits);
-    fc_kernel<TX, TW, TY><<<grid, 256, smem, st>>>(a);
+    pdl_launch(fc_kernel<TX, TW, TY>, grid, 256, smem, st, a);
     cudaError_t e = cudaGetLastError();
     if (n_kernels) *n_kernels = 1;
     if (e != cudaSuccess || splits == 1) return e;
     if (n_kernels) *n_kernels = 2;
     const long long total = (long long)a.B * (a.n_out + 1);
-    fc_reduce_kernel<TX, TY><<<(int)std::min<long long>((total + 255) / 256, 4096), 256, 0, st>>>(a, splits);
+    pdl_launch(fc_reduce_kernel<TX, TY>, (int)std::min<long long>((total + 255) / 256, 4096), 256, 0, st, a, splits);
     return cudaGetLastError();
 }
 
@@ -395,33 +413,33 @@ cudaError_t launch_maxpool(const PoolArgs &a, bool half, cudaStream_t st) {
     const int64_t pix = (int64_t)a.N * a.P * a.Q;
     if (a.C % ve == 0 && pix * (a.C / ve + 1) < (1ll << 31)) {
         const int64_t n = pix * (a.C / ve + (a.cs_in ? 1 : 0));
-        if (half) maxpool_kernel<__half><<<grid_for(n, 256), 256, 0, st>>>(a);
-        else maxpool_kernel<float><<<grid_for(n, 256), 256, 0, st>>>(a);
+        if (half) pdl_launch(maxpool_kernel<__half>, grid_for(n, 256), 256, 0, st, a);
+        else pdl_launch(maxpool_kernel<float>, grid_for(n, 256), 256, 0, st, a);
     } else {
         const int64_t n = pix * (a.C + (a.cs_in ? 1 : 0));
-        if (half) maxpool_scalar_kernel<__half><<<grid_for(n, 256), 256, 0, st>>>(a);
-        else maxpool_scalar_kernel<float><<<grid_for(n, 256), 256, 0, st>>>(a);
+        if (half) pdl_launch(maxpool_scalar_kernel<__half>, grid_for(n, 256), 256, 0, st, a);
+        else pdl_launch(maxpool_scalar_kernel<float>, grid_for(n, 256), 256, 0, st, a);
     }
     return cudaGetLastError();
 }
 
 cudaError_t launch_gap(const PoolArgs &a, bool half, cudaStream_t st) {
     dim3 grid((a.C + 1 + 127) / 128, a.N);
-    if (half) gap_kernel<__half><<<grid, 128, 0, st>>>(a);
-    else gap_kernel<float><<<grid, 128, 0, st>>>(a);
+    if (half) pdl_launch(gap_kernel<__half>, grid, 128, 0, st, a);
+    else pdl_launch(gap_kernel<float>, grid, 128, 0, st, a);
     return cudaGetLastError();
 }
 
 cudaError_t launch_convert_input(const float *in, void *out, int N, int C, int Cp, int H, int W, bool half,
                                  cudaStream_t st) {
     const int64_t n = (int64_t)N * H * W;
-    if (half) convert_input_kernel<__half><<<grid_for(n, 256), 256, 0, st>>>(in, (__half *)out, N, C, Cp, H, W);
-    else convert_input_kernel<float><<<grid_for(n, 256), 256, 0, st>>>(in, (float *)out, N, C, Cp, H, W);
+    if (half) pdl_launch(convert_input_kernel<__half>, grid_for(n, 256), 256, 0, st, in, (__half *)out, N, C, Cp, H, W);
+    else pdl_launch(convert_input_kernel<float>, grid_for(n, 256), 256, 0, st, in, (float *)out, N, C, Cp, H, W);
     return cudaGetLastError();
 }
 
 cudaError_t launch_xor_bit(void *base, int64_t word, int bit, int word_bytes, cudaStream_t st) {
-    xor_bit_kernel<<<1, 1, 0, st>>>(base, word, bit, word_bytes);
+    pdl_launch(xor_bit_kernel, 1, 1, 0, st, base, word, bit, word_bytes);
     return cudaGetLastError();
 }
 
@@ -430,14 +448,14 @@ cudaError_t launch_gather_images(const float *in, float *out, const int32_t *idx
     if (n <= 0) return cudaSuccess;
     const int64_t blocks = (per_image / 4 + 255) / 256 + 1;
     dim3 grid((unsigned)(blocks > 64 ? 64 : blocks), n);
-    gather_images_kernel<<<grid, 256, 0, st>>>(in, out, idx, per_image);
+    pdl_launch(gather_images_kernel, grid, 256, 0, st, in, out, idx, per_image);
     return cudaGetLastError();
 }
 
 cudaError_t launch_scatter_rows(const float *src, float *dst, const int32_t *idx, int n, int row,
                                 cudaStream_t st) {
     if (n <= 0) return cudaSuccess;
-    scatter_rows_kernel<<<grid_for((int64_t)n * row, 256), 256, 0, st>>>(src, dst, idx, n, row);
+    pdl_launch(scatter_rows_kernel, grid_for((int64_t)n * row, 256), 256, 0, st, src, dst, idx, n, row);
     return cudaGetLastError();
 }
 

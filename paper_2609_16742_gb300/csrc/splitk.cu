@@ -37,6 +37,8 @@ __device__ __forceinline__ float fault_source(const ConvArgs &a, int n, int p, i
 // one thread: 8 channels of one output pixel, or (chunk == K / 8) its checksum
 template <typename T>
 __global__ void splitk_reduce_kernel(const ConvArgs a, int splits, int ws_ld) {
+    pdl_wait();
+    pdl_trigger();
     const int M = a.N * a.P * a.Q;
     const int chunks = a.K / 8 + (a.cs_out ? 1 : 0);
     const long long total = (long long)M * chunks;
@@ -149,8 +151,8 @@ cudaError_t launch_splitk_reduce(const ConvArgs &a, int splits, int ws_ld, bool 
     const int threads = 256;
     const long long want = (total + threads - 1) / threads;
     const int grid = (int)std::min<long long>(std::max<long long>(want, 1), 4096);
-    if (half) splitk_reduce_kernel<__half><<<grid, threads, 0, st>>>(a, splits, ws_ld);
-    else splitk_reduce_kernel<float><<<grid, threads, 0, st>>>(a, splits, ws_ld);
+    if (half) pdl_launch(splitk_reduce_kernel<__half>, grid, threads, 0, st, a, splits, ws_ld);
+    else pdl_launch(splitk_reduce_kernel<float>, grid, threads, 0, st, a, splits, ws_ld);
     return cudaGetLastError();
 }
 
