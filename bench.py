@@ -18,7 +18,10 @@ use a collective.
 from __future__ import annotations
 
 import argparse
+import glob
+import hashlib
 import json
+import re
 import os
 import statistics
 import subprocess
@@ -36,8 +39,8 @@ import synth  # noqa: E402
 METRIC = "protected images/sec and checksum overhead % vs unprotected; conv % of GB300 peak"
 DEFAULT_WORKLOAD = "resnet18_imagenet"
 # bounded oracle samples (images) per workload: roughly 10-30 s of CPU work
-ORACLE_SAMPLE = {"lenet5": 256, "resnet18_cifar": 24, "campaign_resnet18_cifar": 24,
-                 "resnet18_imagenet": 16, "vgg16": 3}
+ORACLE_SAMPLE = {"lenet5": 4096, "resnet18_cifar": 512, "campaign_resnet18_cifar": 512,
+                 "resnet18_imagenet": 256, "vgg16": 32}
 
 
 def peaks():
@@ -151,6 +154,30 @@ def run_reference(args, wl, rank, world):
     print(json.dumps(line), flush=True)
 
 
+def source_fingerprint():
+    """Hash of the CUDA sources; ties recorded counters to the kernels they measured."""
+    h = hashlib.sha1()
+    for f in sorted(glob.glob(os.path.join(ROOT, "paper_2609_16742_gb300", "csrc", "*"))):
+        if f.endswith((".cu", ".cuh", ".h")):
+            with open(f, "rb") as fh:
+                h.update(fh.read())
+    return h.hexdigest()[:12]
+
+
+def recorded_traffic(workload, batch):
+    """DRAM bytes per launch of the tensor-core conv family from the committed
+    ncu summary of this workload, or None when the kernels changed since."""
+    path = os.path.join(ROOT, "profiles", "dram_traffic_%s_b%d.md" % (workload, batch))
+    if not os.path.exists(path):
+        return None, None
+    txt = open(path).read()
+    fp = re.search(r"source fingerprint: (\w+)", txt)
+    val = re.search(r"tensor-core conv family: \d+ launches, DRAM bytes per launch: (\d+)", txt)
+    if not fp or not val or fp.group(1) != source_fingerprint():
+        return None, os.path.relpath(path, ROOT) + " (kernels changed since the capture)"
+    return int(val.group(1)), os.path.relpath(path, ROOT)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -160,6 +187,8 @@ def main():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
     ap.add_argument("--simt-only", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--campaign-faults", type=int, default=1000,
+                    help="faults per precision of the fault-injection campaign (0: skip)")
     args = ap.parse_args()
 
     rank = int(os.environ.get("RANK", "0"))
@@ -322,7 +351,7 @@ def main():
                 "launches": si_n, "avg_launch_us": 1e3 * si_ms / max(si_n, 1),
                 "flops_per_launch": si_fl / max(si_n, 1)}
     roof["frac"] = roof["achieved"] / roof["peak"]
-    roof["traffic"] = None
+    roof["traffic"], roof["traffic_source"] = recorded_traffic(wl.name, B)
     roof["conv_share_of_step"] = (tc_ms + si_ms) / ms_p if ms_p else None
 
     cpu = None
@@ -331,6 +360,23 @@ def main():
         v, cores, dt = oracle_rate(wl, n_img)
         cpu = {"value": v, "unit": "images/s", "cores": cores, "kind": "oracle",
                "sample": "%d images of %s, one forward pass (%.1f s)" % (n_img, wl.name, dt)}
+
+    # fault-injection campaign on the CIFAR ResNet-18 (FP32 and FP16): detected
+    # fraction of critical faults and end-to-end time including re-execution
+    camp = None
+    if args.campaign_faults > 0:
+        from paper_2609_16742_gb300 import campaign
+        camp = {}
+        for prec in ("fp32", "fp16"):
+            c = campaign.run(prec, args.campaign_faults, seed=0, device=local)
+            camp[prec] = {"faults": c["faults"], "batch": c["batch"],
+                          "detected_fraction_of_critical": c["all"]["detected_fraction_of_critical"],
+                          "critical": c["all"]["critical"], "trials": c["all"]["trials"],
+                          "false_alarm_rate": c["all"]["false_alarm_rate"],
+                          "weights": c["weights"]["detected_fraction_of_critical"],
+                          "activations": c["activations"]["detected_fraction_of_critical"],
+                          "wall_s": c["wall_s"], "time_relative_to_fault_free": c["time_relative_to_fault_free"],
+                          "reexecuted_images": c["reexecuted_images"], "device_error": c["device_error"]}
 
     in_bytes = B * int(np.prod(wl.in_shape)) * 4
     out_bytes = B * (wl.n_classes * 4 + 4 + 1)
@@ -363,6 +409,7 @@ def main():
         "clocks": clocks,
         "device_error": err,
         "threshold": {"reference": r, "tau": tau},
+        "campaign": camp,
     }
     print(json.dumps(line), flush=True)
     if dist is not None:

@@ -1,0 +1,164 @@
+"""Fault-injection campaign (Sec. III-A) on the CIFAR-shaped ResNet-18.
+
+One trial = one seeded single-bit flip, drawn uniformly over the union of
+(element, bit) pairs of every convolution weight tensor and every
+convolution input activation tensor (ct_buffer_info), injected into one
+inference of a fixed batch (ct_inject + ct_infer), followed by
+ct_reexecute of the flagged images, as deployed.
+
+A weight flip touches every image of the batch: each image is one trial.
+An activation flip touches one image: that image is the trial.  An image is
+critical when its top-1 class differs from the fault-free run (a NaN logit
+counts as class -1, so it is always critical; ties go to the lowest index),
+detected when it is critical and flagged, a false alarm when it is flagged
+but not critical.
+
+Weights are those of the CIFAR ResNet-18 workload; evaluation and
+calibration inputs use the campaign workload's seeds.  The threshold
+(reference r and tau) is calibrated on calib_images fault-free images at
+alpha (nearest-rank quantile of |S - r|).
+
+    python -m paper_2609_16742_gb300.campaign --precision fp16 --faults 100000
+
+prints one JSON object.  The bookkeeping runs on the GPU (torch ops on the
+library's outputs); the host only draws the fault list and launches.
+"""
+import argparse
+import json
+import os
+import sys
+import time
+
+
+def run(precision="fp32", faults=1000, seed=0, batch=None, calib_images=10000, alpha=0.01, device=0,
+        reexecute=True):
+    sys.path.insert(0, os.path.dirname(os.path.dirname(os.path.abspath(__file__))))
+    import numpy as np
+    import torch
+    import synth
+    import paper_2609_16742_gb300 as ct
+
+    torch.cuda.set_device(device)
+    net = synth.workload("resnet18_cifar")            # weights
+    wl = synth.workload("campaign_resnet18_cifar")    # evaluation and calibration inputs
+    B = batch or wl.batch
+    m = ct.ct_build_workload(net, synth.make_params(net.layers, net.seed), precision=precision, max_batch=B,
+                             device=device)
+    stream = torch.cuda.current_stream()
+    # ---- calibration (fault-free) ----
+    n_cal = ((calib_images + B - 1) // B) * B
+    xc = torch.from_numpy(synth.make_input(wl, batch=n_cal, seed=wl.calib_seed)).cuda()
+    Sc = torch.empty(n_cal, device="cuda")
+    lc = torch.empty(B, wl.n_classes, device="cuda")
+    for i in range(0, n_cal, B):
+        ct.ct_infer(m, xc[i:i + B], B, lc, Sc[i:i + B], None, stream)
+    torch.cuda.synchronize()
+    r, tau = ct.ct_calibrate(Sc.cpu().numpy(), alpha)
+    ct.ct_set_threshold(m, r, tau)
+    del xc
+    # ---- fault-free evaluation batch ----
+    x = torch.from_numpy(synth.make_input(wl, batch=B)).cuda()
+    logits = torch.empty(B, wl.n_classes, device="cuda")
+    S = torch.empty(B, device="cuda")
+    flag = torch.empty(B, dtype=torch.uint8, device="cuda")
+
+    def top1(lg):
+        return torch.where(torch.isnan(lg).any(1), torch.full((lg.shape[0],), -1, device=lg.device,
+                                                               dtype=torch.long), lg.argmax(1))
+
+    ct.ct_infer(m, x, B, logits, S, flag, stream)
+    golden = top1(logits).clone()
+    ff_flags = int(flag.sum().item())
+    # fault-free step time (infer + re-execution of its flags) for the relative cost
+    for _ in range(3):
+        ct.ct_infer(m, x, B, logits, S, flag, stream)
+        ct.ct_reexecute(m, x, B, flag, logits, S, stream)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    n_ff = 20
+    for _ in range(n_ff):
+        ct.ct_infer(m, x, B, logits, S, flag, stream)
+        ct.ct_reexecute(m, x, B, flag, logits, S, stream)
+    torch.cuda.synchronize()
+    ff_step_s = (time.perf_counter() - t0) / n_ff
+
+    # ---- campaign ----
+    bufs = ct.ct_buffers(m, B)
+    sites = synth.draw_faults(bufs, faults, seed)
+    per_img = {}
+    for kind, layer, n_el, bits in bufs:
+        if kind == 1:
+            per_img[layer] = n_el // B
+    nb = 32 if precision == "fp32" else 16
+    # [kind, bit] counters on the GPU: trials, critical, detected, false alarms
+    cnt = torch.zeros(2, nb, 4, dtype=torch.long, device="cuda")
+    n_rerun = 0
+    ct.ct_kernel_count(m)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for kind, layer, e, bit in sites.tolist():
+        ct.ct_inject(m, kind, layer, e, bit)
+        ct.ct_infer(m, x, B, logits, S, flag, stream)
+        crit = top1(logits) != golden
+        fl = flag != 0
+        if kind == 0:
+            row = torch.stack([torch.full_like(crit, True).sum(), crit.sum(), (crit & fl).sum(),
+                               (~crit & fl).sum()])
+        else:
+            i = e // per_img[layer]
+            c, f = crit[i], fl[i]
+            row = torch.stack([torch.ones_like(c, dtype=torch.long), c.long(), (c & f).long(),
+                               (~c & f).long()])
+        cnt[kind, bit] += row
+        if reexecute:
+            n_rerun += ct.ct_reexecute(m, x, B, flag, logits, S, stream)
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - t0
+    kernels = ct.ct_kernel_count(m)
+    err = ct.ct_device_error(m)
+    c = cnt.cpu().numpy()
+
+    def summary(a):
+        trials, crit, det, fa = (int(v) for v in a)
+        non = trials - crit
+        return {"trials": trials, "critical": crit, "detected": det, "false_alarms": fa,
+                "detected_fraction_of_critical": det / crit if crit else None,
+                "false_alarm_rate": fa / non if non else None}
+
+    tot = c.sum(axis=(0, 1))
+    out = {
+        "precision": precision, "faults": int(faults), "seed": int(seed), "batch": B,
+        "threshold": {"reference": r, "tau": tau, "alpha": alpha, "calibration_images": n_cal},
+        "fault_free_flagged_images": ff_flags,
+        "all": summary(tot),
+        "weights": summary(c[0].sum(axis=0)),
+        "activations": summary(c[1].sum(axis=0)),
+        "by_bit": {str(b): summary(c[:, b].sum(axis=0)) for b in range(nb)},
+        "wall_s": wall,
+        "fault_free_wall_s": ff_step_s * faults,
+        "time_relative_to_fault_free": wall / (ff_step_s * faults),
+        "reexecuted_images": n_rerun,
+        "kernels_launched": kernels,
+        "device_error": err,
+    }
+    m.close()
+    return out
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
+    ap.add_argument("--precision", default="fp32", choices=["fp32", "fp16"])
+    ap.add_argument("--faults", type=int, default=1000)
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--calib-images", type=int, default=10000)
+    ap.add_argument("--alpha", type=float, default=0.01)
+    ap.add_argument("--no-reexecute", action="store_true")
+    args = ap.parse_args(argv)
+    out = run(args.precision, args.faults, args.seed, calib_images=args.calib_images, alpha=args.alpha,
+              reexecute=not args.no_reexecute)
+    print(json.dumps(out))
+    return 0 if out["device_error"] == 0 else 1
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,80 @@
+"""The fault-injection campaign of Sec. III-A on the CIFAR ResNet-18: a seeded
+subset of its faults against the oracle (per-image critical and flagged
+verdicts), and the campaign runner's bookkeeping."""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from _cache import params
+from _gpu import TOL, ct, onet, run, same_class
+
+pytestmark = pytest.mark.gpu
+
+
+def _model(prec, B):
+    net = synth.workload("resnet18_cifar")
+    return ct().ct_build_workload(net, params("resnet18_cifar"), precision=prec, max_batch=B)
+
+
+@pytest.mark.parametrize("prec", ["fp32", "fp16"])
+def test_campaign_faults_match_oracle(prec):
+    B, n_faults = 16, 24
+    wl = synth.workload("campaign_resnet18_cifar")
+    m = _model(prec, B)
+    net = onet("resnet18_cifar", prec)
+    x = synth.make_input(wl, batch=B)
+    xc = synth.make_input(wl, batch=256, seed=wl.calib_seed)
+    r, tau = oracle.calibrate(oracle.forward(net, xc)["S"], 0.01)
+    ct().ct_set_threshold(m, r, tau)
+    g_lg, _, _ = run(m, x)
+    o_g = oracle.forward(net, x)
+    top_o = oracle.top1(o_g["logits"])
+    bufs = ct().ct_buffers(m, B)
+    assert bufs == oracle.fault_buffers(net, B)
+    faults = synth.draw_faults(bufs, n_faults, seed=11)
+    per_img = {layer: n // B for kind, layer, n, bits in bufs if kind == 1}
+    n_cmp = n_near = crit_mismatch = 0
+    for kind, layer, e, bit in faults.tolist():
+        ct().ct_inject(m, kind, layer, e, bit)
+        lg, S, fl = run(m, x)
+        if kind == 0:
+            imgs, f = list(range(4)), oracle.Fault(0, layer, e, bit)
+        else:
+            img, off = divmod(e, per_img[layer])
+            imgs, f = [img], oracle.Fault(1, layer, off, bit)
+        o = oracle.forward(net, x[imgs], f)
+        for j, i in enumerate(imgs):
+            so, sg = o["S"][j], S[i]
+            assert same_class(sg, so), (kind, layer, e, bit, sg, so)
+            if np.isfinite(so):
+                assert abs(sg - so) <= TOL[prec] * max(abs(so), 1e-6), (kind, layer, e, bit, sg, so)
+            near = np.isfinite(so) and abs(abs(so - r) - tau) <= 0.01 * tau
+            if near:
+                n_near += 1
+            else:
+                assert bool(fl[i]) == bool(oracle.verdict([so], r, tau)[0]), (kind, layer, e, bit, sg, so)
+            lo = o["logits"][j]
+            crit_o = oracle.top1(lo[None])[0] != top_o[i]
+            crit_g = oracle.top1(lg[i][None])[0] != oracle.top1(g_lg[i][None])[0]
+            if crit_o != crit_g:
+                srt = np.sort(lo[np.isfinite(lo)])
+                assert len(srt) > 1 and srt[-1] - srt[-2] <= 2 * TOL[prec] * np.abs(lo).max()
+                crit_mismatch += 1
+            n_cmp += 1
+    assert n_cmp >= n_faults and crit_mismatch <= 1
+
+
+def test_campaign_runner_bookkeeping():
+    from paper_2609_16742_gb300 import campaign
+    out = campaign.run("fp16", faults=48, seed=3, calib_images=512)
+    assert out["device_error"] == 0
+    a = out["all"]
+    assert a["detected"] <= a["critical"] <= a["trials"]
+    assert a["false_alarms"] <= a["trials"] - a["critical"]
+    # a weight flip is one trial per image, an activation flip one trial
+    w, act = out["weights"], out["activations"]
+    assert w["trials"] % out["batch"] == 0
+    assert w["trials"] // out["batch"] + act["trials"] == 48
+    assert sum(v["trials"] for v in out["by_bit"].values()) == a["trials"]
+    assert out["kernels_launched"] > 48
