@@ -51,6 +51,12 @@ constexpr int BK = 64;             // channels per K block (128 bytes of fp16)
 constexpr int A_BYTES = BM * BK * 2;
 constexpr int NTHREADS = 320;      // 1 TMA warp, 1 MMA warp, 8 epilogue warps
 constexpr int N_EPI_WARPS = 8;
+// conv_tc_kernel: TC_NPROD TMA producer warps, one MMA warp, 8 epilogue warps
+constexpr int TC_NPROD = 4;
+constexpr int TC_MMA_WARP = TC_NPROD;
+constexpr int TC_EPI_WARP0 = TC_NPROD + 1;
+constexpr int TC_THREADS = 32 * (TC_NPROD + 1 + N_EPI_WARPS);
+constexpr int TC_CS = 4;           // CTAs per cluster sharing each B tile (N = 128, 256)
 
 enum CtMode { CT_NONE_ = 0, CT_MERGED = 1, CT_SEPARATE = 2 };
 
@@ -61,19 +67,23 @@ struct TcGeom {
     int tmem_cols;
     int m_tiles, n_tiles;
     int splits, kps, ws_ld;      // split-K: K blocks per split, workspace row length
+    int m_groups;                // clusters of CS consecutive M tiles (CS = 1: m_tiles)
     uint16_t coef_h;
 };
 
-// K-block range [lo, hi) and output tile of persistent work item `tile`
+// K-block range [lo, hi) and output tile of persistent work item `item`.
+// A work item of a cluster of cs CTAs is a group of cs consecutive M tiles
+// with the same N tile and K range; CTA `crank` of the cluster takes M tile
+// group * cs + crank (past the last M tile it computes rows it never stores).
 struct TileRef {
     int m0, n_tile, sp, kb_lo, kb_hi;
 };
-__device__ __forceinline__ TileRef tile_ref(int tile, const TcGeom &g) {
+__device__ __forceinline__ TileRef tile_ref(int item, const TcGeom &g, int cs, int crank) {
     TileRef t;
-    const int per = g.m_tiles * g.n_tiles;
-    t.sp = tile / per;
-    const int rt = tile - t.sp * per;
-    t.m0 = (rt / g.n_tiles) * BM;
+    const int per = g.m_groups * g.n_tiles;
+    t.sp = item / per;
+    const int rt = item - t.sp * per;
+    t.m0 = ((rt / g.n_tiles) * cs + crank) * BM;
     t.n_tile = rt % g.n_tiles;
     t.kb_lo = t.sp * g.kps;
     t.kb_hi = min(g.n_kb, t.kb_lo + g.kps);
@@ -221,8 +231,8 @@ __device__ __forceinline__ void store_checksum_pre(float ctv, const CsIn &c, con
 // barrier round trip).  A single TMEM buffer holds the chains; for
 // BN <= 128 the epilogue copies it to registers and releases it before its
 // global stores, so the next tile's MMAs overlap the stores.
-template <int BN, int STAGES, int SUB, int NCH>
-__global__ void __launch_bounds__(NTHREADS, 1)
+template <int BN, int STAGES, int SUB, int NCH, int CS>
+__global__ void __launch_bounds__(TC_THREADS, 1)
 conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
                const ConvArgs a, const TcGeom g) {
     constexpr int B_ROWS = BN + 16;                       // 16 constant carry-through rows
@@ -230,40 +240,62 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
     constexpr int B_TMA_BYTES = BN * BK * 2;
     constexpr int CH = BN + 16;                           // TMEM columns per chain
     constexpr bool EARLY = BN <= 128;                     // release TMEM before the stores
+    // N = 256: two 256-column accumulators fill TMEM, so the carry-through
+    // column is summed on CUDA cores from the centre-tap A tiles in shared
+    // memory by the warps of the producer group that do not issue copies
+    // (they consume every stage, like the MMA warp), and the epilogue of one
+    // tile overlaps the MMAs of the next
+    constexpr bool DBUF = !EARLY;
+    static_assert(!DBUF || CS == 1, "the carry-through warps release stages of their own CTA only");
+    // producer warps (each owns whole ring slots) and carry-through warps
+    constexpr int NPROD = DBUF ? 2 : STAGES % 4 == 0 ? 4 : STAGES % 3 == 0 ? 3 : STAGES % 2 == 0 ? 2 : 1;
+    constexpr int NCT = DBUF ? TC_NPROD - NPROD : 0;
+    static_assert(NPROD <= TC_NPROD && STAGES % NPROD == 0, "producer warps must own whole ring slots");
+    static_assert(!DBUF || (NCT > 0 && BM % (32 * NCT) == 0), "carry-through warps split the tile rows");
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint8_t *As = smem;                                   // [STAGES][SUB][A_BYTES]
     uint8_t *Bs = As + STAGES * SUB * A_BYTES;            // [STAGES][SUB][B_SUB_BYTES]
     uint8_t *CTt = Bs + STAGES * SUB * B_SUB_BYTES;       // separate 16-row carry-through tile
-    uint64_t *full = (uint64_t *)(CTt + 16 * BK * 2);
+    float *ct_sum = (float *)(CTt + 16 * BK * 2);          // [2][BM] carry-through sums (DBUF)
+    uint64_t *full = (uint64_t *)(ct_sum + 2 * BM);
     uint64_t *empty = full + STAGES;
-    uint64_t *acc_full = empty + STAGES;
-    uint64_t *acc_empty = acc_full + 1;
-    uint32_t *tmem_holder = (uint32_t *)(acc_empty + 1);
+    uint64_t *acc_full = empty + STAGES;                  // [2]
+    uint64_t *acc_empty = acc_full + 2;                   // [2]
+    uint64_t *ct_ready = acc_empty + 2;                   // [2]
+    uint32_t *tmem_holder = (uint32_t *)(ct_ready + 2);
     volatile uint32_t *abort_flag = tmem_holder + 1;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int num_tiles = g.m_tiles * g.n_tiles * g.splits;
+    // clusters of CS CTAs share each B tile: CTA r loads rows r * BN / CS ..
+    // of it and multicasts them to the whole cluster
+    const int crank = CS > 1 ? (int)cluster_ctarank() : 0;
+    const int cid = blockIdx.x / CS, ncl = gridDim.x / CS;
+    const uint16_t cmask = (uint16_t)((1u << CS) - 1u);
+    const int num_items = g.m_groups * g.n_tiles * g.splits;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(smem_u32(&full[s]), 1);
-            mbar_init(smem_u32(&empty[s]), 1);
+            mbar_init(smem_u32(&empty[s]), CS + NCT);   // MMA commits (every CTA) + carry-through warps
         }
-        mbar_init(smem_u32(acc_full), 1);
-        mbar_init(smem_u32(acc_empty), N_EPI_WARPS);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(smem_u32(&acc_full[b]), 1);
+            mbar_init(smem_u32(&acc_empty[b]), N_EPI_WARPS);
+            mbar_init(smem_u32(&ct_ready[b]), NCT > 0 ? NCT : 1);
+        }
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
-    if (warp == 1) {
+    if (warp == TC_MMA_WARP) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_holder)),
                      "r"((uint32_t)g.tmem_cols));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
     }
-    if (warp >= 2) {
+    if (warp >= TC_EPI_WARP0) {
         // constant carry-through rows: row 0 = coef, rows 1..15 = 0 (swizzle-invariant)
         const uint32_t coef2 = (uint32_t)g.coef_h | ((uint32_t)g.coef_h << 16);
-        const int t = threadIdx.x - 64;
+        const int t = threadIdx.x - 32 * TC_EPI_WARP0;
         for (int sb = 0; sb < STAGES * SUB; ++sb) {
             uint32_t *rows = (uint32_t *)(Bs + sb * B_SUB_BYTES + BN * BK * 2);
             for (int i = t; i < 16 * BK / 2; i += 32 * N_EPI_WARPS) rows[i] = (i < BK / 2) ? coef2 : 0u;
@@ -274,23 +306,31 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
     }
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
+    // peers multicast into this CTA's shared memory and barriers only after
+    // every CTA of the cluster has initialised its barriers
+    if (CS > 1) cluster_sync();
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem = *tmem_holder;
     // the previous kernel's outputs (and any fault flip) are visible from here
     pdl_wait();
     pdl_trigger();
 
-    if (warp == 0) {
-        // ---------------- TMA producer (whole warp, one lane issues) ----------------
+    if (warp < NPROD) {
+        // ---------------- TMA producers ----------------
+        // One lane of one thread issues TMA copies one after another, so the
+        // ring slots are dealt to NPROD producer warps whose copies proceed
+        // in parallel.  Slot s always belongs to warp s % NPROD (NPROD
+        // divides STAGES): every slot is refilled by one warp in order, so a
+        // parity wait on its empty barrier can never see a phase two ahead.
         if (elect_one()) {
             asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&amap) : "memory");
             asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&bmap) : "memory");
         }
         __syncwarp();
         int it = 0;
-        for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
+        for (int tile = cid; tile < num_items; tile += ncl) {
             if (__any_sync(0xffffffffu, *abort_flag)) break;
-            const TileRef tr = tile_ref(tile, g);
+            const TileRef tr = tile_ref(tile, g, CS, crank);
             const int m0 = tr.m0, n_tile = tr.n_tile;
             const int nimg = m0 / g.PQ, rem = m0 % g.PQ;
             const int p = rem / g.Q, q = rem % g.Q;
@@ -298,6 +338,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
             bool ok = true;
             for (int kb0 = tr.kb_lo; kb0 < tr.kb_hi; kb0 += SUB, ++it) {
                 const int s = it % STAGES;
+                if (s % NPROD != warp) continue;
                 const uint32_t ph = (uint32_t)(it / STAGES) & 1u;
                 if (!warp_wait(smem_u32(&empty[s]), ph ^ 1u, a.err, 1u)) { ok = false; break; }
                 const int nsub = min(SUB, tr.kb_hi - kb0);
@@ -311,27 +352,33 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
                         const int r = tap / g.S, sx = tap % g.S;
                         tma_load_im2col(smem_u32(As + (s * SUB + j) * A_BYTES), &amap, fb, c0, w0, h0, nimg,
                                         (uint16_t)sx, (uint16_t)r);
-                        tma_load_2d(smem_u32(Bs + (s * SUB + j) * B_SUB_BYTES), &bmap, fb, tap * g.C + c0,
-                                    n_tile * BN);
+                        if (CS == 1)
+                            tma_load_2d(smem_u32(Bs + (s * SUB + j) * B_SUB_BYTES), &bmap, fb, tap * g.C + c0,
+                                        n_tile * BN);
+                        else
+                            tma_load_2d_mc(smem_u32(Bs + (s * SUB + j) * B_SUB_BYTES + crank * (BN / CS) * BK * 2),
+                                           &bmap, fb, tap * g.C + c0, n_tile * BN + crank * (BN / CS), cmask);
                     }
                 }
                 __syncwarp();
             }
             if (!ok) { if (lane == 0) *abort_flag = 1; break; }
         }
-    } else if (warp == 1) {
+    } else if (warp == TC_MMA_WARP) {
         // ---------------- MMA issuer (whole warp, one lane issues) ----------------
         const uint32_t id_main = idesc_f16(BM, BN);
         const uint32_t id_merged = idesc_f16(BM, BN + 16);
         const uint32_t id_ct = idesc_f16(BM, 16);
         const uint32_t ct_base = smem_u32(CTt);
         int it = 0, lt = 0;
-        for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++lt) {
+        for (int tile = cid; tile < num_items; tile += ncl, ++lt) {
             if (__any_sync(0xffffffffu, *abort_flag)) break;
-            const TileRef tr = tile_ref(tile, g);
+            const TileRef tr = tile_ref(tile, g, CS, crank);
             const int n_tile = tr.n_tile;
             const bool ct_here = g.ct_mode != CT_NONE_ && n_tile == 0;
-            if (!warp_wait(smem_u32(acc_empty), ((uint32_t)lt & 1u) ^ 1u, a.err, 8u)) {
+            const int ab = DBUF ? (lt & 1) : 0;
+            const uint32_t aph = DBUF ? ((uint32_t)(lt >> 1) & 1u) : ((uint32_t)lt & 1u);
+            if (!warp_wait(smem_u32(&acc_empty[ab]), aph ^ 1u, a.err, 8u)) {
                 if (lane == 0) *abort_flag = 1;
                 break;
             }
@@ -347,7 +394,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
                 for (int j = 0; j < nsub; ++j) {
                     const int kb = kb0 + j;
                     const int kr = kb - tr.kb_lo;               // position within this split
-                    const uint32_t d = tmem + (uint32_t)((kr % NCH) * CH);
+                    const uint32_t d = DBUF ? tmem + (uint32_t)(ab * BN) : tmem + (uint32_t)((kr % NCH) * CH);
                     const bool centre = kb < g.cpb;
                     const uint32_t a_base = smem_u32(As + (s * SUB + j) * A_BYTES);
                     const uint32_t b_base = smem_u32(Bs + (s * SUB + j) * B_SUB_BYTES);
@@ -357,7 +404,9 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
                         const uint64_t bd = smem_desc_sw128(b_base + k16 * 32);
                         const uint32_t acc = (kr >= NCH || k16 > 0) ? 1u : 0u;   // first use of the chain
                         if (leader) {
-                            if (ct_here && centre && g.ct_mode == CT_MERGED) {
+                            if (DBUF) {
+                                umma_f16(d, ad, bd, id_main, acc);
+                            } else if (ct_here && centre && g.ct_mode == CT_MERGED) {
                                 umma_f16(d, ad, bd, id_merged, acc);
                             } else {
                                 umma_f16(d, ad, bd, id_main, acc);
@@ -367,16 +416,78 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
                         }
                     }
                 }
-                if (leader) umma_commit(smem_u32(&empty[s]));
+                if (leader) {
+                    if (CS == 1) umma_commit(smem_u32(&empty[s]));
+                    else umma_commit_mc(smem_u32(&empty[s]), cmask);
+                }
                 __syncwarp();
             }
             if (!ok) { if (lane == 0) *abort_flag = 1; break; }
-            if (elect_one()) umma_commit(smem_u32(acc_full));   // fires when the tile's MMAs have completed
+            if (elect_one()) umma_commit(smem_u32(&acc_full[ab]));   // fires when the tile's MMAs have completed
             __syncwarp();
         }
-    } else {
-        // ---------------- epilogue: warps 2..9 ----------------
-        const int ep = warp - 2;
+    } else if (warp < TC_NPROD) {
+        if (NCT > 0) {
+            // ---------------- carry-through sums (N = 256) ----------------
+            // Consumes every stage in order (arrives on its empty barrier);
+            // on the centre-tap K blocks of the first N tile it adds each A
+            // row's 64 channels (the 128-byte swizzle only permutes chunks
+            // within a row).  Carry-through warp w takes tile rows
+            // lane + 32 (w + NCT i).
+            constexpr int RPL = BM / (32 * (NCT > 0 ? NCT : 1));   // rows per lane
+            const float coef = __half2float(__ushort_as_half(g.coef_h));
+            const int w = warp - NPROD;
+            int it = 0, lt = 0;
+            bool ok = true;
+            for (int tile = cid; tile < num_items && ok; tile += ncl, ++lt) {
+                if (__any_sync(0xffffffffu, *abort_flag)) break;
+                const TileRef tr = tile_ref(tile, g, CS, crank);
+                const bool ct_here = g.ct_mode != CT_NONE_ && tr.n_tile == 0;
+                const int ab = lt & 1;
+                float acc[RPL];
+#pragma unroll
+                for (int i = 0; i < RPL; ++i) acc[i] = 0.f;
+                for (int kb0 = tr.kb_lo; kb0 < tr.kb_hi; kb0 += SUB, ++it) {
+                    const int s = it % STAGES;
+                    if (!warp_wait(smem_u32(&full[s]), (uint32_t)(it / STAGES) & 1u, a.err, 2u)) { ok = false; break; }
+                    const int nsub = min(SUB, tr.kb_hi - kb0);
+                    for (int j = 0; j < nsub; ++j) {
+                        if (!(ct_here && kb0 + j < g.cpb)) continue;
+#pragma unroll
+                        for (int i = 0; i < RPL; ++i) {
+                            const int row = lane + 32 * (w + NCT * i);
+                            const uint4 *rp = reinterpret_cast<const uint4 *>(As + (s * SUB + j) * A_BYTES + row * 128);
+                            float sum = 0.f;
+#pragma unroll
+                            for (int c = 0; c < 8; ++c) {
+                                const uint4 v = rp[c];
+                                const __half2 *h = reinterpret_cast<const __half2 *>(&v);
+#pragma unroll
+                                for (int e = 0; e < 4; ++e) {
+                                    const float2 f = __half22float2(h[e]);
+                                    sum += f.x + f.y;
+                                }
+                            }
+                            acc[i] += sum;
+                        }
+                    }
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(smem_u32(&empty[s]));
+                }
+                if (!ok) break;
+                // ct_sum[ab] is free once the epilogue released accumulator ab
+                if (!warp_wait(smem_u32(&acc_empty[ab]), ((uint32_t)(lt >> 1) & 1u) ^ 1u, a.err, 8u)) { ok = false; break; }
+#pragma unroll
+                for (int i = 0; i < RPL; ++i) ct_sum[ab * BM + lane + 32 * (w + NCT * i)] = coef * acc[i];
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&ct_ready[ab]));
+            }
+            if (!ok && lane == 0) *abort_flag = 1;
+        }
+    } else if (warp >= TC_EPI_WARP0) {
+        // ---------------- epilogue: 8 warps ----------------
+        // (producer warps beyond NPROD have no role)
+        const int ep = warp - TC_EPI_WARP0;
         const int quad = warp & 3;                 // TMEM lanes this warp may read
         const int half = ep >> 2;                  // which half of the tile's channels
         const int row = quad * 32 + lane;
@@ -384,8 +495,8 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
         const FaultDelta fd = a.fd;
         const bool split = g.splits > 1;
         int lt = 0;
-        for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++lt) {
-            const TileRef tr = tile_ref(tile, g);
+        for (int tile = cid; tile < num_items; tile += ncl, ++lt) {
+            const TileRef tr = tile_ref(tile, g, CS, crank);
             const int m0 = tr.m0, n_tile = tr.n_tile;
             // residual loads in flight while the MMAs run
             Res16 rs[BN / 32];
@@ -408,11 +519,14 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
             const int chains = min(NCH, tr.kb_hi - tr.kb_lo);                    // chains that received MMAs
             // chains whose first K block is a centre block hold a carry-through column
             const int ct_chains = max(0, min(NCH, min(g.cpb, tr.kb_hi) - tr.kb_lo));
-            bool ok = mbar_wait(smem_u32(acc_full), (uint32_t)lt & 1u, a.err, 4u) && !*abort_flag;
+            const int ab = DBUF ? (lt & 1) : 0;
+            const uint32_t aph = DBUF ? ((uint32_t)(lt >> 1) & 1u) : ((uint32_t)lt & 1u);
+            bool ok = mbar_wait(smem_u32(&acc_full[ab]), aph, a.err, 4u) && !*abort_flag;
+            if (DBUF) ok = ok && mbar_wait(smem_u32(&ct_ready[ab]), aph, a.err, 4u);
             ok = __all_sync(0xffffffffu, ok);      // tcgen05.ld below is warp-collective
             if (!ok) break;
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-            const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
+            const uint32_t trow = tmem + (uint32_t)(ab * BN) + ((uint32_t)(quad * 32) << 16);
             const int m = m0 + row;
             const bool valid = m < g.M;
             const int mm = valid ? m : 0;
@@ -444,7 +558,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
                     for (int ch = 0; ch < ct_chains; ++ch) ctv += tmem_ld1(trow + ch * CH + BN);
                 asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
                 __syncwarp();
-                if (lane == 0) mbar_arrive(smem_u32(acc_empty));   // accumulators free for the next tile
+                if (lane == 0) mbar_arrive(smem_u32(&acc_empty[0]));   // accumulators free for the next tile
                 if (valid && split) {
                     float *wrow = a.ws + ((size_t)tr.sp * g.M + m) * g.ws_ld;
 #pragma unroll
@@ -477,19 +591,24 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
                         store_chunk_pre(v, rs[(c - half * (BN / 2)) / 16], a, g.K, (size_t)m, n0 + c, fsrc);
                     }
                 }
-                if (do_cs && g.ct_mode != CT_NONE_)
-                    for (int ch = 0; ch < ct_chains; ++ch) ctv += tmem_ld1(trow + ch * CH + BN);
+                if (do_cs && g.ct_mode != CT_NONE_) ctv = ct_sum[ab * BM + row];
                 if (do_cs && valid && split) a.ws[((size_t)tr.sp * g.M + m) * g.ws_ld + g.K] = ctv;
                 else if (do_cs && valid) store_checksum_pre(ctv, csv, a, g, m, fsrc);
                 asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
                 __syncwarp();
-                if (lane == 0) mbar_arrive(smem_u32(acc_empty));
+                if (lane == 0) mbar_arrive(smem_u32(&acc_empty[ab]));
             }
         }
     }
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
-    if (warp == 1) {
+    if (CS > 1) {
+        // the MMAs of this CTA have completed (the epilogue saw every tile);
+        // their commits may still arrive on the peers' barriers: no CTA
+        // leaves before the whole cluster is done
+        cluster_sync();
+    }
+    if (warp == TC_MMA_WARP) {
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)g.tmem_cols));
     }
@@ -1115,7 +1234,8 @@ bool load_encoders() {
 
 template <int BN, int STAGES, int SUB>
 size_t smem_bytes() {
-    return 1024 + (size_t)STAGES * SUB * (A_BYTES + (BN + 16) * BK * 2) + 16 * BK * 2 + 8 * (2 * STAGES + 2) + 16;
+    return 1024 + (size_t)STAGES * SUB * (A_BYTES + (BN + 16) * BK * 2) + 16 * BK * 2 + 2 * BM * 4 +
+           8 * (2 * STAGES + 6) + 16;
 }
 
 uint16_t coef_half_bits(float c) {
@@ -1140,8 +1260,10 @@ int device_sm_count() {
 struct TcPlan {
     CUtensorMap amap;
     CUtensorMap bmap;
+    CUtensorMap bmap_mc;         // B slices of BN / cs rows for the cluster kernels
     TcGeom g;
     int BN, n_tiles, sms;
+    int cs, max_clusters;        // cluster size of the multicast variant (1: none)
     size_t smem;
 };
 
@@ -1195,15 +1317,44 @@ TcPlan *tc_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, cons
     cudaError_t e;
     if (pl->BN == 64) {
         pl->smem = smem_bytes<64, 4, 2>();
-        e = cudaFuncSetAttribute(conv_tc_kernel<64, 4, 2, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
+        e = cudaFuncSetAttribute(conv_tc_kernel<64, 4, 2, 4, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
     } else if (pl->BN == 128) {
         pl->smem = smem_bytes<128, 3, 2>();
-        e = cudaFuncSetAttribute(conv_tc_kernel<128, 3, 2, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
+        e = cudaFuncSetAttribute(conv_tc_kernel<128, 3, 2, 2, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(conv_tc_kernel<128, 3, 2, 2, TC_CS>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
     } else {
         pl->smem = smem_bytes<256, 4, 1>();
-        e = cudaFuncSetAttribute(conv_tc_kernel<256, 4, 1, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
+        e = cudaFuncSetAttribute(conv_tc_kernel<256, 4, 1, 1, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
     }
     if (e != cudaSuccess) { if (why) *why = "shared memory attribute"; delete pl; return nullptr; }
+    // cluster variant: B slices of BN / TC_CS rows multicast to TC_CS CTAs
+    pl->cs = 1;
+    pl->max_clusters = 0;
+    if (pl->BN == 128) {
+        cuuint32_t box_mc[2] = {BK, (cuuint32_t)(pl->BN / TC_CS)};
+        r = g_encode_tiled(&pl->bmap_mc, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void *>(w_dev), bdim, bstr,
+                           box_mc, bes, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(TC_CS * 64);
+        cfg.blockDim = dim3(TC_THREADS);
+        cfg.dynamicSmemBytes = pl->smem;
+        cudaLaunchAttribute at[1];
+        at[0].id = cudaLaunchAttributeClusterDimension;
+        at[0].val.clusterDim.x = TC_CS;
+        at[0].val.clusterDim.y = 1;
+        at[0].val.clusterDim.z = 1;
+        cfg.attrs = at;
+        cfg.numAttrs = 1;
+        int n = 0;
+        cudaError_t oe = cudaOccupancyMaxActiveClusters(&n, conv_tc_kernel<128, 3, 2, 2, TC_CS>, &cfg);
+        if (r == CUDA_SUCCESS && oe == cudaSuccess && n > 0) {
+            pl->cs = TC_CS;
+            pl->max_clusters = n;
+        }
+        cudaGetLastError();
+    }
     return pl;
 }
 
@@ -1217,11 +1368,22 @@ cudaError_t launch_conv_tc(const ConvArgs &a, const void *plan, cudaStream_t st,
     g.ws_ld = (g.K + 1 + 3) & ~3;
     g.splits = (a.K % 8 == 0) ? splitk_choose(tiles, g.n_kb, 4, pl->sms, g.M, g.ws_ld, a.ws ? a.ws_bytes : 0) : 1;
     g.kps = (g.n_kb + g.splits - 1) / g.splits;
-    const int items = tiles * g.splits;
-    dim3 grid(items < pl->sms ? items : pl->sms);
-    if (pl->BN == 64) pdl_launch(conv_tc_kernel<64, 4, 2, 4>, grid, NTHREADS, pl->smem, st, pl->amap, pl->bmap, a, g);
-    else if (pl->BN == 128) pdl_launch(conv_tc_kernel<128, 3, 2, 2>, grid, NTHREADS, pl->smem, st, pl->amap, pl->bmap, a, g);
-    else pdl_launch(conv_tc_kernel<256, 4, 1, 1>, grid, NTHREADS, pl->smem, st, pl->amap, pl->bmap, a, g);
+    g.m_groups = g.m_tiles;
+    if (pl->cs > 1 && g.splits == 1 && g.m_tiles >= 4 * pl->cs) {
+        // clusters of cs CTAs on groups of cs consecutive M tiles, sharing B
+        g.m_groups = (g.m_tiles + pl->cs - 1) / pl->cs;
+        const int items = g.m_groups * g.n_tiles;
+        const int ncl = items < pl->max_clusters ? items : pl->max_clusters;
+        dim3 grid(ncl * pl->cs);
+        pdl_launch_cluster(conv_tc_kernel<128, 3, 2, 2, TC_CS>, grid, TC_THREADS, pl->smem, st, TC_CS, pl->amap,
+                           pl->bmap_mc, a, g);
+    } else {
+        const int items = tiles * g.splits;
+        dim3 grid(items < pl->sms ? items : pl->sms);
+        if (pl->BN == 64) pdl_launch(conv_tc_kernel<64, 4, 2, 4, 1>, grid, TC_THREADS, pl->smem, st, pl->amap, pl->bmap, a, g);
+        else if (pl->BN == 128) pdl_launch(conv_tc_kernel<128, 3, 2, 2, 1>, grid, TC_THREADS, pl->smem, st, pl->amap, pl->bmap, a, g);
+        else pdl_launch(conv_tc_kernel<256, 4, 1, 1, 1>, grid, TC_THREADS, pl->smem, st, pl->amap, pl->bmap, a, g);
+    }
     cudaError_t e = cudaGetLastError();
     if (n_kernels) *n_kernels = 1;
     if (e != cudaSuccess || g.splits == 1) return e;
