@@ -251,7 +251,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
     constexpr int NPROD = DBUF ? 2 : STAGES % 4 == 0 ? 4 : STAGES % 3 == 0 ? 3 : STAGES % 2 == 0 ? 2 : 1;
     constexpr int NCT = DBUF ? TC_NPROD - NPROD : 0;
     static_assert(NPROD <= TC_NPROD && STAGES % NPROD == 0, "producer warps must own whole ring slots");
-    static_assert(!DBUF || (NCT > 0 && BM % (32 * NCT) == 0), "carry-through warps split the tile rows");
+    static_assert(!DBUF || (NCT > 0 && BM % (32 * (NCT > 0 ? NCT : 1)) == 0), "carry-through warps split the tile rows");
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint8_t *As = smem;                                   // [STAGES][SUB][A_BYTES]
@@ -390,33 +390,34 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
                 if (!warp_wait(smem_u32(&full[s]), ph, a.err, 2u)) { ok = false; break; }
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                 const int nsub = min(SUB, tr.kb_hi - kb0);
-                const bool leader = elect_one();
-                for (int j = 0; j < nsub; ++j) {
-                    const int kb = kb0 + j;
-                    const int kr = kb - tr.kb_lo;               // position within this split
-                    const uint32_t d = DBUF ? tmem + (uint32_t)(ab * BN) : tmem + (uint32_t)((kr % NCH) * CH);
-                    const bool centre = kb < g.cpb;
-                    const uint32_t a_base = smem_u32(As + (s * SUB + j) * A_BYTES);
-                    const uint32_t b_base = smem_u32(Bs + (s * SUB + j) * B_SUB_BYTES);
+                if (elect_one()) {
+                    // descriptors advance 32 bytes (2 in the 16-byte address field)
+                    // per 16-element K step; the instruction choice is per K block
+                    for (int j = 0; j < nsub; ++j) {
+                        const int kb = kb0 + j;
+                        const int kr = kb - tr.kb_lo;               // position within this split
+                        const uint32_t d = DBUF ? tmem + (uint32_t)(ab * BN) : tmem + (uint32_t)((kr % NCH) * CH);
+                        const bool centre = kb < g.cpb;
+                        const uint64_t ad0 = smem_desc_sw128(smem_u32(As + (s * SUB + j) * A_BYTES));
+                        const uint64_t bd0 = smem_desc_sw128(smem_u32(Bs + (s * SUB + j) * B_SUB_BYTES));
+                        const uint32_t acc0 = kr >= NCH ? 1u : 0u;  // first use of the chain
+                        if (!DBUF && ct_here && centre && g.ct_mode == CT_SEPARATE) {
+                            const uint64_t cd0 = smem_desc_sw128(ct_base);
 #pragma unroll
-                    for (int k16 = 0; k16 < BK / 16; ++k16) {
-                        const uint64_t ad = smem_desc_sw128(a_base + k16 * 32);
-                        const uint64_t bd = smem_desc_sw128(b_base + k16 * 32);
-                        const uint32_t acc = (kr >= NCH || k16 > 0) ? 1u : 0u;   // first use of the chain
-                        if (leader) {
-                            if (DBUF) {
-                                umma_f16(d, ad, bd, id_main, acc);
-                            } else if (ct_here && centre && g.ct_mode == CT_MERGED) {
-                                umma_f16(d, ad, bd, id_merged, acc);
-                            } else {
-                                umma_f16(d, ad, bd, id_main, acc);
-                                if (ct_here && centre && g.ct_mode == CT_SEPARATE)
-                                    umma_f16(d + BN, ad, smem_desc_sw128(ct_base + k16 * 32), id_ct, acc);
+                            for (int k16 = 0; k16 < BK / 16; ++k16) {
+                                umma_f16(d, ad0 + 2 * k16, bd0 + 2 * k16, id_main, k16 ? 1u : acc0);
+                                umma_f16(d + BN, ad0 + 2 * k16, cd0 + 2 * k16, id_ct, k16 ? 1u : acc0);
                             }
+                        } else {
+                            const uint32_t idm = (!DBUF && ct_here && centre && g.ct_mode == CT_MERGED) ? id_merged : id_main;
+#pragma unroll
+                            for (int k16 = 0; k16 < BK / 16; ++k16)
+                                umma_f16(d, ad0 + 2 * k16, bd0 + 2 * k16, idm, k16 ? 1u : acc0);
                         }
                     }
                 }
-                if (leader) {
+                __syncwarp();
+                if (elect_one()) {
                     if (CS == 1) umma_commit(smem_u32(&empty[s]));
                     else umma_commit_mc(smem_u32(&empty[s]), cmask);
                 }
@@ -1364,9 +1365,11 @@ cudaError_t launch_conv_tc(const ConvArgs &a, const void *plan, cudaStream_t st,
     g.M = a.N * a.P * a.Q;
     g.m_tiles = (g.M + BM - 1) / BM;
     const int tiles = g.m_tiles * g.n_tiles;
-    // split K when the output tiles leave most SMs idle (at least 4 K blocks per split)
+    // split K when the output tiles leave most SMs idle (at least 4 K blocks
+    // per split; about half the SMs busy: more splits cost more in partial
+    // sums than they gain, measured on 4-16 image batches)
     g.ws_ld = (g.K + 1 + 3) & ~3;
-    g.splits = (a.K % 8 == 0) ? splitk_choose(tiles, g.n_kb, 4, pl->sms, g.M, g.ws_ld, a.ws ? a.ws_bytes : 0) : 1;
+    g.splits = (a.K % 8 == 0) ? splitk_choose(tiles, g.n_kb, 4, pl->sms / 2, g.M, g.ws_ld, a.ws ? a.ws_bytes : 0) : 1;
     g.kps = (g.n_kb + g.splits - 1) / g.splits;
     g.m_groups = g.m_tiles;
     if (pl->cs > 1 && g.splits == 1 && g.m_tiles >= 4 * pl->cs) {
