@@ -222,6 +222,17 @@ ct_status ct_run_host(ct_model *m, const float *input_host, int32_t batch, float
 ct_status ct_calibrate(const float *S_host, int64_t n, double alpha, double *reference,
                        double *tau);
 
+/* ct_fi_threshold -- Sec. II-C FI-based threshold, host arithmetic: from a
+ * fault-injection campaign on calibration inputs, with S_host[i] the
+ * accumulated-checksum neuron of image trial i and critical[i] != 0 when
+ * the fault changed its top-1 class, tau = the nearest-rank
+ * ceil((1 - alpha) * m)-th smallest |S - reference| over the m non-critical
+ * trials (a non-finite S counts as an infinite deviation), so that at most
+ * alpha of them are flagged.  CT_EINVAL for n < 1, alpha outside [0, 1) or
+ * no non-critical trial. */
+ct_status ct_fi_threshold(const float *S_host, const uint8_t *critical, int64_t n, double reference,
+                          double alpha, double *tau);
+
 /* Fault-able buffers of the protected network for a given batch, in the
  * order used by campaign drivers: every conv weight tensor, then every
  * distinct tensor read by a convolution (the network input excluded),

@@ -492,6 +492,38 @@ def calibrate(S: np.ndarray, alpha: float):
     return r, float(dev[rank - 1])
 
 
+def fi_threshold(S: np.ndarray, critical: np.ndarray, r: float, alpha: float) -> float:
+    """Sec. II-C FI-based threshold: tau such that at most alpha of the
+    non-critical fault trials of a calibration campaign are flagged.
+
+    Deviations |S - r| of the non-critical trials (a non-finite S is an
+    infinite deviation); tau is their nearest-rank ceil((1 - alpha) * m)-th
+    smallest value, as in calibrate().
+    """
+    S = np.asarray(S, dtype=np.float64)
+    crit = np.asarray(critical).astype(bool)
+    dev = np.abs(S[~crit] - r)
+    dev = np.where(np.isfinite(dev), dev, np.inf)
+    assert dev.size > 0
+    dev = np.sort(dev)
+    rank = int(math.ceil((1.0 - alpha) * len(dev)))
+    rank = min(max(rank, 1), len(dev))
+    return float(dev[rank - 1])
+
+
+def detection_rates(S: np.ndarray, critical: np.ndarray, r: float, tau: float):
+    """Sec. III-A metrics: (TPR, FPR, Youden's J = TPR - FPR).
+
+    TPR = flagged fraction of critical trials, FPR = flagged fraction of
+    non-critical trials, with the verdict of Sec. II-B (NOT |S - r| <= tau).
+    """
+    crit = np.asarray(critical).astype(bool)
+    flag = verdict(np.asarray(S, dtype=np.float64), r, tau).astype(bool)
+    tpr = float(flag[crit].mean()) if crit.any() else float("nan")
+    fpr = float(flag[~crit].mean()) if (~crit).any() else float("nan")
+    return tpr, fpr, tpr - fpr
+
+
 # ---------------------------------------------------------------------------
 # Second code path: the checksum recursion on the unprotected network
 # ---------------------------------------------------------------------------

@@ -35,6 +35,7 @@ _STATUS = {0: "CT_OK", 1: "CT_EINVAL", 2: "CT_ENOMEM", 3: "CT_ECUDA", 4: "CT_EST
 EXPORTS = ["ct_build", "ct_set_threshold", "ct_get_threshold", "ct_infer", "ct_inject",
            "ct_clear_faults", "ct_reexecute", "ct_run_host", "ct_calibrate", "ct_buffer_count",
            "ct_buffer_info", "ct_profile_enable", "ct_profile_read", "ct_launches_per_infer", "ct_kernel_count",
+           "ct_fi_threshold",
            "ct_copy_activation", "ct_device_error", "ct_destroy", "ct_strerror",
            "ct_reexecute_noalloc"]
 
@@ -89,6 +90,7 @@ def lib():
             "ct_reexecute_noalloc": [vp, vp, i32, vp, vp, vp, P(i32), vp],
             "ct_run_host": [vp, vp, i32, vp, vp, vp, P(i32), vp],
             "ct_calibrate": [vp, i64, dbl, P(dbl), P(dbl)],
+            "ct_fi_threshold": [vp, vp, i64, dbl, dbl, P(dbl)],
             "ct_buffer_count": [vp, i32, P(i32)],
             "ct_buffer_info": [vp, i32, i32, P(i32), P(i32), P(i64), P(i32)],
             "ct_profile_enable": [vp, i32],
@@ -264,6 +266,18 @@ def ct_calibrate(S_host: np.ndarray, alpha: float):
     _check(lib().ct_calibrate(S.ctypes.data, S.size, alpha, ctypes.byref(r), ctypes.byref(t)),
            "ct_calibrate")
     return r.value, t.value
+
+
+def ct_fi_threshold(S_host: np.ndarray, critical: np.ndarray, reference: float, alpha: float) -> float:
+    """Sec. II-C FI-based threshold from campaign trials (S, critical)."""
+    S = np.ascontiguousarray(S_host, dtype=np.float32)
+    c = np.ascontiguousarray(critical, dtype=np.uint8)
+    if S.shape != c.shape:
+        raise ValueError("S and critical must have the same shape")
+    t = ctypes.c_double()
+    _check(lib().ct_fi_threshold(S.ctypes.data, c.ctypes.data, S.size, reference, alpha, ctypes.byref(t)),
+           "ct_fi_threshold")
+    return t.value
 
 
 def ct_buffers(m: Model, batch: int) -> List[tuple]:

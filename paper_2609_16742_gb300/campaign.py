@@ -22,6 +22,13 @@ alpha (nearest-rank quantile of |S - r|).
 
 prints one JSON object.  The bookkeeping runs on the GPU (torch ops on the
 library's outputs); the host only draws the fault list and launches.
+
+With --sweep it instead compares the two threshold methods of Sec. II-C
+over alpha in {0.1, 1, 5}% (Sec. III-A): the distribution-based tau from
+fault-free calibration images, and the FI-based tau from a campaign on the
+calibration images (at most alpha of its non-critical trials flagged), each
+scored on a campaign with other faults on the evaluation images: TPR, FPR
+and Youden's J = TPR - FPR.
 """
 import argparse
 import json
@@ -30,10 +37,9 @@ import sys
 import time
 
 
-def run(precision="fp32", faults=1000, seed=0, batch=None, calib_images=10000, alpha=0.01, device=0,
-        reexecute=True):
+def _setup(precision, batch, calib_images, device):
+    """Model, workload and fault-free calibration S values."""
     sys.path.insert(0, os.path.dirname(os.path.dirname(os.path.abspath(__file__))))
-    import numpy as np
     import torch
     import synth
     import paper_2609_16742_gb300 as ct
@@ -45,7 +51,6 @@ def run(precision="fp32", faults=1000, seed=0, batch=None, calib_images=10000, a
     m = ct.ct_build_workload(net, synth.make_params(net.layers, net.seed), precision=precision, max_batch=B,
                              device=device)
     stream = torch.cuda.current_stream()
-    # ---- calibration (fault-free) ----
     n_cal = ((calib_images + B - 1) // B) * B
     xc = torch.from_numpy(synth.make_input(wl, batch=n_cal, seed=wl.calib_seed)).cuda()
     Sc = torch.empty(n_cal, device="cuda")
@@ -53,19 +58,102 @@ def run(precision="fp32", faults=1000, seed=0, batch=None, calib_images=10000, a
     for i in range(0, n_cal, B):
         ct.ct_infer(m, xc[i:i + B], B, lc, Sc[i:i + B], None, stream)
     torch.cuda.synchronize()
-    r, tau = ct.ct_calibrate(Sc.cpu().numpy(), alpha)
+    return m, wl, B, stream, Sc.cpu().numpy(), n_cal
+
+
+def _top1(lg):
+    import torch
+    return torch.where(torch.isnan(lg).any(1), torch.full((lg.shape[0],), -1, device=lg.device, dtype=torch.long),
+                       lg.argmax(1))
+
+
+def _trials(m, x, B, sites, stream, reexecute=False):
+    """Run one campaign on the batch x: per image trial its S and whether it
+    was critical (GPU bookkeeping), plus the counters of run()."""
+    import torch
+    import paper_2609_16742_gb300 as ct
+    n_classes = m.n_classes
+    logits = torch.empty(B, n_classes, device="cuda")
+    S = torch.empty(B, device="cuda")
+    flag = torch.empty(B, dtype=torch.uint8, device="cuda")
+    ct.ct_infer(m, x, B, logits, S, flag, stream)
+    golden = _top1(logits).clone()
+    per_img = {}
+    for kind, layer, n_el, bits in ct.ct_buffers(m, B):
+        if kind == 1:
+            per_img[layer] = n_el // B
+    S_rec, c_rec = [], []
+    n_rerun = 0
+    for kind, layer, e, bit in sites.tolist():
+        ct.ct_inject(m, kind, layer, e, bit)
+        ct.ct_infer(m, x, B, logits, S, flag, stream)
+        crit = _top1(logits) != golden
+        if kind == 0:
+            S_rec.append(S.clone())
+            c_rec.append(crit)
+        else:
+            i = e // per_img[layer]
+            S_rec.append(S[i:i + 1].clone())
+            c_rec.append(crit[i:i + 1])
+        if reexecute:
+            n_rerun += ct.ct_reexecute(m, x, B, flag, logits, S, stream)
+    torch.cuda.synchronize()
+    return torch.cat(S_rec).cpu().numpy(), torch.cat(c_rec).cpu().numpy(), n_rerun
+
+
+def sweep(precision="fp32", faults=2000, seed_cal=1, seed_eval=2, alphas=(0.001, 0.01, 0.05), batch=None,
+          calib_images=10000, device=0):
+    """Distribution-based vs FI-based thresholds over alpha (Sec. II-C, III-A)."""
+    import numpy as np
+    import torch
+    import synth
+    import paper_2609_16742_gb300 as ct
+
+    m, wl, B, stream, S_ff, n_cal = _setup(precision, batch, calib_images, device)
+    bufs = ct.ct_buffers(m, B)
+    # FI campaign on calibration images ("training set") and on evaluation images ("test set")
+    x_cal = torch.from_numpy(synth.make_input(wl, batch=B, seed=wl.calib_seed)).cuda()
+    x_eval = torch.from_numpy(synth.make_input(wl, batch=B)).cuda()
+    S_c, crit_c, _ = _trials(m, x_cal, B, synth.draw_faults(bufs, faults, seed_cal), stream)
+    S_e, crit_e, _ = _trials(m, x_eval, B, synth.draw_faults(bufs, faults, seed_eval), stream)
+    rows = []
+    for alpha in alphas:
+        r, tau_d = ct.ct_calibrate(S_ff, alpha)
+        tau_f = ct.ct_fi_threshold(S_c, crit_c.astype(np.uint8), r, alpha)
+        for method, tau in (("distribution", tau_d), ("fi", tau_f)):
+            flag = ~(np.abs(S_e.astype(np.float64) - r) <= tau)
+            crit = crit_e.astype(bool)
+            tpr = float(flag[crit].mean()) if crit.any() else None
+            fpr = float(flag[~crit].mean()) if (~crit).any() else None
+            rows.append({"method": method, "alpha": alpha, "tau": tau, "reference": r, "tpr": tpr, "fpr": fpr,
+                         "youden_j": (tpr - fpr) if tpr is not None and fpr is not None else None})
+    best = {meth: max((row for row in rows if row["method"] == meth), key=lambda row: row["youden_j"])["alpha"]
+            for meth in ("distribution", "fi")}
+    out = {"precision": precision, "faults_per_campaign": faults, "batch": B, "calibration_images": n_cal,
+           "calibration_trials": int(S_c.size), "calibration_critical": int(crit_c.sum()),
+           "evaluation_trials": int(S_e.size), "evaluation_critical": int(crit_e.sum()),
+           "table": rows, "best_alpha_by_youden_j": best, "device_error": ct.ct_device_error(m)}
+    m.close()
+    return out
+
+
+def run(precision="fp32", faults=1000, seed=0, batch=None, calib_images=10000, alpha=0.01, device=0,
+        reexecute=True):
+    import numpy as np
+    import torch
+    import synth
+    import paper_2609_16742_gb300 as ct
+
+    m, wl, B, stream, S_ff, n_cal = _setup(precision, batch, calib_images, device)
+    r, tau = ct.ct_calibrate(S_ff, alpha)
     ct.ct_set_threshold(m, r, tau)
-    del xc
     # ---- fault-free evaluation batch ----
     x = torch.from_numpy(synth.make_input(wl, batch=B)).cuda()
     logits = torch.empty(B, wl.n_classes, device="cuda")
     S = torch.empty(B, device="cuda")
     flag = torch.empty(B, dtype=torch.uint8, device="cuda")
 
-    def top1(lg):
-        return torch.where(torch.isnan(lg).any(1), torch.full((lg.shape[0],), -1, device=lg.device,
-                                                               dtype=torch.long), lg.argmax(1))
-
+    top1 = _top1
     ct.ct_infer(m, x, B, logits, S, flag, stream)
     golden = top1(logits).clone()
     ff_flags = int(flag.sum().item())
@@ -153,7 +241,14 @@ def main(argv=None):
     ap.add_argument("--calib-images", type=int, default=10000)
     ap.add_argument("--alpha", type=float, default=0.01)
     ap.add_argument("--no-reexecute", action="store_true")
+    ap.add_argument("--sweep", action="store_true",
+                    help="compare distribution-based and FI-based thresholds over alpha in {0.1, 1, 5}%%")
     args = ap.parse_args(argv)
+    if args.sweep:
+        out = sweep(args.precision, args.faults, seed_cal=args.seed + 1, seed_eval=args.seed + 2,
+                    calib_images=args.calib_images)
+        print(json.dumps(out))
+        return 0 if out["device_error"] == 0 else 1
     out = run(args.precision, args.faults, args.seed, calib_images=args.calib_images, alpha=args.alpha,
               reexecute=not args.no_reexecute)
     print(json.dumps(out))

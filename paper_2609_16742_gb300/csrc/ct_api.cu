@@ -896,6 +896,25 @@ ct_status ct_calibrate(const float *S_host, int64_t n, double alpha, double *ref
     return CT_OK;
 }
 
+ct_status ct_fi_threshold(const float *S_host, const uint8_t *critical, int64_t n, double reference,
+                          double alpha, double *tau) {
+    if (!S_host || !critical || n < 1 || !(alpha >= 0.0 && alpha < 1.0) || !tau) return CT_EINVAL;
+    std::vector<double> dev;
+    dev.reserve((size_t)n);
+    for (int64_t i = 0; i < n; ++i) {
+        if (critical[i]) continue;
+        const double d = fabs((double)S_host[i] - reference);
+        dev.push_back(d == d ? d : INFINITY);    // a non-finite S deviates without bound
+    }
+    if (dev.empty()) return CT_EINVAL;
+    std::sort(dev.begin(), dev.end());
+    const int64_t m = (int64_t)dev.size();
+    int64_t rank = (int64_t)ceil((1.0 - alpha) * (double)m);
+    rank = std::min<int64_t>(std::max<int64_t>(rank, 1), m);
+    *tau = dev[rank - 1];
+    return CT_OK;
+}
+
 ct_status ct_buffer_count(const ct_model *m, int32_t batch, int32_t *n) {
     if (!m || !n || batch < 1) return CT_EINVAL;
     int cnt = 0;

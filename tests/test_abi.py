@@ -80,3 +80,16 @@ def test_build_without_device_fails_cleanly(ct):
     with pytest.raises(ct.CtError) as ei:
         ct.ct_build_workload(wl)
     assert ei.value.status == 3          # CT_ECUDA
+
+
+def test_fi_threshold_matches_oracle(ct):
+    rng = np.random.default_rng(9)
+    S = rng.normal(2000.0, 80.0, 3001).astype(np.float32)
+    S[rng.integers(0, 3001, 25)] = np.float32(np.nan)
+    S[rng.integers(0, 3001, 5)] = np.float32(np.inf)
+    crit = (rng.random(3001) < 0.03).astype(np.uint8)
+    for alpha in (0.0, 0.001, 0.01, 0.05, 0.5):
+        got = ct.ct_fi_threshold(S, crit, 2001.5, alpha)
+        assert got == oracle.fi_threshold(S.astype(np.float64), crit, 2001.5, alpha)
+    with pytest.raises(ct.CtError):
+        ct.ct_fi_threshold(S, np.ones(3001, np.uint8), 0.0, 0.01)

@@ -78,3 +78,41 @@ def test_campaign_runner_bookkeeping():
     assert w["trials"] // out["batch"] + act["trials"] == 48
     assert sum(v["trials"] for v in out["by_bit"].values()) == a["trials"]
     assert out["kernels_launched"] > 48
+
+
+def test_threshold_sweep_rows():
+    """Sec. II-C / III-A: distribution-based and FI-based taus over alpha; each
+    row's rates are those the oracle's detection_rates gives for its tau on
+    the evaluation trials, and the FI tau keeps the calibration campaign's
+    false-alarm rate at or below alpha."""
+    from paper_2609_16742_gb300 import campaign
+    rec = {}
+    orig = campaign._trials
+
+    def spy(m, x, B, sites, stream, reexecute=False):
+        out = orig(m, x, B, sites, stream, reexecute)
+        rec.setdefault("runs", []).append(out)
+        return out
+
+    campaign._trials = spy
+    try:
+        out = campaign.sweep("fp32", faults=64, calib_images=512)
+    finally:
+        campaign._trials = orig
+    assert out["device_error"] == 0
+    (S_c, crit_c, _), (S_e, crit_e, _) = rec["runs"]
+    assert S_c.size == out["calibration_trials"] and S_e.size == out["evaluation_trials"]
+    assert len(out["table"]) == 6
+    for row in out["table"]:
+        tpr, fpr, j = oracle.detection_rates(S_e, crit_e, row["reference"], row["tau"])
+        assert row["fpr"] == pytest.approx(fpr, abs=1e-12)
+        if tpr is not None and row["tpr"] is not None:
+            assert row["tpr"] == pytest.approx(tpr, abs=1e-12)
+        if row["method"] == "fi":
+            assert row["tau"] == oracle.fi_threshold(S_c, crit_c, row["reference"], row["alpha"])
+            _, fpr_c, _ = oracle.detection_rates(S_c, crit_c, row["reference"], row["tau"])
+            assert fpr_c <= row["alpha"] + 1e-12
+    # a larger alpha never raises tau
+    for meth in ("distribution", "fi"):
+        taus = [row["tau"] for row in out["table"] if row["method"] == meth]
+        assert all(a >= b for a, b in zip(taus, taus[1:]))

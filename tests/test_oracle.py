@@ -486,3 +486,28 @@ def test_fault_buffers_resnet18_cifar():
     assert all(b[3] == 32 for b in bufs)
     n_conv = sum(1 for L in wl.layers if L.op == "conv")
     assert len(w) == n_conv
+
+
+def test_fi_threshold_and_detection_rates_by_hand():
+    # Sec. II-C FI-based threshold and the Sec. III-A rates on a worked example
+    S = np.array([10.0, 11.0, 9.0, 30.0, np.nan, 12.0, 10.5, 8.0])
+    crit = np.array([0, 0, 0, 1, 0, 0, 1, 0])
+    r = 10.0
+    # non-critical deviations: 0, 1, 1, inf (NaN), 2, 2 -> sorted 0 1 1 2 2 inf
+    assert oracle.fi_threshold(S, crit, r, 0.2) == 2.0      # rank ceil(0.8 * 6) = 5
+    assert oracle.fi_threshold(S, crit, r, 0.5) == 1.0      # rank 3
+    assert oracle.fi_threshold(S, crit, r, 0.0) == np.inf   # rank 6
+    tpr, fpr, j = oracle.detection_rates(S, crit, r, 2.0)
+    # flagged: 30 (critical) and NaN (non-critical); 12 and 8 sit exactly at tau
+    assert tpr == 0.5 and fpr == 1.0 / 6.0 and j == tpr - fpr
+
+
+def test_fi_threshold_bounds_the_false_alarm_rate():
+    rng = np.random.default_rng(4)
+    S = rng.normal(100.0, 5.0, 5000)
+    S[rng.integers(0, 5000, 40)] = np.inf
+    crit = rng.random(5000) < 0.05
+    for alpha in (0.001, 0.01, 0.05):
+        tau = oracle.fi_threshold(S, crit, 100.0, alpha)
+        _, fpr, _ = oracle.detection_rates(S, crit, 100.0, tau)
+        assert fpr <= alpha + 1e-12
