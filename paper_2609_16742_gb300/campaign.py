@@ -127,8 +127,10 @@ def sweep(precision="fp32", faults=2000, seed_cal=1, seed_eval=2, alphas=(0.001,
             fpr = float(flag[~crit].mean()) if (~crit).any() else None
             rows.append({"method": method, "alpha": alpha, "tau": tau, "reference": r, "tpr": tpr, "fpr": fpr,
                          "youden_j": (tpr - fpr) if tpr is not None and fpr is not None else None})
-    best = {meth: max((row for row in rows if row["method"] == meth), key=lambda row: row["youden_j"])["alpha"]
-            for meth in ("distribution", "fi")}
+    best = {}
+    for meth in ("distribution", "fi"):
+        scored = [row for row in rows if row["method"] == meth and row["youden_j"] is not None]
+        best[meth] = max(scored, key=lambda row: row["youden_j"])["alpha"] if scored else None
     out = {"precision": precision, "faults_per_campaign": faults, "batch": B, "calibration_images": n_cal,
            "calibration_trials": int(S_c.size), "calibration_critical": int(crit_c.sum()),
            "evaluation_trials": int(S_e.size), "evaluation_critical": int(crit_e.sum()),

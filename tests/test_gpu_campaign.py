@@ -96,13 +96,14 @@ def test_threshold_sweep_rows():
 
     campaign._trials = spy
     try:
-        out = campaign.sweep("fp32", faults=64, calib_images=512)
+        out = campaign.sweep("fp16", faults=256, calib_images=512)
     finally:
         campaign._trials = orig
     assert out["device_error"] == 0
     (S_c, crit_c, _), (S_e, crit_e, _) = rec["runs"]
     assert S_c.size == out["calibration_trials"] and S_e.size == out["evaluation_trials"]
     assert len(out["table"]) == 6
+    assert out["evaluation_critical"] > 0 and out["calibration_critical"] > 0
     for row in out["table"]:
         tpr, fpr, j = oracle.detection_rates(S_e, crit_e, row["reference"], row["tau"])
         assert row["fpr"] == pytest.approx(fpr, abs=1e-12)
