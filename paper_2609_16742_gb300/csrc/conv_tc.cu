@@ -251,7 +251,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
     constexpr int NPROD = DBUF ? 2 : STAGES % 4 == 0 ? 4 : STAGES % 3 == 0 ? 3 : STAGES % 2 == 0 ? 2 : 1;
     constexpr int NCT = DBUF ? TC_NPROD - NPROD : 0;
     static_assert(NPROD <= TC_NPROD && STAGES % NPROD == 0, "producer warps must own whole ring slots");
-    static_assert(!DBUF || (NCT > 0 && BM % (32 * (NCT > 0 ? NCT : 1)) == 0), "carry-through warps split the tile rows");
+    static_assert(!DBUF || (NCT > 0 && BM % (16 * (NCT > 0 ? NCT : 1)) == 0), "carry-through warps split the tile rows");
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint8_t *As = smem;                                   // [STAGES][SUB][A_BYTES]
@@ -432,12 +432,18 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
             // ---------------- carry-through sums (N = 256) ----------------
             // Consumes every stage in order (arrives on its empty barrier);
             // on the centre-tap K blocks of the first N tile it adds each A
-            // row's 64 channels (the 128-byte swizzle only permutes chunks
-            // within a row).  Carry-through warp w takes tile rows
-            // lane + 32 (w + NCT i).
-            constexpr int RPL = BM / (32 * (NCT > 0 ? NCT : 1));   // rows per lane
+            // row's 64 channels.  The row sums run on the warp-level MMA
+            // against a B of ones (FP32 accumulation, like the tcgen05
+            // column of the other kernels): per K block and 64-row share,
+            // 16 ldmatrix + 16 MMAs.  Rows are read through the 128-byte
+            // swizzle (chunk c of row r sits at chunk c ^ (r & 7)), so the
+            // eight rows of one 8x8 matrix hit eight different bank groups.
+            constexpr int ROWS_W = BM / (NCT > 0 ? NCT : 1);       // rows per carry-through warp
+            constexpr int MT = ROWS_W / 16;                          // 16-row MMA tiles per warp
             const float coef = __half2float(__ushort_as_half(g.coef_h));
             const int w = warp - NPROD;
+            // ldmatrix row address of this lane: matrix lane / 8 = (rows +8, chunk +1) bits
+            const int lm_row = (lane & 7) + ((lane >> 3) & 1) * 8, lm_chk = lane >> 4;
             int it = 0, lt = 0;
             bool ok = true;
             for (int tile = cid; tile < num_items && ok; tile += ncl, ++lt) {
@@ -445,31 +451,29 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
                 const TileRef tr = tile_ref(tile, g, CS, crank);
                 const bool ct_here = g.ct_mode != CT_NONE_ && tr.n_tile == 0;
                 const int ab = lt & 1;
-                float acc[RPL];
+                float acc[MT][4];
 #pragma unroll
-                for (int i = 0; i < RPL; ++i) acc[i] = 0.f;
+                for (int m = 0; m < MT; ++m)
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) acc[m][e] = 0.f;
                 for (int kb0 = tr.kb_lo; kb0 < tr.kb_hi; kb0 += SUB, ++it) {
                     const int s = it % STAGES;
                     if (!warp_wait(smem_u32(&full[s]), (uint32_t)(it / STAGES) & 1u, a.err, 2u)) { ok = false; break; }
                     const int nsub = min(SUB, tr.kb_hi - kb0);
                     for (int j = 0; j < nsub; ++j) {
                         if (!(ct_here && kb0 + j < g.cpb)) continue;
+                        const uint32_t tbase = smem_u32(As + (s * SUB + j) * A_BYTES);
 #pragma unroll
-                        for (int i = 0; i < RPL; ++i) {
-                            const int row = lane + 32 * (w + NCT * i);
-                            const uint4 *rp = reinterpret_cast<const uint4 *>(As + (s * SUB + j) * A_BYTES + row * 128);
-                            float sum = 0.f;
+                        for (int m = 0; m < MT; ++m) {
+                            const int row = w * ROWS_W + m * 16 + lm_row;
+                            const uint32_t rbase = tbase + (uint32_t)row * 128u;
 #pragma unroll
-                            for (int c = 0; c < 8; ++c) {
-                                const uint4 v = rp[c];
-                                const __half2 *h = reinterpret_cast<const __half2 *>(&v);
-#pragma unroll
-                                for (int e = 0; e < 4; ++e) {
-                                    const float2 f = __half22float2(h[e]);
-                                    sum += f.x + f.y;
-                                }
+                            for (int t = 0; t < 4; ++t) {
+                                const uint32_t chk = (uint32_t)((2 * t + lm_chk) ^ (row & 7));
+                                uint32_t a0, a1, a2, a3;
+                                ldsm_x4(rbase + chk * 16u, a0, a1, a2, a3);
+                                mma_rowsum_16x16(acc[m], a0, a1, a2, a3);
                             }
-                            acc[i] += sum;
                         }
                     }
                     __syncwarp();
@@ -478,8 +482,15 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
                 if (!ok) break;
                 // ct_sum[ab] is free once the epilogue released accumulator ab
                 if (!warp_wait(smem_u32(&acc_empty[ab]), ((uint32_t)(lt >> 1) & 1u) ^ 1u, a.err, 8u)) { ok = false; break; }
+                // D fragment: lane l holds rows l / 4 (acc[m][0]) and l / 4 + 8 (acc[m][2]) of tile m
+                if ((lane & 3) == 0) {
 #pragma unroll
-                for (int i = 0; i < RPL; ++i) ct_sum[ab * BM + lane + 32 * (w + NCT * i)] = coef * acc[i];
+                    for (int m = 0; m < MT; ++m) {
+                        const int r0 = w * ROWS_W + m * 16 + (lane >> 2);
+                        ct_sum[ab * BM + r0] = coef * acc[m][0];
+                        ct_sum[ab * BM + r0 + 8] = coef * acc[m][2];
+                    }
+                }
                 __syncwarp();
                 if (lane == 0) mbar_arrive(smem_u32(&ct_ready[ab]));
             }
@@ -910,15 +921,19 @@ struct HaloMaps {
     CUtensorMap amap, bmap, rmap, cmap, qmap;
 };
 
-// Epilogue operand ring (R): per tile, the residual tile (BN channels of
-// its 128 pixels, pixel-major) and the incoming / residual checksum values
-// of its pixels, fetched by the producer warp with TMA several tiles ahead
-// so that the epilogue reads them from shared memory.
+// Epilogue operand ring (R): per tile, the residual tile and the incoming /
+// residual checksum values of its pixels, fetched by the producer warp with
+// TMA several tiles ahead so that the epilogue reads them from shared
+// memory.  The residual is BN / 64 blocks of [128 pixels][64 channels], each
+// copied with the 128-byte swizzle (16-byte chunk c of pixel r at chunk
+// c ^ (r & 7)): the epilogue lane of pixel r reads 16 bytes of its own
+// 128-byte row, and without the swizzle the 32 lanes of a warp would all hit
+// the same four banks.
 template <int BN>
 struct HaloR {
     static constexpr int RES = 128 * BN * 2;
     static constexpr int CS = 128 * 2;
-    static constexpr int STAGE = RES + 2 * CS;       // multiple of 128
+    static constexpr int STAGE = (RES + 2 * CS + 1023) / 1024 * 1024;   // swizzle atoms stay 1024-byte aligned
 };
 
 template <int BN, bool BRES, int NA, int NB, int NR>
@@ -1031,7 +1046,10 @@ conv_tc_halo_kernel(const __grid_constant__ HaloMaps maps, const ConvArgs a, con
                         const uint32_t rb = smem_u32(&r_full[rs]);
                         uint8_t *st = Rs + rs * R::STAGE;
                         mbar_arrive_expect_tx(rb, r_bytes);
-                        if (hg.res) tma_load_4d(smem_u32(st), &maps.rmap, rb, ht.nt * BN, ht.x0, ht.y0, ht.n);
+                        if (hg.res)
+                            for (int cb = 0; cb < BN / 64; ++cb)
+                                tma_load_4d(smem_u32(st + cb * 128 * 128), &maps.rmap, rb, ht.nt * BN + cb * 64, ht.x0,
+                                            ht.y0, ht.n);
                         if (hg.csin) tma_load_3d(smem_u32(st + R::RES), &maps.cmap, rb, ht.x0, ht.y0, ht.n);
                         if (hg.rescs) tma_load_3d(smem_u32(st + R::RES + R::CS), &maps.qmap, rb, ht.x0, ht.y0, ht.n);
                     }
@@ -1171,9 +1189,12 @@ conv_tc_halo_kernel(const __grid_constant__ HaloMaps maps, const ConvArgs a, con
 #pragma unroll
             for (int c = 0; c < BN / 32; ++c) {
                 if (hg.res) {
-                    const uint4 *rp = reinterpret_cast<const uint4 *>(rst + ((size_t)row * BN + half * (BN / 2) + 16 * c) * 2);
-                    rs[c].r0 = rp[0];
-                    rs[c].r1 = rp[1];
+                    // channels ch .. ch + 15: 64-channel block ch / 64, chunks (ch % 64) / 8 and the next
+                    const int ch = half * (BN / 2) + 16 * c;
+                    const uint8_t *rrow = rst + (ch / 64) * 128 * 128 + row * 128;
+                    const int ck = (ch % 64) / 8, sw = row & 7;
+                    rs[c].r0 = *reinterpret_cast<const uint4 *>(rrow + ((ck ^ sw) << 4));
+                    rs[c].r1 = *reinterpret_cast<const uint4 *>(rrow + (((ck + 1) ^ sw) << 4));
                 } else {
                     rs[c].r0 = rs[c].r1 = make_uint4(0u, 0u, 0u, 0u);
                 }
@@ -1532,12 +1553,12 @@ HaloPlan *halo_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, 
                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) { if (why) *why = "weight tensor map"; delete pl; return nullptr; }
     if (res_dev) {
-        // residual [max_batch, H, W, K]: boxes of BN channels x 8 x 16 pixels, pixel-major
+        // residual [max_batch, H, W, K]: boxes of 64 channels x 8 x 16 pixels, pixel-major, 128-byte swizzle
         cuuint64_t rdim[4] = {(cuuint64_t)a.K, (cuuint64_t)a.W, (cuuint64_t)a.H, (cuuint64_t)max_batch};
         cuuint64_t rstr[3] = {(cuuint64_t)a.K * 2, (cuuint64_t)a.W * a.K * 2, (cuuint64_t)a.H * a.W * a.K * 2};
-        cuuint32_t rbox[4] = {(cuuint32_t)pl->BN, HT_TW, HT_TH, 1};
+        cuuint32_t rbox[4] = {64, HT_TW, HT_TH, 1};
         if (g_encode_tiled(&pl->maps.rmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<void *>(res_dev), rdim, rstr,
-                           rbox, aes, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                           rbox, aes, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                            CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS) {
             if (why) *why = "residual tensor map";
             delete pl;

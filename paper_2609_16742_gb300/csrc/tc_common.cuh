@@ -148,6 +148,24 @@ __device__ __forceinline__ float tmem_ld1(uint32_t taddr) {
 
 __device__ __forceinline__ float relu_keep_nan(float v) { return v < 0.f ? 0.f : v; }
 
+// Four 8x8 b16 matrices from shared memory; lane l supplies the row address
+// of row l % 8 of matrix l / 8 (warp-level, non-transposed).
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(addr));
+}
+
+// Warp-level D += A (16x16, f16, row) x B (16x8, f16, col) with FP32 D.
+// With every B element 1 each column of D accumulates the row sums of A.
+__device__ __forceinline__ void mma_rowsum_16x16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3) {
+    const uint32_t one2 = 0x3C003C00u;   // two f16 ones
+    asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+                 "{%8, %9}, {%0, %1, %2, %3};"
+                 : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+                 : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(one2), "r"(one2));
+}
+
 __device__ __forceinline__ float ldh(const __half *p, size_t i) { return __half2float(p[i]); }
 
 // UMMA shared-memory descriptor without swizzle, K-major: core matrices of
