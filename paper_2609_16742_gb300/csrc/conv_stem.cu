@@ -327,7 +327,11 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
 #pragma unroll
         for (int i = 0; i < 32; ++i) bias[i] = __ldg(a.bias + k0 + i);
         const bool has_cs = a.cs_out != nullptr;
-        // pooling role: column jj, channels 16 * cq .. 16 * cq + 15
+        // pooling role: column jj, channels 8 cq .. 8 cq + 7 and 32 + 8 cq ..
+        // 32 + 8 cq + 7 (16-byte chunks cq and cq + 4 of a 128-byte pixel):
+        // with the 144-byte row-buffer pitch and stride-2 columns, the 32
+        // lanes of a warp then start on every 16-byte bank group equally
+        // often (contiguous 32-byte quarters would use half the banks)
         const int jj = et >> 2, cq = et & 3;
         const bool pool_data = jj < g.Q2;
         const bool pool_cs = has_cs && et < g.Q2;
@@ -399,8 +403,8 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
                 for (int dc = -1; dc <= 1; ++dc) {
                     const int col = 2 * jj + dc;
                     if (col < 0 || col >= g.Q) continue;
-                    const uint4 *src = reinterpret_cast<const uint4 *>(rb + col * ST_PIX_H + 16 * cq);
-                    const uint4 s0 = src[0], s1 = src[1];
+                    const uint4 *src = reinterpret_cast<const uint4 *>(rb + col * ST_PIX_H + 8 * cq);
+                    const uint4 s0 = src[0], s1 = src[4];
                     h[0] = hmax2u(h[0], s0.x); h[1] = hmax2u(h[1], s0.y);
                     h[2] = hmax2u(h[2], s0.z); h[3] = hmax2u(h[3], s0.w);
                     h[4] = hmax2u(h[4], s1.x); h[5] = hmax2u(h[5], s1.y);
@@ -423,9 +427,9 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
                 if (store) {
                     const int i2 = (p & 1) ? (p - 1) / 2 : p / 2;
                     uint4 *dst = reinterpret_cast<uint4 *>(static_cast<__half *>(a.y) +
-                                                            (((size_t)jb.n * g.P2 + i2) * g.Q2 + jj) * ST_K + 16 * cq);
+                                                            (((size_t)jb.n * g.P2 + i2) * g.Q2 + jj) * ST_K + 8 * cq);
                     dst[0] = make_uint4(accv[0], accv[1], accv[2], accv[3]);
-                    dst[1] = make_uint4(accv[4], accv[5], accv[6], accv[7]);
+                    dst[4] = make_uint4(accv[4], accv[5], accv[6], accv[7]);
                 }
             }
             if (pool_cs) {
