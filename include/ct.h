@@ -178,6 +178,36 @@ ct_status ct_reexecute(ct_model *m, const float *input_dev, int32_t batch,
                        const uint8_t *flag_dev, float *logits_dev, float *S_dev,
                        int32_t *n_rerun, void *stream);
 
+/* ct_infer_reexec -- ct_infer of `batch` new images (input_dev, logits_dev,
+ * S_dev, flag_dev as for ct_infer) that also carries out the Sec. II-B
+ * re-execution of a PREVIOUS inference's flagged images, deferred into this
+ * one: the images of prev_input_dev [prev_batch, C, H, W] whose
+ * prev_flag_dev entry is non-zero are appended as extra rows of this
+ * inference (the same kernels over batch + n images), and their re-run
+ * logits and S overwrite their rows of prev_logits_dev / prev_S_dev
+ * (prev_S_dev may be NULL).  The re-run's flags are ignored and
+ * prev_flag_dev is not modified.  A flagged image thus costs one more image
+ * of a large batch instead of a separate small-batch pass.  Within one
+ * inference every image's row is computed independently of the others, so
+ * the re-run rows equal those of a fault-free ct_infer of the same images
+ * at a batch size with the same tiling.
+ *   - prev_input_dev NULL (or prev_batch 0): exactly ct_infer; *n_rerun = 0.
+ *   - Synchronises `stream` once to read prev_flag_dev, like ct_reexecute.
+ *   - The combined batch must fit max_batch: when batch + n > max_batch, or
+ *     when a fault is armed (a re-run must be fault-free), the previous
+ *     batch is re-executed first exactly as by ct_reexecute and then this
+ *     batch is inferred as by ct_infer (the armed fault goes to it).
+ *   - The previous batch's buffers must stay valid until the stream reaches
+ *     this call's kernels; none of them may alias this call's outputs.
+ *   - *n_rerun (host, may be NULL): images of the previous batch re-run.
+ * Errors: CT_EINVAL (null model, input or logits; prev_input_dev given
+ * without prev_flag_dev or prev_logits_dev), CT_ERANGE (batch or prev_batch
+ * outside 1..max_batch), CT_ECUDA, and those of ct_infer. */
+ct_status ct_infer_reexec(ct_model *m, const float *input_dev, int32_t batch, float *logits_dev,
+                          float *S_dev, uint8_t *flag_dev, const float *prev_input_dev,
+                          int32_t prev_batch, const uint8_t *prev_flag_dev, float *prev_logits_dev,
+                          float *prev_S_dev, int32_t *n_rerun, void *stream);
+
 /* ct_reexecute_noalloc -- the same re-execution as ct_reexecute, for callers
  * that must not allocate device memory while they run: real-time loops whose
  * device memory is fixed at start-up so that a request can never fail for

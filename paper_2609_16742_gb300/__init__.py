@@ -33,7 +33,7 @@ _STATUS = {0: "CT_OK", 1: "CT_EINVAL", 2: "CT_ENOMEM", 3: "CT_ECUDA", 4: "CT_EST
 
 # every exported symbol of include/ct.h
 EXPORTS = ["ct_build", "ct_set_threshold", "ct_get_threshold", "ct_infer", "ct_inject",
-           "ct_clear_faults", "ct_reexecute", "ct_run_host", "ct_calibrate", "ct_buffer_count",
+           "ct_clear_faults", "ct_reexecute", "ct_infer_reexec", "ct_run_host", "ct_calibrate", "ct_buffer_count",
            "ct_buffer_info", "ct_profile_enable", "ct_profile_read", "ct_launches_per_infer", "ct_kernel_count",
            "ct_fi_threshold",
            "ct_copy_activation", "ct_device_error", "ct_destroy", "ct_strerror",
@@ -87,6 +87,7 @@ def lib():
             "ct_inject": [vp, i32, i32, i64, i32],
             "ct_clear_faults": [vp],
             "ct_reexecute": [vp, vp, i32, vp, vp, vp, P(i32), vp],
+            "ct_infer_reexec": [vp, vp, i32, vp, vp, vp, vp, i32, vp, vp, vp, P(i32), vp],
             "ct_reexecute_noalloc": [vp, vp, i32, vp, vp, vp, P(i32), vp],
             "ct_run_host": [vp, vp, i32, vp, vp, vp, P(i32), vp],
             "ct_calibrate": [vp, i64, dbl, P(dbl), P(dbl)],
@@ -237,6 +238,18 @@ def ct_reexecute(m: Model, input_dev, batch: int, flag_dev, logits_dev, S_dev=No
     n = ctypes.c_int32()
     _check(lib().ct_reexecute(m.handle, _ptr(input_dev), batch, _ptr(flag_dev), _ptr(logits_dev),
                               _ptr(S_dev), ctypes.byref(n), _stream(stream)), "ct_reexecute")
+    return n.value
+
+
+def ct_infer_reexec(m: Model, input_dev, batch: int, logits_dev, S_dev=None, flag_dev=None,
+                    prev_input_dev=None, prev_batch: int = 0, prev_flag_dev=None, prev_logits_dev=None,
+                    prev_S_dev=None, stream=None) -> int:
+    """ct_infer of a new batch that re-executes the previous batch's flagged
+    images as extra rows of the same inference; returns how many were re-run."""
+    n = ctypes.c_int32()
+    _check(lib().ct_infer_reexec(m.handle, _ptr(input_dev), batch, _ptr(logits_dev), _ptr(S_dev), _ptr(flag_dev),
+                                 _ptr(prev_input_dev), prev_batch, _ptr(prev_flag_dev), _ptr(prev_logits_dev),
+                                 _ptr(prev_S_dev), ctypes.byref(n), _stream(stream)), "ct_infer_reexec")
     return n.value
 
 

@@ -128,9 +128,17 @@ __device__ __forceinline__ uint32_t hmax2u(uint32_t a, uint32_t b) {
     return *reinterpret_cast<uint32_t *>(&r);
 }
 
-__device__ __forceinline__ float image_half(const float *x, const StemGeom &g, int n, int c, int h, int w) {
+// image n of the batch: images n >= n_split come from the second input
+// (re-executed images appended to a batch)
+__device__ __forceinline__ const float *image_base(const ConvArgs &a, const StemGeom &g, int n) {
+    const size_t chw = (size_t)g.C * g.H * g.W;
+    if (a.x2 && n >= a.n_split) return static_cast<const float *>(a.x2) + (size_t)(n - a.n_split) * chw;
+    return static_cast<const float *>(a.x) + (size_t)n * chw;
+}
+
+__device__ __forceinline__ float image_half(const float *img, const StemGeom &g, int c, int h, int w) {
     if (c >= g.C || h < 0 || h >= g.H || w < 0 || w >= g.W) return 0.f;
-    return __half2float(__float2half_rn(x[(((size_t)n * g.C + c) * g.H + h) * g.W + w]));
+    return __half2float(__float2half_rn(img[((size_t)c * g.H + h) * g.W + w]));
 }
 
 __global__ void __launch_bounds__(ST_THREADS, 1)
@@ -152,7 +160,6 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
     volatile uint32_t *abort_flag = tmem_holder + 1;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const float *x = static_cast<const float *>(a.x);
     const int units = g.N * g.P2;
     const int u0 = (int)((long long)blockIdx.x * units / gridDim.x);
     const int u1 = (int)((long long)(blockIdx.x + 1) * units / gridDim.x);
@@ -227,6 +234,7 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
                 if (!warp_wait(smem_u32(&empty[slot]), ph ^ 1u, a.err, 1u)) { ok = false; break; }
                 const int y = y0 + t;
                 const bool row_ok = y >= 0 && y < g.H;
+                const float *img = image_base(a, g, jb.n);
                 float v[8][4];
 #pragma unroll
                 for (int it = 0; it < 8; ++it) {
@@ -235,7 +243,7 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
                     for (int c = 0; c < 4; ++c) {
                         v[it][c] = 0.f;
                         if (row_ok && col < g.W && c < g.C)
-                            v[it][c] = __ldg(x + (((size_t)jb.n * g.C + c) * g.H + y) * g.W + col);
+                            v[it][c] = __ldg(img + ((size_t)c * g.H + y) * g.W + col);
                     }
                 }
                 uint8_t *E = ring + slot * ST_SLOT_BYTES;
@@ -361,7 +369,7 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
                 if (q < g.Q) {
                     float fsrc = 0.f;
                     if (fd.active)
-                        fsrc = image_half(x, g, jb.n, fd.cin, 2 * jb.p + fd.r - 3, 2 * q + fd.s - 3);
+                        fsrc = image_half(image_base(a, g, jb.n), g, fd.cin, 2 * jb.p + fd.r - 3, 2 * q + fd.s - 3);
                     uint32_t pk[16];
 #pragma unroll
                     for (int i = 0; i < 32; i += 2) {

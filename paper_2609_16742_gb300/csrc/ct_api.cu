@@ -551,8 +551,11 @@ ct_status act_fault_word(const ct_model *m, int slot, int batch, int64_t e, void
 // inference
 // ---------------------------------------------------------------------------
 
+// input2 / n_split: images n >= n_split of the batch are image n - n_split
+// of input2 (re-executed images appended to a batch); the rest of the
+// network is unaware of it
 ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, float *S,
-                     uint8_t *flag, cudaStream_t st) {
+                     uint8_t *flag, cudaStream_t st, const float *input2 = nullptr, int n_split = 0) {
     const bool half = m->prec == CT_FP16;
     const int wb = half ? 2 : 4;
     const bool armed = m->armed;
@@ -566,10 +569,18 @@ ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, 
         if (act_fault_word(m, act_slot, batch, m->f_elem, &act_base, &act_word) != CT_OK) return CT_ERANGE;
     }
     Slot &s0 = m->slots[0];
-    if (s0.stored)
+    const int n_first = input2 ? n_split : batch;
+    if (s0.stored) {
         CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] {
-            return launch_convert_input(input, s0.data, batch, s0.C, s0.cp, s0.H, s0.W, half, st);
+            return launch_convert_input(input, s0.data, n_first, s0.C, s0.cp, s0.H, s0.W, half, st);
         }));
+        if (input2) {
+            void *dst2 = static_cast<uint8_t *>(s0.data) + (size_t)n_split * s0.H * s0.W * s0.cp * wb;
+            CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] {
+                return launch_convert_input(input2, dst2, batch - n_split, s0.C, s0.cp, s0.H, s0.W, half, st);
+            }));
+        }
+    }
     if (act_slot == 0) CUDA_TRY(xor_bit(m, act_base, act_word, m->f_bit, wb, st));
     for (size_t i = 0; i < m->L.size(); ++i) {
         LayerRT &l = m->L[i];
@@ -599,6 +610,8 @@ ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, 
                 // the fused kernel reads the FP32 image and writes the max-pool's output
                 const Slot &po = m->slots[m->L[i + 1].d.dst];
                 a.x = input;
+                a.x2 = input2;
+                a.n_split = n_first;
                 a.y = po.data;
                 a.cs_out = po.has_cs ? po.cs : nullptr;
                 CUDA_TRY(launch(m, FAM_TC, flops, st, [&] { return launch_stem_pool(a, l.stplan, st); }));
@@ -729,6 +742,47 @@ ct_status reexec_impl(ct_model *m, const float *input, int batch, const uint8_t 
     return CT_OK;
 }
 
+// Inference of `batch` new images with the previous batch's flagged images
+// re-executed as extra rows of the same launch sequence (Sec. II-B): their
+// cost is that of the extra images, not of a separate small-batch pass.
+// Falls back to reexec_impl + infer_impl when a fault is armed (the re-run
+// must be fault-free) or the rows do not fit max_batch.
+ct_status infer_reexec_impl(ct_model *m, const float *input, int batch, float *logits, float *S, uint8_t *flag,
+                            const float *prev_input, int prev_batch, const uint8_t *prev_flag, float *prev_logits,
+                            float *prev_S, int *n_rerun, cudaStream_t st) {
+    if (n_rerun) *n_rerun = 0;
+    if (!prev_input || prev_batch == 0) return infer_impl(m, input, batch, logits, S, flag, st);
+    CUDA_TRY(cudaMemcpyAsync(m->h_flags, prev_flag, prev_batch, cudaMemcpyDeviceToHost, st));
+    CUDA_TRY(cudaStreamSynchronize(st));
+    int n = 0;
+    for (int i = 0; i < prev_batch; ++i)
+        if (m->h_flags[i]) m->h_idx[n++] = i;
+    if (n == 0) return infer_impl(m, input, batch, logits, S, flag, st);
+    if (m->armed || batch + n > m->max_batch) {
+        int nr = 0;
+        ct_status s = reexec_impl(m, prev_input, prev_batch, prev_flag, prev_logits, prev_S, &nr, st);
+        if (s != CT_OK) return s;
+        if (n_rerun) *n_rerun = nr;
+        return infer_impl(m, input, batch, logits, S, flag, st);
+    }
+    if (n_rerun) *n_rerun = n;
+    CUDA_TRY(cudaMemcpyAsync(m->re_idx, m->h_idx, sizeof(int32_t) * n, cudaMemcpyHostToDevice, st));
+    const int64_t per = (int64_t)m->in_c * m->in_h * m->in_w;
+    CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] { return launch_gather_images(prev_input, m->re_input, m->re_idx, n, per, st); }));
+    const int tot = batch + n;
+    ct_status s = infer_impl(m, input, tot, m->re_logits, m->re_S, m->re_flag, st, m->re_input, batch);
+    if (s != CT_OK) return s;
+    // rows < batch: this batch; rows >= batch: the re-run, whose flag is ignored
+    CUDA_TRY(cudaMemcpyAsync(logits, m->re_logits, sizeof(float) * m->n_classes * batch, cudaMemcpyDeviceToDevice, st));
+    if (S) CUDA_TRY(cudaMemcpyAsync(S, m->re_S, sizeof(float) * batch, cudaMemcpyDeviceToDevice, st));
+    if (flag) CUDA_TRY(cudaMemcpyAsync(flag, m->re_flag, batch, cudaMemcpyDeviceToDevice, st));
+    CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] {
+        return launch_scatter_rows(m->re_logits + (size_t)batch * m->n_classes, prev_logits, m->re_idx, n, m->n_classes, st);
+    }));
+    if (prev_S) CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] { return launch_scatter_rows(m->re_S + batch, prev_S, m->re_idx, n, 1, st); }));
+    return CT_OK;
+}
+
 }  // namespace
 
 namespace ct {
@@ -850,6 +904,25 @@ ct_status ct_reexecute(ct_model *m, const float *input_dev, int32_t batch, const
     DeviceGuard g(m->device);
     int n = 0;
     ct_status s = reexec_impl(m, input_dev, batch, flag_dev, logits_dev, S_dev, &n, (cudaStream_t)stream);
+    if (n_rerun) *n_rerun = n;
+    return s;
+}
+
+ct_status ct_infer_reexec(ct_model *m, const float *input_dev, int32_t batch, float *logits_dev, float *S_dev,
+                          uint8_t *flag_dev, const float *prev_input_dev, int32_t prev_batch,
+                          const uint8_t *prev_flag_dev, float *prev_logits_dev, float *prev_S_dev, int32_t *n_rerun,
+                          void *stream) {
+    if (!m || !input_dev || !logits_dev) return CT_EINVAL;
+    if (batch < 1 || batch > m->max_batch) return CT_ERANGE;
+    if (prev_input_dev) {
+        if (!prev_flag_dev || !prev_logits_dev) return CT_EINVAL;
+        if (prev_batch < 1 || prev_batch > m->max_batch) return CT_ERANGE;
+    }
+    DeviceGuard g(m->device);
+    int n = 0;
+    ct_status s = infer_reexec_impl(m, input_dev, batch, logits_dev, S_dev, flag_dev, prev_input_dev,
+                                    prev_input_dev ? prev_batch : 0, prev_flag_dev, prev_logits_dev, prev_S_dev, &n,
+                                    (cudaStream_t)stream);
     if (n_rerun) *n_rerun = n;
     return s;
 }

@@ -43,6 +43,8 @@ struct ConvArgs {
                           // is the sum of cs_in[m * cs_rowsum .. m * cs_rowsum + cs_rowsum)
     float *ws;            // split-K workspace (null: never split)
     size_t ws_bytes;
+    const void *x2;       // first layer only: images n >= n_split are image n - n_split of x2
+    int n_split;          // (null x2: every image comes from x)
 };
 
 struct FcArgs {
