@@ -255,30 +255,20 @@ def main():
         ct.ct_infer(mp, x, B, logits, S, flag, stream)
         return ct.ct_reexecute(mp, x, B, flag, logits, S, stream)
 
-    def deferred_steps(steps, h2d=None, d2h=None):
+    def deferred_steps(steps):
         """`steps` protected steps in which the flagged images of each batch
         are re-executed as extra rows of the next batch's inference
-        (ct_infer_reexec); the last batch's are re-run at the end.  With
-        h2d / d2h, each step copies its input in from pinned host memory and
-        the completed batch's results out."""
+        (ct_infer_reexec); the last batch's are re-run at the end."""
         n_re, prev = 0, None
         for i in range(steps):
             cur = bufs[i % 2]
-            if h2d is not None:
-                cur["x"].copy_(h2d[i % 2], non_blocking=True)
             if prev is None:
                 n_re += ct.ct_infer_reexec(mp, cur["x"], B, cur["lg"], cur["S"], cur["fl"], stream=stream)
             else:
                 n_re += ct.ct_infer_reexec(mp, cur["x"], B, cur["lg"], cur["S"], cur["fl"], prev["x"], B,
                                            prev["fl"], prev["lg"], prev["S"], stream)
-                if d2h is not None:
-                    for k_ in ("lg", "S", "fl"):
-                        d2h[k_].copy_(prev[k_], non_blocking=True)
             prev = cur
         n_re += ct.ct_reexecute(mp, prev["x"], B, prev["fl"], prev["lg"], prev["S"], stream)
-        if d2h is not None:
-            for k_ in ("lg", "S", "fl"):
-                d2h[k_].copy_(prev[k_], non_blocking=True)
         return n_re
 
     def step_unprotected():
@@ -356,16 +346,52 @@ def main():
         return v
 
     # end to end through the public API from pinned host memory: every step
-    # copies its input in, runs ct_infer_reexec, and copies the completed
-    # batch's logits, S and flags out (the last batch after its re-run)
+    # copies its input in (on a copy stream, overlapping the previous step's
+    # kernels; three input slots), runs ct_infer_reexec, and copies the
+    # completed batch's logits, S and flags out (the last batch after its
+    # re-run).  Slot i % 3 is free for step i + 1's input once ct_infer_reexec
+    # of step i returns: that call waited for step i - 1's kernels, the last
+    # to read it.
     xh2 = [torch.from_numpy(xh_).pin_memory() for xh_ in x_hosts]
     d2h = {"lg": torch.empty(B, wl.n_classes, dtype=torch.float32).pin_memory(),
            "S": torch.empty(B, dtype=torch.float32).pin_memory(),
            "fl": torch.empty(B, dtype=torch.uint8).pin_memory()}
-    deferred_steps(2, h2d=xh2, d2h=d2h)
+    ebufs = [{"x": torch.empty_like(bufs[0]["x"]), "lg": torch.empty_like(bufs[0]["lg"]),
+              "S": torch.empty_like(bufs[0]["S"]), "fl": torch.empty_like(bufs[0]["fl"])} for _ in range(3)]
+    copy_stream = torch.cuda.Stream()
+    ev_in = [torch.cuda.Event() for _ in range(3)]
+
+    def copy_in(i):
+        with torch.cuda.stream(copy_stream):
+            ebufs[i % 3]["x"].copy_(xh2[i % 2], non_blocking=True)
+            ev_in[i % 3].record(copy_stream)
+
+    def e2e_steps(steps):
+        n_re, prev = 0, None
+        copy_in(0)
+        for i in range(steps):
+            cur = ebufs[i % 3]
+            stream.wait_event(ev_in[i % 3])
+            if prev is None:
+                n_re += ct.ct_infer_reexec(mp, cur["x"], B, cur["lg"], cur["S"], cur["fl"], stream=stream)
+            else:
+                n_re += ct.ct_infer_reexec(mp, cur["x"], B, cur["lg"], cur["S"], cur["fl"], prev["x"], B,
+                                           prev["fl"], prev["lg"], prev["S"], stream)
+            if i + 1 < steps:
+                copy_in(i + 1)
+            if prev is not None:
+                for k_ in ("lg", "S", "fl"):
+                    d2h[k_].copy_(prev[k_], non_blocking=True)
+            prev = cur
+        n_re += ct.ct_reexecute(mp, prev["x"], B, prev["fl"], prev["lg"], prev["S"], stream)
+        for k_ in ("lg", "S", "fl"):
+            d2h[k_].copy_(prev[k_], non_blocking=True)
+        return n_re
+
+    e2e_steps(3)
     barrier()
     t0 = time.perf_counter()
-    deferred_steps(args.steps, h2d=xh2, d2h=d2h)
+    e2e_steps(args.steps)
     barrier()
     e2e_s = max_over_ranks(time.perf_counter() - t0)
 
@@ -470,7 +496,8 @@ def main():
         "cpu_baseline": cpu,
         "e2e": {"value": world * B * args.steps / e2e_s, "unit": "images/s",
                 "h2d_bytes_per_step": in_bytes, "d2h_bytes_per_step": out_bytes,
-                "api": "ct_infer_reexec with pinned host copies in and out on the launch stream"},
+                "api": "ct_infer_reexec; pinned host copies in (copy stream, overlapping the previous "
+                       "step) and out (launch stream)"},
         "e2e_sync_reexec": {"value": world * B * args.steps / e2e_sync_s, "unit": "images/s",
                             "api": "ct_run_host (host buffers, synchronous re-execution)"},
         "kernel_families": {nm: {"launches": fam_stats[i][0], "ms": fam_stats[i][1],
