@@ -141,6 +141,88 @@ __device__ __forceinline__ float image_half(const float *img, const StemGeom &g,
     return __half2float(__float2half_rn(img[((size_t)c * g.H + h) * g.W + w]));
 }
 
+// The ring entries in production order: a CTA's convolution rows each need
+// the input rows not already in the ring (7 at the start of a run within an
+// image, then 2).  Entry e is produced by warp e % 4.
+struct RowIter {
+    StemJobs jb;
+    bool have;
+    int ecount, t, n_new, y0;
+    int n_of_last;        // image of the entry last returned
+
+    __device__ void set_job() {
+        n_new = jb.seg_start ? 7 : 2;
+        y0 = jb.seg_start ? 2 * jb.p - 3 : 2 * jb.p + 2;
+    }
+    __device__ void init(int u0, int u1, const StemGeom &g) {
+        have = jb.first(u0, u1, g);
+        ecount = 0;
+        t = 0;
+        n_of_last = 0;
+        if (have) set_job();
+    }
+    // next entry of warp w: its index e and input row y
+    __device__ bool next(int w, int &e, int &y, const StemGeom &g) {
+        while (have) {
+            while (t < n_new) {
+                const int ee = ecount + t, tt = t;
+                ++t;
+                if ((ee & 3) == w) {
+                    e = ee;
+                    y = y0 + tt;
+                    n_of_last = jb.n;
+                    return true;
+                }
+            }
+            ecount += n_new;
+            t = 0;
+            have = jb.next(g);
+            if (have) set_job();
+        }
+        return false;
+    }
+};
+
+// one input row (image img, row y) as FP32 values: lane owns columns lane + 32 it
+__device__ __forceinline__ void load_image_row(float (&v)[8][4], const float *img, const StemGeom &g, int y,
+                                               int lane) {
+    const bool row_ok = y >= 0 && y < g.H;
+#pragma unroll
+    for (int it = 0; it < 8; ++it) {
+        const int col = lane + 32 * it;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            v[it][c] = 0.f;
+            if (row_ok && col < g.W && c < g.C) v[it][c] = __ldg(img + ((size_t)c * g.H + y) * g.W + col);
+        }
+    }
+}
+
+// waits for ring slot e % ST_NSLOT, writes the row's two FP16 copies (E:
+// pixel x at byte 8 (x + 3), O: at byte 8 (x + 4)) and marks it full
+__device__ __forceinline__ bool store_ring_row(const float (&v)[8][4], uint8_t *ring, uint64_t *full,
+                                               uint64_t *empty, int e, const StemGeom &g, int lane, uint32_t *err) {
+    const int slot = e % ST_NSLOT;
+    const uint32_t ph = (uint32_t)(e / ST_NSLOT) & 1u;
+    if (!warp_wait(smem_u32(&empty[slot]), ph ^ 1u, err, 1u)) return false;
+    uint8_t *E = ring + slot * ST_SLOT_BYTES;
+    uint8_t *O = E + ST_ROW_BYTES;
+#pragma unroll
+    for (int it = 0; it < 8; ++it) {
+        const int col = lane + 32 * it;
+        if (col < g.W) {
+            __half2 lo = __floats2half2_rn(v[it][0], v[it][1]);
+            __half2 hi = __floats2half2_rn(v[it][2], v[it][3]);
+            const uint2 pk = make_uint2(*reinterpret_cast<uint32_t *>(&lo), *reinterpret_cast<uint32_t *>(&hi));
+            *reinterpret_cast<uint2 *>(E + (col + 3) * 8) = pk;
+            *reinterpret_cast<uint2 *>(O + (col + 4) * 8) = pk;
+        }
+    }
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    mbar_arrive(smem_u32(&full[slot]));
+    return true;
+}
+
 __global__ void __launch_bounds__(ST_THREADS, 1)
 stem_pool_kernel(const ConvArgs a, const StemGeom g) {
     pdl_wait();
@@ -218,54 +300,28 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
 
     if (warp < 4) {
         // ---------------- ring producers ----------------
-        StemJobs jb;
-        bool have = jb.first(u0, u1, g);
-        int ecount = 0;
-        while (have) {
+        // Each warp produces every fourth ring entry.  The global loads of
+        // its next entry are issued before it waits for the current entry's
+        // slot and stores it, so two input rows per warp (eight per CTA) are
+        // in flight against the DRAM latency.
+        RowIter ri;
+        ri.init(u0, u1, g);
+        float va[8][4], vb[8][4];
+        int ea = 0, ya = 0, eb = 0, yb = 0;
+        bool ok = true;
+        bool ha = ri.next(warp, ea, ya, g);
+        if (ha) load_image_row(va, image_base(a, g, ri.n_of_last), g, ya, lane);
+        while (ha) {
             if (__any_sync(0xffffffffu, *abort_flag)) break;
-            const int n_new = jb.seg_start ? 7 : 2;
-            const int y0 = jb.seg_start ? 2 * jb.p - 3 : 2 * jb.p + 2;
-            bool ok = true;
-            for (int t = 0; t < n_new; ++t) {
-                const int e = ecount + t;
-                if ((e & 3) != warp) continue;
-                const int slot = e % ST_NSLOT;
-                const uint32_t ph = (uint32_t)(e / ST_NSLOT) & 1u;
-                if (!warp_wait(smem_u32(&empty[slot]), ph ^ 1u, a.err, 1u)) { ok = false; break; }
-                const int y = y0 + t;
-                const bool row_ok = y >= 0 && y < g.H;
-                const float *img = image_base(a, g, jb.n);
-                float v[8][4];
-#pragma unroll
-                for (int it = 0; it < 8; ++it) {
-                    const int col = lane + 32 * it;
-#pragma unroll
-                    for (int c = 0; c < 4; ++c) {
-                        v[it][c] = 0.f;
-                        if (row_ok && col < g.W && c < g.C)
-                            v[it][c] = __ldg(img + ((size_t)c * g.H + y) * g.W + col);
-                    }
-                }
-                uint8_t *E = ring + slot * ST_SLOT_BYTES;
-                uint8_t *O = E + ST_ROW_BYTES;
-#pragma unroll
-                for (int it = 0; it < 8; ++it) {
-                    const int col = lane + 32 * it;
-                    if (col < g.W) {
-                        __half2 lo = __floats2half2_rn(v[it][0], v[it][1]);
-                        __half2 hi = __floats2half2_rn(v[it][2], v[it][3]);
-                        const uint2 pk = make_uint2(*reinterpret_cast<uint32_t *>(&lo), *reinterpret_cast<uint32_t *>(&hi));
-                        *reinterpret_cast<uint2 *>(E + (col + 3) * 8) = pk;
-                        *reinterpret_cast<uint2 *>(O + (col + 4) * 8) = pk;
-                    }
-                }
-                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-                mbar_arrive(smem_u32(&full[slot]));
-            }
-            if (!ok) { if (lane == 0) *abort_flag = 1; break; }
-            ecount += n_new;
-            have = jb.next(g);
+            const bool hb = ri.next(warp, eb, yb, g);
+            if (hb) load_image_row(vb, image_base(a, g, ri.n_of_last), g, yb, lane);
+            if (!(ok = store_ring_row(va, ring, full, empty, ea, g, lane, a.err))) break;
+            if (!hb) break;
+            ha = ri.next(warp, ea, ya, g);
+            if (ha) load_image_row(va, image_base(a, g, ri.n_of_last), g, ya, lane);
+            if (!(ok = store_ring_row(vb, ring, full, empty, eb, g, lane, a.err))) break;
         }
+        if (!ok && lane == 0) *abort_flag = 1;
     } else if (warp == 4) {
         // ---------------- MMA issuer (whole warp, one lane issues) ----------------
         const uint32_t id64 = idesc_f16(128, ST_K);

@@ -1393,8 +1393,10 @@ cudaError_t launch_conv_tc(const ConvArgs &a, const void *plan, cudaStream_t st,
     g.splits = (a.K % 8 == 0) ? splitk_choose(tiles, g.n_kb, 4, pl->sms / 2, g.M, g.ws_ld, a.ws ? a.ws_bytes : 0) : 1;
     g.kps = (g.n_kb + g.splits - 1) / g.splits;
     g.m_groups = g.m_tiles;
-    if (pl->cs > 1 && g.splits == 1 && g.m_tiles >= 4 * pl->cs) {
+    if (pl->cs > 1 && g.splits == 1 && g.m_tiles >= 4 * pl->cs && g.n_kb >= 4) {
         // clusters of cs CTAs on groups of cs consecutive M tiles, sharing B
+        // (not for a few K blocks per tile: little B to share, and the
+        // cluster's CTAs advance in lockstep)
         g.m_groups = (g.m_tiles + pl->cs - 1) / pl->cs;
         const int items = g.m_groups * g.n_tiles;
         const int ncl = items < pl->max_clusters ? items : pl->max_clusters;
