@@ -40,8 +40,10 @@ exact on stored values; the global average pool and the final FC layer
 produce fp32.  Biases are stored in fp32 in every precision.  Precision
 "fp64" rounds nowhere (used by the exact pins).
 
-Readings of points the paper leaves open are listed in the design doc and
-repeated next to the code that takes them.
+Readings of points the paper leaves open are stated next to the code that
+takes them.  The paper's own replace-mode construction (prune the least
+important channel and put the carry-through filter in its place) is in
+``oracle/replace.py``.
 """
 from __future__ import annotations
 
