@@ -96,10 +96,37 @@ typedef struct {
 /* flags for ct_build_opts.flags */
 #define CT_FLAG_SIMT_ONLY 1u      /* use the CUDA-core conv kernels everywhere */
 
+/* ct_build_opts.protect: how the scheme of Sec. II-A is built in.
+ *   CT_PROTECT_NONE     the network as described (the unprotected baseline);
+ *   CT_PROTECT_WIDEN    every carry-through filter is an EXTRA output channel
+ *                       (kept beside the tensor as a checksum plane) and every
+ *                       hidden FC layer gets an extra neuron: the data path is
+ *                       the unprotected one, bit for bit;
+ *   CT_PROTECT_REPLACE  the paper's construction: in every tensor the least
+ *                       important channel is pruned and the carry-through
+ *                       filter (or neuron) takes its place as the LAST
+ *                       channel, so widths and costs are those of the
+ *                       unprotected network.  Importance: the combined L1 norm
+ *                       of the channel's filters (before BatchNorm folding) in
+ *                       its writers and of its slices in its readers, summed
+ *                       over tensors tied by a residual add or a pooling; the
+ *                       smallest, lowest index on ties.  A residual block's
+ *                       first convolution gets an all-zero last channel, the
+ *                       1x1 shortcut a pass-through one (CT_DS_ZERO: zero);
+ *                       the slices of the incoming checksum are zero weights
+ *                       that are multiplied like any other.  No fine-tuning.
+ *                       The classifier keeps its classes and gets the
+ *                       accumulated-checksum neuron (sum of all its inputs,
+ *                       the checksum channel's features included).
+ * Faults (ct_inject) address the stored tensors: for CT_PROTECT_REPLACE the
+ * literal layout is the original shape. */
+#define CT_PROTECT_NONE 0
+#define CT_PROTECT_WIDEN 1
+#define CT_PROTECT_REPLACE 2
+
 typedef struct {
     int32_t precision;   /* ct_precision: storage type of weights and activations */
-    int32_t protect;     /* 1: add carry-through filters and the checksum neuron;
-                            0: the same network and kernels without them */
+    int32_t protect;     /* CT_PROTECT_NONE / _WIDEN / _REPLACE (see above) */
     int32_t ds_mode;     /* ct_ds_mode */
     int32_t device;      /* CUDA device ordinal */
     int32_t max_batch;   /* workspaces are sized for this many images */

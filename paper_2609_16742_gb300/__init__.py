@@ -25,6 +25,7 @@ CT_OP_CONV, CT_OP_MAXPOOL, CT_OP_GAP, CT_OP_FC = 0, 1, 2, 3
 CT_ROLE_CT, CT_ROLE_NONE, CT_ROLE_PASS = 0, 1, 2
 CT_BUF_WEIGHT, CT_BUF_ACT = 0, 1
 CT_DS_PASS, CT_DS_ZERO = 0, 1
+CT_PROTECT_NONE, CT_PROTECT_WIDEN, CT_PROTECT_REPLACE = 0, 1, 2
 CT_FLAG_SIMT_ONLY = 1
 FAM_TC, FAM_SIMT, FAM_FC, FAM_POOL, FAM_OTHER = 0, 1, 2, 3, 4
 
@@ -176,8 +177,11 @@ class Model:
 def ct_build(layers: Sequence, params: Sequence[dict], in_shape, n_classes: int,
              precision: str = "fp32", protect: bool = True, ds_mode: str = "pass",
              device: int = 0, max_batch: int = 64, simt_only: bool = False,
-             bn_eps: float = 1e-5) -> Model:
-    """Build a model from synth-style layers and float32 parameter dicts."""
+             bn_eps: float = 1e-5, replace: bool = False) -> Model:
+    """Build a model from synth-style layers and float32 parameter dicts.
+
+    protect=True adds the carry-through filters as extra channels (widened);
+    replace=True builds the paper's prune-and-replace construction instead."""
     n = len(layers)
     arr = (LayerDesc * n)()
     keep = []
@@ -192,12 +196,13 @@ def ct_build(layers: Sequence, params: Sequence[dict], in_shape, n_classes: int,
                 keep.append(a)
                 wp[6 * i + j] = a.ctypes.data
     desc = ModelDesc(n, arr, in_shape[0], in_shape[1], in_shape[2], n_classes, bn_eps)
-    opts = BuildOpts(CT_FP16 if precision == "fp16" else CT_FP32, int(protect),
+    mode = CT_PROTECT_REPLACE if replace else (CT_PROTECT_WIDEN if protect else CT_PROTECT_NONE)
+    opts = BuildOpts(CT_FP16 if precision == "fp16" else CT_FP32, mode,
                      CT_DS_ZERO if ds_mode == "zero" else CT_DS_PASS, device, max_batch,
                      CT_FLAG_SIMT_ONLY if simt_only else 0)
     h = ctypes.c_void_p()
     _check(lib().ct_build(ctypes.byref(desc), wp, ctypes.byref(opts), ctypes.byref(h)), "ct_build")
-    return Model(h.value, n_classes, in_shape, precision, protect, max_batch)
+    return Model(h.value, n_classes, in_shape, precision, protect or replace, max_batch)
 
 
 def ct_build_workload(wl, params=None, **kw) -> Model:

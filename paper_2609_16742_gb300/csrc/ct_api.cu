@@ -115,7 +115,8 @@ constexpr size_t SPLITK_WS_BYTES = 32ull << 20;
 struct ct_model {
     int device = 0;
     int prec = CT_FP32;
-    bool protect = true;
+    bool protect = true;         // widened construction: checksum planes beside the tensors
+    bool replace = false;        // replace construction: checksum inside the pruned tensors
     int ds_mode = CT_DS_PASS;
     int max_batch = 0;
     uint32_t flags = 0;
@@ -262,6 +263,93 @@ cudaError_t launch(ct_model *m, int fam, double flops, cudaStream_t st, F &&fn, 
 // build
 // ---------------------------------------------------------------------------
 
+// Replace construction (Sec. II-A): per slot, the output channel pruned to
+// make room for the carry-through filter (-1: none).  Slots tied by a
+// residual add, a max-pool or the global average pool form one stream with
+// one index: the channel whose combined L1 norm over the stream's writers
+// (their output filters, before BatchNorm folding) and readers (their input
+// slices; an FC reader's H*W columns of the channel) is smallest, the lowest
+// such index on ties.  The network input and the classifier output are not
+// pruned.
+std::vector<int> replace_prune_index(const ct_model_desc *desc, const float *const *wts, int n_slots) {
+    const int nL = desc->n_layers;
+    std::vector<int> parent(n_slots);
+    for (int i = 0; i < n_slots; ++i) parent[i] = i;
+    auto find = [&](int a) {
+        while (parent[a] != a) a = parent[a] = parent[parent[a]];
+        return a;
+    };
+    auto unite = [&](int a, int b) {
+        a = find(a); b = find(b);
+        if (a != b) parent[std::max(a, b)] = std::min(a, b);
+    };
+    std::vector<int> ch(n_slots, 0), hw(n_slots, 1);
+    ch[0] = desc->in_c;
+    std::vector<int> H(n_slots, 0), W(n_slots, 0);
+    H[0] = desc->in_h; W[0] = desc->in_w;
+    int final_dst = -1;
+    for (int i = 0; i < nL; ++i) {
+        const ct_layer_desc &d = desc->layers[i];
+        if (d.op == CT_OP_CONV) {
+            ch[d.dst] = d.cout;
+            H[d.dst] = (H[d.src] + 2 * d.pad - d.k) / d.stride + 1;
+            W[d.dst] = (W[d.src] + 2 * d.pad - d.k) / d.stride + 1;
+            if (d.res >= 0) unite(d.dst, d.res);
+        } else if (d.op == CT_OP_MAXPOOL) {
+            ch[d.dst] = ch[d.src];
+            H[d.dst] = (H[d.src] + 2 * d.pad - d.k) / d.stride + 1;
+            W[d.dst] = (W[d.src] + 2 * d.pad - d.k) / d.stride + 1;
+            unite(d.dst, d.src);
+        } else if (d.op == CT_OP_GAP) {
+            ch[d.dst] = ch[d.src]; H[d.dst] = W[d.dst] = 1;
+            unite(d.dst, d.src);
+        } else {
+            ch[d.dst] = d.cout; H[d.dst] = W[d.dst] = 1;
+            if (d.final) final_dst = d.dst;
+        }
+    }
+    std::vector<std::vector<double>> score(n_slots);
+    auto add = [&](int slot, int c, double v) {
+        const int r = find(slot);
+        if (r == find(0) || (final_dst >= 0 && r == find(final_dst))) return;
+        if ((int)score[r].size() < ch[slot]) score[r].resize(ch[slot], 0.0);
+        score[r][c] += v;
+    };
+    for (int i = 0; i < nL; ++i) {
+        const ct_layer_desc &d = desc->layers[i];
+        const float *w = wts[CT_WEIGHTS_PER_LAYER * i];
+        if (d.op == CT_OP_CONV) {
+            const int RS = d.k * d.k;
+            for (int k = 0; k < d.cout; ++k)
+                for (int c = 0; c < d.cin; ++c) {
+                    double a = 0.0;
+                    for (int t = 0; t < RS; ++t) a += fabs((double)w[((size_t)k * d.cin + c) * RS + t]);
+                    add(d.dst, k, a);
+                    add(d.src, c, a);
+                }
+        } else if (d.op == CT_OP_FC) {
+            const int C = ch[d.src], P = H[d.src] * W[d.src];
+            for (int j = 0; j < d.cout; ++j)
+                for (int c = 0; c < C; ++c) {
+                    double a = 0.0;
+                    for (int p = 0; p < P; ++p) a += fabs((double)w[(size_t)j * d.cin + (size_t)c * P + p]);
+                    if (!d.final) add(d.dst, j, a);
+                    add(d.src, c, a);
+                }
+        }
+    }
+    std::vector<int> out(n_slots, -1);
+    for (int sl = 0; sl < n_slots; ++sl) {
+        const std::vector<double> &v = score[find(sl)];
+        if (v.empty()) continue;
+        int best = 0;
+        for (int c = 1; c < (int)v.size(); ++c)
+            if (v[c] < v[best]) best = c;
+        out[sl] = best;
+    }
+    return out;
+}
+
 ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const *wts) {
     const int nL = desc->n_layers;
     int max_slot = 0;
@@ -279,6 +367,9 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
     const size_t esz = m->esz();
     const int B = m->max_batch;
     int n_final = 0;
+    // replace construction: pruned channel per slot (-1 elsewhere and in the other modes)
+    const std::vector<int> pj = m->replace ? replace_prune_index(desc, wts, max_slot + 1)
+                                           : std::vector<int>(max_slot + 1, -1);
 
     for (int i = 0; i < nL; ++i) {
         const ct_layer_desc &d = desc->layers[i];
@@ -343,7 +434,24 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
             if (l.tc_small) src.cp = 4;
             std::vector<uint8_t> hw((size_t)l.K * l.w_ld * esz, 0);
             std::vector<float> hb(l.K, 0.f);
-            for (int k = 0; k < l.K; ++k) {
+            // replace construction: stored output channel kk holds original
+            // channel kk (+1 past the pruned one); the last holds the
+            // carry-through filter (zero for a block's first convolution,
+            // pass-through for the shortcut); stored input channel cc likewise,
+            // the last (the incoming checksum) being a zero slice
+            const int jo = pj[d.dst], ji = pj[d.src];
+            if (jo >= 0) {
+                const int ctr = (l.R - 1) / 2;
+                const int kk = l.K - 1;
+                for (int cc = 0; cc < l.C; ++cc) {
+                    double v = 0.0;
+                    if (d.role == CT_ROLE_CT) v = l.coef;
+                    else if (d.role == CT_ROLE_PASS && m->ds_mode == CT_DS_PASS && cc == l.C - 1 && ji >= 0) v = 1.0;
+                    if (v != 0.0) put(hw, (size_t)weight_word(l, kk, ctr, ctr, cc), v, prec);
+                }
+            }
+            for (int kk = 0; kk < l.K - (jo >= 0 ? 1 : 0); ++kk) {
+                const int k = (jo >= 0 && kk >= jo) ? kk + 1 : kk;
                 double scale = 1.0, shift = bias ? (double)bias[k] : 0.0;
                 if (d.bn) {
                     const float *g = wts[CT_WEIGHTS_PER_LAYER * i + 2], *be = wts[CT_WEIGHTS_PER_LAYER * i + 3];
@@ -353,13 +461,15 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
                     double t = (shift - (double)mu[k]) * scale;
                     shift = t + (double)be[k];
                 }
-                hb[k] = (float)shift;
-                for (int c = 0; c < l.C; ++c)
+                hb[kk] = (float)shift;
+                for (int cc = 0; cc < l.C - (ji >= 0 ? 1 : 0); ++cc) {
+                    const int c = (ji >= 0 && cc >= ji) ? cc + 1 : cc;
                     for (int r = 0; r < l.R; ++r)
                         for (int s = 0; s < l.S; ++s) {
                             double v = (double)W[(((size_t)k * l.C + c) * l.R + r) * l.S + s] * scale;
-                            put(hw, (size_t)weight_word(l, k, r, s, c), v, prec);
+                            put(hw, (size_t)weight_word(l, kk, r, s, cc), v, prec);
                         }
+                }
             }
             ct_status st;
             if ((st = dalloc(m, &l.w, hw.size())) != CT_OK) return st;
@@ -391,14 +501,25 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
             l.fc_tc = prec == CT_FP16 && !(m->flags & CT_FLAG_SIMT_ONLY) && !d.final && !src.is_float &&
                       tc_supported(l.n_in, l.n_out, 1, 1, 1, 0, &why);
             // weights: columns permuted from (c, h, w) to the NHWC flatten (h, w, c)
-            std::vector<uint8_t> hw((size_t)l.n_out * l.n_in * esz);
+            std::vector<uint8_t> hw((size_t)l.n_out * l.n_in * esz, 0);
             std::vector<float> hb(l.n_out, 0.f);
-            for (int j = 0; j < l.n_out; ++j) {
-                hb[j] = bias ? bias[j] : 0.f;
-                for (int c = 0; c < src.C; ++c)
+            // replace construction: neuron jj holds original neuron jj (+1 past
+            // the pruned one), the last a carry-through neuron of weight coef;
+            // input channel cc likewise, the last (checksum) zero in every
+            // normal neuron.  The classifier keeps its neurons; its
+            // accumulated-checksum neuron is computed by the FC kernel.
+            const int jo = d.final ? -1 : pj[d.dst], ji = pj[d.src];
+            if (jo >= 0)
+                for (int q = 0; q < l.n_in; ++q) put(hw, (size_t)(l.n_out - 1) * l.n_in + q, l.coef, prec);
+            for (int jj = 0; jj < l.n_out - (jo >= 0 ? 1 : 0); ++jj) {
+                const int j = (jo >= 0 && jj >= jo) ? jj + 1 : jj;
+                hb[jj] = bias ? bias[j] : 0.f;
+                for (int cc = 0; cc < src.C - (ji >= 0 ? 1 : 0); ++cc) {
+                    const int c = (ji >= 0 && cc >= ji) ? cc + 1 : cc;
                     for (int p = 0; p < HW; ++p)
-                        put(hw, (size_t)j * l.n_in + (size_t)p * src.C + c,
+                        put(hw, (size_t)jj * l.n_in + (size_t)p * src.C + cc,
                             (double)W[(size_t)j * l.n_in + (size_t)c * HW + p], prec);
+                }
             }
             ct_status st;
             if ((st = dalloc(m, &l.w, hw.size())) != CT_OK) return st;
@@ -655,7 +776,10 @@ ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, 
             FcArgs a{};
             a.x = src.data; a.xcs = src.has_cs ? src.cs : nullptr; a.w = l.w; a.bias = l.bias;
             a.B = batch; a.n_in = l.n_in; a.n_cs = l.n_cs; a.n_out = l.n_out;
-            a.relu = d.relu; a.final_layer = d.final; a.protect = m->protect; a.coef = l.coef;
+            a.relu = d.relu; a.final_layer = d.final; a.coef = l.coef;
+            // replace construction: the classifier's accumulated-checksum neuron
+            // sums every input feature (the checksum channel is one of them)
+            a.protect = m->protect || (m->replace && d.final);
             a.ref = m->ref; a.tau = m->tau;
             if (d.final) { a.y = logits; a.S = S; a.flag = flag; }
             else { a.y = dst.data; a.ycs = dst.has_cs ? dst.cs : nullptr; }
@@ -819,6 +943,7 @@ ct_status ct_build(const ct_model_desc *desc, const float *const *weights, const
                    ct_model **out) {
     if (!desc || !weights || !opts || !out || desc->n_layers < 1 || !desc->layers) return CT_EINVAL;
     if (opts->precision != CT_FP32 && opts->precision != CT_FP16) return CT_EINVAL;
+    if (opts->protect < CT_PROTECT_NONE || opts->protect > CT_PROTECT_REPLACE) return CT_EINVAL;
     if (opts->max_batch < 1 || desc->in_c < 1 || desc->in_h < 1 || desc->in_w < 1 || desc->n_classes < 1)
         return CT_EINVAL;
     *out = nullptr;
@@ -832,7 +957,8 @@ ct_status ct_build(const ct_model_desc *desc, const float *const *weights, const
     if (!m) return CT_ENOMEM;
     m->device = opts->device;
     m->prec = opts->precision;
-    m->protect = opts->protect != 0;
+    m->protect = opts->protect == CT_PROTECT_WIDEN;
+    m->replace = opts->protect == CT_PROTECT_REPLACE;
     m->ds_mode = opts->ds_mode;
     m->max_batch = opts->max_batch;
     m->flags = opts->flags;
