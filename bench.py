@@ -226,17 +226,26 @@ def main():
     # room for the previous batch's flagged images riding along (deferred re-execution)
     mp = ct.ct_build_workload(wl, params, device=local, simt_only=args.simt_only, max_batch=B + REEXEC_ROOM)
     mu = ct.ct_build_workload(wl, params, device=local, simt_only=args.simt_only, protect=False)
+    # the paper's prune-and-replace construction of the same network
+    mr = ct.ct_build_workload(wl, params, device=local, simt_only=args.simt_only, replace=True,
+                              max_batch=B + REEXEC_ROOM)
 
     # calibration (Sec. II-C, distribution-based, alpha = 1%) on seeded fault-free images
     calib_n = 2 * B
     xc = torch.from_numpy(synth.make_input(wl, batch=calib_n, seed=wl.calib_seed)).cuda()
     Sc = torch.empty(calib_n, device="cuda")
     lc = torch.empty(B, wl.n_classes, device="cuda")
-    for i in range(0, calib_n, B):
-        ct.ct_infer(mp, xc[i:i + B], B, lc, Sc[i:i + B], None)
-    torch.cuda.synchronize()
-    r, tau = ct.ct_calibrate(Sc.cpu().numpy(), 0.01)
-    ct.ct_set_threshold(mp, r, tau)
+
+    def calibrate(model):
+        for i in range(0, calib_n, B):
+            ct.ct_infer(model, xc[i:i + B], B, lc, Sc[i:i + B], None)
+        torch.cuda.synchronize()
+        rr, tt = ct.ct_calibrate(Sc.cpu().numpy(), 0.01)
+        ct.ct_set_threshold(model, rr, tt)
+        return rr, tt
+
+    r, tau = calibrate(mp)
+    r_rep, tau_rep = calibrate(mr)
     del xc
 
     # evaluation batches for this rank (distinct slices of the seeded set per
@@ -255,20 +264,21 @@ def main():
         ct.ct_infer(mp, x, B, logits, S, flag, stream)
         return ct.ct_reexecute(mp, x, B, flag, logits, S, stream)
 
-    def deferred_steps(steps):
+    def deferred_steps(steps, model=None):
         """`steps` protected steps in which the flagged images of each batch
         are re-executed as extra rows of the next batch's inference
         (ct_infer_reexec); the last batch's are re-run at the end."""
+        model = model or mp
         n_re, prev = 0, None
         for i in range(steps):
             cur = bufs[i % 2]
             if prev is None:
-                n_re += ct.ct_infer_reexec(mp, cur["x"], B, cur["lg"], cur["S"], cur["fl"], stream=stream)
+                n_re += ct.ct_infer_reexec(model, cur["x"], B, cur["lg"], cur["S"], cur["fl"], stream=stream)
             else:
-                n_re += ct.ct_infer_reexec(mp, cur["x"], B, cur["lg"], cur["S"], cur["fl"], prev["x"], B,
+                n_re += ct.ct_infer_reexec(model, cur["x"], B, cur["lg"], cur["S"], cur["fl"], prev["x"], B,
                                            prev["fl"], prev["lg"], prev["S"], stream)
             prev = cur
-        n_re += ct.ct_reexecute(mp, prev["x"], B, prev["fl"], prev["lg"], prev["S"], stream)
+        n_re += ct.ct_reexecute(model, prev["x"], B, prev["fl"], prev["lg"], prev["S"], stream)
         return n_re
 
     def step_unprotected():
@@ -303,6 +313,7 @@ def main():
         step_protected()
         step_unprotected()
     deferred_steps(max(args.warmup, 3))
+    deferred_steps(max(args.warmup, 3), mr)
     torch.cuda.synchronize()
 
     # unprotected reference (same kernels, no carry-through filters)
@@ -327,6 +338,16 @@ def main():
     # synchronous re-execution (each batch's flagged images as their own
     # small batch, replayed from a CUDA graph), for comparison
     ms_ps, n_rerun_s = timed(step_protected, args.steps)
+
+    # the paper's prune-and-replace construction: same steps, and its
+    # inference alone
+    ms_r, n_rerun_r = timed(lambda k: deferred_steps(k, mr), args.steps, loop=True)
+
+    def step_replace_infer():
+        ct.ct_infer(mr, x, B, logits, S, flag, stream)
+        return 0
+    ms_ri, _ = timed(step_replace_infer, args.steps)
+    err_r = ct.ct_device_error(mr)
 
     # the headline steps again with CUDA events around every kernel on the
     # launch stream: per-family launches, device time and FLOPs for the roofline
@@ -491,6 +512,15 @@ def main():
         "value_sync_reexec": world * B * args.steps / (ms_ps / 1e3),
         "overhead_reexec_sync_pct": 100.0 * (ms_ps - ms_pi) / ms_u,
         "reexecuted_images_per_step_sync": n_rerun_s / args.steps,
+        "replace_construction": {
+            "what": "Sec. II-A prune-and-replace (ct_build CT_PROTECT_REPLACE): the least important channel of "
+                    "every tensor gives its place to the carry-through filter; no fine-tuning",
+            "value": world * B * args.steps / (ms_r / 1e3), "unit": "images/s",
+            "overhead_pct": 100.0 * (ms_r / ms_u - 1.0),
+            "overhead_filters_pct": 100.0 * (ms_ri / ms_u - 1.0),
+            "reexecuted_images_per_step": n_rerun_r / args.steps,
+            "threshold": {"reference": r_rep, "tau": tau_rep},
+            "device_error": err_r},
         "conv_tflop_per_batch": conv_flops(wl) / 1e12,
         "roofline": roof,
         "cpu_baseline": cpu,
