@@ -235,6 +235,42 @@ ct_status ct_infer_reexec(ct_model *m, const float *input_dev, int32_t batch, fl
                           int32_t prev_batch, const uint8_t *prev_flag_dev, float *prev_logits_dev,
                           float *prev_S_dev, int32_t *n_rerun, void *stream);
 
+/* One fault of a batched campaign: the arguments of ct_inject. */
+typedef struct {
+    int32_t kind;        /* ct_buf_kind */
+    int32_t layer;       /* index into desc->layers of a convolution */
+    int64_t element;     /* literal-layout element, as for ct_inject */
+    int32_t bit;
+} ct_fault;
+
+/* ct_campaign_batched -- Sec. III-A fault-injection campaign, many faults
+ * in ONE launch: for fault f and image n of the batch input_dev
+ * [batch, C, H, W] (FP32, device), the result of ct_inject(faults[f]) +
+ * ct_infer of that batch, without re-execution:
+ *   S_dev[f * batch + n] (FP32), top1_dev[f * batch + n] (int32: argmax of
+ *   the logits, lowest index on ties, -1 if any logit is NaN),
+ *   flag_dev[f * batch + n] (uint8: NOT(|S - reference| <= tau)).
+ * A weight fault (CT_BUF_WEIGHT, a convolution's literal weight layout)
+ * touches every image, so all `batch` entries of its row are written.  An
+ * activation fault (CT_BUF_ACT, element of [batch, C_tot, H, W] of the
+ * second convolution's input) touches one image: only that image's entry is
+ * written, the rest of the row is left as it was.
+ * Each CTA holds its own copy of the convolution weights in shared memory,
+ * flipped for its fault, and runs the whole network for its images; the
+ * model's weights are never modified.  Supported networks: FP32, widened
+ * (CT_PROTECT_WIDEN), the LeNet-5 shape -- an unpadded stride-1
+ * convolution with a carry-through filter, 2x2 stride-2 max-pool, the same
+ * again, then FC, FC, classifier, with ReLU after every convolution and
+ * hidden FC -- small enough for one CTA's shared memory; CT_EUNSUPPORTED
+ * otherwise.  The first convolution's input (the image) is not a fault site.
+ * `faults` is host memory, read before the call returns.  Asynchronous on
+ * `stream` after one synchronisation (the previous call's fault list).
+ * Errors: CT_EINVAL, CT_ERANGE (batch, layer, element or bit out of range),
+ * CT_EUNSUPPORTED, CT_ENOMEM, CT_ECUDA. */
+ct_status ct_campaign_batched(ct_model *m, const float *input_dev, int32_t batch,
+                              const ct_fault *faults, int32_t n_faults, float *S_dev,
+                              int32_t *top1_dev, uint8_t *flag_dev, void *stream);
+
 /* ct_reexecute_noalloc -- the same re-execution as ct_reexecute, for callers
  * that must not allocate device memory while they run: real-time loops whose
  * device memory is fixed at start-up so that a request can never fail for

@@ -38,7 +38,7 @@ EXPORTS = ["ct_build", "ct_set_threshold", "ct_get_threshold", "ct_infer", "ct_i
            "ct_buffer_info", "ct_profile_enable", "ct_profile_read", "ct_launches_per_infer", "ct_kernel_count",
            "ct_fi_threshold",
            "ct_copy_activation", "ct_device_error", "ct_destroy", "ct_strerror",
-           "ct_reexecute_noalloc"]
+           "ct_reexecute_noalloc", "ct_campaign_batched"]
 
 CT_NOALLOC_SCRATCH_BYTES = 16 * 1024 * 1024
 
@@ -59,6 +59,11 @@ class ModelDesc(ctypes.Structure):
     _fields_ = [("n_layers", ctypes.c_int32), ("layers", ctypes.POINTER(LayerDesc)),
                 ("in_c", ctypes.c_int32), ("in_h", ctypes.c_int32), ("in_w", ctypes.c_int32),
                 ("n_classes", ctypes.c_int32), ("bn_eps", ctypes.c_double)]
+
+
+class FaultDesc(ctypes.Structure):
+    _fields_ = [("kind", ctypes.c_int32), ("layer", ctypes.c_int32), ("element", ctypes.c_int64),
+                ("bit", ctypes.c_int32)]
 
 
 class BuildOpts(ctypes.Structure):
@@ -101,6 +106,7 @@ def lib():
             "ct_kernel_count": [vp, P(i64)],
             "ct_copy_activation": [vp, i32, i32, vp, vp, P(i32), P(i32), P(i32), P(i32), P(i32), vp],
             "ct_device_error": [vp, P(ctypes.c_uint32)],
+            "ct_campaign_batched": [vp, vp, i32, P(FaultDesc), i32, vp, vp, vp, vp],
         }
         for name, args in sig.items():
             f = getattr(L, name)
@@ -256,6 +262,17 @@ def ct_infer_reexec(m: Model, input_dev, batch: int, logits_dev, S_dev=None, fla
                                  _ptr(prev_input_dev), prev_batch, _ptr(prev_flag_dev), _ptr(prev_logits_dev),
                                  _ptr(prev_S_dev), ctypes.byref(n), _stream(stream)), "ct_infer_reexec")
     return n.value
+
+
+def ct_campaign_batched(m: Model, input_dev, batch: int, faults, S_dev, top1_dev, flag_dev, stream=None):
+    """Many faults in one launch.  faults: rows (kind, layer, element, bit);
+    outputs [n_faults, batch] device tensors (float32, int32, uint8)."""
+    f = np.asarray(faults, dtype=np.int64).reshape(-1, 4)
+    arr = (FaultDesc * max(len(f), 1))()
+    for i, (kind, layer, el, bit) in enumerate(f.tolist()):
+        arr[i] = FaultDesc(kind, layer, el, bit)
+    _check(lib().ct_campaign_batched(m.handle, _ptr(input_dev), batch, arr, len(f), _ptr(S_dev), _ptr(top1_dev),
+                                     _ptr(flag_dev), _stream(stream)), "ct_campaign_batched")
 
 
 def ct_reexecute_noalloc(m: Model, input_dev, batch: int, flag_dev, logits_dev, S_dev=None,

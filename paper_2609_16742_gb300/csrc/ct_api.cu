@@ -134,6 +134,9 @@ struct ct_model {
     int32_t *re_idx = nullptr;
     uint8_t *h_flags = nullptr;
     int32_t *h_idx = nullptr;
+    // batched campaign: resolved faults (device) and their pinned staging
+    CampFault *camp_d = nullptr, *camp_h = nullptr;
+    int camp_cap = 0;
     float *rh_input = nullptr, *rh_logits = nullptr, *rh_S = nullptr;
     uint8_t *rh_flag = nullptr;
     uint32_t *d_err = nullptr;
@@ -189,6 +192,8 @@ void free_all(ct_model *m) {
     for (void *p : m->dev_allocs) cudaFree(p);
     m->dev_allocs.clear();
     if (m->h_flags) cudaFreeHost(m->h_flags);
+    if (m->camp_h) cudaFreeHost(m->camp_h);
+    if (m->camp_d) cudaFree(m->camp_d);
     if (m->h_idx) cudaFreeHost(m->h_idx);
     for (auto &e : m->ev_pool) { cudaEventDestroy(e.first); cudaEventDestroy(e.second); }
     m->ev_pool.clear();
@@ -1051,6 +1056,104 @@ ct_status ct_infer_reexec(ct_model *m, const float *input_dev, int32_t batch, fl
                                     (cudaStream_t)stream);
     if (n_rerun) *n_rerun = n;
     return s;
+}
+
+// The LeNet shape the batched campaign kernel runs (FP32, widened):
+// conv -> pool -> conv -> pool -> fc -> fc -> fc, with ReLU after every conv
+// and hidden FC, 2x2 stride-2 pools, unpadded stride-1 convolutions with a
+// carry-through filter.
+static bool small_net_of(const ct_model *m, SmallNet *g) {
+    if (m->prec != CT_FP32 || !m->protect || m->L.size() != 7) return false;
+    const LayerRT &c1 = m->L[0], &p1 = m->L[1], &c2 = m->L[2], &p2 = m->L[3];
+    const LayerRT &f1 = m->L[4], &f2 = m->L[5], &f3 = m->L[6];
+    auto conv_ok = [](const LayerRT &l) {
+        return l.d.op == CT_OP_CONV && l.d.stride == 1 && l.d.pad == 0 && l.d.relu && l.d.res < 0 &&
+               l.role == CT_ROLE_CT && l.R == l.S && l.w_ld == l.R * l.S * l.C && l.c_stride == l.C;
+    };
+    auto pool_ok = [](const LayerRT &l) { return l.d.op == CT_OP_MAXPOOL && l.d.k == 2 && l.d.stride == 2 && l.d.pad == 0; };
+    if (!conv_ok(c1) || !pool_ok(p1) || !conv_ok(c2) || !pool_ok(p2)) return false;
+    if (c1.d.src != 0 || p1.d.src != c1.d.dst || c2.d.src != p1.d.dst || p2.d.src != c2.d.dst) return false;
+    if (f1.d.op != CT_OP_FC || f2.d.op != CT_OP_FC || f3.d.op != CT_OP_FC || !f1.d.relu || !f2.d.relu ||
+        !f3.d.final || f1.d.src != p2.d.dst || f2.d.src != f1.d.dst || f3.d.src != f2.d.dst)
+        return false;
+    if (c1.cs_in || !c2.cs_in || f1.x_float || f1.fc_tc || f2.fc_tc) return false;
+    const Slot &s1 = m->slots[p1.d.dst], &s2 = m->slots[p2.d.dst];
+    SmallNet &n = *g;
+    memset(&n, 0, sizeof(n));
+    n.C0 = c1.C; n.H0 = c1.H; n.W0 = c1.W;
+    n.K1 = c1.K; n.R1 = c1.R; n.H1 = c1.P; n.W1 = c1.Q; n.Hp1 = s1.H; n.Wp1 = s1.W;
+    n.K2 = c2.K; n.R2 = c2.R; n.H2 = c2.P; n.W2 = c2.Q; n.Hp2 = s2.H; n.Wp2 = s2.W;
+    n.NIN1 = f1.n_in; n.N1 = f1.n_out; n.N2 = f2.n_out; n.N3 = f3.n_out;
+    if (n.NIN1 != n.K2 * n.Hp2 * n.Wp2 || f1.n_cs != n.Hp2 * n.Wp2 || f2.n_in != n.N1 || f3.n_in != n.N2) return false;
+    n.w1 = (const float *)c1.w; n.b1 = c1.bias; n.w2 = (const float *)c2.w; n.b2 = c2.bias;
+    n.wf1 = (const float *)f1.w; n.bf1 = f1.bias; n.wf2 = (const float *)f2.w; n.bf2 = f2.bias;
+    n.wf3 = (const float *)f3.w; n.bf3 = f3.bias;
+    n.coef1 = c1.coef; n.coef2 = c2.coef; n.coeff1 = f1.coef; n.coeff2 = f2.coef; n.coeff3 = f3.coef;
+    n.ref = m->ref; n.tau = m->tau;
+    return campaign_small_smem(n) <= 200 * 1024;
+}
+
+ct_status ct_campaign_batched(ct_model *m, const float *input_dev, int32_t batch, const ct_fault *faults,
+                              int32_t n_faults, float *S_dev, int32_t *top1_dev, uint8_t *flag_dev, void *stream) {
+    if (!m || !input_dev || (n_faults > 0 && (!faults || !S_dev || !top1_dev || !flag_dev)) || n_faults < 0)
+        return CT_EINVAL;
+    if (batch < 1 || batch > m->max_batch) return CT_ERANGE;
+    SmallNet g;
+    if (!small_net_of(m, &g)) return CT_EUNSUPPORTED;
+    if (n_faults == 0) return CT_OK;
+    g.B = batch;
+    g.x = input_dev;
+    DeviceGuard dg(m->device);
+    cudaStream_t st = (cudaStream_t)stream;
+    // resolve every fault on the host, as ct_inject + ct_infer would
+    if (n_faults > m->camp_cap) {
+        CUDA_TRY(cudaStreamSynchronize(st));
+        if (m->camp_h) cudaFreeHost(m->camp_h);
+        if (m->camp_d) cudaFree(m->camp_d);
+        m->camp_h = nullptr; m->camp_d = nullptr; m->camp_cap = 0;
+        if (cudaMallocHost((void **)&m->camp_h, sizeof(CampFault) * n_faults) != cudaSuccess ||
+            cudaMalloc((void **)&m->camp_d, sizeof(CampFault) * n_faults) != cudaSuccess) {
+            cudaGetLastError();
+            return CT_ENOMEM;
+        }
+        m->camp_cap = n_faults;
+    } else {
+        CUDA_TRY(cudaStreamSynchronize(st));        // the staging of the previous call was copied
+    }
+    const int per_img = (g.K1 + 1) * g.Hp1 * g.Wp1;
+    for (int i = 0; i < n_faults; ++i) {
+        const ct_fault &fi = faults[i];
+        CampFault &cf = m->camp_h[i];
+        memset(&cf, 0, sizeof(cf));
+        cf.kind = fi.kind;
+        cf.bit = fi.bit;
+        cf.word = -1;
+        if (fi.bit < 0 || fi.bit >= 32) return CT_ERANGE;
+        if (fi.kind == CT_BUF_WEIGHT) {
+            if (fi.layer != 0 && fi.layer != 2) return CT_ERANGE;
+            const LayerRT &l = m->L[fi.layer];
+            const int64_t n_el = (int64_t)(l.K + 1) * (l.C + (l.cs_in ? 1 : 0)) * l.R * l.S;
+            if (fi.element < 0 || fi.element >= n_el) return CT_ERANGE;
+            cf.layer = fi.layer == 0 ? 0 : 1;
+            const WeightFault wf = resolve_weight_fault(m, l, fi.element, fi.bit);
+            if (wf.explicit_word) cf.word = wf.word;
+            else cf.fd = wf.fd;
+        } else if (fi.kind == CT_BUF_ACT) {
+            // the second convolution's input; the network input is not a fault site
+            if (fi.layer != 2 || fi.element < 0 || fi.element >= (int64_t)batch * per_img) return CT_ERANGE;
+            cf.img = (int)(fi.element / per_img);
+            const int within = (int)(fi.element % per_img);
+            cf.act_c = within / (g.Hp1 * g.Wp1);
+            cf.act_hw = within % (g.Hp1 * g.Wp1);
+        } else {
+            return CT_EINVAL;
+        }
+    }
+    CUDA_TRY(cudaMemcpyAsync(m->camp_d, m->camp_h, sizeof(CampFault) * n_faults, cudaMemcpyHostToDevice, st));
+    CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] {
+        return launch_campaign_small(g, m->camp_d, n_faults, S_dev, top1_dev, flag_dev, st);
+    }));
+    return CT_OK;
 }
 
 ct_status ct_run_host(ct_model *m, const float *input_host, int32_t batch, float *logits_host,

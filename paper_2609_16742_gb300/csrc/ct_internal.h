@@ -47,6 +47,34 @@ struct ConvArgs {
     int n_split;          // (null x2: every image comes from x)
 };
 
+// Batched campaign on a LeNet-shaped FP32 network (campaign_small.cu):
+// shapes, the model's device weights (convolutions KRSC, FC rows with
+// columns in the NHWC flatten order), coefficients and threshold.
+struct SmallNet {
+    int B, C0, H0, W0;
+    int K1, R1, H1, W1, Hp1, Wp1;
+    int K2, R2, H2, W2, Hp2, Wp2;
+    int NIN1, N1, N2, N3;
+    const float *x;                       // [B, C0, H0, W0] FP32 images
+    const float *w1, *b1, *w2, *b2, *wf1, *bf1, *wf2, *bf2, *wf3, *bf3;
+    float coef1, coef2, coeff1, coeff2, coeff3;
+    double ref, tau;
+};
+
+// One fault of a batched campaign, resolved on the host.
+struct CampFault {
+    int kind;            // 0 weight, 1 activation
+    int layer;           // weight: 0 first convolution, 1 second
+    long long word;      // weight: stored word to flip (-1: use fd)
+    int bit;
+    FaultDelta fd;       // weight: element of the construction that is not stored
+    int img, act_c, act_hw;   // activation: image, channel (K1 = checksum), pixel of the first pool's output
+};
+
+size_t campaign_small_smem(const SmallNet &g);
+cudaError_t launch_campaign_small(const SmallNet &g, const CampFault *faults, int n_faults, float *S, int32_t *top1,
+                                  uint8_t *flag, cudaStream_t st);
+
 struct FcArgs {
     const void *x;        // [B, n_in] data features
     const void *xcs;      // [B, n_cs] checksum features or null
