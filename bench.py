@@ -488,6 +488,14 @@ def main():
                           "activations": c["activations"]["detected_fraction_of_critical"],
                           "wall_s": c["wall_s"], "time_relative_to_fault_free": c["time_relative_to_fault_free"],
                           "reexecuted_images": c["reexecuted_images"], "device_error": c["device_error"]}
+        # LeNet-5 (FP32): 100,000 faults in one launch of the batched campaign kernel
+        cb = campaign.run_batched(faults=100 * args.campaign_faults, seed=0, device=local)
+        camp["lenet5_batched"] = {"faults": cb["faults"], "batch": cb["batch"], "wall_s": cb["wall_s"],
+                                  "faults_per_s": cb["faults_per_s"],
+                                  "detected_fraction_of_critical": cb["all"]["detected_fraction_of_critical"],
+                                  "critical": cb["all"]["critical"], "trials": cb["all"]["trials"],
+                                  "false_alarm_rate": cb["all"]["false_alarm_rate"],
+                                  "device_error": cb["device_error"]}
 
     in_bytes = B * int(np.prod(wl.in_shape)) * 4
     out_bytes = B * (wl.n_classes * 4 + 4 + 1)

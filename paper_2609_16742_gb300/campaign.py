@@ -235,6 +235,68 @@ def run(precision="fp32", faults=1000, seed=0, batch=None, calib_images=10000, a
     return out
 
 
+def run_batched(faults=100000, seed=0, calib_images=10000, alpha=0.01, device=0):
+    """The campaign of run() on LeNet-5 (FP32) with ct_campaign_batched: all
+    faults in one launch (no re-execution).  Returns the same counters."""
+    sys.path.insert(0, os.path.dirname(os.path.dirname(os.path.abspath(__file__))))
+    import numpy as np
+    import torch
+    import synth
+    import paper_2609_16742_gb300 as ct
+
+    torch.cuda.set_device(device)
+    wl = synth.workload("lenet5")
+    B = wl.batch
+    m = ct.ct_build_workload(wl, synth.make_params(wl.layers, wl.seed), max_batch=B, device=device)
+    stream = torch.cuda.current_stream()
+    n_cal = ((calib_images + B - 1) // B) * B
+    xc = torch.from_numpy(synth.make_input(wl, batch=n_cal, seed=wl.calib_seed)).cuda()
+    Sc = torch.empty(n_cal, device="cuda")
+    lc = torch.empty(B, wl.n_classes, device="cuda")
+    for i in range(0, n_cal, B):
+        ct.ct_infer(m, xc[i:i + B], B, lc, Sc[i:i + B], None, stream)
+    torch.cuda.synchronize()
+    r, tau = ct.ct_calibrate(Sc.cpu().numpy(), alpha)
+    ct.ct_set_threshold(m, r, tau)
+    x = torch.from_numpy(synth.make_input(wl, batch=B)).cuda()
+    logits = torch.empty(B, wl.n_classes, device="cuda")
+    ct.ct_infer(m, x, B, logits, None, None, stream)
+    golden = _top1(logits).to(torch.int32)
+    bufs = ct.ct_buffers(m, B)
+    sites = synth.draw_faults(bufs, faults, seed)
+    F = len(sites)
+    S = torch.full((F, B), float("nan"), device="cuda")
+    top1 = torch.full((F, B), -2, dtype=torch.int32, device="cuda")
+    flag = torch.zeros((F, B), dtype=torch.uint8, device="cuda")
+    ct.ct_campaign_batched(m, x, B, sites[:1], S, top1, flag, stream)      # warm-up
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    ct.ct_campaign_batched(m, x, B, sites, S, top1, flag, stream)
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - t0
+    # trials: every image of a weight fault, the hit image of an activation fault
+    valid = top1 != -2
+    crit = valid & (top1 != golden[None, :])
+    fl = valid & (flag != 0)
+    kinds = torch.from_numpy(np.ascontiguousarray(sites[:, 0])).cuda()
+
+    def summary(sel):
+        v, c, f_ = valid[sel], crit[sel], fl[sel]
+        trials, critical = int(v.sum()), int(c.sum())
+        det, fa = int((c & f_).sum()), int((~c & f_ & v).sum())
+        non = trials - critical
+        return {"trials": trials, "critical": critical, "detected": det, "false_alarms": fa,
+                "detected_fraction_of_critical": det / critical if critical else None,
+                "false_alarm_rate": fa / non if non else None}
+
+    out = {"network": "lenet5", "precision": "fp32", "faults": F, "seed": seed, "batch": B,
+           "threshold": {"reference": r, "tau": tau, "alpha": alpha, "calibration_images": n_cal},
+           "all": summary(slice(None)), "weights": summary(kinds == 0), "activations": summary(kinds == 1),
+           "wall_s": wall, "faults_per_s": F / wall, "device_error": ct.ct_device_error(m)}
+    m.close()
+    return out
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
     ap.add_argument("--precision", default="fp32", choices=["fp32", "fp16"])
@@ -243,9 +305,15 @@ def main(argv=None):
     ap.add_argument("--calib-images", type=int, default=10000)
     ap.add_argument("--alpha", type=float, default=0.01)
     ap.add_argument("--no-reexecute", action="store_true")
+    ap.add_argument("--batched-lenet", action="store_true",
+                    help="LeNet-5 FP32 campaign, all faults in one launch (ct_campaign_batched)")
     ap.add_argument("--sweep", action="store_true",
                     help="compare distribution-based and FI-based thresholds over alpha in {0.1, 1, 5}%%")
     args = ap.parse_args(argv)
+    if args.batched_lenet:
+        out = run_batched(args.faults, args.seed, calib_images=args.calib_images, alpha=args.alpha)
+        print(json.dumps(out))
+        return 0 if out["device_error"] == 0 else 1
     if args.sweep:
         out = sweep(args.precision, args.faults, seed_cal=args.seed + 1, seed_eval=args.seed + 2,
                     calib_images=args.calib_images)

@@ -140,3 +140,14 @@ def test_batched_rejects_other_networks_and_sites():
     with pytest.raises(ct().CtError):              # the image is not a fault site
         _batched(m, x, np.array([[1, 0, 0, 1]]))
     m.close()
+
+
+def test_batched_campaign_runner_bookkeeping():
+    from paper_2609_16742_gb300 import campaign
+    out = campaign.run_batched(faults=2000, seed=4, calib_images=512)
+    assert out["device_error"] == 0
+    a, w, act = out["all"], out["weights"], out["activations"]
+    assert a["detected"] <= a["critical"] <= a["trials"]
+    assert w["trials"] % out["batch"] == 0
+    assert w["trials"] // out["batch"] + act["trials"] == 2000
+    assert a["trials"] == w["trials"] + act["trials"]
