@@ -156,6 +156,31 @@ def conv2d(x: np.ndarray, w: np.ndarray, skip: Optional[np.ndarray], stride: int
     return y
 
 
+def depthwise2d(x: np.ndarray, w: np.ndarray, skip: Optional[np.ndarray], stride: int, pad: int) -> np.ndarray:
+    """Depthwise convolution of one image x [C, H, W] with w [C, 1, R, S]
+    (double): output channel c is the correlation of input channel c with
+    its filter, taps added in (r, s) order; skipped taps are not multiplied."""
+    C, H, W = x.shape
+    K, one, R, S = w.shape
+    assert K == C and one == 1, (w.shape, x.shape)
+    P = (H + 2 * pad - R) // stride + 1
+    Q = (W + 2 * pad - S) // stride + 1
+    xp = np.zeros((C, H + 2 * pad, W + 2 * pad))
+    xp[:, pad:pad + H, pad:pad + W] = x
+    y = np.zeros((C, P, Q))
+    for r in range(R):
+        for s_ in range(S):
+            win = xp[:, r:r + stride * (P - 1) + 1:stride, s_:s_ + stride * (Q - 1) + 1:stride]
+            tap = w[:, 0, r, s_].astype(np.float64)
+            if skip is not None:
+                tap = np.where(skip[:, 0, r, s_] != 0, 0.0, tap)
+                live = skip[:, 0, r, s_] == 0
+                y[live] += tap[live, None, None] * win[live]
+            else:
+                y += tap[:, None, None] * win
+    return y
+
+
 def relu(y: np.ndarray) -> np.ndarray:
     """max(y, 0) that keeps NaN (and -0.0) as they are: y < 0 -> +0."""
     return np.where(y < 0, 0.0, y)
@@ -200,6 +225,7 @@ class OLayer:
     pad: int = 0
     k: int = 1
     ct: str = "none"
+    groups: int = 1                     # > 1: depthwise (W is [K_tot, 1, k, k])
     W: Optional[np.ndarray] = None      # literal weights (float64 holding storage values)
     skip: Optional[np.ndarray] = None   # structural zeros of the construction
     b: Optional[np.ndarray] = None      # fp32 biases as float64
@@ -225,7 +251,39 @@ def build(layers: Sequence[synth.Layer], params, prec: str, protected: bool = Tr
     n_data = {0: in_shape[0] if in_shape else None}
     out: List[OLayer] = []
     for L, P in zip(layers, params):
-        if L.op == "conv":
+        if L.op == "conv" and L.groups > 1:
+            # Depthwise (reading: the paper builds the carry-through filter for
+            # dense convolutions only).  The checksum is one more group: its
+            # filter sees only the incoming checksum channel, so it passes the
+            # checksum through at the centre tap (weight 1); off-centre taps
+            # of that filter are structural zeros.  Without an incoming
+            # checksum there is nothing to pass.
+            assert L.groups == L.cin == L.cout
+            cs_in = has_cs[L.src]
+            w = P["w"].astype(np.float64)
+            b = P["b"].astype(np.float64)
+            if L.bn:
+                w, b = fold_bn(w, b, P, bn_eps)
+            w = round_to(w, prec)
+            b = round_to(b, "fp32") if prec != "fp64" else b
+            passes = protected and cs_in and L.ct != "none"
+            K = L.cout + (1 if passes else 0)
+            W = np.zeros((K, 1, L.k, L.k))
+            skip = np.zeros((K, 1, L.k, L.k), dtype=np.uint8)
+            W[:L.cout] = w
+            ctr = (L.k - 1) // 2
+            if passes:
+                skip[L.cout] = 1
+                skip[L.cout, 0, ctr, ctr] = 0
+                W[L.cout, 0, ctr, ctr] = 1.0
+            bb = np.zeros(K)
+            bb[:L.cout] = b
+            has_cs[L.dst] = passes
+            n_data[L.dst] = L.cout
+            out.append(OLayer("conv", L.src, L.dst, res=L.res, relu=L.relu, stride=L.stride,
+                              pad=L.pad, k=L.k, ct="pass" if passes else "none", groups=L.groups, W=W,
+                              skip=skip, b=bb, n_data_out=L.cout, has_ct_out=passes))
+        elif L.op == "conv":
             ct = L.ct if protected else "none"
             if ct == "pass" and ds_mode == "zero":
                 ct = "none"
@@ -322,12 +380,19 @@ def weight_shape(net: ONet, layer: int) -> tuple:
     return net.layers[layer].W.shape
 
 
+def _in_channels(net: ONet, L: OLayer) -> int:
+    """Channels of a convolution's input tensor, checksum included."""
+    if L.groups > 1:
+        return net.n_data[L.src] + (1 if net.has_cs[L.src] else 0)
+    return L.W.shape[1]
+
+
 def act_shape(net: ONet, layer: int, batch: int) -> tuple:
     """Literal layout [B, C_tot, H, W] of the input tensor of conv ``layer``."""
     L = net.layers[layer]
     assert L.op == "conv"
     H, W = slot_hw(net)[L.src]
-    return (batch, L.W.shape[1], H, W)
+    return (batch, _in_channels(net, L), H, W)
 
 
 def slot_hw(net: ONet) -> Dict[int, tuple]:
@@ -363,7 +428,7 @@ def fault_buffers(net: ONet, batch: int, include_input: bool = False) -> List[tu
             seen.add(L.src)
             if L.src == 0 and not include_input:
                 continue
-            C = L.W.shape[1]
+            C = _in_channels(net, L)
             H, W = hw[L.src]
             bufs.append((1, i, int(batch * C * H * W), bits))
     return bufs
@@ -396,7 +461,12 @@ def forward(net: ONet, x: np.ndarray, fault: Optional[Fault] = None, keep: bool 
                 if wfault_layer is not None and wfault_layer[0] == li:
                     W, sk = wfault_layer[1], wfault_layer[2]
                 xin = acts[L.src]
-                y = conv2d(xin, W, sk, L.stride, L.pad) + L.b[:, None, None]
+                if L.groups > 1:
+                    # the filters read the first K_tot input channels (the
+                    # checksum filter the checksum channel, when it exists)
+                    y = depthwise2d(xin[:W.shape[0]], W, sk, L.stride, L.pad) + L.b[:, None, None]
+                else:
+                    y = conv2d(xin, W, sk, L.stride, L.pad) + L.b[:, None, None]
                 if L.res >= 0:
                     r = acts[L.res]
                     nd = L.n_data_out

@@ -140,6 +140,8 @@ class Layer:
       "none" : the layer gets none (first conv of a residual block)
       "pass" : a 1x1 shortcut convolution
     How each role is realised is decided by the consumer.
+    ``groups`` > 1 is a depthwise convolution (groups == cin == cout):
+    output channel c reads input channel c only.
     """
     op: str
     src: int
@@ -155,6 +157,7 @@ class Layer:
     res: int = -1
     final: bool = False
     ct_shift: int = 0      # carry-through coefficient is 2**-ct_shift
+    groups: int = 1
 
 
 @dataclass
@@ -246,6 +249,59 @@ def vgg16(n_classes: int = 1000, fc1_shift: int = 0) -> List[Layer]:
     return L
 
 
+def mobilenet_v2(n_classes: int = 10) -> List[Layer]:
+    """MobileNet-V2 for 32 x 32 inputs (first convolution and first
+    bottleneck stage at stride 1): stem 3x3 -> 32, inverted-residual
+    bottlenecks (t, c, n, s) = (1,16,1,1) (6,24,2,1) (6,32,3,2) (6,64,4,2)
+    (6,96,3,1) (6,160,3,2) (6,320,1,1), 1x1 -> 1280, global average pool,
+    FC.  A bottleneck is 1x1 expand (t * cin, BN, ReLU; absent for t = 1),
+    3x3 depthwise (BN, ReLU), 1x1 project (BN, no activation), plus the
+    block input when the stride is 1 and cin == cout.  ReLU stands for the
+    ReLU6 of the original network (Sec. II-A: ReLU6 would saturate the
+    checksum).  Roles: a block with a residual input gets no carry-through
+    filter on its first convolution (Sec. II-A); depthwise layers have the
+    role "pass" (their checksum group sees only the incoming checksum)."""
+    L: List[Layer] = []
+    slot = 0
+
+    def new() -> int:
+        nonlocal slot
+        slot += 1
+        return slot
+
+    s1 = new()
+    L.append(Layer("conv", 0, s1, cin=3, cout=32, k=3, stride=1, pad=1, ct="ct", bn=True, relu=True))
+    x, cin = s1, 32
+    for t, c, n, s in ((1, 16, 1, 1), (6, 24, 2, 1), (6, 32, 3, 2), (6, 64, 4, 2), (6, 96, 3, 1),
+                       (6, 160, 3, 2), (6, 320, 1, 1)):
+        for i in range(n):
+            stride = s if i == 0 else 1
+            residual = stride == 1 and cin == c
+            h, hid = x, cin
+            first = True
+            if t != 1:
+                hid = t * cin
+                e = new()
+                L.append(Layer("conv", x, e, cin=cin, cout=hid, k=1, stride=1, pad=0,
+                               ct="none" if residual else "ct", bn=True, relu=True))
+                h, first = e, False
+            d = new()
+            L.append(Layer("conv", h, d, cin=hid, cout=hid, k=3, stride=stride, pad=1,
+                           ct="pass", bn=True, relu=True, groups=hid))
+            y = new()
+            L.append(Layer("conv", d, y, cin=hid, cout=c, k=1, stride=1, pad=0, ct="ct", bn=True,
+                           relu=False, res=x if residual else -1))
+            assert not (first and residual)
+            x, cin = y, c
+    f = new()
+    L.append(Layer("conv", x, f, cin=cin, cout=1280, k=1, stride=1, pad=0, ct="ct", bn=True, relu=True))
+    g = new()
+    L.append(Layer("gap", f, g))
+    o = new()
+    L.append(Layer("fc", g, o, cin=1280, cout=n_classes, final=True))
+    return L
+
+
 WORKLOADS: Dict[str, Workload] = {
     "lenet5": Workload("lenet5", lenet5(), (1, 28, 28), 10, 64, "fp32", 0, "uniform01",
                        calib_seed=100),
@@ -260,6 +316,8 @@ WORKLOADS: Dict[str, Workload] = {
     "campaign_resnet18_cifar": Workload("campaign_resnet18_cifar", resnet18(False, 10),
                                         (3, 32, 32), 10, 128, "fp32", 5, "normal",
                                         calib_seed=105),
+    "mobilenetv2_cifar": Workload("mobilenetv2_cifar", mobilenet_v2(10), (3, 32, 32), 10, 128,
+                                  "fp32", 6, "normal", calib_seed=106),
 }
 
 
@@ -299,7 +357,7 @@ def shapes(layers: List[Layer], in_shape: tuple) -> Dict[int, tuple]:
 def make_params(layers: List[Layer], seed: int) -> List[Dict[str, np.ndarray]]:
     """Seeded float32 parameters, one dict per layer (empty for pools).
 
-    conv: "w" [cout, cin, k, k] Kaiming-normal (std sqrt(2/(cin*k*k))),
+    conv: "w" [cout, cin / groups, k, k] Kaiming-normal (std sqrt(2/fan_in)),
           "b" zeros [cout]; with bn also "gamma" U[0.9,1.1], "beta" N(0,0.1^2),
           "mean" N(0,0.1^2), "var" U[1,2] (all [cout]).
     fc:   "w" [cout, cin] Kaiming-normal (std sqrt(2/cin)), "b" zeros [cout].
@@ -309,10 +367,11 @@ def make_params(layers: List[Layer], seed: int) -> List[Dict[str, np.ndarray]]:
         st = 16 * (li + 1)
         p: Dict[str, np.ndarray] = {}
         if L.op == "conv":
-            fan = L.cin * L.k * L.k
+            cg = L.cin // L.groups                 # input channels each filter reads
+            fan = cg * L.k * L.k
             n = L.cout * fan
             p["w"] = (normal(seed, st, n) * math.sqrt(2.0 / fan)).astype(np.float32).reshape(
-                L.cout, L.cin, L.k, L.k)
+                L.cout, cg, L.k, L.k)
             p["b"] = np.zeros(L.cout, np.float32)
             if L.bn:
                 p["gamma"] = (0.9 + 0.2 * uniform(seed, st + 1, L.cout)).astype(np.float32)

@@ -28,7 +28,7 @@ def int_params(layers, seed, lo=-2, hi=2, bn=False):
     for L in layers:
         p = {}
         if L.op == "conv":
-            p["w"] = rng.integers(lo, hi + 1, size=(L.cout, L.cin, L.k, L.k)).astype(np.float32)
+            p["w"] = rng.integers(lo, hi + 1, size=(L.cout, L.cin // L.groups, L.k, L.k)).astype(np.float32)
             p["b"] = rng.integers(-2, 3, size=L.cout).astype(np.float32)
             if L.bn:
                 # eps = 0, var = 4, gamma = 1: the folded scale is exactly 0.5
@@ -243,10 +243,68 @@ def test_protected_logits_equal_unprotected(name, prec):
 # O-T3 / O-T4: the checksum equals its closed-form recursion; S sums the FC inputs
 # ---------------------------------------------------------------------------
 
-@pytest.mark.parametrize("which", ["identity", "downsample-pass", "downsample-zero", "lenet"])
+def tiny_mobilenet():
+    """Two inverted-residual blocks (the second with a residual input) around
+    depthwise 3x3 convolutions, one of them stride 2."""
+    return [Layer("conv", 0, 1, cin=2, cout=4, k=3, stride=1, pad=1, ct="ct", bn=True, relu=True),
+            Layer("conv", 1, 2, cin=4, cout=8, k=1, ct="ct", bn=True, relu=True),
+            Layer("conv", 2, 3, cin=8, cout=8, k=3, stride=2, pad=1, ct="pass", bn=True, relu=True, groups=8),
+            Layer("conv", 3, 4, cin=8, cout=4, k=1, ct="ct", bn=True),
+            Layer("conv", 4, 5, cin=4, cout=8, k=1, ct="none", bn=True, relu=True),
+            Layer("conv", 5, 6, cin=8, cout=8, k=3, stride=1, pad=1, ct="pass", bn=True, relu=True, groups=8),
+            Layer("conv", 6, 7, cin=8, cout=4, k=1, ct="ct", bn=True, res=4),
+            Layer("gap", 7, 8),
+            Layer("fc", 8, 9, cin=4, cout=3, final=True)]
+
+
+def test_depthwise_equals_block_diagonal_dense_convolution():
+    """A depthwise convolution is the dense one whose filter k is zero on
+    every input channel but k (brute force through the pinned dense path)."""
+    rng = np.random.default_rng(8)
+    for stride in (1, 2):
+        x = rng.normal(size=(5, 7, 6))
+        w = rng.normal(size=(5, 1, 3, 3))
+        dense = np.zeros((5, 5, 3, 3))
+        for k in range(5):
+            dense[k, k] = w[k, 0]
+        y = oracle.depthwise2d(x, w, None, stride, 1)
+        y_ref = oracle.conv2d(x, dense, None, stride, 1)
+        assert np.allclose(y, y_ref, rtol=1e-13, atol=1e-13)
+        # a skipped tap is not multiplied: an infinite input there stays out
+        sk = np.zeros(w.shape, np.uint8)
+        sk[2, 0, 0, 0] = 1
+        xi = x.copy()
+        xi[2] = np.inf
+        assert not np.isfinite(oracle.depthwise2d(xi, w, None, stride, 1)[2]).all()
+        w0 = w.copy()
+        w0[2, 0, 0, 0] = 0.0
+        y_sk = oracle.depthwise2d(x, w, sk, stride, 1)
+        assert np.allclose(y_sk, oracle.depthwise2d(x, w0, None, stride, 1), rtol=1e-13, atol=1e-13)
+
+
+def test_depthwise_passes_the_checksum_through():
+    """The depthwise layer's checksum group reads only the incoming checksum:
+    its checksum output is the input checksum at the sampled centre (ReLU'd,
+    and the input checksum is already >= 0)."""
+    layers = tiny_mobilenet()
+    params = int_params(layers, 5, bn=True)
+    net = oracle.build(layers, params, "fp64", True, bn_eps=0.0, in_shape=(2, 8, 8), n_classes=3)
+    x = np.random.default_rng(6).integers(-4, 5, size=(1, 2, 8, 8)).astype(np.float32)
+    a = oracle.forward(net, x, keep=True)["acts"][0]
+    assert np.array_equal(a[3][-1], a[2][-1][::2, ::2])          # stride 2, pad 1: centre = 2p
+    assert a[3].shape[0] == 8 + 1
+    # the second block's first convolution has no checksum, so its depthwise
+    # layer has nothing to pass: no extra group, no checksum channel
+    assert a[5].shape[0] == 8 and a[6].shape[0] == 8
+    assert net.layers[5].W.shape == (8, 1, 3, 3) and net.layers[2].W.shape == (9, 1, 3, 3)
+
+
+@pytest.mark.parametrize("which", ["identity", "downsample-pass", "downsample-zero", "lenet", "mobilenet"])
 def test_closed_form_exact_on_integer_nets(which):
     if which == "lenet":
         layers, shape = tiny_lenet(), (1, 10, 10)
+    elif which == "mobilenet":
+        layers, shape = tiny_mobilenet(), (2, 8, 8)
     else:
         layers, shape = tiny_resnet(ds=which != "identity"), (2, 8, 8)
     ds_mode = "zero" if which.endswith("zero") else "pass"
@@ -266,7 +324,7 @@ def test_closed_form_exact_on_integer_nets(which):
         assert cf != 0.0
 
 
-@pytest.mark.parametrize("name", ["lenet5", "resnet18_cifar", "resnet18_imagenet", "vgg16"])
+@pytest.mark.parametrize("name", ["lenet5", "resnet18_cifar", "resnet18_imagenet", "vgg16", "mobilenetv2_cifar"])
 def test_closed_form_gaussian_nets(name):
     wl = synth.workload(name)
     params = cached_params(name)
