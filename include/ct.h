@@ -75,6 +75,15 @@ typedef struct {
     int32_t role;
     int32_t bn, relu, final;
     int32_t ct_shift;
+    int32_t groups;   /* CONV: 1 (dense) or cin == cout (depthwise; weights
+                         [cout, 1, k, k]).  The paper constructs the
+                         carry-through filter for dense convolutions; in a
+                         depthwise layer the checksum is one more group, whose
+                         filter sees only the incoming checksum channel, so it
+                         passes the checksum through at the centre tap (role
+                         CT or PASS; nothing when the input carries no
+                         checksum).  Its literal weight layout is
+                         [cout (+1), 1, k, k].  Not with CT_PROTECT_REPLACE. */
 } ct_layer_desc;
 
 typedef struct {

@@ -52,7 +52,7 @@ class CtError(RuntimeError):
 class LayerDesc(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in
                 ("op", "src", "dst", "res", "cin", "cout", "k", "stride", "pad", "role", "bn",
-                 "relu", "final", "ct_shift")]
+                 "relu", "final", "ct_shift", "groups")]
 
 
 class ModelDesc(ctypes.Structure):
@@ -195,7 +195,7 @@ def ct_build(layers: Sequence, params: Sequence[dict], in_shape, n_classes: int,
     for i, (L, p) in enumerate(zip(layers, params)):
         arr[i] = LayerDesc(_OPS[L.op], L.src, L.dst, L.res, L.cin, L.cout, L.k, L.stride, L.pad,
                            _ROLES.get(L.ct, CT_ROLE_NONE), int(L.bn), int(L.relu), int(L.final),
-                           int(L.ct_shift))
+                           int(L.ct_shift), int(getattr(L, "groups", 1)))
         for j, key in enumerate(("w", "b", "gamma", "beta", "mean", "var")):
             if key in p:
                 a = np.ascontiguousarray(p[key], dtype=np.float32)

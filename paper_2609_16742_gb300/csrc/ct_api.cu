@@ -103,7 +103,11 @@ struct LayerRT {
     int n_in = 0, n_cs = 0, n_out = 0;
     bool x_float = false;
     bool fc_tc = false;          // hidden FC run on the tensor-core conv kernel as a 1x1 conv
+    bool dw = false;             // depthwise convolution: weights [R*S][C]
 };
+
+// input channels a filter of this convolution spans in the literal layout
+int weight_in_channels(const LayerRT &l) { return l.dw ? 1 : l.C + (l.cs_in ? 1 : 0); }
 
 struct EvRec { int fam; int ev; double flops; int nk; };
 
@@ -223,6 +227,7 @@ float flipped(double stored, int bit, int prec) {
 
 // stored word of data-filter weight (k, r, s, c) in the device weight array
 int64_t weight_word(const LayerRT &l, int k, int r, int s, int c) {
+    if (l.dw) return ((int64_t)r * l.S + s) * l.C + k;      // c is 0: the filter's one channel
     if (l.stem) return (int64_t)k * l.w_ld + stem_kidx(r, s, c);
     return (int64_t)k * l.w_ld + ((int64_t)r * l.S + s) * l.c_stride + c;
 }
@@ -323,7 +328,9 @@ std::vector<int> replace_prune_index(const ct_model_desc *desc, const float *con
     for (int i = 0; i < nL; ++i) {
         const ct_layer_desc &d = desc->layers[i];
         const float *w = wts[CT_WEIGHTS_PER_LAYER * i];
+        if (!w) continue;
         if (d.op == CT_OP_CONV) {
+            if (d.groups > 1) continue;
             const int RS = d.k * d.k;
             for (int k = 0; k < d.cout; ++k)
                 for (int c = 0; c < d.cin; ++c) {
@@ -372,7 +379,12 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
     const size_t esz = m->esz();
     const int B = m->max_batch;
     int n_final = 0;
-    // replace construction: pruned channel per slot (-1 elsewhere and in the other modes)
+    // replace construction: pruned channel per slot (-1 elsewhere and in the other
+    // modes).  Its scores read every weight as a dense [cout, cin, k, k] array, so
+    // grouped convolutions are rejected before any weight is read.
+    if (m->replace)
+        for (int i = 0; i < nL; ++i)
+            if (desc->layers[i].op == CT_OP_CONV && desc->layers[i].groups > 1) return CT_EUNSUPPORTED;
     const std::vector<int> pj = m->replace ? replace_prune_index(desc, wts, max_slot + 1)
                                            : std::vector<int>(max_slot + 1, -1);
 
@@ -389,9 +401,15 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
         if (d.op == CT_OP_CONV) {
             if (src.is_float || d.cin != src.C || d.k < 1 || d.stride < 1 || d.pad < 0 || d.cout < 1 || !W)
                 return CT_EINVAL;
+            const int groups = d.groups < 1 ? 1 : d.groups;
+            l.dw = groups > 1;
+            if (l.dw && (groups != d.cin || groups != d.cout || m->replace || !dw_supported(d.cin, d.cout, prec == CT_FP16)))
+                return CT_EUNSUPPORTED;
             int role = m->protect ? d.role : CT_ROLE_NONE;
-            if (role == CT_ROLE_PASS && m->ds_mode == CT_DS_ZERO) role = CT_ROLE_NONE;
+            if (role == CT_ROLE_PASS && m->ds_mode == CT_DS_ZERO && !l.dw) role = CT_ROLE_NONE;
             if (role < CT_ROLE_CT || role > CT_ROLE_PASS) return CT_EINVAL;
+            // depthwise: the checksum group passes the incoming checksum through
+            if (l.dw) role = (role != CT_ROLE_NONE && src.has_cs) ? CT_ROLE_PASS : CT_ROLE_NONE;
             l.role = role;
             l.C = d.cin; l.K = d.cout; l.R = l.S = d.k;
             l.H = src.H; l.W = src.W;
@@ -411,9 +429,9 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
             // scale 1 and bias 0 because its filter is never folded ----
             const int RSC = l.R * l.S * l.C;
             std::string why;
-            l.tc = prec == CT_FP16 && !(m->flags & CT_FLAG_SIMT_ONLY) &&
+            l.tc = !l.dw && prec == CT_FP16 && !(m->flags & CT_FLAG_SIMT_ONLY) &&
                    tc_supported(l.C, l.K, l.R, l.S, d.stride, d.pad, &why);
-            if (prec == CT_FP16 && !(m->flags & CT_FLAG_SIMT_ONLY) && d.src == 0 && d.res < 0 && i + 1 < nL &&
+            if (!l.dw && prec == CT_FP16 && !(m->flags & CT_FLAG_SIMT_ONLY) && d.src == 0 && d.res < 0 && i + 1 < nL &&
                 stem_pool_supported(l.C, l.K, l.R, l.S, d.stride, d.pad, l.H, l.W)) {
                 // the image and the unpooled output must have no other reader
                 const ct_layer_desc &nx = desc->layers[i + 1];
@@ -426,7 +444,7 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
                          nx.pad == 1 && readers_in == 1 && readers_mid == 1;
                 if (l.stem) { src.stored = false; dst.stored = false; }
             }
-            if (!l.stem && prec == CT_FP16 && !(m->flags & CT_FLAG_SIMT_ONLY) && d.src == 0 &&
+            if (!l.dw && !l.stem && prec == CT_FP16 && !(m->flags & CT_FLAG_SIMT_ONLY) && d.src == 0 &&
                 tc_small_supported(l.C, l.K, l.R, l.S, d.stride, d.pad)) {
                 int readers = 0;               // the padded image must have no other reader
                 for (int j = 0; j < nL; ++j)
@@ -434,7 +452,7 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
                 l.tc_small = readers == 1;
             }
             if (l.stem) l.tc = false;
-            l.w_ld = l.stem ? stem_klen() : l.tc_small ? tc_small_kpad(l.R, l.S) : RSC;
+            l.w_ld = l.dw ? l.R * l.S : l.stem ? stem_klen() : l.tc_small ? tc_small_kpad(l.R, l.S) : RSC;
             l.c_stride = l.tc_small ? 4 : l.C;
             if (l.tc_small) src.cp = 4;
             std::vector<uint8_t> hw((size_t)l.K * l.w_ld * esz, 0);
@@ -467,6 +485,13 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
                     shift = t + (double)be[k];
                 }
                 hb[kk] = (float)shift;
+                if (l.dw) {
+                    for (int r = 0; r < l.R; ++r)
+                        for (int s = 0; s < l.S; ++s)
+                            put(hw, (size_t)weight_word(l, kk, r, s, 0),
+                                (double)W[((size_t)k * l.R + r) * l.S + s] * scale, prec);
+                    continue;
+                }
                 for (int cc = 0; cc < l.C - (ji >= 0 ? 1 : 0); ++cc) {
                     const int c = (ji >= 0 && cc >= ji) ? cc + 1 : cc;
                     for (int r = 0; r < l.R; ++r)
@@ -635,21 +660,21 @@ struct WeightFault {
 // or pass-through row), whose flipped value enters the epilogue as
 // dv * input, dv = flipped - stored.
 WeightFault resolve_weight_fault(const ct_model *m, const LayerRT &l, int64_t e, int bit) {
-    const int Ct = l.C + (l.cs_in ? 1 : 0);
+    const int Ct = weight_in_channels(l);
     const int RS = l.R * l.S;
     const int k = (int)(e / ((int64_t)Ct * RS));
     const int c = (int)((e / RS) % Ct);
     const int r = (int)((e / l.S) % l.R), s = (int)(e % l.S);
     const bool centre = r == (l.R - 1) / 2 && s == (l.S - 1) / 2;
     WeightFault f;
-    if (k < l.K && c < l.C) {
+    if (k < l.K && (l.dw || c < l.C)) {
         f.explicit_word = true;
         f.word = weight_word(l, k, r, s, c);
         return f;
     }
     double stored = 0.0;                      // zero slice and off-centre taps
     if (k == l.K && l.role == CT_ROLE_CT && centre) stored = l.coef;
-    if (k == l.K && l.role == CT_ROLE_PASS && centre && c == l.C) stored = 1.0;
+    if (k == l.K && l.role == CT_ROLE_PASS && centre && (l.dw || c == l.C)) stored = 1.0;
     const float v = flipped(stored, bit, m->prec);
     f.fd.active = 1;
     f.fd.kout = k;
@@ -741,6 +766,9 @@ ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, 
                 a.y = po.data;
                 a.cs_out = po.has_cs ? po.cs : nullptr;
                 CUDA_TRY(launch(m, FAM_TC, flops, st, [&] { return launch_stem_pool(a, l.stplan, st); }));
+            } else if (l.dw) {
+                const double dw_flops = 2.0 * batch * l.P * l.Q * (double)l.K * l.R * l.S;
+                CUDA_TRY(launch(m, FAM_OTHER, dw_flops, st, [&] { return launch_conv_dw(a, half, st); }));
             } else if (l.tc_small) {
                 CUDA_TRY(launch(m, FAM_TC, flops, st, [&] { return launch_conv_tc_small(a, l.splan, st); }));
             } else {
@@ -1010,7 +1038,7 @@ ct_status ct_inject(ct_model *m, int32_t kind, int32_t layer, int64_t element, i
     if (bit < 0 || bit >= bits) return CT_ERANGE;
     if (kind == CT_BUF_WEIGHT) {
         const int Kt = l.K + ((l.role == CT_ROLE_CT || l.role == CT_ROLE_PASS) ? 1 : 0);
-        const int Ct = l.C + (l.cs_in ? 1 : 0);
+        const int Ct = weight_in_channels(l);
         if (element < 0 || element >= (int64_t)Kt * Ct * l.R * l.S) return CT_ERANGE;
     } else {
         const Slot &sl = m->slots[l.d.src];
@@ -1243,7 +1271,7 @@ ct_status ct_buffer_info(const ct_model *m, int32_t batch, int32_t i, int32_t *k
         if (l.d.op != CT_OP_CONV) continue;
         if (idx++ == i) {
             const int Kt = l.K + ((l.role == CT_ROLE_CT || l.role == CT_ROLE_PASS) ? 1 : 0);
-            const int Ct = l.C + (l.cs_in ? 1 : 0);
+            const int Ct = weight_in_channels(l);
             *kind = CT_BUF_WEIGHT; *layer = (int)li; *n_elements = (int64_t)Kt * Ct * l.R * l.S; *bits = b;
             return CT_OK;
         }

@@ -71,6 +71,9 @@ struct CampFault {
     int img, act_c, act_hw;   // activation: image, channel (K1 = checksum), pixel of the first pool's output
 };
 
+bool dw_supported(int C, int K, bool half);
+cudaError_t launch_conv_dw(const ConvArgs &a, bool half, cudaStream_t st);
+
 size_t campaign_small_smem(const SmallNet &g);
 cudaError_t launch_campaign_small(const SmallNet &g, const CampFault *faults, int n_faults, float *S, int32_t *top1,
                                   uint8_t *flag, cudaStream_t st);

@@ -94,3 +94,11 @@ def test_replace_flips_match_oracle():
                 assert abs(sg - so) <= TOL[prec] * max(abs(so), 1e-6), (kind, layer, e, bit, sg, so)
     assert ct().ct_device_error(m) == 0
     m.close()
+
+
+def test_replace_rejects_depthwise_networks():
+    """The pruning scores read dense filters; a network with depthwise
+    convolutions is refused before any weight is read."""
+    with pytest.raises(ct().CtError) as e:
+        rmodel("mobilenetv2_cifar", "fp32", max_batch=2)
+    assert e.value.status == 6
