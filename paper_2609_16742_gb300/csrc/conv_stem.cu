@@ -415,10 +415,17 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
             if (ok) {
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                 const uint32_t trow = tmem + (uint32_t)(ab * 128) + ((uint32_t)(quad * 32) << 16);
+                // all of the row's TMEM loads in flight, one wait
                 float v[32];
-                tmem_ld16(trow + k0, v);
-                tmem_ld16(trow + k0 + 16, v + 16);
-                const float ctv = (has_cs && g.ct && half_id == 0) ? tmem_ld1(trow + ST_K) : 0.f;
+                uint32_t r0[16], r1[16], rc = 0;
+                const bool want_ct = has_cs && g.ct && half_id == 0;      // warp-uniform
+                tmem_ld16_nw(trow + k0, r0);
+                tmem_ld16_nw(trow + k0 + 16, r1);
+                if (want_ct) tmem_ld1_nw(trow + ST_K, rc);
+                tmem_wait_ld();
+                tmem_done16(r0, v);
+                tmem_done16(r1, v + 16);
+                const float ctv = want_ct ? tmem_done(rc) : 0.f;
                 asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
                 __syncwarp();
                 if (lane == 0) mbar_arrive(smem_u32(&acc_empty[ab]));

@@ -1176,10 +1176,17 @@ conv_tc_halo_kernel(const __grid_constant__ HaloMaps maps, const ConvArgs a, con
             if (!ok) break;
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
             const uint32_t trow = tmem + (uint32_t)(ab * CH) + ((uint32_t)(quad * 32) << 16);
+            // all of the tile's TMEM loads in flight, one wait
             float vals[BN / 2];
+            uint32_t rr[BN / 32][16], rc = 0;
+            const bool want_ct = do_cs && hg.ct;                      // warp-uniform
 #pragma unroll
-            for (int c = 0; c < BN / 2; c += 16) tmem_ld16(trow + half * (BN / 2) + c, vals + c);
-            const float ctv = (do_cs && hg.ct) ? tmem_ld1(trow + BN) : 0.f;
+            for (int c = 0; c < BN / 2; c += 16) tmem_ld16_nw(trow + half * (BN / 2) + c, rr[c / 16]);
+            if (want_ct) tmem_ld1_nw(trow + BN, rc);
+            tmem_wait_ld();
+#pragma unroll
+            for (int c = 0; c < BN / 2; c += 16) tmem_done16(rr[c / 16], vals + c);
+            const float ctv = want_ct ? tmem_done(rc) : 0.f;
             asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&acc_empty[ab]));
