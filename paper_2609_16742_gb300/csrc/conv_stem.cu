@@ -13,9 +13,10 @@
 // in step 1), each tap with 4 channels (the image's C <= 4 channels, then
 // zeros).
 //
-// No im2col tile is built.  The producer warps convert input rows from FP32
-// NCHW to FP16 pixels of 4 channels (8 bytes) in a ring of shared-memory
-// rows.  With stride 2, output column q reads input pixels 2q + s - 3, so in
+// No im2col tile is built.  Image rows arrive by bulk copies (one per
+// channel row) in a staging ring, four rows per producer warp in flight;
+// the producer warps convert them from FP32 NCHW to FP16 pixels of 4
+// channels (8 bytes) in a ring of shared-memory rows.  With stride 2, output column q reads input pixels 2q + s - 3, so in
 // such a row the A operand of one step is a strided view: A row q starts
 // 16 bytes after row q - 1 and each 8-element K chunk (2 taps) 16 bytes after
 // the previous one.  That is a no-swizzle K-major UMMA descriptor with row
@@ -68,8 +69,14 @@ constexpr int ST_TMEM_COLS = 128 * ST_NACC;
 constexpr size_t ST_OFF_B = (size_t)ST_NSLOT * ST_SLOT_BYTES;
 constexpr size_t ST_OFF_ROW = ST_OFF_B + (size_t)ST_KSTEPS * ST_B_STEP;
 constexpr size_t ST_OFF_CS = ST_OFF_ROW + 2ull * 128 * ST_PIX_H * 2;
-constexpr size_t ST_OFF_BAR = ST_OFF_CS + 2ull * 128 * 2;
-constexpr size_t ST_SMEM = 1024 + ST_OFF_BAR + 8 * (2 * ST_NSLOT + 2 * ST_NACC + 1) + 16;
+// staging of FP32 image rows (bulk copies): 4 per producer warp, up to 4
+// channels of 256 pixels each
+constexpr int ST_STG_W = 4;                  // staging slots per producer warp
+constexpr int ST_NSTG = 4 * ST_STG_W;
+constexpr int ST_STG_BYTES = 4 * 256 * 4;
+constexpr size_t ST_OFF_STG = ST_OFF_CS + 2ull * 128 * 2;
+constexpr size_t ST_OFF_BAR = ST_OFF_STG + (size_t)ST_NSTG * ST_STG_BYTES;
+constexpr size_t ST_SMEM = 1024 + ST_OFF_BAR + 8 * (2 * ST_NSLOT + 2 * ST_NACC + 1 + ST_NSTG) + 16;
 
 struct StemGeom {
     int N, C, H, W, P, Q, P2, Q2;
@@ -183,46 +190,6 @@ struct RowIter {
     }
 };
 
-// one input row (image img, row y) as FP32 values: lane owns columns lane + 32 it
-__device__ __forceinline__ void load_image_row(float (&v)[8][4], const float *img, const StemGeom &g, int y,
-                                               int lane) {
-    const bool row_ok = y >= 0 && y < g.H;
-#pragma unroll
-    for (int it = 0; it < 8; ++it) {
-        const int col = lane + 32 * it;
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-            v[it][c] = 0.f;
-            if (row_ok && col < g.W && c < g.C) v[it][c] = __ldg(img + ((size_t)c * g.H + y) * g.W + col);
-        }
-    }
-}
-
-// waits for ring slot e % ST_NSLOT, writes the row's two FP16 copies (E:
-// pixel x at byte 8 (x + 3), O: at byte 8 (x + 4)) and marks it full
-__device__ __forceinline__ bool store_ring_row(const float (&v)[8][4], uint8_t *ring, uint64_t *full,
-                                               uint64_t *empty, int e, const StemGeom &g, int lane, uint32_t *err) {
-    const int slot = e % ST_NSLOT;
-    const uint32_t ph = (uint32_t)(e / ST_NSLOT) & 1u;
-    if (!warp_wait(smem_u32(&empty[slot]), ph ^ 1u, err, 1u)) return false;
-    uint8_t *E = ring + slot * ST_SLOT_BYTES;
-    uint8_t *O = E + ST_ROW_BYTES;
-#pragma unroll
-    for (int it = 0; it < 8; ++it) {
-        const int col = lane + 32 * it;
-        if (col < g.W) {
-            __half2 lo = __floats2half2_rn(v[it][0], v[it][1]);
-            __half2 hi = __floats2half2_rn(v[it][2], v[it][3]);
-            const uint2 pk = make_uint2(*reinterpret_cast<uint32_t *>(&lo), *reinterpret_cast<uint32_t *>(&hi));
-            *reinterpret_cast<uint2 *>(E + (col + 3) * 8) = pk;
-            *reinterpret_cast<uint2 *>(O + (col + 4) * 8) = pk;
-        }
-    }
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-    mbar_arrive(smem_u32(&full[slot]));
-    return true;
-}
-
 __global__ void __launch_bounds__(ST_THREADS, 1)
 stem_pool_kernel(const ConvArgs a, const StemGeom g) {
     pdl_wait();
@@ -238,7 +205,9 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
     uint64_t *acc_full = empty + ST_NSLOT;
     uint64_t *acc_empty = acc_full + ST_NACC;
     uint64_t *mma_done = acc_empty + ST_NACC;
-    uint32_t *tmem_holder = (uint32_t *)(mma_done + 1);
+    uint64_t *stg_full = mma_done + 1;                       // [ST_NSTG]
+    float *stg = (float *)(smem + ST_OFF_STG);
+    uint32_t *tmem_holder = (uint32_t *)(stg_full + ST_NSTG);
     volatile uint32_t *abort_flag = tmem_holder + 1;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -285,6 +254,7 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
             mbar_init(smem_u32(&acc_empty[b]), ST_EPI / 32);
         }
         mbar_init(smem_u32(mma_done), 1);
+        for (int s = 0; s < ST_NSTG; ++s) mbar_init(smem_u32(&stg_full[s]), 1);
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -300,28 +270,77 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
 
     if (warp < 4) {
         // ---------------- ring producers ----------------
-        // Each warp produces every fourth ring entry.  The global loads of
-        // its next entry are issued before it waits for the current entry's
-        // slot and stores it, so two input rows per warp (eight per CTA) are
-        // in flight against the DRAM latency.
+        // Each warp produces every fourth ring entry.  Its next ST_STG_W
+        // entries' image rows are in flight as bulk copies (one per channel
+        // row of W FP32 values) into its own staging slots; the warp then
+        // converts a landed row to the two FP16 copies of its ring slot.
+        // Rows outside the image are not copied (their slot reads as zero).
         RowIter ri;
         ri.init(u0, u1, g);
-        float va[8][4], vb[8][4];
-        int ea = 0, ya = 0, eb = 0, yb = 0;
-        bool ok = true;
-        bool ha = ri.next(warp, ea, ya, g);
-        if (ha) load_image_row(va, image_base(a, g, ri.n_of_last), g, ya, lane);
-        while (ha) {
-            if (__any_sync(0xffffffffu, *abort_flag)) break;
-            const bool hb = ri.next(warp, eb, yb, g);
-            if (hb) load_image_row(vb, image_base(a, g, ri.n_of_last), g, yb, lane);
-            if (!(ok = store_ring_row(va, ring, full, empty, ea, g, lane, a.err))) break;
-            if (!hb) break;
-            ha = ri.next(warp, ea, ya, g);
-            if (ha) load_image_row(va, image_base(a, g, ri.n_of_last), g, ya, lane);
-            if (!(ok = store_ring_row(vb, ring, full, empty, eb, g, lane, a.err))) break;
+        int ent_e[ST_STG_W], ent_y[ST_STG_W];
+        int k_issue = 0, k_done = 0;
+        bool ok = true, more = true;
+        const uint32_t row_bytes = (uint32_t)g.W * 4u;
+        while (ok) {
+            // keep ST_STG_W entries in flight
+            while (more && k_issue - k_done < ST_STG_W) {
+                int e, y;
+                more = ri.next(warp, e, y, g);
+                if (!more) break;
+                const int i = k_issue % ST_STG_W, sl = warp * ST_STG_W + i;
+                ent_e[i] = e; ent_y[i] = y;
+                if (lane == 0) {
+                    const uint32_t bar = smem_u32(&stg_full[sl]);
+                    if (y >= 0 && y < g.H) {
+                        const float *img = image_base(a, g, ri.n_of_last);
+                        mbar_arrive_expect_tx(bar, row_bytes * (uint32_t)g.C);
+                        for (int c = 0; c < g.C; ++c)
+                            bulk_load(smem_u32(stg + (size_t)sl * (ST_STG_BYTES / 4) + c * g.W),
+                                      img + ((size_t)c * g.H + y) * g.W, row_bytes, bar);
+                    } else {
+                        mbar_arrive(bar);
+                    }
+                }
+                ++k_issue;
+            }
+            if (k_done == k_issue) break;
+            if (__any_sync(0xffffffffu, *abort_flag)) { ok = false; break; }
+            const int i = k_done % ST_STG_W, sl = warp * ST_STG_W + i;
+            if (!warp_wait(smem_u32(&stg_full[sl]), (uint32_t)(k_done / ST_STG_W) & 1u, a.err, 1u)) { ok = false; break; }
+            const int e = ent_e[i], y = ent_y[i];
+            const int slot = e % ST_NSLOT;
+            if (!warp_wait(smem_u32(&empty[slot]), ((uint32_t)(e / ST_NSLOT) & 1u) ^ 1u, a.err, 1u)) { ok = false; break; }
+            const bool row_ok = y >= 0 && y < g.H;
+            const float *sr = stg + (size_t)sl * (ST_STG_BYTES / 4);
+            uint8_t *E = ring + slot * ST_SLOT_BYTES;
+            uint8_t *O = E + ST_ROW_BYTES;
+#pragma unroll
+            for (int it = 0; it < 8; ++it) {
+                const int col = lane + 32 * it;
+                if (col < g.W) {
+                    float v[4];
+#pragma unroll
+                    for (int c = 0; c < 4; ++c) v[c] = (row_ok && c < g.C) ? sr[c * g.W + col] : 0.f;
+                    __half2 lo = __floats2half2_rn(v[0], v[1]);
+                    __half2 hi = __floats2half2_rn(v[2], v[3]);
+                    const uint2 pk = make_uint2(*reinterpret_cast<uint32_t *>(&lo), *reinterpret_cast<uint32_t *>(&hi));
+                    *reinterpret_cast<uint2 *>(E + (col + 3) * 8) = pk;
+                    *reinterpret_cast<uint2 *>(O + (col + 4) * 8) = pk;
+                }
+            }
+            // the staging slot is refilled by a bulk copy (async proxy) after these reads
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            __syncwarp();
+            mbar_arrive(smem_u32(&full[slot]));
+            ++k_done;
         }
-        if (!ok && lane == 0) *abort_flag = 1;
+        if (!ok) {
+            if (lane == 0) *abort_flag = 1;
+            // copies still in flight land before the CTA leaves
+            for (int k = k_done; k < k_issue; ++k)
+                warp_wait(smem_u32(&stg_full[warp * ST_STG_W + k % ST_STG_W]), (uint32_t)(k / ST_STG_W) & 1u,
+                          a.err, 1u);
+        }
     } else if (warp == 4) {
         // ---------------- MMA issuer (whole warp, one lane issues) ----------------
         const uint32_t id64 = idesc_f16(128, ST_K);
@@ -549,7 +568,8 @@ int stem_klen() { return ST_KLEN; }
 bool stem_pool_supported(int C, int K, int R, int S, int stride, int pad, int H, int W) {
     if (C < 1 || C > 4 || K != ST_K || R != ST_R || S != ST_R || stride != 2 || pad != 3) return false;
     const int P = (H + 2 * pad - R) / stride + 1, Q = (W + 2 * pad - S) / stride + 1;
-    return P >= 2 && Q >= 2 && Q <= 128 && W + 4 <= ST_RP && W <= 256;
+    // W % 4: image rows are bulk-copied, which needs 16-byte multiples
+    return P >= 2 && Q >= 2 && Q <= 128 && W + 4 <= ST_RP && W <= 256 && W % 4 == 0;
 }
 
 StemPlan *stem_plan_create(const ConvArgs &a, std::string *why) {

@@ -89,6 +89,14 @@ __device__ __forceinline__ void tma_load_im2col(uint32_t dst, const CUtensorMap 
         : "memory");
 }
 
+// plain bulk copy global -> shared of `bytes` (16-byte aligned addresses, a
+// multiple of 16 bytes), completing on the mbarrier's transaction count
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void *src, uint32_t bytes, uint32_t bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+                 "l"((uint64_t)src), "r"(bytes), "r"(bar)
+                 : "memory");
+}
+
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, uint32_t bar, int x, int y) {
     asm volatile(
         "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
