@@ -51,11 +51,16 @@ constexpr int BK = 64;             // channels per K block (128 bytes of fp16)
 constexpr int A_BYTES = BM * BK * 2;
 constexpr int NTHREADS = 320;      // 1 TMA warp, 1 MMA warp, 8 epilogue warps
 constexpr int N_EPI_WARPS = 8;
-// conv_tc_kernel: TC_NPROD TMA producer warps, one MMA warp, 8 epilogue warps
-constexpr int TC_NPROD = 4;
-constexpr int TC_MMA_WARP = TC_NPROD;
-constexpr int TC_EPI_WARP0 = TC_NPROD + 1;
-constexpr int TC_THREADS = 32 * (TC_NPROD + 1 + N_EPI_WARPS);
+// conv_tc_kernel: a producer group (TMA producer warps, each owning whole ring
+// slots, plus for N = 256 two carry-through warps), one MMA warp, 8 epilogue
+// warps.  The group is as large as the variant needs: a warp fewer raises the
+// register budget of a 1-CTA-per-SM kernel (384 threads: 168 registers, 416:
+// 128).
+constexpr int tc_nprod(int BN, int STAGES) {
+    return BN > 128 ? 2 : STAGES % 4 == 0 ? 4 : STAGES % 3 == 0 ? 3 : STAGES % 2 == 0 ? 2 : 1;
+}
+constexpr int tc_npg(int BN, int STAGES) { return BN > 128 ? 4 : tc_nprod(BN, STAGES); }
+constexpr int tc_threads(int BN, int STAGES) { return 32 * (tc_npg(BN, STAGES) + 1 + N_EPI_WARPS); }
 constexpr int TC_CS = 4;           // CTAs per cluster sharing each B tile (N = 128, 256)
 
 enum CtMode { CT_NONE_ = 0, CT_MERGED = 1, CT_SEPARATE = 2 };
@@ -232,7 +237,7 @@ __device__ __forceinline__ void store_checksum_pre(float ctv, const CsIn &c, con
 // BN <= 128 the epilogue copies it to registers and releases it before its
 // global stores, so the next tile's MMAs overlap the stores.
 template <int BN, int STAGES, int SUB, int NCH, int CS>
-__global__ void __launch_bounds__(TC_THREADS, 1)
+__global__ void __launch_bounds__(tc_threads(BN, STAGES), 1)
 conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
                const ConvArgs a, const TcGeom g) {
     constexpr int B_ROWS = BN + 16;                       // 16 constant carry-through rows
@@ -248,9 +253,13 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
     constexpr bool DBUF = !EARLY;
     static_assert(!DBUF || CS == 1, "the carry-through warps release stages of their own CTA only");
     // producer warps (each owns whole ring slots) and carry-through warps
-    constexpr int NPROD = DBUF ? 2 : STAGES % 4 == 0 ? 4 : STAGES % 3 == 0 ? 3 : STAGES % 2 == 0 ? 2 : 1;
-    constexpr int NCT = DBUF ? TC_NPROD - NPROD : 0;
-    static_assert(NPROD <= TC_NPROD && STAGES % NPROD == 0, "producer warps must own whole ring slots");
+    constexpr int NPROD = tc_nprod(BN, STAGES);
+    constexpr int NPG = tc_npg(BN, STAGES);               // producer group: producers + carry-through warps
+    constexpr int NCT = DBUF ? NPG - NPROD : 0;
+    constexpr int TC_MMA_WARP = NPG;
+    constexpr int TC_EPI_WARP0 = NPG + 1;
+    static_assert(STAGES % NPROD == 0, "producer warps must own whole ring slots");
+    static_assert(DBUF ? NCT > 0 : NCT == 0, "carry-through warps only beside double-buffered accumulators");
     static_assert(!DBUF || (NCT > 0 && BM % (16 * (NCT > 0 ? NCT : 1)) == 0), "carry-through warps split the tile rows");
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -427,7 +436,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
             if (elect_one()) umma_commit(smem_u32(&acc_full[ab]));   // fires when the tile's MMAs have completed
             __syncwarp();
         }
-    } else if (warp < TC_NPROD) {
+    } else if (warp < NPG) {
         if (NCT > 0) {
             // ---------------- carry-through sums (N = 256) ----------------
             // Consumes every stage in order (arrives on its empty barrier);
@@ -1367,7 +1376,7 @@ TcPlan *tc_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, cons
                            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(TC_CS * 64);
-        cfg.blockDim = dim3(TC_THREADS);
+        cfg.blockDim = dim3(tc_threads(128, 3));
         cfg.dynamicSmemBytes = pl->smem;
         cudaLaunchAttribute at[1];
         at[0].id = cudaLaunchAttributeClusterDimension;
@@ -1408,14 +1417,14 @@ cudaError_t launch_conv_tc(const ConvArgs &a, const void *plan, cudaStream_t st,
         const int items = g.m_groups * g.n_tiles;
         const int ncl = items < pl->max_clusters ? items : pl->max_clusters;
         dim3 grid(ncl * pl->cs);
-        pdl_launch_cluster(conv_tc_kernel<128, 3, 2, 2, TC_CS>, grid, TC_THREADS, pl->smem, st, TC_CS, pl->amap,
+        pdl_launch_cluster(conv_tc_kernel<128, 3, 2, 2, TC_CS>, grid, tc_threads(128, 3), pl->smem, st, TC_CS, pl->amap,
                            pl->bmap_mc, a, g);
     } else {
         const int items = tiles * g.splits;
         dim3 grid(items < pl->sms ? items : pl->sms);
-        if (pl->BN == 64) pdl_launch(conv_tc_kernel<64, 4, 2, 4, 1>, grid, TC_THREADS, pl->smem, st, pl->amap, pl->bmap, a, g);
-        else if (pl->BN == 128) pdl_launch(conv_tc_kernel<128, 3, 2, 2, 1>, grid, TC_THREADS, pl->smem, st, pl->amap, pl->bmap, a, g);
-        else pdl_launch(conv_tc_kernel<256, 4, 1, 1, 1>, grid, TC_THREADS, pl->smem, st, pl->amap, pl->bmap, a, g);
+        if (pl->BN == 64) pdl_launch(conv_tc_kernel<64, 4, 2, 4, 1>, grid, tc_threads(64, 4), pl->smem, st, pl->amap, pl->bmap, a, g);
+        else if (pl->BN == 128) pdl_launch(conv_tc_kernel<128, 3, 2, 2, 1>, grid, tc_threads(128, 3), pl->smem, st, pl->amap, pl->bmap, a, g);
+        else pdl_launch(conv_tc_kernel<256, 4, 1, 1, 1>, grid, tc_threads(256, 4), pl->smem, st, pl->amap, pl->bmap, a, g);
     }
     cudaError_t e = cudaGetLastError();
     if (n_kernels) *n_kernels = 1;
