@@ -32,9 +32,11 @@ __global__ void __launch_bounds__(256) fc_kernel(FcArgs a) {
     pdl_wait();
     pdl_trigger();
     extern __shared__ __align__(16) float smem[];
-    float *Xs = smem;                              // [FC_KC][FC_IMG + 1]
-    float *Ws = Xs + FC_KC * (FC_IMG + 1);         // [FC_KC][FC_J]; offset 4160 floats: 16-byte aligned
-    float *red = Ws + FC_KC * FC_J;                // [FC_WARPS][FC_J + 1][FC_IMG]
+    // two stages of [FC_KC][FC_IMG + 1] inputs and [FC_KC][FC_J] weights (each
+    // offset a multiple of 4 floats: 16-byte aligned float4 reads), then the
+    // cross-warp reduction [FC_WARPS][FC_J + 1][FC_IMG]
+    constexpr int XS = FC_KC * (FC_IMG + 1), WS = FC_KC * FC_J;
+    float *red = smem + 2 * (XS + WS);
     const TX *x = static_cast<const TX *>(a.x);
     const TW *w = static_cast<const TW *>(a.w);
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -50,26 +52,55 @@ __global__ void __launch_bounds__(256) fc_kernel(FcArgs a) {
     const int nkc = (a.n_in + FC_KC - 1) / FC_KC;
     const int kc_per = (nkc + gridDim.z - 1) / gridDim.z;
     const int k_lo = blockIdx.z * kc_per * FC_KC, k_hi = min(a.n_in, k_lo + kc_per * FC_KC);
-    for (int k0 = k_lo; k0 < k_hi; k0 += FC_KC) {
-        // stage x[b0 .. b0+63][k0 .. k0+63] transposed, and W[j0..j0+15][k0..k0+63]
-        for (int e = tid; e < FC_KC * FC_IMG; e += 256) {
-            int kk = e % FC_KC, bb = e / FC_KC;
-            int b = b0 + bb, k = k0 + kk;
-            Xs[kk * (FC_IMG + 1) + bb] = (b < a.B && k < k_hi) ? to_f(x[(size_t)b * a.n_in + k]) : 0.f;
+    // x[b0 .. b0+63][k0 .. k0+63] (transposed) and W[j0..j0+15][k0..k0+63]:
+    // the next chunk's values are loaded into registers while this chunk is
+    // multiplied, then stored to the other stage
+    constexpr int XR = FC_KC * FC_IMG / 256, WR = FC_KC * FC_J / 256;
+    float xr[XR], wr[WR];
+    auto load_chunk = [&](int k0) {
+#pragma unroll
+        for (int i = 0; i < XR; ++i) {
+            const int e = tid + 256 * i, kk = e % FC_KC, bb = e / FC_KC;
+            const int b = b0 + bb, k = k0 + kk;
+            xr[i] = (b < a.B && k < k_hi) ? to_f(x[(size_t)b * a.n_in + k]) : 0.f;
         }
-        for (int e = tid; e < FC_KC * FC_J; e += 256) {
-            int kk = e % FC_KC, jj = e / FC_KC;
-            int j = j0 + jj, k = k0 + kk;
-            Ws[kk * FC_J + jj] = (j < a.n_out && k < k_hi) ? to_f(w[(size_t)j * a.n_in + k]) : 0.f;
+#pragma unroll
+        for (int i = 0; i < WR; ++i) {
+            const int e = tid + 256 * i, kk = e % FC_KC, jj = e / FC_KC;
+            const int j = j0 + jj, k = k0 + kk;
+            wr[i] = (j < a.n_out && k < k_hi) ? to_f(w[(size_t)j * a.n_in + k]) : 0.f;
         }
-        __syncthreads();
+    };
+    auto store_chunk = [&](int stage) {
+        float *Xd = smem + stage * (XS + WS), *Wd = Xd + XS;
+#pragma unroll
+        for (int i = 0; i < XR; ++i) {
+            const int e = tid + 256 * i;
+            Xd[(e % FC_KC) * (FC_IMG + 1) + e / FC_KC] = xr[i];
+        }
+#pragma unroll
+        for (int i = 0; i < WR; ++i) {
+            const int e = tid + 256 * i;
+            Wd[(e % FC_KC) * FC_J + e / FC_KC] = wr[i];
+        }
+    };
+    if (k_lo < k_hi) {
+        load_chunk(k_lo);
+        store_chunk(0);
+    }
+    __syncthreads();
+    int stage = 0;
+    for (int k0 = k_lo; k0 < k_hi; k0 += FC_KC, stage ^= 1) {
+        const bool more = k0 + FC_KC < k_hi;
+        if (more) load_chunk(k0 + FC_KC);
+        const float *Xs = smem + stage * (XS + WS), *Ws = Xs + XS;
 #pragma unroll 2
         for (int kk = warp; kk < FC_KC; kk += FC_WARPS) {
             float x0 = Xs[kk * (FC_IMG + 1) + lane], x1 = Xs[kk * (FC_IMG + 1) + lane + 32];
-            const float4 *wr = reinterpret_cast<const float4 *>(&Ws[kk * FC_J]);
+            const float4 *wrow = reinterpret_cast<const float4 *>(&Ws[kk * FC_J]);
 #pragma unroll
             for (int q = 0; q < FC_J / 4; ++q) {
-                float4 wv = wr[q];
+                float4 wv = wrow[q];
                 acc[4 * q + 0][0] = fmaf(wv.x, x0, acc[4 * q + 0][0]);
                 acc[4 * q + 0][1] = fmaf(wv.x, x1, acc[4 * q + 0][1]);
                 acc[4 * q + 1][0] = fmaf(wv.y, x0, acc[4 * q + 1][0]);
@@ -81,6 +112,7 @@ __global__ void __launch_bounds__(256) fc_kernel(FcArgs a) {
             }
             if (ct_block) { act[0] += x0; act[1] += x1; }
         }
+        if (more) store_chunk(stage ^ 1);
         __syncthreads();
     }
     // cross-warp reduction
@@ -374,7 +406,7 @@ int grid_for(int64_t n, int threads) {
 template <typename TX, typename TW, typename TY>
 cudaError_t fc_go(const FcArgs &a, cudaStream_t st, int *n_kernels) {
     const size_t smem =
-        sizeof(float) * (FC_KC * (FC_IMG + 1) + FC_KC * FC_J + FC_WARPS * (FC_J + 1) * FC_IMG);
+        sizeof(float) * (2 * (FC_KC * (FC_IMG + 1) + FC_KC * FC_J) + FC_WARPS * (FC_J + 1) * FC_IMG);
     static bool attr = false;
     if (!attr) {
         cudaError_t e = cudaFuncSetAttribute(fc_kernel<TX, TW, TY>,
