@@ -14,7 +14,7 @@
 // zeros).
 //
 // No im2col tile is built.  Image rows arrive by bulk copies (one per
-// channel row) in a staging ring, four rows per producer warp in flight;
+// channel row) in a staging ring, two rows per producer warp in flight;
 // the producer warps convert them from FP32 NCHW to FP16 pixels of 4
 // channels (8 bytes) in a ring of shared-memory rows.  With stride 2, output column q reads input pixels 2q + s - 3, so in
 // such a row the A operand of one step is a strided view: A row q starts
@@ -56,7 +56,7 @@ constexpr int ST_KLEN = 16 * ST_KSTEPS;      // 224: weight row length
 constexpr int ST_RP = 264;                   // ring row pitch in pixels (8 bytes each)
 constexpr int ST_ROW_BYTES = ST_RP * 8;      // one copy of one input row
 constexpr int ST_SLOT_BYTES = 2 * ST_ROW_BYTES;
-constexpr int ST_NSLOT = 16;                 // ring rows
+constexpr int ST_NSLOT = 24;                 // ring rows: the producers run up to ~8 convolution rows ahead
 constexpr int ST_B_STEP = ST_NB * 32;        // B bytes per K16 step (two core-matrix columns)
 constexpr int ST_B_LBO = ST_NB * 16;         // between the two K chunks of a step
 constexpr int ST_PIX_H = 72;                 // halves per pixel in the epilogue row buffer (144 B)
@@ -69,9 +69,12 @@ constexpr int ST_TMEM_COLS = 128 * ST_NACC;
 constexpr size_t ST_OFF_B = (size_t)ST_NSLOT * ST_SLOT_BYTES;
 constexpr size_t ST_OFF_ROW = ST_OFF_B + (size_t)ST_KSTEPS * ST_B_STEP;
 constexpr size_t ST_OFF_CS = ST_OFF_ROW + 2ull * 128 * ST_PIX_H * 2;
-// staging of FP32 image rows (bulk copies): 4 per producer warp, up to 4
-// channels of 256 pixels each
-constexpr int ST_STG_W = 4;                  // staging slots per producer warp
+// staging of FP32 image rows (bulk copies): ST_STG_W per producer warp, up
+// to 4 channels of 256 pixels each.  Shared memory goes to ring depth first:
+// the producer, MMA and epilogue stages only overlap when the ring holds
+// several convolution rows beyond the 7-row window (16 slots: 275 us at 256
+// images, 24: 238 us; deeper staging gained nothing)
+constexpr int ST_STG_W = 2;                  // staging slots per producer warp
 constexpr int ST_NSTG = 4 * ST_STG_W;
 constexpr int ST_STG_BYTES = 4 * 256 * 4;
 constexpr size_t ST_OFF_STG = ST_OFF_CS + 2ull * 128 * 2;
