@@ -1,34 +1,38 @@
-// Tensor-core (tcgen05) implicit-GEMM convolution with the carry-through
+// Tensor-core (tcgen05) implicit-GEMM convolutions with the carry-through
 // filter, FP16 storage, FP32 accumulation in TMEM.
 //
 // GEMM view: D[m, n] = sum_k A[m, k] B[n, k] with m = output pixel (n, p, q),
 // n = output channel, k = (tap, channel), channels innermost.
 //   A (128 pixels x 64 channels of one tap) is fetched by TMA in im2col mode
-//     from the NHWC input: the TMA unit walks consecutive output pixels,
-//     applies stride and zero padding, and writes the 128-byte swizzled
-//     K-major tile the MMA reads.
+//     from the NHWC input (conv_tc_kernel), or as one 18 x 10 pixel patch
+//     whose nine shifted views are the nine taps (conv_tc_halo_kernel); the
+//     tiles are 128-byte swizzled and K-major.
 //   B (BN channels x 64) is fetched by tiled TMA from the KRSC weights.
 //   The carry-through filter of Sec. II-A is one more GEMM row: coef at the
-//     centre tap of every input channel, 0 elsewhere.  Its non-zero part is a
-//     constant 16-row tile (row 0 = coef, rows 1-15 = 0) kept in shared
-//     memory, so the tensor core itself computes the checksum column on the
-//     centre-tap K blocks, which the K loop visits first: as 16 extra columns
-//     of the same MMA when BN + 16 <= 256, else as a separate N = 16 MMA.
-//   The incoming checksum plane (weight coef at the centre) and the
-//   epilogue (bias, residual, ReLU) are applied by the epilogue warps.
+//     centre tap of every input channel, 0 elsewhere.  For BN <= 128 its
+//     non-zero part is a constant 16-row tile (row 0 = coef) kept after the
+//     weight rows in shared memory, and the centre-tap K blocks, which the
+//     K loop visits first, are issued with N = BN + 16: the tensor core
+//     computes the checksum column.  For BN = 256 two spare warps compute it
+//     from the same A tiles with warp-level MMAs against a ones vector.
+//   The incoming checksum plane (weight coef at the centre), the residual
+//   checksum and the epilogue (bias, residual, ReLU) are applied by the
+//   epilogue warps.
 //
 // The kernels are persistent: one CTA per SM walks a static list of output
-// tiles.  The TMA producer runs ahead across tile boundaries through a ring
+// tiles.  The TMA producers run ahead across tile boundaries through a ring
 // of shared-memory stages.  Consecutive K blocks accumulate into up to four
 // independent TMEM accumulators (chains), because back-to-back MMAs into one
-// accumulator wait on each other; the epilogue sums the chains, and for
-// N <= 128 releases TMEM before its global stores so that the next tile's
-// MMAs overlap them.
+// accumulator wait on each other; the epilogue sums the chains.  For
+// N <= 128 it releases TMEM before its global stores so that the next
+// tile's MMAs overlap them; for N = 256 two accumulators alternate.
 //
-// Warp roles (320 threads): warp 0 issues TMA, warp 1 allocates TMEM and
-// issues tcgen05.mma (one elected lane), warps 2-9 read the accumulator:
-// each TMEM lane quadrant (32 output pixels) is read by two warps, each
-// taking half of the tile's channels.
+// Warp roles.  conv_tc_kernel: a producer group (producer warps, each owning
+// whole ring slots, plus for N = 256 the two carry-through warps), one MMA
+// warp (one elected lane issues tcgen05.mma), eight epilogue warps.
+// conv_tc_halo_kernel (320 threads): warp 0 issues TMA, warp 1 the MMAs,
+// warps 2-9 the epilogue.  Each TMEM lane quadrant (32 output pixels) is
+// read by two epilogue warps, each taking half of the tile's channels.
 // Every mbarrier wait is bounded; on expiry the kernel records an error code
 // in a device word, stops issuing work and exits after releasing TMEM.
 #include <cuda.h>
@@ -246,10 +250,10 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
     constexpr int CH = BN + 16;                           // TMEM columns per chain
     constexpr bool EARLY = BN <= 128;                     // release TMEM before the stores
     // N = 256: two 256-column accumulators fill TMEM, so the carry-through
-    // column is summed on CUDA cores from the centre-tap A tiles in shared
-    // memory by the warps of the producer group that do not issue copies
-    // (they consume every stage, like the MMA warp), and the epilogue of one
-    // tile overlaps the MMAs of the next
+    // column is summed (warp-level MMAs against a ones vector) from the
+    // centre-tap A tiles in shared memory by the warps of the producer group
+    // that do not issue copies (they consume every stage, like the MMA warp),
+    // and the epilogue of one tile overlaps the MMAs of the next
     constexpr bool DBUF = !EARLY;
     static_assert(!DBUF || CS == 1, "the carry-through warps release stages of their own CTA only");
     // producer warps (each owns whole ring slots) and carry-through warps
