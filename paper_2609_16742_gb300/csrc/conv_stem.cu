@@ -133,6 +133,14 @@ __device__ __forceinline__ bool epi_bar_or(bool pred) {
     return r != 0;
 }
 
+// two FP32 values to an FP16 pair (round to nearest) with ReLU in one
+// conversion: negative values become 0, NaN stays NaN
+__device__ __forceinline__ uint32_t cvt_relu_h2(float lo, float hi) {
+    uint32_t r;
+    asm("cvt.rn.relu.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+    return r;
+}
+
 __device__ __forceinline__ uint32_t hmax2u(uint32_t a, uint32_t b) {
     __half2 r = __hmax2_nan(*reinterpret_cast<__half2 *>(&a), *reinterpret_cast<__half2 *>(&b));
     return *reinterpret_cast<uint32_t *>(&r);
@@ -421,9 +429,18 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
         const int jj = et >> 2, cq = et & 3;
         const bool pool_data = jj < g.Q2;
         const bool pool_cs = has_cs && et < g.Q2;
-        uint32_t accv[8], carry[8];
-        __half acc_cs = __ushort_as_half((unsigned short)0xFC00), carry_cs = acc_cs;
+        const bool want_ct = has_cs && g.ct && half_id == 0;      // warp-uniform
+        const bool keep_cs = has_cs && half_id == 0;
+        // vertical max-pool state of this thread's column q, carried across
+        // convolution rows: after an odd row p it holds row p (shared with
+        // the next pooled row), after an even row the maximum of rows p - 1
+        // and p
+        uint32_t vs[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) vs[i] = 0xFC00FC00u;
+        __half vs_cs = __ushort_as_half((unsigned short)0xFC00);
         bool acc_valid = false, has_carry = false;
+        int n_st = 0;                                   // pooled rows written: row-buffer parity
         StemJobs jb;
         bool have = jb.first(u0, u1, g);
         int j = 0;
@@ -432,15 +449,19 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
             const uint32_t use = (uint32_t)(j / ST_NACC) & 1u;
             bool ok = mbar_wait(smem_u32(&acc_full[ab]), use, a.err, 4u);
             ok = __all_sync(0xffffffffu, ok) && !*abort_flag;
-            __half *rb = rowbuf + (size_t)(j & 1) * 128 * ST_PIX_H;
-            __half *cb = csbuf + (j & 1) * 128;
+            const int p = jb.p;
+            const bool close_even = (p & 1) == 0 && p == g.P - 1;
+            if (jb.seg_start) { acc_valid = false; has_carry = false; }
+            // this row completes pooled row i2 (uniform over the epilogue)
+            const bool store = (p & 1) ? acc_valid : close_even;
+            __half *rb = rowbuf + (size_t)(n_st & 1) * 128 * ST_PIX_H;
+            __half *cb = csbuf + (n_st & 1) * 128;
             if (ok) {
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                 const uint32_t trow = tmem + (uint32_t)(ab * 128) + ((uint32_t)(quad * 32) << 16);
                 // all of the row's TMEM loads in flight, one wait
                 float v[32];
                 uint32_t r0[16], r1[16], rc = 0;
-                const bool want_ct = has_cs && g.ct && half_id == 0;      // warp-uniform
                 tmem_ld16_nw(trow + k0, r0);
                 tmem_ld16_nw(trow + k0 + 16, r1);
                 if (want_ct) tmem_ld1_nw(trow + ST_K, rc);
@@ -451,98 +472,98 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
                 asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
                 __syncwarp();
                 if (lane == 0) mbar_arrive(smem_u32(&acc_empty[ab]));
-                if (q < g.Q) {
-                    float fsrc = 0.f;
-                    if (fd.active)
-                        fsrc = image_half(image_base(a, g, jb.n), g, fd.cin, 2 * jb.p + fd.r - 3, 2 * q + fd.s - 3);
-                    uint32_t pk[16];
+                // bias, ReLU, FP16: one conversion per channel pair on the
+                // common path
+                uint32_t u[16];
+                float o_cs = (a.role == CT_ROLE_CT) ? ctv : 0.f;
+                if (!fd.active) {
+                    if (a.relu) {
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) u[i] = cvt_relu_h2(v[2 * i] + bias[2 * i], v[2 * i + 1] + bias[2 * i + 1]);
+                    } else {
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) {
+                            __half2 hh = __floats2half2_rn(v[2 * i] + bias[2 * i], v[2 * i + 1] + bias[2 * i + 1]);
+                            u[i] = *reinterpret_cast<uint32_t *>(&hh);
+                        }
+                    }
+                } else {
+                    const float fsrc = q < g.Q
+                        ? image_half(image_base(a, g, jb.n), g, fd.cin, 2 * p + fd.r - 3, 2 * q + fd.s - 3) : 0.f;
 #pragma unroll
                     for (int i = 0; i < 32; i += 2) {
                         float o[2];
 #pragma unroll
                         for (int t = 0; t < 2; ++t) {
                             float s = v[i + t] + bias[i + t];
-                            if (fd.active && fd.kout == k0 + i + t) s += fd.dv * fsrc;
+                            if (fd.kout == k0 + i + t) s += fd.dv * fsrc;
                             if (a.relu) s = relu_keep_nan(s);
                             o[t] = s;
                         }
                         __half2 hh = __floats2half2_rn(o[0], o[1]);
-                        pk[i / 2] = *reinterpret_cast<uint32_t *>(&hh);
+                        u[i / 2] = *reinterpret_cast<uint32_t *>(&hh);
                     }
+                    if (fd.kout == ST_K) o_cs += fd.dv * fsrc;
+                }
+                if (a.relu) o_cs = relu_keep_nan(o_cs);
+                const __half u_cs = __float2half_rn(o_cs);
+                // vertical pooling in registers
+                uint32_t out[16];
+                __half out_cs = u_cs;
+                if (p & 1) {
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) { out[i] = hmax2u(vs[i], u[i]); vs[i] = u[i]; }
+                    out_cs = __hmax_nan(vs_cs, u_cs);
+                    vs_cs = u_cs;
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) { vs[i] = has_carry ? hmax2u(vs[i], u[i]) : u[i]; out[i] = vs[i]; }
+                    vs_cs = has_carry ? __hmax_nan(vs_cs, u_cs) : u_cs;
+                    out_cs = vs_cs;
+                }
+                if (store && q < g.Q) {
                     uint4 *dst = reinterpret_cast<uint4 *>(rb + q * ST_PIX_H + k0);
 #pragma unroll
-                    for (int i = 0; i < 4; ++i) dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
-                    if (has_cs && half_id == 0) {
-                        float o = (a.role == CT_ROLE_CT) ? ctv : 0.f;
-                        if (fd.active && fd.kout == ST_K) o += fd.dv * fsrc;
-                        if (a.relu) o = relu_keep_nan(o);
-                        cb[q] = __float2half_rn(o);
-                    }
+                    for (int i = 0; i < 4; ++i) dst[i] = make_uint4(out[4 * i], out[4 * i + 1], out[4 * i + 2], out[4 * i + 3]);
+                    if (keep_cs) cb[q] = out_cs;
                 }
             }
             if (epi_bar_or(!ok)) {
                 if (et == 0) *abort_flag = 1;
                 break;
             }
-            // ---- column max over 2jj - 1 .. 2jj + 1, then the row logic ----
-            const int p = jb.p;
-            const bool close_even = (p & 1) == 0 && p == g.P - 1;
-            if (jb.seg_start) { acc_valid = false; has_carry = false; }
-            if (pool_data) {
-                uint32_t h[8];
+            // ---- a completed pooled row: column max over 2jj - 1 .. 2jj + 1 ----
+            if (store) {
+                const int i2 = (p & 1) ? (p - 1) / 2 : p / 2;
+                if (pool_data) {
+                    uint32_t h[8];
 #pragma unroll
-                for (int i = 0; i < 8; ++i) h[i] = 0xFC00FC00u;
+                    for (int i = 0; i < 8; ++i) h[i] = 0xFC00FC00u;
 #pragma unroll
-                for (int dc = -1; dc <= 1; ++dc) {
-                    const int col = 2 * jj + dc;
-                    if (col < 0 || col >= g.Q) continue;
-                    const uint4 *src = reinterpret_cast<const uint4 *>(rb + col * ST_PIX_H + 8 * cq);
-                    const uint4 s0 = src[0], s1 = src[4];
-                    h[0] = hmax2u(h[0], s0.x); h[1] = hmax2u(h[1], s0.y);
-                    h[2] = hmax2u(h[2], s0.z); h[3] = hmax2u(h[3], s0.w);
-                    h[4] = hmax2u(h[4], s1.x); h[5] = hmax2u(h[5], s1.y);
-                    h[6] = hmax2u(h[6], s1.z); h[7] = hmax2u(h[7], s1.w);
-                }
-                bool store = false;
-                if (p & 1) {
-                    if (acc_valid) {
-#pragma unroll
-                        for (int i = 0; i < 8; ++i) accv[i] = hmax2u(accv[i], h[i]);
-                        store = true;
+                    for (int dc = -1; dc <= 1; ++dc) {
+                        const int col = 2 * jj + dc;
+                        if (col < 0 || col >= g.Q) continue;
+                        const uint4 *src = reinterpret_cast<const uint4 *>(rb + col * ST_PIX_H + 8 * cq);
+                        const uint4 s0 = src[0], s1 = src[4];
+                        h[0] = hmax2u(h[0], s0.x); h[1] = hmax2u(h[1], s0.y);
+                        h[2] = hmax2u(h[2], s0.z); h[3] = hmax2u(h[3], s0.w);
+                        h[4] = hmax2u(h[4], s1.x); h[5] = hmax2u(h[5], s1.y);
+                        h[6] = hmax2u(h[6], s1.z); h[7] = hmax2u(h[7], s1.w);
                     }
-#pragma unroll
-                    for (int i = 0; i < 8; ++i) carry[i] = h[i];
-                } else {
-#pragma unroll
-                    for (int i = 0; i < 8; ++i) accv[i] = has_carry ? hmax2u(carry[i], h[i]) : h[i];
-                    store = close_even;
-                }
-                if (store) {
-                    const int i2 = (p & 1) ? (p - 1) / 2 : p / 2;
                     uint4 *dst = reinterpret_cast<uint4 *>(static_cast<__half *>(a.y) +
                                                             (((size_t)jb.n * g.P2 + i2) * g.Q2 + jj) * ST_K + 8 * cq);
-                    dst[0] = make_uint4(accv[0], accv[1], accv[2], accv[3]);
-                    dst[4] = make_uint4(accv[4], accv[5], accv[6], accv[7]);
+                    dst[0] = make_uint4(h[0], h[1], h[2], h[3]);
+                    dst[4] = make_uint4(h[4], h[5], h[6], h[7]);
                 }
-            }
-            if (pool_cs) {
-                __half h = __ushort_as_half((unsigned short)0xFC00);
-                for (int dc = -1; dc <= 1; ++dc) {
-                    const int col = 2 * et + dc;
-                    if (col >= 0 && col < g.Q) h = __hmax_nan(h, cb[col]);
+                if (pool_cs) {
+                    __half h = __ushort_as_half((unsigned short)0xFC00);
+                    for (int dc = -1; dc <= 1; ++dc) {
+                        const int col = 2 * et + dc;
+                        if (col >= 0 && col < g.Q) h = __hmax_nan(h, cb[col]);
+                    }
+                    static_cast<__half *>(a.cs_out)[((size_t)jb.n * g.P2 + i2) * g.Q2 + et] = h;
                 }
-                bool store = false;
-                if (p & 1) {
-                    if (acc_valid) { acc_cs = __hmax_nan(acc_cs, h); store = true; }
-                    carry_cs = h;
-                } else {
-                    acc_cs = has_carry ? __hmax_nan(carry_cs, h) : h;
-                    store = close_even;
-                }
-                if (store) {
-                    const int i2 = (p & 1) ? (p - 1) / 2 : p / 2;
-                    static_cast<__half *>(a.cs_out)[((size_t)jb.n * g.P2 + i2) * g.Q2 + et] = acc_cs;
-                }
+                ++n_st;
             }
             if (p & 1) { acc_valid = false; has_carry = true; }
             else { acc_valid = !close_even; }
