@@ -27,14 +27,15 @@
 // Work unit: one pooled output row (n, i), which takes convolution rows
 // 2i - 1, 2i, 2i + 1.  Each CTA owns a contiguous range of units and computes
 // their convolution rows in order, so a row shared by two units is computed
-// once (plus one row at the start of each CTA's range in an image).  The
-// epilogue keeps the column-pooled row of the previous odd convolution row
-// in registers and writes each pooled row when its last convolution row is
-// done.
+// once (plus one row at the start of each CTA's range in an image).  Each
+// epilogue thread keeps the vertical maximum of its output column in
+// registers; when a convolution row completes a pooled row, those column
+// maxima go through a shared-memory row buffer for the 3-wide horizontal
+// maximum and the pooled row is written.
 //
-// Warp roles (416 threads): warps 0-3 fill ring rows (entry e goes to warp
-// e % 4), warp 4 allocates TMEM and issues tcgen05.mma (one elected lane),
-// warps 5-12 are the epilogue: each TMEM lane quadrant is read by two warps,
+// Warp roles (480 threads): warps 0-5 fill ring rows (entry e goes to warp
+// e % 6), warp 6 allocates TMEM and issues tcgen05.mma (one elected lane),
+// warps 7-14 are the epilogue: each TMEM lane quadrant is read by two warps,
 // each taking 32 of the 64 channels.  Four TMEM accumulators rotate over
 // consecutive convolution rows, so the MMAs run up to three rows ahead of
 // the epilogue.  Every mbarrier wait is bounded; on
@@ -60,8 +61,10 @@ constexpr int ST_NSLOT = 24;                 // ring rows: the producers run up 
 constexpr int ST_B_STEP = ST_NB * 32;        // B bytes per K16 step (two core-matrix columns)
 constexpr int ST_B_LBO = ST_NB * 16;         // between the two K chunks of a step
 constexpr int ST_PIX_H = 72;                 // halves per pixel in the epilogue row buffer (144 B)
-constexpr int ST_THREADS = 416;
-constexpr int ST_EPI0 = 160;                 // first epilogue thread
+constexpr int ST_NPROD = 6;                  // ring producer warps
+constexpr int ST_MMA_WARP = ST_NPROD;
+constexpr int ST_EPI0 = 32 * (ST_NPROD + 1); // first epilogue thread
+constexpr int ST_THREADS = ST_EPI0 + 256;
 constexpr int ST_EPI = 256;                  // epilogue threads
 constexpr int ST_NACC = 4;                   // TMEM accumulators (rows in flight between MMA and epilogue)
 constexpr int ST_TMEM_COLS = 128 * ST_NACC;
@@ -75,7 +78,7 @@ constexpr size_t ST_OFF_CS = ST_OFF_ROW + 2ull * 128 * ST_PIX_H * 2;
 // several convolution rows beyond the 7-row window (16 slots: 275 us at 256
 // images, 24: 238 us; deeper staging gained nothing)
 constexpr int ST_STG_W = 2;                  // staging slots per producer warp
-constexpr int ST_NSTG = 4 * ST_STG_W;
+constexpr int ST_NSTG = ST_NPROD * ST_STG_W;
 constexpr int ST_STG_BYTES = 4 * 256 * 4;
 constexpr size_t ST_OFF_STG = ST_OFF_CS + 2ull * 128 * 2;
 constexpr size_t ST_OFF_BAR = ST_OFF_STG + (size_t)ST_NSTG * ST_STG_BYTES;
@@ -161,7 +164,7 @@ __device__ __forceinline__ float image_half(const float *img, const StemGeom &g,
 
 // The ring entries in production order: a CTA's convolution rows each need
 // the input rows not already in the ring (7 at the start of a run within an
-// image, then 2).  Entry e is produced by warp e % 4.
+// image, then 2).  Entry e is produced by warp e % ST_NPROD.
 struct RowIter {
     StemJobs jb;
     bool have;
@@ -185,7 +188,7 @@ struct RowIter {
             while (t < n_new) {
                 const int ee = ecount + t, tt = t;
                 ++t;
-                if ((ee & 3) == w) {
+                if (ee % ST_NPROD == w) {
                     e = ee;
                     y = y0 + tt;
                     n_of_last = jb.n;
@@ -269,7 +272,7 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
-    if (warp == 4) {
+    if (warp == ST_MMA_WARP) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_holder)),
                      "r"((uint32_t)ST_TMEM_COLS));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
@@ -279,9 +282,9 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem = *tmem_holder;
 
-    if (warp < 4) {
+    if (warp < ST_NPROD) {
         // ---------------- ring producers ----------------
-        // Each warp produces every fourth ring entry.  Its next ST_STG_W
+        // Each warp produces every ST_NPROD-th ring entry.  Its next ST_STG_W
         // entries' image rows are in flight as bulk copies (one per channel
         // row of W FP32 values) into its own staging slots; the warp then
         // converts a landed row to the two FP16 copies of its ring slot.
@@ -352,7 +355,7 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
                 warp_wait(smem_u32(&stg_full[warp * ST_STG_W + k % ST_STG_W]), (uint32_t)(k / ST_STG_W) & 1u,
                           a.err, 1u);
         }
-    } else if (warp == 4) {
+    } else if (warp == ST_MMA_WARP) {
         // ---------------- MMA issuer (whole warp, one lane issues) ----------------
         const uint32_t id64 = idesc_f16(128, ST_K);
         const uint32_t id80 = idesc_f16(128, ST_NB);
@@ -410,10 +413,10 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
             warp_wait(smem_u32(mma_done), 0u, a.err, 16u);
         }
     } else {
-        // ---------------- epilogue: warps 5..12 ----------------
+        // ---------------- epilogue: warps 7..14 ----------------
         const int et = threadIdx.x - ST_EPI0;
         const int quad = warp & 3;
-        const int half_id = (warp - 5) >> 2;            // channels 32 * half_id ..
+        const int half_id = (warp - ST_MMA_WARP - 1) >> 2;           // channels 32 * half_id ..
         const int q = quad * 32 + lane;                 // output column of this thread
         const int k0 = 32 * half_id;
         const FaultDelta fd = a.fd;
@@ -573,7 +576,7 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
     }
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
-    if (warp == 4) {
+    if (warp == ST_MMA_WARP) {
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)ST_TMEM_COLS));
     }
