@@ -27,9 +27,15 @@
 // N <= 128 it releases TMEM before its global stores so that the next
 // tile's MMAs overlap them; for N = 256 two accumulators alternate.
 //
+// With N = 256 and no split K, conv_tc_pair_kernel runs the tiles on pairs of
+// CTAs (a cluster of two, tcgen05 cta_group::2): one M = 256 MMA reads the
+// 128 A rows and 128 weight rows each CTA holds, which halves the weight
+// bytes every SM copies and reads per step.
+//
 // Warp roles.  conv_tc_kernel: a producer group (producer warps, each owning
 // whole ring slots, plus for N = 256 the two carry-through warps), one MMA
-// warp (one elected lane issues tcgen05.mma), eight epilogue warps.
+// warp (one elected lane issues tcgen05.mma), eight epilogue warps;
+// conv_tc_pair_kernel the same, with the MMAs issued by the even CTA.
 // conv_tc_halo_kernel (320 threads): warp 0 issues TMA, warp 1 the MMAs,
 // warps 2-9 the epilogue.  Each TMEM lane quadrant (32 output pixels) is
 // read by two epilogue warps, each taking half of the tile's channels.
@@ -636,6 +642,305 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
     if (warp == TC_MMA_WARP) {
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)g.tmem_cols));
+    }
+}
+
+// ---------------------------------------------------------------------------
+// N = 256 over CTA pairs (tcgen05 cta_group::2).  A cluster of two CTAs
+// computes a 256-pixel x 256-channel tile: each CTA copies its own 128 A rows
+// and its half (128 rows) of the tile's weights; the even CTA issues M = 256
+// MMAs that read both CTAs' shared memory and leave each CTA's 128 rows of D
+// in its own TMEM.  Per SM and 128 x 256 x 16 step the shared memory then
+// takes 8 KB of copies and 8 KB of MMA reads instead of 12 + 12, the bound
+// of the single-CTA N = 256 tiles.  Hand-over (all waits bounded):
+//   full[s]        even CTA: stage s landed in both CTAs (one expect_tx
+//                  arrival + the bytes of both CTAs' copies)
+//   consumed[s]    each CTA: the pair's MMAs on stage s completed (commit
+//                  multicast); the carry-through warps then sum their A rows
+//   empty[s]       each CTA: stage s may be refilled (carry-through warps)
+//   acc_full[b]    each CTA: accumulator b complete (commit multicast)
+//   acc_empty[b]   each CTA: its epilogue has read accumulator b
+//   pair_empty[b]  even CTA: both epilogues have read accumulator b
+//   ct_ready[b]    each CTA: carry-through sums of accumulator b in ct_sum[b]
+//   mma_done       each CTA: every MMA of the pair completed (before dealloc)
+constexpr int PR_STAGES = 6;
+constexpr int PR_NPROD = 2, PR_NCT = 2;
+constexpr int PR_MMA_WARP = PR_NPROD + PR_NCT;
+constexpr int PR_EPI_WARP0 = PR_MMA_WARP + 1;
+constexpr int PR_THREADS = 32 * (PR_EPI_WARP0 + N_EPI_WARPS);
+constexpr int PR_BH_BYTES = BM * BK * 2;                  // this CTA's 128 weight rows of a stage
+constexpr int PR_NBAR = 3 * PR_STAGES + 9;
+
+size_t pair_smem_bytes() {
+    return 1024 + (size_t)PR_STAGES * (A_BYTES + PR_BH_BYTES) + 2 * BM * 4 + 8 * PR_NBAR + 16;
+}
+
+__global__ void __launch_bounds__(PR_THREADS, 1)
+conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
+                    const ConvArgs a, const TcGeom g) {
+    constexpr int BN = 256;
+    static_assert(PR_STAGES % PR_NPROD == 0, "producer warps must own whole ring slots");
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint8_t *As = smem;                                    // [STAGES][A_BYTES]
+    uint8_t *Bs = As + PR_STAGES * A_BYTES;                // [STAGES][PR_BH_BYTES]
+    float *ct_sum = (float *)(Bs + PR_STAGES * PR_BH_BYTES);   // [2][BM]
+    uint64_t *full = (uint64_t *)(ct_sum + 2 * BM);
+    uint64_t *consumed = full + PR_STAGES;
+    uint64_t *empty = consumed + PR_STAGES;
+    uint64_t *acc_full = empty + PR_STAGES;                // [2]
+    uint64_t *acc_empty = acc_full + 2;                    // [2]
+    uint64_t *pair_empty = acc_empty + 2;                  // [2]
+    uint64_t *ct_ready = pair_empty + 2;                   // [2]
+    uint64_t *mma_done = ct_ready + 2;
+    uint32_t *tmem_holder = (uint32_t *)(mma_done + 1);
+    volatile uint32_t *abort_flag = tmem_holder + 1;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t crank = cluster_ctarank();
+    const bool leader = crank == 0;
+    const int cid = blockIdx.x >> 1, ncl = gridDim.x >> 1;
+    const int m_pairs = (g.m_tiles + 1) >> 1;
+    const int num_items = m_pairs * g.n_tiles;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < PR_STAGES; ++s) {
+            mbar_init(smem_u32(&full[s]), 1);
+            mbar_init(smem_u32(&consumed[s]), 1);
+            mbar_init(smem_u32(&empty[s]), PR_NCT);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(smem_u32(&acc_full[b]), 1);
+            mbar_init(smem_u32(&acc_empty[b]), N_EPI_WARPS);
+            mbar_init(smem_u32(&pair_empty[b]), 2 * N_EPI_WARPS);
+            mbar_init(smem_u32(&ct_ready[b]), PR_NCT);
+        }
+        mbar_init(smem_u32(mma_done), 1);
+        *abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == PR_MMA_WARP) {
+        // one warp of each CTA of the pair allocates the same columns in both
+        asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_holder)),
+                     "r"(512u));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;");
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    // the peer's barriers are initialised before any copy or arrival targets them
+    cluster_sync();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tmem = *tmem_holder;
+    pdl_wait();
+    pdl_trigger();
+
+    if (warp < PR_NPROD) {
+        // ---------------- TMA producers (slot s belongs to warp s % PR_NPROD) ----------------
+        if (elect_one()) {
+            asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&amap) : "memory");
+            asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&bmap) : "memory");
+        }
+        __syncwarp();
+        const uint32_t full_even = mapa_shared(smem_u32(full), 0u);
+        int it = 0;
+        bool ok = true;
+        for (int item = cid; item < num_items && ok; item += ncl) {
+            if (__any_sync(0xffffffffu, *abort_flag)) break;
+            const int m_pair = item / g.n_tiles, n_tile = item % g.n_tiles;
+            const int m0 = (2 * m_pair + (int)crank) * BM;       // past M: rows that are never stored
+            const int nimg = m0 / g.PQ, rem = m0 % g.PQ;
+            const int p = rem / g.Q, q = rem % g.Q;
+            const int w0 = q * g.stride - g.pad, h0 = p * g.stride - g.pad;
+            for (int kb = 0; kb < g.n_kb; ++kb, ++it) {
+                const int s = it % PR_STAGES;
+                if (s % PR_NPROD != warp) continue;
+                if (!warp_wait(smem_u32(&empty[s]), ((uint32_t)(it / PR_STAGES) & 1u) ^ 1u, a.err, 1u)) { ok = false; break; }
+                if (elect_one()) {
+                    const uint32_t fb = full_even + (uint32_t)(s * 8);
+                    if (leader) mbar_arrive_expect_tx(smem_u32(&full[s]), 2u * (A_BYTES + PR_BH_BYTES));
+                    const int tap = tap_of(kb / g.cpb, g.ctr_tap);
+                    const int c0 = (kb % g.cpb) * BK;
+                    const int r = tap / g.S, sx = tap % g.S;
+                    tma_load_im2col_pair(smem_u32(As + s * A_BYTES), &amap, fb, c0, w0, h0, nimg, (uint16_t)sx,
+                                         (uint16_t)r);
+                    tma_load_2d_pair(smem_u32(Bs + s * PR_BH_BYTES), &bmap, fb, tap * g.C + c0,
+                                     n_tile * BN + (int)crank * BM);
+                }
+                __syncwarp();
+            }
+        }
+        if (!ok && lane == 0) *abort_flag = 1;
+    } else if (warp < PR_MMA_WARP) {
+        // ---------------- carry-through sums (as in conv_tc_kernel, N = 256) ----------------
+        // This CTA's A rows of every stage, read after the pair's MMAs used
+        // the stage; then the stage goes back to the producers.
+        constexpr int ROWS_W = BM / PR_NCT;
+        constexpr int MT = ROWS_W / 16;
+        const float coef = __half2float(__ushort_as_half(g.coef_h));
+        const int w = warp - PR_NPROD;
+        const int lm_row = (lane & 7) + ((lane >> 3) & 1) * 8, lm_chk = lane >> 4;
+        int it = 0, lt = 0;
+        bool ok = true;
+        for (int item = cid; item < num_items && ok; item += ncl, ++lt) {
+            if (__any_sync(0xffffffffu, *abort_flag)) break;
+            const bool ct_here = g.ct_mode != CT_NONE_ && item % g.n_tiles == 0;
+            const int ab = lt & 1;
+            float acc[MT][4];
+#pragma unroll
+            for (int m = 0; m < MT; ++m)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) acc[m][e] = 0.f;
+            for (int kb = 0; kb < g.n_kb; ++kb, ++it) {
+                const int s = it % PR_STAGES;
+                if (!warp_wait(smem_u32(&consumed[s]), (uint32_t)(it / PR_STAGES) & 1u, a.err, 2u)) { ok = false; break; }
+                if (ct_here && kb < g.cpb) {
+                    const uint32_t tbase = smem_u32(As + s * A_BYTES);
+#pragma unroll
+                    for (int m = 0; m < MT; ++m) {
+                        const int row = w * ROWS_W + m * 16 + lm_row;
+                        const uint32_t rbase = tbase + (uint32_t)row * 128u;
+#pragma unroll
+                        for (int t = 0; t < 4; ++t) {
+                            const uint32_t chk = (uint32_t)((2 * t + lm_chk) ^ (row & 7));
+                            uint32_t a0, a1, a2, a3;
+                            ldsm_x4(rbase + chk * 16u, a0, a1, a2, a3);
+                            mma_rowsum_16x16(acc[m], a0, a1, a2, a3);
+                        }
+                    }
+                }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&empty[s]));
+            }
+            if (!ok) break;
+            if (!warp_wait(smem_u32(&acc_empty[ab]), ((uint32_t)(lt >> 1) & 1u) ^ 1u, a.err, 8u)) { ok = false; break; }
+            if ((lane & 3) == 0) {
+#pragma unroll
+                for (int m = 0; m < MT; ++m) {
+                    const int r0 = w * ROWS_W + m * 16 + (lane >> 2);
+                    ct_sum[ab * BM + r0] = coef * acc[m][0];
+                    ct_sum[ab * BM + r0 + 8] = coef * acc[m][2];
+                }
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&ct_ready[ab]));
+        }
+        if (!ok && lane == 0) *abort_flag = 1;
+    } else if (warp == PR_MMA_WARP) {
+        // ---------------- MMA issuer: the even CTA, one elected lane ----------------
+        if (leader) {
+            const uint32_t idesc = idesc_f16(2 * BM, BN);
+            int it = 0, lt = 0;
+            for (int item = cid; item < num_items; item += ncl, ++lt) {
+                if (__any_sync(0xffffffffu, *abort_flag)) break;
+                const int ab = lt & 1;
+                if (!warp_wait(smem_u32(&pair_empty[ab]), ((uint32_t)(lt >> 1) & 1u) ^ 1u, a.err, 8u)) {
+                    if (lane == 0) *abort_flag = 1;
+                    break;
+                }
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                bool ok = true;
+                for (int kb = 0; kb < g.n_kb; ++kb, ++it) {
+                    const int s = it % PR_STAGES;
+                    if (!warp_wait(smem_u32(&full[s]), (uint32_t)(it / PR_STAGES) & 1u, a.err, 2u)) { ok = false; break; }
+                    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                    if (elect_one()) {
+                        const uint32_t d = tmem + (uint32_t)(ab * BN);
+                        const uint64_t ad0 = smem_desc_sw128(smem_u32(As + s * A_BYTES));
+                        const uint64_t bd0 = smem_desc_sw128(smem_u32(Bs + s * PR_BH_BYTES));
+#pragma unroll
+                        for (int k16 = 0; k16 < BK / 16; ++k16)
+                            umma_f16_pair(d, ad0 + 2 * k16, bd0 + 2 * k16, idesc, (kb > 0 || k16 > 0) ? 1u : 0u);
+                        umma_commit_pair_mc(smem_u32(&consumed[s]), (uint16_t)3u);
+                    }
+                    __syncwarp();
+                }
+                if (!ok) { if (lane == 0) *abort_flag = 1; break; }
+                if (elect_one()) umma_commit_pair_mc(smem_u32(&acc_full[ab]), (uint16_t)3u);
+                __syncwarp();
+            }
+            // fires in both CTAs once every MMA issued above has completed
+            if (elect_one()) umma_commit_pair_mc(smem_u32(mma_done), (uint16_t)3u);
+            __syncwarp();
+        }
+    } else {
+        // ---------------- epilogue: 8 warps, this CTA's 128 rows ----------------
+        const int ep = warp - PR_EPI_WARP0;
+        const int quad = warp & 3;
+        const int half = ep >> 2;
+        const int row = quad * 32 + lane;
+        const __half *x = static_cast<const __half *>(a.x);
+        const FaultDelta fd = a.fd;
+        const uint32_t pair_empty_even = mapa_shared(smem_u32(pair_empty), 0u);
+        int lt = 0;
+        for (int item = cid; item < num_items; item += ncl, ++lt) {
+            const int m_pair = item / g.n_tiles, n_tile = item % g.n_tiles;
+            const int m0 = (2 * m_pair + (int)crank) * BM;
+            Res16 rs[BN / 32];
+            {
+                const int mp = m0 + row;
+#pragma unroll
+                for (int c = 0; c < BN / 32; ++c)
+                    rs[c] = mp < g.M ? load_res16(a, g.K, (size_t)mp, n_tile * BN + half * (BN / 2) + 16 * c)
+                                     : Res16{make_uint4(0u, 0u, 0u, 0u), make_uint4(0u, 0u, 0u, 0u)};
+            }
+            CsIn csv{0.f, 0.f};
+            {
+                const int mp = m0 + row;
+                if (half == 0 && a.cs_out != nullptr && n_tile == 0 && mp < g.M) {
+                    const int ni = mp / g.PQ, rm = mp % g.PQ;
+                    csv = load_cs_inputs(a, g, mp, ni, rm / g.Q, rm % g.Q);
+                }
+            }
+            const int ab = lt & 1;
+            const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
+            bool ok = mbar_wait(smem_u32(&acc_full[ab]), aph, a.err, 4u) && !*abort_flag;
+            ok = ok && mbar_wait(smem_u32(&ct_ready[ab]), aph, a.err, 4u);
+            ok = __all_sync(0xffffffffu, ok);      // tcgen05.ld below is warp-collective
+            if (!ok) break;
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            const uint32_t trow = tmem + (uint32_t)(ab * BN) + ((uint32_t)(quad * 32) << 16);
+            const int m = m0 + row;
+            const bool valid = m < g.M;
+            const int mm = valid ? m : 0;
+            const int nimg = mm / g.PQ, rem = mm % g.PQ, p = rem / g.Q, q = rem % g.Q;
+            float fsrc = 0.f;
+            if (fd.active) {
+                const int h = p * g.stride + fd.r - g.pad, w = q * g.stride + fd.s - g.pad;
+                if (h >= 0 && h < a.H && w >= 0 && w < a.W) {
+                    if (fd.cin < g.C) fsrc = ldh(x, (((size_t)nimg * a.H + h) * a.W + w) * g.C + fd.cin);
+                    else if (a.cs_in) fsrc = ldh(static_cast<const __half *>(a.cs_in), ((size_t)nimg * a.H + h) * a.W + w);
+                }
+            }
+            const int n0 = n_tile * BN;
+            const bool do_cs = half == 0 && a.cs_out != nullptr && n_tile == 0;
+#pragma unroll
+            for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 16) {
+                float v[16];
+                tmem_ld16(trow + c, v);
+                if (valid) store_chunk_pre(v, rs[(c - half * (BN / 2)) / 16], a, g.K, (size_t)m, n0 + c, fsrc);
+            }
+            if (do_cs && valid) {
+                const float ctv = g.ct_mode != CT_NONE_ ? ct_sum[ab * BM + row] : 0.f;
+                store_checksum_pre(ctv, csv, a, g, m, fsrc);
+            }
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            __syncwarp();
+            if (lane == 0) {
+                mbar_arrive(smem_u32(&acc_empty[ab]));
+                mbar_arrive_cluster(pair_empty_even + (uint32_t)(ab * 8));
+            }
+        }
+    }
+    // every MMA of the pair has completed before TMEM is freed in either CTA
+    if (warp == PR_MMA_WARP) warp_wait(smem_u32(mma_done), 0u, a.err, 16u);
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    // no CTA leaves while its peer may still read its shared memory or
+    // arrive on its barriers
+    cluster_sync();
+    if (warp == PR_MMA_WARP) {
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(512u));
     }
 }
 
@@ -1307,6 +1612,9 @@ struct TcPlan {
     int BN, n_tiles, sms;
     int cs, max_clusters;        // cluster size of the multicast variant (1: none)
     size_t smem;
+    CUtensorMap bmap_pair;       // N = 256 over CTA pairs: 128-row weight halves
+    int pair_clusters;           // resident CTA pairs (0: no pair variant)
+    size_t pair_smem;
 };
 
 bool tc_supported(int C, int K, int R, int S, int stride, int pad, std::string *why) {
@@ -1370,6 +1678,34 @@ TcPlan *tc_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, cons
         e = cudaFuncSetAttribute(conv_tc_kernel<256, 4, 1, 1, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
     }
     if (e != cudaSuccess) { if (why) *why = "shared memory attribute"; delete pl; return nullptr; }
+    // N = 256 over CTA pairs (cta_group::2): each CTA copies 128 of the 256 weight rows
+    pl->pair_clusters = 0;
+    if (pl->BN == 256) {
+        cuuint32_t box_h[2] = {BK, (cuuint32_t)BM};
+        r = g_encode_tiled(&pl->bmap_pair, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void *>(w_dev), bdim, bstr,
+                           box_h, bes, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        pl->pair_smem = pair_smem_bytes();
+        cudaError_t pe = cudaFuncSetAttribute(conv_tc_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              (int)pl->pair_smem);
+        if (r == CUDA_SUCCESS && pe == cudaSuccess) {
+            cudaLaunchConfig_t cfg = {};
+            cfg.gridDim = dim3(2 * 64);
+            cfg.blockDim = dim3(PR_THREADS);
+            cfg.dynamicSmemBytes = pl->pair_smem;
+            cudaLaunchAttribute at[1];
+            at[0].id = cudaLaunchAttributeClusterDimension;
+            at[0].val.clusterDim.x = 2;
+            at[0].val.clusterDim.y = 1;
+            at[0].val.clusterDim.z = 1;
+            cfg.attrs = at;
+            cfg.numAttrs = 1;
+            int n = 0;
+            if (cudaOccupancyMaxActiveClusters(&n, conv_tc_pair_kernel, &cfg) == cudaSuccess && n > 0)
+                pl->pair_clusters = n;
+        }
+        cudaGetLastError();
+    }
     // cluster variant: B slices of BN / TC_CS rows multicast to TC_CS CTAs
     pl->cs = 1;
     pl->max_clusters = 0;
@@ -1413,7 +1749,13 @@ cudaError_t launch_conv_tc(const ConvArgs &a, const void *plan, cudaStream_t st,
     g.splits = (a.K % 8 == 0) ? splitk_choose(tiles, g.n_kb, 4, pl->sms / 2, g.M, g.ws_ld, a.ws ? a.ws_bytes : 0) : 1;
     g.kps = (g.n_kb + g.splits - 1) / g.splits;
     g.m_groups = g.m_tiles;
-    if (pl->cs > 1 && g.splits == 1 && g.m_tiles >= 4 * pl->cs && g.n_kb >= 4) {
+    if (pl->pair_clusters > 0 && g.splits == 1 && g.m_tiles >= 2) {
+        // N = 256 tiles over CTA pairs: 256 pixels x 256 channels per pair
+        const int items = ((g.m_tiles + 1) / 2) * g.n_tiles;
+        const int ncl = items < pl->pair_clusters ? items : pl->pair_clusters;
+        pdl_launch_cluster(conv_tc_pair_kernel, dim3(2 * ncl), PR_THREADS, pl->pair_smem, st, 2, pl->amap,
+                           pl->bmap_pair, a, g);
+    } else if (pl->cs > 1 && g.splits == 1 && g.m_tiles >= 4 * pl->cs && g.n_kb >= 4) {
         // clusters of cs CTAs on groups of cs consecutive M tiles, sharing B
         // (not for a few K blocks per tile: little B to share, and the
         // cluster's CTAs advance in lockstep)

@@ -5,7 +5,7 @@ import pytest
 
 import oracle
 from _cache import inputs
-from _gpu import assert_parity, ct, model, onet, run
+from _gpu import TOL, assert_parity, ct, model, onet, run, same_class
 
 pytestmark = pytest.mark.gpu
 
@@ -49,6 +49,34 @@ def test_resnet18_imagenet_fp16_full_batch_sampled():
     idx = [0, 129, 255]
     o = _oracle("resnet18_imagenet", "fp16", x[idx])
     assert_parity(lg[idx], S[idx], o["logits"], o["S"], "fp16", "resnet18_imagenet")
+
+
+def test_resnet18_imagenet_fp16_odd_tile_count_and_flip():
+    """131 images: the 256-channel layers have an odd number of 128-row
+    tiles (201 at 14 x 14, 51 at 7 x 7), so the last pair of CTAs that share
+    a 256-row tile has its second CTA past the output; the last image's rows
+    lie in that pair's first CTA.  Then one weight flip in the first
+    256-channel convolution, compared on the same images."""
+    name, B = "resnet18_imagenet", 131
+    m = model(name, max_batch=B)
+    x = inputs(name, B)
+    lg, S, _ = run(m, x)
+    idx = [0, 130]
+    net = onet(name, "fp16")
+    o = oracle.forward(net, x[idx])
+    assert_parity(lg[idx], S[idx], o["logits"], o["S"], "fp16", "resnet18_imagenet b131")
+    layer = [i for i, L in enumerate(net.layers) if L.op == "conv" and L.n_data_out == 256][0]
+    n_w = [n for kind, lay, n, bits in ct().ct_buffers(m, B) if kind == 0 and lay == layer][0]
+    e, bit = n_w // 3 + 7, 13
+    ct().ct_inject(m, 0, layer, e, bit)
+    lg, S, _ = run(m, x)
+    o = oracle.forward(net, x[idx], oracle.Fault(0, layer, e, bit))
+    for j, i in enumerate(idx):
+        assert same_class(S[i], o["S"][j]), (i, S[i], o["S"][j])
+        if np.isfinite(o["S"][j]):
+            assert abs(S[i] - o["S"][j]) <= TOL["fp16"] * max(abs(o["S"][j]), 1e-6), (i, S[i], o["S"][j])
+    assert ct().ct_device_error(m) == 0
+    m.close()
 
 
 def test_vgg16_fp16_full_batch_sampled():
