@@ -462,7 +462,8 @@ def main():
     tc_n, tc_ms, tc_fl = fam_stats[0]
     si_n, si_ms, si_fl = fam_stats[1]
     if tc_ms >= si_ms and tc_n:
-        roof = {"kernel": "conv_tc_kernel (tcgen05, fp16 in / fp32 acc)", "bound": "tensor",
+        roof = {"kernel": "tcgen05 convolution family: stem_pool, conv_tc_halo, conv_tc, conv_tc_pair "
+                          "(fp16 in / fp32 acc)", "bound": "tensor",
                 "achieved": tc_fl / (tc_ms / 1e3) / 1e12, "peak": pk["bf16_tflops"],
                 "unit": "TFLOP/s",
                 "peak_source": "%s bf16 dense burst; fp16 has the bf16 rate" % pk_kind,
