@@ -104,14 +104,17 @@ def get_threads() -> int:
 # ---------------------------------------------------------------------------
 
 def round_to(x, prec: str) -> np.ndarray:
-    """Round float64 values to the storage precision (nearest-even)."""
+    """Round float64 values to the storage precision (nearest-even).  Values
+    beyond the format's range become +-inf, as in the stored tensors (bit
+    flips in exponents produce them on purpose), without a warning."""
     x = np.asarray(x, dtype=np.float64)
     if prec == "fp64":
         return x.copy()
-    if prec == "fp32":
-        return x.astype(np.float32).astype(np.float64)
-    if prec == "fp16":
-        return x.astype(np.float16).astype(np.float64)
+    with np.errstate(over="ignore"):
+        if prec == "fp32":
+            return x.astype(np.float32).astype(np.float64)
+        if prec == "fp16":
+            return x.astype(np.float16).astype(np.float64)
     raise ValueError(prec)
 
 
