@@ -652,27 +652,29 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
 // MMAs that read both CTAs' shared memory and leave each CTA's 128 rows of D
 // in its own TMEM.  Per SM and 128 x 256 x 16 step the shared memory then
 // takes 8 KB of copies and 8 KB of MMA reads instead of 12 + 12, the bound
-// of the single-CTA N = 256 tiles.  Hand-over (all waits bounded):
+// of the single-CTA N = 256 tiles.
+//
+// The carry-through column at the centre tap is coef * the channel sum of
+// one input pixel, so each epilogue thread adds it up from the input tensor
+// (rows of C FP16 values, just copied through L2) with FP32 accumulation;
+// the stage pipeline carries only the GEMM.  Hand-over (all waits bounded):
 //   full[s]        even CTA: stage s landed in both CTAs (one expect_tx
 //                  arrival + the bytes of both CTAs' copies)
-//   consumed[s]    each CTA: the pair's MMAs on stage s completed (commit
-//                  multicast); the carry-through warps then sum their A rows
-//   empty[s]       each CTA: stage s may be refilled (carry-through warps)
+//   empty[s]       each CTA: the pair's MMAs on stage s completed (commit
+//                  multicast): the stage may be refilled
 //   acc_full[b]    each CTA: accumulator b complete (commit multicast)
-//   acc_empty[b]   each CTA: its epilogue has read accumulator b
 //   pair_empty[b]  even CTA: both epilogues have read accumulator b
-//   ct_ready[b]    each CTA: carry-through sums of accumulator b in ct_sum[b]
 //   mma_done       each CTA: every MMA of the pair completed (before dealloc)
 constexpr int PR_STAGES = 6;
-constexpr int PR_NPROD = 2, PR_NCT = 2;
-constexpr int PR_MMA_WARP = PR_NPROD + PR_NCT;
+constexpr int PR_NPROD = 2;
+constexpr int PR_MMA_WARP = PR_NPROD;
 constexpr int PR_EPI_WARP0 = PR_MMA_WARP + 1;
 constexpr int PR_THREADS = 32 * (PR_EPI_WARP0 + N_EPI_WARPS);
 constexpr int PR_BH_BYTES = BM * BK * 2;                  // this CTA's 128 weight rows of a stage
-constexpr int PR_NBAR = 3 * PR_STAGES + 9;
+constexpr int PR_NBAR = 2 * PR_STAGES + 5;                // full, empty per stage; acc_full, pair_empty, mma_done
 
 size_t pair_smem_bytes() {
-    return 1024 + (size_t)PR_STAGES * (A_BYTES + PR_BH_BYTES) + 2 * BM * 4 + 8 * PR_NBAR + 16;
+    return 1024 + (size_t)PR_STAGES * (A_BYTES + PR_BH_BYTES) + 8 * PR_NBAR + 16;
 }
 
 __global__ void __launch_bounds__(PR_THREADS, 1)
@@ -684,15 +686,11 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint8_t *As = smem;                                    // [STAGES][A_BYTES]
     uint8_t *Bs = As + PR_STAGES * A_BYTES;                // [STAGES][PR_BH_BYTES]
-    float *ct_sum = (float *)(Bs + PR_STAGES * PR_BH_BYTES);   // [2][BM]
-    uint64_t *full = (uint64_t *)(ct_sum + 2 * BM);
-    uint64_t *consumed = full + PR_STAGES;
-    uint64_t *empty = consumed + PR_STAGES;
+    uint64_t *full = (uint64_t *)(Bs + PR_STAGES * PR_BH_BYTES);
+    uint64_t *empty = full + PR_STAGES;
     uint64_t *acc_full = empty + PR_STAGES;                // [2]
-    uint64_t *acc_empty = acc_full + 2;                    // [2]
-    uint64_t *pair_empty = acc_empty + 2;                  // [2]
-    uint64_t *ct_ready = pair_empty + 2;                   // [2]
-    uint64_t *mma_done = ct_ready + 2;
+    uint64_t *pair_empty = acc_full + 2;                   // [2]
+    uint64_t *mma_done = pair_empty + 2;
     uint32_t *tmem_holder = (uint32_t *)(mma_done + 1);
     volatile uint32_t *abort_flag = tmem_holder + 1;
 
@@ -706,14 +704,11 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
     if (threadIdx.x == 0) {
         for (int s = 0; s < PR_STAGES; ++s) {
             mbar_init(smem_u32(&full[s]), 1);
-            mbar_init(smem_u32(&consumed[s]), 1);
-            mbar_init(smem_u32(&empty[s]), PR_NCT);
+            mbar_init(smem_u32(&empty[s]), 1);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(smem_u32(&acc_full[b]), 1);
-            mbar_init(smem_u32(&acc_empty[b]), N_EPI_WARPS);
             mbar_init(smem_u32(&pair_empty[b]), 2 * N_EPI_WARPS);
-            mbar_init(smem_u32(&ct_ready[b]), PR_NCT);
         }
         mbar_init(smem_u32(mma_done), 1);
         *abort_flag = 0;
@@ -770,61 +765,6 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
             }
         }
         if (!ok && lane == 0) *abort_flag = 1;
-    } else if (warp < PR_MMA_WARP) {
-        // ---------------- carry-through sums (as in conv_tc_kernel, N = 256) ----------------
-        // This CTA's A rows of every stage, read after the pair's MMAs used
-        // the stage; then the stage goes back to the producers.
-        constexpr int ROWS_W = BM / PR_NCT;
-        constexpr int MT = ROWS_W / 16;
-        const float coef = __half2float(__ushort_as_half(g.coef_h));
-        const int w = warp - PR_NPROD;
-        const int lm_row = (lane & 7) + ((lane >> 3) & 1) * 8, lm_chk = lane >> 4;
-        int it = 0, lt = 0;
-        bool ok = true;
-        for (int item = cid; item < num_items && ok; item += ncl, ++lt) {
-            if (__any_sync(0xffffffffu, *abort_flag)) break;
-            const bool ct_here = g.ct_mode != CT_NONE_ && item % g.n_tiles == 0;
-            const int ab = lt & 1;
-            float acc[MT][4];
-#pragma unroll
-            for (int m = 0; m < MT; ++m)
-#pragma unroll
-                for (int e = 0; e < 4; ++e) acc[m][e] = 0.f;
-            for (int kb = 0; kb < g.n_kb; ++kb, ++it) {
-                const int s = it % PR_STAGES;
-                if (!warp_wait(smem_u32(&consumed[s]), (uint32_t)(it / PR_STAGES) & 1u, a.err, 2u)) { ok = false; break; }
-                if (ct_here && kb < g.cpb) {
-                    const uint32_t tbase = smem_u32(As + s * A_BYTES);
-#pragma unroll
-                    for (int m = 0; m < MT; ++m) {
-                        const int row = w * ROWS_W + m * 16 + lm_row;
-                        const uint32_t rbase = tbase + (uint32_t)row * 128u;
-#pragma unroll
-                        for (int t = 0; t < 4; ++t) {
-                            const uint32_t chk = (uint32_t)((2 * t + lm_chk) ^ (row & 7));
-                            uint32_t a0, a1, a2, a3;
-                            ldsm_x4(rbase + chk * 16u, a0, a1, a2, a3);
-                            mma_rowsum_16x16(acc[m], a0, a1, a2, a3);
-                        }
-                    }
-                }
-                __syncwarp();
-                if (lane == 0) mbar_arrive(smem_u32(&empty[s]));
-            }
-            if (!ok) break;
-            if (!warp_wait(smem_u32(&acc_empty[ab]), ((uint32_t)(lt >> 1) & 1u) ^ 1u, a.err, 8u)) { ok = false; break; }
-            if ((lane & 3) == 0) {
-#pragma unroll
-                for (int m = 0; m < MT; ++m) {
-                    const int r0 = w * ROWS_W + m * 16 + (lane >> 2);
-                    ct_sum[ab * BM + r0] = coef * acc[m][0];
-                    ct_sum[ab * BM + r0 + 8] = coef * acc[m][2];
-                }
-            }
-            __syncwarp();
-            if (lane == 0) mbar_arrive(smem_u32(&ct_ready[ab]));
-        }
-        if (!ok && lane == 0) *abort_flag = 1;
     } else if (warp == PR_MMA_WARP) {
         // ---------------- MMA issuer: the even CTA, one elected lane ----------------
         if (leader) {
@@ -850,7 +790,7 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
 #pragma unroll
                         for (int k16 = 0; k16 < BK / 16; ++k16)
                             umma_f16_pair(d, ad0 + 2 * k16, bd0 + 2 * k16, idesc, (kb > 0 || k16 > 0) ? 1u : 0u);
-                        umma_commit_pair_mc(smem_u32(&consumed[s]), (uint16_t)3u);
+                        umma_commit_pair_mc(smem_u32(&empty[s]), (uint16_t)3u);
                     }
                     __syncwarp();
                 }
@@ -870,39 +810,54 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
         const int row = quad * 32 + lane;
         const __half *x = static_cast<const __half *>(a.x);
         const FaultDelta fd = a.fd;
+        const float coef = __half2float(__ushort_as_half(g.coef_h));
+        const int ctr_r = g.ctr_tap / g.S, ctr_s = g.ctr_tap % g.S;
         const uint32_t pair_empty_even = mapa_shared(smem_u32(pair_empty), 0u);
         int lt = 0;
         for (int item = cid; item < num_items; item += ncl, ++lt) {
             const int m_pair = item / g.n_tiles, n_tile = item % g.n_tiles;
             const int m0 = (2 * m_pair + (int)crank) * BM;
+            const int m = m0 + row;
+            const bool valid = m < g.M;
+            const int mm = valid ? m : 0;
+            const int nimg = mm / g.PQ, rem = mm % g.PQ, p = rem / g.Q, q = rem % g.Q;
+            const bool do_cs = half == 0 && a.cs_out != nullptr && n_tile == 0;
             Res16 rs[BN / 32];
-            {
-                const int mp = m0 + row;
 #pragma unroll
-                for (int c = 0; c < BN / 32; ++c)
-                    rs[c] = mp < g.M ? load_res16(a, g.K, (size_t)mp, n_tile * BN + half * (BN / 2) + 16 * c)
-                                     : Res16{make_uint4(0u, 0u, 0u, 0u), make_uint4(0u, 0u, 0u, 0u)};
-            }
+            for (int c = 0; c < BN / 32; ++c)
+                rs[c] = valid ? load_res16(a, g.K, (size_t)m, n_tile * BN + half * (BN / 2) + 16 * c)
+                              : Res16{make_uint4(0u, 0u, 0u, 0u), make_uint4(0u, 0u, 0u, 0u)};
             CsIn csv{0.f, 0.f};
-            {
-                const int mp = m0 + row;
-                if (half == 0 && a.cs_out != nullptr && n_tile == 0 && mp < g.M) {
-                    const int ni = mp / g.PQ, rm = mp % g.PQ;
-                    csv = load_cs_inputs(a, g, mp, ni, rm / g.Q, rm % g.Q);
+            // carry-through column: coef * sum of the C channels of the centre-tap pixel
+            float ctv = 0.f;
+            if (do_cs && valid) {
+                csv = load_cs_inputs(a, g, m, nimg, p, q);
+                if (g.ct_mode != CT_NONE_) {
+                    const int h = p * g.stride + ctr_r - g.pad, w = q * g.stride + ctr_s - g.pad;
+                    if (h >= 0 && h < a.H && w >= 0 && w < a.W) {
+                        const uint4 *src = reinterpret_cast<const uint4 *>(x + (((size_t)nimg * a.H + h) * a.W + w) * g.C);
+                        float acc[4] = {0.f, 0.f, 0.f, 0.f};
+                        for (int c8 = 0; c8 < g.C / 8; ++c8) {
+                            const uint4 u = __ldg(src + c8);
+                            const __half2 *hh = reinterpret_cast<const __half2 *>(&u);
+#pragma unroll
+                            for (int i = 0; i < 4; ++i) {
+                                const float2 f = __half22float2(hh[i]);
+                                acc[i] += f.x;
+                                acc[i] += f.y;
+                            }
+                        }
+                        ctv = coef * ((acc[0] + acc[1]) + (acc[2] + acc[3]));
+                    }
                 }
             }
             const int ab = lt & 1;
             const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
             bool ok = mbar_wait(smem_u32(&acc_full[ab]), aph, a.err, 4u) && !*abort_flag;
-            ok = ok && mbar_wait(smem_u32(&ct_ready[ab]), aph, a.err, 4u);
             ok = __all_sync(0xffffffffu, ok);      // tcgen05.ld below is warp-collective
             if (!ok) break;
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
             const uint32_t trow = tmem + (uint32_t)(ab * BN) + ((uint32_t)(quad * 32) << 16);
-            const int m = m0 + row;
-            const bool valid = m < g.M;
-            const int mm = valid ? m : 0;
-            const int nimg = mm / g.PQ, rem = mm % g.PQ, p = rem / g.Q, q = rem % g.Q;
             float fsrc = 0.f;
             if (fd.active) {
                 const int h = p * g.stride + fd.r - g.pad, w = q * g.stride + fd.s - g.pad;
@@ -912,23 +867,16 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
                 }
             }
             const int n0 = n_tile * BN;
-            const bool do_cs = half == 0 && a.cs_out != nullptr && n_tile == 0;
 #pragma unroll
             for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 16) {
                 float v[16];
                 tmem_ld16(trow + c, v);
                 if (valid) store_chunk_pre(v, rs[(c - half * (BN / 2)) / 16], a, g.K, (size_t)m, n0 + c, fsrc);
             }
-            if (do_cs && valid) {
-                const float ctv = g.ct_mode != CT_NONE_ ? ct_sum[ab * BM + row] : 0.f;
-                store_checksum_pre(ctv, csv, a, g, m, fsrc);
-            }
+            if (do_cs && valid) store_checksum_pre(ctv, csv, a, g, m, fsrc);
             asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
             __syncwarp();
-            if (lane == 0) {
-                mbar_arrive(smem_u32(&acc_empty[ab]));
-                mbar_arrive_cluster(pair_empty_even + (uint32_t)(ab * 8));
-            }
+            if (lane == 0) mbar_arrive_cluster(pair_empty_even + (uint32_t)(ab * 8));
         }
     }
     // every MMA of the pair has completed before TMEM is freed in either CTA
