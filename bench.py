@@ -39,6 +39,7 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 import synth  # noqa: E402
+from paper_2609_16742_gb300 import replicas  # noqa: E402
 
 METRIC = "protected images/sec and checksum overhead % vs unprotected; conv % of GB300 peak"
 DEFAULT_WORKLOAD = "resnet18_imagenet"
@@ -259,7 +260,7 @@ def main():
     # evaluation batches for this rank (distinct slices of the seeded set per
     # rank); two, alternating, so that each step's re-run images come from
     # the batch before it
-    x_hosts = [synth.make_input(wl, batch=B, first=(2 * rank + j) * B) for j in range(2)]
+    x_hosts = [synth.make_input(wl, batch=B, first=f) for f in replicas.input_slices(rank, B)]
     x_host = x_hosts[0]
     bufs = [{"x": torch.from_numpy(xh_).cuda(), "lg": torch.empty(B, wl.n_classes, device="cuda"),
              "S": torch.empty(B, device="cuda"), "fl": torch.empty(B, dtype=torch.uint8, device="cuda")}
@@ -310,11 +311,7 @@ def main():
                 n_re += fn()
         e1.record(stream)
         barrier()
-        ms = e0.elapsed_time(e1)
-        if dist is not None:
-            t = torch.tensor([ms], device="cuda")
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ms = float(t.item())
+        ms = replicas.reduce_max(e0.elapsed_time(e1), dist, "cuda")
         return ms, n_re
 
     for _ in range(max(args.warmup, 3)):
@@ -361,7 +358,7 @@ def main():
         replace_leg = {
             "what": "Sec. II-A prune-and-replace (ct_build CT_PROTECT_REPLACE): the least important channel of "
                     "every tensor gives its place to the carry-through filter; no fine-tuning",
-            "value": world * B * args.steps / (ms_r / 1e3), "unit": "images/s",
+            "value": replicas.job_throughput(world, B, args.steps, ms_r / 1e3), "unit": "images/s",
             "overhead_pct": 100.0 * (ms_r / ms_u - 1.0),
             "overhead_filters_pct": 100.0 * (ms_ri / ms_u - 1.0),
             "reexecuted_images_per_step": n_rerun_r / args.steps,
@@ -379,11 +376,7 @@ def main():
     err = ct.ct_device_error(mp)
 
     def max_over_ranks(v):
-        if dist is not None:
-            t = torch.tensor([v], device="cuda")
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            v = float(t.item())
-        return v
+        return replicas.reduce_max(v, dist, "cuda")
 
     # end to end through the public API from pinned host memory: every step
     # copies its input in (on a copy stream, overlapping the previous step's
@@ -457,8 +450,8 @@ def main():
         return
 
     pk, pk_kind = peaks()
-    value = world * B * args.steps / (ms_p / 1e3)
-    value_u = world * B * args.steps / (ms_u / 1e3)
+    value = replicas.job_throughput(world, B, args.steps, ms_p / 1e3)
+    value_u = replicas.job_throughput(world, B, args.steps, ms_u / 1e3)
     props = torch.cuda.get_device_properties(local)
     # dominant kernel: the convolution family that carries the FLOPs
     tc_n, tc_ms, tc_fl = fam_stats[0]
@@ -537,18 +530,18 @@ def main():
         "overhead_filters_pct": 100.0 * (ms_pi / ms_u - 1.0),
         "overhead_reexec_pct": 100.0 * (ms_p - ms_pi) / ms_u,
         "reexecuted_images_per_step": n_rerun / args.steps,
-        "value_sync_reexec": world * B * args.steps / (ms_ps / 1e3),
+        "value_sync_reexec": replicas.job_throughput(world, B, args.steps, ms_ps / 1e3),
         "overhead_reexec_sync_pct": 100.0 * (ms_ps - ms_pi) / ms_u,
         "reexecuted_images_per_step_sync": n_rerun_s / args.steps,
         "replace_construction": replace_leg,
         "conv_tflop_per_batch": conv_flops(wl) / 1e12,
         "roofline": roof,
         "cpu_baseline": cpu,
-        "e2e": {"value": world * B * args.steps / e2e_s, "unit": "images/s",
+        "e2e": {"value": replicas.job_throughput(world, B, args.steps, e2e_s), "unit": "images/s",
                 "h2d_bytes_per_step": in_bytes, "d2h_bytes_per_step": out_bytes,
                 "api": "ct_infer_reexec; pinned host copies in (copy stream, overlapping the previous "
                        "step) and out (launch stream)"},
-        "e2e_sync_reexec": {"value": world * B * args.steps / e2e_sync_s, "unit": "images/s",
+        "e2e_sync_reexec": {"value": replicas.job_throughput(world, B, args.steps, e2e_sync_s), "unit": "images/s",
                             "api": "ct_run_host (host buffers, synchronous re-execution)"},
         "kernel_families": {nm: {"launches": fam_stats[i][0], "ms": fam_stats[i][1],
                                  "tflop": fam_stats[i][2] / 1e12}
