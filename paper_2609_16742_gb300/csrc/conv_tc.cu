@@ -14,7 +14,9 @@
 //     weight rows in shared memory, and the centre-tap K blocks, which the
 //     K loop visits first, are issued with N = BN + 16: the tensor core
 //     computes the checksum column.  For BN = 256 two spare warps compute it
-//     from the same A tiles with warp-level MMAs against a ones vector.
+//     from the same A tiles with warp-level MMAs against a ones vector
+//     (conv_tc_kernel), or the epilogue adds up the centre-tap pixel's
+//     channels (conv_tc_pair_kernel).
 //   The incoming checksum plane (weight coef at the centre), the residual
 //   checksum and the epilogue (bias, residual, ReLU) are applied by the
 //   epilogue warps.
@@ -30,12 +32,14 @@
 // With N = 256 and no split K, conv_tc_pair_kernel runs the tiles on pairs of
 // CTAs (a cluster of two, tcgen05 cta_group::2): one M = 256 MMA reads the
 // 128 A rows and 128 weight rows each CTA holds, which halves the weight
-// bytes every SM copies and reads per step.
+// bytes every SM copies and reads per step.  Its epilogue sums the
+// carry-through column from the centre-tap input pixel.
 //
 // Warp roles.  conv_tc_kernel: a producer group (producer warps, each owning
 // whole ring slots, plus for N = 256 the two carry-through warps), one MMA
 // warp (one elected lane issues tcgen05.mma), eight epilogue warps;
-// conv_tc_pair_kernel the same, with the MMAs issued by the even CTA.
+// conv_tc_pair_kernel: two producer warps, the MMA warp (issuing in the even
+// CTA only), eight epilogue warps.
 // conv_tc_halo_kernel (320 threads): warp 0 issues TMA, warp 1 the MMAs,
 // warps 2-9 the epilogue.  Each TMEM lane quadrant (32 output pixels) is
 // read by two epilogue warps, each taking half of the tile's channels.
