@@ -256,6 +256,10 @@ def main():
     r, tau = calibrate(mp)
     r_rep, tau_rep = calibrate(mr) if mr is not None else (None, None)
     del xc
+    # every re-execution graph is captured before anything is timed
+    for model_ in (mp, mr):
+        if model_ is not None:
+            ct.ct_reexecute_prepare(model_, B + REEXEC_ROOM)
 
     # evaluation batches for this rank (distinct slices of the seeded set per
     # rank); two, alternating, so that each step's re-run images come from
@@ -525,11 +529,6 @@ def main():
                    "simt_only": bool(args.simt_only)},
         "reexecution": "deferred: each batch's flagged images ride as extra rows of the next batch's "
                        "inference (ct_infer_reexec); the last batch's are re-run at the end of the timed region",
-        "unprotected_value": value_u,
-        "overhead_pct": 100.0 * (ms_p / ms_u - 1.0),
-        "overhead_filters_pct": 100.0 * (ms_pi / ms_u - 1.0),
-        "overhead_reexec_pct": 100.0 * (ms_p - ms_pi) / ms_u,
-        "reexecuted_images_per_step": n_rerun / args.steps,
         "value_sync_reexec": replicas.job_throughput(world, B, args.steps, ms_ps / 1e3),
         "overhead_reexec_sync_pct": 100.0 * (ms_ps - ms_pi) / ms_u,
         "reexecuted_images_per_step_sync": n_rerun_s / args.steps,
@@ -553,6 +552,14 @@ def main():
         "threshold": {"reference": r, "tau": tau},
         "campaign": camp,
     }
+    # the headline figures last, so that a truncated tail of the line keeps them
+    line["reexecuted_images_per_step"] = n_rerun / args.steps
+    line["roofline_frac"] = roof["frac"]
+    line["unprotected_value"] = value_u
+    line["overhead_reexec_pct"] = 100.0 * (ms_p - ms_pi) / ms_u
+    line["overhead_filters_pct"] = 100.0 * (ms_pi / ms_u - 1.0)
+    line["overhead_pct"] = 100.0 * (ms_p / ms_u - 1.0)
+    line["value_images_per_s"] = value
     print(json.dumps(line), flush=True)
     if dist is not None:
         dist.destroy_process_group()

@@ -52,8 +52,10 @@ typedef enum { CT_OP_CONV = 0, CT_OP_MAXPOOL = 1, CT_OP_GAP = 2, CT_OP_FC = 3 } 
  *                paragraph);
  *   CT_ROLE_PASS a 1x1 downsample shortcut: its checksum output is the
  *                incoming checksum at the sampled position (or nothing when
- *                the model is built with CT_DS_ZERO). */
-typedef enum { CT_ROLE_CT = 0, CT_ROLE_NONE = 1, CT_ROLE_PASS = 2 } ct_role;
+ *                the model is built with CT_DS_ZERO);
+ *   CT_ROLE_AUTO derived from the network graph by the residual rule (see
+ *                ct_resolve_roles). */
+typedef enum { CT_ROLE_CT = 0, CT_ROLE_NONE = 1, CT_ROLE_PASS = 2, CT_ROLE_AUTO = 3 } ct_role;
 
 typedef enum { CT_BUF_WEIGHT = 0, CT_BUF_ACT = 1 } ct_buf_kind;
 
@@ -144,6 +146,21 @@ typedef struct {
 
 typedef struct ct_model ct_model;
 
+/* ct_resolve_roles -- Sec. II-A residual rule, host only (no device is
+ * touched).  A convolution whose input tensor is also read by another layer
+ * (as the `src` of another layer or as a `res` operand: the shortcut of a
+ * residual block) must not carry a carry-through filter: that tensor's
+ * checksum already reaches the block's residual add along the shortcut, and
+ * a filter on the other path would count it twice.  roles[i] (one per layer,
+ * written for every layer) receives the effective role of convolution i, -1
+ * for other layers.  CT_ROLE_AUTO resolves to CT_ROLE_CT for a convolution
+ * whose input has no other reader; otherwise to CT_ROLE_PASS when its
+ * output goes to nothing but a residual add (the shortcut), else to
+ * CT_ROLE_NONE.  Explicit roles are kept.
+ * Errors: CT_EINVAL for a malformed description or a CT_ROLE_CT
+ * convolution that the rule forbids. */
+ct_status ct_resolve_roles(const ct_model_desc *desc, int32_t *roles);
+
 /* ct_build -- Sec. II-A/II-B construction.  Folds BatchNorm (Eq. 1) into the
  * convolutions in double precision with the identity (scale exactly 1, bias
  * 0) on every checksum channel; appends a carry-through filter to every
@@ -155,9 +172,12 @@ typedef struct ct_model ct_model;
  * 4 channels with 64 filters, followed by a 3x3 stride-2 padding-1 max-pool
  * that is its only reader, runs as one fused kernel: the FP16 copy of the
  * image and the unpooled convolution output are then never stored.
+ * Roles are resolved and checked by the rule of ct_resolve_roles first,
+ * before any device is touched.
  * Synchronous.  On success *out owns device memory until ct_destroy.
- * Errors: CT_EINVAL (malformed description), CT_EUNSUPPORTED, CT_ENOMEM,
- * CT_ECUDA.  Nothing is allocated on failure. */
+ * Errors: CT_EINVAL (malformed description, or a carry-through filter that
+ * the residual rule forbids), CT_EUNSUPPORTED, CT_ENOMEM, CT_ECUDA.  Nothing
+ * is allocated on failure. */
 ct_status ct_build(const ct_model_desc *desc, const float *const *weights,
                    const ct_build_opts *opts, ct_model **out);
 
@@ -202,17 +222,26 @@ ct_status ct_clear_faults(ct_model *m);
  * logits_dev and S_dev (the re-run's own flags are ignored; flag_dev is not
  * modified).  Synchronises `stream` once to read the flags.  *n_rerun
  * (host) receives the number of images re-run.  Same buffers as ct_infer.
- * The re-run batch is padded to the next power of two by repeating the
- * last flagged image.  Its inference is captured into a CUDA graph on a
- * model-owned stream the first time that padded size occurs (that call is
- * slower) and replayed afterwards; with profiling on (ct_profile_enable) the
- * kernels are launched one by one instead.  A re-run row equals a fault-free
+ * The re-run batch is padded to the next power of two (or to max_batch when
+ * that is smaller) by repeating the last flagged image.  Its inference is
+ * captured into a CUDA graph on a model-owned stream the first time that
+ * padded size occurs (that call is slower; ct_reexecute_prepare captures
+ * them ahead of time) and replayed afterwards; with profiling on
+ * (ct_profile_enable) the kernels are launched one by one instead.  A re-run row equals a fault-free
  * ct_infer of the padded batch; because small batches split K differently,
  * it can differ from the same image's row of a full batch by summation
  * order.  An armed fault stays armed for the next ct_infer. */
 ct_status ct_reexecute(ct_model *m, const float *input_dev, int32_t batch,
                        const uint8_t *flag_dev, float *logits_dev, float *S_dev,
                        int32_t *n_rerun, void *stream);
+
+/* ct_reexecute_prepare -- captures, ahead of time, the re-execution graphs
+ * ct_reexecute replays (Sec. II-B mitigation): one per padded re-run size
+ * (1, 2, 4, ... up to the first power of two >= max_images, capped at
+ * max_batch), so that no later ct_reexecute pays a capture.  Synchronous;
+ * launches nothing.  Errors: CT_EINVAL (null model), CT_ERANGE (max_images
+ * outside 1..max_batch), CT_ECUDA (capture or instantiation failed). */
+ct_status ct_reexecute_prepare(ct_model *m, int32_t max_images);
 
 /* ct_infer_reexec -- ct_infer of `batch` new images (input_dev, logits_dev,
  * S_dev, flag_dev as for ct_infer) that also carries out the Sec. II-B
@@ -297,9 +326,12 @@ ct_status ct_campaign_batched(ct_model *m, const float *input_dev, int32_t batch
  *     4*n (indices), 4*n*in_c*in_h*in_w (images), 4*n*n_classes (logits),
  *     4*n (S) and n (flags) bytes for n flagged images.  If it does not,
  *     or batch > 65536, the call returns CT_ERANGE and runs nothing.
- *   - The first call on a device looks up the array's device address
- *     (cudaGetSymbolAddress) with that device current; make that first
- *     call before any stream capture.
+ *   - ct_build looks up the array's device address (cudaGetSymbolAddress)
+ *     with the model's device current.  That lookup loads the array's
+ *     module, which commits its CT_NOALLOC_SCRATCH_BYTES on the device, so
+ *     the memory is taken when a model is built, never by this call.
+ *   - *n_rerun is the number of images re-run: 0 when the call returns
+ *     CT_ERANGE (nothing ran).
  *   - Every call on a device shares the one array and it keeps the last
  *     call's contents; calls that can overlap on the GPU race on it, so
  *     serialise them (one stream, or a wait between streams).  Host-side

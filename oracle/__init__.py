@@ -529,6 +529,40 @@ def _maybe_flip_act(y: np.ndarray, slot: int, target_slot: int, fault: Fault, n:
     return y
 
 
+def residual_roles(layers: Sequence[synth.Layer]) -> List[Optional[str]]:
+    """Sec. II-A, residual networks: the role of each convolution that the
+    network graph fixes (None for other layers).
+
+    A tensor read by two layers reaches a later residual add along two paths
+    (the block's main path and its shortcut), and its checksum arrives along
+    the shortcut already.  So a convolution reading such a tensor gets no
+    carry-through filter ("none"), or the checksum would be accumulated
+    twice -- unless it is the shortcut itself: a convolution whose output
+    goes to nothing but a residual add passes the checksum through ("pass").
+    A depthwise convolution passes its incoming checksum through as well
+    (its checksum group sees only the checksum channel); every other
+    convolution carries a carry-through filter ("ct").
+    """
+    uses: Dict[int, int] = {}
+    added: set = set()
+    for L in layers:
+        uses[L.src] = uses.get(L.src, 0) + 1
+        if L.res >= 0:
+            uses[L.res] = uses.get(L.res, 0) + 1
+            added.add(L.res)
+    out: List[Optional[str]] = []
+    for L in layers:
+        if L.op != "conv":
+            out.append(None)
+        elif uses[L.src] > 1:
+            out.append("pass" if L.dst in added and uses[L.dst] == 1 else "none")
+        elif L.groups > 1:
+            out.append("pass")
+        else:
+            out.append("ct")
+    return out
+
+
 def top1(logits: np.ndarray) -> np.ndarray:
     """Top-1 class per row; ties go to the lowest index; any NaN gives -1."""
     logits = np.asarray(logits, dtype=np.float64)

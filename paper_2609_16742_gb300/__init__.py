@@ -22,7 +22,7 @@ LIB_PATH = os.path.join(_HERE, "_lib", "libct.so")
 
 CT_FP32, CT_FP16 = 0, 1
 CT_OP_CONV, CT_OP_MAXPOOL, CT_OP_GAP, CT_OP_FC = 0, 1, 2, 3
-CT_ROLE_CT, CT_ROLE_NONE, CT_ROLE_PASS = 0, 1, 2
+CT_ROLE_CT, CT_ROLE_NONE, CT_ROLE_PASS, CT_ROLE_AUTO = 0, 1, 2, 3
 CT_BUF_WEIGHT, CT_BUF_ACT = 0, 1
 CT_DS_PASS, CT_DS_ZERO = 0, 1
 CT_PROTECT_NONE, CT_PROTECT_WIDEN, CT_PROTECT_REPLACE = 0, 1, 2
@@ -38,7 +38,8 @@ EXPORTS = ["ct_build", "ct_set_threshold", "ct_get_threshold", "ct_infer", "ct_i
            "ct_buffer_info", "ct_profile_enable", "ct_profile_read", "ct_launches_per_infer", "ct_kernel_count",
            "ct_fi_threshold",
            "ct_copy_activation", "ct_device_error", "ct_destroy", "ct_strerror",
-           "ct_reexecute_noalloc", "ct_campaign_batched"]
+           "ct_reexecute_noalloc", "ct_campaign_batched", "ct_resolve_roles",
+           "ct_reexecute_prepare"]
 
 CT_NOALLOC_SCRATCH_BYTES = 16 * 1024 * 1024
 
@@ -107,6 +108,8 @@ def lib():
             "ct_copy_activation": [vp, i32, i32, vp, vp, P(i32), P(i32), P(i32), P(i32), P(i32), vp],
             "ct_device_error": [vp, P(ctypes.c_uint32)],
             "ct_campaign_batched": [vp, vp, i32, P(FaultDesc), i32, vp, vp, vp, vp],
+            "ct_resolve_roles": [P(ModelDesc), P(i32)],
+            "ct_reexecute_prepare": [vp, i32],
         }
         for name, args in sig.items():
             f = getattr(L, name)
@@ -153,7 +156,8 @@ def _stream(stream) -> Optional[int]:
 
 
 _OPS = {"conv": CT_OP_CONV, "maxpool": CT_OP_MAXPOOL, "gap": CT_OP_GAP, "fc": CT_OP_FC}
-_ROLES = {"ct": CT_ROLE_CT, "none": CT_ROLE_NONE, "pass": CT_ROLE_PASS}
+_ROLES = {"ct": CT_ROLE_CT, "none": CT_ROLE_NONE, "pass": CT_ROLE_PASS, "auto": CT_ROLE_AUTO}
+_ROLE_NAMES = {v: k for k, v in _ROLES.items()}
 
 
 class Model:
@@ -180,6 +184,27 @@ class Model:
             pass
 
 
+def _layer_descs(layers: Sequence):
+    n = len(layers)
+    arr = (LayerDesc * n)()
+    for i, L in enumerate(layers):
+        arr[i] = LayerDesc(_OPS[L.op], L.src, L.dst, L.res, L.cin, L.cout, L.k, L.stride, L.pad,
+                           _ROLES.get(L.ct, CT_ROLE_NONE), int(L.bn), int(L.relu), int(L.final),
+                           int(L.ct_shift), int(getattr(L, "groups", 1)))
+    return arr
+
+
+def ct_resolve_roles(layers: Sequence, in_shape, n_classes: int) -> List[Optional[str]]:
+    """Sec. II-A residual rule as the library applies it: the effective role
+    of every convolution ("ct", "none", "pass"; "auto" resolved), None for
+    other layers.  Raises CtError (CT_EINVAL) when a "ct" role breaks the rule."""
+    arr = _layer_descs(layers)
+    desc = ModelDesc(len(layers), arr, in_shape[0], in_shape[1], in_shape[2], n_classes, 1e-5)
+    out = (ctypes.c_int32 * len(layers))()
+    _check(lib().ct_resolve_roles(ctypes.byref(desc), out), "ct_resolve_roles")
+    return [None if r < 0 else _ROLE_NAMES[r] for r in out]
+
+
 def ct_build(layers: Sequence, params: Sequence[dict], in_shape, n_classes: int,
              precision: str = "fp32", protect: bool = True, ds_mode: str = "pass",
              device: int = 0, max_batch: int = 64, simt_only: bool = False,
@@ -189,13 +214,10 @@ def ct_build(layers: Sequence, params: Sequence[dict], in_shape, n_classes: int,
     protect=True adds the carry-through filters as extra channels (widened);
     replace=True builds the paper's prune-and-replace construction instead."""
     n = len(layers)
-    arr = (LayerDesc * n)()
+    arr = _layer_descs(layers)
     keep = []
     wp = (ctypes.c_void_p * (6 * n))()
     for i, (L, p) in enumerate(zip(layers, params)):
-        arr[i] = LayerDesc(_OPS[L.op], L.src, L.dst, L.res, L.cin, L.cout, L.k, L.stride, L.pad,
-                           _ROLES.get(L.ct, CT_ROLE_NONE), int(L.bn), int(L.relu), int(L.final),
-                           int(L.ct_shift), int(getattr(L, "groups", 1)))
         for j, key in enumerate(("w", "b", "gamma", "beta", "mean", "var")):
             if key in p:
                 a = np.ascontiguousarray(p[key], dtype=np.float32)
@@ -250,6 +272,11 @@ def ct_reexecute(m: Model, input_dev, batch: int, flag_dev, logits_dev, S_dev=No
     _check(lib().ct_reexecute(m.handle, _ptr(input_dev), batch, _ptr(flag_dev), _ptr(logits_dev),
                               _ptr(S_dev), ctypes.byref(n), _stream(stream)), "ct_reexecute")
     return n.value
+
+
+def ct_reexecute_prepare(m: Model, max_images: int):
+    """Capture the re-execution graphs of every padded size up to max_images."""
+    _check(lib().ct_reexecute_prepare(m.handle, max_images), "ct_reexecute_prepare")
 
 
 def ct_infer_reexec(m: Model, input_dev, batch: int, logits_dev, S_dev=None, flag_dev=None,

@@ -159,20 +159,9 @@ def run(precision="fp32", faults=1000, seed=0, batch=None, calib_images=10000, a
     ct.ct_infer(m, x, B, logits, S, flag, stream)
     golden = top1(logits).clone()
     ff_flags = int(flag.sum().item())
-    # fault-free step time (infer + re-execution of its flags) for the relative cost
-    for _ in range(3):
-        ct.ct_infer(m, x, B, logits, S, flag, stream)
-        ct.ct_reexecute(m, x, B, flag, logits, S, stream)
-    torch.cuda.synchronize()
-    t0 = time.perf_counter()
-    n_ff = 20
-    for _ in range(n_ff):
-        ct.ct_infer(m, x, B, logits, S, flag, stream)
-        ct.ct_reexecute(m, x, B, flag, logits, S, stream)
-    torch.cuda.synchronize()
-    ff_step_s = (time.perf_counter() - t0) / n_ff
+    # every re-execution graph is captured before anything is timed
+    ct.ct_reexecute_prepare(m, B)
 
-    # ---- campaign ----
     bufs = ct.ct_buffers(m, B)
     sites = synth.draw_faults(bufs, faults, seed)
     per_img = {}
@@ -182,12 +171,13 @@ def run(precision="fp32", faults=1000, seed=0, batch=None, calib_images=10000, a
     nb = 32 if precision == "fp32" else 16
     # [kind, bit] counters on the GPU: trials, critical, detected, false alarms
     cnt = torch.zeros(2, nb, 4, dtype=torch.long, device="cuda")
-    n_rerun = 0
-    ct.ct_kernel_count(m)
-    torch.cuda.synchronize()
-    t0 = time.perf_counter()
-    for kind, layer, e, bit in sites.tolist():
-        ct.ct_inject(m, kind, layer, e, bit)
+    scratch = torch.zeros_like(cnt)
+
+    def trial(kind, layer, e, bit, counters, inject=True):
+        """One inference of the batch (with the fault armed when inject),
+        the per-image bookkeeping, and the re-execution of its flagged images."""
+        if inject:
+            ct.ct_inject(m, kind, layer, e, bit)
         ct.ct_infer(m, x, B, logits, S, flag, stream)
         crit = top1(logits) != golden
         fl = flag != 0
@@ -199,9 +189,29 @@ def run(precision="fp32", faults=1000, seed=0, batch=None, calib_images=10000, a
             c, f = crit[i], fl[i]
             row = torch.stack([torch.ones_like(c, dtype=torch.long), c.long(), (c & f).long(),
                                (~c & f).long()])
-        cnt[kind, bit] += row
-        if reexecute:
-            n_rerun += ct.ct_reexecute(m, x, B, flag, logits, S, stream)
+        counters[kind, bit] += row
+        return ct.ct_reexecute(m, x, B, flag, logits, S, stream) if reexecute else 0
+
+    # fault-free time of the same steps (the same bookkeeping and re-execution,
+    # no fault armed) for the relative cost
+    n_ff = min(200, max(20, faults // 50))
+    ff_sites = sites[np.arange(n_ff) % len(sites)].tolist()
+    for kind, layer, e, bit in ff_sites[:5]:
+        trial(kind, layer, e, bit, scratch, inject=False)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for kind, layer, e, bit in ff_sites:
+        trial(kind, layer, e, bit, scratch, inject=False)
+    torch.cuda.synchronize()
+    ff_step_s = (time.perf_counter() - t0) / n_ff
+
+    # ---- campaign ----
+    n_rerun = 0
+    ct.ct_kernel_count(m)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for kind, layer, e, bit in sites.tolist():
+        n_rerun += trial(kind, layer, e, bit, cnt)
     torch.cuda.synchronize()
     wall = time.perf_counter() - t0
     kernels = ct.ct_kernel_count(m)

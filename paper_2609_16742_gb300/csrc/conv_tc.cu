@@ -75,7 +75,6 @@ constexpr int tc_nprod(int BN, int STAGES) {
 }
 constexpr int tc_npg(int BN, int STAGES) { return BN > 128 ? 4 : tc_nprod(BN, STAGES); }
 constexpr int tc_threads(int BN, int STAGES) { return 32 * (tc_npg(BN, STAGES) + 1 + N_EPI_WARPS); }
-constexpr int TC_CS = 4;           // CTAs per cluster sharing each B tile (N = 128, 256)
 
 enum CtMode { CT_NONE_ = 0, CT_MERGED = 1, CT_SEPARATE = 2 };
 
@@ -86,23 +85,19 @@ struct TcGeom {
     int tmem_cols;
     int m_tiles, n_tiles;
     int splits, kps, ws_ld;      // split-K: K blocks per split, workspace row length
-    int m_groups;                // clusters of CS consecutive M tiles (CS = 1: m_tiles)
     uint16_t coef_h;
 };
 
 // K-block range [lo, hi) and output tile of persistent work item `item`.
-// A work item of a cluster of cs CTAs is a group of cs consecutive M tiles
-// with the same N tile and K range; CTA `crank` of the cluster takes M tile
-// group * cs + crank (past the last M tile it computes rows it never stores).
 struct TileRef {
     int m0, n_tile, sp, kb_lo, kb_hi;
 };
-__device__ __forceinline__ TileRef tile_ref(int item, const TcGeom &g, int cs, int crank) {
+__device__ __forceinline__ TileRef tile_ref(int item, const TcGeom &g) {
     TileRef t;
-    const int per = g.m_groups * g.n_tiles;
+    const int per = g.m_tiles * g.n_tiles;
     t.sp = item / per;
     const int rt = item - t.sp * per;
-    t.m0 = ((rt / g.n_tiles) * cs + crank) * BM;
+    t.m0 = (rt / g.n_tiles) * BM;
     t.n_tile = rt % g.n_tiles;
     t.kb_lo = t.sp * g.kps;
     t.kb_hi = min(g.n_kb, t.kb_lo + g.kps);
@@ -250,7 +245,7 @@ __device__ __forceinline__ void store_checksum_pre(float ctv, const CsIn &c, con
 // barrier round trip).  A single TMEM buffer holds the chains; for
 // BN <= 128 the epilogue copies it to registers and releases it before its
 // global stores, so the next tile's MMAs overlap the stores.
-template <int BN, int STAGES, int SUB, int NCH, int CS>
+template <int BN, int STAGES, int SUB, int NCH>
 __global__ void __launch_bounds__(tc_threads(BN, STAGES), 1)
 conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
                const ConvArgs a, const TcGeom g) {
@@ -265,7 +260,6 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
     // that do not issue copies (they consume every stage, like the MMA warp),
     // and the epilogue of one tile overlaps the MMAs of the next
     constexpr bool DBUF = !EARLY;
-    static_assert(!DBUF || CS == 1, "the carry-through warps release stages of their own CTA only");
     // producer warps (each owns whole ring slots) and carry-through warps
     constexpr int NPROD = tc_nprod(BN, STAGES);
     constexpr int NPG = tc_npg(BN, STAGES);               // producer group: producers + carry-through warps
@@ -290,17 +284,13 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
     volatile uint32_t *abort_flag = tmem_holder + 1;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    // clusters of CS CTAs share each B tile: CTA r loads rows r * BN / CS ..
-    // of it and multicasts them to the whole cluster
-    const int crank = CS > 1 ? (int)cluster_ctarank() : 0;
-    const int cid = blockIdx.x / CS, ncl = gridDim.x / CS;
-    const uint16_t cmask = (uint16_t)((1u << CS) - 1u);
-    const int num_items = g.m_groups * g.n_tiles * g.splits;
+    const int cid = blockIdx.x, ncl = gridDim.x;
+    const int num_items = g.m_tiles * g.n_tiles * g.splits;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(smem_u32(&full[s]), 1);
-            mbar_init(smem_u32(&empty[s]), CS + NCT);   // MMA commits (every CTA) + carry-through warps
+            mbar_init(smem_u32(&empty[s]), 1 + NCT);   // MMA commit + carry-through warps
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(smem_u32(&acc_full[b]), 1);
@@ -329,9 +319,6 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
     }
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
-    // peers multicast into this CTA's shared memory and barriers only after
-    // every CTA of the cluster has initialised its barriers
-    if (CS > 1) cluster_sync();
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem = *tmem_holder;
     // the previous kernel's outputs (and any fault flip) are visible from here
@@ -353,7 +340,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
         int it = 0;
         for (int tile = cid; tile < num_items; tile += ncl) {
             if (__any_sync(0xffffffffu, *abort_flag)) break;
-            const TileRef tr = tile_ref(tile, g, CS, crank);
+            const TileRef tr = tile_ref(tile, g);
             const int m0 = tr.m0, n_tile = tr.n_tile;
             const int nimg = m0 / g.PQ, rem = m0 % g.PQ;
             const int p = rem / g.Q, q = rem % g.Q;
@@ -375,12 +362,8 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
                         const int r = tap / g.S, sx = tap % g.S;
                         tma_load_im2col(smem_u32(As + (s * SUB + j) * A_BYTES), &amap, fb, c0, w0, h0, nimg,
                                         (uint16_t)sx, (uint16_t)r);
-                        if (CS == 1)
-                            tma_load_2d(smem_u32(Bs + (s * SUB + j) * B_SUB_BYTES), &bmap, fb, tap * g.C + c0,
-                                        n_tile * BN);
-                        else
-                            tma_load_2d_mc(smem_u32(Bs + (s * SUB + j) * B_SUB_BYTES + crank * (BN / CS) * BK * 2),
-                                           &bmap, fb, tap * g.C + c0, n_tile * BN + crank * (BN / CS), cmask);
+                        tma_load_2d(smem_u32(Bs + (s * SUB + j) * B_SUB_BYTES), &bmap, fb, tap * g.C + c0,
+                                    n_tile * BN);
                     }
                 }
                 __syncwarp();
@@ -396,7 +379,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
         int it = 0, lt = 0;
         for (int tile = cid; tile < num_items; tile += ncl, ++lt) {
             if (__any_sync(0xffffffffu, *abort_flag)) break;
-            const TileRef tr = tile_ref(tile, g, CS, crank);
+            const TileRef tr = tile_ref(tile, g);
             const int n_tile = tr.n_tile;
             const bool ct_here = g.ct_mode != CT_NONE_ && n_tile == 0;
             const int ab = DBUF ? (lt & 1) : 0;
@@ -440,10 +423,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
                     }
                 }
                 __syncwarp();
-                if (elect_one()) {
-                    if (CS == 1) umma_commit(smem_u32(&empty[s]));
-                    else umma_commit_mc(smem_u32(&empty[s]), cmask);
-                }
+                if (elect_one()) umma_commit(smem_u32(&empty[s]));
                 __syncwarp();
             }
             if (!ok) { if (lane == 0) *abort_flag = 1; break; }
@@ -471,7 +451,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
             bool ok = true;
             for (int tile = cid; tile < num_items && ok; tile += ncl, ++lt) {
                 if (__any_sync(0xffffffffu, *abort_flag)) break;
-                const TileRef tr = tile_ref(tile, g, CS, crank);
+                const TileRef tr = tile_ref(tile, g);
                 const bool ct_here = g.ct_mode != CT_NONE_ && tr.n_tile == 0;
                 const int ab = lt & 1;
                 float acc[MT][4];
@@ -531,7 +511,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
         const bool split = g.splits > 1;
         int lt = 0;
         for (int tile = cid; tile < num_items; tile += ncl, ++lt) {
-            const TileRef tr = tile_ref(tile, g, CS, crank);
+            const TileRef tr = tile_ref(tile, g);
             const int m0 = tr.m0, n_tile = tr.n_tile;
             // residual loads in flight while the MMAs run
             Res16 rs[BN / 32];
@@ -637,12 +617,6 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
     }
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
-    if (CS > 1) {
-        // the MMAs of this CTA have completed (the epilogue saw every tile);
-        // their commits may still arrive on the peers' barriers: no CTA
-        // leaves before the whole cluster is done
-        cluster_sync();
-    }
     if (warp == TC_MMA_WARP) {
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)g.tmem_cols));
@@ -1559,10 +1533,8 @@ int device_sm_count() {
 struct TcPlan {
     CUtensorMap amap;
     CUtensorMap bmap;
-    CUtensorMap bmap_mc;         // B slices of BN / cs rows for the cluster kernels
     TcGeom g;
     int BN, n_tiles, sms;
-    int cs, max_clusters;        // cluster size of the multicast variant (1: none)
     size_t smem;
     CUtensorMap bmap_pair;       // N = 256 over CTA pairs: 128-row weight halves
     int pair_clusters;           // resident CTA pairs (0: no pair variant)
@@ -1619,15 +1591,13 @@ TcPlan *tc_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, cons
     cudaError_t e;
     if (pl->BN == 64) {
         pl->smem = smem_bytes<64, 4, 2>();
-        e = cudaFuncSetAttribute(conv_tc_kernel<64, 4, 2, 4, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
+        e = cudaFuncSetAttribute(conv_tc_kernel<64, 4, 2, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
     } else if (pl->BN == 128) {
         pl->smem = smem_bytes<128, 3, 2>();
-        e = cudaFuncSetAttribute(conv_tc_kernel<128, 3, 2, 2, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
-        if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(conv_tc_kernel<128, 3, 2, 2, TC_CS>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
+        e = cudaFuncSetAttribute(conv_tc_kernel<128, 3, 2, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
     } else {
         pl->smem = smem_bytes<256, 4, 1>();
-        e = cudaFuncSetAttribute(conv_tc_kernel<256, 4, 1, 1, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
+        e = cudaFuncSetAttribute(conv_tc_kernel<256, 4, 1, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
     }
     if (e != cudaSuccess) { if (why) *why = "shared memory attribute"; delete pl; return nullptr; }
     // N = 256 over CTA pairs (cta_group::2): each CTA copies 128 of the 256 weight rows
@@ -1658,33 +1628,6 @@ TcPlan *tc_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, cons
         }
         cudaGetLastError();
     }
-    // cluster variant: B slices of BN / TC_CS rows multicast to TC_CS CTAs
-    pl->cs = 1;
-    pl->max_clusters = 0;
-    if (pl->BN == 128) {
-        cuuint32_t box_mc[2] = {BK, (cuuint32_t)(pl->BN / TC_CS)};
-        r = g_encode_tiled(&pl->bmap_mc, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void *>(w_dev), bdim, bstr,
-                           box_mc, bes, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-        cudaLaunchConfig_t cfg = {};
-        cfg.gridDim = dim3(TC_CS * 64);
-        cfg.blockDim = dim3(tc_threads(128, 3));
-        cfg.dynamicSmemBytes = pl->smem;
-        cudaLaunchAttribute at[1];
-        at[0].id = cudaLaunchAttributeClusterDimension;
-        at[0].val.clusterDim.x = TC_CS;
-        at[0].val.clusterDim.y = 1;
-        at[0].val.clusterDim.z = 1;
-        cfg.attrs = at;
-        cfg.numAttrs = 1;
-        int n = 0;
-        cudaError_t oe = cudaOccupancyMaxActiveClusters(&n, conv_tc_kernel<128, 3, 2, 2, TC_CS>, &cfg);
-        if (r == CUDA_SUCCESS && oe == cudaSuccess && n > 0) {
-            pl->cs = TC_CS;
-            pl->max_clusters = n;
-        }
-        cudaGetLastError();
-    }
     return pl;
 }
 
@@ -1700,29 +1643,18 @@ cudaError_t launch_conv_tc(const ConvArgs &a, const void *plan, cudaStream_t st,
     g.ws_ld = (g.K + 1 + 3) & ~3;
     g.splits = (a.K % 8 == 0) ? splitk_choose(tiles, g.n_kb, 4, pl->sms / 2, g.M, g.ws_ld, a.ws ? a.ws_bytes : 0) : 1;
     g.kps = (g.n_kb + g.splits - 1) / g.splits;
-    g.m_groups = g.m_tiles;
     if (pl->pair_clusters > 0 && g.splits == 1 && g.m_tiles >= 2) {
         // N = 256 tiles over CTA pairs: 256 pixels x 256 channels per pair
         const int items = ((g.m_tiles + 1) / 2) * g.n_tiles;
         const int ncl = items < pl->pair_clusters ? items : pl->pair_clusters;
         pdl_launch_cluster(conv_tc_pair_kernel, dim3(2 * ncl), PR_THREADS, pl->pair_smem, st, 2, pl->amap,
                            pl->bmap_pair, a, g);
-    } else if (pl->cs > 1 && g.splits == 1 && g.m_tiles >= 4 * pl->cs && g.n_kb >= 4) {
-        // clusters of cs CTAs on groups of cs consecutive M tiles, sharing B
-        // (not for a few K blocks per tile: little B to share, and the
-        // cluster's CTAs advance in lockstep)
-        g.m_groups = (g.m_tiles + pl->cs - 1) / pl->cs;
-        const int items = g.m_groups * g.n_tiles;
-        const int ncl = items < pl->max_clusters ? items : pl->max_clusters;
-        dim3 grid(ncl * pl->cs);
-        pdl_launch_cluster(conv_tc_kernel<128, 3, 2, 2, TC_CS>, grid, tc_threads(128, 3), pl->smem, st, TC_CS, pl->amap,
-                           pl->bmap_mc, a, g);
     } else {
         const int items = tiles * g.splits;
         dim3 grid(items < pl->sms ? items : pl->sms);
-        if (pl->BN == 64) pdl_launch(conv_tc_kernel<64, 4, 2, 4, 1>, grid, tc_threads(64, 4), pl->smem, st, pl->amap, pl->bmap, a, g);
-        else if (pl->BN == 128) pdl_launch(conv_tc_kernel<128, 3, 2, 2, 1>, grid, tc_threads(128, 3), pl->smem, st, pl->amap, pl->bmap, a, g);
-        else pdl_launch(conv_tc_kernel<256, 4, 1, 1, 1>, grid, tc_threads(256, 4), pl->smem, st, pl->amap, pl->bmap, a, g);
+        if (pl->BN == 64) pdl_launch(conv_tc_kernel<64, 4, 2, 4>, grid, tc_threads(64, 4), pl->smem, st, pl->amap, pl->bmap, a, g);
+        else if (pl->BN == 128) pdl_launch(conv_tc_kernel<128, 3, 2, 2>, grid, tc_threads(128, 3), pl->smem, st, pl->amap, pl->bmap, a, g);
+        else pdl_launch(conv_tc_kernel<256, 4, 1, 1>, grid, tc_threads(256, 4), pl->smem, st, pl->amap, pl->bmap, a, g);
     }
     cudaError_t e = cudaGetLastError();
     if (n_kernels) *n_kernels = 1;

@@ -362,6 +362,44 @@ std::vector<int> replace_prune_index(const ct_model_desc *desc, const float *con
     return out;
 }
 
+// Sec. II-A, residual networks: a convolution whose input tensor is also
+// read by another layer (the shortcut of a residual block) gets no
+// carry-through filter, because that tensor's checksum already reaches the
+// block's residual add along the shortcut; a filter on the other path would
+// add it a second time.  Resolves CT_ROLE_AUTO per convolution into roles[i]
+// (one whose input has another reader: the shortcut, PASS, if its output
+// goes to nothing but a residual add, else NONE; otherwise CT) and rejects
+// an explicit CT_ROLE_CT that the rule forbids.  roles[i] is -1 for layers
+// that are not convolutions.
+ct_status resolve_roles(const ct_model_desc *desc, int32_t *roles) {
+    const int nL = desc->n_layers;
+    int max_slot = 0;
+    for (int i = 0; i < nL; ++i) {
+        const ct_layer_desc &d = desc->layers[i];
+        if (d.src < 0 || d.dst <= 0 || d.res < -1) return CT_EINVAL;
+        max_slot = std::max(max_slot, std::max(std::max(d.dst, d.src), d.res));
+    }
+    std::vector<int> readers(max_slot + 1, 0), is_res(max_slot + 1, 0);
+    for (int i = 0; i < nL; ++i) {
+        const ct_layer_desc &d = desc->layers[i];
+        ++readers[d.src];
+        if (d.res >= 0) { ++readers[d.res]; is_res[d.res] = 1; }
+    }
+    for (int i = 0; i < nL; ++i) {
+        const ct_layer_desc &d = desc->layers[i];
+        roles[i] = -1;
+        if (d.op != CT_OP_CONV) continue;
+        const bool shared_input = readers[d.src] > 1;
+        int r = d.role;
+        if (r == CT_ROLE_AUTO)
+            r = !shared_input ? CT_ROLE_CT : (is_res[d.dst] && readers[d.dst] == 1) ? CT_ROLE_PASS : CT_ROLE_NONE;
+        if (r < CT_ROLE_CT || r > CT_ROLE_PASS) return CT_EINVAL;
+        if (r == CT_ROLE_CT && shared_input) return CT_EINVAL;
+        roles[i] = r;
+    }
+    return CT_OK;
+}
+
 ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const *wts) {
     const int nL = desc->n_layers;
     int max_slot = 0;
@@ -387,6 +425,8 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
             if (desc->layers[i].op == CT_OP_CONV && desc->layers[i].groups > 1) return CT_EUNSUPPORTED;
     const std::vector<int> pj = m->replace ? replace_prune_index(desc, wts, max_slot + 1)
                                            : std::vector<int>(max_slot + 1, -1);
+    std::vector<int32_t> roles(nL);
+    if (resolve_roles(desc, roles.data()) != CT_OK) return CT_EINVAL;
 
     for (int i = 0; i < nL; ++i) {
         const ct_layer_desc &d = desc->layers[i];
@@ -396,6 +436,7 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
         Slot &dst = m->slots[d.dst];
         LayerRT l;
         l.d = d;
+        if (d.op == CT_OP_CONV) l.d.role = roles[i];
         const float *W = wts[CT_WEIGHTS_PER_LAYER * i + 0];
         const float *bias = wts[CT_WEIGHTS_PER_LAYER * i + 1];
         if (d.op == CT_OP_CONV) {
@@ -405,7 +446,7 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
             l.dw = groups > 1;
             if (l.dw && (groups != d.cin || groups != d.cout || m->replace || !dw_supported(d.cin, d.cout, prec == CT_FP16)))
                 return CT_EUNSUPPORTED;
-            int role = m->protect ? d.role : CT_ROLE_NONE;
+            int role = m->protect ? l.d.role : CT_ROLE_NONE;
             if (role == CT_ROLE_PASS && m->ds_mode == CT_DS_ZERO && !l.dw) role = CT_ROLE_NONE;
             if (role < CT_ROLE_CT || role > CT_ROLE_PASS) return CT_EINVAL;
             // depthwise: the checksum group passes the incoming checksum through
@@ -468,8 +509,8 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
                 const int kk = l.K - 1;
                 for (int cc = 0; cc < l.C; ++cc) {
                     double v = 0.0;
-                    if (d.role == CT_ROLE_CT) v = l.coef;
-                    else if (d.role == CT_ROLE_PASS && m->ds_mode == CT_DS_PASS && cc == l.C - 1 && ji >= 0) v = 1.0;
+                    if (l.d.role == CT_ROLE_CT) v = l.coef;
+                    else if (l.d.role == CT_ROLE_PASS && m->ds_mode == CT_DS_PASS && cc == l.C - 1 && ji >= 0) v = 1.0;
                     if (v != 0.0) put(hw, (size_t)weight_word(l, kk, ctr, ctr, cc), v, prec);
                 }
             }
@@ -870,11 +911,13 @@ ct_status reexec_impl(ct_model *m, const float *input, int batch, const uint8_t 
         if (m->h_flags[i]) m->h_idx[n++] = i;
     if (n_rerun) *n_rerun = n;
     if (n == 0) return CT_OK;
-    // the re-run batch is padded to a power of two by repeating the last
-    // flagged image; only the first n rows are scattered back
+    // the re-run batch is padded to a power of two (at most max_batch) by
+    // repeating the last flagged image; only the first n rows are scattered
+    // back.  Each bucket size has its own graph slot (ceil log2), and
+    // max_batch is the only size in the last slot.
     int bucket = 1;
     while (bucket < n) bucket <<= 1;
-    if (bucket > m->max_batch) bucket = n;
+    if (bucket > m->max_batch) bucket = m->max_batch;
     for (int i = n; i < bucket; ++i) m->h_idx[i] = m->h_idx[n - 1];
     CUDA_TRY(cudaMemcpyAsync(m->re_idx, m->h_idx, sizeof(int32_t) * bucket, cudaMemcpyHostToDevice, st));
     const int64_t per = (int64_t)m->in_c * m->in_h * m->in_w;
@@ -964,6 +1007,16 @@ ct_status infer_fault_free(ct_model *m, const float *input, int batch, float *lo
     return s;
 }
 
+cudaError_t reexec_gather(ct_model *m, const float *in, float *out, const int32_t *idx, int n, int64_t per_image,
+                          cudaStream_t st) {
+    return launch(m, FAM_OTHER, 0, st, [&] { return launch_gather_images(in, out, idx, n, per_image, st); });
+}
+
+cudaError_t reexec_scatter(ct_model *m, const float *src, float *dst, const int32_t *idx, int n, int row,
+                           cudaStream_t st) {
+    return launch(m, FAM_OTHER, 0, st, [&] { return launch_scatter_rows(src, dst, idx, n, row, st); });
+}
+
 }  // namespace ct
 
 // ===========================================================================
@@ -971,6 +1024,11 @@ ct_status infer_fault_free(ct_model *m, const float *input, int batch, float *lo
 // ===========================================================================
 
 extern "C" {
+
+ct_status ct_resolve_roles(const ct_model_desc *desc, int32_t *roles) {
+    if (!desc || !roles || desc->n_layers < 1 || !desc->layers) return CT_EINVAL;
+    return resolve_roles(desc, roles);
+}
 
 ct_status ct_build(const ct_model_desc *desc, const float *const *weights, const ct_build_opts *opts,
                    ct_model **out) {
@@ -980,6 +1038,11 @@ ct_status ct_build(const ct_model_desc *desc, const float *const *weights, const
     if (opts->max_batch < 1 || desc->in_c < 1 || desc->in_h < 1 || desc->in_w < 1 || desc->n_classes < 1)
         return CT_EINVAL;
     *out = nullptr;
+    {
+        // the description is checked against the residual rule before any device work
+        std::vector<int32_t> roles(desc->n_layers);
+        if (resolve_roles(desc, roles.data()) != CT_OK) return CT_EINVAL;
+    }
     int ndev = 0;
     if (cudaGetDeviceCount(&ndev) != cudaSuccess || opts->device < 0 || opts->device >= ndev) {
         cudaGetLastError();
@@ -998,6 +1061,9 @@ ct_status ct_build(const ct_model_desc *desc, const float *const *weights, const
     m->in_c = desc->in_c; m->in_h = desc->in_h; m->in_w = desc->in_w;
     m->n_classes = desc->n_classes;
     ct_status s = build_impl(m, desc, weights);
+    // the static scratch of ct_reexecute_noalloc is committed here, not on
+    // its first call
+    if (s == CT_OK) s = noalloc_scratch_setup(m->device);
     if (s != CT_OK) {
         free_all(m);
         delete m;
@@ -1065,6 +1131,19 @@ ct_status ct_reexecute(ct_model *m, const float *input_dev, int32_t batch, const
     ct_status s = reexec_impl(m, input_dev, batch, flag_dev, logits_dev, S_dev, &n, (cudaStream_t)stream);
     if (n_rerun) *n_rerun = n;
     return s;
+}
+
+ct_status ct_reexecute_prepare(ct_model *m, int32_t max_images) {
+    if (!m) return CT_EINVAL;
+    if (max_images < 1 || max_images > m->max_batch) return CT_ERANGE;
+    DeviceGuard g(m->device);
+    // the same buckets reexec_impl uses: powers of two, the last one capped at max_batch
+    for (int b = 1;; b <<= 1) {
+        const int bucket = b > m->max_batch ? m->max_batch : b;
+        if (!reexec_graph(m, bucket)) return CT_ECUDA;
+        if (b >= max_images) break;
+    }
+    return CT_OK;
 }
 
 ct_status ct_infer_reexec(ct_model *m, const float *input_dev, int32_t batch, float *logits_dev, float *S_dev,

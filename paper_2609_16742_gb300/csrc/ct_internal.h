@@ -181,6 +181,16 @@ ct_status model_info(const ct_model *m, ModelInfo *out);
 // ct_infer on device buffers with any armed fault left armed for the next ct_infer.
 ct_status infer_fault_free(ct_model *m, const float *input, int batch, float *logits, float *S,
                            uint8_t *flag, cudaStream_t st);
+// The re-execution gather and scatter launched for model m: counted by
+// ct_kernel_count and timed under ct_profile_enable like every kernel of m.
+cudaError_t reexec_gather(ct_model *m, const float *in, float *out, const int32_t *idx, int n, int64_t per_image,
+                          cudaStream_t st);
+cudaError_t reexec_scatter(ct_model *m, const float *src, float *dst, const int32_t *idx, int n, int row,
+                           cudaStream_t st);
+// Looks up, with `device` current, the device address of the static scratch
+// of ct_reexecute_noalloc (loading its module commits the array); ct_build
+// calls it so that no request-serving call does.
+ct_status noalloc_scratch_setup(int device);
 
 // number of SMs of the current device (148 if the query fails)
 int device_sm_count();

@@ -13,7 +13,9 @@
 // Host code must not pass g_reexec_scratch to a kernel: on the host the name
 // stands for a host-side shadow, not a device address.  The device address is
 // looked up once per device with cudaGetSymbolAddress, with that device
-// current, on the first call made on the device.
+// current, by ct_build (noalloc_scratch_setup).  The lookup loads this file's
+// module, which commits the array on that device; doing it in ct_build keeps
+// that commitment out of the calls that serve requests.
 #include <string.h>
 
 #include "ct_internal.h"
@@ -31,11 +33,34 @@ int32_t g_host_idx[kMaxBatch];
 
 size_t up256(size_t x) { return (x + 255) & ~(size_t)255; }
 
+// device address of the array on the current device, looked up once
+ct_status lookup(int device) {
+    if (g_scratch_ready[device]) return CT_OK;
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_reexec_scratch) != cudaSuccess || p == nullptr) {
+        cudaGetLastError();
+        return CT_ECUDA;
+    }
+    g_scratch_dev[device] = static_cast<unsigned char *>(p);
+    g_scratch_ready[device] = true;
+    return CT_OK;
+}
+
 }  // namespace
+
+namespace ct {
+
+ct_status noalloc_scratch_setup(int device) {
+    if (device < 0 || device >= kMaxDevices) return CT_EINVAL;
+    return lookup(device);
+}
+
+}  // namespace ct
 
 extern "C" ct_status ct_reexecute_noalloc(ct_model *m, const float *input_dev, int32_t batch,
                                           const uint8_t *flag_dev, float *logits_dev, float *S_dev,
                                           int32_t *n_rerun, void *stream) {
+    if (n_rerun) *n_rerun = 0;
     if (!m || !input_dev || !flag_dev || !logits_dev) return CT_EINVAL;
     ct::ModelInfo mi;
     ct_status s = ct::model_info(m, &mi);
@@ -50,16 +75,9 @@ extern "C" ct_status ct_reexecute_noalloc(ct_model *m, const float *input_dev, i
         ~Restore() { if (prev >= 0 && prev != dev) cudaSetDevice(prev); }
     } restore{mi.device, prev};
 
-    // set-up, once per device, with the device current
-    if (!g_scratch_ready[mi.device]) {
-        void *p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_reexec_scratch) != cudaSuccess || p == nullptr) {
-            cudaGetLastError();
-            return CT_ECUDA;
-        }
-        g_scratch_dev[mi.device] = static_cast<unsigned char *>(p);
-        g_scratch_ready[mi.device] = true;
-    }
+    // ct_build looked the address up for this device; the lookup here only
+    // runs if that failed to happen (it is a no-op otherwise)
+    if ((s = lookup(mi.device)) != CT_OK) return s;
     unsigned char *base = g_scratch_dev[mi.device];
     cudaStream_t st = (cudaStream_t)stream;
 
@@ -70,7 +88,6 @@ extern "C" ct_status ct_reexecute_noalloc(ct_model *m, const float *input_dev, i
     int n = 0;
     for (int i = 0; i < batch; ++i)
         if (g_host_flags[i]) g_host_idx[n++] = i;
-    if (n_rerun) *n_rerun = n;
     if (n == 0) return CT_OK;
 
     // scratch layout: index list | compacted images | logits | S | flags
@@ -82,6 +99,7 @@ extern "C" ct_status ct_reexecute_noalloc(ct_model *m, const float *input_dev, i
     const size_t off_fl = up256(off_S + sizeof(float) * n);
     const size_t need = off_fl + (size_t)n;
     if (need > (size_t)CT_NOALLOC_SCRATCH_BYTES) return CT_ERANGE;
+    if (n_rerun) *n_rerun = n;
     int32_t *idx = reinterpret_cast<int32_t *>(base + off_idx);
     float *cin = reinterpret_cast<float *>(base + off_in);
     float *clg = reinterpret_cast<float *>(base + off_lg);
@@ -90,10 +108,10 @@ extern "C" ct_status ct_reexecute_noalloc(ct_model *m, const float *input_dev, i
 
     if (cudaMemcpyAsync(idx, g_host_idx, sizeof(int32_t) * n, cudaMemcpyHostToDevice, st) != cudaSuccess)
         return CT_ECUDA;
-    if (ct::launch_gather_images(input_dev, cin, idx, n, per, st) != cudaSuccess) return CT_ECUDA;
+    if (ct::reexec_gather(m, input_dev, cin, idx, n, per, st) != cudaSuccess) return CT_ECUDA;
     s = ct::infer_fault_free(m, cin, n, clg, cS, cfl, st);
     if (s != CT_OK) return s;
-    if (ct::launch_scatter_rows(clg, logits_dev, idx, n, mi.n_classes, st) != cudaSuccess) return CT_ECUDA;
-    if (S_dev && ct::launch_scatter_rows(cS, S_dev, idx, n, 1, st) != cudaSuccess) return CT_ECUDA;
+    if (ct::reexec_scatter(m, clg, logits_dev, idx, n, mi.n_classes, st) != cudaSuccess) return CT_ECUDA;
+    if (S_dev && ct::reexec_scatter(m, cS, S_dev, idx, n, 1, st) != cudaSuccess) return CT_ECUDA;
     return CT_OK;
 }

@@ -93,3 +93,56 @@ def test_fi_threshold_matches_oracle(ct):
         assert got == oracle.fi_threshold(S.astype(np.float64), crit, 2001.5, alpha)
     with pytest.raises(ct.CtError):
         ct.ct_fi_threshold(S, np.ones(3001, np.uint8), 0.0, 0.01)
+
+
+@pytest.mark.parametrize("name", ["lenet5", "resnet18_cifar", "resnet18_imagenet", "vgg16",
+                                  "mobilenetv2_cifar"])
+def test_library_derives_the_residual_roles(ct, name):
+    """Sec. II-A residual rule in the library (host only): with every role left
+    to the library (CT_ROLE_AUTO) it derives the declared roles; the declared
+    roles pass unchanged."""
+    import dataclasses
+    import synth
+    wl = synth.workload(name)
+    declared = [L.ct if L.op == "conv" else None for L in wl.layers]
+    auto = [dataclasses.replace(L, ct="auto") if L.op == "conv" else L for L in wl.layers]
+    got = ct.ct_resolve_roles(auto, wl.in_shape, wl.n_classes)
+    # depthwise layers: the library keeps the role it is given and decides the
+    # pass-through when it builds them; compare the dense convolutions
+    dense = [i for i, L in enumerate(wl.layers) if L.op == "conv" and L.groups == 1]
+    assert [got[i] for i in dense] == [declared[i] for i in dense]
+    assert ct.ct_resolve_roles(wl.layers, wl.in_shape, wl.n_classes) == declared
+
+
+def test_library_rejects_a_filter_the_residual_rule_forbids(ct):
+    """A block whose first convolution is labelled "ct" (its input is also the
+    shortcut) is rejected by ct_resolve_roles and by ct_build before any
+    device work (CT_EINVAL), GPU or not."""
+    import dataclasses
+    import synth
+    wl = synth.workload("resnet18_cifar")
+    first = next(i for i, L in enumerate(wl.layers) if L.op == "conv" and L.ct == "none")
+    bad = [dataclasses.replace(L, ct="ct") if i == first else L for i, L in enumerate(wl.layers)]
+    with pytest.raises(ct.CtError) as ei:
+        ct.ct_resolve_roles(bad, wl.in_shape, wl.n_classes)
+    assert ei.value.status == 1
+    params = [{} for _ in bad]
+    with pytest.raises(ct.CtError) as ei:
+        ct.ct_build(bad, params, wl.in_shape, wl.n_classes, max_batch=1)
+    assert ei.value.status == 1
+    # a downsample shortcut labelled "ct" breaks the rule too
+    ds = next(i for i, L in enumerate(wl.layers) if L.op == "conv" and L.ct == "pass")
+    bad = [dataclasses.replace(L, ct="ct") if i == ds else L for i, L in enumerate(wl.layers)]
+    with pytest.raises(ct.CtError):
+        ct.ct_resolve_roles(bad, wl.in_shape, wl.n_classes)
+
+
+def test_no_multicast_load_in_the_library():
+    """The library runs on every rank of a multi-GPU run: no TMA load may use
+    cluster multicast (mbarrier arrivals of tcgen05.commit are not loads)."""
+    csrc = os.path.join(ROOT, "paper_2609_16742_gb300", "csrc")
+    for f in sorted(os.listdir(csrc)):
+        txt = open(os.path.join(csrc, f)).read()
+        for line in txt.splitlines():
+            if "cp.async.bulk" in line:
+                assert "multicast" not in line, (f, line)

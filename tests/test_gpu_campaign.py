@@ -1,5 +1,5 @@
-"""The fault-injection campaign of Sec. III-A on the CIFAR ResNet-18: a seeded
-subset of its faults against the oracle (per-image critical and flagged
+"""The fault-injection campaign of Sec. III-A on the CIFAR ResNet-18: its
+first 500 seeded faults against the oracle (per-image critical and flagged
 verdicts), and the campaign runner's bookkeeping."""
 import numpy as np
 import pytest
@@ -19,27 +19,35 @@ def _model(prec, B):
 
 @pytest.mark.parametrize("prec", ["fp32", "fp16"])
 def test_campaign_faults_match_oracle(prec):
-    B, n_faults = 16, 24
+    """The first 500 faults of the campaign (the same seeded draw as
+    campaign.run with seed 0, over the campaign's batch of 128 images)
+    against the oracle: per image trial, S within tolerance and the verdict
+    identical (near-threshold images counted apart), and the critical
+    verdict identical unless the oracle's top two logits are within the
+    tolerance of each other.  A weight fault is compared on the first 8
+    images, an activation fault on the image it hits."""
     wl = synth.workload("campaign_resnet18_cifar")
+    B, n_faults = wl.batch, 500
     m = _model(prec, B)
     net = onet("resnet18_cifar", prec)
     x = synth.make_input(wl, batch=B)
-    xc = synth.make_input(wl, batch=256, seed=wl.calib_seed)
+    xc = synth.make_input(wl, batch=128, seed=wl.calib_seed)
     r, tau = oracle.calibrate(oracle.forward(net, xc)["S"], 0.01)
     ct().ct_set_threshold(m, r, tau)
     g_lg, _, _ = run(m, x)
     o_g = oracle.forward(net, x)
     top_o = oracle.top1(o_g["logits"])
+    top_g = oracle.top1(g_lg)
     bufs = ct().ct_buffers(m, B)
     assert bufs == oracle.fault_buffers(net, B)
-    faults = synth.draw_faults(bufs, n_faults, seed=11)
+    faults = synth.draw_faults(bufs, n_faults, seed=0)
     per_img = {layer: n // B for kind, layer, n, bits in bufs if kind == 1}
-    n_cmp = n_near = crit_mismatch = 0
+    n_cmp = n_near = crit_mismatch = n_crit = n_flag = 0
     for kind, layer, e, bit in faults.tolist():
         ct().ct_inject(m, kind, layer, e, bit)
         lg, S, fl = run(m, x)
         if kind == 0:
-            imgs, f = list(range(4)), oracle.Fault(0, layer, e, bit)
+            imgs, f = list(range(8)), oracle.Fault(0, layer, e, bit)
         else:
             img, off = divmod(e, per_img[layer])
             imgs, f = [img], oracle.Fault(1, layer, off, bit)
@@ -56,13 +64,18 @@ def test_campaign_faults_match_oracle(prec):
                 assert bool(fl[i]) == bool(oracle.verdict([so], r, tau)[0]), (kind, layer, e, bit, sg, so)
             lo = o["logits"][j]
             crit_o = oracle.top1(lo[None])[0] != top_o[i]
-            crit_g = oracle.top1(lg[i][None])[0] != oracle.top1(g_lg[i][None])[0]
+            crit_g = oracle.top1(lg[i][None])[0] != top_g[i]
             if crit_o != crit_g:
                 srt = np.sort(lo[np.isfinite(lo)])
                 assert len(srt) > 1 and srt[-1] - srt[-2] <= 2 * TOL[prec] * np.abs(lo).max()
                 crit_mismatch += 1
+            n_crit += int(crit_o)
+            n_flag += int(bool(fl[i]))
             n_cmp += 1
-    assert n_cmp >= n_faults and crit_mismatch <= 1
+    assert n_cmp >= n_faults and crit_mismatch <= max(2, n_cmp // 500)
+    assert ct().ct_device_error(m) == 0
+    print("%s: %d trials, %d critical, %d flagged, %d near-threshold, %d critical mismatches"
+          % (prec, n_cmp, n_crit, n_flag, n_near, crit_mismatch))
 
 
 def test_campaign_runner_bookkeeping():

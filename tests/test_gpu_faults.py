@@ -5,7 +5,7 @@ import pytest
 import oracle
 import synth
 from _cache import inputs
-from _gpu import TOL, ct, kept_checksum_pixel, model, onet, rel_err_rows, run, same_class
+from _gpu import TOL, assert_parity, ct, kept_checksum_pixel, model, onet, rel_err_rows, run, same_class
 
 pytestmark = pytest.mark.gpu
 
@@ -133,6 +133,33 @@ def test_reexecute_restores_flagged_rows():
     assert np.array_equal(Sn[keep], g_S[keep].astype(np.float32))
     assert rel_err_rows(lgn[5], g_lg[5])[0] <= 1e-5
     assert abs(Sn[5] - g_S[5]) <= 1e-5 * abs(g_S[5])
+
+
+def test_reexecute_rows_match_oracle_every_bucket():
+    """Sec. II-B re-execution against the oracle: with the graphs captured
+    ahead of time (ct_reexecute_prepare) and a max_batch that is not a power
+    of two (6), 1 to 6 flagged images (padded batches 1, 2, 4 and the capped
+    6, which 5 flagged images also use) are re-run into poisoned rows; each
+    re-run row matches the oracle and no other row is written."""
+    import torch
+    name, B = "resnet18_cifar", 6
+    m = model(name, max_batch=B)
+    ct().ct_reexecute_prepare(m, B)
+    x = inputs(name, B)
+    o = oracle.forward(onet(name, "fp32"), x)
+    xd = torch.from_numpy(x).cuda()
+    for n in (1, 2, 3, 5, 6, 5):
+        fl = torch.zeros(B, dtype=torch.uint8, device="cuda")
+        fl[B - n:] = 1
+        lg = torch.full((B, m.n_classes), float("nan"), device="cuda")
+        S = torch.full((B,), float("nan"), device="cuda")
+        assert ct().ct_reexecute(m, xd, B, fl, lg, S) == n
+        torch.cuda.synchronize()
+        lgn, Sn = lg.cpu().numpy().astype(np.float64), S.cpu().numpy().astype(np.float64)
+        assert np.isnan(lgn[:B - n]).all() and np.isnan(Sn[:B - n]).all()
+        assert_parity(lgn[B - n:], Sn[B - n:], o["logits"][B - n:], o["S"][B - n:], "fp32",
+                      "re-run of %d images" % n)
+    assert ct().ct_device_error(m) == 0
 
 
 def test_run_host_matches_device_path():

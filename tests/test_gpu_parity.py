@@ -126,3 +126,21 @@ def test_fault_buffers_match_oracle():
     assert ct().ct_buffers(m, 128) == oracle.fault_buffers(onet("resnet18_cifar", "fp32"), 128)
     m16 = model("resnet18_imagenet", max_batch=2)
     assert ct().ct_buffers(m16, 2) == oracle.fault_buffers(onet("resnet18_imagenet", "fp16"), 2)
+
+
+def test_roles_derived_by_the_library_build_the_same_network():
+    """Sec. II-A residual rule: the network built with every role left to the
+    library (CT_ROLE_AUTO) is the one built from the declared roles, bit for
+    bit."""
+    import dataclasses
+    import synth
+    from _cache import params
+    name = "resnet18_cifar"
+    wl = synth.workload(name)
+    auto = [dataclasses.replace(L, ct="auto") if L.op == "conv" else L for L in wl.layers]
+    x = inputs(name, 4)
+    ma = ct().ct_build(auto, params(name), wl.in_shape, wl.n_classes, max_batch=4)
+    la, Sa, _ = run(ma, x)
+    lm, Sm, _ = run(model(name, max_batch=4), x)
+    assert np.array_equal(la, lm) and np.array_equal(Sa, Sm)
+    ma.close()

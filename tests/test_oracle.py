@@ -351,6 +351,53 @@ def test_residual_rule_prevents_double_count():
     assert bad != good
 
 
+def test_residual_roles_hand_built_graphs():
+    """Sec. II-A residual rule on hand-built graphs: a tensor read twice gives
+    its convolution readers no carry-through filter; the convolution whose
+    output is the residual operand is the shortcut."""
+    # identity block: slot 1 is read by conv1 (src) and by the add of conv2 (res)
+    assert oracle.residual_roles(tiny_resnet(ds=False)) == ["ct", "none", "ct", None, None]
+    # downsample block: slot 1 is read by conv1 and by the 1x1 shortcut
+    assert oracle.residual_roles(tiny_resnet(ds=True)) == ["ct", "none", "pass", "ct", None, None]
+    # no residual anywhere: every convolution carries a filter
+    assert oracle.residual_roles(tiny_lenet()) == ["ct", None, "ct", None, None]
+    # a tensor read by two convolutions whose outputs meet only in an FC-free
+    # branch: both readers lose the filter, the depthwise layer passes through
+    L = [Layer("conv", 0, 1, cin=1, cout=2, k=3, pad=1),
+         Layer("conv", 1, 2, cin=2, cout=2, k=3, pad=1),
+         Layer("conv", 1, 3, cin=2, cout=2, k=3, pad=1, groups=2),
+         Layer("conv", 3, 4, cin=2, cout=2, k=3, pad=1, groups=2)]
+    assert oracle.residual_roles(L) == ["ct", "none", "none", "pass"]
+
+
+@pytest.mark.parametrize("name", ["lenet5", "resnet18_cifar", "resnet18_imagenet", "vgg16",
+                                  "mobilenetv2_cifar"])
+def test_workload_roles_follow_the_residual_rule(name):
+    """The roles the workloads declare (and the oracle and the library read)
+    are those the residual rule derives from the graph."""
+    wl = synth.workload(name)
+    declared = [L.ct if L.op == "conv" else None for L in wl.layers]
+    assert oracle.residual_roles(wl.layers) == declared
+
+
+def test_top1_pins():
+    """Sec. II-B "change of the golden classification": argmax with ties to the
+    lowest index, any NaN logit gives class -1; infinities order as numbers."""
+    nan, inf = float("nan"), float("inf")
+    rows = [([1.0, 3.0, 2.0], 1), ([5.0, 5.0, 1.0], 0), ([1.0, 5.0, 5.0], 1),
+            ([nan, 1.0, 2.0], -1), ([1.0, 2.0, nan], -1), ([nan, nan], -1),
+            ([1.0, inf, 2.0], 1), ([inf, inf, 0.0], 0), ([-inf, -inf, -inf], 0), ([-inf, -5.0], 1),
+            ([-0.0, 0.0], 0), ([0.0, -0.0], 0), ([7.0], 0), ([-1e30, -1e31, -1e29], 2)]
+    for row, want in rows:
+        assert oracle.top1(np.array([row]))[0] == want, (row, want)
+    # without ties or NaN it is numpy's argmax (first maximum)
+    x = np.random.default_rng(3).standard_normal((200, 17))
+    assert (oracle.top1(x) == np.argmax(x, axis=1)).all()
+    # float32 logits promoted to double keep their order
+    assert oracle.top1(np.array([[np.float32(1.0), np.nextafter(np.float32(1.0), np.float32(2.0))]],
+                                dtype=np.float32))[0] == 1
+
+
 # ---------------------------------------------------------------------------
 # O-T5: brute-force single-bit flips on a tiny net against a separate scalar model
 # ---------------------------------------------------------------------------

@@ -68,3 +68,28 @@ def test_noalloc_rejects_a_batch_beyond_its_scratch():
     assert ct().ct_reexecute_noalloc(m, xd, B, fl, lg, S) == 2
     torch.cuda.synchronize()
     assert np.isfinite(lg[:2].cpu().numpy()).all() and float(lg[2:].abs().sum()) == 0.0
+
+
+def test_noalloc_leaves_device_free_memory_unchanged():
+    """The reason the entry point exists: a call takes no device memory.  A
+    re-run of 8 flagged 3x224x224 images needs ~5 MB of scratch; after the
+    model's kernels have run once (so their modules are loaded), the device's
+    free memory is the same before and after two calls."""
+    import torch
+    name, B = "resnet18_imagenet", 8
+    m = model(name, max_batch=B)
+    xd = torch.from_numpy(inputs(name, B)).cuda()
+    lg = torch.zeros(B, m.n_classes, device="cuda")
+    S = torch.zeros(B, device="cuda")
+    fl = torch.ones(B, dtype=torch.uint8, device="cuda")
+    lg0 = torch.zeros_like(lg)
+    ct().ct_infer(m, xd, B, lg0, None, None)       # loads the modules of a batch-8 inference
+    torch.cuda.synchronize()
+    free0 = torch.cuda.mem_get_info()[0]
+    for _ in range(2):
+        assert ct().ct_reexecute_noalloc(m, xd, B, fl, lg, S) == B
+    torch.cuda.synchronize()
+    assert torch.cuda.mem_get_info()[0] == free0
+    a, b = lg0.cpu().numpy(), lg.cpu().numpy()
+    err = np.abs(a - b).max(axis=1) / np.maximum(np.abs(a).max(axis=1), 1e-6)
+    assert (err <= TOL["fp16"]).all()
