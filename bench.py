@@ -5,12 +5,15 @@ One step = one batch through the whole inference path on each GPU:
 carry-through convolutions, FC layers with the checksum neurons, per-image
 verification, and re-execution of the flagged images (fault-free run: the
 flagged images are the false alarms of the distribution-based threshold,
-alpha = 1%).  The headline re-executes each batch's flagged images as extra
-rows of the next batch's inference (ct_infer_reexec; the last batch's at the
-end of the timed region); the same steps with a separate re-run per batch
+alpha = 1%).  The headline runs the K timed batches through one
+ct_infer_batches call, which re-executes each batch's flagged images as
+extra rows of the inference two batches later (the last two batches' at the
+end of the call); the same steps with a separate re-run per batch
 (ct_infer + ct_reexecute) are reported beside it.  The same model built
 without carry-through filters gives the unprotected throughput and the
-overhead.
+overhead.  The end-to-end figure runs the same batches from pinned host
+memory through ct_run_host_batches (copies in and out inside the call,
+overlapped with the inferences).
 
 Prints ONE JSON line (rank 0).  Multi-GPU (torchrun): independent replicas,
 each rank runs its own batch; only the barrier and the max-over-ranks timing
@@ -189,7 +192,7 @@ def recorded_traffic(workload, batch):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=40)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
@@ -277,22 +280,20 @@ def main():
         ct.ct_infer(mp, x, B, logits, S, flag, stream)
         return ct.ct_reexecute(mp, x, B, flag, logits, S, stream)
 
+    # outputs of the batch-list calls: four rotating sets (a batch's re-run rows
+    # are written two batches after it)
+    outs = [{"lg": torch.empty(B, wl.n_classes, device="cuda"), "S": torch.empty(B, device="cuda"),
+             "fl": torch.empty(B, dtype=torch.uint8, device="cuda")} for _ in range(4)]
+
     def deferred_steps(steps, model=None):
-        """`steps` protected steps in which the flagged images of each batch
-        are re-executed as extra rows of the next batch's inference
-        (ct_infer_reexec); the last batch's are re-run at the end."""
+        """`steps` protected steps in one ct_infer_batches call: each batch's
+        flagged images are re-executed as extra rows of the inference two
+        batches later, the last two batches' at the end of the call."""
         model = model or mp
-        n_re, prev = 0, None
-        for i in range(steps):
-            cur = bufs[i % 2]
-            if prev is None:
-                n_re += ct.ct_infer_reexec(model, cur["x"], B, cur["lg"], cur["S"], cur["fl"], stream=stream)
-            else:
-                n_re += ct.ct_infer_reexec(model, cur["x"], B, cur["lg"], cur["S"], cur["fl"], prev["x"], B,
-                                           prev["fl"], prev["lg"], prev["S"], stream)
-            prev = cur
-        n_re += ct.ct_reexecute(model, prev["x"], B, prev["fl"], prev["lg"], prev["S"], stream)
-        return n_re
+        xs = [bufs[i % 2]["x"] for i in range(steps)]
+        return ct.ct_infer_batches(model, xs, B, [outs[i % 4]["lg"] for i in range(steps)],
+                                   [outs[i % 4]["S"] for i in range(steps)],
+                                   [outs[i % 4]["fl"] for i in range(steps)], stream)
 
     def step_unprotected():
         ct.ct_infer(mu, x, B, logits, None, None, stream)
@@ -382,48 +383,20 @@ def main():
     def max_over_ranks(v):
         return replicas.reduce_max(v, dist, "cuda")
 
-    # end to end through the public API from pinned host memory: every step
-    # copies its input in (on a copy stream, overlapping the previous step's
-    # kernels; three input slots), runs ct_infer_reexec, and copies the
-    # completed batch's logits, S and flags out (the last batch after its
-    # re-run).  Slot i % 3 is free for step i + 1's input once ct_infer_reexec
-    # of step i returns: that call waited for step i - 1's kernels, the last
-    # to read it.
+    # end to end through the public API from pinned host memory: one
+    # ct_run_host_batches call over the K batches copies each batch in on the
+    # library's copy stream while earlier batches run, and copies each
+    # batch's logits, S and flags out once its re-run rows are final
     xh2 = [torch.from_numpy(xh_).pin_memory() for xh_ in x_hosts]
-    d2h = {"lg": torch.empty(B, wl.n_classes, dtype=torch.float32).pin_memory(),
-           "S": torch.empty(B, dtype=torch.float32).pin_memory(),
-           "fl": torch.empty(B, dtype=torch.uint8).pin_memory()}
-    ebufs = [{"x": torch.empty_like(bufs[0]["x"]), "lg": torch.empty_like(bufs[0]["lg"]),
-              "S": torch.empty_like(bufs[0]["S"]), "fl": torch.empty_like(bufs[0]["fl"])} for _ in range(3)]
-    copy_stream = torch.cuda.Stream()
-    ev_in = [torch.cuda.Event() for _ in range(3)]
-
-    def copy_in(i):
-        with torch.cuda.stream(copy_stream):
-            ebufs[i % 3]["x"].copy_(xh2[i % 2], non_blocking=True)
-            ev_in[i % 3].record(copy_stream)
+    hout = [{"lg": torch.empty(B, wl.n_classes, dtype=torch.float32).pin_memory(),
+             "S": torch.empty(B, dtype=torch.float32).pin_memory(),
+             "fl": torch.empty(B, dtype=torch.uint8).pin_memory()} for _ in range(4)]
 
     def e2e_steps(steps):
-        n_re, prev = 0, None
-        copy_in(0)
-        for i in range(steps):
-            cur = ebufs[i % 3]
-            stream.wait_event(ev_in[i % 3])
-            if prev is None:
-                n_re += ct.ct_infer_reexec(mp, cur["x"], B, cur["lg"], cur["S"], cur["fl"], stream=stream)
-            else:
-                n_re += ct.ct_infer_reexec(mp, cur["x"], B, cur["lg"], cur["S"], cur["fl"], prev["x"], B,
-                                           prev["fl"], prev["lg"], prev["S"], stream)
-            if i + 1 < steps:
-                copy_in(i + 1)
-            if prev is not None:
-                for k_ in ("lg", "S", "fl"):
-                    d2h[k_].copy_(prev[k_], non_blocking=True)
-            prev = cur
-        n_re += ct.ct_reexecute(mp, prev["x"], B, prev["fl"], prev["lg"], prev["S"], stream)
-        for k_ in ("lg", "S", "fl"):
-            d2h[k_].copy_(prev[k_], non_blocking=True)
-        return n_re
+        return ct.ct_run_host_batches(mp, [xh2[i % 2] for i in range(steps)], B,
+                                      [hout[i % 4]["lg"] for i in range(steps)],
+                                      [hout[i % 4]["S"] for i in range(steps)],
+                                      [hout[i % 4]["fl"] for i in range(steps)], stream)
 
     e2e_steps(3)
     barrier()
@@ -431,6 +404,16 @@ def main():
     e2e_steps(args.steps)
     barrier()
     e2e_s = max_over_ranks(time.perf_counter() - t0)
+    # what the host link gives one batch's input alone (pinned host -> device)
+    xd_probe = torch.empty_like(bufs[0]["x"])
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for _ in range(5):
+        xd_probe.copy_(xh2[0], non_blocking=True)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    h2d_gbs = 5 * xh2[0].numel() * 4 / (ev0.elapsed_time(ev1) / 1e3) / 1e9
+    del xd_probe
 
     # the same through the host-buffer entry point ct_run_host (H2D, infer,
     # synchronous re-execution, D2H inside the call)
@@ -527,8 +510,9 @@ def main():
                    "parallelism": "replicas x%d" % world, "alpha": 0.01,
                    "l2": "inputs and activations larger than L2 (no flush)",
                    "simt_only": bool(args.simt_only)},
-        "reexecution": "deferred: each batch's flagged images ride as extra rows of the next batch's "
-                       "inference (ct_infer_reexec); the last batch's are re-run at the end of the timed region",
+        "reexecution": "deferred by two batches (ct_infer_batches): each batch's flagged images ride as extra "
+                       "rows of the inference two batches later; the last two batches' are re-run at the end of "
+                       "the call, inside the timed region",
         "value_sync_reexec": replicas.job_throughput(world, B, args.steps, ms_ps / 1e3),
         "overhead_reexec_sync_pct": 100.0 * (ms_ps - ms_pi) / ms_u,
         "reexecuted_images_per_step_sync": n_rerun_s / args.steps,
@@ -538,8 +522,10 @@ def main():
         "cpu_baseline": cpu,
         "e2e": {"value": replicas.job_throughput(world, B, args.steps, e2e_s), "unit": "images/s",
                 "h2d_bytes_per_step": in_bytes, "d2h_bytes_per_step": out_bytes,
-                "api": "ct_infer_reexec; pinned host copies in (copy stream, overlapping the previous "
-                       "step) and out (launch stream)"},
+                "api": "ct_run_host_batches: one call over the K batches from pinned host memory, copies in "
+                       "and out overlapped with the inferences, deferred re-execution",
+                "h2d_gbs_alone": h2d_gbs,
+                "h2d_bound_images_per_s": h2d_gbs * 1e9 / (in_bytes / B) * world},
         "e2e_sync_reexec": {"value": replicas.job_throughput(world, B, args.steps, e2e_sync_s), "unit": "images/s",
                             "api": "ct_run_host (host buffers, synchronous re-execution)"},
         "kernel_families": {nm: {"launches": fam_stats[i][0], "ms": fam_stats[i][1],

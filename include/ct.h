@@ -342,6 +342,48 @@ ct_status ct_reexecute_noalloc(ct_model *m, const float *input_dev, int32_t batc
                                const uint8_t *flag_dev, float *logits_dev, float *S_dev,
                                int32_t *n_rerun, void *stream);
 
+/* ct_infer_batches -- Sec. II-B over a list of batches resident on the
+ * device: inference and verification of each batch, and re-execution of
+ * every flagged image, deferred by two batches (Sec. II-B, last paragraph:
+ * re-execute flagged inferences once, ignore the re-run's flag).  Step i
+ * infers batch i and re-runs, as extra rows of that same inference, the
+ * flagged images of batch i - 2, whose flags the library copied to pinned
+ * host memory when that batch's inference ended; the host waits only for
+ * that copy, which the device finished while it went on with batch i - 1,
+ * so the device never idles for a flag read-back.  The last two batches'
+ * flagged images are re-run on their own at the end.
+ *   - input_dev[i], logits_dev[i], S_dev[i], flag_dev[i]: host arrays of
+ *     n_batches device pointers (FP32 NCHW [batch, C, H, W]; FP32
+ *     [batch, n_classes]; FP32 [batch]; uint8 [batch]), as for ct_infer.
+ *     Every one must stay valid for the whole call; a re-run row overwrites
+ *     its image's logits and S; the flags are the first run's.
+ *   - The re-run rows must fit max_batch (batch + flagged images); when they
+ *     do not, or a fault is armed, that batch's flagged images are re-run as
+ *     by ct_reexecute instead (the armed fault goes to the next inference).
+ *   - Returns after every result is final (the call synchronises `stream`).
+ *   - *n_rerun (host, may be NULL): images re-run in all.
+ * Errors: CT_EINVAL (null arrays or entries), CT_ERANGE (batch outside
+ * 1..max_batch), CT_ENOMEM (first call: pinned host memory), CT_ECUDA. */
+ct_status ct_infer_batches(ct_model *m, int32_t n_batches, int32_t batch, const float *const *input_dev,
+                           float *const *logits_dev, float *const *S_dev, uint8_t *const *flag_dev,
+                           int32_t *n_rerun, void *stream);
+
+/* ct_run_host_batches -- ct_infer_batches for callers whose inputs and
+ * results live in HOST memory: batch i's input (input_host[i], FP32 NCHW) is
+ * copied into one of six library-owned device slots on a library copy
+ * stream while the device still works on earlier batches, and its logits
+ * (logits_host[i]), S (S_host[i]) and flags (flag_host[i]) are copied back
+ * once its re-run rows are written (two batches later).  S_host and
+ * flag_host, or any of their entries, may be NULL (not copied back).  With
+ * pinned host buffers the copies overlap the inferences; pageable buffers
+ * work, serialised.  The first call allocates the device slots (6 x
+ * max_batch images and their results) and pinned flag buffers; they live
+ * until ct_destroy.  Returns after every result is in host memory.
+ * Errors as for ct_infer_batches. */
+ct_status ct_run_host_batches(ct_model *m, int32_t n_batches, int32_t batch, const float *const *input_host,
+                              float *const *logits_host, float *const *S_host, uint8_t *const *flag_host,
+                              int32_t *n_rerun, void *stream);
+
 /* ct_run_host -- end-to-end call for callers with host buffers: copies the
  * input from host memory, runs ct_infer and ct_reexecute, and copies
  * logits, S and flags back.  Returns after the results are in host memory.

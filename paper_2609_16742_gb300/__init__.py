@@ -39,7 +39,7 @@ EXPORTS = ["ct_build", "ct_set_threshold", "ct_get_threshold", "ct_infer", "ct_i
            "ct_fi_threshold",
            "ct_copy_activation", "ct_device_error", "ct_destroy", "ct_strerror",
            "ct_reexecute_noalloc", "ct_campaign_batched", "ct_resolve_roles",
-           "ct_reexecute_prepare"]
+           "ct_reexecute_prepare", "ct_infer_batches", "ct_run_host_batches"]
 
 CT_NOALLOC_SCRATCH_BYTES = 16 * 1024 * 1024
 
@@ -110,6 +110,8 @@ def lib():
             "ct_campaign_batched": [vp, vp, i32, P(FaultDesc), i32, vp, vp, vp, vp],
             "ct_resolve_roles": [P(ModelDesc), P(i32)],
             "ct_reexecute_prepare": [vp, i32],
+            "ct_infer_batches": [vp, i32, i32, P(vp), P(vp), P(vp), P(vp), P(i32), vp],
+            "ct_run_host_batches": [vp, i32, i32, P(vp), P(vp), P(vp), P(vp), P(i32), vp],
         }
         for name, args in sig.items():
             f = getattr(L, name)
@@ -277,6 +279,35 @@ def ct_reexecute(m: Model, input_dev, batch: int, flag_dev, logits_dev, S_dev=No
 def ct_reexecute_prepare(m: Model, max_images: int):
     """Capture the re-execution graphs of every padded size up to max_images."""
     _check(lib().ct_reexecute_prepare(m.handle, max_images), "ct_reexecute_prepare")
+
+
+def _ptr_array(items):
+    """ctypes array of addresses (None entries stay NULL), or None for None."""
+    if items is None:
+        return None
+    return (ctypes.c_void_p * max(len(items), 1))(*[_ptr(t) for t in items])
+
+
+def ct_infer_batches(m: Model, inputs_dev, batch: int, logits_dev, S_dev, flag_dev, stream=None) -> int:
+    """Inference of a list of device-resident batches with each batch's
+    flagged images re-run two batches later (Sec. II-B); returns the images
+    re-run.  Each argument is a list with one device tensor per batch."""
+    n = ctypes.c_int32()
+    _check(lib().ct_infer_batches(m.handle, len(inputs_dev), batch, _ptr_array(inputs_dev), _ptr_array(logits_dev),
+                                  _ptr_array(S_dev), _ptr_array(flag_dev), ctypes.byref(n), _stream(stream)),
+           "ct_infer_batches")
+    return n.value
+
+
+def ct_run_host_batches(m: Model, inputs_host, batch: int, logits_host, S_host=None, flag_host=None,
+                        stream=None) -> int:
+    """ct_infer_batches for host buffers (numpy arrays or pinned CPU tensors):
+    input copies and result copies overlap the device's work."""
+    n = ctypes.c_int32()
+    _check(lib().ct_run_host_batches(m.handle, len(inputs_host), batch, _ptr_array(inputs_host),
+                                     _ptr_array(logits_host), _ptr_array(S_host), _ptr_array(flag_host),
+                                     ctypes.byref(n), _stream(stream)), "ct_run_host_batches")
+    return n.value
 
 
 def ct_infer_reexec(m: Model, input_dev, batch: int, logits_dev, S_dev=None, flag_dev=None,

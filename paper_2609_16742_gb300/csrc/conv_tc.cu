@@ -201,6 +201,50 @@ __device__ __forceinline__ void store_chunk_pre(const float *v, const Res16 &r, 
     yp[1] = make_uint4(packed[4], packed[5], packed[6], packed[7]);
 }
 
+// Fault-free epilogue of 16 channels k0 .. k0 + 15 of one pixel: the same
+// FP32 operations in the same order as store_chunk_pre without a fault
+// ((accumulator + bias) + residual, then ReLU), with the bias read as four
+// 16-byte vectors and ReLU and the FP16 rounding (nearest even) fused into
+// one conversion per channel pair (negative values become +0, NaN stays NaN).
+struct Bias16 {
+    float4 q[4];
+};
+__device__ __forceinline__ Bias16 load_bias16(const float *bias, int k0) {
+    const float4 *p = reinterpret_cast<const float4 *>(bias + k0);
+    Bias16 b;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) b.q[i] = __ldg(p + i);
+    return b;
+}
+__device__ __forceinline__ uint32_t cvt_h2(float lo, float hi, bool relu) {
+    uint32_t r;
+    if (relu) asm("cvt.rn.relu.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+    else asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+    return r;
+}
+__device__ __forceinline__ void store16_fast(const float *v, const Bias16 &b, const Res16 &r, bool res, bool relu,
+                                             __half *dst) {
+    const float *bb = reinterpret_cast<const float *>(b.q);
+    float t[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) t[i] = v[i] + bb[i];
+    if (res) {
+        const __half2 *h0 = reinterpret_cast<const __half2 *>(&r.r0);
+        const __half2 *h1 = reinterpret_cast<const __half2 *>(&r.r1);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float2 f0 = __half22float2(h0[i]), f1 = __half22float2(h1[i]);
+            t[2 * i] += f0.x; t[2 * i + 1] += f0.y; t[8 + 2 * i] += f1.x; t[8 + 2 * i + 1] += f1.y;
+        }
+    }
+    uint32_t pk[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) pk[i] = cvt_h2(t[2 * i], t[2 * i + 1], relu);
+    uint4 *yp = reinterpret_cast<uint4 *>(dst);
+    yp[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+    yp[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+}
+
 // The checksum output of one pixel: carry-through column + coef * incoming
 // checksum (centre pixel, or the sum of an FC layer's checksum features),
 // fault delta, residual checksum, ReLU.
@@ -509,6 +553,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
         const __half *x = static_cast<const __half *>(a.x);
         const FaultDelta fd = a.fd;
         const bool split = g.splits > 1;
+        const bool has_res = a.res != nullptr, relu = a.relu != 0;
         int lt = 0;
         for (int tile = cid; tile < num_items; tile += ncl, ++lt) {
             const TileRef tr = tile_ref(tile, g);
@@ -581,11 +626,18 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
                         *reinterpret_cast<float4 *>(wrow + n0 + half * (BN / 2) + c) =
                             make_float4(vals[c], vals[c + 1], vals[c + 2], vals[c + 3]);
                     if (do_cs) wrow[g.K] = ctv;
-                } else if (valid) {
+                } else if (valid && fd.active) {
 #pragma unroll
                     for (int c = 0; c < BN / 2; c += 16)
                         store_chunk_pre(vals + c, rs[c / 16], a, g.K, (size_t)m, n0 + half * (BN / 2) + c, fsrc);
                     if (do_cs) store_checksum_pre(ctv, csv, a, g, m, fsrc);
+                } else if (valid) {
+                    __half *yrow = static_cast<__half *>(a.y) + (size_t)m * g.K + n0 + half * (BN / 2);
+#pragma unroll
+                    for (int c = 0; c < BN / 2; c += 16)
+                        store16_fast(vals + c, load_bias16(a.bias, n0 + half * (BN / 2) + c), rs[c / 16], has_res,
+                                     relu, yrow + c);
+                    if (do_cs) store_checksum_pre(ctv, csv, a, g, m, 0.f);
                 }
             } else {
 #pragma unroll
@@ -602,8 +654,11 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
                         float4 *wp = reinterpret_cast<float4 *>(a.ws + ((size_t)tr.sp * g.M + m) * g.ws_ld + n0 + c);
 #pragma unroll
                         for (int i = 0; i < 4; ++i) wp[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
-                    } else if (valid) {
+                    } else if (valid && fd.active) {
                         store_chunk_pre(v, rs[(c - half * (BN / 2)) / 16], a, g.K, (size_t)m, n0 + c, fsrc);
+                    } else if (valid) {
+                        store16_fast(v, load_bias16(a.bias, n0 + c), rs[(c - half * (BN / 2)) / 16], has_res, relu,
+                                     static_cast<__half *>(a.y) + (size_t)m * g.K + n0 + c);
                     }
                 }
                 if (do_cs && g.ct_mode != CT_NONE_) ctv = ct_sum[ab * BM + row];
@@ -791,6 +846,7 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
         const float coef = __half2float(__ushort_as_half(g.coef_h));
         const int ctr_r = g.ctr_tap / g.S, ctr_s = g.ctr_tap % g.S;
         const uint32_t pair_empty_even = mapa_shared(smem_u32(pair_empty), 0u);
+        const bool has_res = a.res != nullptr, relu = a.relu != 0;
         int lt = 0;
         for (int item = cid; item < num_items; item += ncl, ++lt) {
             const int m_pair = item / g.n_tiles, n_tile = item % g.n_tiles;
@@ -849,7 +905,10 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
             for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 16) {
                 float v[16];
                 tmem_ld16(trow + c, v);
-                if (valid) store_chunk_pre(v, rs[(c - half * (BN / 2)) / 16], a, g.K, (size_t)m, n0 + c, fsrc);
+                if (valid && fd.active) store_chunk_pre(v, rs[(c - half * (BN / 2)) / 16], a, g.K, (size_t)m, n0 + c, fsrc);
+                else if (valid)
+                    store16_fast(v, load_bias16(a.bias, n0 + c), rs[(c - half * (BN / 2)) / 16], has_res, relu,
+                                 static_cast<__half *>(a.y) + (size_t)m * g.K + n0 + c);
             }
             if (do_cs && valid) store_checksum_pre(ctv, csv, a, g, m, fsrc);
             asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -1180,6 +1239,14 @@ struct HaloR {
     static constexpr int STAGE = (RES + 2 * CS + 1023) / 1024 * 1024;   // swizzle atoms stay 1024-byte aligned
 };
 
+// Resident weights (one channel block, one N tile): tap visit i (the centre
+// tap first) at offset halo_bres_off(i); only the centre tap is followed by
+// the 16 constant carry-through rows.
+template <int BN>
+__host__ __device__ constexpr int halo_bres_off(int i) {
+    return i == 0 ? 0 : (BN + 16) * BK * 2 + (i - 1) * BN * BK * 2;
+}
+
 template <int BN, bool BRES, int NA, int NB, int NR>
 __global__ void __launch_bounds__(NTHREADS, 1)
 conv_tc_halo_kernel(const __grid_constant__ HaloMaps maps, const ConvArgs a, const HaloGeom hg, const TcGeom g) {
@@ -1187,13 +1254,14 @@ conv_tc_halo_kernel(const __grid_constant__ HaloMaps maps, const ConvArgs a, con
     constexpr int B_STAGE = B_ROWS * BK * 2;
     constexpr int B_TMA = BN * BK * 2;
     constexpr int NBS = BRES ? 9 : NB;
+    constexpr int B_AREA = BRES ? halo_bres_off<BN>(9) : NB * B_STAGE;
     constexpr int CH = BN + 16;
     using R = HaloR<BN>;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint8_t *As = smem;
     uint8_t *Bs = As + NA * HT_A_STAGE;
-    uint8_t *Rs = Bs + NBS * B_STAGE;
+    uint8_t *Rs = Bs + B_AREA;
     uint64_t *a_full = (uint64_t *)(Rs + NR * R::STAGE);
     uint64_t *a_empty = a_full + NA;
     uint64_t *b_full = a_empty + NA;
@@ -1240,7 +1308,7 @@ conv_tc_halo_kernel(const __grid_constant__ HaloMaps maps, const ConvArgs a, con
         // row 0 = coef, rows 1..15 = 0 (swizzle-invariant)
         const uint32_t coef2 = (uint32_t)hg.coef_h | ((uint32_t)hg.coef_h << 16);
         const int t = threadIdx.x - 64;
-        for (int sb = 0; sb < NBS; ++sb) {
+        for (int sb = 0; sb < (BRES ? 1 : NBS); ++sb) {
             uint32_t *rows = (uint32_t *)(Bs + sb * B_STAGE + BN * BK * 2);
             for (int i = t; i < 16 * BK / 2; i += 32 * N_EPI_WARPS) rows[i] = (i < BK / 2) ? coef2 : 0u;
         }
@@ -1262,7 +1330,8 @@ conv_tc_halo_kernel(const __grid_constant__ HaloMaps maps, const ConvArgs a, con
             if (BRES) {
                 for (int i = 0; i < 9; ++i) {
                     mbar_arrive_expect_tx(smem_u32(&b_full[i]), B_TMA);
-                    tma_load_2d(smem_u32(Bs + i * B_STAGE), &maps.bmap, smem_u32(&b_full[i]), tap_of(i, 4) * hg.C, 0);
+                    tma_load_2d(smem_u32(Bs + halo_bres_off<BN>(i)), &maps.bmap, smem_u32(&b_full[i]),
+                                tap_of(i, 4) * hg.C, 0);
                 }
             }
         }
@@ -1349,7 +1418,7 @@ conv_tc_halo_kernel(const __grid_constant__ HaloMaps maps, const ConvArgs a, con
                         for (int i = 0; i < 9; ++i) {
                             const int tap = tap_of(i, 4);
                             const uint32_t a_tap = a_base + (uint32_t)(((tap / 3) * HT_PW + tap % 3) * BK * 2);
-                            const uint32_t b_base = b0 + (uint32_t)(i * B_STAGE);
+                            const uint32_t b_base = b0 + (uint32_t)halo_bres_off<BN>(i);
 #pragma unroll
                             for (int k16 = 0; k16 < BK / 16; ++k16) {
                                 const uint64_t ad = smem_desc_sw128_sbo(a_tap + k16 * 32, HT_ROW);
@@ -1404,6 +1473,12 @@ conv_tc_halo_kernel(const __grid_constant__ HaloMaps maps, const ConvArgs a, con
         const int row = quad * 32 + lane;
         const __half *x = static_cast<const __half *>(a.x);
         const FaultDelta fd = a.fd;
+        const bool has_res = hg.res != 0, relu = a.relu != 0;
+        // one N tile: this thread's channels are the same in every tile
+        constexpr int NBIAS = BN <= 64 ? BN / 32 : 1;
+        Bias16 bias_r[NBIAS];
+#pragma unroll
+        for (int c = 0; c < NBIAS; ++c) bias_r[c] = load_bias16(a.bias, half * (BN / 2) + 16 * c);
         int lt = 0;
         for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++lt) {
             const HaloTile ht = halo_tile(tile, hg);
@@ -1468,8 +1543,17 @@ conv_tc_halo_kernel(const __grid_constant__ HaloMaps maps, const ConvArgs a, con
                         else if (a.cs_in) fsrc = ldh(static_cast<const __half *>(a.cs_in), ((size_t)ht.n * hg.H + h) * hg.W + w);
                     }
                 }
+                if (fd.active) {
 #pragma unroll
-                for (int c = 0; c < BN / 2; c += 16) store_chunk_pre(vals + c, rs[c / 16], a, hg.K, (size_t)m, n0 + c, fsrc);
+                    for (int c = 0; c < BN / 2; c += 16)
+                        store_chunk_pre(vals + c, rs[c / 16], a, hg.K, (size_t)m, n0 + c, fsrc);
+                } else {
+                    __half *yrow = static_cast<__half *>(a.y) + (size_t)m * hg.K + n0;
+#pragma unroll
+                    for (int c = 0; c < BN / 2; c += 16)
+                        store16_fast(vals + c, BN <= 64 ? bias_r[(c / 16) % NBIAS] : load_bias16(a.bias, n0 + c),
+                                     rs[c / 16], has_res, relu, yrow + c);
+                }
                 if (do_cs) store_checksum_pre(ctv, csv, a, g, m, fsrc);
             }
         }
@@ -1574,10 +1658,13 @@ TcPlan *tc_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, cons
     int lower[2] = {-a.pad, -a.pad};
     int upper[2] = {a.pad - (a.S - 1), a.pad - (a.R - 1)};
     cuuint32_t estr[4] = {1, (cuuint32_t)a.stride, (cuuint32_t)a.stride, 1};
+    // a strided 1x1 convolution reads every other pixel: 256-byte L2
+    // promotion would also fetch the pixels it skips (64 channels = 128 bytes)
+    const CUtensorMapL2promotion apromo =
+        (a.R == 1 && a.stride > 1) ? CU_TENSOR_MAP_L2_PROMOTION_L2_128B : CU_TENSOR_MAP_L2_PROMOTION_L2_256B;
     CUresult r = g_encode_im2col(&pl->amap, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<void *>(x_dev), gdim, gstr,
                                  lower, upper, BK, BM, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                                 CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+                                 CU_TENSOR_MAP_SWIZZLE_128B, apromo, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) { if (why) *why = "im2col tensor map"; delete pl; return nullptr; }
     // B: weights [K, R*S*C] fp16, K-major rows
     cuuint64_t bdim[2] = {(cuuint64_t)g.RSC, (cuuint64_t)a.K};
@@ -1738,7 +1825,8 @@ struct HaloPlan {
 template <int BN, bool BRES, int NA, int NB, int NR>
 size_t halo_smem() {
     const int nbs = BRES ? 9 : NB;
-    return 1024 + (size_t)NA * HT_A_STAGE + (size_t)nbs * (BN + 16) * BK * 2 + (size_t)NR * HaloR<BN>::STAGE +
+    const size_t b_area = BRES ? (size_t)halo_bres_off<BN>(9) : (size_t)NB * (BN + 16) * BK * 2;
+    return 1024 + (size_t)NA * HT_A_STAGE + b_area + (size_t)NR * HaloR<BN>::STAGE +
            8 * (2 * NA + 2 * nbs + 2 * NR + 4) + 16;
 }
 
@@ -1822,8 +1910,8 @@ HaloPlan *halo_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, 
     cudaError_t e;
     if (pl->BN == 64 && hg.ncb == 1) {
         pl->kind = 0;
-        pl->smem = halo_smem<64, true, 3, 0, 3>();
-        e = cudaFuncSetAttribute(conv_tc_halo_kernel<64, true, 3, 0, 3>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
+        pl->smem = halo_smem<64, true, 4, 0, 3>();
+        e = cudaFuncSetAttribute(conv_tc_halo_kernel<64, true, 4, 0, 3>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
     } else if (pl->BN == 64) {
         pl->kind = 1;
         pl->smem = halo_smem<64, false, 3, 6, 3>();
@@ -1851,7 +1939,7 @@ cudaError_t launch_conv_tc_halo(const ConvArgs &a, const HaloPlan *pl, cudaStrea
     g.M = a.N * a.P * a.Q;
     const int tiles = halo_tiles(pl, a.N);
     dim3 grid(tiles < pl->sms ? tiles : pl->sms);
-    if (pl->kind == 0) pdl_launch(conv_tc_halo_kernel<64, true, 3, 0, 3>, grid, NTHREADS, pl->smem, st, pl->maps, a, hg, g);
+    if (pl->kind == 0) pdl_launch(conv_tc_halo_kernel<64, true, 4, 0, 3>, grid, NTHREADS, pl->smem, st, pl->maps, a, hg, g);
     else if (pl->kind == 1) pdl_launch(conv_tc_halo_kernel<64, false, 3, 6, 3>, grid, NTHREADS, pl->smem, st, pl->maps, a, hg, g);
     else pdl_launch(conv_tc_halo_kernel<128, false, 3, 4, 2>, grid, NTHREADS, pl->smem, st, pl->maps, a, hg, g);
     return cudaGetLastError();

@@ -153,6 +153,19 @@ struct ct_model {
     int n_kernels_last = -1;     // kernels launched by the last inference
     int n_kernels_run = 0;
     std::vector<void *> dev_allocs;
+    // ct_infer_batches / ct_run_host_batches: per pipeline slot a pinned copy
+    // of the batch's flags, a pinned index list, events; a copy stream and
+    // (host buffers) device slots for inputs and results; made on first use
+    static constexpr int PIPE = 6;
+    uint8_t *pipe_flags_h = nullptr;      // [PIPE][max_batch]
+    int32_t *pipe_idx_h = nullptr;        // [PIPE + 2][max_batch]
+    cudaEvent_t pipe_ev_flags[PIPE] = {}, pipe_ev_step[PIPE] = {}, pipe_ev_in[PIPE] = {}, pipe_ev_out[PIPE] = {};
+    cudaEvent_t pipe_ev_tail = nullptr;
+    bool pipe_ready = false;
+    cudaStream_t pipe_copy = nullptr;     // input copies
+    cudaStream_t pipe_copy_out = nullptr; // result copies
+    float *pipe_in_d = nullptr, *pipe_lg_d = nullptr, *pipe_S_d = nullptr;
+    uint8_t *pipe_fl_d = nullptr;
     // profiling
     bool prof = false;
     std::vector<std::pair<cudaEvent_t, cudaEvent_t>> ev_pool;
@@ -206,6 +219,18 @@ void free_all(ct_model *m) {
     m->re_graph.clear();
     if (m->cap_stream) cudaStreamDestroy(m->cap_stream);
     m->cap_stream = nullptr;
+    if (m->pipe_flags_h) cudaFreeHost(m->pipe_flags_h);
+    if (m->pipe_idx_h) cudaFreeHost(m->pipe_idx_h);
+    m->pipe_flags_h = nullptr;
+    m->pipe_idx_h = nullptr;
+    for (int i = 0; i < ct_model::PIPE; ++i)
+        for (cudaEvent_t *e : {&m->pipe_ev_flags[i], &m->pipe_ev_step[i], &m->pipe_ev_in[i], &m->pipe_ev_out[i]})
+            if (*e) { cudaEventDestroy(*e); *e = nullptr; }
+    if (m->pipe_ev_tail) cudaEventDestroy(m->pipe_ev_tail);
+    m->pipe_ev_tail = nullptr;
+    if (m->pipe_copy) cudaStreamDestroy(m->pipe_copy);
+    if (m->pipe_copy_out) cudaStreamDestroy(m->pipe_copy_out);
+    m->pipe_copy = m->pipe_copy_out = nullptr;
 }
 
 // store a double as the storage word (fp32 or fp16) into a byte buffer
@@ -902,24 +927,26 @@ cudaGraphExec_t reexec_graph(ct_model *m, int bucket) {
     return ex;
 }
 
-ct_status reexec_impl(ct_model *m, const float *input, int batch, const uint8_t *flag, float *logits,
-                      float *S, int *n_rerun, cudaStream_t st) {
-    CUDA_TRY(cudaMemcpyAsync(m->h_flags, flag, batch, cudaMemcpyDeviceToHost, st));
-    CUDA_TRY(cudaStreamSynchronize(st));
+// Re-execution of the images whose host-side flag is set (Sec. II-B, last
+// paragraph): gather them into a batch of their own, padded to a power of
+// two (at most max_batch) by repeating the last one, run it fault-free
+// (graph replay, or direct launches when profiling) and scatter the first n
+// rows back.  idx_host: a pinned index buffer of max_batch entries that no
+// copy still in flight reads.
+ct_status reexec_rows(ct_model *m, const float *input, int batch, const uint8_t *flags_host, float *logits,
+                      float *S, int *n_rerun, int32_t *idx_host, cudaStream_t st) {
     int n = 0;
     for (int i = 0; i < batch; ++i)
-        if (m->h_flags[i]) m->h_idx[n++] = i;
+        if (flags_host[i]) idx_host[n++] = i;
     if (n_rerun) *n_rerun = n;
     if (n == 0) return CT_OK;
-    // the re-run batch is padded to a power of two (at most max_batch) by
-    // repeating the last flagged image; only the first n rows are scattered
-    // back.  Each bucket size has its own graph slot (ceil log2), and
-    // max_batch is the only size in the last slot.
+    // each bucket size has its own graph slot (ceil log2); max_batch is the
+    // only size in the last slot
     int bucket = 1;
     while (bucket < n) bucket <<= 1;
     if (bucket > m->max_batch) bucket = m->max_batch;
-    for (int i = n; i < bucket; ++i) m->h_idx[i] = m->h_idx[n - 1];
-    CUDA_TRY(cudaMemcpyAsync(m->re_idx, m->h_idx, sizeof(int32_t) * bucket, cudaMemcpyHostToDevice, st));
+    for (int i = n; i < bucket; ++i) idx_host[i] = idx_host[n - 1];
+    CUDA_TRY(cudaMemcpyAsync(m->re_idx, idx_host, sizeof(int32_t) * bucket, cudaMemcpyHostToDevice, st));
     const int64_t per = (int64_t)m->in_c * m->in_h * m->in_w;
     CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] { return launch_gather_images(input, m->re_input, m->re_idx, bucket, per, st); }));
     // fault-free re-run: an armed fault stays armed for the next ct_infer
@@ -942,31 +969,43 @@ ct_status reexec_impl(ct_model *m, const float *input, int batch, const uint8_t 
     return CT_OK;
 }
 
-// Inference of `batch` new images with the previous batch's flagged images
-// re-executed as extra rows of the same launch sequence (Sec. II-B): their
-// cost is that of the extra images, not of a separate small-batch pass.
-// Falls back to reexec_impl + infer_impl when a fault is armed (the re-run
-// must be fault-free) or the rows do not fit max_batch.
-ct_status infer_reexec_impl(ct_model *m, const float *input, int batch, float *logits, float *S, uint8_t *flag,
-                            const float *prev_input, int prev_batch, const uint8_t *prev_flag, float *prev_logits,
-                            float *prev_S, int *n_rerun, cudaStream_t st) {
-    if (n_rerun) *n_rerun = 0;
-    if (!prev_input || prev_batch == 0) return infer_impl(m, input, batch, logits, S, flag, st);
-    CUDA_TRY(cudaMemcpyAsync(m->h_flags, prev_flag, prev_batch, cudaMemcpyDeviceToHost, st));
+// the device flags of a finished inference, read on the host (one stream synchronisation)
+ct_status read_flags(ct_model *m, const uint8_t *flag, int batch, cudaStream_t st) {
+    CUDA_TRY(cudaMemcpyAsync(m->h_flags, flag, batch, cudaMemcpyDeviceToHost, st));
     CUDA_TRY(cudaStreamSynchronize(st));
+    return CT_OK;
+}
+
+ct_status reexec_impl(ct_model *m, const float *input, int batch, const uint8_t *flag, float *logits,
+                      float *S, int *n_rerun, cudaStream_t st) {
+    ct_status s = read_flags(m, flag, batch, st);
+    if (s != CT_OK) return s;
+    return reexec_rows(m, input, batch, m->h_flags, logits, S, n_rerun, m->h_idx, st);
+}
+
+// Inference of `batch` new images with the flagged images of a previous
+// batch (host-side flags) re-executed as extra rows of the same launch
+// sequence (Sec. II-B): their cost is that of the extra images, not of a
+// separate small-batch pass.  Falls back to reexec_rows + infer_impl when a
+// fault is armed (the re-run must be fault-free) or the rows do not fit
+// max_batch.  idx_host as for reexec_rows.
+ct_status infer_with_reruns(ct_model *m, const float *input, int batch, float *logits, float *S, uint8_t *flag,
+                            const float *prev_input, int prev_batch, const uint8_t *prev_flags_host,
+                            float *prev_logits, float *prev_S, int *n_rerun, int32_t *idx_host, cudaStream_t st) {
+    if (n_rerun) *n_rerun = 0;
     int n = 0;
     for (int i = 0; i < prev_batch; ++i)
-        if (m->h_flags[i]) m->h_idx[n++] = i;
+        if (prev_flags_host[i]) idx_host[n++] = i;
     if (n == 0) return infer_impl(m, input, batch, logits, S, flag, st);
     if (m->armed || batch + n > m->max_batch) {
         int nr = 0;
-        ct_status s = reexec_impl(m, prev_input, prev_batch, prev_flag, prev_logits, prev_S, &nr, st);
+        ct_status s = reexec_rows(m, prev_input, prev_batch, prev_flags_host, prev_logits, prev_S, &nr, idx_host, st);
         if (s != CT_OK) return s;
         if (n_rerun) *n_rerun = nr;
         return infer_impl(m, input, batch, logits, S, flag, st);
     }
     if (n_rerun) *n_rerun = n;
-    CUDA_TRY(cudaMemcpyAsync(m->re_idx, m->h_idx, sizeof(int32_t) * n, cudaMemcpyHostToDevice, st));
+    CUDA_TRY(cudaMemcpyAsync(m->re_idx, idx_host, sizeof(int32_t) * n, cudaMemcpyHostToDevice, st));
     const int64_t per = (int64_t)m->in_c * m->in_h * m->in_w;
     CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] { return launch_gather_images(prev_input, m->re_input, m->re_idx, n, per, st); }));
     const int tot = batch + n;
@@ -980,6 +1019,216 @@ ct_status infer_reexec_impl(ct_model *m, const float *input, int batch, float *l
         return launch_scatter_rows(m->re_logits + (size_t)batch * m->n_classes, prev_logits, m->re_idx, n, m->n_classes, st);
     }));
     if (prev_S) CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] { return launch_scatter_rows(m->re_S + batch, prev_S, m->re_idx, n, 1, st); }));
+    return CT_OK;
+}
+
+ct_status infer_reexec_impl(ct_model *m, const float *input, int batch, float *logits, float *S, uint8_t *flag,
+                            const float *prev_input, int prev_batch, const uint8_t *prev_flag, float *prev_logits,
+                            float *prev_S, int *n_rerun, cudaStream_t st) {
+    if (n_rerun) *n_rerun = 0;
+    if (!prev_input || prev_batch == 0) return infer_impl(m, input, batch, logits, S, flag, st);
+    ct_status s = read_flags(m, prev_flag, prev_batch, st);
+    if (s != CT_OK) return s;
+    return infer_with_reruns(m, input, batch, logits, S, flag, prev_input, prev_batch, m->h_flags, prev_logits, prev_S,
+                             n_rerun, m->h_idx, st);
+}
+
+// Re-execution of the flagged images of nb <= 2 batches (host flags) as one
+// padded batch: each batch's images are gathered after the previous ones'
+// and their rows scattered back to that batch's outputs.  idx_host holds
+// 2 * max_batch entries that no copy in flight reads.  When the combined
+// count exceeds max_batch, each batch is re-run on its own.
+template <typename In, typename Fl, typename Lg, typename Sv>
+ct_status reexec_rows_of(ct_model *m, int nb, In in, Fl fl, Lg lg, Sv Sp, int batch, int *n_rerun, int32_t *idx_host,
+                         cudaStream_t st) {
+    int tot = 0;
+    for (int j = 0; j < nb; ++j)
+        for (int i = 0; i < batch; ++i) tot += fl(j)[i] ? 1 : 0;
+    if (n_rerun) *n_rerun = tot;
+    if (tot == 0) return CT_OK;
+    if (nb == 1 || tot > m->max_batch) {
+        for (int j = 0; j < nb; ++j) {
+            int nr = 0;
+            ct_status s = reexec_rows(m, in(j), batch, fl(j), lg(j), Sp(j), &nr, idx_host + (size_t)j * m->max_batch, st);
+            if (s != CT_OK) return s;
+        }
+        return CT_OK;
+    }
+    int bucket = 1;
+    while (bucket < tot) bucket <<= 1;
+    if (bucket > m->max_batch) bucket = m->max_batch;
+    // gather lists: per batch its own flagged indices, then the padded combined list
+    const int64_t per = (int64_t)m->in_c * m->in_h * m->in_w;
+    int32_t *lists = idx_host;                     // [nb][<= batch] flagged indices
+    int off = 0;
+    std::vector<int> cnt(nb);
+    for (int j = 0; j < nb; ++j) {
+        int c = 0;
+        for (int i = 0; i < batch; ++i)
+            if (fl(j)[i]) lists[off + c++] = i;
+        cnt[j] = c;
+        off += c;
+    }
+    CUDA_TRY(cudaMemcpyAsync(m->re_idx, lists, sizeof(int32_t) * tot, cudaMemcpyHostToDevice, st));
+    // rows [o_j, o_j + cnt_j) of the re-run batch: batch j's images; padding repeats the last one
+    for (int j = 0, o = 0; j < nb; o += cnt[j], ++j) {
+        if (!cnt[j]) continue;
+        const int c = cnt[j];
+        float *dst = m->re_input + (size_t)o * per;
+        CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] { return launch_gather_images(in(j), dst, m->re_idx + o, c, per, st); }));
+    }
+    for (int r = tot; r < bucket; ++r)           // padding: copies of the last gathered image
+        CUDA_TRY(cudaMemcpyAsync(m->re_input + (size_t)r * per, m->re_input + (size_t)(tot - 1) * per,
+                                 sizeof(float) * per, cudaMemcpyDeviceToDevice, st));
+    const bool armed = m->armed;
+    m->armed = false;
+    ct_status s = CT_OK;
+    cudaGraphExec_t ex = m->prof ? nullptr : reexec_graph(m, bucket);
+    if (ex) {
+        int slot = 0;
+        while ((1 << slot) < bucket) ++slot;
+        if (cudaGraphLaunch(ex, st) != cudaSuccess) s = CT_ECUDA;
+        else m->kernels_total += m->re_graph_nk[slot];
+    } else {
+        s = infer_impl(m, m->re_input, bucket, m->re_logits, m->re_S, m->re_flag, st);
+    }
+    m->armed = armed;
+    if (s != CT_OK) return s;
+    for (int j = 0, o = 0; j < nb; o += cnt[j], ++j) {
+        if (!cnt[j]) continue;
+        const int c = cnt[j];
+        float *L = lg(j), *Sj = Sp(j);
+        CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] {
+            return launch_scatter_rows(m->re_logits + (size_t)o * m->n_classes, L, m->re_idx + o, c, m->n_classes, st);
+        }));
+        if (Sj) CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] { return launch_scatter_rows(m->re_S + o, Sj, m->re_idx + o, c, 1, st); }));
+    }
+    return CT_OK;
+}
+
+// Pipeline resources of ct_infer_batches / ct_run_host_batches, made on the
+// first call (host slots only for the host-buffer call).
+ct_status pipe_setup(ct_model *m, bool host) {
+    if (!m->pipe_ready) {
+        const size_t B = (size_t)m->max_batch;
+        if (cudaMallocHost((void **)&m->pipe_flags_h, ct_model::PIPE * B) != cudaSuccess ||
+            cudaMallocHost((void **)&m->pipe_idx_h, sizeof(int32_t) * (ct_model::PIPE + 2) * B) != cudaSuccess) {
+            cudaGetLastError();
+            return CT_ENOMEM;
+        }
+        for (int i = 0; i < ct_model::PIPE; ++i)
+            for (cudaEvent_t *e : {&m->pipe_ev_flags[i], &m->pipe_ev_step[i], &m->pipe_ev_in[i], &m->pipe_ev_out[i]})
+                CUDA_TRY(cudaEventCreateWithFlags(e, cudaEventDisableTiming));
+        CUDA_TRY(cudaEventCreateWithFlags(&m->pipe_ev_tail, cudaEventDisableTiming));
+        CUDA_TRY(cudaStreamCreateWithFlags(&m->pipe_copy, cudaStreamNonBlocking));
+        CUDA_TRY(cudaStreamCreateWithFlags(&m->pipe_copy_out, cudaStreamNonBlocking));
+        m->pipe_ready = true;
+    }
+    if (host && !m->pipe_in_d) {
+        const size_t B = (size_t)m->max_batch, per = (size_t)m->in_c * m->in_h * m->in_w;
+        ct_status st;
+        if ((st = dalloc(m, (void **)&m->pipe_in_d, sizeof(float) * ct_model::PIPE * B * per)) != CT_OK ||
+            (st = dalloc(m, (void **)&m->pipe_lg_d, sizeof(float) * ct_model::PIPE * B * m->n_classes)) != CT_OK ||
+            (st = dalloc(m, (void **)&m->pipe_S_d, sizeof(float) * ct_model::PIPE * B)) != CT_OK ||
+            (st = dalloc(m, (void **)&m->pipe_fl_d, ct_model::PIPE * B)) != CT_OK)
+            return st;
+    }
+    return CT_OK;
+}
+
+// Buffers of one call of ct_infer_batches (device) or ct_run_host_batches (host).
+struct BatchIO {
+    const float *const *in;
+    float *const *lg;
+    float *const *S;
+    uint8_t *const *fl;
+};
+
+// n batches of `batch` images with the re-execution of Sec. II-B deferred by
+// two batches: step i infers batch i and re-runs, as extra rows of the same
+// inference, the flagged images of batch i - 2.  The flags of every batch
+// are copied to pinned host memory when its inference ends, and the host
+// waits for batch i - 2's copy before it launches step i; the device is then
+// working on batch i - 1, so the wait does not idle it, and the host stays
+// at most two batches ahead.  Host buffers: batch i's input is copied into
+// device slot i % PIPE on a copy stream (overlapping the device's work on
+// earlier batches) and batch i's results are copied back once its re-run
+// rows are written (after step i + 2).  The last two batches' flagged
+// images are re-run on their own at the end.  Returns after every result is
+// final (and, for host buffers, copied back).
+ct_status run_batches(ct_model *m, int n, int batch, const BatchIO &io, bool host, int *n_rerun, cudaStream_t st) {
+    constexpr int P = ct_model::PIPE;
+    const size_t B = (size_t)m->max_batch, per = (size_t)m->in_c * m->in_h * m->in_w, nc = (size_t)m->n_classes;
+    const cudaStream_t cs = m->pipe_copy, co = m->pipe_copy_out;   // inputs in, results out
+    int reruns = 0;
+    auto dev_in = [&](int i) -> const float * { return host ? m->pipe_in_d + (size_t)(i % P) * B * per : io.in[i]; };
+    auto dev_lg = [&](int i) -> float * { return host ? m->pipe_lg_d + (size_t)(i % P) * B * nc : io.lg[i]; };
+    auto dev_S = [&](int i) -> float * { return host ? m->pipe_S_d + (size_t)(i % P) * B : io.S[i]; };
+    auto dev_fl = [&](int i) -> uint8_t * { return host ? m->pipe_fl_d + (size_t)(i % P) * B : io.fl[i]; };
+    auto copy_out = [&](int i) -> ct_status {       // host: results of batch i (co waits for them first)
+        const int q = i % P;
+        CUDA_TRY(cudaMemcpyAsync(io.lg[i], dev_lg(i), sizeof(float) * nc * batch, cudaMemcpyDeviceToHost, co));
+        if (io.S && io.S[i]) CUDA_TRY(cudaMemcpyAsync(io.S[i], dev_S(i), sizeof(float) * batch, cudaMemcpyDeviceToHost, co));
+        if (io.fl && io.fl[i]) CUDA_TRY(cudaMemcpyAsync(io.fl[i], dev_fl(i), batch, cudaMemcpyDeviceToHost, co));
+        CUDA_TRY(cudaEventRecord(m->pipe_ev_out[q], co));
+        return CT_OK;
+    };
+    for (int i = 0; i < n; ++i) {
+        const int s = i % P;
+        if (host) {
+            // slot s last held batch i - P: its input was last read by step i - P + 2
+            // (the re-run gather) and its results were copied out after that step
+            if (i >= P) CUDA_TRY(cudaStreamWaitEvent(cs, m->pipe_ev_step[(i - P + 2) % P], 0));
+            CUDA_TRY(cudaMemcpyAsync(const_cast<float *>(dev_in(i)), io.in[i], sizeof(float) * per * batch,
+                                     cudaMemcpyHostToDevice, cs));
+            CUDA_TRY(cudaEventRecord(m->pipe_ev_in[s], cs));
+            CUDA_TRY(cudaStreamWaitEvent(st, m->pipe_ev_in[s], 0));
+            if (i >= P) CUDA_TRY(cudaStreamWaitEvent(st, m->pipe_ev_out[s], 0));
+        }
+        ct_status r;
+        int nr = 0;
+        if (i >= 2) {
+            const int q = (i - 2) % P;
+            CUDA_TRY(cudaEventSynchronize(m->pipe_ev_flags[q]));
+            r = infer_with_reruns(m, dev_in(i), batch, dev_lg(i), dev_S(i), dev_fl(i), dev_in(i - 2), batch,
+                                  m->pipe_flags_h + (size_t)q * B, dev_lg(i - 2), dev_S(i - 2), &nr,
+                                  m->pipe_idx_h + (size_t)s * B, st);
+        } else {
+            r = infer_impl(m, dev_in(i), batch, dev_lg(i), dev_S(i), dev_fl(i), st);
+        }
+        if (r != CT_OK) return r;
+        reruns += nr;
+        CUDA_TRY(cudaMemcpyAsync(m->pipe_flags_h + (size_t)s * B, dev_fl(i), batch, cudaMemcpyDeviceToHost, st));
+        CUDA_TRY(cudaEventRecord(m->pipe_ev_flags[s], st));
+        CUDA_TRY(cudaEventRecord(m->pipe_ev_step[s], st));
+        if (host && i >= 2) {
+            CUDA_TRY(cudaStreamWaitEvent(co, m->pipe_ev_step[s], 0));
+            ct_status c = copy_out(i - 2);
+            if (c != CT_OK) return c;
+        }
+    }
+    // the last two batches: their flagged images re-run together, one batch
+    const int k0 = n >= 2 ? n - 2 : 0;
+    for (int k = k0; k < n; ++k) CUDA_TRY(cudaEventSynchronize(m->pipe_ev_flags[k % P]));
+    int nr = 0;
+    ct_status r = reexec_rows_of(m, n - k0, [&](int j) { return dev_in(k0 + j); },
+                                 [&](int j) { return (const uint8_t *)(m->pipe_flags_h + (size_t)((k0 + j) % P) * B); },
+                                 [&](int j) { return dev_lg(k0 + j); }, [&](int j) { return dev_S(k0 + j); }, batch, &nr,
+                                 m->pipe_idx_h + (size_t)P * B, st);
+    if (r != CT_OK) return r;
+    reruns += nr;
+    if (host) {
+        CUDA_TRY(cudaEventRecord(m->pipe_ev_tail, st));
+        CUDA_TRY(cudaStreamWaitEvent(co, m->pipe_ev_tail, 0));
+        for (int k = k0; k < n; ++k) {
+            ct_status c = copy_out(k);
+            if (c != CT_OK) return c;
+        }
+        CUDA_TRY(cudaStreamSynchronize(cs));
+        CUDA_TRY(cudaStreamSynchronize(co));
+    }
+    CUDA_TRY(cudaStreamSynchronize(st));
+    if (n_rerun) *n_rerun = reruns;
     return CT_OK;
 }
 
@@ -1261,6 +1510,44 @@ ct_status ct_campaign_batched(ct_model *m, const float *input_dev, int32_t batch
         return launch_campaign_small(g, m->camp_d, n_faults, S_dev, top1_dev, flag_dev, st);
     }));
     return CT_OK;
+}
+
+ct_status ct_infer_batches(ct_model *m, int32_t n_batches, int32_t batch, const float *const *input_dev,
+                           float *const *logits_dev, float *const *S_dev, uint8_t *const *flag_dev, int32_t *n_rerun,
+                           void *stream) {
+    if (n_rerun) *n_rerun = 0;
+    if (!m || n_batches < 0 || (n_batches > 0 && (!input_dev || !logits_dev || !S_dev || !flag_dev))) return CT_EINVAL;
+    if (batch < 1 || batch > m->max_batch) return CT_ERANGE;
+    for (int i = 0; i < n_batches; ++i)
+        if (!input_dev[i] || !logits_dev[i] || !S_dev[i] || !flag_dev[i]) return CT_EINVAL;
+    if (n_batches == 0) return CT_OK;
+    DeviceGuard g(m->device);
+    ct_status s = pipe_setup(m, false);
+    if (s != CT_OK) return s;
+    int nr = 0;
+    s = run_batches(m, n_batches, batch, BatchIO{input_dev, logits_dev, S_dev, flag_dev}, false, &nr,
+                    (cudaStream_t)stream);
+    if (n_rerun) *n_rerun = nr;
+    return s;
+}
+
+ct_status ct_run_host_batches(ct_model *m, int32_t n_batches, int32_t batch, const float *const *input_host,
+                              float *const *logits_host, float *const *S_host, uint8_t *const *flag_host,
+                              int32_t *n_rerun, void *stream) {
+    if (n_rerun) *n_rerun = 0;
+    if (!m || n_batches < 0 || (n_batches > 0 && (!input_host || !logits_host))) return CT_EINVAL;
+    if (batch < 1 || batch > m->max_batch) return CT_ERANGE;
+    for (int i = 0; i < n_batches; ++i)
+        if (!input_host[i] || !logits_host[i]) return CT_EINVAL;
+    if (n_batches == 0) return CT_OK;
+    DeviceGuard g(m->device);
+    ct_status s = pipe_setup(m, true);
+    if (s != CT_OK) return s;
+    int nr = 0;
+    s = run_batches(m, n_batches, batch, BatchIO{input_host, logits_host, S_host, flag_host}, true, &nr,
+                    (cudaStream_t)stream);
+    if (n_rerun) *n_rerun = nr;
+    return s;
 }
 
 ct_status ct_run_host(ct_model *m, const float *input_host, int32_t batch, float *logits_host,

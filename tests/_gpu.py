@@ -80,3 +80,29 @@ def kept_checksum_pixel(net, x1, slot, n_ds=3):
     kept[::2 ** n_ds, ::2 ** n_ds] = True
     pix = int(np.argmax(np.where(kept, cs, -1.0)))
     return pix, float(cs.reshape(-1)[pix])
+
+
+def ulp16(x):
+    """Spacing of binary16 values at |x| (normal range; 2**-24 below it)."""
+    a = np.abs(np.asarray(x, dtype=np.float64))
+    e = np.floor(np.log2(np.maximum(a, 2.0 ** -14)))
+    return 2.0 ** (e - 10)
+
+
+def near_threshold(S_o, r, tau, prec, S_g=None):
+    """Images on which the GPU and the oracle may legitimately decide
+    differently: the oracle's S lies within 1% of tau of the threshold (the
+    stated band), or -- FP16 storage only -- the two S values fall on opposite
+    sides of the threshold while differing by at most two binary16 ulps of S.
+    With FP16 storage S is an FP32 sum of FP16-rounded features, the largest
+    of which (the carried checksum) is close to S itself; two correct
+    implementations that accumulate in different orders can round it one ulp
+    apart (16 at S ~ 3.2e4 on VGG-16, against 1% of tau ~ 1.4)."""
+    S_o = np.asarray(S_o, dtype=np.float64)
+    near = np.isfinite(S_o) & (np.abs(np.abs(S_o - r) - tau) <= 0.01 * tau)
+    if prec == "fp16" and S_g is not None:
+        S_g = np.asarray(S_g, dtype=np.float64)
+        import oracle
+        straddle = oracle.verdict(S_g, r, tau) != oracle.verdict(S_o, r, tau)
+        near |= np.isfinite(S_o) & np.isfinite(S_g) & straddle & (np.abs(S_g - S_o) <= 2.0 * ulp16(S_o))
+    return near

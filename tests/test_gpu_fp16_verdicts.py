@@ -2,18 +2,21 @@
 VGG-16, batch 64): every row's logits and S against the oracle, and the
 per-image verdict of Sec. II-B (flag = NOT(|S - r| <= tau)) identical on
 both sides for one shared (r, tau), fault-free and under seeded single-bit
-flips (Sec. III-A).  Images whose oracle S lies within 1% of tau of the
-threshold (| |S - r| - tau | <= 0.01 tau) are counted separately as
-near-threshold, not compared: FP16 storage moves S by up to the 2e-2
-relative tolerance, which at these S values (~7e3 against tau ~90) is more
-than tau itself."""
+flips (Sec. III-A).  The GPU's flag is the rule applied to its own S, on
+every image.  Near-threshold images are counted separately, not compared:
+the oracle's S within 1% of tau of the threshold, or the two S values on
+opposite sides of it while at most two binary16 ulps apart -- with FP16
+storage S is an FP32 sum of FP16-rounded features, the largest of which
+(the carried checksum) is near S itself, so two correct implementations can
+round it one ulp apart (16 at S ~ 3.2e4 on VGG-16, against 1% of tau ~
+1.4).  Their number is bounded and reported."""
 import numpy as np
 import pytest
 
 import oracle
 import synth
 from _cache import inputs
-from _gpu import TOL, assert_parity, ct, model, onet, run, same_class
+from _gpu import TOL, assert_parity, ct, model, near_threshold, onet, run, same_class
 
 pytestmark = pytest.mark.gpu
 
@@ -23,7 +26,9 @@ CASES = {"resnet18_imagenet": {"calib": 64, "weight_imgs": 8, "faults": 6},
 
 def _verdicts_agree(S_g, flag_g, S_o, r, tau, what):
     """Identical verdicts except near-threshold images; returns (compared, near)."""
-    near = np.isfinite(S_o) & (np.abs(np.abs(S_o - r) - tau) <= 0.01 * tau)
+    own = oracle.verdict(S_g, r, tau)
+    assert (flag_g.astype(bool) == own).all(), (what, np.nonzero(flag_g.astype(bool) != own)[0][:8])
+    near = near_threshold(S_o, r, tau, "fp16", S_g)
     want = oracle.verdict(S_o, r, tau)
     bad = np.nonzero((flag_g.astype(bool) != want) & ~near)[0]
     assert bad.size == 0, (what, bad[:8], S_g[bad[:8]], S_o[bad[:8]], r, tau)
@@ -54,7 +59,7 @@ def test_fp16_logits_and_verdicts_every_row(name):
         c, nn = _verdicts_agree(S, flag, o["S"], rr, tt, name)
         n_cmp += c
         n_near += nn
-    assert n_cmp >= 2 * B - 4, (n_cmp, n_near)
+    assert n_cmp + n_near == 2 * B and n_near <= max(3, 2 * B // 50), (n_cmp, n_near)
 
     # seeded single-bit flips over the literal layout's conv weights and
     # conv-input activations; a weight flip is compared on the first images,

@@ -57,7 +57,8 @@ def layer_errors(name, prec, batch, simt_only=False, first=0):
     ("resnet18_imagenet", "fp16", 8, False),
     ("resnet18_cifar", "fp16", 20, False),
     ("vgg16", "fp16", 2, False),
-    # a batch whose N = 128 / 256 layers run in clusters that share weight tiles
+    # a batch whose N = 128 layers fill the GPU with im2col tiles and whose
+    # N = 256 layers run on CTA pairs
     ("resnet18_cifar", "fp16", 160, False),
 ])
 def test_every_stored_tensor_matches_oracle(name, prec, batch, simt_only):
