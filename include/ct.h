@@ -106,6 +106,8 @@ typedef struct {
 
 /* flags for ct_build_opts.flags */
 #define CT_FLAG_SIMT_ONLY 1u      /* use the CUDA-core conv kernels everywhere */
+#define CT_FLAG_LAYERWISE 2u      /* one kernel per layer even where the whole network
+                                     fits one kernel (the LeNet-5 shape, FP32) */
 
 /* ct_build_opts.protect: how the scheme of Sec. II-A is built in.
  *   CT_PROTECT_NONE     the network as described (the unprotected baseline);
@@ -172,6 +174,16 @@ ct_status ct_resolve_roles(const ct_model_desc *desc, int32_t *roles);
  * 4 channels with 64 filters, followed by a 3x3 stride-2 padding-1 max-pool
  * that is its only reader, runs as one fused kernel: the FP16 copy of the
  * image and the unpooled convolution output are then never stored.
+ * An FP32 network of the LeNet-5 shape (conv, 2x2 max-pool, conv, 2x2
+ * max-pool, three FC layers; widened or unprotected) runs as ONE kernel
+ * whose CTAs take one image each through the whole network in shared
+ * memory; an armed fault is applied inside it (its intermediate tensors are
+ * then not stored, and a fault in the image is rejected with CT_ERANGE).
+ * CT_FLAG_LAYERWISE keeps one kernel per layer.
+ * With FP16 storage, a stride-1 3x3 convolution followed by a 2x2 stride-2
+ * max-pool that is its only reader applies the pool in its epilogue (data
+ * and checksum channels together) whenever it runs on halo tiles (batches
+ * that fill the GPU with them): its unpooled output is then not stored.
  * Roles are resolved and checked by the rule of ct_resolve_roles first,
  * before any device is touched.
  * Synchronous.  On success *out owns device memory until ct_destroy.
@@ -453,7 +465,8 @@ ct_status ct_kernel_count(ct_model *m, int64_t *n);
  * first with data_host = NULL to query).  Synchronous.  CT_ERANGE for a slot
  * that is not kept (the classifier output) or batch > max_batch; CT_ESTATE
  * for a tensor that a fused kernel computes without storing (slot 0 and the
- * unpooled stem output of a model with a fused stem). */
+ * unpooled stem output of a model with a fused stem; the unpooled output of
+ * a convolution whose max-pool ran in its kernel in the last inference). */
 ct_status ct_copy_activation(ct_model *m, int32_t slot, int32_t batch, void *data_host, void *cs_host,
                              int32_t *C, int32_t *H, int32_t *W, int32_t *has_cs,
                              int32_t *elem_bytes, void *stream);

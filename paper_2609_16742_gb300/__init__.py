@@ -27,6 +27,7 @@ CT_BUF_WEIGHT, CT_BUF_ACT = 0, 1
 CT_DS_PASS, CT_DS_ZERO = 0, 1
 CT_PROTECT_NONE, CT_PROTECT_WIDEN, CT_PROTECT_REPLACE = 0, 1, 2
 CT_FLAG_SIMT_ONLY = 1
+CT_FLAG_LAYERWISE = 2
 FAM_TC, FAM_SIMT, FAM_FC, FAM_POOL, FAM_OTHER = 0, 1, 2, 3, 4
 
 _STATUS = {0: "CT_OK", 1: "CT_EINVAL", 2: "CT_ENOMEM", 3: "CT_ECUDA", 4: "CT_ESTATE",
@@ -210,11 +211,12 @@ def ct_resolve_roles(layers: Sequence, in_shape, n_classes: int) -> List[Optiona
 def ct_build(layers: Sequence, params: Sequence[dict], in_shape, n_classes: int,
              precision: str = "fp32", protect: bool = True, ds_mode: str = "pass",
              device: int = 0, max_batch: int = 64, simt_only: bool = False,
-             bn_eps: float = 1e-5, replace: bool = False) -> Model:
+             bn_eps: float = 1e-5, replace: bool = False, layerwise: bool = False) -> Model:
     """Build a model from synth-style layers and float32 parameter dicts.
 
     protect=True adds the carry-through filters as extra channels (widened);
-    replace=True builds the paper's prune-and-replace construction instead."""
+    replace=True builds the paper's prune-and-replace construction instead;
+    layerwise=True keeps one kernel per layer for the LeNet-5 shape."""
     n = len(layers)
     arr = _layer_descs(layers)
     keep = []
@@ -229,7 +231,7 @@ def ct_build(layers: Sequence, params: Sequence[dict], in_shape, n_classes: int,
     mode = CT_PROTECT_REPLACE if replace else (CT_PROTECT_WIDEN if protect else CT_PROTECT_NONE)
     opts = BuildOpts(CT_FP16 if precision == "fp16" else CT_FP32, mode,
                      CT_DS_ZERO if ds_mode == "zero" else CT_DS_PASS, device, max_batch,
-                     CT_FLAG_SIMT_ONLY if simt_only else 0)
+                     (CT_FLAG_SIMT_ONLY if simt_only else 0) | (CT_FLAG_LAYERWISE if layerwise else 0))
     h = ctypes.c_void_p()
     _check(lib().ct_build(ctypes.byref(desc), wp, ctypes.byref(opts), ctypes.byref(h)), "ct_build")
     return Model(h.value, n_classes, in_shape, precision, protect or replace, max_batch)

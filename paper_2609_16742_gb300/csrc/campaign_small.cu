@@ -1,5 +1,8 @@
-// Batched fault-injection campaign for small networks (Sec. III-A): one
-// launch evaluates many single-bit faults.  CTA (f, y) runs fault f on images
+// Whole-network kernel for small networks (the LeNet-5 shape), used two ways:
+// inference of a batch (ct_infer on such a model: one launch instead of one
+// per layer, with any armed fault applied inside the kernel), and the
+// batched fault-injection campaign of Sec. III-A (ct_campaign_batched: one
+// launch evaluates many single-bit faults).  CTA (f, y) runs fault f on images
 // y * ipc .. y * ipc + ipc - 1 of a fixed batch through the whole protected
 // network in shared memory: conv -> ReLU -> 2x2 max-pool -> conv -> ReLU ->
 // 2x2 max-pool -> FC -> ReLU -> FC -> ReLU -> FC (the LeNet-5 shape), FP32,
@@ -77,13 +80,25 @@ __host__ __device__ inline SmLayout sm_layout(const SmallNet &g) {
     return L;
 }
 
-__global__ void __launch_bounds__(256) campaign_small_kernel(const SmallNet g, const CampFault *faults, int ipc,
-                                                              float *S_out, int32_t *top1_out, uint8_t *flag_out) {
+// faults == null: inference -- one fault, `single` (kind 2: none), and every
+// image of the batch is computed (an activation fault changes only its
+// image); rows B .. B + rr.n - 1 are the re-run list: image rr.idx[j] of
+// rr.x, whose logits and S go to row rr.idx[j] of rr.logits / rr.S (no
+// flag).  logits_out, top1_out may be null.  Without protection
+// (g.protect == 0) no checksum channel or neuron is computed, S is NaN and
+// the flag 0, as for the per-layer kernels.
+__global__ void __launch_bounds__(1024) campaign_small_kernel(const SmallNet g, const CampFault *faults,
+                                                               const CampFault single, int ipc, float *S_out,
+                                                               int32_t *top1_out, uint8_t *flag_out, float *logits_out,
+                                                               const SmallRerun rr) {
     pdl_wait();
     pdl_trigger();
-    const CampFault f = faults[blockIdx.x];
-    const int n_lo = blockIdx.y * ipc, n_hi = min(g.B, n_lo + ipc);
-    if (f.kind == 1 && (f.img < n_lo || f.img >= n_hi)) return;      // only the hit image's CTA works
+    const CampFault f = faults ? faults[blockIdx.x] : single;
+    const bool campaign = faults != nullptr;
+    const int pc = g.protect ? 1 : 0;            // checksum channels / neurons
+    const int n_lo = blockIdx.y * ipc, n_hi = min(g.B + (campaign ? 0 : rr.n), n_lo + ipc);
+    // a campaign's activation fault: only the hit image's CTA works
+    if (campaign && f.kind == 1 && (f.img < n_lo || f.img >= n_hi)) return;
     extern __shared__ __align__(16) float sm[];
     const SmLayout L = sm_layout(g);
     float *w1 = sm + L.w1, *w2 = sm + L.w2, *img = sm + L.img, *a1 = sm + L.a1, *c1 = sm + L.c1;
@@ -101,16 +116,21 @@ __global__ void __launch_bounds__(256) campaign_small_kernel(const SmallNet g, c
     const bool fd1 = f.kind == 0 && f.layer == 0 && f.fd.active;
     const bool fd2 = f.kind == 0 && f.layer == 1 && f.fd.active;
     __syncthreads();
-    const int n_first = f.kind == 1 ? f.img : n_lo, n_last = f.kind == 1 ? f.img + 1 : n_hi;
+    const int n_first = (campaign && f.kind == 1) ? f.img : n_lo;
+    const int n_last = (campaign && f.kind == 1) ? f.img + 1 : n_hi;
     const int ctr1 = (g.R1 - 1) / 2, ctr2 = (g.R2 - 1) / 2;
     const int HW0 = g.H0 * g.W0, HW1 = g.H1 * g.W1, HWp1 = g.Hp1 * g.Wp1, HW2 = g.H2 * g.W2, HWp2 = g.Hp2 * g.Wp2;
     for (int n = n_first; n < n_last; ++n) {
         // ---- image [C0][H0][W0] ----
-        const float *xn = g.x + (size_t)n * g.C0 * HW0;
+        const bool rerun = n >= g.B;             // a row of the re-run list
+        const int src_n = rerun ? rr.idx[n - g.B] : n;
+        const float *xn = rerun ? rr.x + (size_t)src_n * g.C0 * HW0
+                        : (g.x2 && n >= g.n_split) ? g.x2 + (size_t)(n - g.n_split) * g.C0 * HW0
+                                                   : g.x + (size_t)n * g.C0 * HW0;
         for (int i = tid; i < g.C0 * HW0; i += blockDim.x) img[i] = __ldg(xn + i);
         __syncthreads();
         // ---- conv1 + ReLU, its carry-through channel ----
-        for (int e = tid; e < (g.K1 + 1) * HW1; e += blockDim.x) {
+        for (int e = tid; e < (g.K1 + pc) * HW1; e += blockDim.x) {
             const int k = e / HW1, pq = e % HW1, p = pq / g.W1, q = pq % g.W1;
             float o;
             if (k < g.K1) {
@@ -133,7 +153,7 @@ __global__ void __launch_bounds__(256) campaign_small_kernel(const SmallNet g, c
         }
         __syncthreads();
         // ---- 2x2 max-pool (data and checksum); an activation flip of this image ----
-        for (int e = tid; e < (g.K1 + 1) * HWp1; e += blockDim.x) {
+        for (int e = tid; e < (g.K1 + pc) * HWp1; e += blockDim.x) {
             const int k = e / HWp1, pq = e % HWp1, p = pq / g.Wp1, q = pq % g.Wp1;
             const float *src = k < g.K1 ? a1 + k * HW1 : c1;
             float mx = -INFINITY;
@@ -145,7 +165,7 @@ __global__ void __launch_bounds__(256) campaign_small_kernel(const SmallNet g, c
         __syncthreads();
         // ---- conv2 + ReLU (the checksum input is skipped by data filters),
         // carry-through channel over data and checksum inputs ----
-        for (int e = tid; e < (g.K2 + 1) * HW2; e += blockDim.x) {
+        for (int e = tid; e < (g.K2 + pc) * HW2; e += blockDim.x) {
             const int k = e / HW2, pq = e % HW2, p = pq / g.W2, q = pq % g.W2;
             float o;
             if (k < g.K2) {
@@ -170,7 +190,7 @@ __global__ void __launch_bounds__(256) campaign_small_kernel(const SmallNet g, c
         }
         __syncthreads();
         // ---- 2x2 max-pool into the FC input: data in (h, w, c) order, checksum plane ----
-        for (int e = tid; e < (g.K2 + 1) * HWp2; e += blockDim.x) {
+        for (int e = tid; e < (g.K2 + pc) * HWp2; e += blockDim.x) {
             const int k = e / HWp2, pq = e % HWp2, p = pq / g.Wp2, q = pq % g.Wp2;
             const float *src = k < g.K2 ? a2 + k * HW2 : c2;
             float mx = -INFINITY;
@@ -180,7 +200,7 @@ __global__ void __launch_bounds__(256) campaign_small_kernel(const SmallNet g, c
         }
         __syncthreads();
         // ---- FC1 + ReLU; carry-through neuron ----
-        for (int j = warp; j <= g.N1; j += blockDim.x / 32) {
+        for (int j = warp; j < g.N1 + pc; j += blockDim.x / 32) {
             float o;
             if (j < g.N1) o = warp_dot(g.wf1 + (size_t)j * g.NIN1, p2, g.NIN1, lane) + __ldg(g.bf1 + j);
             else o = g.coeff1 * (warp_sum(p2, g.NIN1, lane) + warp_sum(q2, HWp2, lane));
@@ -188,7 +208,7 @@ __global__ void __launch_bounds__(256) campaign_small_kernel(const SmallNet g, c
         }
         __syncthreads();
         // ---- FC2 + ReLU; carry-through neuron ----
-        for (int j = warp; j <= g.N2; j += blockDim.x / 32) {
+        for (int j = warp; j < g.N2 + pc; j += blockDim.x / 32) {
             float o;
             if (j < g.N2) o = warp_dot(g.wf2 + (size_t)j * g.N1, f1, g.N1, lane) + __ldg(g.bf2 + j);
             else o = g.coeff2 * (warp_sum(f1, g.N1, lane) + f1[g.N1]);
@@ -196,13 +216,22 @@ __global__ void __launch_bounds__(256) campaign_small_kernel(const SmallNet g, c
         }
         __syncthreads();
         // ---- classifier; accumulated-checksum neuron S ----
-        for (int j = warp; j <= g.N3; j += blockDim.x / 32) {
+        for (int j = warp; j < g.N3 + pc; j += blockDim.x / 32) {
             float o;
             if (j < g.N3) o = warp_dot(g.wf3 + (size_t)j * g.N2, f2, g.N2, lane) + __ldg(g.bf3 + j);
             else o = g.coeff3 * (warp_sum(f2, g.N2, lane) + f2[g.N2]);
             if (lane == 0) f3[j] = o;
         }
         __syncthreads();
+        const size_t o = (size_t)blockIdx.x * g.B + n;
+        if (rerun) {
+            for (int j = tid; j < g.N3; j += blockDim.x) rr.logits[(size_t)src_n * g.N3 + j] = f3[j];
+            if (tid == 0 && rr.S) rr.S[src_n] = g.protect ? f3[g.N3] : __int_as_float(0x7fc00000);
+            __syncthreads();
+            continue;
+        }
+        if (logits_out)
+            for (int j = tid; j < g.N3; j += blockDim.x) logits_out[o * g.N3 + j] = f3[j];
         if (tid == 0) {
             // top-1: a NaN logit gives -1; ties go to the lowest index
             int best = 0;
@@ -211,11 +240,12 @@ __global__ void __launch_bounds__(256) campaign_small_kernel(const SmallNet g, c
                 if (f3[j] != f3[j]) nan = true;
                 else if (f3[j] > f3[best]) best = j;
             }
-            const float S = f3[g.N3];
-            const size_t o = (size_t)blockIdx.x * g.B + n;
-            S_out[o] = S;
-            top1_out[o] = nan ? -1 : best;
-            flag_out[o] = !(fabs((double)S - g.ref) <= g.tau);
+            const float S = g.protect ? f3[g.N3] : __int_as_float(0x7fc00000);
+            if (S_out) S_out[o] = S;
+            if (top1_out) top1_out[o] = nan ? -1 : best;
+            const uint8_t fv = g.protect ? !(fabs((double)S - g.ref) <= g.tau) : 0;
+            if (flag_out) flag_out[o] = fv;
+            if (!campaign && g.flag2) g.flag2[n] = fv;
         }
         __syncthreads();
     }
@@ -236,7 +266,26 @@ cudaError_t launch_campaign_small(const SmallNet &g, const CampFault *faults, in
         if (e != cudaSuccess) return e;
     }
     dim3 grid(n_faults, (g.B + IPC - 1) / IPC);
-    pdl_launch(campaign_small_kernel, grid, 256, smem, st, g, faults, IPC, S, top1, flag);
+    CampFault none{};
+    none.kind = 2;
+    SmallRerun rr{};
+    pdl_launch(campaign_small_kernel, grid, 256, smem, st, g, faults, none, IPC, S, top1, flag, (float *)nullptr, rr);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_small_infer(const SmallNet &g, const CampFault &fault, float *logits, float *S, uint8_t *flag,
+                               const SmallRerun &rr, cudaStream_t st) {
+    const size_t smem = campaign_small_smem(g);
+    if (smem > 48 * 1024) {
+        cudaError_t e = cudaFuncSetAttribute(campaign_small_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)smem);
+        if (e != cudaSuccess) return e;
+    }
+    // one image per CTA of 1024 threads: the images of a batch (and the
+    // re-run list) run side by side
+    dim3 grid(1, g.B + rr.n);
+    pdl_launch(campaign_small_kernel, grid, 1024, smem, st, g, (const CampFault *)nullptr, fault, 1, S,
+               (int32_t *)nullptr, flag, logits, rr);
     return cudaGetLastError();
 }
 

@@ -54,8 +54,18 @@ __device__ __forceinline__ float load_x(const T *x, int n, int h, int w, int c, 
     return to_f(x[(((size_t)n * H + h) * W + w) * C + c]);
 }
 
+// Output column j (0 .. TN) of thread column tx within the block's BN columns:
+// groups of 4 consecutive columns, the groups of one thread BN / (TN / 4)
+// apart, so that the 16-byte shared-memory reads of a warp's threads cover
+// consecutive 16-byte pieces (no bank conflicts) for every TN.
+template <int BN, int TN>
+__device__ __forceinline__ int col_of(int tx, int j) {
+    return (j / 4) * (BN / (TN / 4)) + tx * 4 + (j % 4);
+}
+
+// two blocks per SM: 256-thread blocks stay at or below 128 registers
 template <typename T, int BM, int BN, int BK, int TM, int TN, bool VEC>
-__global__ void __launch_bounds__((BM / TM) * (BN / TN))
+__global__ void __launch_bounds__((BM / TM) * (BN / TN), 2)
 conv_simt_kernel(ConvArgs a) {
     pdl_wait();
     pdl_trigger();
@@ -106,15 +116,19 @@ conv_simt_kernel(ConvArgs a) {
 
     auto load_tiles = [&](int kt) {
         const int k0 = kt * BK;
+        // the tap and channel of this K tile (C is a multiple of BK on the
+        // vector path: one tap per K tile), computed once per tile
+        const int tap_k = VEC ? k0 / a.C : 0;
+        const int c_k = VEC ? k0 - tap_k * a.C : 0;
+        const int r_k = VEC ? tap_k / a.S : 0, s_k = VEC ? tap_k - r_k * a.S : 0;
 #pragma unroll
         for (int i = 0; i < A_PER; ++i) {
 #pragma unroll
             for (int e = 0; e < AE; ++e) areg[i][e] = 0.f;
             if (a_n[i] < 0) continue;
             if (VEC) {
-                int tap = k0 / a.C, c0 = k0 % a.C + a_sub[i];
-                int r = tap / a.S, s = tap % a.S;
-                int h = a_h0[i] + r, ww = a_w0[i] + s;
+                const int c0 = c_k + a_sub[i];
+                const int h = a_h0[i] + r_k, ww = a_w0[i] + s_k;
                 if (h >= 0 && h < a.H && ww >= 0 && ww < a.W) {
                     const typename Vec<T>::type *p = reinterpret_cast<const typename Vec<T>::type *>(
                         x + (((size_t)a_n[i] * a.H + h) * a.W + ww) * a.C + c0);
@@ -185,34 +199,51 @@ conv_simt_kernel(ConvArgs a) {
         store_tiles(0);
     }
     __syncthreads();
+    // one K step: TM x TN FFMAs from two rows of the staged tiles; on the
+    // centre tap's K tiles of the first channel tile the A values are also
+    // summed for the carry-through output (same order as before: k ascending)
+    auto kstep = [&](int buf, int kk, bool ctr) {
+        float av[TM], bv[TN];
+#pragma unroll
+        for (int i = 0; i < TM; i += 4) {
+            float4 v = *reinterpret_cast<const float4 *>(&As[buf][kk][ty * TM + i]);
+            av[i] = v.x; av[i + 1] = v.y; av[i + 2] = v.z; av[i + 3] = v.w;
+        }
+#pragma unroll
+        for (int j = 0; j < TN; j += 4) {
+            float4 v = *reinterpret_cast<const float4 *>(&Bs[buf][kk][col_of<BN, TN>(tx, j)]);
+            bv[j] = v.x; bv[j + 1] = v.y; bv[j + 2] = v.z; bv[j + 3] = v.w;
+        }
+#pragma unroll
+        for (int i = 0; i < TM; ++i)
+#pragma unroll
+            for (int j = 0; j < TN; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
+        if (ctr) {
+#pragma unroll
+            for (int i = 0; i < TM; ++i) csum[i] += av[i];
+        }
+    };
     for (int kt = kt_lo; kt < kt_hi; ++kt) {
         const int buf = (kt - kt_lo) & 1;
         if (kt + 1 < kt_hi) load_tiles(kt + 1);
         const int k0 = kt * BK;
+        // a K tile lies wholly inside or outside the centre tap's K range
+        // when C is a multiple of BK (vector path); otherwise test each k
+        if (!do_cs) {
 #pragma unroll
-        for (int kk = 0; kk < BK; ++kk) {
-            float av[TM], bv[TN];
+            for (int kk = 0; kk < BK; ++kk) kstep(buf, kk, false);
+        } else if (VEC) {
+            const bool ctr = k0 >= ctr_lo && k0 < ctr_hi;
+            if (ctr) {
 #pragma unroll
-            for (int i = 0; i < TM; i += 4) {
-                float4 v = *reinterpret_cast<const float4 *>(&As[buf][kk][ty * TM + i]);
-                av[i] = v.x; av[i + 1] = v.y; av[i + 2] = v.z; av[i + 3] = v.w;
+                for (int kk = 0; kk < BK; ++kk) kstep(buf, kk, true);
+            } else {
+#pragma unroll
+                for (int kk = 0; kk < BK; ++kk) kstep(buf, kk, false);
             }
+        } else {
 #pragma unroll
-            for (int j = 0; j < TN; j += 4) {
-                float4 v = *reinterpret_cast<const float4 *>(&Bs[buf][kk][tx * TN + j]);
-                bv[j] = v.x; bv[j + 1] = v.y; bv[j + 2] = v.z; bv[j + 3] = v.w;
-            }
-#pragma unroll
-            for (int i = 0; i < TM; ++i)
-#pragma unroll
-                for (int j = 0; j < TN; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
-            if (do_cs) {
-                const int k = k0 + kk;
-                if (k >= ctr_lo && k < ctr_hi) {
-#pragma unroll
-                    for (int i = 0; i < TM; ++i) csum[i] += av[i];
-                }
-            }
+            for (int kk = 0; kk < BK; ++kk) kstep(buf, kk, k0 + kk >= ctr_lo && k0 + kk < ctr_hi);
         }
         if (kt + 1 < kt_hi) store_tiles(buf ^ 1);
         __syncthreads();
@@ -228,7 +259,7 @@ conv_simt_kernel(ConvArgs a) {
             if (m >= M) break;
 #pragma unroll
             for (int j = 0; j < TN; ++j) {
-                const int k = n0 + tx * TN + j;
+                const int k = n0 + col_of<BN, TN>(tx, j);
                 if (k < a.K) wz[(size_t)m * ws_ld + k] = acc[i][j];
             }
             if (a.cs_out != nullptr && blockIdx.y == 0 && tx == 0)
@@ -250,7 +281,7 @@ conv_simt_kernel(ConvArgs a) {
         float v[TN];
 #pragma unroll
         for (int j = 0; j < TN; ++j) {
-            const int k = n0 + tx * TN + j;
+            const int k = n0 + col_of<BN, TN>(tx, j);
             v[j] = 0.f;
             if (k >= a.K) continue;
             float o = acc[i][j] + a.bias[k];
@@ -266,28 +297,26 @@ conv_simt_kernel(ConvArgs a) {
             if (a.relu) o = relu_keep_nan(o);
             v[j] = o;
         }
-        const int kb = n0 + tx * TN;
-        if (kb + TN <= a.K && (a.K % 4) == 0) {
-            if constexpr (sizeof(T) == 4) {
+        // groups of 4 consecutive columns: vector stores when the group is whole
 #pragma unroll
-                for (int j = 0; j < TN; j += 4)
-                    *reinterpret_cast<float4 *>(&y[(size_t)m * a.K + kb + j]) =
-                        make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
-            } else {
-#pragma unroll
-                for (int j = 0; j < TN; j += 4) {
+        for (int j = 0; j < TN; j += 4) {
+            const int kb = n0 + col_of<BN, TN>(tx, j);
+            if (kb + 4 <= a.K && (a.K % 4) == 0) {
+                if constexpr (sizeof(T) == 4) {
+                    *reinterpret_cast<float4 *>(&y[(size_t)m * a.K + kb]) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
+                } else {
                     __half2 h0 = __floats2half2_rn(v[j], v[j + 1]);
                     __half2 h1 = __floats2half2_rn(v[j + 2], v[j + 3]);
                     uint2 pk;
                     pk.x = *reinterpret_cast<uint32_t *>(&h0);
                     pk.y = *reinterpret_cast<uint32_t *>(&h1);
-                    *reinterpret_cast<uint2 *>(&y[(size_t)m * a.K + kb + j]) = pk;
+                    *reinterpret_cast<uint2 *>(&y[(size_t)m * a.K + kb]) = pk;
                 }
-            }
-        } else {
+            } else {
 #pragma unroll
-            for (int j = 0; j < TN; ++j)
-                if (kb + j < a.K) y[(size_t)m * a.K + kb + j] = from_f<T>(v[j]);
+                for (int e = 0; e < 4; ++e)
+                    if (kb + e < a.K) y[(size_t)m * a.K + kb + e] = from_f<T>(v[j + e]);
+            }
         }
         // checksum output: one thread column of the first channel tile
         if (a.cs_out != nullptr && blockIdx.y == 0 && tx == 0) {

@@ -245,6 +245,44 @@ __device__ __forceinline__ void store16_fast(const float *v, const Bias16 &b, co
     yp[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
 }
 
+// Epilogue values of 16 channels k0 .. k0 + 15 of one pixel in FP32, in the
+// order of store_chunk_pre: accumulator + bias, fault delta, residual, ReLU.
+__device__ __forceinline__ void epi16_vals(const float *v, const Bias16 &b, const Res16 &r, bool res, bool relu,
+                                           const FaultDelta &fd, int k0, float fsrc, float *t) {
+    const float *bb = reinterpret_cast<const float *>(b.q);
+    float rv[16];
+    {
+        const __half2 *h0 = reinterpret_cast<const __half2 *>(&r.r0);
+        const __half2 *h1 = reinterpret_cast<const __half2 *>(&r.r1);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float2 f0 = __half22float2(h0[i]), f1 = __half22float2(h1[i]);
+            rv[2 * i] = f0.x; rv[2 * i + 1] = f0.y; rv[8 + 2 * i] = f1.x; rv[8 + 2 * i + 1] = f1.y;
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+        float x = v[i] + bb[i];
+        if (fd.active && fd.kout == k0 + i) x += fd.dv * fsrc;
+        if (res) x += rv[i];
+        if (relu) x = relu_keep_nan(x);
+        t[i] = x;
+    }
+}
+
+// Maximum over the 2 x 2 window of a halo tile's epilogue lanes: a warp holds
+// four tile rows of 8 pixels, lane = 8 * row + column, so the window's other
+// pixels are lanes l ^ 1 and l ^ 8.  NaN wins (a window with a NaN is NaN).
+__device__ __forceinline__ float fmax_nan(float a, float b) {
+    float r;
+    asm("max.NaN.f32 %0, %1, %2;" : "=f"(r) : "f"(a), "f"(b));
+    return r;
+}
+__device__ __forceinline__ float pool2x2_lanes(float v) {
+    v = fmax_nan(v, __shfl_xor_sync(0xffffffffu, v, 1));
+    return fmax_nan(v, __shfl_xor_sync(0xffffffffu, v, 8));
+}
+
 // The checksum output of one pixel: carry-through column + coef * incoming
 // checksum (centre pixel, or the sum of an FC layer's checksum features),
 // fault delta, residual checksum, ReLU.
@@ -270,15 +308,20 @@ __device__ __forceinline__ CsIn load_cs_inputs(const ConvArgs &a, const TcGeom &
     return c;
 }
 
-__device__ __forceinline__ void store_checksum_pre(float ctv, const CsIn &c, const ConvArgs &a, const TcGeom &g,
-                                                   int m, float fsrc) {
+__device__ __forceinline__ float checksum_value(float ctv, const CsIn &c, const ConvArgs &a, const TcGeom &g,
+                                                float fsrc) {
     float o = 0.f;
     if (a.role == CT_ROLE_CT) o = ctv + a.coef * c.cin;
     else if (a.role == CT_ROLE_PASS) o = c.cin;
     if (a.fd.active && a.fd.kout == g.K) o += a.fd.dv * fsrc;
     if (a.res_cs) o += c.rcs;
     if (a.relu) o = relu_keep_nan(o);
-    static_cast<__half *>(a.cs_out)[m] = __float2half_rn(o);
+    return o;
+}
+
+__device__ __forceinline__ void store_checksum_pre(float ctv, const CsIn &c, const ConvArgs &a, const TcGeom &g,
+                                                   int m, float fsrc) {
+    static_cast<__half *>(a.cs_out)[m] = __float2half_rn(checksum_value(ctv, c, a, g, fsrc));
 }
 
 
@@ -1247,7 +1290,10 @@ __host__ __device__ constexpr int halo_bres_off(int i) {
     return i == 0 ? 0 : (BN + 16) * BK * 2 + (i - 1) * BN * BK * 2;
 }
 
-template <int BN, bool BRES, int NA, int NB, int NR>
+// POOL: the 2 x 2 stride-2 max-pool that follows the convolution is applied
+// in the epilogue (data and checksum alike); a.y / a.cs_out are then the
+// pooled tensor [N, H / 2, W / 2, K] and its checksum plane.
+template <int BN, bool BRES, int NA, int NB, int NR, bool POOL>
 __global__ void __launch_bounds__(NTHREADS, 1)
 conv_tc_halo_kernel(const __grid_constant__ HaloMaps maps, const ConvArgs a, const HaloGeom hg, const TcGeom g) {
     constexpr int B_ROWS = BN + 16;                       // 16 constant carry-through rows
@@ -1534,7 +1580,39 @@ conv_tc_halo_kernel(const __grid_constant__ HaloMaps maps, const ConvArgs a, con
                 __syncwarp();
                 if (lane == 0) mbar_arrive(smem_u32(&r_empty[rsl]));
             }
-            if (valid) {
+            if (POOL) {
+                // every lane computes its pixel (the shuffles need the whole warp);
+                // the window's top-left lane stores the pooled pixel
+                float fsrc = 0.f;
+                if (fd.active && valid) {
+                    const int h = p + fd.r - 1, w = q + fd.s - 1;
+                    if (h >= 0 && h < hg.H && w >= 0 && w < hg.W) {
+                        if (fd.cin < hg.C) fsrc = ldh(x, (((size_t)ht.n * hg.H + h) * hg.W + w) * hg.C + fd.cin);
+                        else if (a.cs_in) fsrc = ldh(static_cast<const __half *>(a.cs_in), ((size_t)ht.n * hg.H + h) * hg.W + w);
+                    }
+                }
+                const bool writer = valid && (row & 1) == 0 && (row & 8) == 0;
+                const size_t mp = ((size_t)ht.n * (hg.H / 2) + p / 2) * (hg.W / 2) + q / 2;
+#pragma unroll
+                for (int c = 0; c < BN / 2; c += 16) {
+                    float t[16];
+                    epi16_vals(vals + c, BN <= 64 ? bias_r[(c / 16) % NBIAS] : load_bias16(a.bias, n0 + c), rs[c / 16],
+                               has_res, relu, fd, n0 + c, fsrc, t);
+                    uint32_t pk[8];
+#pragma unroll
+                    for (int i = 0; i < 8; ++i)
+                        pk[i] = cvt_h2(pool2x2_lanes(t[2 * i]), pool2x2_lanes(t[2 * i + 1]), false);
+                    if (writer) {
+                        uint4 *yp = reinterpret_cast<uint4 *>(static_cast<__half *>(a.y) + mp * hg.K + n0 + c);
+                        yp[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+                        yp[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+                    }
+                }
+                if (do_cs) {
+                    const float o = pool2x2_lanes(checksum_value(ctv, csv, a, g, fsrc));
+                    if (writer) static_cast<__half *>(a.cs_out)[mp] = __float2half_rn(o);
+                }
+            } else if (valid) {
                 float fsrc = 0.f;
                 if (fd.active) {
                     const int h = p + fd.r - 1, w = q + fd.s - 1;
@@ -1817,18 +1895,24 @@ struct HaloPlan {
     HaloMaps maps;
     HaloGeom hg;
     TcGeom g;
-    int BN, kind, sms;
+    int BN, kind, pool, sms;
     size_t smem;
     const void *res, *csin, *rescs;   // tensors the R-ring maps point at
 };
 
-template <int BN, bool BRES, int NA, int NB, int NR>
+template <int BN, bool BRES, int NA, int NB, int NR, bool POOL>
 size_t halo_smem() {
     const int nbs = BRES ? 9 : NB;
     const size_t b_area = BRES ? (size_t)halo_bres_off<BN>(9) : (size_t)NB * (BN + 16) * BK * 2;
     return 1024 + (size_t)NA * HT_A_STAGE + b_area + (size_t)NR * HaloR<BN>::STAGE +
            8 * (2 * NA + 2 * nbs + 2 * NR + 4) + 16;
 }
+
+// halo kernel variants <BN, resident weights, patch stages, weight stages,
+// operand-ring stages>; each also with the fused 2 x 2 max-pool
+#define HK0 64, true, 4, 0, 3
+#define HK1 64, false, 3, 6, 3
+#define HK2 128, false, 3, 4, 2
 
 // Tiles that overhang the image waste MMA rows: require whole 8-column tiles
 // and at most one partly filled row of tiles on a tall image.
@@ -1849,8 +1933,9 @@ static bool encode_plane_map(CUtensorMap *map, const void *plane, int N, int H, 
 }
 
 HaloPlan *halo_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, const void *x_dev, const void *res_dev,
-                           const void *csin_dev, const void *rescs_dev, std::string *why) {
+                           const void *csin_dev, const void *rescs_dev, bool pool, std::string *why) {
     if (!halo_supported(a.C, a.K, a.R, a.S, a.stride, a.pad, a.H, a.W)) { if (why) *why = "shape"; return nullptr; }
+    if (pool && (a.H % 2 || a.W % 2)) { if (why) *why = "pooled shape"; return nullptr; }
     if (!load_encoders()) { if (why) *why = "tensor-map encoders unavailable"; return nullptr; }
     HaloPlan *pl = new HaloPlan();
     memset(pl, 0, sizeof(*pl));
@@ -1908,19 +1993,15 @@ HaloPlan *halo_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, 
         return nullptr;
     }
     cudaError_t e;
-    if (pl->BN == 64 && hg.ncb == 1) {
-        pl->kind = 0;
-        pl->smem = halo_smem<64, true, 4, 0, 3>();
-        e = cudaFuncSetAttribute(conv_tc_halo_kernel<64, true, 4, 0, 3>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
-    } else if (pl->BN == 64) {
-        pl->kind = 1;
-        pl->smem = halo_smem<64, false, 3, 6, 3>();
-        e = cudaFuncSetAttribute(conv_tc_halo_kernel<64, false, 3, 6, 3>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
-    } else {
-        pl->kind = 2;
-        pl->smem = halo_smem<128, false, 3, 4, 2>();
-        e = cudaFuncSetAttribute(conv_tc_halo_kernel<128, false, 3, 4, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
-    }
+    pl->pool = pool ? 1 : 0;
+    pl->kind = (pl->BN == 64 && hg.ncb == 1) ? 0 : pl->BN == 64 ? 1 : 2;
+#define HALO_ATTR(P, ...)                                                                                        \
+    (pl->smem = halo_smem<__VA_ARGS__, P>(),                                                                       \
+     cudaFuncSetAttribute(conv_tc_halo_kernel<__VA_ARGS__, P>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem))
+    if (pl->kind == 0) e = pool ? HALO_ATTR(true, HK0) : HALO_ATTR(false, HK0);
+    else if (pl->kind == 1) e = pool ? HALO_ATTR(true, HK1) : HALO_ATTR(false, HK1);
+    else e = pool ? HALO_ATTR(true, HK2) : HALO_ATTR(false, HK2);
+#undef HALO_ATTR
     if (e != cudaSuccess) { cudaGetLastError(); if (why) *why = "shared memory attribute"; delete pl; return nullptr; }
     return pl;
 }
@@ -1939,9 +2020,12 @@ cudaError_t launch_conv_tc_halo(const ConvArgs &a, const HaloPlan *pl, cudaStrea
     g.M = a.N * a.P * a.Q;
     const int tiles = halo_tiles(pl, a.N);
     dim3 grid(tiles < pl->sms ? tiles : pl->sms);
-    if (pl->kind == 0) pdl_launch(conv_tc_halo_kernel<64, true, 4, 0, 3>, grid, NTHREADS, pl->smem, st, pl->maps, a, hg, g);
-    else if (pl->kind == 1) pdl_launch(conv_tc_halo_kernel<64, false, 3, 6, 3>, grid, NTHREADS, pl->smem, st, pl->maps, a, hg, g);
-    else pdl_launch(conv_tc_halo_kernel<128, false, 3, 4, 2>, grid, NTHREADS, pl->smem, st, pl->maps, a, hg, g);
+#define HALO_LAUNCH(P, ...) \
+    pdl_launch(conv_tc_halo_kernel<__VA_ARGS__, P>, grid, NTHREADS, pl->smem, st, pl->maps, a, hg, g)
+    if (pl->kind == 0) pl->pool ? HALO_LAUNCH(true, HK0) : HALO_LAUNCH(false, HK0);
+    else if (pl->kind == 1) pl->pool ? HALO_LAUNCH(true, HK1) : HALO_LAUNCH(false, HK1);
+    else pl->pool ? HALO_LAUNCH(true, HK2) : HALO_LAUNCH(false, HK2);
+#undef HALO_LAUNCH
     return cudaGetLastError();
 }
 

@@ -77,6 +77,7 @@ struct Slot {
     bool has_cs = false;
     bool is_float = false;       // GAP output: fp32 features whatever the precision
     bool stored = true;          // false: computed inside a fused kernel, never in HBM
+    bool skipped_last = false;   // the last inference computed its reader (a fused max-pool) without storing it
     void *data = nullptr;
     void *cs = nullptr;
 };
@@ -98,6 +99,7 @@ struct LayerRT {
     bool stem = false;           // fused image stem: this conv and the max-pool after it
     StemPlan *stplan = nullptr;
     bool fused = false;          // max-pool computed by the preceding fused stem
+    bool pool_fuse = false;      // conv: its halo kernel applies the 2 x 2 max-pool that follows (layer + 1)
     int w_ld = 0, c_stride = 0;  // weight row length and channel stride within a tap
     // fc
     int n_in = 0, n_cs = 0, n_out = 0;
@@ -151,13 +153,17 @@ struct ct_model {
     std::vector<int> re_graph_nk;        // kernels in each graph
     int64_t kernels_total = 0;           // kernels launched since the last ct_kernel_count
     int n_kernels_last = -1;     // kernels launched by the last inference
+    bool small = false;          // the whole network runs as one kernel (LeNet-5 shape)
+    uint8_t *flag_mirror = nullptr;   // set by run_batches: the final kernel also writes the flags here
+    double small_flops = 0;      // its convolutions' multiply-adds per image
     int n_kernels_run = 0;
     std::vector<void *> dev_allocs;
     // ct_infer_batches / ct_run_host_batches: per pipeline slot a pinned copy
     // of the batch's flags, a pinned index list, events; a copy stream and
     // (host buffers) device slots for inputs and results; made on first use
     static constexpr int PIPE = 6;
-    uint8_t *pipe_flags_h = nullptr;      // [PIPE][max_batch]
+    uint8_t *pipe_flags_h = nullptr;      // [PIPE][max_batch], host memory mapped for the device
+    uint8_t *pipe_flags_d = nullptr;      // its device address
     int32_t *pipe_idx_h = nullptr;        // [PIPE + 2][max_batch]
     cudaEvent_t pipe_ev_flags[PIPE] = {}, pipe_ev_step[PIPE] = {}, pipe_ev_in[PIPE] = {}, pipe_ev_out[PIPE] = {};
     cudaEvent_t pipe_ev_tail = nullptr;
@@ -425,6 +431,8 @@ ct_status resolve_roles(const ct_model_desc *desc, int32_t *roles) {
     return CT_OK;
 }
 
+static bool small_net_of(const ct_model *m, SmallNet *g);
+
 ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const *wts) {
     const int nL = desc->n_layers;
     int max_slot = 0;
@@ -683,11 +691,28 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
             const Slot &sx = m->slots[l.d.src];
             const Slot *sr = l.d.res >= 0 ? &m->slots[l.d.res] : nullptr;
             const bool cs_out = l.cs_out;
+            // a 2 x 2 stride-2 max-pool that is the only reader of this output
+            // runs in the halo kernel's epilogue
+            const size_t li = (size_t)(&l - m->L.data());
+            if (li + 1 < m->L.size() && l.P % 2 == 0 && l.Q % 2 == 0) {
+                const ct_layer_desc &nx = m->L[li + 1].d;
+                int readers = 0;
+                for (auto &o : m->L) readers += (o.d.src == l.d.dst) + (o.d.res == l.d.dst);
+                l.pool_fuse = nx.op == CT_OP_MAXPOOL && nx.src == l.d.dst && nx.k == 2 && nx.stride == 2 &&
+                              nx.pad == 0 && readers == 1;
+            }
             l.hplan = halo_plan_create(a, B, l.w, sx.data, sr ? sr->data : nullptr,
                                        (cs_out && sx.has_cs) ? sx.cs : nullptr,
-                                       (cs_out && sr && sr->has_cs) ? sr->cs : nullptr, &why);
+                                       (cs_out && sr && sr->has_cs) ? sr->cs : nullptr, l.pool_fuse, &why);
             if (!l.hplan) return CT_ECUDA;
         }
+    }
+    // ---- the LeNet-5 shape runs as one whole-network kernel ----
+    {
+        SmallNet g;
+        m->small = !(m->flags & CT_FLAG_LAYERWISE) && small_net_of(m, &g);
+        if (m->small)
+            m->small_flops = (double)g.K1 * g.H1 * g.W1 * g.R1 * g.R1 * g.C0 + (double)g.K2 * g.H2 * g.W2 * g.R2 * g.R2 * g.K1;
     }
     // ---- scratch for re-execution and host runs ----
     const size_t per_img = (size_t)m->in_c * m->in_h * m->in_w;
@@ -768,13 +793,97 @@ ct_status act_fault_word(const ct_model *m, int slot, int batch, int64_t e, void
 // inference
 // ---------------------------------------------------------------------------
 
+// The LeNet shape the whole-network kernel runs (FP32, widened or
+// unprotected): conv -> pool -> conv -> pool -> fc -> fc -> fc, with ReLU
+// after every conv and hidden FC, 2x2 stride-2 pools, unpadded stride-1
+// convolutions with a carry-through filter (widened).
+static bool small_net_of(const ct_model *m, SmallNet *g) {
+    if (m->prec != CT_FP32 || m->replace || m->L.size() != 7) return false;
+    const LayerRT &c1 = m->L[0], &p1 = m->L[1], &c2 = m->L[2], &p2 = m->L[3];
+    const LayerRT &f1 = m->L[4], &f2 = m->L[5], &f3 = m->L[6];
+    const int want_role = m->protect ? CT_ROLE_CT : CT_ROLE_NONE;
+    auto conv_ok = [&](const LayerRT &l) {
+        return l.d.op == CT_OP_CONV && l.d.stride == 1 && l.d.pad == 0 && l.d.relu && l.d.res < 0 &&
+               l.role == want_role && l.R == l.S && l.w_ld == l.R * l.S * l.C && l.c_stride == l.C && !l.dw;
+    };
+    auto pool_ok = [](const LayerRT &l) { return l.d.op == CT_OP_MAXPOOL && l.d.k == 2 && l.d.stride == 2 && l.d.pad == 0; };
+    if (!conv_ok(c1) || !pool_ok(p1) || !conv_ok(c2) || !pool_ok(p2)) return false;
+    if (c1.d.src != 0 || p1.d.src != c1.d.dst || c2.d.src != p1.d.dst || p2.d.src != c2.d.dst) return false;
+    if (f1.d.op != CT_OP_FC || f2.d.op != CT_OP_FC || f3.d.op != CT_OP_FC || !f1.d.relu || !f2.d.relu ||
+        !f3.d.final || f1.d.src != p2.d.dst || f2.d.src != f1.d.dst || f3.d.src != f2.d.dst)
+        return false;
+    if (c1.cs_in || c2.cs_in != m->protect || f1.x_float || f1.fc_tc || f2.fc_tc) return false;
+    const Slot &s1 = m->slots[p1.d.dst], &s2 = m->slots[p2.d.dst];
+    SmallNet &n = *g;
+    memset(&n, 0, sizeof(n));
+    n.protect = m->protect ? 1 : 0;
+    n.C0 = c1.C; n.H0 = c1.H; n.W0 = c1.W;
+    n.K1 = c1.K; n.R1 = c1.R; n.H1 = c1.P; n.W1 = c1.Q; n.Hp1 = s1.H; n.Wp1 = s1.W;
+    n.K2 = c2.K; n.R2 = c2.R; n.H2 = c2.P; n.W2 = c2.Q; n.Hp2 = s2.H; n.Wp2 = s2.W;
+    n.NIN1 = f1.n_in; n.N1 = f1.n_out; n.N2 = f2.n_out; n.N3 = f3.n_out;
+    if (n.NIN1 != n.K2 * n.Hp2 * n.Wp2 || f1.n_cs != (m->protect ? n.Hp2 * n.Wp2 : 0) || f2.n_in != n.N1 ||
+        f3.n_in != n.N2)
+        return false;
+    n.w1 = (const float *)c1.w; n.b1 = c1.bias; n.w2 = (const float *)c2.w; n.b2 = c2.bias;
+    n.wf1 = (const float *)f1.w; n.bf1 = f1.bias; n.wf2 = (const float *)f2.w; n.bf2 = f2.bias;
+    n.wf3 = (const float *)f3.w; n.bf3 = f3.bias;
+    n.coef1 = c1.coef; n.coef2 = c2.coef; n.coeff1 = f1.coef; n.coeff2 = f2.coef; n.coeff3 = f3.coef;
+    n.ref = m->ref; n.tau = m->tau;
+    return campaign_small_smem(n) <= 200 * 1024;
+}
+
 // input2 / n_split: images n >= n_split of the batch are image n - n_split
 // of input2 (re-executed images appended to a batch); the rest of the
 // network is unaware of it
 ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, float *S,
-                     uint8_t *flag, cudaStream_t st, const float *input2 = nullptr, int n_split = 0) {
+                     uint8_t *flag, cudaStream_t st, const float *input2 = nullptr, int n_split = 0,
+                     const SmallRerun *rerun = nullptr) {
     const bool half = m->prec == CT_FP16;
     const int wb = half ? 2 : 4;
+    if (m->small) {
+        // the whole network in one kernel; an armed fault is applied inside it
+        SmallNet g;
+        small_net_of(m, &g);
+        g.B = batch;
+        g.x = input;
+        g.x2 = input2;
+        g.n_split = input2 ? n_split : batch;
+        g.ref = m->ref;
+        g.tau = m->tau;
+        g.flag2 = m->flag_mirror;
+        CampFault f{};
+        f.kind = 2;
+        if (m->armed) {
+            const LayerRT &l = m->L[m->f_layer];
+            f.kind = m->f_kind;
+            f.bit = m->f_bit;
+            f.word = -1;
+            if (m->f_kind == CT_BUF_WEIGHT) {
+                f.layer = m->f_layer == 0 ? 0 : 1;
+                const WeightFault wf = resolve_weight_fault(m, l, m->f_elem, m->f_bit);
+                if (wf.explicit_word) f.word = wf.word;
+                else f.fd = wf.fd;
+            } else {
+                const int per_img = (g.K1 + (g.protect ? 1 : 0)) * g.Hp1 * g.Wp1;
+                if (m->f_layer != 2 || m->f_elem < 0 || m->f_elem >= (int64_t)batch * per_img) return CT_ERANGE;
+                f.img = (int)(m->f_elem / per_img);
+                const int within = (int)(m->f_elem % per_img);
+                f.act_c = within / (g.Hp1 * g.Wp1);
+                f.act_hw = within % (g.Hp1 * g.Wp1);
+            }
+        }
+        m->armed = false;
+        m->n_kernels_run = 0;
+        for (auto &sl : m->slots) sl.skipped_last = true;
+        m->slots[0].skipped_last = false;
+        SmallRerun none{};
+        const SmallRerun &rr = rerun ? *rerun : none;
+        CUDA_TRY(launch(m, FAM_SIMT, 2.0 * (batch + rr.n) * m->small_flops, st,
+                        [&] { return launch_small_infer(g, f, logits, S, flag, rr, st); }));
+        m->n_kernels_last = m->n_kernels_run;
+        return CT_OK;
+    }
+    for (auto &sl : m->slots) sl.skipped_last = false;
     const bool armed = m->armed;
     m->armed = false;
     m->n_kernels_run = 0;
@@ -799,6 +908,7 @@ ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, 
         }
     }
     if (act_slot == 0) CUDA_TRY(xor_bit(m, act_base, act_word, m->f_bit, wb, st));
+    size_t pool_done = (size_t)-1;               // a max-pool applied by the preceding conv kernel
     for (size_t i = 0; i < m->L.size(); ++i) {
         LayerRT &l = m->L[i];
         const ct_layer_desc &d = l.d;
@@ -840,14 +950,23 @@ ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, 
             } else {
                 a.ws = m->ws; a.ws_bytes = SPLITK_WS_BYTES;
                 int nk = 1;
-                if (l.hplan && halo_tiles(l.hplan, batch) >= halo_sms(l.hplan))
+                const bool halo = l.hplan && halo_tiles(l.hplan, batch) >= halo_sms(l.hplan);
+                dst.skipped_last = halo && l.pool_fuse;
+                if (halo && l.pool_fuse) {
+                    // the kernel writes the max-pool's output; this output is never stored
+                    const Slot &po = m->slots[m->L[i + 1].d.dst];
+                    a.y = po.data;
+                    a.cs_out = po.has_cs ? po.cs : nullptr;
+                    pool_done = i + 1;
+                }
+                if (halo)
                     CUDA_TRY(launch(m, FAM_TC, flops, st, [&] { return launch_conv_tc_halo(a, l.hplan, st); }));
                 else if (l.tc) CUDA_TRY(launch(m, FAM_TC, flops, st, [&] { return launch_conv_tc(a, l.plan, st, &nk); }, &nk));
                 else CUDA_TRY(launch(m, FAM_SIMT, flops, st, [&] { return launch_conv_simt(a, half, st, &nk); }, &nk));
             }
             if (wfault && wf.explicit_word) CUDA_TRY(xor_bit(m, l.w, wf.word, m->f_bit, wb, st));
-        } else if (l.fused) {
-            // computed by the fused stem
+        } else if (l.fused || i == pool_done) {
+            // computed by the fused stem, or by the halo kernel of the conv before it
         } else if (d.op == CT_OP_MAXPOOL || d.op == CT_OP_GAP) {
             PoolArgs a{};
             a.x = src.data; a.cs_in = src.has_cs ? src.cs : nullptr;
@@ -880,7 +999,7 @@ ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, 
             // sums every input feature (the checksum channel is one of them)
             a.protect = m->protect || (m->replace && d.final);
             a.ref = m->ref; a.tau = m->tau;
-            if (d.final) { a.y = logits; a.S = S; a.flag = flag; }
+            if (d.final) { a.y = logits; a.S = S; a.flag = flag; a.flag2 = m->flag_mirror; }
             else { a.y = dst.data; a.ycs = dst.has_cs ? dst.cs : nullptr; }
             a.ws = m->ws; a.ws_bytes = SPLITK_WS_BYTES;
             const double flops = 2.0 * batch * (double)l.n_in * l.n_out;
@@ -914,7 +1033,10 @@ cudaGraphExec_t reexec_graph(ct_model *m, int bucket) {
         return nullptr;
     }
     const int64_t before = m->kernels_total;
+    uint8_t *const mirror = m->flag_mirror;      // a re-run never writes a batch's flag copy
+    m->flag_mirror = nullptr;
     const ct_status s = infer_impl(m, m->re_input, bucket, m->re_logits, m->re_S, m->re_flag, m->cap_stream);
+    m->flag_mirror = mirror;
     m->re_graph_nk[slot] = (int)(m->kernels_total - before);
     m->kernels_total = before;           // captured, not launched
     cudaGraph_t g = nullptr;
@@ -949,9 +1071,12 @@ ct_status reexec_rows(ct_model *m, const float *input, int batch, const uint8_t 
     CUDA_TRY(cudaMemcpyAsync(m->re_idx, idx_host, sizeof(int32_t) * bucket, cudaMemcpyHostToDevice, st));
     const int64_t per = (int64_t)m->in_c * m->in_h * m->in_w;
     CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] { return launch_gather_images(input, m->re_input, m->re_idx, bucket, per, st); }));
-    // fault-free re-run: an armed fault stays armed for the next ct_infer
+    // fault-free re-run: an armed fault stays armed for the next ct_infer;
+    // it writes no batch's flag copy
     const bool armed = m->armed;
     m->armed = false;
+    uint8_t *const mirror = m->flag_mirror;
+    m->flag_mirror = nullptr;
     ct_status s = CT_OK;
     cudaGraphExec_t ex = m->prof ? nullptr : reexec_graph(m, bucket);
     if (ex) {
@@ -963,6 +1088,7 @@ ct_status reexec_rows(ct_model *m, const float *input, int batch, const uint8_t 
         s = infer_impl(m, m->re_input, bucket, m->re_logits, m->re_S, m->re_flag, st);
     }
     m->armed = armed;
+    m->flag_mirror = mirror;
     if (s != CT_OK) return s;
     CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] { return launch_scatter_rows(m->re_logits, logits, m->re_idx, n, m->n_classes, st); }));
     if (S) CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] { return launch_scatter_rows(m->re_S, S, m->re_idx, n, 1, st); }));
@@ -1005,6 +1131,16 @@ ct_status infer_with_reruns(ct_model *m, const float *input, int batch, float *l
         return infer_impl(m, input, batch, logits, S, flag, st);
     }
     if (n_rerun) *n_rerun = n;
+    if (m->small && n <= SMALL_MAX_RERUN) {
+        // the whole-network kernel reads the re-run images and writes their rows itself
+        SmallRerun rr{};
+        rr.x = prev_input;
+        rr.logits = prev_logits;
+        rr.S = prev_S;
+        rr.n = n;
+        for (int j = 0; j < n; ++j) rr.idx[j] = idx_host[j];
+        return infer_impl(m, input, batch, logits, S, flag, st, nullptr, 0, &rr);
+    }
     CUDA_TRY(cudaMemcpyAsync(m->re_idx, idx_host, sizeof(int32_t) * n, cudaMemcpyHostToDevice, st));
     const int64_t per = (int64_t)m->in_c * m->in_h * m->in_w;
     CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] { return launch_gather_images(prev_input, m->re_input, m->re_idx, n, per, st); }));
@@ -1082,6 +1218,8 @@ ct_status reexec_rows_of(ct_model *m, int nb, In in, Fl fl, Lg lg, Sv Sp, int ba
                                  sizeof(float) * per, cudaMemcpyDeviceToDevice, st));
     const bool armed = m->armed;
     m->armed = false;
+    uint8_t *const mirror = m->flag_mirror;
+    m->flag_mirror = nullptr;
     ct_status s = CT_OK;
     cudaGraphExec_t ex = m->prof ? nullptr : reexec_graph(m, bucket);
     if (ex) {
@@ -1093,6 +1231,7 @@ ct_status reexec_rows_of(ct_model *m, int nb, In in, Fl fl, Lg lg, Sv Sp, int ba
         s = infer_impl(m, m->re_input, bucket, m->re_logits, m->re_S, m->re_flag, st);
     }
     m->armed = armed;
+    m->flag_mirror = mirror;
     if (s != CT_OK) return s;
     for (int j = 0, o = 0; j < nb; o += cnt[j], ++j) {
         if (!cnt[j]) continue;
@@ -1111,7 +1250,8 @@ ct_status reexec_rows_of(ct_model *m, int nb, In in, Fl fl, Lg lg, Sv Sp, int ba
 ct_status pipe_setup(ct_model *m, bool host) {
     if (!m->pipe_ready) {
         const size_t B = (size_t)m->max_batch;
-        if (cudaMallocHost((void **)&m->pipe_flags_h, ct_model::PIPE * B) != cudaSuccess ||
+        if (cudaHostAlloc((void **)&m->pipe_flags_h, ct_model::PIPE * B, cudaHostAllocMapped) != cudaSuccess ||
+            cudaHostGetDevicePointer((void **)&m->pipe_flags_d, m->pipe_flags_h, 0) != cudaSuccess ||
             cudaMallocHost((void **)&m->pipe_idx_h, sizeof(int32_t) * (ct_model::PIPE + 2) * B) != cudaSuccess) {
             cudaGetLastError();
             return CT_ENOMEM;
@@ -1187,6 +1327,8 @@ ct_status run_batches(ct_model *m, int n, int batch, const BatchIO &io, bool hos
         }
         ct_status r;
         int nr = 0;
+        // the final kernel writes this batch's flags to the mapped host ring too
+        m->flag_mirror = m->pipe_flags_d + (size_t)s * B;
         if (i >= 2) {
             const int q = (i - 2) % P;
             CUDA_TRY(cudaEventSynchronize(m->pipe_ev_flags[q]));
@@ -1196,9 +1338,9 @@ ct_status run_batches(ct_model *m, int n, int batch, const BatchIO &io, bool hos
         } else {
             r = infer_impl(m, dev_in(i), batch, dev_lg(i), dev_S(i), dev_fl(i), st);
         }
+        m->flag_mirror = nullptr;
         if (r != CT_OK) return r;
         reruns += nr;
-        CUDA_TRY(cudaMemcpyAsync(m->pipe_flags_h + (size_t)s * B, dev_fl(i), batch, cudaMemcpyDeviceToHost, st));
         CUDA_TRY(cudaEventRecord(m->pipe_ev_flags[s], st));
         CUDA_TRY(cudaEventRecord(m->pipe_ev_step[s], st));
         if (host && i >= 2) {
@@ -1414,48 +1556,13 @@ ct_status ct_infer_reexec(ct_model *m, const float *input_dev, int32_t batch, fl
     return s;
 }
 
-// The LeNet shape the batched campaign kernel runs (FP32, widened):
-// conv -> pool -> conv -> pool -> fc -> fc -> fc, with ReLU after every conv
-// and hidden FC, 2x2 stride-2 pools, unpadded stride-1 convolutions with a
-// carry-through filter.
-static bool small_net_of(const ct_model *m, SmallNet *g) {
-    if (m->prec != CT_FP32 || !m->protect || m->L.size() != 7) return false;
-    const LayerRT &c1 = m->L[0], &p1 = m->L[1], &c2 = m->L[2], &p2 = m->L[3];
-    const LayerRT &f1 = m->L[4], &f2 = m->L[5], &f3 = m->L[6];
-    auto conv_ok = [](const LayerRT &l) {
-        return l.d.op == CT_OP_CONV && l.d.stride == 1 && l.d.pad == 0 && l.d.relu && l.d.res < 0 &&
-               l.role == CT_ROLE_CT && l.R == l.S && l.w_ld == l.R * l.S * l.C && l.c_stride == l.C;
-    };
-    auto pool_ok = [](const LayerRT &l) { return l.d.op == CT_OP_MAXPOOL && l.d.k == 2 && l.d.stride == 2 && l.d.pad == 0; };
-    if (!conv_ok(c1) || !pool_ok(p1) || !conv_ok(c2) || !pool_ok(p2)) return false;
-    if (c1.d.src != 0 || p1.d.src != c1.d.dst || c2.d.src != p1.d.dst || p2.d.src != c2.d.dst) return false;
-    if (f1.d.op != CT_OP_FC || f2.d.op != CT_OP_FC || f3.d.op != CT_OP_FC || !f1.d.relu || !f2.d.relu ||
-        !f3.d.final || f1.d.src != p2.d.dst || f2.d.src != f1.d.dst || f3.d.src != f2.d.dst)
-        return false;
-    if (c1.cs_in || !c2.cs_in || f1.x_float || f1.fc_tc || f2.fc_tc) return false;
-    const Slot &s1 = m->slots[p1.d.dst], &s2 = m->slots[p2.d.dst];
-    SmallNet &n = *g;
-    memset(&n, 0, sizeof(n));
-    n.C0 = c1.C; n.H0 = c1.H; n.W0 = c1.W;
-    n.K1 = c1.K; n.R1 = c1.R; n.H1 = c1.P; n.W1 = c1.Q; n.Hp1 = s1.H; n.Wp1 = s1.W;
-    n.K2 = c2.K; n.R2 = c2.R; n.H2 = c2.P; n.W2 = c2.Q; n.Hp2 = s2.H; n.Wp2 = s2.W;
-    n.NIN1 = f1.n_in; n.N1 = f1.n_out; n.N2 = f2.n_out; n.N3 = f3.n_out;
-    if (n.NIN1 != n.K2 * n.Hp2 * n.Wp2 || f1.n_cs != n.Hp2 * n.Wp2 || f2.n_in != n.N1 || f3.n_in != n.N2) return false;
-    n.w1 = (const float *)c1.w; n.b1 = c1.bias; n.w2 = (const float *)c2.w; n.b2 = c2.bias;
-    n.wf1 = (const float *)f1.w; n.bf1 = f1.bias; n.wf2 = (const float *)f2.w; n.bf2 = f2.bias;
-    n.wf3 = (const float *)f3.w; n.bf3 = f3.bias;
-    n.coef1 = c1.coef; n.coef2 = c2.coef; n.coeff1 = f1.coef; n.coeff2 = f2.coef; n.coeff3 = f3.coef;
-    n.ref = m->ref; n.tau = m->tau;
-    return campaign_small_smem(n) <= 200 * 1024;
-}
-
 ct_status ct_campaign_batched(ct_model *m, const float *input_dev, int32_t batch, const ct_fault *faults,
                               int32_t n_faults, float *S_dev, int32_t *top1_dev, uint8_t *flag_dev, void *stream) {
     if (!m || !input_dev || (n_faults > 0 && (!faults || !S_dev || !top1_dev || !flag_dev)) || n_faults < 0)
         return CT_EINVAL;
     if (batch < 1 || batch > m->max_batch) return CT_ERANGE;
     SmallNet g;
-    if (!small_net_of(m, &g)) return CT_EUNSUPPORTED;
+    if (!m->protect || !small_net_of(m, &g)) return CT_EUNSUPPORTED;
     if (n_faults == 0) return CT_OK;
     g.B = batch;
     g.x = input_dev;
@@ -1710,7 +1817,7 @@ ct_status ct_copy_activation(ct_model *m, int32_t slot, int32_t batch, void *dat
     if (!m) return CT_EINVAL;
     if (slot < 0 || slot >= (int)m->slots.size() || batch < 1 || batch > m->max_batch) return CT_ERANGE;
     const Slot &sl = m->slots[slot];
-    if (!sl.stored) return CT_ESTATE;
+    if (!sl.stored || sl.skipped_last) return CT_ESTATE;
     if (!sl.data) return CT_ERANGE;
     const size_t e = sl.is_float ? 4 : m->esz();
     if (C) *C = sl.cp;

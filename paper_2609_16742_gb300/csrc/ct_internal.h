@@ -52,6 +52,10 @@ struct ConvArgs {
 // columns in the NHWC flatten order), coefficients and threshold.
 struct SmallNet {
     int B, C0, H0, W0;
+    int protect;                          // widened construction (0: the network alone)
+    const float *x2;                      // images n >= n_split are image n - n_split of x2 (null: none)
+    int n_split;
+    uint8_t *flag2;                       // inference: a second copy of the flags (host-mapped) or null
     int K1, R1, H1, W1, Hp1, Wp1;
     int K2, R2, H2, W2, Hp2, Wp2;
     int NIN1, N1, N2, N3;
@@ -63,7 +67,7 @@ struct SmallNet {
 
 // One fault of a batched campaign, resolved on the host.
 struct CampFault {
-    int kind;            // 0 weight, 1 activation
+    int kind;            // 0 weight, 1 activation, 2 none
     int layer;           // weight: 0 first convolution, 1 second
     long long word;      // weight: stored word to flip (-1: use fd)
     int bit;
@@ -77,6 +81,20 @@ cudaError_t launch_conv_dw(const ConvArgs &a, bool half, cudaStream_t st);
 size_t campaign_small_smem(const SmallNet &g);
 cudaError_t launch_campaign_small(const SmallNet &g, const CampFault *faults, int n_faults, float *S, int32_t *top1,
                                   uint8_t *flag, cudaStream_t st);
+// Re-run list of a whole-network inference: images idx[0 .. n) of x, their
+// logits and S written to those rows of logits / S.
+constexpr int SMALL_MAX_RERUN = 128;
+struct SmallRerun {
+    const float *x;
+    float *logits, *S;
+    int n;
+    int idx[SMALL_MAX_RERUN];
+};
+// Inference of g.B images with the whole-network kernel: logits [B, N3],
+// S [B] and flags [B] (each may be null), with `fault` (kind 2: none)
+// applied, plus the fault-free re-run list rr (rr.n = 0: none).
+cudaError_t launch_small_infer(const SmallNet &g, const CampFault &fault, float *logits, float *S, uint8_t *flag,
+                               const SmallRerun &rr, cudaStream_t st);
 
 struct FcArgs {
     const void *x;        // [B, n_in] data features
@@ -87,6 +105,7 @@ struct FcArgs {
     void *ycs;            // [B] carry-through neuron (hidden) or null
     float *S;             // final: [B] or null
     uint8_t *flag;        // final: [B] or null
+    uint8_t *flag2;       // final: a second copy of the flags (host-mapped memory) or null
     int B, n_in, n_cs, n_out;
     int relu, final_layer, protect;
     float coef;
@@ -218,8 +237,11 @@ struct HaloPlan;
 bool halo_supported(int C, int K, int R, int S, int stride, int pad, int H, int W);
 // res_dev / csin_dev / rescs_dev: residual tensor, incoming and residual
 // checksum planes the layer reads (null if none); launches must pass them.
+// pool: the layer's 2 x 2 stride-2 max-pool is applied in the epilogue (even
+// H and W); launches then pass the pooled tensor and plane as y / cs_out.
 HaloPlan *halo_plan_create(const ConvArgs &shape_args, int max_batch, const void *w_dev, const void *x_dev,
-                           const void *res_dev, const void *csin_dev, const void *rescs_dev, std::string *why);
+                           const void *res_dev, const void *csin_dev, const void *rescs_dev, bool pool,
+                           std::string *why);
 void halo_plan_destroy(HaloPlan *p);
 int halo_tiles(const HaloPlan *p, int batch);
 int halo_sms(const HaloPlan *p);

@@ -159,6 +159,7 @@ __global__ void __launch_bounds__(256) fc_kernel(FcArgs a) {
                 if (b >= a.B) continue;
                 if (a.S) a.S[b] = __int_as_float(0x7fc00000);
                 if (a.flag) a.flag[b] = 0;
+                if (a.flag2) a.flag2[b] = 0;
             }
         }
         return;
@@ -174,7 +175,9 @@ __global__ void __launch_bounds__(256) fc_kernel(FcArgs a) {
         s *= a.coef;
         if (a.final_layer) {
             if (a.S) a.S[b] = s;
-            if (a.flag) a.flag[b] = !(fabs((double)s - a.ref) <= a.tau);
+            const uint8_t fv = !(fabs((double)s - a.ref) <= a.tau);
+            if (a.flag) a.flag[b] = fv;
+            if (a.flag2) a.flag2[b] = fv;
         } else {
             if (a.relu) s = relu_keep_nan(s);
             static_cast<TY *>(a.ycs)[b] = from_f<TY>(s);
@@ -209,6 +212,7 @@ __global__ void fc_reduce_kernel(FcArgs a, int splits) {
             if (a.final_layer) {
                 if (a.S) a.S[b] = __int_as_float(0x7fc00000);
                 if (a.flag) a.flag[b] = 0;
+                if (a.flag2) a.flag2[b] = 0;
             }
             continue;
         }
@@ -220,7 +224,9 @@ __global__ void fc_reduce_kernel(FcArgs a, int splits) {
         s *= a.coef;
         if (a.final_layer) {
             if (a.S) a.S[b] = s;
-            if (a.flag) a.flag[b] = !(fabs((double)s - a.ref) <= a.tau);
+            const uint8_t fv = !(fabs((double)s - a.ref) <= a.tau);
+            if (a.flag) a.flag[b] = fv;
+            if (a.flag2) a.flag2[b] = fv;
         } else {
             if (a.relu) s = relu_keep_nan(s);
             static_cast<TY *>(a.ycs)[b] = from_f<TY>(s);

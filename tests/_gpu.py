@@ -25,11 +25,11 @@ def ct():
 
 
 def model(name: str, prec: str = None, protect: bool = True, simt_only: bool = False,
-          max_batch: int = None, ds_mode: str = "pass"):
+          max_batch: int = None, ds_mode: str = "pass", layerwise: bool = False):
     wl = synth.workload(name)
     return ct().ct_build_workload(wl, params(name), precision=prec or wl.precision,
                                   protect=protect, simt_only=simt_only,
-                                  max_batch=max_batch or wl.batch, ds_mode=ds_mode)
+                                  max_batch=max_batch or wl.batch, ds_mode=ds_mode, layerwise=layerwise)
 
 
 def run(m, x_np):

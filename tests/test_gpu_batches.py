@@ -73,3 +73,37 @@ def test_host_batches_equal_device_batches():
                   "fp32", "host batches")
     # a second call reuses the library's slots
     assert ct().ct_run_host_batches(m, xh[:2], B, lh[:2], None, None) == 0
+
+
+def test_lenet5_whole_network_kernel_reruns_inside_the_kernel():
+    """LeNet-5 runs as one whole-network kernel per batch; a flagged image's
+    re-run is a row of that same kernel (it reads the image from the earlier
+    batch and writes its logits and S there).  An activation flip (bit 30 of
+    the largest checksum value of conv2's input, image 5 of batch 0) makes S
+    explode; after the call every image matches the oracle."""
+    import torch
+    name, Bl, nb = "lenet5", 16, 4
+    net = onet(name, "fp32")
+    x = inputs(name, Bl * nb)
+    o = oracle.forward(net, x, keep=True)
+    m = model(name, max_batch=Bl + 8)
+    r = float(np.mean(o["S"]))
+    ct().ct_set_threshold(m, r, float(np.abs(o["S"] - r).max()) * 1.01)
+    cs = o["acts"][5][2][-1]                        # checksum plane of conv2's input, image 5
+    kept = np.zeros_like(cs, dtype=bool)
+    kept[2:-2, 2:-2] = True                         # the centre taps conv2 (5x5, no padding) samples
+    pix = int(np.argmax(np.where(kept, cs, -1.0)))
+    assert 0.5 <= cs.reshape(-1)[pix] < 2.0
+    per = int(np.prod(oracle.act_shape(net, 2, 1)[1:]))
+    ct().ct_inject(m, 1, 2, 5 * per + (per - cs.size) + pix, 30)
+    xs = [torch.from_numpy(x[i * Bl:(i + 1) * Bl]).cuda() for i in range(nb)]
+    lg = [torch.full((Bl, m.n_classes), float("nan"), device="cuda") for _ in range(nb)]
+    S = [torch.full((Bl,), float("nan"), device="cuda") for _ in range(nb)]
+    fl = [torch.full((Bl,), 7, dtype=torch.uint8, device="cuda") for _ in range(nb)]
+    n = ct().ct_infer_batches(m, xs, Bl, lg, S, fl)
+    flags = torch.cat(fl).cpu().numpy()
+    assert flags[5] == 1 and flags.sum() == 1 and n == 1, (flags.nonzero(), n)
+    assert_parity(torch.cat(lg).cpu().numpy().astype(np.float64), torch.cat(S).cpu().numpy().astype(np.float64),
+                  o["logits"], o["S"], "fp32", "lenet5 batches")
+    assert ct().ct_launches_per_infer(m) == 1
+    assert ct().ct_device_error(m) == 0

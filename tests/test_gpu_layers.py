@@ -14,9 +14,11 @@ CT_ESTATE = 4
 
 
 def layer_errors(name, prec, batch, simt_only=False, first=0):
-    """[(slot, op, data_rel_err, cs_rel_err)] for one inference; raises on a device error."""
+    """[(slot, op, data_rel_err, cs_rel_err)] for one inference, one kernel per
+    layer (LeNet-5 otherwise runs as one whole-network kernel that stores no
+    intermediate tensor); raises on a device error."""
     wl = synth.workload(name)
-    m = model(name, prec=prec, simt_only=simt_only, max_batch=batch)
+    m = model(name, prec=prec, simt_only=simt_only, max_batch=batch, layerwise=True)
     x = inputs(name, batch, first)
     run(m, x)
     code = ct().ct_device_error(m)
@@ -75,3 +77,16 @@ def test_small_batches_split_k():
     base = ct().ct_launches_per_infer(m)
     run(m, inputs("resnet18_imagenet", 2))
     assert ct().ct_launches_per_infer(m) > base
+
+
+def test_whole_network_kernel_stores_no_intermediate_tensor():
+    """LeNet-5 (FP32) runs as one kernel: its logits and S match the oracle
+    (test_gpu_parity) and its intermediate tensors are reported as not
+    stored."""
+    m = model("lenet5", max_batch=4)
+    run(m, inputs("lenet5", 4))
+    assert ct().ct_launches_per_infer(m) == 1
+    for slot in (1, 2, 3, 4):
+        with pytest.raises(ct().CtError) as ei:
+            ct().ct_copy_activation(m, slot, 4)
+        assert ei.value.status == CT_ESTATE

@@ -144,3 +144,37 @@ def test_roles_derived_by_the_library_build_the_same_network():
     lm, Sm, _ = run(model(name, max_batch=4), x)
     assert np.array_equal(la, lm) and np.array_equal(Sa, Sm)
     ma.close()
+
+
+def test_vgg16_fused_pool_under_weight_faults():
+    """VGG-16's first two stride-1 layers apply the following 2 x 2 max-pool in
+    their halo-tile epilogue.  Single-bit flips in conv1_2's weights -- a
+    stored data weight, the carry-through row off its centre tap and the
+    zero checksum slice (the last two are implicit and enter the epilogue as
+    a delta) -- give the oracle's S and logits on the images they touch."""
+    name, B = "vgg16", 2
+    m = model(name, max_batch=B)
+    net = onet(name, "fp16")
+    x = inputs(name, B)
+    lg, S, _ = run(m, x)
+    o = oracle.forward(net, x)
+    assert_parity(lg, S, o["logits"], o["S"], "fp16", "vgg16 fused pools")
+    with pytest.raises(ct().CtError) as ei:          # the unpooled conv1_2 output is not stored
+        ct().ct_copy_activation(m, 2, B)
+    assert ei.value.status == 4
+    layer = 1                                         # conv1_2: 64 -> 64 (+1), input 64 (+1) channels
+    K, C = 64, 64
+    def el(k, c, r, s_):
+        return ((k * (C + 1) + c) * 3 + r) * 3 + s_
+    for e, bit in [(el(5, 7, 1, 1), 14), (el(K, 3, 0, 2), 14), (el(9, C, 1, 1), 13)]:
+        ct().ct_inject(m, 0, layer, e, bit)
+        lg, S, _ = run(m, x)
+        of = oracle.forward(net, x, oracle.Fault(0, layer, e, bit))
+        for i in range(B):
+            assert same_class(S[i], of["S"][i]), (e, bit, S[i], of["S"][i])
+            if np.isfinite(of["S"][i]):
+                assert abs(S[i] - of["S"][i]) <= TOL["fp16"] * max(abs(of["S"][i]), 1e-6), (e, bit, S[i], of["S"][i])
+            if np.isfinite(of["logits"][i]).all():
+                err = np.abs(lg[i] - of["logits"][i]).max() / max(np.abs(of["logits"][i]).max(), 1e-6)
+                assert err <= TOL["fp16"], (e, bit, err)
+    assert ct().ct_device_error(m) == 0
