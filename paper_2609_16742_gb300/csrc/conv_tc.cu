@@ -85,6 +85,10 @@ struct TcGeom {
     int tmem_cols;
     int m_tiles, n_tiles;
     int splits, kps, ws_ld;      // split-K: K blocks per split, workspace row length
+    // conv_tc_pair_kernel<true>: tiles t_first .. end are each run as two
+    // 128-channel halves, units 0 .. units - t_first - 1 (unit 2 * (tile -
+    // t_first) + half); whole tiles 0 .. t_first - 1 follow them
+    int t_first, units;
     uint16_t coef_h;
 };
 
@@ -215,6 +219,30 @@ __device__ __forceinline__ Bias16 load_bias16(const float *bias, int k0) {
 #pragma unroll
     for (int i = 0; i < 4; ++i) b.q[i] = __ldg(p + i);
     return b;
+}
+// Bias of the conv kernels' epilogue: a copy in shared memory (up to
+// BIAS_SMEM output channels), filled once per CTA, so that the per-chunk
+// bias read costs no global-memory round trip; else the global array.
+constexpr int BIAS_SMEM = 1024;
+__device__ __forceinline__ Bias16 bias16_at(const float *bias_s, const float *bias_g, bool in_smem, int k0) {
+    if (in_smem) {
+        const float4 *p = reinterpret_cast<const float4 *>(bias_s + k0);
+        Bias16 b;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) b.q[i] = p[i];
+        return b;
+    }
+    return load_bias16(bias_g, k0);
+}
+// Copy of the bias into shared memory by the epilogue warps (named barrier 1
+// over those warps only).  Returns whether the copy was made.
+__device__ __forceinline__ bool stage_bias(float *bias_s, const float *bias_g, int K, int t, int nthreads) {
+    const bool in_smem = bias_g != nullptr && K <= BIAS_SMEM;
+    if (in_smem) {
+        for (int i = t; i < K; i += nthreads) bias_s[i] = __ldg(bias_g + i);
+        asm volatile("bar.sync 1, %0;" ::"r"(nthreads) : "memory");
+    }
+    return in_smem;
 }
 __device__ __forceinline__ uint32_t cvt_h2(float lo, float hi, bool relu) {
     uint32_t r;
@@ -369,6 +397,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
     uint64_t *ct_ready = acc_empty + 2;                   // [2]
     uint32_t *tmem_holder = (uint32_t *)(ct_ready + 2);
     volatile uint32_t *abort_flag = tmem_holder + 1;
+    float *bias_s = (float *)(((uintptr_t)(tmem_holder + 2) + 15) & ~(uintptr_t)15);   // [BIAS_SMEM]
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int cid = blockIdx.x, ncl = gridDim.x;
@@ -597,6 +626,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
         const FaultDelta fd = a.fd;
         const bool split = g.splits > 1;
         const bool has_res = a.res != nullptr, relu = a.relu != 0;
+        const bool bias_sm = stage_bias(bias_s, a.bias, g.K, threadIdx.x - 32 * TC_EPI_WARP0, 32 * N_EPI_WARPS);
         int lt = 0;
         for (int tile = cid; tile < num_items; tile += ncl, ++lt) {
             const TileRef tr = tile_ref(tile, g);
@@ -678,7 +708,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
                     __half *yrow = static_cast<__half *>(a.y) + (size_t)m * g.K + n0 + half * (BN / 2);
 #pragma unroll
                     for (int c = 0; c < BN / 2; c += 16)
-                        store16_fast(vals + c, load_bias16(a.bias, n0 + half * (BN / 2) + c), rs[c / 16], has_res,
+                        store16_fast(vals + c, bias16_at(bias_s, a.bias, bias_sm, n0 + half * (BN / 2) + c), rs[c / 16], has_res,
                                      relu, yrow + c);
                     if (do_cs) store_checksum_pre(ctv, csv, a, g, m, 0.f);
                 }
@@ -700,8 +730,8 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
                     } else if (valid && fd.active) {
                         store_chunk_pre(v, rs[(c - half * (BN / 2)) / 16], a, g.K, (size_t)m, n0 + c, fsrc);
                     } else if (valid) {
-                        store16_fast(v, load_bias16(a.bias, n0 + c), rs[(c - half * (BN / 2)) / 16], has_res, relu,
-                                     static_cast<__half *>(a.y) + (size_t)m * g.K + n0 + c);
+                        store16_fast(v, bias16_at(bias_s, a.bias, bias_sm, n0 + c), rs[(c - half * (BN / 2)) / 16], has_res,
+                                     relu, static_cast<__half *>(a.y) + (size_t)m * g.K + n0 + c);
                     }
                 }
                 if (do_cs && g.ct_mode != CT_NONE_) ctv = ct_sum[ab * BM + row];
@@ -741,6 +771,13 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
 //   acc_full[b]    each CTA: accumulator b complete (commit multicast)
 //   pair_empty[b]  even CTA: both epilogues have read accumulator b
 //   mma_done       each CTA: every MMA of the pair completed (before dealloc)
+//
+// Last-round balance (conv_tc_pair_kernel<true>).  When the last round of
+// tiles would leave more than half the pairs idle, each tile of that round
+// runs as two units of 128 channels (M = 256, N = 128 MMAs: each CTA copies
+// 64 weight rows), on different pairs and before the whole tiles.  Every
+// output is still one full-K accumulation, so the result does not depend on
+// the split.
 constexpr int PR_STAGES = 6;
 constexpr int PR_NPROD = 2;
 constexpr int PR_MMA_WARP = PR_NPROD;
@@ -749,13 +786,26 @@ constexpr int PR_THREADS = 32 * (PR_EPI_WARP0 + N_EPI_WARPS);
 constexpr int PR_BH_BYTES = BM * BK * 2;                  // this CTA's 128 weight rows of a stage
 constexpr int PR_NBAR = 2 * PR_STAGES + 5;                // full, empty per stage; acc_full, pair_empty, mma_done
 
-size_t pair_smem_bytes() {
-    return 1024 + (size_t)PR_STAGES * (A_BYTES + PR_BH_BYTES) + 8 * PR_NBAR + 16;
+// Work unit u of a pair kernel: its 256 x 256 tile and channel half (-1:
+// all 256 channels).
+struct PairUnit {
+    int item, nh;
+};
+template <bool SPLIT>
+__device__ __forceinline__ PairUnit pair_unit(int u, const TcGeom &g) {
+    const int n_h = SPLIT ? g.units - g.t_first : 0;
+    if (u >= n_h) return PairUnit{u - n_h, -1};
+    return PairUnit{g.t_first + (u >> 1), u & 1};
 }
 
+size_t pair_smem_bytes() {
+    return 1024 + (size_t)PR_STAGES * (A_BYTES + PR_BH_BYTES) + 8 * PR_NBAR + 16 + 16 + 4 * BIAS_SMEM;
+}
+
+template <bool SPLIT>
 __global__ void __launch_bounds__(PR_THREADS, 1)
 conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
-                    const ConvArgs a, const TcGeom g) {
+                    const __grid_constant__ CUtensorMap bmap64, const ConvArgs a, const TcGeom g) {
     constexpr int BN = 256;
     static_assert(PR_STAGES % PR_NPROD == 0, "producer warps must own whole ring slots");
     extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -769,13 +819,13 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
     uint64_t *mma_done = pair_empty + 2;
     uint32_t *tmem_holder = (uint32_t *)(mma_done + 1);
     volatile uint32_t *abort_flag = tmem_holder + 1;
+    float *bias_s = (float *)(((uintptr_t)(tmem_holder + 2) + 15) & ~(uintptr_t)15);   // [BIAS_SMEM]
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t crank = cluster_ctarank();
     const bool leader = crank == 0;
     const int cid = blockIdx.x >> 1, ncl = gridDim.x >> 1;
-    const int m_pairs = (g.m_tiles + 1) >> 1;
-    const int num_items = m_pairs * g.n_tiles;
+    const int num_units = SPLIT ? g.units : ((g.m_tiles + 1) >> 1) * g.n_tiles;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < PR_STAGES; ++s) {
@@ -810,14 +860,17 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
         if (elect_one()) {
             asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&amap) : "memory");
             asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&bmap) : "memory");
+            if (SPLIT) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&bmap64) : "memory");
         }
         __syncwarp();
         const uint32_t full_even = mapa_shared(smem_u32(full), 0u);
         int it = 0;
         bool ok = true;
-        for (int item = cid; item < num_items && ok; item += ncl) {
+        for (int u = cid; u < num_units && ok; u += ncl) {
             if (__any_sync(0xffffffffu, *abort_flag)) break;
-            const int m_pair = item / g.n_tiles, n_tile = item % g.n_tiles;
+            const PairUnit pu = pair_unit<SPLIT>(u, g);
+            const bool hu = SPLIT && pu.nh >= 0;                  // a 128-channel half
+            const int m_pair = pu.item / g.n_tiles, n_tile = pu.item % g.n_tiles;
             const int m0 = (2 * m_pair + (int)crank) * BM;       // past M: rows that are never stored
             const int nimg = m0 / g.PQ, rem = m0 % g.PQ;
             const int p = rem / g.Q, q = rem % g.Q;
@@ -828,14 +881,19 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
                 if (!warp_wait(smem_u32(&empty[s]), ((uint32_t)(it / PR_STAGES) & 1u) ^ 1u, a.err, 1u)) { ok = false; break; }
                 if (elect_one()) {
                     const uint32_t fb = full_even + (uint32_t)(s * 8);
-                    if (leader) mbar_arrive_expect_tx(smem_u32(&full[s]), 2u * (A_BYTES + PR_BH_BYTES));
+                    if (leader)
+                        mbar_arrive_expect_tx(smem_u32(&full[s]), 2u * (A_BYTES + (hu ? PR_BH_BYTES / 2 : PR_BH_BYTES)));
                     const int tap = tap_of(kb / g.cpb, g.ctr_tap);
                     const int c0 = (kb % g.cpb) * BK;
                     const int r = tap / g.S, sx = tap % g.S;
                     tma_load_im2col_pair(smem_u32(As + s * A_BYTES), &amap, fb, c0, w0, h0, nimg, (uint16_t)sx,
                                          (uint16_t)r);
-                    tma_load_2d_pair(smem_u32(Bs + s * PR_BH_BYTES), &bmap, fb, tap * g.C + c0,
-                                     n_tile * BN + (int)crank * BM);
+                    if (hu)
+                        tma_load_2d_pair(smem_u32(Bs + s * PR_BH_BYTES), &bmap64, fb, tap * g.C + c0,
+                                         n_tile * BN + pu.nh * (BN / 2) + (int)crank * (BM / 2));
+                    else
+                        tma_load_2d_pair(smem_u32(Bs + s * PR_BH_BYTES), &bmap, fb, tap * g.C + c0,
+                                         n_tile * BN + (int)crank * BM);
                 }
                 __syncwarp();
             }
@@ -844,10 +902,11 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
     } else if (warp == PR_MMA_WARP) {
         // ---------------- MMA issuer: the even CTA, one elected lane ----------------
         if (leader) {
-            const uint32_t idesc = idesc_f16(2 * BM, BN);
             int it = 0, lt = 0;
-            for (int item = cid; item < num_items; item += ncl, ++lt) {
+            for (int u = cid; u < num_units; u += ncl, ++lt) {
                 if (__any_sync(0xffffffffu, *abort_flag)) break;
+                const bool hu = SPLIT && pair_unit<SPLIT>(u, g).nh >= 0;
+                const uint32_t idesc = idesc_f16(2 * BM, hu ? BN / 2 : BN);
                 const int ab = lt & 1;
                 if (!warp_wait(smem_u32(&pair_empty[ab]), ((uint32_t)(lt >> 1) & 1u) ^ 1u, a.err, 8u)) {
                     if (lane == 0) *abort_flag = 1;
@@ -890,20 +949,28 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
         const int ctr_r = g.ctr_tap / g.S, ctr_s = g.ctr_tap % g.S;
         const uint32_t pair_empty_even = mapa_shared(smem_u32(pair_empty), 0u);
         const bool has_res = a.res != nullptr, relu = a.relu != 0;
+        const bool bias_sm = stage_bias(bias_s, a.bias, g.K, threadIdx.x - 32 * PR_EPI_WARP0, 32 * N_EPI_WARPS);
         int lt = 0;
-        for (int item = cid; item < num_items; item += ncl, ++lt) {
-            const int m_pair = item / g.n_tiles, n_tile = item % g.n_tiles;
+        for (int u = cid; u < num_units; u += ncl, ++lt) {
+            const PairUnit pu = pair_unit<SPLIT>(u, g);
+            const bool hu = SPLIT && pu.nh >= 0;
+            const int m_pair = pu.item / g.n_tiles, n_tile = pu.item % g.n_tiles;
             const int m0 = (2 * m_pair + (int)crank) * BM;
             const int m = m0 + row;
             const bool valid = m < g.M;
             const int mm = valid ? m : 0;
             const int nimg = mm / g.PQ, rem = mm % g.PQ, p = rem / g.Q, q = rem % g.Q;
-            const bool do_cs = half == 0 && a.cs_out != nullptr && n_tile == 0;
+            const bool do_cs = half == 0 && a.cs_out != nullptr && n_tile == 0 && !(hu && pu.nh > 0);
+            // this warp's channels: cols [cw, cw + ncw) of the accumulator,
+            // output channels nw + (0 .. ncw)
+            const int ncw = hu ? BN / 4 : BN / 2;
+            const int cw = half * ncw;
+            const int nw = n_tile * BN + (hu ? pu.nh * (BN / 2) : 0) + cw;
             Res16 rs[BN / 32];
 #pragma unroll
             for (int c = 0; c < BN / 32; ++c)
-                rs[c] = valid ? load_res16(a, g.K, (size_t)m, n_tile * BN + half * (BN / 2) + 16 * c)
-                              : Res16{make_uint4(0u, 0u, 0u, 0u), make_uint4(0u, 0u, 0u, 0u)};
+                rs[c] = (valid && 16 * c < ncw) ? load_res16(a, g.K, (size_t)m, nw + 16 * c)
+                                                : Res16{make_uint4(0u, 0u, 0u, 0u), make_uint4(0u, 0u, 0u, 0u)};
             CsIn csv{0.f, 0.f};
             // carry-through column: coef * sum of the C channels of the centre-tap pixel
             float ctv = 0.f;
@@ -943,15 +1010,15 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
                     else if (a.cs_in) fsrc = ldh(static_cast<const __half *>(a.cs_in), ((size_t)nimg * a.H + h) * a.W + w);
                 }
             }
-            const int n0 = n_tile * BN;
 #pragma unroll
-            for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 16) {
+            for (int c = 0; c < BN / 2; c += 16) {
+                if (c >= ncw) break;
                 float v[16];
-                tmem_ld16(trow + c, v);
-                if (valid && fd.active) store_chunk_pre(v, rs[(c - half * (BN / 2)) / 16], a, g.K, (size_t)m, n0 + c, fsrc);
+                tmem_ld16(trow + cw + c, v);
+                if (valid && fd.active) store_chunk_pre(v, rs[c / 16], a, g.K, (size_t)m, nw + c, fsrc);
                 else if (valid)
-                    store16_fast(v, load_bias16(a.bias, n0 + c), rs[(c - half * (BN / 2)) / 16], has_res, relu,
-                                 static_cast<__half *>(a.y) + (size_t)m * g.K + n0 + c);
+                    store16_fast(v, bias16_at(bias_s, a.bias, bias_sm, nw + c), rs[c / 16], has_res, relu,
+                                 static_cast<__half *>(a.y) + (size_t)m * g.K + nw + c);
             }
             if (do_cs && valid) store_checksum_pre(ctv, csv, a, g, m, fsrc);
             asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -1670,7 +1737,7 @@ bool load_encoders() {
 template <int BN, int STAGES, int SUB>
 size_t smem_bytes() {
     return 1024 + (size_t)STAGES * SUB * (A_BYTES + (BN + 16) * BK * 2) + 16 * BK * 2 + 2 * BM * 4 +
-           8 * (2 * STAGES + 6) + 16;
+           8 * (2 * STAGES + 6) + 16 + 16 + 4 * BIAS_SMEM;
 }
 
 uint16_t coef_half_bits(float c) {
@@ -1699,6 +1766,7 @@ struct TcPlan {
     int BN, n_tiles, sms;
     size_t smem;
     CUtensorMap bmap_pair;       // N = 256 over CTA pairs: 128-row weight halves
+    CUtensorMap bmap_pair64;     // 128-channel half tiles: 64-row weight quarters
     int pair_clusters;           // resident CTA pairs (0: no pair variant)
     size_t pair_smem;
 };
@@ -1772,9 +1840,17 @@ TcPlan *tc_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, cons
         r = g_encode_tiled(&pl->bmap_pair, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void *>(w_dev), bdim, bstr,
                            box_h, bes, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        cuuint32_t box_q[2] = {BK, (cuuint32_t)(BM / 2)};
+        if (r == CUDA_SUCCESS)
+            r = g_encode_tiled(&pl->bmap_pair64, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void *>(w_dev), bdim,
+                               bstr, box_q, bes, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
         pl->pair_smem = pair_smem_bytes();
-        cudaError_t pe = cudaFuncSetAttribute(conv_tc_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        cudaError_t pe = cudaFuncSetAttribute(conv_tc_pair_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                               (int)pl->pair_smem);
+        if (pe == cudaSuccess)
+            pe = cudaFuncSetAttribute(conv_tc_pair_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      (int)pl->pair_smem);
         if (r == CUDA_SUCCESS && pe == cudaSuccess) {
             cudaLaunchConfig_t cfg = {};
             cfg.gridDim = dim3(2 * 64);
@@ -1788,7 +1864,7 @@ TcPlan *tc_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, cons
             cfg.attrs = at;
             cfg.numAttrs = 1;
             int n = 0;
-            if (cudaOccupancyMaxActiveClusters(&n, conv_tc_pair_kernel, &cfg) == cudaSuccess && n > 0)
+            if (cudaOccupancyMaxActiveClusters(&n, conv_tc_pair_kernel<false>, &cfg) == cudaSuccess && n > 0)
                 pl->pair_clusters = n;
         }
         cudaGetLastError();
@@ -1811,9 +1887,20 @@ cudaError_t launch_conv_tc(const ConvArgs &a, const void *plan, cudaStream_t st,
     if (pl->pair_clusters > 0 && g.splits == 1 && g.m_tiles >= 2) {
         // N = 256 tiles over CTA pairs: 256 pixels x 256 channels per pair
         const int items = ((g.m_tiles + 1) / 2) * g.n_tiles;
-        const int ncl = items < pl->pair_clusters ? items : pl->pair_clusters;
-        pdl_launch_cluster(conv_tc_pair_kernel, dim3(2 * ncl), PR_THREADS, pl->pair_smem, st, 2, pl->amap,
-                           pl->bmap_pair, a, g);
+        const int P = pl->pair_clusters;
+        // last round: rem tiles on P pairs; as 2 * rem half tiles when they
+        // fit in one round (the round then takes half a tile time)
+        const int rem = items % P;
+        const bool halves = rem > 0 && 2 * rem <= P;
+        g.t_first = halves ? items - rem : items;
+        g.units = halves ? items + rem : items;
+        const int ncl = g.units < P ? g.units : P;
+        if (halves)
+            pdl_launch_cluster(conv_tc_pair_kernel<true>, dim3(2 * ncl), PR_THREADS, pl->pair_smem, st, 2, pl->amap,
+                               pl->bmap_pair, pl->bmap_pair64, a, g);
+        else
+            pdl_launch_cluster(conv_tc_pair_kernel<false>, dim3(2 * ncl), PR_THREADS, pl->pair_smem, st, 2, pl->amap,
+                               pl->bmap_pair, pl->bmap_pair64, a, g);
     } else {
         const int items = tiles * g.splits;
         dim3 grid(items < pl->sms ? items : pl->sms);

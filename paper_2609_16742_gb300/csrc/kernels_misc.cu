@@ -28,7 +28,7 @@ constexpr int FC_J = 16, FC_IMG = 64, FC_KC = 64, FC_WARPS = 8;
 static_assert((FC_KC * (FC_IMG + 1)) % 4 == 0, "weight tile must start 16-byte aligned (float4 reads)");
 
 template <typename TX, typename TW, typename TY>
-__global__ void __launch_bounds__(256) fc_kernel(FcArgs a) {
+__global__ void __launch_bounds__(256, 2) fc_kernel(FcArgs a) {
     pdl_wait();
     pdl_trigger();
     extern __shared__ __align__(16) float smem[];

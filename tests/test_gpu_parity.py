@@ -178,3 +178,28 @@ def test_vgg16_fused_pool_under_weight_faults():
                 err = np.abs(lg[i] - of["logits"][i]).max() / max(np.abs(of["logits"][i]).max(), 1e-6)
                 assert err <= TOL["fp16"], (e, bit, err)
     assert ct().ct_device_error(m) == 0
+
+
+def test_half_tiles_of_the_last_round_give_whole_tile_bits():
+    """A 512 -> 512 3 x 3 convolution on 7 x 7 maps: 256 images make 98
+    CTA-pair tiles for 76 pairs, and the 22 tiles of the last round (images
+    199-255) run as 44 half tiles of 128 channels; 128 images make 50 tiles,
+    all whole.  Each output is the same full-K accumulation either way, so
+    images 128-255 give the same bits (data and checksum) in both runs."""
+    import synth
+    from synth import Layer
+    shape = (512, 7, 7)
+    layers = [Layer("conv", 0, 1, cin=512, cout=512, k=3, stride=1, pad=1, ct="ct", bn=True, relu=True),
+              Layer("gap", 1, 2), Layer("fc", 2, 3, cin=512, cout=10, final=True)]
+    params = synth.make_params(layers, 11)
+    x = np.random.default_rng(5).standard_normal((256,) + shape).astype(np.float32)
+    out = {}
+    for B in (256, 128):
+        m = ct().ct_build(layers, params, shape, 10, precision="fp16", max_batch=B)
+        run(m, x[256 - B:])
+        out[B] = ct().ct_copy_activation(m, 1, B)
+        assert ct().ct_device_error(m) == 0
+        m.close()
+    (d256, c256), (d128, c128) = out[256], out[128]
+    assert np.isfinite(d256).all() and np.abs(d256).max() > 0
+    assert np.array_equal(d256[128:], d128) and np.array_equal(c256[128:], c128)
