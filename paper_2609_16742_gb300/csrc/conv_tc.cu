@@ -38,8 +38,9 @@
 // Warp roles.  conv_tc_kernel: a producer group (producer warps, each owning
 // whole ring slots, plus for N = 256 the two carry-through warps), one MMA
 // warp (one elected lane issues tcgen05.mma), eight epilogue warps;
-// conv_tc_pair_kernel: two producer warps, the MMA warp (issuing in the even
-// CTA only), eight epilogue warps.
+// conv_tc_pair_kernel: three producer warps, each owning two ring slots (with
+// two, the copy issue held the 7 x 7 layers back by 8%, measured), the MMA
+// warp (issuing in the even CTA only), eight epilogue warps.
 // conv_tc_halo_kernel (320 threads): warp 0 issues TMA, warp 1 the MMAs,
 // warps 2-9 the epilogue.  Each TMEM lane quadrant (32 output pixels) is
 // read by two epilogue warps, each taking half of the tile's channels.
@@ -779,30 +780,36 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
 // output is still one full-K accumulation, so the result does not depend on
 // the split.
 constexpr int PR_STAGES = 6;
-constexpr int PR_NPROD = 2;
+constexpr int PR_NPROD = 3;
 constexpr int PR_MMA_WARP = PR_NPROD;
 constexpr int PR_EPI_WARP0 = PR_MMA_WARP + 1;
 constexpr int PR_THREADS = 32 * (PR_EPI_WARP0 + N_EPI_WARPS);
 constexpr int PR_BH_BYTES = BM * BK * 2;                  // this CTA's 128 weight rows of a stage
 constexpr int PR_NBAR = 2 * PR_STAGES + 5;                // full, empty per stage; acc_full, pair_empty, mma_done
 
-// Work unit u of a pair kernel: its 256 x 256 tile and channel half (-1:
-// all 256 channels).
+// Work unit u of a pair kernel: its tile (256 pixels x 256 channels), first
+// output channel, and whether it is a 128-channel half (else all 256).
 struct PairUnit {
-    int item, nh;
+    int item, nb;
+    bool narrow;
 };
-template <bool SPLIT>
+template <bool VARN>
 __device__ __forceinline__ PairUnit pair_unit(int u, const TcGeom &g) {
-    const int n_h = SPLIT ? g.units - g.t_first : 0;
-    if (u >= n_h) return PairUnit{u - n_h, -1};
-    return PairUnit{g.t_first + (u >> 1), u & 1};
+    if (!VARN) return PairUnit{u, (u % g.n_tiles) * 256, false};
+    const int n_h = g.units - g.t_first;
+    if (u >= n_h) {
+        const int it = u - n_h;
+        return PairUnit{it, (it % g.n_tiles) * 256, false};
+    }
+    const int it = g.t_first + (u >> 1);
+    return PairUnit{it, (it % g.n_tiles) * 256 + (u & 1) * 128, true};
 }
 
 size_t pair_smem_bytes() {
     return 1024 + (size_t)PR_STAGES * (A_BYTES + PR_BH_BYTES) + 8 * PR_NBAR + 16 + 16 + 4 * BIAS_SMEM;
 }
 
-template <bool SPLIT>
+template <bool VARN>
 __global__ void __launch_bounds__(PR_THREADS, 1)
 conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
                     const __grid_constant__ CUtensorMap bmap64, const ConvArgs a, const TcGeom g) {
@@ -825,7 +832,7 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
     const uint32_t crank = cluster_ctarank();
     const bool leader = crank == 0;
     const int cid = blockIdx.x >> 1, ncl = gridDim.x >> 1;
-    const int num_units = SPLIT ? g.units : ((g.m_tiles + 1) >> 1) * g.n_tiles;
+    const int num_units = VARN ? g.units : ((g.m_tiles + 1) >> 1) * g.n_tiles;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < PR_STAGES; ++s) {
@@ -860,7 +867,7 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
         if (elect_one()) {
             asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&amap) : "memory");
             asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&bmap) : "memory");
-            if (SPLIT) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&bmap64) : "memory");
+            if (VARN) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&bmap64) : "memory");
         }
         __syncwarp();
         const uint32_t full_even = mapa_shared(smem_u32(full), 0u);
@@ -868,9 +875,9 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
         bool ok = true;
         for (int u = cid; u < num_units && ok; u += ncl) {
             if (__any_sync(0xffffffffu, *abort_flag)) break;
-            const PairUnit pu = pair_unit<SPLIT>(u, g);
-            const bool hu = SPLIT && pu.nh >= 0;                  // a 128-channel half
-            const int m_pair = pu.item / g.n_tiles, n_tile = pu.item % g.n_tiles;
+            const PairUnit pu = pair_unit<VARN>(u, g);
+            const bool hu = VARN && pu.narrow;                    // 128 channels
+            const int m_pair = pu.item / g.n_tiles;
             const int m0 = (2 * m_pair + (int)crank) * BM;       // past M: rows that are never stored
             const int nimg = m0 / g.PQ, rem = m0 % g.PQ;
             const int p = rem / g.Q, q = rem % g.Q;
@@ -890,10 +897,10 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
                                          (uint16_t)r);
                     if (hu)
                         tma_load_2d_pair(smem_u32(Bs + s * PR_BH_BYTES), &bmap64, fb, tap * g.C + c0,
-                                         n_tile * BN + pu.nh * (BN / 2) + (int)crank * (BM / 2));
+                                         pu.nb + (int)crank * (BM / 2));
                     else
                         tma_load_2d_pair(smem_u32(Bs + s * PR_BH_BYTES), &bmap, fb, tap * g.C + c0,
-                                         n_tile * BN + (int)crank * BM);
+                                         pu.nb + (int)crank * BM);
                 }
                 __syncwarp();
             }
@@ -905,7 +912,7 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
             int it = 0, lt = 0;
             for (int u = cid; u < num_units; u += ncl, ++lt) {
                 if (__any_sync(0xffffffffu, *abort_flag)) break;
-                const bool hu = SPLIT && pair_unit<SPLIT>(u, g).nh >= 0;
+                const bool hu = VARN && pair_unit<VARN>(u, g).narrow;
                 const uint32_t idesc = idesc_f16(2 * BM, hu ? BN / 2 : BN);
                 const int ab = lt & 1;
                 if (!warp_wait(smem_u32(&pair_empty[ab]), ((uint32_t)(lt >> 1) & 1u) ^ 1u, a.err, 8u)) {
@@ -952,20 +959,20 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
         const bool bias_sm = stage_bias(bias_s, a.bias, g.K, threadIdx.x - 32 * PR_EPI_WARP0, 32 * N_EPI_WARPS);
         int lt = 0;
         for (int u = cid; u < num_units; u += ncl, ++lt) {
-            const PairUnit pu = pair_unit<SPLIT>(u, g);
-            const bool hu = SPLIT && pu.nh >= 0;
-            const int m_pair = pu.item / g.n_tiles, n_tile = pu.item % g.n_tiles;
+            const PairUnit pu = pair_unit<VARN>(u, g);
+            const bool hu = VARN && pu.narrow;
+            const int m_pair = pu.item / g.n_tiles;
             const int m0 = (2 * m_pair + (int)crank) * BM;
             const int m = m0 + row;
             const bool valid = m < g.M;
             const int mm = valid ? m : 0;
             const int nimg = mm / g.PQ, rem = mm % g.PQ, p = rem / g.Q, q = rem % g.Q;
-            const bool do_cs = half == 0 && a.cs_out != nullptr && n_tile == 0 && !(hu && pu.nh > 0);
+            const bool do_cs = half == 0 && a.cs_out != nullptr && pu.nb == 0;
             // this warp's channels: cols [cw, cw + ncw) of the accumulator,
             // output channels nw + (0 .. ncw)
             const int ncw = hu ? BN / 4 : BN / 2;
             const int cw = half * ncw;
-            const int nw = n_tile * BN + (hu ? pu.nh * (BN / 2) : 0) + cw;
+            const int nw = pu.nb + cw;
             Res16 rs[BN / 32];
 #pragma unroll
             for (int c = 0; c < BN / 32; ++c)
@@ -1833,7 +1840,9 @@ TcPlan *tc_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, cons
         e = cudaFuncSetAttribute(conv_tc_kernel<256, 4, 1, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
     }
     if (e != cudaSuccess) { if (why) *why = "shared memory attribute"; delete pl; return nullptr; }
-    // N = 256 over CTA pairs (cta_group::2): each CTA copies 128 of the 256 weight rows
+    // N = 256 over CTA pairs (cta_group::2): each CTA copies half of the
+    // tile's weight rows.  (128-channel layers stay on the single-CTA
+    // kernel: on CTA pairs they ran 10-30% slower, measured.)
     pl->pair_clusters = 0;
     if (pl->BN == 256) {
         cuuint32_t box_h[2] = {BK, (cuuint32_t)BM};
@@ -1885,11 +1894,11 @@ cudaError_t launch_conv_tc(const ConvArgs &a, const void *plan, cudaStream_t st,
     g.splits = (a.K % 8 == 0) ? splitk_choose(tiles, g.n_kb, 4, pl->sms / 2, g.M, g.ws_ld, a.ws ? a.ws_bytes : 0) : 1;
     g.kps = (g.n_kb + g.splits - 1) / g.splits;
     if (pl->pair_clusters > 0 && g.splits == 1 && g.m_tiles >= 2) {
-        // N = 256 tiles over CTA pairs: 256 pixels x 256 channels per pair
+        // tiles over CTA pairs: 256 pixels x 256 channels per pair
         const int items = ((g.m_tiles + 1) / 2) * g.n_tiles;
         const int P = pl->pair_clusters;
-        // last round: rem tiles on P pairs; as 2 * rem half tiles when they
-        // fit in one round (the round then takes half a tile time)
+        // last round of 256-channel tiles: rem tiles on P pairs; as 2 * rem
+        // half tiles when they fit in one round (it then takes half a tile time)
         const int rem = items % P;
         const bool halves = rem > 0 && 2 * rem <= P;
         g.t_first = halves ? items - rem : items;
