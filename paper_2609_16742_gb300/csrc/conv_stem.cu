@@ -33,10 +33,13 @@
 // maxima go through a shared-memory row buffer for the 3-wide horizontal
 // maximum and the pooled row is written.
 //
-// Warp roles (480 threads): warps 0-5 fill ring rows (entry e goes to warp
-// e % 6), warp 6 allocates TMEM and issues tcgen05.mma (one elected lane),
-// warps 7-14 are the epilogue: each TMEM lane quadrant is read by two warps,
-// each taking 32 of the 64 channels.  Four TMEM accumulators rotate over
+// Warp roles (512 threads): warps 0-5 fill ring rows (entry e goes to warp
+// e % 6), warps 6 and 7 issue tcgen05.mma (one elected lane each, for
+// alternate convolution rows: issuing one row's 14 MMAs and 3 commits takes
+// a thread about 900 cycles, so one issuer left the tensor core idle half the
+// time, measured), warp 6 also allocates TMEM, warps 8-15 are the epilogue:
+// each TMEM lane quadrant is read by two warps, each taking 32 of the 64
+// channels.  Four TMEM accumulators rotate over
 // consecutive convolution rows, so the MMAs run up to three rows ahead of
 // the epilogue.  Every mbarrier wait is bounded; on
 // expiry the kernel records an error code, stops and frees TMEM.
@@ -62,8 +65,9 @@ constexpr int ST_B_STEP = ST_NB * 32;        // B bytes per K16 step (two core-m
 constexpr int ST_B_LBO = ST_NB * 16;         // between the two K chunks of a step
 constexpr int ST_PIX_H = 72;                 // halves per pixel in the epilogue row buffer (144 B)
 constexpr int ST_NPROD = 6;                  // ring producer warps
-constexpr int ST_MMA_WARP = ST_NPROD;
-constexpr int ST_EPI0 = 32 * (ST_NPROD + 1); // first epilogue thread
+constexpr int ST_NMMA = 2;                   // MMA warps: convolution rows alternate between them
+constexpr int ST_MMA_WARP = ST_NPROD;        // the first also allocates TMEM
+constexpr int ST_EPI0 = 32 * (ST_NPROD + ST_NMMA);   // first epilogue thread
 constexpr int ST_THREADS = ST_EPI0 + 256;
 constexpr int ST_EPI = 256;                  // epilogue threads
 constexpr int ST_NACC = 4;                   // TMEM accumulators (rows in flight between MMA and epilogue)
@@ -82,7 +86,7 @@ constexpr int ST_NSTG = ST_NPROD * ST_STG_W;
 constexpr int ST_STG_BYTES = 4 * 256 * 4;
 constexpr size_t ST_OFF_STG = ST_OFF_CS + 2ull * 128 * 2;
 constexpr size_t ST_OFF_BAR = ST_OFF_STG + (size_t)ST_NSTG * ST_STG_BYTES;
-constexpr size_t ST_SMEM = 1024 + ST_OFF_BAR + 8 * (2 * ST_NSLOT + 2 * ST_NACC + 1 + ST_NSTG) + 16;
+constexpr size_t ST_SMEM = 1024 + ST_OFF_BAR + 8 * (2 * ST_NSLOT + 2 * ST_NACC + ST_NMMA + ST_NSTG) + 16;
 
 struct StemGeom {
     int N, C, H, W, P, Q, P2, Q2;
@@ -218,8 +222,8 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
     uint64_t *empty = full + ST_NSLOT;
     uint64_t *acc_full = empty + ST_NSLOT;
     uint64_t *acc_empty = acc_full + ST_NACC;
-    uint64_t *mma_done = acc_empty + ST_NACC;
-    uint64_t *stg_full = mma_done + 1;                       // [ST_NSTG]
+    uint64_t *mma_done = acc_empty + ST_NACC;                // [ST_NMMA]
+    uint64_t *stg_full = mma_done + ST_NMMA;                 // [ST_NSTG]
     float *stg = (float *)(smem + ST_OFF_STG);
     uint32_t *tmem_holder = (uint32_t *)(stg_full + ST_NSTG);
     volatile uint32_t *abort_flag = tmem_holder + 1;
@@ -261,13 +265,13 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
     if (threadIdx.x == 0) {
         for (int s = 0; s < ST_NSLOT; ++s) {
             mbar_init(smem_u32(&full[s]), 32);
-            mbar_init(smem_u32(&empty[s]), 1);
+            mbar_init(smem_u32(&empty[s]), ST_NMMA);      // one release per MMA warp
         }
         for (int b = 0; b < ST_NACC; ++b) {
             mbar_init(smem_u32(&acc_full[b]), 1);
             mbar_init(smem_u32(&acc_empty[b]), ST_EPI / 32);
         }
-        mbar_init(smem_u32(mma_done), 1);
+        for (int w = 0; w < ST_NMMA; ++w) mbar_init(smem_u32(&mma_done[w]), 1);
         for (int s = 0; s < ST_NSTG; ++s) mbar_init(smem_u32(&stg_full[s]), 1);
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -355,68 +359,105 @@ stem_pool_kernel(const ConvArgs a, const StemGeom g) {
                 warp_wait(smem_u32(&stg_full[warp * ST_STG_W + k % ST_STG_W]), (uint32_t)(k / ST_STG_W) & 1u,
                           a.err, 1u);
         }
-    } else if (warp == ST_MMA_WARP) {
-        // ---------------- MMA issuer (whole warp, one lane issues) ----------------
+    } else if (warp < ST_MMA_WARP + ST_NMMA) {
+        // ---------------- MMA issuers: job j goes to MMA warp j % ST_NMMA ----------------
+        // One elected lane issues a job's 14 MMAs; the issue of one job and
+        // the barrier waits of the next overlap across the two warps.  A ring
+        // row is released once by each MMA warp, in row order, as soon as
+        // none of that warp's later jobs reads it: after its job j, the rows
+        // below the window of its next job j + 2 (all remaining rows after its
+        // last job).  The release is a commit, so it also waits for the MMAs.
+        const int mw = warp - ST_MMA_WARP;
         const uint32_t id64 = idesc_f16(128, ST_K);
         const uint32_t id80 = idesc_f16(128, ST_NB);
         const uint32_t ring_base = smem_u32(ring), b_base = smem_u32(Bs);
-        StemJobs jb;
-        bool have = jb.first(u0, u1, g);
-        int ecount = 0, j = 0;
-        bool issued = false;
-        while (have) {
-            if (__any_sync(0xffffffffu, *abort_flag)) break;
-            const int wstart = jb.seg_start ? ecount : ecount - 5;
-            ecount += jb.seg_start ? 7 : 2;
-            StemJobs nx = jb;
-            const bool have_next = nx.next(g);
-            const int nrel = (have_next && !nx.seg_start) ? 2 : 7;
-            const int ab = j % ST_NACC;
-            const uint32_t use = (uint32_t)(j / ST_NACC) & 1u;
-            bool ok = warp_wait(smem_u32(&acc_empty[ab]), use ^ 1u, a.err, 8u);
-            // only the rows new to this window: the others were waited for by
-            // an earlier row of the run and stay until it releases them
-            for (int r = jb.seg_start ? 0 : ST_R - 2; r < ST_R && ok; ++r) {
-                const int e = wstart + r;
-                ok = warp_wait(smem_u32(&full[e % ST_NSLOT]), (uint32_t)(e / ST_NSLOT) & 1u, a.err, 2u);
-            }
-            if (!ok) { if (lane == 0) *abort_flag = 1; break; }
-            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-            if (elect_one()) {
-                const uint32_t d = tmem + (uint32_t)(ab * 128);
+        // descriptors: the weights' are fixed; a ring row's is the ring base
+        // descriptor plus the row's offset in 16-byte units (the start
+        // address field of a no-swizzle descriptor is addr >> 4)
+        uint64_t bd[ST_KSTEPS];
 #pragma unroll
-                for (int i = 0; i < ST_R; ++i) {
-                    const int r = i == 0 ? 3 : (i <= 3 ? i - 1 : i);    // centre row first
-                    const uint32_t row = ring_base + (uint32_t)(((wstart + r) % ST_NSLOT) * ST_SLOT_BYTES);
-                    const uint64_t a0 = smem_desc_noswz(row, 16, 128);
-                    const uint64_t a1 = smem_desc_noswz(row + ST_ROW_BYTES + 32, 16, 128);
-                    const uint64_t b0 = smem_desc_noswz(b_base + (2 * r) * ST_B_STEP, ST_B_LBO, 128);
-                    const uint64_t b1 = smem_desc_noswz(b_base + (2 * r + 1) * ST_B_STEP, ST_B_LBO, 128);
-                    // the first MMA (centre row) writes all 80 columns when the
-                    // carry-through row is present
-                    umma_f16(d, a0, b0, (i == 0 && g.ct) ? id80 : id64, i > 0 ? 1u : 0u);
-                    umma_f16(d, a1, b1, id64, 1u);
-                }
-                umma_commit(smem_u32(&acc_full[ab]));
-                for (int t = 0; t < nrel; ++t) umma_commit(smem_u32(&empty[(wstart + t) % ST_NSLOT]));
+        for (int t = 0; t < ST_KSTEPS; ++t) bd[t] = smem_desc_noswz(b_base + t * ST_B_STEP, ST_B_LBO, 128);
+        const uint64_t ad_base = smem_desc_noswz(ring_base, 16, 128);
+        // window starts of jobs j, j + 1, j + 2 (scanned ahead of the issue)
+        StemJobs scan;
+        bool scan_have = scan.first(u0, u1, g);
+        int scan_ec = 0;                       // ring entries of the jobs scanned so far
+        int ws[3];
+        bool hv[3];
+        auto scan_one = [&](int &w, bool &h) {
+            h = scan_have;
+            w = 0;
+            if (scan_have) {
+                w = scan.seg_start ? scan_ec : scan_ec - 5;
+                scan_ec += scan.seg_start ? 7 : 2;
+                scan_have = scan.next(g);
             }
-            __syncwarp();
-            issued = true;
-            jb = nx;
-            have = have_next;
+        };
+        scan_one(ws[0], hv[0]);
+        scan_one(ws[1], hv[1]);
+        scan_one(ws[2], hv[2]);
+        int j = 0, waited = 0, rel = 0;
+        bool issued = false, ok = true;
+        while (hv[0]) {
+            if (j % ST_NMMA == mw) {
+                if (__any_sync(0xffffffffu, *abort_flag)) { ok = false; break; }
+                const int wstart = ws[0];
+                const int ab = j % ST_NACC;
+                const uint32_t use = (uint32_t)(j / ST_NACC) & 1u;
+                ok = warp_wait(smem_u32(&acc_empty[ab]), use ^ 1u, a.err, 8u);
+                // the rows of the window this warp has not waited for
+                for (int e = max(waited, wstart); e < wstart + ST_R && ok; ++e)
+                    ok = warp_wait(smem_u32(&full[e % ST_NSLOT]), (uint32_t)(e / ST_NSLOT) & 1u, a.err, 2u);
+                if (!ok) { if (lane == 0) *abort_flag = 1; break; }
+                waited = wstart + ST_R;
+                const int rel_end = hv[ST_NMMA] ? ws[ST_NMMA] : scan_ec;
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                if (elect_one()) {
+                    const uint32_t d = tmem + (uint32_t)(ab * 128);
+                    int slot = wstart % ST_NSLOT;
+                    uint64_t ad[ST_R];
+#pragma unroll
+                    for (int r = 0; r < ST_R; ++r) {
+                        ad[r] = ad_base + (uint64_t)((slot * ST_SLOT_BYTES) >> 4);
+                        slot = slot + 1 == ST_NSLOT ? 0 : slot + 1;
+                    }
+#pragma unroll
+                    for (int i = 0; i < ST_R; ++i) {
+                        const int r = i == 0 ? 3 : (i <= 3 ? i - 1 : i);    // centre row first
+                        // the first MMA (centre row) writes all 80 columns when the
+                        // carry-through row is present
+                        umma_f16(d, ad[r], bd[2 * r], (i == 0 && g.ct) ? id80 : id64, i > 0 ? 1u : 0u);
+                        umma_f16(d, ad[r] + (uint64_t)((ST_ROW_BYTES + 32) >> 4), bd[2 * r + 1], id64, 1u);
+                    }
+                    umma_commit(smem_u32(&acc_full[ab]));
+                    for (int e = rel; e < rel_end; ++e) umma_commit(smem_u32(&empty[e % ST_NSLOT]));
+                }
+                __syncwarp();
+                rel = max(rel, rel_end);
+                issued = true;
+            }
+            ws[0] = ws[1]; hv[0] = hv[1];
+            ws[1] = ws[2]; hv[1] = hv[2];
+            scan_one(ws[2], hv[2]);
             ++j;
+        }
+        // a warp with no job after some rows (or none at all) still releases them
+        if (ok && rel < scan_ec) {
+            if (elect_one())
+                for (int e = rel; e < scan_ec; ++e) umma_commit(smem_u32(&empty[e % ST_NSLOT]));
+            __syncwarp();
         }
         // every issued MMA has completed before TMEM can be freed
         if (issued) {
-            if (elect_one()) umma_commit(smem_u32(mma_done));
+            if (elect_one()) umma_commit(smem_u32(&mma_done[mw]));
             __syncwarp();
-            warp_wait(smem_u32(mma_done), 0u, a.err, 16u);
+            warp_wait(smem_u32(&mma_done[mw]), 0u, a.err, 16u);
         }
     } else {
-        // ---------------- epilogue: warps 7..14 ----------------
+        // ---------------- epilogue: warps 8..15 ----------------
         const int et = threadIdx.x - ST_EPI0;
         const int quad = warp & 3;
-        const int half_id = (warp - ST_MMA_WARP - 1) >> 2;           // channels 32 * half_id ..
+        const int half_id = (warp - ST_MMA_WARP - ST_NMMA) >> 2;     // channels 32 * half_id ..
         const int q = quad * 32 + lane;                 // output column of this thread
         const int k0 = 32 * half_id;
         const FaultDelta fd = a.fd;
