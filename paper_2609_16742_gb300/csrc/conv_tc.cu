@@ -161,9 +161,11 @@ struct Res16 {
 __device__ __forceinline__ Res16 load_res16(const ConvArgs &a, int K, size_t m, int k0) {
     Res16 r;
     if (a.res) {
-        const uint4 *rp = reinterpret_cast<const uint4 *>(static_cast<const __half *>(a.res) + m * K + k0);
-        r.r0 = rp[0];
-        r.r1 = rp[1];
+        // K and k0 are multiples of 16 channels: 32-byte aligned
+        uint32_t w[8];
+        ld_global_nc_v8(static_cast<const __half *>(a.res) + m * K + k0, w);
+        r.r0 = make_uint4(w[0], w[1], w[2], w[3]);
+        r.r1 = make_uint4(w[4], w[5], w[6], w[7]);
     } else {
         r.r0 = r.r1 = make_uint4(0u, 0u, 0u, 0u);
     }
@@ -269,9 +271,7 @@ __device__ __forceinline__ void store16_fast(const float *v, const Bias16 &b, co
     uint32_t pk[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i) pk[i] = cvt_h2(t[2 * i], t[2 * i + 1], relu);
-    uint4 *yp = reinterpret_cast<uint4 *>(dst);
-    yp[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-    yp[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+    st_global_v8(dst, pk);          // 16 channels of one pixel: 32-byte aligned
 }
 
 // Epilogue values of 16 channels k0 .. k0 + 15 of one pixel in FP32, in the
@@ -1676,11 +1676,7 @@ conv_tc_halo_kernel(const __grid_constant__ HaloMaps maps, const ConvArgs a, con
 #pragma unroll
                     for (int i = 0; i < 8; ++i)
                         pk[i] = cvt_h2(pool2x2_lanes(t[2 * i]), pool2x2_lanes(t[2 * i + 1]), false);
-                    if (writer) {
-                        uint4 *yp = reinterpret_cast<uint4 *>(static_cast<__half *>(a.y) + mp * hg.K + n0 + c);
-                        yp[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-                        yp[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
-                    }
+                    if (writer) st_global_v8(static_cast<__half *>(a.y) + mp * hg.K + n0 + c, pk);
                 }
                 if (do_cs) {
                     const float o = pool2x2_lanes(checksum_value(ctv, csv, a, g, fsrc));

@@ -62,6 +62,20 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint32_
     }
 }
 
+// 32-byte global accesses (one request instead of two 16-byte ones; the
+// epilogues write 32 bytes of one pixel's row per lane, so a warp store
+// touches 32 rows either way).  Addresses must be 32-byte aligned.
+__device__ __forceinline__ void st_global_v8(void *p, const uint32_t (&v)[8]) {
+    asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p), "r"(v[0]), "r"(v[1]),
+                 "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7])
+                 : "memory");
+}
+__device__ __forceinline__ void ld_global_nc_v8(const void *p, uint32_t (&v)[8]) {
+    asm volatile("ld.global.nc.v8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+                 : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7])
+                 : "l"(p));
+}
+
 // One lane of a converged warp: issues TMA / tcgen05 instructions while the
 // whole warp computes their (warp-uniform) operands.
 __device__ __forceinline__ bool elect_one() {

@@ -6,8 +6,9 @@ is collected last on purpose."""
 import numpy as np
 import pytest
 
+import oracle
 from _cache import inputs
-from _gpu import TOL, ct, model, run
+from _gpu import TOL, assert_parity, ct, model, onet, run
 
 pytestmark = pytest.mark.gpu
 
@@ -48,6 +49,11 @@ def test_noalloc_reexecute_matches_reexecute_twice():
         assert (err <= TOL["fp32"]).all(), (call, err.max())
         sa, sb = S_a.cpu().numpy(), S_b.cpu().numpy()
         assert (np.abs(sa - sb) <= TOL["fp32"] * np.abs(sa)).all(), call
+        # and the re-run rows against the oracle (Sec. II-B: a fault-free
+        # re-execution of the flagged images)
+        rows = np.nonzero(flags.cpu().numpy())[0][:3]
+        o = oracle.forward(onet(name, "fp32"), x[rows])
+        assert_parity(b[rows], sb[rows], o["logits"], o["S"], "fp32", "noalloc re-run rows")
 
 
 def test_noalloc_rejects_a_batch_beyond_its_scratch():
