@@ -154,10 +154,14 @@ __device__ __forceinline__ uint32_t hmax2u(uint32_t a, uint32_t b) {
 }
 
 // image n of the batch: images n >= n_split come from the second input
-// (re-executed images appended to a batch)
+// (re-executed images appended to a batch), directly or through the index
+// list x2_idx
 __device__ __forceinline__ const float *image_base(const ConvArgs &a, const StemGeom &g, int n) {
     const size_t chw = (size_t)g.C * g.H * g.W;
-    if (a.x2 && n >= a.n_split) return static_cast<const float *>(a.x2) + (size_t)(n - a.n_split) * chw;
+    if (a.x2 && n >= a.n_split) {
+        const int i = a.x2_idx ? a.x2_idx[n - a.n_split] : n - a.n_split;
+        return static_cast<const float *>(a.x2) + (size_t)i * chw;
+    }
     return static_cast<const float *>(a.x) + (size_t)n * chw;
 }
 

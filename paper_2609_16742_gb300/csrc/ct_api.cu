@@ -139,7 +139,8 @@ struct ct_model {
     uint8_t *re_flag = nullptr;
     int32_t *re_idx = nullptr;
     uint8_t *h_flags = nullptr;
-    int32_t *h_idx = nullptr;
+    int32_t *h_idx = nullptr;          // host memory mapped for the device
+    int32_t *h_idx_d = nullptr;        // its device address
     // batched campaign: resolved faults (device) and their pinned staging
     CampFault *camp_d = nullptr, *camp_h = nullptr;
     int camp_cap = 0;
@@ -164,7 +165,8 @@ struct ct_model {
     static constexpr int PIPE = 6;
     uint8_t *pipe_flags_h = nullptr;      // [PIPE][max_batch], host memory mapped for the device
     uint8_t *pipe_flags_d = nullptr;      // its device address
-    int32_t *pipe_idx_h = nullptr;        // [PIPE + 2][max_batch]
+    int32_t *pipe_idx_h = nullptr;        // [PIPE + 2][max_batch], host memory mapped for the device
+    int32_t *pipe_idx_d = nullptr;        // its device address
     cudaEvent_t pipe_ev_flags[PIPE] = {}, pipe_ev_step[PIPE] = {}, pipe_ev_in[PIPE] = {}, pipe_ev_out[PIPE] = {};
     cudaEvent_t pipe_ev_tail = nullptr;
     bool pipe_ready = false;
@@ -229,6 +231,7 @@ void free_all(ct_model *m) {
     if (m->pipe_idx_h) cudaFreeHost(m->pipe_idx_h);
     m->pipe_flags_h = nullptr;
     m->pipe_idx_h = nullptr;
+    m->pipe_idx_d = nullptr;
     for (int i = 0; i < ct_model::PIPE; ++i)
         for (cudaEvent_t *e : {&m->pipe_ev_flags[i], &m->pipe_ev_step[i], &m->pipe_ev_in[i], &m->pipe_ev_out[i]})
             if (*e) { cudaEventDestroy(*e); *e = nullptr; }
@@ -730,7 +733,9 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
     if ((st = dalloc(m, (void **)&m->ws, SPLITK_WS_BYTES)) != CT_OK) return st;
     CUDA_TRY(cudaMemset(m->d_err, 0, sizeof(uint32_t)));
     if (cudaMallocHost((void **)&m->h_flags, B) != cudaSuccess) return CT_ENOMEM;
-    if (cudaMallocHost((void **)&m->h_idx, sizeof(int32_t) * B) != cudaSuccess) return CT_ENOMEM;
+    if (cudaHostAlloc((void **)&m->h_idx, sizeof(int32_t) * B, cudaHostAllocMapped) != cudaSuccess ||
+        cudaHostGetDevicePointer((void **)&m->h_idx_d, m->h_idx, 0) != cudaSuccess)
+        return CT_ENOMEM;
     CUDA_TRY(cudaDeviceSynchronize());
     return CT_OK;
 }
@@ -835,9 +840,17 @@ static bool small_net_of(const ct_model *m, SmallNet *g) {
 // input2 / n_split: images n >= n_split of the batch are image n - n_split
 // of input2 (re-executed images appended to a batch); the rest of the
 // network is unaware of it
+// Re-executed images appended to an inference as rows n_split .. batch - 1:
+// image idx[j] of the earlier batch's input (input2), whose logits and S
+// rows they write.  idx is device-visible (mapped host memory).
+struct RerunRows {
+    const int32_t *idx;
+    float *logits, *S;
+};
+
 ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, float *S,
                      uint8_t *flag, cudaStream_t st, const float *input2 = nullptr, int n_split = 0,
-                     const SmallRerun *rerun = nullptr) {
+                     const SmallRerun *rerun = nullptr, const RerunRows *rows = nullptr) {
     const bool half = m->prec == CT_FP16;
     const int wb = half ? 2 : 4;
     if (m->small) {
@@ -903,7 +916,8 @@ ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, 
         if (input2) {
             void *dst2 = static_cast<uint8_t *>(s0.data) + (size_t)n_split * s0.H * s0.W * s0.cp * wb;
             CUDA_TRY(launch(m, FAM_OTHER, 0, st, [&] {
-                return launch_convert_input(input2, dst2, batch - n_split, s0.C, s0.cp, s0.H, s0.W, half, st);
+                return launch_convert_input(input2, dst2, batch - n_split, s0.C, s0.cp, s0.H, s0.W, half, st,
+                                            rows ? rows->idx : nullptr);
             }));
         }
     }
@@ -939,6 +953,7 @@ ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, 
                 a.x = input;
                 a.x2 = input2;
                 a.n_split = n_first;
+                a.x2_idx = rows ? rows->idx : nullptr;
                 a.y = po.data;
                 a.cs_out = po.has_cs ? po.cs : nullptr;
                 CUDA_TRY(launch(m, FAM_TC, flops, st, [&] { return launch_stem_pool(a, l.stplan, st); }));
@@ -999,7 +1014,10 @@ ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, 
             // sums every input feature (the checksum channel is one of them)
             a.protect = m->protect || (m->replace && d.final);
             a.ref = m->ref; a.tau = m->tau;
-            if (d.final) { a.y = logits; a.S = S; a.flag = flag; a.flag2 = m->flag_mirror; }
+            if (d.final) {
+                a.y = logits; a.S = S; a.flag = flag; a.flag2 = m->flag_mirror;
+                if (rows) { a.rr_split = n_split; a.rr_idx = rows->idx; a.rr_y = rows->logits; a.rr_S = rows->S; }
+            }
             else { a.y = dst.data; a.ycs = dst.has_cs ? dst.cs : nullptr; }
             a.ws = m->ws; a.ws_bytes = SPLITK_WS_BYTES;
             const double flops = 2.0 * batch * (double)l.n_in * l.n_out;
@@ -1117,7 +1135,8 @@ ct_status reexec_impl(ct_model *m, const float *input, int batch, const uint8_t 
 // max_batch.  idx_host as for reexec_rows.
 ct_status infer_with_reruns(ct_model *m, const float *input, int batch, float *logits, float *S, uint8_t *flag,
                             const float *prev_input, int prev_batch, const uint8_t *prev_flags_host,
-                            float *prev_logits, float *prev_S, int *n_rerun, int32_t *idx_host, cudaStream_t st) {
+                            float *prev_logits, float *prev_S, int *n_rerun, int32_t *idx_host, cudaStream_t st,
+                            const int32_t *idx_dev = nullptr) {
     if (n_rerun) *n_rerun = 0;
     int n = 0;
     for (int i = 0; i < prev_batch; ++i)
@@ -1140,6 +1159,13 @@ ct_status infer_with_reruns(ct_model *m, const float *input, int batch, float *l
         rr.n = n;
         for (int j = 0; j < n; ++j) rr.idx[j] = idx_host[j];
         return infer_impl(m, input, batch, logits, S, flag, st, nullptr, 0, &rr);
+    }
+    if (idx_dev) {
+        // the first layer reads the re-run images through the index list and
+        // the final FC writes their rows to the earlier batch's outputs: no
+        // gather, copy or scatter around the inference
+        const RerunRows rows{idx_dev, prev_logits, prev_S};
+        return infer_impl(m, input, batch + n, logits, S, flag, st, prev_input, batch, nullptr, &rows);
     }
     CUDA_TRY(cudaMemcpyAsync(m->re_idx, idx_host, sizeof(int32_t) * n, cudaMemcpyHostToDevice, st));
     const int64_t per = (int64_t)m->in_c * m->in_h * m->in_w;
@@ -1166,7 +1192,7 @@ ct_status infer_reexec_impl(ct_model *m, const float *input, int batch, float *l
     ct_status s = read_flags(m, prev_flag, prev_batch, st);
     if (s != CT_OK) return s;
     return infer_with_reruns(m, input, batch, logits, S, flag, prev_input, prev_batch, m->h_flags, prev_logits, prev_S,
-                             n_rerun, m->h_idx, st);
+                             n_rerun, m->h_idx, st, m->h_idx_d);
 }
 
 // Re-execution of the flagged images of nb <= 2 batches (host flags) as one
@@ -1252,7 +1278,9 @@ ct_status pipe_setup(ct_model *m, bool host) {
         const size_t B = (size_t)m->max_batch;
         if (cudaHostAlloc((void **)&m->pipe_flags_h, ct_model::PIPE * B, cudaHostAllocMapped) != cudaSuccess ||
             cudaHostGetDevicePointer((void **)&m->pipe_flags_d, m->pipe_flags_h, 0) != cudaSuccess ||
-            cudaMallocHost((void **)&m->pipe_idx_h, sizeof(int32_t) * (ct_model::PIPE + 2) * B) != cudaSuccess) {
+            cudaHostAlloc((void **)&m->pipe_idx_h, sizeof(int32_t) * (ct_model::PIPE + 2) * B, cudaHostAllocMapped) !=
+                cudaSuccess ||
+            cudaHostGetDevicePointer((void **)&m->pipe_idx_d, m->pipe_idx_h, 0) != cudaSuccess) {
             cudaGetLastError();
             return CT_ENOMEM;
         }
@@ -1334,7 +1362,7 @@ ct_status run_batches(ct_model *m, int n, int batch, const BatchIO &io, bool hos
             CUDA_TRY(cudaEventSynchronize(m->pipe_ev_flags[q]));
             r = infer_with_reruns(m, dev_in(i), batch, dev_lg(i), dev_S(i), dev_fl(i), dev_in(i - 2), batch,
                                   m->pipe_flags_h + (size_t)q * B, dev_lg(i - 2), dev_S(i - 2), &nr,
-                                  m->pipe_idx_h + (size_t)s * B, st);
+                                  m->pipe_idx_h + (size_t)s * B, st, m->pipe_idx_d + (size_t)s * B);
         } else {
             r = infer_impl(m, dev_in(i), batch, dev_lg(i), dev_S(i), dev_fl(i), st);
         }

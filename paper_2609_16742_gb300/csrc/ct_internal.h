@@ -45,6 +45,8 @@ struct ConvArgs {
     size_t ws_bytes;
     const void *x2;       // first layer only: images n >= n_split are image n - n_split of x2
     int n_split;          // (null x2: every image comes from x)
+    const int32_t *x2_idx;  // non-null: image n >= n_split is image x2_idx[n - n_split] of x2
+                            // (device-visible: mapped host memory)
 };
 
 // Batched campaign on a LeNet-shaped FP32 network (campaign_small.cu):
@@ -112,6 +114,14 @@ struct FcArgs {
     double ref, tau;
     float *ws;            // split-K workspace (null: never split)
     size_t ws_bytes;
+    // final layer with re-run rows: rows b >= rr_split are re-executed images
+    // of an earlier batch; their logits and S go to row rr_idx[b - rr_split]
+    // of rr_y / rr_S (rr_S may be null) and their flags are not written
+    // (rr_idx null: every row is a row of this batch)
+    int rr_split;
+    const int32_t *rr_idx;
+    float *rr_y;
+    float *rr_S;
 };
 
 struct PoolArgs {
@@ -184,8 +194,9 @@ cudaError_t launch_splitk_reduce(const ConvArgs &a, int splits, int ws_ld, bool 
 cudaError_t launch_fc(const FcArgs &a, bool half, bool x_float, cudaStream_t st, int *n_kernels);
 cudaError_t launch_maxpool(const PoolArgs &a, bool half, cudaStream_t st);
 cudaError_t launch_gap(const PoolArgs &a, bool half, cudaStream_t st);
+// idx non-null: row n of out is image idx[n] of in (device-visible idx)
 cudaError_t launch_convert_input(const float *in, void *out, int N, int C, int Cp, int H, int W, bool half,
-                                 cudaStream_t st);
+                                 cudaStream_t st, const int32_t *idx = nullptr);
 cudaError_t launch_xor_bit(void *base, int64_t word, int bit, int word_bytes, cudaStream_t st);
 cudaError_t launch_gather_images(const float *in, float *out, const int32_t *idx, int n,
                                  int64_t per_image, cudaStream_t st);

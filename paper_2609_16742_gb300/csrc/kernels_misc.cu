@@ -25,6 +25,25 @@ __device__ __forceinline__ float relu_keep_nan(float v) { return v < 0.f ? 0.f :
 // FMAs and one staged weight value is a broadcast.
 // ---------------------------------------------------------------------------
 constexpr int FC_J = 16, FC_IMG = 64, FC_KC = 64, FC_WARPS = 8;
+
+// Row b of a layer's output: a row of this batch, or (final layer with
+// re-run rows) the re-executed image's row of the earlier batch's logits
+template <typename TY>
+__device__ __forceinline__ TY *fc_out_row(const FcArgs &a, int b) {
+    if (a.rr_idx && b >= a.rr_split) return reinterpret_cast<TY *>(a.rr_y) + (size_t)a.rr_idx[b - a.rr_split] * a.n_out;
+    return static_cast<TY *>(a.y) + (size_t)b * a.n_out;
+}
+// S and verdict of image row b of the final layer; a re-run row writes its
+// S to the earlier batch and no flag (Sec. II-B: the re-run's flag is ignored)
+__device__ __forceinline__ void fc_final_out(const FcArgs &a, int b, float s, uint8_t fv) {
+    if (a.rr_idx && b >= a.rr_split) {
+        if (a.rr_S) a.rr_S[a.rr_idx[b - a.rr_split]] = s;
+        return;
+    }
+    if (a.S) a.S[b] = s;
+    if (a.flag) a.flag[b] = fv;
+    if (a.flag2) a.flag2[b] = fv;
+}
 static_assert((FC_KC * (FC_IMG + 1)) % 4 == 0, "weight tile must start 16-byte aligned (float4 reads)");
 
 template <typename TX, typename TW, typename TY>
@@ -150,16 +169,14 @@ __global__ void __launch_bounds__(256, 2) fc_kernel(FcArgs a) {
         for (int wv = 0; wv < FC_WARPS; ++wv) s += red[(wv * (FC_J + 1) + jj) * FC_IMG + bb];
         s += a.bias[j];
         if (a.relu) s = relu_keep_nan(s);
-        static_cast<TY *>(a.y)[(size_t)b * a.n_out + j] = from_f<TY>(s);
+        fc_out_row<TY>(a, b)[j] = from_f<TY>(s);
     }
     if (!ct_block) {
         if (a.final_layer && blockIdx.x == 0 && !a.protect) {
             for (int bb = tid; bb < FC_IMG; bb += 256) {
                 int b = b0 + bb;
                 if (b >= a.B) continue;
-                if (a.S) a.S[b] = __int_as_float(0x7fc00000);
-                if (a.flag) a.flag[b] = 0;
-                if (a.flag2) a.flag2[b] = 0;
+                fc_final_out(a, b, __int_as_float(0x7fc00000), 0);
             }
         }
         return;
@@ -174,10 +191,7 @@ __global__ void __launch_bounds__(256, 2) fc_kernel(FcArgs a) {
             for (int i = 0; i < a.n_cs; ++i) s += to_f(xcs[(size_t)b * a.n_cs + i]);
         s *= a.coef;
         if (a.final_layer) {
-            if (a.S) a.S[b] = s;
-            const uint8_t fv = !(fabs((double)s - a.ref) <= a.tau);
-            if (a.flag) a.flag[b] = fv;
-            if (a.flag2) a.flag2[b] = fv;
+            fc_final_out(a, b, s, !(fabs((double)s - a.ref) <= a.tau));
         } else {
             if (a.relu) s = relu_keep_nan(s);
             static_cast<TY *>(a.ycs)[b] = from_f<TY>(s);
@@ -205,15 +219,11 @@ __global__ void fc_reduce_kernel(FcArgs a, int splits) {
             for (int z = 0; z < splits; ++z) s += a.ws[z * plane + (size_t)b * ldw + j];
             s += a.bias[j];
             if (a.relu) s = relu_keep_nan(s);
-            static_cast<TY *>(a.y)[(size_t)b * a.n_out + j] = from_f<TY>(s);
+            fc_out_row<TY>(a, b)[j] = from_f<TY>(s);
             continue;
         }
         if (!a.protect) {
-            if (a.final_layer) {
-                if (a.S) a.S[b] = __int_as_float(0x7fc00000);
-                if (a.flag) a.flag[b] = 0;
-                if (a.flag2) a.flag2[b] = 0;
-            }
+            if (a.final_layer) fc_final_out(a, b, __int_as_float(0x7fc00000), 0);
             continue;
         }
         float s = 0.f;
@@ -223,10 +233,7 @@ __global__ void fc_reduce_kernel(FcArgs a, int splits) {
             for (int i = 0; i < a.n_cs; ++i) s += to_f(xcs[(size_t)b * a.n_cs + i]);
         s *= a.coef;
         if (a.final_layer) {
-            if (a.S) a.S[b] = s;
-            const uint8_t fv = !(fabs((double)s - a.ref) <= a.tau);
-            if (a.flag) a.flag[b] = fv;
-            if (a.flag2) a.flag2[b] = fv;
+            fc_final_out(a, b, s, !(fabs((double)s - a.ref) <= a.tau));
         } else {
             if (a.relu) s = relu_keep_nan(s);
             static_cast<TY *>(a.ycs)[b] = from_f<TY>(s);
@@ -355,14 +362,14 @@ __global__ void gap_kernel(PoolArgs a) {
 // NCHW fp32 -> NHWC storage type, one thread per pixel; channels C..Cp-1
 // of the output (padding to Cp channels) are written as zeros.
 template <typename T>
-__global__ void convert_input_kernel(const float *in, T *out, int N, int C, int Cp, int H, int W) {
+__global__ void convert_input_kernel(const float *in, T *out, int N, int C, int Cp, int H, int W, const int32_t *idx) {
     pdl_wait();
     pdl_trigger();
     const int HW = H * W;
     const int total = N * HW;
     for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < total; e += gridDim.x * blockDim.x) {
         const int n = e / HW, hw = e % HW;
-        const float *src = in + (size_t)n * C * HW + hw;
+        const float *src = in + (size_t)(idx ? idx[n] : n) * C * HW + hw;
         T *dst = out + (size_t)e * Cp;
         for (int c = 0; c < Cp; ++c) dst[c] = from_f<T>(c < C ? src[(size_t)c * HW] : 0.f);
     }
@@ -469,10 +476,10 @@ cudaError_t launch_gap(const PoolArgs &a, bool half, cudaStream_t st) {
 }
 
 cudaError_t launch_convert_input(const float *in, void *out, int N, int C, int Cp, int H, int W, bool half,
-                                 cudaStream_t st) {
+                                 cudaStream_t st, const int32_t *idx) {
     const int64_t n = (int64_t)N * H * W;
-    if (half) pdl_launch(convert_input_kernel<__half>, grid_for(n, 256), 256, 0, st, in, (__half *)out, N, C, Cp, H, W);
-    else pdl_launch(convert_input_kernel<float>, grid_for(n, 256), 256, 0, st, in, (float *)out, N, C, Cp, H, W);
+    if (half) pdl_launch(convert_input_kernel<__half>, grid_for(n, 256), 256, 0, st, in, (__half *)out, N, C, Cp, H, W, idx);
+    else pdl_launch(convert_input_kernel<float>, grid_for(n, 256), 256, 0, st, in, (float *)out, N, C, Cp, H, W, idx);
     return cudaGetLastError();
 }
 
