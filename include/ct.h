@@ -107,7 +107,8 @@ typedef struct {
 /* flags for ct_build_opts.flags */
 #define CT_FLAG_SIMT_ONLY 1u      /* use the CUDA-core conv kernels everywhere */
 #define CT_FLAG_LAYERWISE 2u      /* one kernel per layer even where the whole network
-                                     fits one kernel (the LeNet-5 shape, FP32) */
+                                     fits one kernel (the LeNet-5 shape, FP32) or a
+                                     shortcut could share its block's first launch */
 
 /* ct_build_opts.protect: how the scheme of Sec. II-A is built in.
  *   CT_PROTECT_NONE     the network as described (the unprotected baseline);
@@ -180,6 +181,11 @@ ct_status ct_resolve_roles(const ct_model_desc *desc, int32_t *roles);
  * memory; an armed fault is applied inside it (its intermediate tensors are
  * then not stored, and a fault in the image is rejected with CT_ERANGE).
  * CT_FLAG_LAYERWISE keeps one kernel per layer.
+ * With FP16 storage, a 1x1 shortcut convolution listed right after its
+ * block's first convolution, reading the same tensor at the same stride
+ * (the shortcut's pixel is that convolution's centre tap), runs in the same
+ * launch on the tensor cores whenever both are whole N = 128 or N = 256
+ * tiles (unless CT_FLAG_LAYERWISE); its outputs are the same bits.
  * With FP16 storage, a stride-1 3x3 convolution followed by a 2x2 stride-2
  * max-pool that is its only reader applies the pool in its epilogue (data
  * and checksum channels together) whenever it runs on halo tiles (batches

@@ -216,7 +216,8 @@ def ct_build(layers: Sequence, params: Sequence[dict], in_shape, n_classes: int,
 
     protect=True adds the carry-through filters as extra channels (widened);
     replace=True builds the paper's prune-and-replace construction instead;
-    layerwise=True keeps one kernel per layer for the LeNet-5 shape."""
+    layerwise=True keeps one kernel per layer: for the LeNet-5 shape, and for
+    1x1 shortcuts that would otherwise run in their block's first launch."""
     n = len(layers)
     arr = _layer_descs(layers)
     keep = []

@@ -50,7 +50,9 @@
 #include <cudaTypedefs.h>
 #include <string.h>
 
+#include <algorithm>
 #include <mutex>
+#include <vector>
 
 #include "ct_internal.h"
 #include "tc_common.cuh"
@@ -90,6 +92,11 @@ struct TcGeom {
     // 128-channel halves, units 0 .. units - t_first - 1 (unit 2 * (tile -
     // t_first) + half); whole tiles 0 .. t_first - 1 follow them
     int t_first, units;
+    // a 1x1 shortcut convolution run by the same launch (its items follow
+    // this layer's; see UnitSeq): its item count (0: none), and its split:
+    // CTAs (or pairs) 0 .. sc_s0 - 1 share items 0 .. sc_x - 1 evenly, the
+    // others the rest
+    int sc_items, sc_s0, sc_x;
     uint16_t coef_h;
 };
 
@@ -109,6 +116,42 @@ __device__ __forceinline__ TileRef tile_ref(int item, const TcGeom &g) {
     return t;
 }
 
+
+// Work units of one CTA (or CTA pair) cid of ncl: first this layer's n1
+// units, round-robin (cid, cid + ncl, ...), then a contiguous share of the
+// shortcut's items: CTAs 0 .. sc_s0 - 1 split items 0 .. sc_x - 1 evenly and
+// the others split the rest, so that the host can give more of them to the
+// CTAs with fewer units of this layer.
+// The shortcut is a 1x1 convolution of the same input at the same stride,
+// whose pixel is this layer's centre tap: its A operand is this layer's
+// centre-tap K blocks (same tensor map and coordinates); its weights,
+// epilogue arguments and geometry are its own.  Its units are numbered
+// n1 + item.
+struct UnitSeq {
+    int n1, k1, lo, cnt;
+};
+template <bool SC>
+__device__ __forceinline__ UnitSeq unit_seq(int cid, int ncl, int n1, const TcGeom &g) {
+    UnitSeq s;
+    s.n1 = n1;
+    s.k1 = cid < n1 ? (n1 - 1 - cid) / ncl + 1 : 0;
+    s.lo = 0;
+    s.cnt = 0;
+    if (SC && g.sc_items > 0) {
+        if (cid < g.sc_s0) {
+            s.lo = (int)(((long long)cid * g.sc_x) / g.sc_s0);
+            s.cnt = (int)(((long long)(cid + 1) * g.sc_x) / g.sc_s0) - s.lo;
+        } else {
+            const int nc = ncl - g.sc_s0, c = cid - g.sc_s0, rest = g.sc_items - g.sc_x;
+            s.lo = g.sc_x + (int)(((long long)c * rest) / nc);
+            s.cnt = g.sc_x + (int)(((long long)(c + 1) * rest) / nc) - s.lo;
+        }
+    }
+    return s;
+}
+__device__ __forceinline__ int unit_at(const UnitSeq &s, int k, int cid, int ncl) {
+    return k < s.k1 ? cid + k * ncl : s.n1 + s.lo + (k - s.k1);
+}
 
 // tap visited at K-block kb: the centre tap first, the others in order
 __device__ __forceinline__ int tap_of(int t, int ctr) { return t == 0 ? ctr : (t <= ctr ? t - 1 : t); }
@@ -247,6 +290,20 @@ __device__ __forceinline__ bool stage_bias(float *bias_s, const float *bias_g, i
     }
     return in_smem;
 }
+// stage_bias for a launch that also runs a shortcut convolution: the
+// shortcut's bias follows this layer's (bias_s[K .. 2K)).
+__device__ __forceinline__ bool stage_bias2(float *bias_s, const float *b1, const float *b2, int K, int t,
+                                            int nthreads) {
+    const bool in_smem = b1 != nullptr && b2 != nullptr && 2 * K <= BIAS_SMEM;
+    if (in_smem) {
+        for (int i = t; i < K; i += nthreads) {
+            bias_s[i] = __ldg(b1 + i);
+            bias_s[K + i] = __ldg(b2 + i);
+        }
+        asm volatile("bar.sync 1, %0;" ::"r"(nthreads) : "memory");
+    }
+    return in_smem;
+}
 __device__ __forceinline__ uint32_t cvt_h2(float lo, float hi, bool relu) {
     uint32_t r;
     if (relu) asm("cvt.rn.relu.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
@@ -319,31 +376,38 @@ __device__ __forceinline__ float pool2x2_lanes(float v) {
 // incoming checksum at the centre pixel (or the sum of an FC layer's
 // checksum features) and the residual checksum.  Loaded before the
 // accumulator is ready so that their latency overlaps the MMAs.
+// The centre-pixel and residual checksums are kept as FP16 bits and
+// converted where they are used, so that their loads stay in flight while
+// the epilogue waits for the accumulator (a conversion right after the load
+// would stall the warp on it).
 struct CsIn {
-    float cin, rcs;
+    float cin_sum;                 // FC layer: the sum of its incoming checksum features
+    unsigned short cin_h, rcs_h;   // FP16 bits of the incoming and residual checksums (0: +0)
 };
+__device__ __forceinline__ float h2f_bits(unsigned short b) { return __half2float(__ushort_as_half(b)); }
 __device__ __forceinline__ CsIn load_cs_inputs(const ConvArgs &a, const TcGeom &g, int m, int nimg, int p, int q) {
-    CsIn c{0.f, 0.f};
+    CsIn c{0.f, 0, 0};
     const __half *csi = static_cast<const __half *>(a.cs_in);
     const int ctr_r = g.ctr_tap / g.S, ctr_s = g.ctr_tap % g.S;
     const int hc = p * g.stride + ctr_r - g.pad, wc = q * g.stride + ctr_s - g.pad;
     const bool inb = hc >= 0 && hc < a.H && wc >= 0 && wc < a.W;
     if (csi && a.cs_rowsum > 0) {                  // FC layer: every incoming checksum feature
-        for (int i = 0; i < a.cs_rowsum; ++i) c.cin += ldh(csi, (size_t)m * a.cs_rowsum + i);
+        for (int i = 0; i < a.cs_rowsum; ++i) c.cin_sum += ldh(csi, (size_t)m * a.cs_rowsum + i);
     } else if (csi && inb) {
-        c.cin = ldh(csi, ((size_t)nimg * a.H + hc) * a.W + wc);
+        c.cin_h = __ldg(reinterpret_cast<const unsigned short *>(csi) + ((size_t)nimg * a.H + hc) * a.W + wc);
     }
-    if (a.res_cs) c.rcs = ldh(static_cast<const __half *>(a.res_cs), (size_t)m);
+    if (a.res_cs) c.rcs_h = __ldg(static_cast<const unsigned short *>(a.res_cs) + m);
     return c;
 }
 
 __device__ __forceinline__ float checksum_value(float ctv, const CsIn &c, const ConvArgs &a, const TcGeom &g,
                                                 float fsrc) {
+    const float cin = a.cs_rowsum > 0 ? c.cin_sum : h2f_bits(c.cin_h);
     float o = 0.f;
-    if (a.role == CT_ROLE_CT) o = ctv + a.coef * c.cin;
-    else if (a.role == CT_ROLE_PASS) o = c.cin;
+    if (a.role == CT_ROLE_CT) o = ctv + a.coef * cin;
+    else if (a.role == CT_ROLE_PASS) o = cin;
     if (a.fd.active && a.fd.kout == g.K) o += a.fd.dv * fsrc;
-    if (a.res_cs) o += c.rcs;
+    if (a.res_cs) o += h2f_bits(c.rcs_h);
     if (a.relu) o = relu_keep_nan(o);
     return o;
 }
@@ -361,10 +425,14 @@ __device__ __forceinline__ void store_checksum_pre(float ctv, const CsIn &c, con
 // barrier round trip).  A single TMEM buffer holds the chains; for
 // BN <= 128 the epilogue copies it to registers and releases it before its
 // global stores, so the next tile's MMAs overlap the stores.
-template <int BN, int STAGES, int SUB, int NCH>
+// SC: the launch also runs a 1x1 shortcut convolution (bmap2, a2, g2; see
+// UnitSeq); otherwise those arguments are unused.
+template <int BN, int STAGES, int SUB, int NCH, bool SC>
 __global__ void __launch_bounds__(tc_threads(BN, STAGES), 1)
 conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
-               const ConvArgs a, const TcGeom g) {
+               const __grid_constant__ ConvArgs a, const __grid_constant__ TcGeom g,
+               const __grid_constant__ CUtensorMap bmap2, const __grid_constant__ ConvArgs a2,
+               const __grid_constant__ TcGeom g2) {
     constexpr int B_ROWS = BN + 16;                       // 16 constant carry-through rows
     constexpr int B_SUB_BYTES = B_ROWS * BK * 2;
     constexpr int B_TMA_BYTES = BN * BK * 2;
@@ -376,6 +444,11 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
     // that do not issue copies (they consume every stage, like the MMA warp),
     // and the epilogue of one tile overlaps the MMAs of the next
     constexpr bool DBUF = !EARLY;
+    // accumulator buffers, 256 TMEM columns apart: two when both fit (N =
+    // 256; N <= 128 with one chain), so that a tile's MMAs never wait for
+    // the previous tile's epilogue to read TMEM
+    constexpr int NACC = (DBUF || 2 * NCH * CH <= 512) ? 2 : 1;
+    static_assert(NACC == 1 || DBUF || NCH * CH <= 256, "an accumulator buffer spans at most 256 columns");
     // producer warps (each owns whole ring slots) and carry-through warps
     constexpr int NPROD = tc_nprod(BN, STAGES);
     constexpr int NPG = tc_npg(BN, STAGES);               // producer group: producers + carry-through warps
@@ -385,6 +458,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
     static_assert(STAGES % NPROD == 0, "producer warps must own whole ring slots");
     static_assert(DBUF ? NCT > 0 : NCT == 0, "carry-through warps only beside double-buffered accumulators");
     static_assert(!DBUF || (NCT > 0 && BM % (16 * (NCT > 0 ? NCT : 1)) == 0), "carry-through warps split the tile rows");
+    static_assert(!SC || !DBUF, "a shortcut only beside single-buffered accumulators");
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint8_t *As = smem;                                   // [STAGES][SUB][A_BYTES]
@@ -402,7 +476,9 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int cid = blockIdx.x, ncl = gridDim.x;
-    const int num_items = g.m_tiles * g.n_tiles * g.splits;
+    const int n1 = g.m_tiles * g.n_tiles * g.splits;     // this layer's items
+    const UnitSeq us = unit_seq<SC>(cid, ncl, n1, g);
+    const int n_units = us.k1 + us.cnt;                 // this CTA's units
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -452,12 +528,17 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
         if (elect_one()) {
             asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&amap) : "memory");
             asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&bmap) : "memory");
+            if (SC) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&bmap2) : "memory");
         }
         __syncwarp();
         int it = 0;
-        for (int tile = cid; tile < num_items; tile += ncl) {
+        for (int k = 0; k < n_units; ++k) {
             if (__any_sync(0xffffffffu, *abort_flag)) break;
-            const TileRef tr = tile_ref(tile, g);
+            const int unit = unit_at(us, k, cid, ncl);
+            const bool sc = SC && unit >= n1;
+            // A coordinates: this layer's geometry (a shortcut reads its centre tap)
+            const TileRef tr = sc ? tile_ref(unit - n1, g2) : tile_ref(unit, g);
+            const CUtensorMap *bm = sc ? &bmap2 : &bmap;
             const int m0 = tr.m0, n_tile = tr.n_tile;
             const int nimg = m0 / g.PQ, rem = m0 % g.PQ;
             const int p = rem / g.Q, q = rem % g.Q;
@@ -479,7 +560,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
                         const int r = tap / g.S, sx = tap % g.S;
                         tma_load_im2col(smem_u32(As + (s * SUB + j) * A_BYTES), &amap, fb, c0, w0, h0, nimg,
                                         (uint16_t)sx, (uint16_t)r);
-                        tma_load_2d(smem_u32(Bs + (s * SUB + j) * B_SUB_BYTES), &bmap, fb, tap * g.C + c0,
+                        tma_load_2d(smem_u32(Bs + (s * SUB + j) * B_SUB_BYTES), bm, fb, (sc ? 0 : tap) * g.C + c0,
                                     n_tile * BN);
                     }
                 }
@@ -493,14 +574,17 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
         const uint32_t id_merged = idesc_f16(BM, BN + 16);
         const uint32_t id_ct = idesc_f16(BM, 16);
         const uint32_t ct_base = smem_u32(CTt);
-        int it = 0, lt = 0;
-        for (int tile = cid; tile < num_items; tile += ncl, ++lt) {
+        int it = 0;
+        for (int lt = 0; lt < n_units; ++lt) {
             if (__any_sync(0xffffffffu, *abort_flag)) break;
-            const TileRef tr = tile_ref(tile, g);
+            const int unit = unit_at(us, lt, cid, ncl);
+            const bool sc = SC && unit >= n1;
+            const TcGeom &G = sc ? g2 : g;
+            const TileRef tr = tile_ref(sc ? unit - n1 : unit, G);
             const int n_tile = tr.n_tile;
-            const bool ct_here = g.ct_mode != CT_NONE_ && n_tile == 0;
-            const int ab = DBUF ? (lt & 1) : 0;
-            const uint32_t aph = DBUF ? ((uint32_t)(lt >> 1) & 1u) : ((uint32_t)lt & 1u);
+            const bool ct_here = G.ct_mode != CT_NONE_ && n_tile == 0;
+            const int ab = NACC == 2 ? (lt & 1) : 0;
+            const uint32_t aph = NACC == 2 ? ((uint32_t)(lt >> 1) & 1u) : ((uint32_t)lt & 1u);
             if (!warp_wait(smem_u32(&acc_empty[ab]), aph ^ 1u, a.err, 8u)) {
                 if (lane == 0) *abort_flag = 1;
                 break;
@@ -519,12 +603,12 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
                     for (int j = 0; j < nsub; ++j) {
                         const int kb = kb0 + j;
                         const int kr = kb - tr.kb_lo;               // position within this split
-                        const uint32_t d = DBUF ? tmem + (uint32_t)(ab * BN) : tmem + (uint32_t)((kr % NCH) * CH);
-                        const bool centre = kb < g.cpb;
+                        const uint32_t d = tmem + (uint32_t)(ab * 256 + (kr % NCH) * CH);
+                        const bool centre = kb < G.cpb;
                         const uint64_t ad0 = smem_desc_sw128(smem_u32(As + (s * SUB + j) * A_BYTES));
                         const uint64_t bd0 = smem_desc_sw128(smem_u32(Bs + (s * SUB + j) * B_SUB_BYTES));
                         const uint32_t acc0 = kr >= NCH ? 1u : 0u;  // first use of the chain
-                        if (!DBUF && ct_here && centre && g.ct_mode == CT_SEPARATE) {
+                        if (!DBUF && ct_here && centre && G.ct_mode == CT_SEPARATE) {
                             const uint64_t cd0 = smem_desc_sw128(ct_base);
 #pragma unroll
                             for (int k16 = 0; k16 < BK / 16; ++k16) {
@@ -532,7 +616,7 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
                                 umma_f16(d + BN, ad0 + 2 * k16, cd0 + 2 * k16, id_ct, k16 ? 1u : acc0);
                             }
                         } else {
-                            const uint32_t idm = (!DBUF && ct_here && centre && g.ct_mode == CT_MERGED) ? id_merged : id_main;
+                            const uint32_t idm = (!DBUF && ct_here && centre && G.ct_mode == CT_MERGED) ? id_merged : id_main;
 #pragma unroll
                             for (int k16 = 0; k16 < BK / 16; ++k16)
                                 umma_f16(d, ad0 + 2 * k16, bd0 + 2 * k16, idm, k16 ? 1u : acc0);
@@ -564,11 +648,11 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
             const int w = warp - NPROD;
             // ldmatrix row address of this lane: matrix lane / 8 = (rows +8, chunk +1) bits
             const int lm_row = (lane & 7) + ((lane >> 3) & 1) * 8, lm_chk = lane >> 4;
-            int it = 0, lt = 0;
+            int it = 0;
             bool ok = true;
-            for (int tile = cid; tile < num_items && ok; tile += ncl, ++lt) {
+            for (int lt = 0; lt < n_units && ok; ++lt) {
                 if (__any_sync(0xffffffffu, *abort_flag)) break;
-                const TileRef tr = tile_ref(tile, g);
+                const TileRef tr = tile_ref(unit_at(us, lt, cid, ncl), g);
                 const bool ct_here = g.ct_mode != CT_NONE_ && tr.n_tile == 0;
                 const int ab = lt & 1;
                 float acc[MT][4];
@@ -623,14 +707,20 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
         const int quad = warp & 3;                 // TMEM lanes this warp may read
         const int half = ep >> 2;                  // which half of the tile's channels
         const int row = quad * 32 + lane;
-        const __half *x = static_cast<const __half *>(a.x);
-        const FaultDelta fd = a.fd;
-        const bool split = g.splits > 1;
-        const bool has_res = a.res != nullptr, relu = a.relu != 0;
-        const bool bias_sm = stage_bias(bias_s, a.bias, g.K, threadIdx.x - 32 * TC_EPI_WARP0, 32 * N_EPI_WARPS);
-        int lt = 0;
-        for (int tile = cid; tile < num_items; tile += ncl, ++lt) {
-            const TileRef tr = tile_ref(tile, g);
+        const int et = threadIdx.x - 32 * TC_EPI_WARP0;
+        const bool bias_sm = SC ? stage_bias2(bias_s, a.bias, a2.bias, g.K, et, 32 * N_EPI_WARPS)
+                                : stage_bias(bias_s, a.bias, g.K, et, 32 * N_EPI_WARPS);
+        for (int lt = 0; lt < n_units; ++lt) {
+            const int unit = unit_at(us, lt, cid, ncl);
+            const bool sc = SC && unit >= n1;
+            const ConvArgs &A = sc ? a2 : a;       // this unit's layer
+            const TcGeom &G = sc ? g2 : g;
+            const float *bias_l = bias_s + (sc ? G.K : 0);
+            const __half *x = static_cast<const __half *>(A.x);
+            const FaultDelta fd = A.fd;
+            const bool split = G.splits > 1;
+            const bool has_res = A.res != nullptr, relu = A.relu != 0;
+            const TileRef tr = tile_ref(sc ? unit - n1 : unit, G);
             const int m0 = tr.m0, n_tile = tr.n_tile;
             // residual loads in flight while the MMAs run
             Res16 rs[BN / 32];
@@ -638,80 +728,104 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
                 const int mp = m0 + row;
 #pragma unroll
                 for (int c = 0; c < BN / 32; ++c)
-                    rs[c] = (mp < g.M && g.splits == 1)
-                                ? load_res16(a, g.K, (size_t)mp, n_tile * BN + half * (BN / 2) + 16 * c)
+                    rs[c] = (mp < G.M && G.splits == 1)
+                                ? load_res16(A, G.K, (size_t)mp, n_tile * BN + half * (BN / 2) + 16 * c)
                                 : Res16{make_uint4(0u, 0u, 0u, 0u), make_uint4(0u, 0u, 0u, 0u)};
             }
-            CsIn csv{0.f, 0.f};
+            CsIn csv{0.f, 0, 0};
             {
                 const int mp = m0 + row;
-                if (half == 0 && a.cs_out != nullptr && n_tile == 0 && mp < g.M && g.splits == 1) {
-                    const int ni = mp / g.PQ, rm = mp % g.PQ;
-                    csv = load_cs_inputs(a, g, mp, ni, rm / g.Q, rm % g.Q);
+                if (half == 0 && A.cs_out != nullptr && n_tile == 0 && mp < G.M && G.splits == 1) {
+                    const int ni = mp / G.PQ, rm = mp % G.PQ;
+                    csv = load_cs_inputs(A, G, mp, ni, rm / G.Q, rm % G.Q);
                 }
             }
             const int chains = min(NCH, tr.kb_hi - tr.kb_lo);                    // chains that received MMAs
             // chains whose first K block is a centre block hold a carry-through column
-            const int ct_chains = max(0, min(NCH, min(g.cpb, tr.kb_hi) - tr.kb_lo));
-            const int ab = DBUF ? (lt & 1) : 0;
-            const uint32_t aph = DBUF ? ((uint32_t)(lt >> 1) & 1u) : ((uint32_t)lt & 1u);
-            bool ok = mbar_wait(smem_u32(&acc_full[ab]), aph, a.err, 4u) && !*abort_flag;
-            if (DBUF) ok = ok && mbar_wait(smem_u32(&ct_ready[ab]), aph, a.err, 4u);
+            const int ct_chains = max(0, min(NCH, min(G.cpb, tr.kb_hi) - tr.kb_lo));
+            const int ab = NACC == 2 ? (lt & 1) : 0;
+            const uint32_t aph = NACC == 2 ? ((uint32_t)(lt >> 1) & 1u) : ((uint32_t)lt & 1u);
+            bool ok = mbar_wait(smem_u32(&acc_full[ab]), aph, A.err, 4u) && !*abort_flag;
+            if (DBUF) ok = ok && mbar_wait(smem_u32(&ct_ready[ab]), aph, A.err, 4u);
             ok = __all_sync(0xffffffffu, ok);      // tcgen05.ld below is warp-collective
             if (!ok) break;
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-            const uint32_t trow = tmem + (uint32_t)(ab * BN) + ((uint32_t)(quad * 32) << 16);
+            const uint32_t trow = tmem + (uint32_t)(ab * 256) + ((uint32_t)(quad * 32) << 16);
             const int m = m0 + row;
-            const bool valid = m < g.M;
+            const bool valid = m < G.M;
             const int mm = valid ? m : 0;
-            const int nimg = mm / g.PQ, rem = mm % g.PQ, p = rem / g.Q, q = rem % g.Q;
+            const int nimg = mm / G.PQ, rem = mm % G.PQ, p = rem / G.Q, q = rem % G.Q;
             float fsrc = 0.f;
             if (fd.active && !split) {
-                const int h = p * g.stride + fd.r - g.pad, w = q * g.stride + fd.s - g.pad;
-                if (h >= 0 && h < a.H && w >= 0 && w < a.W) {
-                    if (fd.cin < g.C) fsrc = ldh(x, (((size_t)nimg * a.H + h) * a.W + w) * g.C + fd.cin);
-                    else if (a.cs_in) fsrc = ldh(static_cast<const __half *>(a.cs_in), ((size_t)nimg * a.H + h) * a.W + w);
+                const int h = p * G.stride + fd.r - G.pad, w = q * G.stride + fd.s - G.pad;
+                if (h >= 0 && h < A.H && w >= 0 && w < A.W) {
+                    if (fd.cin < G.C) fsrc = ldh(x, (((size_t)nimg * A.H + h) * A.W + w) * G.C + fd.cin);
+                    else if (A.cs_in) fsrc = ldh(static_cast<const __half *>(A.cs_in), ((size_t)nimg * A.H + h) * A.W + w);
                 }
             }
             const int n0 = n_tile * BN;
-            const bool do_cs = half == 0 && a.cs_out != nullptr && n_tile == 0;
+            const bool do_cs = half == 0 && A.cs_out != nullptr && n_tile == 0;
             float ctv = 0.f;
             if (EARLY) {
+                // TMEM reads in few round trips: chain 0 (all of this warp's
+                // columns) with the carry-through columns, then the other
+                // chains two chunks at a time; the sums keep the order
+                // ((chain 0 + chain 1) + chain 2) + ...
                 float vals[BN / 2];
+                const bool ld_ct = do_cs && G.ct_mode != CT_NONE_;
+                uint32_t ctr[NCH];
+                {
+                    uint32_t tv[BN / 32][16];
 #pragma unroll
-                for (int c = 0; c < BN / 2; c += 16) {
-                    tmem_ld16(trow + half * (BN / 2) + c, vals + c);
-                    for (int ch = 1; ch < chains; ++ch) {
+                    for (int c = 0; c < BN / 2; c += 16) tmem_ld16_nw(trow + half * (BN / 2) + c, tv[c / 16]);
+#pragma unroll
+                    for (int ch = 0; ch < NCH; ++ch)
+                        if (ld_ct && ch < ct_chains) tmem_ld1_nw(trow + ch * CH + BN, ctr[ch]);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int c = 0; c < BN / 2; c += 16) tmem_done16(tv[c / 16], vals + c);
+                }
+                for (int ch = 1; ch < chains; ++ch) {
+#pragma unroll
+                    for (int c = 0; c < BN / 2; c += 32) {
+                        uint32_t t2[2][16];
+                        tmem_ld16_nw(trow + ch * CH + half * (BN / 2) + c, t2[0]);
+                        tmem_ld16_nw(trow + ch * CH + half * (BN / 2) + c + 16, t2[1]);
+                        tmem_wait_ld();
                         float t[16];
-                        tmem_ld16(trow + ch * CH + half * (BN / 2) + c, t);
+                        tmem_done16(t2[0], t);
 #pragma unroll
                         for (int i = 0; i < 16; ++i) vals[c + i] += t[i];
+                        tmem_done16(t2[1], t);
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) vals[c + 16 + i] += t[i];
                     }
                 }
-                if (do_cs && g.ct_mode != CT_NONE_)
-                    for (int ch = 0; ch < ct_chains; ++ch) ctv += tmem_ld1(trow + ch * CH + BN);
+#pragma unroll
+                for (int ch = 0; ch < NCH; ++ch)
+                    if (ld_ct && ch < ct_chains) ctv += tmem_done(ctr[ch]);
                 asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
                 __syncwarp();
-                if (lane == 0) mbar_arrive(smem_u32(&acc_empty[0]));   // accumulators free for the next tile
+                if (lane == 0) mbar_arrive(smem_u32(&acc_empty[ab]));   // accumulators free for a later tile
                 if (valid && split) {
-                    float *wrow = a.ws + ((size_t)tr.sp * g.M + m) * g.ws_ld;
+                    float *wrow = A.ws + ((size_t)tr.sp * G.M + m) * G.ws_ld;
 #pragma unroll
                     for (int c = 0; c < BN / 2; c += 4)
                         *reinterpret_cast<float4 *>(wrow + n0 + half * (BN / 2) + c) =
                             make_float4(vals[c], vals[c + 1], vals[c + 2], vals[c + 3]);
-                    if (do_cs) wrow[g.K] = ctv;
+                    if (do_cs) wrow[G.K] = ctv;
                 } else if (valid && fd.active) {
 #pragma unroll
                     for (int c = 0; c < BN / 2; c += 16)
-                        store_chunk_pre(vals + c, rs[c / 16], a, g.K, (size_t)m, n0 + half * (BN / 2) + c, fsrc);
-                    if (do_cs) store_checksum_pre(ctv, csv, a, g, m, fsrc);
+                        store_chunk_pre(vals + c, rs[c / 16], A, G.K, (size_t)m, n0 + half * (BN / 2) + c, fsrc);
+                    if (do_cs) store_checksum_pre(ctv, csv, A, G, m, fsrc);
                 } else if (valid) {
-                    __half *yrow = static_cast<__half *>(a.y) + (size_t)m * g.K + n0 + half * (BN / 2);
+                    __half *yrow = static_cast<__half *>(A.y) + (size_t)m * G.K + n0 + half * (BN / 2);
 #pragma unroll
                     for (int c = 0; c < BN / 2; c += 16)
-                        store16_fast(vals + c, bias16_at(bias_s, a.bias, bias_sm, n0 + half * (BN / 2) + c), rs[c / 16], has_res,
+                        store16_fast(vals + c, bias16_at(bias_l, A.bias, bias_sm, n0 + half * (BN / 2) + c), rs[c / 16], has_res,
                                      relu, yrow + c);
-                    if (do_cs) store_checksum_pre(ctv, csv, a, g, m, 0.f);
+                    if (do_cs) store_checksum_pre(ctv, csv, A, G, m, 0.f);
                 }
             } else {
 #pragma unroll
@@ -725,19 +839,19 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
                         for (int i = 0; i < 16; ++i) v[i] += t[i];
                     }
                     if (valid && split) {
-                        float4 *wp = reinterpret_cast<float4 *>(a.ws + ((size_t)tr.sp * g.M + m) * g.ws_ld + n0 + c);
+                        float4 *wp = reinterpret_cast<float4 *>(A.ws + ((size_t)tr.sp * G.M + m) * G.ws_ld + n0 + c);
 #pragma unroll
                         for (int i = 0; i < 4; ++i) wp[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
                     } else if (valid && fd.active) {
-                        store_chunk_pre(v, rs[(c - half * (BN / 2)) / 16], a, g.K, (size_t)m, n0 + c, fsrc);
+                        store_chunk_pre(v, rs[(c - half * (BN / 2)) / 16], A, G.K, (size_t)m, n0 + c, fsrc);
                     } else if (valid) {
-                        store16_fast(v, bias16_at(bias_s, a.bias, bias_sm, n0 + c), rs[(c - half * (BN / 2)) / 16], has_res,
-                                     relu, static_cast<__half *>(a.y) + (size_t)m * g.K + n0 + c);
+                        store16_fast(v, bias16_at(bias_l, A.bias, bias_sm, n0 + c), rs[(c - half * (BN / 2)) / 16], has_res,
+                                     relu, static_cast<__half *>(A.y) + (size_t)m * G.K + n0 + c);
                     }
                 }
-                if (do_cs && g.ct_mode != CT_NONE_) ctv = ct_sum[ab * BM + row];
-                if (do_cs && valid && split) a.ws[((size_t)tr.sp * g.M + m) * g.ws_ld + g.K] = ctv;
-                else if (do_cs && valid) store_checksum_pre(ctv, csv, a, g, m, fsrc);
+                if (do_cs && G.ct_mode != CT_NONE_) ctv = ct_sum[ab * BM + row];
+                if (do_cs && valid && split) A.ws[((size_t)tr.sp * G.M + m) * G.ws_ld + G.K] = ctv;
+                else if (do_cs && valid) store_checksum_pre(ctv, csv, A, G, m, fsrc);
                 asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
                 __syncwarp();
                 if (lane == 0) mbar_arrive(smem_u32(&acc_empty[ab]));
@@ -805,14 +919,26 @@ __device__ __forceinline__ PairUnit pair_unit(int u, const TcGeom &g) {
     return PairUnit{it, (it % g.n_tiles) * 256 + (u & 1) * 128, true};
 }
 
+// unit u of a pair kernel that may also run a shortcut (units n1 ..: its
+// whole tiles)
+template <bool VARN, bool SC>
+__device__ __forceinline__ PairUnit pair_unit_sc(int u, int n1, const TcGeom &g, const TcGeom &g2) {
+    if (SC && u >= n1) return PairUnit{u - n1, ((u - n1) % g2.n_tiles) * 256, false};
+    return pair_unit<VARN>(u, g);
+}
+
 size_t pair_smem_bytes() {
     return 1024 + (size_t)PR_STAGES * (A_BYTES + PR_BH_BYTES) + 8 * PR_NBAR + 16 + 16 + 4 * BIAS_SMEM;
 }
 
-template <bool VARN>
+// SC: the launch also runs a 1x1 shortcut convolution as whole tiles after
+// this layer's units (bmap2: its 128-row weight halves; a2, g2; see UnitSeq).
+template <bool VARN, bool SC>
 __global__ void __launch_bounds__(PR_THREADS, 1)
 conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
-                    const __grid_constant__ CUtensorMap bmap64, const ConvArgs a, const TcGeom g) {
+                    const __grid_constant__ CUtensorMap bmap64, const __grid_constant__ ConvArgs a,
+                    const __grid_constant__ TcGeom g, const __grid_constant__ CUtensorMap bmap2,
+                    const __grid_constant__ ConvArgs a2, const __grid_constant__ TcGeom g2) {
     constexpr int BN = 256;
     static_assert(PR_STAGES % PR_NPROD == 0, "producer warps must own whole ring slots");
     extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -832,7 +958,9 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
     const uint32_t crank = cluster_ctarank();
     const bool leader = crank == 0;
     const int cid = blockIdx.x >> 1, ncl = gridDim.x >> 1;
-    const int num_units = VARN ? g.units : ((g.m_tiles + 1) >> 1) * g.n_tiles;
+    const int n1 = VARN ? g.units : ((g.m_tiles + 1) >> 1) * g.n_tiles;    // this layer's units
+    const UnitSeq us = unit_seq<SC>(cid, ncl, n1, g);
+    const int n_units = us.k1 + us.cnt;                                     // this pair's units
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < PR_STAGES; ++s) {
@@ -868,21 +996,26 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
             asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&amap) : "memory");
             asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&bmap) : "memory");
             if (VARN) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&bmap64) : "memory");
+            if (SC) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&bmap2) : "memory");
         }
         __syncwarp();
         const uint32_t full_even = mapa_shared(smem_u32(full), 0u);
         int it = 0;
         bool ok = true;
-        for (int u = cid; u < num_units && ok; u += ncl) {
+        for (int k = 0; k < n_units && ok; ++k) {
             if (__any_sync(0xffffffffu, *abort_flag)) break;
-            const PairUnit pu = pair_unit<VARN>(u, g);
+            const int u = unit_at(us, k, cid, ncl);
+            const bool sc = SC && u >= n1;
+            const PairUnit pu = pair_unit_sc<VARN, SC>(u, n1, g, g2);
+            const int n_kb = sc ? g2.n_kb : g.n_kb;
             const bool hu = VARN && pu.narrow;                    // 128 channels
-            const int m_pair = pu.item / g.n_tiles;
+            const int m_pair = pu.item / (sc ? g2.n_tiles : g.n_tiles);
             const int m0 = (2 * m_pair + (int)crank) * BM;       // past M: rows that are never stored
             const int nimg = m0 / g.PQ, rem = m0 % g.PQ;
             const int p = rem / g.Q, q = rem % g.Q;
+            // A coordinates: this layer's geometry (a shortcut reads its centre tap)
             const int w0 = q * g.stride - g.pad, h0 = p * g.stride - g.pad;
-            for (int kb = 0; kb < g.n_kb; ++kb, ++it) {
+            for (int kb = 0; kb < n_kb; ++kb, ++it) {
                 const int s = it % PR_STAGES;
                 if (s % PR_NPROD != warp) continue;
                 if (!warp_wait(smem_u32(&empty[s]), ((uint32_t)(it / PR_STAGES) & 1u) ^ 1u, a.err, 1u)) { ok = false; break; }
@@ -898,6 +1031,8 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
                     if (hu)
                         tma_load_2d_pair(smem_u32(Bs + s * PR_BH_BYTES), &bmap64, fb, tap * g.C + c0,
                                          pu.nb + (int)crank * (BM / 2));
+                    else if (sc)
+                        tma_load_2d_pair(smem_u32(Bs + s * PR_BH_BYTES), &bmap2, fb, c0, pu.nb + (int)crank * BM);
                     else
                         tma_load_2d_pair(smem_u32(Bs + s * PR_BH_BYTES), &bmap, fb, tap * g.C + c0,
                                          pu.nb + (int)crank * BM);
@@ -909,10 +1044,12 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
     } else if (warp == PR_MMA_WARP) {
         // ---------------- MMA issuer: the even CTA, one elected lane ----------------
         if (leader) {
-            int it = 0, lt = 0;
-            for (int u = cid; u < num_units; u += ncl, ++lt) {
+            int it = 0;
+            for (int lt = 0; lt < n_units; ++lt) {
                 if (__any_sync(0xffffffffu, *abort_flag)) break;
-                const bool hu = VARN && pair_unit<VARN>(u, g).narrow;
+                const int u = unit_at(us, lt, cid, ncl);
+                const int n_kb = (SC && u >= n1) ? g2.n_kb : g.n_kb;
+                const bool hu = VARN && pair_unit_sc<VARN, SC>(u, n1, g, g2).narrow;
                 const uint32_t idesc = idesc_f16(2 * BM, hu ? BN / 2 : BN);
                 const int ab = lt & 1;
                 if (!warp_wait(smem_u32(&pair_empty[ab]), ((uint32_t)(lt >> 1) & 1u) ^ 1u, a.err, 8u)) {
@@ -921,7 +1058,7 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
                 }
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                 bool ok = true;
-                for (int kb = 0; kb < g.n_kb; ++kb, ++it) {
+                for (int kb = 0; kb < n_kb; ++kb, ++it) {
                     const int s = it % PR_STAGES;
                     if (!warp_wait(smem_u32(&full[s]), (uint32_t)(it / PR_STAGES) & 1u, a.err, 2u)) { ok = false; break; }
                     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
@@ -950,24 +1087,30 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
         const int quad = warp & 3;
         const int half = ep >> 2;
         const int row = quad * 32 + lane;
-        const __half *x = static_cast<const __half *>(a.x);
-        const FaultDelta fd = a.fd;
-        const float coef = __half2float(__ushort_as_half(g.coef_h));
-        const int ctr_r = g.ctr_tap / g.S, ctr_s = g.ctr_tap % g.S;
         const uint32_t pair_empty_even = mapa_shared(smem_u32(pair_empty), 0u);
-        const bool has_res = a.res != nullptr, relu = a.relu != 0;
-        const bool bias_sm = stage_bias(bias_s, a.bias, g.K, threadIdx.x - 32 * PR_EPI_WARP0, 32 * N_EPI_WARPS);
-        int lt = 0;
-        for (int u = cid; u < num_units; u += ncl, ++lt) {
-            const PairUnit pu = pair_unit<VARN>(u, g);
+        const int et = threadIdx.x - 32 * PR_EPI_WARP0;
+        const bool bias_sm = SC ? stage_bias2(bias_s, a.bias, a2.bias, g.K, et, 32 * N_EPI_WARPS)
+                                : stage_bias(bias_s, a.bias, g.K, et, 32 * N_EPI_WARPS);
+        for (int lt = 0; lt < n_units; ++lt) {
+            const int u = unit_at(us, lt, cid, ncl);
+            const bool sc = SC && u >= n1;
+            const ConvArgs &A = sc ? a2 : a;       // this unit's layer
+            const TcGeom &G = sc ? g2 : g;
+            const float *bias_l = bias_s + (sc ? G.K : 0);
+            const __half *x = static_cast<const __half *>(A.x);
+            const FaultDelta fd = A.fd;
+            const float coef = __half2float(__ushort_as_half(G.coef_h));
+            const int ctr_r = G.ctr_tap / G.S, ctr_s = G.ctr_tap % G.S;
+            const bool has_res = A.res != nullptr, relu = A.relu != 0;
+            const PairUnit pu = pair_unit_sc<VARN, SC>(u, n1, g, g2);
             const bool hu = VARN && pu.narrow;
-            const int m_pair = pu.item / g.n_tiles;
+            const int m_pair = pu.item / G.n_tiles;
             const int m0 = (2 * m_pair + (int)crank) * BM;
             const int m = m0 + row;
-            const bool valid = m < g.M;
+            const bool valid = m < G.M;
             const int mm = valid ? m : 0;
-            const int nimg = mm / g.PQ, rem = mm % g.PQ, p = rem / g.Q, q = rem % g.Q;
-            const bool do_cs = half == 0 && a.cs_out != nullptr && pu.nb == 0;
+            const int nimg = mm / G.PQ, rem = mm % G.PQ, p = rem / G.Q, q = rem % G.Q;
+            const bool do_cs = half == 0 && A.cs_out != nullptr && pu.nb == 0;
             // this warp's channels: cols [cw, cw + ncw) of the accumulator,
             // output channels nw + (0 .. ncw)
             const int ncw = hu ? BN / 4 : BN / 2;
@@ -976,19 +1119,19 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
             Res16 rs[BN / 32];
 #pragma unroll
             for (int c = 0; c < BN / 32; ++c)
-                rs[c] = (valid && 16 * c < ncw) ? load_res16(a, g.K, (size_t)m, nw + 16 * c)
+                rs[c] = (valid && 16 * c < ncw) ? load_res16(A, G.K, (size_t)m, nw + 16 * c)
                                                 : Res16{make_uint4(0u, 0u, 0u, 0u), make_uint4(0u, 0u, 0u, 0u)};
-            CsIn csv{0.f, 0.f};
+            CsIn csv{0.f, 0, 0};
             // carry-through column: coef * sum of the C channels of the centre-tap pixel
             float ctv = 0.f;
             if (do_cs && valid) {
-                csv = load_cs_inputs(a, g, m, nimg, p, q);
-                if (g.ct_mode != CT_NONE_) {
-                    const int h = p * g.stride + ctr_r - g.pad, w = q * g.stride + ctr_s - g.pad;
-                    if (h >= 0 && h < a.H && w >= 0 && w < a.W) {
-                        const uint4 *src = reinterpret_cast<const uint4 *>(x + (((size_t)nimg * a.H + h) * a.W + w) * g.C);
+                csv = load_cs_inputs(A, G, m, nimg, p, q);
+                if (G.ct_mode != CT_NONE_) {
+                    const int h = p * G.stride + ctr_r - G.pad, w = q * G.stride + ctr_s - G.pad;
+                    if (h >= 0 && h < A.H && w >= 0 && w < A.W) {
+                        const uint4 *src = reinterpret_cast<const uint4 *>(x + (((size_t)nimg * A.H + h) * A.W + w) * G.C);
                         float acc[4] = {0.f, 0.f, 0.f, 0.f};
-                        for (int c8 = 0; c8 < g.C / 8; ++c8) {
+                        for (int c8 = 0; c8 < G.C / 8; ++c8) {
                             const uint4 u = __ldg(src + c8);
                             const __half2 *hh = reinterpret_cast<const __half2 *>(&u);
 #pragma unroll
@@ -1004,30 +1147,36 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
             }
             const int ab = lt & 1;
             const uint32_t aph = (uint32_t)(lt >> 1) & 1u;
-            bool ok = mbar_wait(smem_u32(&acc_full[ab]), aph, a.err, 4u) && !*abort_flag;
+            bool ok = mbar_wait(smem_u32(&acc_full[ab]), aph, A.err, 4u) && !*abort_flag;
             ok = __all_sync(0xffffffffu, ok);      // tcgen05.ld below is warp-collective
             if (!ok) break;
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
             const uint32_t trow = tmem + (uint32_t)(ab * BN) + ((uint32_t)(quad * 32) << 16);
             float fsrc = 0.f;
             if (fd.active) {
-                const int h = p * g.stride + fd.r - g.pad, w = q * g.stride + fd.s - g.pad;
-                if (h >= 0 && h < a.H && w >= 0 && w < a.W) {
-                    if (fd.cin < g.C) fsrc = ldh(x, (((size_t)nimg * a.H + h) * a.W + w) * g.C + fd.cin);
-                    else if (a.cs_in) fsrc = ldh(static_cast<const __half *>(a.cs_in), ((size_t)nimg * a.H + h) * a.W + w);
+                const int h = p * G.stride + fd.r - G.pad, w = q * G.stride + fd.s - G.pad;
+                if (h >= 0 && h < A.H && w >= 0 && w < A.W) {
+                    if (fd.cin < G.C) fsrc = ldh(x, (((size_t)nimg * A.H + h) * A.W + w) * G.C + fd.cin);
+                    else if (A.cs_in) fsrc = ldh(static_cast<const __half *>(A.cs_in), ((size_t)nimg * A.H + h) * A.W + w);
                 }
             }
+            // TMEM loads one chunk ahead: chunk c + 16 is in flight while chunk c is stored
+            uint32_t tv[2][16];
+            tmem_ld16_nw(trow + cw, tv[0]);
+            tmem_wait_ld();
 #pragma unroll
             for (int c = 0; c < BN / 2; c += 16) {
                 if (c >= ncw) break;
+                if (c + 16 < ncw) tmem_ld16_nw(trow + cw + c + 16, tv[((c / 16) & 1) ^ 1]);
                 float v[16];
-                tmem_ld16(trow + cw + c, v);
-                if (valid && fd.active) store_chunk_pre(v, rs[c / 16], a, g.K, (size_t)m, nw + c, fsrc);
+                tmem_done16(tv[(c / 16) & 1], v);
+                if (valid && fd.active) store_chunk_pre(v, rs[c / 16], A, G.K, (size_t)m, nw + c, fsrc);
                 else if (valid)
-                    store16_fast(v, bias16_at(bias_s, a.bias, bias_sm, nw + c), rs[c / 16], has_res, relu,
-                                 static_cast<__half *>(a.y) + (size_t)m * g.K + nw + c);
+                    store16_fast(v, bias16_at(bias_l, A.bias, bias_sm, nw + c), rs[c / 16], has_res, relu,
+                                 static_cast<__half *>(A.y) + (size_t)m * G.K + nw + c);
+                tmem_wait_ld();
             }
-            if (do_cs && valid) store_checksum_pre(ctv, csv, a, g, m, fsrc);
+            if (do_cs && valid) store_checksum_pre(ctv, csv, A, G, m, fsrc);
             asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
             __syncwarp();
             if (lane == 0) mbar_arrive_cluster(pair_empty_even + (uint32_t)(ab * 8));
@@ -1645,10 +1794,10 @@ conv_tc_halo_kernel(const __grid_constant__ HaloMaps maps, const ConvArgs a, con
                     rs[c].r0 = rs[c].r1 = make_uint4(0u, 0u, 0u, 0u);
                 }
             }
-            CsIn csv{0.f, 0.f};
+            CsIn csv{0.f, 0, 0};
             if (do_cs) {
-                if (hg.csin) csv.cin = __half2float(reinterpret_cast<const __half *>(rst + R::RES)[row]);
-                if (hg.rescs) csv.rcs = __half2float(reinterpret_cast<const __half *>(rst + R::RES + R::CS)[row]);
+                if (hg.csin) csv.cin_h = reinterpret_cast<const unsigned short *>(rst + R::RES)[row];
+                if (hg.rescs) csv.rcs_h = reinterpret_cast<const unsigned short *>(rst + R::RES + R::CS)[row];
             }
             if (ring) {
                 __syncwarp();
@@ -1772,6 +1921,10 @@ struct TcPlan {
     CUtensorMap bmap_pair64;     // 128-channel half tiles: 64-row weight quarters
     int pair_clusters;           // resident CTA pairs (0: no pair variant)
     size_t pair_smem;
+    // launches that also run a shortcut: splits of the shortcut's items
+    // for the last few batch sizes (batch, items, s0, x; batch 0: empty)
+    int sc_cache[8][4];
+    int sc_next;
 };
 
 bool tc_supported(int C, int K, int R, int S, int stride, int pad, std::string *why) {
@@ -1827,13 +1980,19 @@ TcPlan *tc_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, cons
     cudaError_t e;
     if (pl->BN == 64) {
         pl->smem = smem_bytes<64, 4, 2>();
-        e = cudaFuncSetAttribute(conv_tc_kernel<64, 4, 2, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
+        e = cudaFuncSetAttribute(conv_tc_kernel<64, 4, 2, 4, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)pl->smem);
     } else if (pl->BN == 128) {
         pl->smem = smem_bytes<128, 3, 2>();
-        e = cudaFuncSetAttribute(conv_tc_kernel<128, 3, 2, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
+        e = cudaFuncSetAttribute(conv_tc_kernel<128, 3, 2, 1, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)pl->smem);
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(conv_tc_kernel<128, 3, 2, 1, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)pl->smem);
     } else {
         pl->smem = smem_bytes<256, 4, 1>();
-        e = cudaFuncSetAttribute(conv_tc_kernel<256, 4, 1, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->smem);
+        e = cudaFuncSetAttribute(conv_tc_kernel<256, 4, 1, 1, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)pl->smem);
     }
     if (e != cudaSuccess) { if (why) *why = "shared memory attribute"; delete pl; return nullptr; }
     // N = 256 over CTA pairs (cta_group::2): each CTA copies half of the
@@ -1851,11 +2010,11 @@ TcPlan *tc_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, cons
                                bstr, box_q, bes, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                                CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
         pl->pair_smem = pair_smem_bytes();
-        cudaError_t pe = cudaFuncSetAttribute(conv_tc_pair_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                              (int)pl->pair_smem);
-        if (pe == cudaSuccess)
-            pe = cudaFuncSetAttribute(conv_tc_pair_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                      (int)pl->pair_smem);
+        cudaError_t pe = cudaSuccess;
+        for (auto kern : {conv_tc_pair_kernel<false, false>, conv_tc_pair_kernel<true, false>,
+                          conv_tc_pair_kernel<false, true>, conv_tc_pair_kernel<true, true>})
+            if (pe == cudaSuccess)
+                pe = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl->pair_smem);
         if (r == CUDA_SUCCESS && pe == cudaSuccess) {
             cudaLaunchConfig_t cfg = {};
             cfg.gridDim = dim3(2 * 64);
@@ -1869,7 +2028,7 @@ TcPlan *tc_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, cons
             cfg.attrs = at;
             cfg.numAttrs = 1;
             int n = 0;
-            if (cudaOccupancyMaxActiveClusters(&n, conv_tc_pair_kernel<false>, &cfg) == cudaSuccess && n > 0)
+            if (cudaOccupancyMaxActiveClusters(&n, conv_tc_pair_kernel<false, false>, &cfg) == cudaSuccess && n > 0)
                 pl->pair_clusters = n;
         }
         cudaGetLastError();
@@ -1877,8 +2036,81 @@ TcPlan *tc_plan_create(const ConvArgs &a, int max_batch, const void *w_dev, cons
     return pl;
 }
 
-cudaError_t launch_conv_tc(const ConvArgs &a, const void *plan, cudaStream_t st, int *n_kernels) {
-    const TcPlan *pl = static_cast<const TcPlan *>(plan);
+namespace {
+
+// Estimated cost of a work unit, in K-block times: its K blocks or, when
+// more, the time its epilogue takes to store the tile (measured by clock
+// traces: about 4 K blocks for a 128 x 128 tile, 12 for the 256 x 256 tile
+// of a CTA pair), plus one for the accumulator hand-over.
+constexpr double EPI_KB_SINGLE = 4.0, EPI_KB_PAIR = 12.0, UNIT_OVERHEAD_KB = 1.0;
+double unit_cost(double kb, double epi) { return std::max(kb, epi) + UNIT_OVERHEAD_KB; }
+
+// Split of the shortcut's n2 items (UnitSeq: CTAs 0 .. s0 - 1 share items
+// 0 .. x - 1, the others the rest) that minimises the largest estimated
+// load, given each CTA's load of the first layer's units and the cost c2
+// of one shortcut item.  s0 is tried at the CTAs where that load changes
+// (round-robin units give a few levels) and at both ends; for each, the
+// best x balances the two groups' largest loads (the first grows with x,
+// the second shrinks).
+struct ScSplit {
+    int s0, x;
+};
+ScSplit shortcut_split(const std::vector<double> &load, int n2, double c2) {
+    const int ncl = (int)load.size();
+    auto share = [&](int c, int s0, int x) -> long long {
+        if (c < s0) return (c + 1) * (long long)x / s0 - c * (long long)x / s0;
+        const long long nc = ncl - s0, r = n2 - x;
+        return (c - s0 + 1) * r / nc - (c - s0) * r / nc;
+    };
+    auto group_max = [&](int c_lo, int c_hi, int s0, int x) {
+        double mx = 0.0;
+        for (int c = c_lo; c < c_hi; ++c) mx = std::max(mx, load[c] + (double)share(c, s0, x) * c2);
+        return mx;
+    };
+    ScSplit best{0, 0};
+    double best_max = 1e300;
+    for (int s0 = 0; s0 <= ncl; ++s0) {
+        if (s0 > 0 && s0 < ncl && load[s0] == load[s0 - 1]) continue;
+        int x = s0 == 0 ? 0 : n2;
+        if (s0 > 0 && s0 < ncl) {
+            int lo = 0, hi = n2;
+            while (lo < hi) {
+                const int mid = (lo + hi) / 2;
+                if (group_max(0, s0, s0, mid) >= group_max(s0, ncl, s0, mid)) hi = mid;
+                else lo = mid + 1;
+            }
+            x = lo;
+        }
+        for (int xc = x; xc >= std::max(0, x - 1); --xc) {
+            if ((s0 == 0 && xc != 0) || (s0 == ncl && xc != n2)) continue;
+            const double mx = std::max(group_max(0, s0, s0, xc), group_max(s0, ncl, s0, xc));
+            if (mx < best_max) {
+                best_max = mx;
+                best = ScSplit{s0, xc};
+            }
+        }
+    }
+    return best;
+}
+
+// The split for (batch, n2) from the plan's cache, else made by make() and
+// cached (the oldest of the entries is replaced).
+template <typename F>
+ScSplit cached_split(TcPlan *pl, int batch, int n2, F &&make) {
+    for (auto &e : pl->sc_cache)
+        if (e[0] == batch && e[1] == n2) return ScSplit{e[2], e[3]};
+    const ScSplit sp = make();
+    int *e = pl->sc_cache[pl->sc_next];
+    pl->sc_next = (pl->sc_next + 1) % 8;
+    e[0] = batch;
+    e[1] = n2;
+    e[2] = sp.s0;
+    e[3] = sp.x;
+    return sp;
+}
+
+// Geometry of one launch of plan pl: output tiles, K split, CTA pairs.
+TcGeom tc_launch_geom(const ConvArgs &a, const TcPlan *pl, bool *pairs) {
     TcGeom g = pl->g;
     g.M = a.N * a.P * a.Q;
     g.m_tiles = (g.M + BM - 1) / BM;
@@ -1889,7 +2121,51 @@ cudaError_t launch_conv_tc(const ConvArgs &a, const void *plan, cudaStream_t st,
     g.ws_ld = (g.K + 1 + 3) & ~3;
     g.splits = (a.K % 8 == 0) ? splitk_choose(tiles, g.n_kb, 4, pl->sms / 2, g.M, g.ws_ld, a.ws ? a.ws_bytes : 0) : 1;
     g.kps = (g.n_kb + g.splits - 1) / g.splits;
-    if (pl->pair_clusters > 0 && g.splits == 1 && g.m_tiles >= 2) {
+    g.sc_items = 0;
+    g.sc_s0 = 0;
+    g.sc_x = 0;
+    *pairs = pl->pair_clusters > 0 && g.splits == 1 && g.m_tiles >= 2;
+    return g;
+}
+
+}  // namespace
+
+bool tc_shortcut_fits(const ConvArgs &a, const void *plan, const void *plan2) {
+    const TcPlan *pl = static_cast<const TcPlan *>(plan);
+    const TcPlan *pl2 = static_cast<const TcPlan *>(plan2);
+    if (!pl || !pl2) return false;
+    bool pairs = false;
+    const TcGeom g = tc_launch_geom(a, pl, &pairs);
+    // both layers whole (unsplit) N = 128 tiles on single CTAs, or N = 256
+    // tiles on CTA pairs; the shortcut's K blocks are the centre tap's
+    return g.splits == 1 && pl2->BN == pl->BN && pl2->n_tiles == pl->n_tiles && pl2->g.n_kb == pl->g.cpb &&
+           ((pl->BN == 128 && !pairs) || (pl->BN == 256 && pairs));
+}
+
+cudaError_t launch_conv_tc(const ConvArgs &a, const void *plan, cudaStream_t st, int *n_kernels, const ConvArgs *a2,
+                           const void *plan2, bool *merged) {
+    TcPlan *pl = static_cast<TcPlan *>(const_cast<void *>(plan));
+    const TcPlan *pl2 = static_cast<const TcPlan *>(plan2);
+    if (merged) *merged = false;
+    bool pairs = false;
+    TcGeom g = tc_launch_geom(a, pl, &pairs);
+    const int tiles = g.m_tiles * g.n_tiles;
+    // a 1x1 shortcut of the same input (a2, plan2) joins this launch when the
+    // tiles allow; the caller launches it on its own otherwise
+    const bool sc = a2 && tc_shortcut_fits(a, plan, plan2);
+    TcGeom g2 = sc ? pl2->g : g;
+    if (sc) {
+        g2.M = g.M;
+        g2.m_tiles = g.m_tiles;
+        g2.ws_ld = g.ws_ld;
+        g2.splits = 1;
+        g2.kps = g2.n_kb;
+        g2.t_first = g2.units = 0;
+        g2.sc_items = g2.sc_s0 = g2.sc_x = 0;
+    }
+    const ConvArgs &b = sc ? *a2 : a;
+    const CUtensorMap &bm2 = sc ? (pairs ? pl2->bmap_pair : pl2->bmap) : (pairs ? pl->bmap_pair : pl->bmap);
+    if (pairs) {
         // tiles over CTA pairs: 256 pixels x 256 channels per pair
         const int items = ((g.m_tiles + 1) / 2) * g.n_tiles;
         const int P = pl->pair_clusters;
@@ -1899,22 +2175,64 @@ cudaError_t launch_conv_tc(const ConvArgs &a, const void *plan, cudaStream_t st,
         const bool halves = rem > 0 && 2 * rem <= P;
         g.t_first = halves ? items - rem : items;
         g.units = halves ? items + rem : items;
-        const int ncl = g.units < P ? g.units : P;
-        if (halves)
-            pdl_launch_cluster(conv_tc_pair_kernel<true>, dim3(2 * ncl), PR_THREADS, pl->pair_smem, st, 2, pl->amap,
-                               pl->bmap_pair, pl->bmap_pair64, a, g);
+        const int n2 = sc ? ((g.m_tiles + 1) / 2) * g2.n_tiles : 0;
+        const int ncl = g.units + n2 < P ? g.units + n2 : P;
+        if (sc) {
+            g.sc_items = n2;
+            const ScSplit sp = cached_split(pl, a.N, n2, [&] {
+                std::vector<double> load(ncl, 0.0);
+                for (int u = 0; u < g.units; ++u) {
+                    const bool narrow = halves && u < g.units - g.t_first;
+                    // a 128-channel half costs ~0.92 of a whole tile's K block (measured)
+                    load[u % ncl] += unit_cost((narrow ? 0.92 : 1.0) * g.n_kb, EPI_KB_PAIR);
+                }
+                return shortcut_split(load, n2, unit_cost(g2.n_kb, EPI_KB_PAIR));
+            });
+            g.sc_s0 = sp.s0;
+            g.sc_x = sp.x;
+        }
+        if (halves && sc)
+            pdl_launch_cluster(conv_tc_pair_kernel<true, true>, dim3(2 * ncl), PR_THREADS, pl->pair_smem, st, 2,
+                               pl->amap, pl->bmap_pair, pl->bmap_pair64, a, g, bm2, b, g2);
+        else if (sc)
+            pdl_launch_cluster(conv_tc_pair_kernel<false, true>, dim3(2 * ncl), PR_THREADS, pl->pair_smem, st, 2,
+                               pl->amap, pl->bmap_pair, pl->bmap_pair64, a, g, bm2, b, g2);
+        else if (halves)
+            pdl_launch_cluster(conv_tc_pair_kernel<true, false>, dim3(2 * ncl), PR_THREADS, pl->pair_smem, st, 2,
+                               pl->amap, pl->bmap_pair, pl->bmap_pair64, a, g, bm2, b, g2);
         else
-            pdl_launch_cluster(conv_tc_pair_kernel<false>, dim3(2 * ncl), PR_THREADS, pl->pair_smem, st, 2, pl->amap,
-                               pl->bmap_pair, pl->bmap_pair64, a, g);
+            pdl_launch_cluster(conv_tc_pair_kernel<false, false>, dim3(2 * ncl), PR_THREADS, pl->pair_smem, st, 2,
+                               pl->amap, pl->bmap_pair, pl->bmap_pair64, a, g, bm2, b, g2);
     } else {
         const int items = tiles * g.splits;
-        dim3 grid(items < pl->sms ? items : pl->sms);
-        if (pl->BN == 64) pdl_launch(conv_tc_kernel<64, 4, 2, 4>, grid, tc_threads(64, 4), pl->smem, st, pl->amap, pl->bmap, a, g);
-        else if (pl->BN == 128) pdl_launch(conv_tc_kernel<128, 3, 2, 2>, grid, tc_threads(128, 3), pl->smem, st, pl->amap, pl->bmap, a, g);
-        else pdl_launch(conv_tc_kernel<256, 4, 1, 1>, grid, tc_threads(256, 4), pl->smem, st, pl->amap, pl->bmap, a, g);
+        const int n2 = sc ? g2.m_tiles * g2.n_tiles : 0;
+        const int ncl = items + n2 < pl->sms ? items + n2 : pl->sms;
+        dim3 grid(ncl);
+        if (sc) {
+            g.sc_items = n2;
+            const ScSplit sp = cached_split(pl, a.N, n2, [&] {
+                std::vector<double> load(ncl, 0.0);
+                for (int u = 0; u < items; ++u) load[u % ncl] += unit_cost(g.n_kb, EPI_KB_SINGLE);
+                return shortcut_split(load, n2, unit_cost(g2.n_kb, EPI_KB_SINGLE));
+            });
+            g.sc_s0 = sp.s0;
+            g.sc_x = sp.x;
+            pdl_launch(conv_tc_kernel<128, 3, 2, 1, true>, grid, tc_threads(128, 3), pl->smem, st, pl->amap, pl->bmap,
+                       a, g, bm2, b, g2);
+        } else if (pl->BN == 64) {
+            pdl_launch(conv_tc_kernel<64, 4, 2, 4, false>, grid, tc_threads(64, 4), pl->smem, st, pl->amap, pl->bmap, a,
+                       g, bm2, b, g2);
+        } else if (pl->BN == 128) {
+            pdl_launch(conv_tc_kernel<128, 3, 2, 1, false>, grid, tc_threads(128, 3), pl->smem, st, pl->amap, pl->bmap,
+                       a, g, bm2, b, g2);
+        } else {
+            pdl_launch(conv_tc_kernel<256, 4, 1, 1, false>, grid, tc_threads(256, 4), pl->smem, st, pl->amap, pl->bmap,
+                       a, g, bm2, b, g2);
+        }
     }
     cudaError_t e = cudaGetLastError();
     if (n_kernels) *n_kernels = 1;
+    if (e == cudaSuccess && merged) *merged = sc;
     if (e != cudaSuccess || g.splits == 1) return e;
     if (n_kernels) *n_kernels = 2;
     return launch_splitk_reduce(a, g.splits, g.ws_ld, true, st);

@@ -100,6 +100,8 @@ struct LayerRT {
     StemPlan *stplan = nullptr;
     bool fused = false;          // max-pool computed by the preceding fused stem
     bool pool_fuse = false;      // conv: its halo kernel applies the 2 x 2 max-pool that follows (layer + 1)
+    bool sc_next = false;        // conv: layer + 1 is a 1x1 shortcut of the same input that may run in this
+                                 // layer's launch (its A operand is this layer's centre tap)
     int w_ld = 0, c_stride = 0;  // weight row length and channel stride within a tap
     // fc
     int n_in = 0, n_cs = 0, n_out = 0;
@@ -710,6 +712,18 @@ ct_status build_impl(ct_model *m, const ct_model_desc *desc, const float *const 
             if (!l.hplan) return CT_ECUDA;
         }
     }
+    // ---- 1x1 shortcuts that run in the launch of the convolution before them ----
+    // Layer i + 1 reads the same tensor as layer i at the same stride, and
+    // its pixel (p * stride, q * stride) is layer i's centre tap (pad =
+    // (R - 1) / 2): its GEMM operand A is layer i's centre-tap K blocks.
+    for (size_t i = 0; i + 1 < m->L.size() && !(m->flags & CT_FLAG_LAYERWISE); ++i) {
+        LayerRT &l = m->L[i];
+        const LayerRT &n = m->L[i + 1];
+        l.sc_next = l.tc && l.plan && n.tc && n.plan && !l.stem && !n.stem && l.d.op == CT_OP_CONV &&
+                    n.d.op == CT_OP_CONV && n.d.src == l.d.src && n.R == 1 && n.S == 1 && n.d.pad == 0 &&
+                    n.d.stride == l.d.stride && l.R == l.S && l.d.pad == (l.R - 1) / 2 && n.C == l.C &&
+                    n.K == l.K && n.d.res < 0 && (l.K == 128 || l.K % 256 == 0);
+    }
     // ---- the LeNet-5 shape runs as one whole-network kernel ----
     {
         SmallNet g;
@@ -923,30 +937,47 @@ ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, 
     }
     if (act_slot == 0) CUDA_TRY(xor_bit(m, act_base, act_word, m->f_bit, wb, st));
     size_t pool_done = (size_t)-1;               // a max-pool applied by the preceding conv kernel
+    size_t sc_done = (size_t)-1;                 // a shortcut run by the preceding conv's launch
+    // arguments of convolution layer li; a weight fault armed on it is
+    // resolved into wf (an explicit word is flipped by the caller around the
+    // launch, an implicit one rides in the epilogue as a delta)
+    auto conv_args = [&](size_t li, ConvArgs &a, WeightFault &wf) -> bool {
+        const LayerRT &l = m->L[li];
+        const ct_layer_desc &d = l.d;
+        const Slot &src = m->slots[d.src];
+        const Slot &dst = m->slots[d.dst];
+        a = ConvArgs{};
+        a.x = src.data; a.cs_in = src.has_cs ? src.cs : nullptr; a.w = l.w; a.bias = l.bias;
+        if (d.res >= 0) {
+            a.res = m->slots[d.res].data;
+            a.res_cs = m->slots[d.res].has_cs ? m->slots[d.res].cs : nullptr;
+        }
+        a.y = dst.data; a.cs_out = dst.has_cs ? dst.cs : nullptr;
+        a.N = batch; a.H = l.H; a.W = l.W; a.C = l.C; a.K = l.K; a.R = l.R; a.S = l.S;
+        a.stride = d.stride; a.pad = d.pad; a.P = l.P; a.Q = l.Q;
+        a.role = l.role; a.relu = d.relu; a.coef = l.coef; a.err = m->d_err;
+        a.ws = m->ws; a.ws_bytes = SPLITK_WS_BYTES;
+        const bool wfault = armed && m->f_kind == CT_BUF_WEIGHT && m->f_layer == (int)li;
+        if (wfault) {
+            wf = resolve_weight_fault(m, l, m->f_elem, m->f_bit);
+            if (!wf.explicit_word) a.fd = wf.fd;
+        }
+        return wfault;
+    };
+    auto conv_flops = [&](const LayerRT &l) { return 2.0 * batch * l.P * l.Q * (double)l.K * l.R * l.S * l.C; };
     for (size_t i = 0; i < m->L.size(); ++i) {
         LayerRT &l = m->L[i];
         const ct_layer_desc &d = l.d;
         Slot &src = m->slots[d.src];
         Slot &dst = m->slots[d.dst];
-        if (d.op == CT_OP_CONV) {
-            ConvArgs a{};
-            a.x = src.data; a.cs_in = src.has_cs ? src.cs : nullptr; a.w = l.w; a.bias = l.bias;
-            if (d.res >= 0) {
-                a.res = m->slots[d.res].data;
-                a.res_cs = m->slots[d.res].has_cs ? m->slots[d.res].cs : nullptr;
-            }
-            a.y = dst.data; a.cs_out = dst.has_cs ? dst.cs : nullptr;
-            a.N = batch; a.H = l.H; a.W = l.W; a.C = l.C; a.K = l.K; a.R = l.R; a.S = l.S;
-            a.stride = d.stride; a.pad = d.pad; a.P = l.P; a.Q = l.Q;
-            a.role = l.role; a.relu = d.relu; a.coef = l.coef; a.err = m->d_err;
+        if (i == sc_done) {
+            // computed by the launch of the convolution before it
+        } else if (d.op == CT_OP_CONV) {
+            ConvArgs a;
             WeightFault wf;
-            const bool wfault = armed && m->f_kind == CT_BUF_WEIGHT && m->f_layer == (int)i;
-            if (wfault) {
-                wf = resolve_weight_fault(m, l, m->f_elem, m->f_bit);
-                if (wf.explicit_word) CUDA_TRY(xor_bit(m, l.w, wf.word, m->f_bit, wb, st));
-                else a.fd = wf.fd;
-            }
-            const double flops = 2.0 * batch * l.P * l.Q * (double)l.K * l.R * l.S * l.C;
+            const bool wfault = conv_args(i, a, wf);
+            if (wfault && wf.explicit_word) CUDA_TRY(xor_bit(m, l.w, wf.word, m->f_bit, wb, st));
+            const double flops = conv_flops(l);
             if (l.stem) {
                 // the fused kernel reads the FP32 image and writes the max-pool's output
                 const Slot &po = m->slots[m->L[i + 1].d.dst];
@@ -963,7 +994,6 @@ ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, 
             } else if (l.tc_small) {
                 CUDA_TRY(launch(m, FAM_TC, flops, st, [&] { return launch_conv_tc_small(a, l.splan, st); }));
             } else {
-                a.ws = m->ws; a.ws_bytes = SPLITK_WS_BYTES;
                 int nk = 1;
                 const bool halo = l.hplan && halo_tiles(l.hplan, batch) >= halo_sms(l.hplan);
                 dst.skipped_last = halo && l.pool_fuse;
@@ -974,10 +1004,27 @@ ct_status infer_impl(ct_model *m, const float *input, int batch, float *logits, 
                     a.cs_out = po.has_cs ? po.cs : nullptr;
                     pool_done = i + 1;
                 }
-                if (halo)
+                const LayerRT *ln = l.sc_next ? &m->L[i + 1] : nullptr;
+                ConvArgs a2;
+                WeightFault wf2;
+                bool wfault2 = false;
+                if (ln) wfault2 = conv_args(i + 1, a2, wf2);
+                if (halo) {
                     CUDA_TRY(launch(m, FAM_TC, flops, st, [&] { return launch_conv_tc_halo(a, l.hplan, st); }));
-                else if (l.tc) CUDA_TRY(launch(m, FAM_TC, flops, st, [&] { return launch_conv_tc(a, l.plan, st, &nk); }, &nk));
-                else CUDA_TRY(launch(m, FAM_SIMT, flops, st, [&] { return launch_conv_simt(a, half, st, &nk); }, &nk));
+                } else if (ln && tc_shortcut_fits(a, l.plan, ln->plan)) {
+                    // the shortcut (layer i + 1) runs in this launch
+                    if (wfault2 && wf2.explicit_word) CUDA_TRY(xor_bit(m, ln->w, wf2.word, m->f_bit, wb, st));
+                    bool merged = false;
+                    CUDA_TRY(launch(m, FAM_TC, flops + conv_flops(*ln), st,
+                                    [&] { return launch_conv_tc(a, l.plan, st, &nk, &a2, ln->plan, &merged); }, &nk));
+                    if (!merged) return CT_ECUDA;
+                    if (wfault2 && wf2.explicit_word) CUDA_TRY(xor_bit(m, ln->w, wf2.word, m->f_bit, wb, st));
+                    sc_done = i + 1;
+                } else if (l.tc) {
+                    CUDA_TRY(launch(m, FAM_TC, flops, st, [&] { return launch_conv_tc(a, l.plan, st, &nk); }, &nk));
+                } else {
+                    CUDA_TRY(launch(m, FAM_SIMT, flops, st, [&] { return launch_conv_simt(a, half, st, &nk); }, &nk));
+                }
             }
             if (wfault && wf.explicit_word) CUDA_TRY(xor_bit(m, l.w, wf.word, m->f_bit, wb, st));
         } else if (l.fused || i == pool_done) {

@@ -184,7 +184,14 @@ inline cudaError_t pdl_launch_cluster(void (*kernel)(KArgs...), dim3 grid, dim3 
 // conv launchers report in *n_kernels (may be null) how many kernels they
 // launched: 2 when K is split (the conv kernel and the split-K reduction)
 cudaError_t launch_conv_simt(const ConvArgs &a, bool half, cudaStream_t st, int *n_kernels);
-cudaError_t launch_conv_tc(const ConvArgs &a, const void *tc_plan, cudaStream_t st, int *n_kernels);
+// a2 / tc_plan2: a 1x1 shortcut convolution of the same input at the same
+// stride whose pixel is the first layer's centre tap; it runs in the same
+// launch when both layers' tiles allow (*merged tells whether it did; if
+// not, the caller launches it itself)
+cudaError_t launch_conv_tc(const ConvArgs &a, const void *tc_plan, cudaStream_t st, int *n_kernels,
+                           const ConvArgs *a2 = nullptr, const void *tc_plan2 = nullptr, bool *merged = nullptr);
+// whether launch_conv_tc(a, tc_plan, ..., a2, tc_plan2) runs both layers in one launch
+bool tc_shortcut_fits(const ConvArgs &a, const void *tc_plan, const void *tc_plan2);
 // Split-K: number of K splits for `tiles` output tiles over n_kblocks K
 // blocks (1 = no split); partial sums [splits][M][ws_ld] must fit ws_bytes.
 int splitk_choose(int tiles, int n_kblocks, int min_kb_per_split, int target_ctas, int M, int ws_ld,

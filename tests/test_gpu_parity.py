@@ -203,3 +203,40 @@ def test_half_tiles_of_the_last_round_give_whole_tile_bits():
     (d256, c256), (d128, c128) = out[256], out[128]
     assert np.isfinite(d256).all() and np.abs(d256).max() > 0
     assert np.array_equal(d256[128:], d128) and np.array_equal(c256[128:], c128)
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("batch", [256, 37])
+def test_shortcuts_in_the_block_launch_give_separate_launch_bits(batch):
+    """ResNet-18 (224 x 224, FP16): each 1 x 1 stride-2 shortcut runs in the
+    launch of its block's first 3 x 3 convolution, reading that
+    convolution's centre-tap K blocks (stage 2 on single CTAs; stages 3-4 on
+    CTA pairs, stage 4 beside half tiles at 256 images); CT_FLAG_LAYERWISE
+    runs each shortcut in its own launch.  Every output is the same MMA
+    sequence either way, so every stored tensor (data and checksum), the
+    logits and S are the same bits; the merged run also launches three
+    kernels fewer at 256 images."""
+    x = inputs("resnet18_imagenet", batch, 3)
+    res = {}
+    for lw in (False, True):
+        m = model("resnet18_imagenet", layerwise=lw, max_batch=batch)
+        lg, S, fl = run(m, x)
+        assert ct().ct_device_error(m) == 0
+        acts = {}
+        for slot in range(2, 23):
+            try:
+                acts[slot] = ct().ct_copy_activation(m, slot, batch)
+            except RuntimeError:
+                pass
+        res[lw] = (lg, S, fl, acts, ct().ct_launches_per_infer(m))
+        m.close()
+    (lg0, S0, f0, a0, k0), (lg1, S1, f1, a1, k1) = res[False], res[True]
+    assert sorted(a0) == sorted(a1) and len(a0) >= 18
+    for slot in a0:
+        (d0, c0), (d1, c1) = a0[slot], a1[slot]
+        assert np.array_equal(d0, d1, equal_nan=True), slot
+        assert (c0 is None) == (c1 is None) and (c0 is None or np.array_equal(c0, c1, equal_nan=True)), slot
+    assert np.array_equal(lg0, lg1, equal_nan=True) and np.array_equal(S0, S1, equal_nan=True)
+    assert np.array_equal(f0, f1)
+    if batch == 256:
+        assert k1 - k0 == 3
