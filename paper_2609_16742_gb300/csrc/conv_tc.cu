@@ -331,6 +331,37 @@ __device__ __forceinline__ void store16_fast(const float *v, const Bias16 &b, co
     st_global_v8(dst, pk);          // 16 channels of one pixel: 32-byte aligned
 }
 
+// store16_fast without a residual, into registers: FP16 pairs of
+// (accumulator + bias), ReLU fused into the rounding (the same bits).
+__device__ __forceinline__ void pack16(const float *v, const Bias16 &b, bool relu, uint32_t (&pk)[8]) {
+    const float *bb = reinterpret_cast<const float *>(b.q);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) pk[i] = cvt_h2(v[2 * i] + bb[2 * i], v[2 * i + 1] + bb[2 * i + 1], relu);
+}
+// 4 x 4 transpose of 32-byte pieces among the lanes 4a .. 4a + 3 of a warp
+// (i = lane & 3): on entry pk[p] is piece p (channels 16p .. 16p + 15) of
+// this lane's pixel, on exit pk[k] is piece i of the pixel of lane 4a + k.
+// Two butterfly rounds of shuffles; then a warp's store of pk[k] writes
+// eight pixels' 64 channels, eight whole 128-byte lines, where a store of
+// each lane's own piece touches 32 lines.
+__device__ __forceinline__ void transpose4_pieces(uint32_t (&pk)[4][8], int i) {
+#pragma unroll
+    for (int mk = 1; mk <= 2; mk <<= 1) {
+        const bool up = (i & mk) != 0;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            if (q & mk) continue;
+#pragma unroll
+            for (int r = 0; r < 8; ++r) {
+                const uint32_t send = up ? pk[q][r] : pk[q + mk][r];
+                const uint32_t recv = __shfl_xor_sync(0xffffffffu, send, mk);
+                if (up) pk[q][r] = recv;
+                else pk[q + mk][r] = recv;
+            }
+        }
+    }
+}
+
 // Epilogue values of 16 channels k0 .. k0 + 15 of one pixel in FP32, in the
 // order of store_chunk_pre: accumulator + bias, fault delta, residual, ReLU.
 __device__ __forceinline__ void epi16_vals(const float *v, const Bias16 &b, const Res16 &r, bool res, bool relu,
@@ -819,6 +850,24 @@ conv_tc_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__
                     for (int c = 0; c < BN / 2; c += 16)
                         store_chunk_pre(vals + c, rs[c / 16], A, G.K, (size_t)m, n0 + half * (BN / 2) + c, fsrc);
                     if (do_cs) store_checksum_pre(ctv, csv, A, G, m, fsrc);
+                } else if (BN == 128 && !split && !fd.active && !has_res) {
+                    // whole lines: the lanes of each group of four swap their
+                    // 16-channel pieces (all lanes take part; stores of pixels
+                    // past M are skipped)
+                    uint32_t pk[4][8];
+#pragma unroll
+                    for (int c = 0; c < 4; ++c)
+                        pack16(vals + 16 * c, bias16_at(bias_l, A.bias, bias_sm, n0 + half * (BN / 2) + 16 * c), relu,
+                               pk[c]);
+                    transpose4_pieces(pk, lane & 3);
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) {
+                        const int mk = m0 + quad * 32 + (lane & ~3) + k;
+                        if (mk < G.M)
+                            st_global_v8(static_cast<__half *>(A.y) + (size_t)mk * G.K + n0 + half * (BN / 2) +
+                                             16 * (lane & 3), pk[k]);
+                    }
+                    if (do_cs && valid) store_checksum_pre(ctv, csv, A, G, m, 0.f);
                 } else if (valid) {
                     __half *yrow = static_cast<__half *>(A.y) + (size_t)m * G.K + n0 + half * (BN / 2);
 #pragma unroll
@@ -1160,21 +1209,40 @@ conv_tc_pair_kernel(const __grid_constant__ CUtensorMap amap, const __grid_const
                     else if (A.cs_in) fsrc = ldh(static_cast<const __half *>(A.cs_in), ((size_t)nimg * A.H + h) * A.W + w);
                 }
             }
-            // TMEM loads one chunk ahead: chunk c + 16 is in flight while chunk c is stored
-            uint32_t tv[2][16];
-            tmem_ld16_nw(trow + cw, tv[0]);
-            tmem_wait_ld();
+            if (!fd.active && !has_res) {
+                // whole lines: per 64 channels the lanes of each group of four
+                // swap their 16-channel pieces (all lanes take part; stores of
+                // pixels past M are skipped)
+#pragma unroll
+                for (int c0 = 0; c0 < BN / 2; c0 += 64) {
+                    if (c0 >= ncw) break;
+                    uint32_t pk[4][8];
+#pragma unroll
+                    for (int c = 0; c < 4; ++c) {
+                        float v[16];
+                        tmem_ld16(trow + cw + c0 + 16 * c, v);
+                        pack16(v, bias16_at(bias_l, A.bias, bias_sm, nw + c0 + 16 * c), relu, pk[c]);
+                    }
+                    transpose4_pieces(pk, lane & 3);
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) {
+                        const int mk = m0 + quad * 32 + (lane & ~3) + k;
+                        if (mk < G.M)
+                            st_global_v8(static_cast<__half *>(A.y) + (size_t)mk * G.K + nw + c0 + 16 * (lane & 3),
+                                         pk[k]);
+                    }
+                }
+            } else {
 #pragma unroll
             for (int c = 0; c < BN / 2; c += 16) {
                 if (c >= ncw) break;
-                if (c + 16 < ncw) tmem_ld16_nw(trow + cw + c + 16, tv[((c / 16) & 1) ^ 1]);
                 float v[16];
-                tmem_done16(tv[(c / 16) & 1], v);
+                tmem_ld16(trow + cw + c, v);
                 if (valid && fd.active) store_chunk_pre(v, rs[c / 16], A, G.K, (size_t)m, nw + c, fsrc);
                 else if (valid)
                     store16_fast(v, bias16_at(bias_l, A.bias, bias_sm, nw + c), rs[c / 16], has_res, relu,
                                  static_cast<__half *>(A.y) + (size_t)m * G.K + nw + c);
-                tmem_wait_ld();
+            }
             }
             if (do_cs && valid) store_checksum_pre(ctv, csv, A, G, m, fsrc);
             asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");

@@ -185,3 +185,37 @@ def test_inject_range_errors():
         ct().ct_inject(m, 0, 0, 0, 32)
     ct().ct_inject(m, 0, 0, 7 * 25 - 1, 31)
     ct().ct_clear_faults(m)
+
+
+def test_faults_in_shortcuts_that_share_their_block_launch():
+    """ResNet-18/224, FP16, 64 images: the 1 x 1 shortcuts of stages 2 and 3
+    (layers 7 and 12) run in the launch of their block's first convolution
+    (layers 6 and 11; single CTAs, CTA pairs).  Weight faults in both layers
+    (flipped words, and epilogue deltas for the shortcut's checksum-channel
+    weights: its pass-through weight and a zero weight from the incoming
+    checksum to a data channel) and activation faults in the tensor both
+    read give the same bits as separate launches (CT_FLAG_LAYERWISE)."""
+    B = 64
+    x = inputs("resnet18_imagenet", B)
+    ms = {lw: model("resnet18_imagenet", layerwise=lw, max_batch=B) for lw in (False, True)}
+    # the merged pairs' weights (layers 6 + 7, 11 + 12) and the tensors they read
+    bufs = [b for b in ct().ct_buffers(ms[False], B) if b[1] in (6, 7, 11, 12)]
+    faults = []
+    for kind, layers, n in ((0, (6, 11), 8), (0, (7, 12), 16), (1, (6, 11), 8)):
+        faults += synth.draw_faults([b for b in bufs if b[0] == kind and b[1] in layers], n, seed=5).tolist()
+    for layer, C, K in ((7, 64, 128), (12, 128, 256)):
+        faults.append([0, layer, K * (C + 1) + C, 14])      # checksum pass-through weight 1.0 -> inf
+        faults.append([0, layer, 5 * (C + 1) + C, 13])      # incoming checksum -> channel 5 (0)
+    assert {f[0] for f in faults} == {0, 1}
+    for kind, layer, e, bit in faults:
+        out = []
+        for lw in (False, True):
+            ct().ct_inject(ms[lw], kind, layer, e, bit)
+            out.append(run(ms[lw], x))
+        (l0, s0, f0), (l1, s1, f1) = out
+        assert np.array_equal(l0, l1, equal_nan=True), (kind, layer, e, bit)
+        assert np.array_equal(s0, s1, equal_nan=True) and np.array_equal(f0, f1), (kind, layer, e, bit)
+    assert ct().ct_launches_per_infer(ms[True]) - ct().ct_launches_per_infer(ms[False]) >= 2
+    for m in ms.values():
+        assert ct().ct_device_error(m) == 0
+        m.close()
