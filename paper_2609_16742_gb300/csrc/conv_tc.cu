@@ -23,11 +23,14 @@
 //
 // The kernels are persistent: one CTA per SM walks a static list of output
 // tiles.  The TMA producers run ahead across tile boundaries through a ring
-// of shared-memory stages.  Consecutive K blocks accumulate into up to four
-// independent TMEM accumulators (chains), because back-to-back MMAs into one
-// accumulator wait on each other; the epilogue sums the chains.  For
-// N <= 128 it releases TMEM before its global stores so that the next
-// tile's MMAs overlap them; for N = 256 two accumulators alternate.
+// of shared-memory stages.  N = 64 tiles spread consecutive K blocks over
+// four independent TMEM accumulators (chains), because back-to-back short
+// MMAs into one accumulator wait on each other; the epilogue sums the
+// chains.  N = 128 and N = 256 tiles use one accumulator, and two of them
+// alternate in TMEM, so that a tile's MMAs overlap the previous tile's
+// epilogue.  A 1x1 shortcut that reads the same input at the same stride
+// (a ResNet downsample) can run in the launch of its block's first
+// convolution, whose centre-tap K blocks are its A operand (UnitSeq).
 //
 // With N = 256 and no split K, conv_tc_pair_kernel runs the tiles on pairs of
 // CTAs (a cluster of two, tcgen05 cta_group::2): one M = 256 MMA reads the
@@ -451,11 +454,11 @@ __device__ __forceinline__ void store_checksum_pre(float ctv, const CsIn &c, con
 
 // K-block kb accumulates into chain kb % NCH: back-to-back MMAs into one
 // TMEM accumulator serialise on it, so NCH independent chains keep the
-// tensor pipe busy when one 128 x BN x 16 MMA is short (BN = 64, 128).  The
+// tensor pipe busy when one 128 x BN x 16 MMA is short (BN = 64).  The
 // epilogue adds the chains.  SUB K-blocks share one pipeline stage (one
-// barrier round trip).  A single TMEM buffer holds the chains; for
-// BN <= 128 the epilogue copies it to registers and releases it before its
-// global stores, so the next tile's MMAs overlap the stores.
+// barrier round trip).  When two buffers of the chains fit in TMEM (NACC),
+// tiles alternate between them; for BN <= 128 the epilogue also copies its
+// buffer to registers and releases it before its global stores.
 // SC: the launch also runs a 1x1 shortcut convolution (bmap2, a2, g2; see
 // UnitSeq); otherwise those arguments are unused.
 template <int BN, int STAGES, int SUB, int NCH, bool SC>
