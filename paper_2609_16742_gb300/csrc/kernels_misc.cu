@@ -25,6 +25,19 @@ __device__ __forceinline__ float relu_keep_nan(float v) { return v < 0.f ? 0.f :
 // FMAs and one staged weight value is a broadcast.
 // ---------------------------------------------------------------------------
 constexpr int FC_J = 16, FC_IMG = 64, FC_KC = 64, FC_WARPS = 8;
+// input rows in shared memory: FC_KC values + 4 of padding (16-byte rows; a
+// warp's 16-byte reads of 32 rows at one k then hit every bank once per phase)
+constexpr int FC_XP = FC_KC + 4;
+static_assert((FC_KC / 4) % FC_WARPS == 0, "each warp takes whole groups of four inputs");
+
+// four consecutive inputs k .. k + 3 of one row as FP32 (16 or 8 bytes, aligned)
+__device__ __forceinline__ float4 load4_f(const float *p) { return *reinterpret_cast<const float4 *>(p); }
+__device__ __forceinline__ float4 load4_f(const __half *p) {
+    const uint2 u = *reinterpret_cast<const uint2 *>(p);
+    const float2 a = __half22float2(*reinterpret_cast<const __half2 *>(&u.x));
+    const float2 b = __half22float2(*reinterpret_cast<const __half2 *>(&u.y));
+    return make_float4(a.x, a.y, b.x, b.y);
+}
 
 // Row b of a layer's output: a row of this batch, or (final layer with
 // re-run rows) the re-executed image's row of the earlier batch's logits
@@ -44,17 +57,17 @@ __device__ __forceinline__ void fc_final_out(const FcArgs &a, int b, float s, ui
     if (a.flag) a.flag[b] = fv;
     if (a.flag2) a.flag2[b] = fv;
 }
-static_assert((FC_KC * (FC_IMG + 1)) % 4 == 0, "weight tile must start 16-byte aligned (float4 reads)");
+static_assert((FC_IMG * FC_XP) % 4 == 0, "weight tile must start 16-byte aligned (float4 reads)");
 
 template <typename TX, typename TW, typename TY>
 __global__ void __launch_bounds__(256, 2) fc_kernel(FcArgs a) {
     pdl_wait();
     pdl_trigger();
     extern __shared__ __align__(16) float smem[];
-    // two stages of [FC_KC][FC_IMG + 1] inputs and [FC_KC][FC_J] weights (each
+    // two stages of [FC_IMG][FC_XP] inputs and [FC_KC][FC_J] weights (each
     // offset a multiple of 4 floats: 16-byte aligned float4 reads), then the
     // cross-warp reduction [FC_WARPS][FC_J + 1][FC_IMG]
-    constexpr int XS = FC_KC * (FC_IMG + 1), WS = FC_KC * FC_J;
+    constexpr int XS = FC_IMG * FC_XP, WS = FC_KC * FC_J;
     float *red = smem + 2 * (XS + WS);
     const TX *x = static_cast<const TX *>(a.x);
     const TW *w = static_cast<const TW *>(a.w);
@@ -71,17 +84,31 @@ __global__ void __launch_bounds__(256, 2) fc_kernel(FcArgs a) {
     const int nkc = (a.n_in + FC_KC - 1) / FC_KC;
     const int kc_per = (nkc + gridDim.z - 1) / gridDim.z;
     const int k_lo = blockIdx.z * kc_per * FC_KC, k_hi = min(a.n_in, k_lo + kc_per * FC_KC);
-    // x[b0 .. b0+63][k0 .. k0+63] (transposed) and W[j0..j0+15][k0..k0+63]:
+    // x[b0 .. b0+63][k0 .. k0+63] and W[j0..j0+15][k0..k0+63] (transposed):
     // the next chunk's values are loaded into registers while this chunk is
-    // multiplied, then stored to the other stage
+    // multiplied, then stored to the other stage.  The inputs move as four
+    // consecutive values per load when every row starts 16-byte aligned
+    // (n_in a multiple of 4; the K ranges end on multiples of 4 then too).
     constexpr int XR = FC_KC * FC_IMG / 256, WR = FC_KC * FC_J / 256;
-    float xr[XR], wr[WR];
+    const bool xvec = (a.n_in & 3) == 0;
+    float4 xr[XR / 4];
+    float xs[XR];
+    float wr[WR];
     auto load_chunk = [&](int k0) {
+        if (xvec) {
 #pragma unroll
-        for (int i = 0; i < XR; ++i) {
-            const int e = tid + 256 * i, kk = e % FC_KC, bb = e / FC_KC;
-            const int b = b0 + bb, k = k0 + kk;
-            xr[i] = (b < a.B && k < k_hi) ? to_f(x[(size_t)b * a.n_in + k]) : 0.f;
+            for (int i = 0; i < XR / 4; ++i) {
+                const int e = tid + 256 * i, k4 = (e % (FC_KC / 4)) * 4, bb = e / (FC_KC / 4);
+                const int b = b0 + bb, k = k0 + k4;
+                xr[i] = (b < a.B && k < k_hi) ? load4_f(x + (size_t)b * a.n_in + k) : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+        } else {
+#pragma unroll
+            for (int i = 0; i < XR; ++i) {
+                const int e = tid + 256 * i, kk = e % FC_KC, bb = e / FC_KC;
+                const int b = b0 + bb, k = k0 + kk;
+                xs[i] = (b < a.B && k < k_hi) ? to_f(x[(size_t)b * a.n_in + k]) : 0.f;
+            }
         }
 #pragma unroll
         for (int i = 0; i < WR; ++i) {
@@ -92,10 +119,18 @@ __global__ void __launch_bounds__(256, 2) fc_kernel(FcArgs a) {
     };
     auto store_chunk = [&](int stage) {
         float *Xd = smem + stage * (XS + WS), *Wd = Xd + XS;
+        if (xvec) {
 #pragma unroll
-        for (int i = 0; i < XR; ++i) {
-            const int e = tid + 256 * i;
-            Xd[(e % FC_KC) * (FC_IMG + 1) + e / FC_KC] = xr[i];
+            for (int i = 0; i < XR / 4; ++i) {
+                const int e = tid + 256 * i;
+                *reinterpret_cast<float4 *>(&Xd[(e / (FC_KC / 4)) * FC_XP + (e % (FC_KC / 4)) * 4]) = xr[i];
+            }
+        } else {
+#pragma unroll
+            for (int i = 0; i < XR; ++i) {
+                const int e = tid + 256 * i;
+                Xd[(e / FC_KC) * FC_XP + e % FC_KC] = xs[i];
+            }
         }
 #pragma unroll
         for (int i = 0; i < WR; ++i) {
@@ -113,23 +148,31 @@ __global__ void __launch_bounds__(256, 2) fc_kernel(FcArgs a) {
         const bool more = k0 + FC_KC < k_hi;
         if (more) load_chunk(k0 + FC_KC);
         const float *Xs = smem + stage * (XS + WS), *Ws = Xs + XS;
-#pragma unroll 2
-        for (int kk = warp; kk < FC_KC; kk += FC_WARPS) {
-            float x0 = Xs[kk * (FC_IMG + 1) + lane], x1 = Xs[kk * (FC_IMG + 1) + lane + 32];
-            const float4 *wrow = reinterpret_cast<const float4 *>(&Ws[kk * FC_J]);
+        // warp w takes the groups of four inputs g = w, w + FC_WARPS, ...;
+        // lanes are images (lane, lane + 32)
 #pragma unroll
-            for (int q = 0; q < FC_J / 4; ++q) {
-                float4 wv = wrow[q];
-                acc[4 * q + 0][0] = fmaf(wv.x, x0, acc[4 * q + 0][0]);
-                acc[4 * q + 0][1] = fmaf(wv.x, x1, acc[4 * q + 0][1]);
-                acc[4 * q + 1][0] = fmaf(wv.y, x0, acc[4 * q + 1][0]);
-                acc[4 * q + 1][1] = fmaf(wv.y, x1, acc[4 * q + 1][1]);
-                acc[4 * q + 2][0] = fmaf(wv.z, x0, acc[4 * q + 2][0]);
-                acc[4 * q + 2][1] = fmaf(wv.z, x1, acc[4 * q + 2][1]);
-                acc[4 * q + 3][0] = fmaf(wv.w, x0, acc[4 * q + 3][0]);
-                acc[4 * q + 3][1] = fmaf(wv.w, x1, acc[4 * q + 3][1]);
+        for (int g = warp; g < FC_KC / 4; g += FC_WARPS) {
+            const float4 x04 = *reinterpret_cast<const float4 *>(&Xs[lane * FC_XP + 4 * g]);
+            const float4 x14 = *reinterpret_cast<const float4 *>(&Xs[(lane + 32) * FC_XP + 4 * g]);
+            const float x0v[4] = {x04.x, x04.y, x04.z, x04.w}, x1v[4] = {x14.x, x14.y, x14.z, x14.w};
+#pragma unroll
+            for (int t = 0; t < 4; ++t) {
+                const float x0 = x0v[t], x1 = x1v[t];
+                const float4 *wrow = reinterpret_cast<const float4 *>(&Ws[(4 * g + t) * FC_J]);
+#pragma unroll
+                for (int q = 0; q < FC_J / 4; ++q) {
+                    float4 wv = wrow[q];
+                    acc[4 * q + 0][0] = fmaf(wv.x, x0, acc[4 * q + 0][0]);
+                    acc[4 * q + 0][1] = fmaf(wv.x, x1, acc[4 * q + 0][1]);
+                    acc[4 * q + 1][0] = fmaf(wv.y, x0, acc[4 * q + 1][0]);
+                    acc[4 * q + 1][1] = fmaf(wv.y, x1, acc[4 * q + 1][1]);
+                    acc[4 * q + 2][0] = fmaf(wv.z, x0, acc[4 * q + 2][0]);
+                    acc[4 * q + 2][1] = fmaf(wv.z, x1, acc[4 * q + 2][1]);
+                    acc[4 * q + 3][0] = fmaf(wv.w, x0, acc[4 * q + 3][0]);
+                    acc[4 * q + 3][1] = fmaf(wv.w, x1, acc[4 * q + 3][1]);
+                }
+                if (ct_block) { act[0] += x0; act[1] += x1; }
             }
-            if (ct_block) { act[0] += x0; act[1] += x1; }
         }
         if (more) store_chunk(stage ^ 1);
         __syncthreads();
@@ -419,7 +462,7 @@ int grid_for(int64_t n, int threads) {
 template <typename TX, typename TW, typename TY>
 cudaError_t fc_go(const FcArgs &a, cudaStream_t st, int *n_kernels) {
     const size_t smem =
-        sizeof(float) * (2 * (FC_KC * (FC_IMG + 1) + FC_KC * FC_J) + FC_WARPS * (FC_J + 1) * FC_IMG);
+        sizeof(float) * (2 * (FC_IMG * FC_XP + FC_KC * FC_J) + FC_WARPS * (FC_J + 1) * FC_IMG);
     static bool attr = false;
     if (!attr) {
         cudaError_t e = cudaFuncSetAttribute(fc_kernel<TX, TW, TY>,
