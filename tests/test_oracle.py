@@ -101,6 +101,26 @@ def test_conv2d_matches_bruteforce(stride, pad):
     np.testing.assert_allclose(y, ref, rtol=1e-12, atol=1e-12)
 
 
+@pytest.mark.parametrize("hw", [(8, 8), (7, 9), (14, 14)])
+def test_strided_shortcut_reads_the_centre_tap_of_the_block_convolution(hw):
+    """A 1 x 1 stride-2 convolution (pad 0) equals a 3 x 3 stride-2 pad-1
+    convolution whose only non-zero tap is the centre: output (p, q) reads
+    input (2p, 2q) in both, for every map size (odd ones too).  This is
+    why a ResNet downsample can use its block's first convolution's
+    centre-tap operand.  Checked against the brute-force loop, integers so
+    that the sums are exact."""
+    rng = np.random.default_rng(hw[0] * 31 + hw[1])
+    x = rng.integers(-3, 4, size=(5,) + hw).astype(np.float64)
+    w1 = rng.integers(-3, 4, size=(6, 5, 1, 1)).astype(np.float64)
+    w3 = np.zeros((6, 5, 3, 3))
+    w3[:, :, 1, 1] = w1[:, :, 0, 0]
+    a = brute_conv(x, w1, 2, 0)
+    b = brute_conv(x, w3, 2, 1)
+    assert a.shape == b.shape == (6, (hw[0] - 1) // 2 + 1, (hw[1] - 1) // 2 + 1)
+    assert np.array_equal(a, b)
+    assert np.array_equal(oracle.conv2d(x, w1, None, 2, 0), a)
+
+
 def test_conv2d_skip_is_structural():
     x = np.ones((2, 4, 4))
     x[1, 1, 1] = np.inf
